@@ -1,0 +1,339 @@
+"""Seeded synthetic workloads: networks, test inputs and mutant descriptor tables.
+
+This module only *generates data*.  It holds none of the method's arithmetic (no
+layer function, no mutation operator, no kill rule) and imports neither the GPU
+binding nor the oracle, so both can be fed the very same arrays.
+
+The paper's trained models and datasets (Table 1: LeNet-5, ResNet, MobileNetV2, FCNN,
+RNN on MNIST-family, SVHN, CIFAR-10, Caltech-101, IMDB, Reuters) are not available
+here.  Random-initialised networks of the same shapes and random inputs of the
+datasets' shapes (28x28x1 / 32x32x3, 10 classes) stand in for them.
+
+Recipe (every choice is seeded):
+  * weights  He-normal, W ~ N(0, 2 / fan_in), numpy PCG64 seeded with `model_seed`
+    (default 0); biases ~ U(-0.05, 0.05).
+  * inputs   U[0,1] for the MLP and LeNet (MNIST-like), N(0,1) per channel for the
+    32x32x3 networks (CIFAR-like); PCG64 seeded with `input_seed` (default 1).
+  * mutants  PCG64 seeded with `mutant_seed` (default 2).  Mutant i: layer uniform over
+    the weighted layers (stress mix: half on layer 0, the rest uniform over the
+    others); operator [GF, NEB, NAI, NS][i % 4]; selection ratio
+    ratios[(i // 4) % len(ratios)]; k = max(1, floor(r * N_l + 0.5)) neurons of layer
+    l drawn without replacement (NS: 2 * max(1, k // 2) neurons, paired in order);
+    GF sigma multiplier 0.1; a 63-bit seed for the operator's random numbers.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+OPS = ("GF", "NEB", "NAI", "NS", "WS", "IDENTITY")
+OP_INDEX = {name: i for i, name in enumerate(OPS)}
+CONFIG_OPS = ("GF", "NEB", "NAI", "NS")
+
+
+@dataclass
+class Node:
+    kind: str                 # conv | dense | maxpool | flatten | add | gap | shortcut
+    inputs: tuple             # node ids; -1 = the model input
+    act: str = "none"         # none | relu
+    kh: int = 1
+    kw: int = 1
+    stride: int = 1
+    pad: int = 0
+    cin: int = 0
+    cout: int = 0
+    W: np.ndarray | None = None   # conv [cout][kh][kw][cin], dense [cout][cin], fp32
+    b: np.ndarray | None = None   # [cout], fp32
+
+
+@dataclass
+class Model:
+    name: str
+    in_shape: tuple           # (H, W, C), NHWC
+    n_classes: int
+    nodes: list = field(default_factory=list)
+
+    def layers(self):
+        """Node ids of the weighted nodes (conv, dense) in node order."""
+        return [v for v, n in enumerate(self.nodes) if n.kind in ("conv", "dense")]
+
+    def n_layers(self):
+        return len(self.layers())
+
+    def layer_width(self, layer):
+        return self.nodes[self.layers()[layer]].cout
+
+
+@dataclass
+class MutantTable:
+    layer: np.ndarray        # int32 [n]
+    op: np.ndarray           # int32 [n], index into OPS
+    n_neurons: np.ndarray    # int32 [n]
+    neuron_off: np.ndarray   # int64 [n]
+    param: np.ndarray        # float32 [n]
+    seed: np.ndarray         # uint64 [n]
+    pool: np.ndarray         # int32 [sum n_neurons]
+    ratio: np.ndarray        # float64 [n] (bookkeeping only)
+
+    def __len__(self):
+        return int(self.layer.shape[0])
+
+    def subset(self, idx):
+        idx = np.asarray(idx, dtype=np.int64)
+        pools, offs, off = [], [], 0
+        for i in idx:
+            a = int(self.neuron_off[i])
+            n = int(self.n_neurons[i])
+            pools.append(self.pool[a:a + n])
+            offs.append(off)
+            off += n
+        pool = np.concatenate(pools).astype(np.int32) if pools else np.zeros(0, np.int32)
+        return MutantTable(self.layer[idx].copy(), self.op[idx].copy(), self.n_neurons[idx].copy(),
+                           np.asarray(offs, np.int64), self.param[idx].copy(), self.seed[idx].copy(),
+                           pool, self.ratio[idx].copy())
+
+
+# ----------------------------------------------------------------- networks --
+
+class _Builder:
+    def __init__(self, name, in_shape, n_classes, seed):
+        self.m = Model(name, tuple(in_shape), n_classes)
+        self.rng = np.random.default_rng(seed)
+        self.shape = {-1: tuple(in_shape)}
+
+    def _add(self, node, shape):
+        self.m.nodes.append(node)
+        v = len(self.m.nodes) - 1
+        self.shape[v] = shape
+        return v
+
+    def _init(self, fan_in, shape_w, cout):
+        W = (self.rng.standard_normal(shape_w) * np.sqrt(2.0 / fan_in)).astype(np.float32)
+        b = self.rng.uniform(-0.05, 0.05, size=cout).astype(np.float32)
+        return W, b
+
+    def conv(self, x, cout, k, stride=1, pad=0, act="relu"):
+        h, w, c = self.shape[x]
+        W, b = self._init(k * k * c, (cout, k, k, c), cout)
+        oh = (h + 2 * pad - k) // stride + 1
+        ow = (w + 2 * pad - k) // stride + 1
+        return self._add(Node("conv", (x,), act, k, k, stride, pad, c, cout, W, b), (oh, ow, cout))
+
+    def dense(self, x, cout, act="relu"):
+        h, w, c = self.shape[x]
+        W, b = self._init(h * w * c, (cout, h * w * c), cout)
+        return self._add(Node("dense", (x,), act, 1, 1, 1, 0, h * w * c, cout, W, b), (1, 1, cout))
+
+    def maxpool(self, x, k=2, stride=2):
+        h, w, c = self.shape[x]
+        return self._add(Node("maxpool", (x,), "none", k, k, stride), ((h - k) // stride + 1, (w - k) // stride + 1, c))
+
+    def flatten(self, x):
+        h, w, c = self.shape[x]
+        return self._add(Node("flatten", (x,)), (1, 1, h * w * c))
+
+    def add(self, a, b, act="relu"):
+        return self._add(Node("add", (a, b), act), self.shape[a])
+
+    def gap(self, x):
+        return self._add(Node("gap", (x,)), (1, 1, self.shape[x][2]))
+
+    def shortcut(self, x, stride, cout):
+        h, w, c = self.shape[x]
+        return self._add(Node("shortcut", (x,), "none", 1, 1, stride, 0, c, cout),
+                         ((h - 1) // stride + 1, (w - 1) // stride + 1, cout))
+
+
+def mlp(seed=0, widths=(784, 128, 64, 10)):
+    """Fully connected 784-128-64-10, ReLU (the paper's FCNN family, Table 1)."""
+    bld = _Builder("mlp", (1, 1, widths[0]), widths[-1], seed)
+    x = -1
+    for i, w in enumerate(widths[1:]):
+        x = bld.dense(x, w, act="relu" if i < len(widths) - 2 else "none")
+    return bld.m
+
+
+def lenet5(seed=0):
+    """LeNet-5 style CNN on 28x28x1 (Table 1): conv5x5(6, pad 2)+ReLU+pool,
+    conv5x5(16, valid)+ReLU+pool, FC 400-120-84-10."""
+    bld = _Builder("lenet5", (28, 28, 1), 10, seed)
+    x = bld.conv(-1, 6, 5, pad=2)
+    x = bld.maxpool(x)
+    x = bld.conv(x, 16, 5, pad=0)
+    x = bld.maxpool(x)
+    x = bld.flatten(x)
+    x = bld.dense(x, 120)
+    x = bld.dense(x, 84)
+    bld.dense(x, 10, act="none")
+    return bld.m
+
+
+def vgg(seed=0):
+    """VGG-style CNN on 32x32x3 with BN folded into the conv biases:
+    [64,64,P][128,128,P][256,256,P], FC 4096-512-10 (8 weighted layers, 3,248,202
+    parameters)."""
+    bld = _Builder("vgg", (32, 32, 3), 10, seed)
+    x = -1
+    for c in (64, 128, 256):
+        x = bld.conv(x, c, 3, pad=1)
+        x = bld.conv(x, c, 3, pad=1)
+        x = bld.maxpool(x)
+    x = bld.flatten(x)
+    x = bld.dense(x, 512)
+    bld.dense(x, 10, act="none")
+    return bld.m
+
+
+def resnet20(seed=0):
+    """ResNet-20 on 32x32x3: stem conv, 3 stages x 3 basic blocks (16/32/64
+    channels, BN folded), parameter-free option-A shortcuts (stride-2 subsampling,
+    zero channels appended), global average pooling, FC 64-10.  19 convs + 1 FC."""
+    bld = _Builder("resnet20", (32, 32, 3), 10, seed)
+    x = bld.conv(-1, 16, 3, pad=1)
+    cin = 16
+    for s, c in enumerate((16, 32, 64)):
+        for blk in range(3):
+            stride = 2 if (s > 0 and blk == 0) else 1
+            a = bld.conv(x, c, 3, stride=stride, pad=1, act="relu")
+            bb = bld.conv(a, c, 3, stride=1, pad=1, act="none")
+            sc = x if (stride == 1 and cin == c) else bld.shortcut(x, stride, c)
+            x = bld.add(bb, sc, act="relu")
+            cin = c
+    x = bld.gap(x)
+    bld.dense(x, 10, act="none")
+    return bld.m
+
+
+MODELS = {"mlp": mlp, "lenet5": lenet5, "vgg": vgg, "resnet20": resnet20}
+
+
+# ------------------------------------------------------------------- inputs --
+
+def inputs(model: Model, n: int, seed: int = 1, dist: str | None = None) -> np.ndarray:
+    """n inputs of the model's shape, [n][H][W][C] float32."""
+    if dist is None:
+        dist = "uniform" if model.in_shape[2] == 1 else "normal"
+    rng = np.random.default_rng(seed)
+    shape = (n,) + tuple(model.in_shape)
+    if dist == "uniform":
+        return rng.random(shape, dtype=np.float32)
+    return rng.standard_normal(shape, dtype=np.float32)
+
+
+# ------------------------------------------------------------------ mutants --
+
+def mutants(model: Model, n: int, seed: int = 2, ratios=(0.01,), ops=CONFIG_OPS,
+            first_layer_share: float | None = None, layers=None) -> MutantTable:
+    """Descriptor table of n single-layer mutants (recipe in the module docstring)."""
+    rng = np.random.default_rng(seed)
+    L = model.n_layers()
+    cand = list(range(L)) if layers is None else list(layers)
+    lay = np.zeros(n, np.int32)
+    opv = np.zeros(n, np.int32)
+    nn = np.zeros(n, np.int32)
+    off = np.zeros(n, np.int64)
+    par = np.zeros(n, np.float32)
+    sd = np.zeros(n, np.uint64)
+    rat = np.zeros(n, np.float64)
+    pool = []
+    pos = 0
+    for i in range(n):
+        if first_layer_share is not None:
+            l = 0 if rng.random() < first_layer_share else int(rng.integers(1, L))
+        else:
+            l = cand[int(rng.integers(0, len(cand)))]
+        op = ops[i % len(ops)]
+        r = ratios[(i // len(ops)) % len(ratios)]
+        N = model.layer_width(l)
+        k = max(1, int(np.floor(r * N + 0.5)))
+        if op == "NS":
+            k = min(2 * max(1, k // 2), N - (N % 2))
+        k = min(k, N)
+        ids = rng.choice(N, size=k, replace=False).astype(np.int32)
+        lay[i] = l
+        opv[i] = OP_INDEX[op]
+        nn[i] = k
+        off[i] = pos
+        par[i] = 0.1 if op == "GF" else 0.0
+        sd[i] = np.uint64(int(rng.integers(0, 2 ** 63 - 1)))
+        rat[i] = r
+        pool.append(ids)
+        pos += k
+    return MutantTable(lay, opv, nn, off, par, sd,
+                       np.concatenate(pool).astype(np.int32) if pool else np.zeros(0, np.int32), rat)
+
+
+def concat(tables) -> MutantTable:
+    """One table holding the rows of several, in order."""
+    tables = list(tables)
+    offs, pos = [], 0
+    for t in tables:
+        offs.append(t.neuron_off + pos)
+        pos += t.pool.size
+    cat = lambda f, dt: np.concatenate([getattr(t, f) for t in tables]).astype(dt) if tables else np.zeros(0, dt)
+    return MutantTable(cat("layer", np.int32), cat("op", np.int32), cat("n_neurons", np.int32),
+                       np.concatenate(offs).astype(np.int64) if tables else np.zeros(0, np.int64),
+                       cat("param", np.float32), cat("seed", np.uint64), cat("pool", np.int32),
+                       cat("ratio", np.float64))
+
+
+def table_from_rows(rows) -> MutantTable:
+    """Build a table from (layer, op_name, neuron_ids, param, seed) tuples."""
+    pool, off, nn = [], [], []
+    for r in rows:
+        off.append(len(pool))
+        nn.append(len(r[2]))
+        pool += list(r[2])
+    n = len(rows)
+    return MutantTable(np.array([r[0] for r in rows], np.int32), np.array([OP_INDEX[r[1]] for r in rows], np.int32),
+                       np.array(nn, np.int32), np.array(off, np.int64),
+                       np.array([r[3] for r in rows], np.float32), np.array([r[4] for r in rows], np.uint64),
+                       np.array(pool, np.int32), np.zeros(n))
+
+
+def stratified(table: MutantTable, model: Model, per_layer_op: int) -> np.ndarray:
+    """Indices of a stratified subsample: the first `per_layer_op` mutants of every
+    (layer, operator) pair, in table order."""
+    picked = []
+    seen = {}
+    for i in range(len(table)):
+        key = (int(table.layer[i]), int(table.op[i]))
+        if seen.get(key, 0) < per_layer_op:
+            seen[key] = seen.get(key, 0) + 1
+            picked.append(i)
+    return np.asarray(picked, np.int64)
+
+
+# ------------------------------------------------------------ named configs --
+
+@dataclass
+class Workload:
+    name: str
+    model: Model
+    X: np.ndarray
+    table: MutantTable
+    labels: np.ndarray | None = None
+
+
+CONFIGS = {
+    # name: (model, n_inputs, n_mutants, ratios, first-layer share)
+    "mlp": ("mlp", 1000, 200, (0.01,), None),
+    "lenet5": ("lenet5", 10000, 2000, (0.01,), None),
+    "vgg": ("vgg", 10000, 5000, (0.005, 0.01, 0.02, 0.05), None),
+    "resnet20": ("resnet20", 10000, 5000, (0.01,), None),
+    "vgg_stress": ("vgg", 20000, 20000, (0.001, 0.01, 0.05, 0.10), 0.5),
+}
+
+
+def workload(name: str, n_inputs: int | None = None, n_mutants: int | None = None,
+             model_seed: int = 0, input_seed: int = 1, mutant_seed: int = 2) -> Workload:
+    """A named configuration, optionally truncated to its first inputs / mutants
+    (the truncated table equals the prefix of the full one)."""
+    mname, n_in, n_mut, ratios, skew = CONFIGS[name]
+    model = MODELS[mname](model_seed)
+    n_in = n_in if n_inputs is None else n_inputs
+    n_mut = n_mut if n_mutants is None else n_mutants
+    X = inputs(model, n_in, input_seed)
+    table = mutants(model, n_mut, mutant_seed, ratios=ratios, first_layer_share=skew)
+    return Workload(name, model, X, table)
