@@ -1,0 +1,234 @@
+/*
+ * mure.h -- C ABI of the GB300 (sm_103a) library for memoized DNN mutation testing.
+ *
+ * The library evaluates weight-level mutants of one feed-forward network on a test
+ * input set and fills the mutants x inputs kill matrix and the mutation score
+ * (Ghanbari et al., "Provably Lossless Acceleration of DNN Mutation Testing via
+ * Memoization", PACMSE/ISSTA 2026; Algorithm 1, Sec. 3 and Sec. 5.2).
+ *
+ * Memoized mode follows Algorithm 1: the original network's activations are computed
+ * once and kept in device memory (the memo table of Algorithm 3, extended to every
+ * layer), mutants are grouped by their first mutated layer (the clusters of
+ * Algorithm 1, lines 3-9), and each mutant runs only from its mutated layer onward
+ * on memo rows (the chopped mutant of Algorithm 4).  Vanilla mode runs every mutant
+ * end to end from the inputs (the paper's exhaustive baseline, Sec. 5.1).
+ *
+ * Conventions for every call
+ *   - Tensors are fp32, NHWC, densely packed, row-major.
+ *   - A status other than MURE_OK leaves every output buffer untouched unless the
+ *     call says otherwise; mure_last_error() then holds a one-line reason.
+ *   - All argument validation happens before any device work is queued.
+ *   - Calls on one context are not thread-safe; use one context per host thread.
+ *   - Every call is synchronous with respect to the host: when it returns, its
+ *     results are in the caller's buffers.  Device work runs on the context's stream.
+ *   - Pointers documented as "host" must be host memory; "device" ones must be memory
+ *     of the context's device.  The caller keeps ownership of everything it passes.
+ */
+#ifndef MURE_H
+#define MURE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MURE_OK = 0,
+    MURE_ERR_INVALID_ARG = 1, /* a bad pointer, size, index, graph or descriptor */
+    MURE_ERR_UNSUPPORTED = 2, /* valid but outside what the kernels implement */
+    MURE_ERR_OOM = 3,         /* device allocation failed (nothing was launched) */
+    MURE_ERR_CUDA = 4,        /* a CUDA runtime call failed */
+    MURE_ERR_TIMEOUT = 5      /* a device-side bounded wait gave up */
+} mure_status;
+
+/* Network node kinds (Sec. 4: a network is a DAG of layer functions). */
+enum {
+    MURE_NODE_CONV2D = 0,   /* zero-padded 2-D convolution + bias + activation */
+    MURE_NODE_DENSE = 1,    /* fully connected + bias + activation */
+    MURE_NODE_MAXPOOL2D = 2,/* max pooling, window kh x kw, stride `stride` (floor) */
+    MURE_NODE_FLATTEN = 3,  /* reshape to a vector (no data movement in NHWC) */
+    MURE_NODE_ADD = 4,      /* element-wise sum of in0 and in1 + activation */
+    MURE_NODE_GAP = 5,      /* global average pooling over H and W */
+    MURE_NODE_SHORTCUT = 6  /* parameter-free residual shortcut: subsample by
+                               `stride`, zero channels appended up to `cout` */
+};
+enum { MURE_ACT_NONE = 0, MURE_ACT_RELU = 1 };
+
+/* Mutation operators (Sec. 3.1; DeepMutation's weight-level mutators).  Neuron j of
+ * a weighted layer is its output channel / output unit j (Sec. 2.1).
+ *   GF  Gaussian fuzzing: w[j][f] += sigma * n, n ~ N(0,1), sigma = param x the
+ *       population standard deviation of the layer's weights (bias excluded).
+ *   NEB neuron effect blocking: the output of neuron j is 0.
+ *   NAI neuron activation inverse: the pre-activation of neuron j is negated.
+ *   NS  neuron switch: neurons j0, j1 (consecutive pool entries) exchange filters
+ *       and biases; n_neurons must be even.
+ *   WS  weight shuffling: the fan-in weights of neuron j are permuted.
+ *   IDENTITY no change (neurons ignored).
+ * GF noise and WS permutations come from the counter-based SplitMix64 generator
+ * (Steele, Lea, Flood, OOPSLA 2014): the stream of neuron slot q of a mutant with
+ * seed s is seeded with draw q of a generator seeded with s; GF's standard normals
+ * come from the Box-Muller transform of draw pairs (2p, 2p+1) in fp64 (cosine for
+ * even, sine for odd index), rounded to fp32 after scaling by sigma; WS uses
+ * Fisher-Yates from the last index down, j = floor(u (i+1)) with u the top 53 bits. */
+enum { MURE_OP_GF = 0, MURE_OP_NEB = 1, MURE_OP_NAI = 2, MURE_OP_NS = 3, MURE_OP_WS = 4, MURE_OP_IDENTITY = 5 };
+
+/* Arithmetic of the layer kernels.  FP32: fp32 FMA chains on the CUDA cores.
+ * TF32X3: tensor cores (tcgen05), fp32 operands split into two TF32 halves, three
+ * products per pair.  BF16: tensor cores, bf16 operands, fp32 accumulation (the
+ * reduced-precision variant).  One model uses one arithmetic for every layer
+ * computation (cache build, vanilla prefix and suffix), so memoized and vanilla
+ * results stay bit-identical under every mode. */
+enum { MURE_PREC_FP32 = 0, MURE_PREC_TF32X3 = 1, MURE_PREC_BF16 = 2 };
+
+/* One node.  in0/in1 are node ids (< this node's id) or -1 for the network input.
+ * Weighted nodes (CONV2D, DENSE) are numbered 0..L-1 in node order: these numbers
+ * are the "layers" of mutant descriptors.  W: conv [cout][kh][kw][cin], dense
+ * [cout][cin]; b: [cout].  W and b are host pointers, copied by mure_model_load. */
+typedef struct {
+    int32_t kind, act, in0, in1;
+    int32_t kh, kw, stride, pad;
+    int32_t cin, cout;
+    const float *W;
+    const float *b;
+} mure_node;
+
+/* Network description.  Nodes in topological order; the last node is the output
+ * (the logits), of size n_classes.  The supported shape of the graph: each
+ * weighted node is followed, before the next weighted node reads it, by at most one
+ * ADD (its other input a network input, a block input or a SHORTCUT of one), then
+ * optional MAXPOOL2D (2x2, stride 2), FLATTEN and GAP nodes; the output node is
+ * the last weighted node.  Other graphs return MURE_ERR_UNSUPPORTED. */
+typedef struct {
+    int32_t in_h, in_w, in_c, n_classes;
+    int32_t n_nodes;
+    int32_t precision; /* MURE_PREC_* */
+    const mure_node *nodes;
+} mure_model_desc;
+
+/* One mutant descriptor (the mutant map of Algorithm 1, with mu(M') = {layer}). */
+typedef struct {
+    int32_t layer;      /* first (and only) mutated weighted layer, 0..L-1 */
+    int32_t op;         /* MURE_OP_* */
+    int32_t n_neurons;  /* neuron ids at neuron_pool[neuron_off .. +n_neurons) */
+    int32_t reserved;   /* must be 0 */
+    int64_t neuron_off;
+    float param;        /* GF: sigma multiplier (e.g. 0.1); ignored otherwise */
+    float reserved2;    /* must be 0 */
+    uint64_t seed;      /* GF / WS random stream */
+} mure_mutant;
+
+/* Device allocator.  When given to mure_create, every device allocation of the
+ * library goes through it (for instance a framework's caching allocator); when
+ * NULL, the library uses cudaMallocAsync / cudaFreeAsync on the context stream.
+ * alloc returns NULL on failure. */
+typedef struct {
+    void *(*alloc)(size_t bytes, void *stream, void *user);
+    void (*free)(void *ptr, void *stream, void *user);
+    void *user;
+} mure_allocator;
+
+typedef struct {
+    int32_t outputs_on_device; /* kill_bits / logits_out are device pointers */
+    int32_t reserved;
+    int64_t workspace_bytes;   /* cap on per-batch scratch (0: 8 GiB) */
+    float *logits_out;         /* nullable; [n_mutants][n_inputs][n_classes]: every
+                                  mutant's logits (for parity checks; slows the run) */
+} mure_eval_opts;
+
+typedef struct {
+    double ms_total;        /* device time of the whole call (CUDA events) */
+    double ms_expand;       /* descriptor expansion (GF noise, WS shuffles) */
+    double ms_suffix;       /* delta + suffix + epilogue kernels */
+    double ms_score;        /* score reduction */
+    int64_t n_rows;         /* (mutant, input) pairs evaluated */
+    int64_t n_near_ties;    /* rows whose top-2 logit margin < 1e-4 |max logit| */
+    int64_t n_groups;       /* first-mutated-layer groups with >= 1 mutant */
+    int64_t n_batches;      /* (group, mutant chunk, input tile) batches */
+    int64_t kernel_launches;/* library kernels launched by the call */
+    int64_t flops;          /* analytic FLOPs of the layer kernels that ran */
+} mure_eval_stats;
+
+typedef struct mure_ctx mure_ctx;
+typedef struct mure_model mure_model;
+typedef struct mure_cache mure_cache;
+
+/* Create a context on CUDA device `device` that queues all work on `cuda_stream`
+ * (a cudaStream_t; NULL = the legacy default stream).  alloc may be NULL.
+ * Errors: INVALID_ARG (out == NULL, bad device), CUDA. */
+mure_status mure_create(int device, void *cuda_stream, const mure_allocator *alloc, mure_ctx **out);
+
+/* Destroy a context.  Models and caches made from it must be freed first. */
+void mure_destroy(mure_ctx *ctx);
+
+/* The reason for the last failed call on this context ("" if none).  Valid until
+ * the next call on the context. */
+const char *mure_last_error(const mure_ctx *ctx);
+
+/* Copy a network to the device and compile it into stages (Algorithm 2: the
+ * dependence graph is read from the nodes' inputs).  Errors: INVALID_ARG
+ * (inconsistent shapes, bad ids, NULL weights), UNSUPPORTED (graph outside the
+ * supported shape, n_classes > 32, unknown precision), OOM, CUDA. */
+mure_status mure_model_load(mure_ctx *ctx, const mure_model_desc *desc, mure_model **out);
+void mure_model_free(mure_model *model);
+
+/* Number of weighted layers L of a loaded model (or -1 for NULL). */
+int32_t mure_model_n_layers(const mure_model *model);
+
+/* Build the prefix-activation cache (the memo table, Algorithm 3 and Algorithm 1
+ * lines 11-12, kept for every layer so every cluster shares one table): one forward
+ * pass of the original network over X [n_inputs][in_h][in_w][in_c] storing, per
+ * input, every weighted layer's input and pre-activation output, plus the original
+ * logits, predictions and labels.  labels [n_inputs] in [0, n_classes) or NULL (then
+ * label = original prediction, and kill reduces to "prediction changed").  X and
+ * labels are device pointers when x_on_device != 0, else host pointers.  n_inputs
+ * may be 0.  Errors: INVALID_ARG (NULL X with n_inputs > 0, label out of range),
+ * OOM, CUDA. */
+mure_status mure_build_prefix_cache(mure_model *model, const float *X, int64_t n_inputs, const int32_t *labels,
+                                    int x_on_device, mure_cache **out);
+void mure_cache_free(mure_cache *cache);
+
+/* Original logits [n_inputs][n_classes] and predictions [n_inputs] held by a cache,
+ * copied to host buffers (either may be NULL). */
+mure_status mure_cache_outputs(mure_cache *cache, float *logits, int32_t *pred);
+
+/* Memoized mutation testing (Algorithm 1).  table [n_mutants] and neuron_pool
+ * [pool_len] are host arrays.  kill_bits [n_mutants][ceil(n_inputs/64)] receives
+ * bit t of row i = kill(mutant i, input t) (Sec. 5.2: the original predicts
+ * label(t) and the mutant does not), least significant bit first; padding bits are
+ * 0.  score_killed_frac = killed mutants / n_mutants; score_deepmutation =
+ * sum_i |killingLabels(i)| / (n_mutants |L|), L the labels present in the inputs
+ * (Sec. 5.2).  Either score pointer may be NULL; stats may be NULL; opts may be
+ * NULL (host outputs, defaults).  n_mutants may be 0.  Errors: INVALID_ARG (bad
+ * descriptor: layer, op, neuron id out of range or repeated, odd NS count,
+ * non-zero reserved fields, pool range), OOM, CUDA, TIMEOUT. */
+mure_status mure_eval_mutants(mure_cache *cache, const mure_mutant *table, int64_t n_mutants,
+                              const int32_t *neuron_pool, int64_t pool_len, const mure_eval_opts *opts,
+                              uint64_t *kill_bits, double *score_killed_frac, double *score_deepmutation,
+                              mure_eval_stats *stats);
+
+/* Vanilla mutation testing (the paper's exhaustive baseline): every mutant is run
+ * end to end from X with no activation reuse across mutants, through the same layer
+ * kernels, so its outputs equal mure_eval_mutants' bit for bit (Theorem 1).
+ * Arguments as in mure_build_prefix_cache followed by mure_eval_mutants. */
+mure_status mure_eval_vanilla(mure_model *model, const float *X, int64_t n_inputs, const int32_t *labels,
+                              int x_on_device, const mure_mutant *table, int64_t n_mutants,
+                              const int32_t *neuron_pool, int64_t pool_len, const mure_eval_opts *opts,
+                              uint64_t *kill_bits, double *score_killed_frac, double *score_deepmutation,
+                              mure_eval_stats *stats);
+
+/* The expanded per-neuron patch of each GF / WS mutant, for checking the random
+ * number streams: for mutant i and neuron slot q, F_l fp32 values at out +
+ * offset[i] + q * F_l, where offset is returned in offsets [n_mutants] (-1 for other
+ * operators).  GF: the noise added to each fan-in weight, fl32(sigma * n_f).  WS:
+ * the permuted weights W[j][perm[f]].  out_len is the capacity of out (host);
+ * Errors: INVALID_ARG (descriptors, or out too small), OOM, CUDA. */
+mure_status mure_expand_patches(mure_model *model, const mure_mutant *table, int64_t n_mutants,
+                                const int32_t *neuron_pool, int64_t pool_len, float *out, int64_t out_len,
+                                int64_t *offsets);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MURE_H */

@@ -1,0 +1,971 @@
+// C ABI of the library: contexts, model compilation (graph -> stages), the prefix
+// activation cache, and the memoized / vanilla mutation-testing schedulers.
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <numeric>
+
+#include "common.cuh"
+#include "device_util.cuh"
+
+using namespace mure;
+
+namespace {
+
+// ------------------------------------------------------------------ plumbing --
+
+struct Fail {
+    mure_status st;
+};
+
+void set_err(mure_ctx *c, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
+void set_err(mure_ctx *c, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (c) c->err = buf;
+}
+
+#define FAILIF(cond, ctx, status, ...)        \
+    do {                                      \
+        if (cond) {                           \
+            set_err(ctx, __VA_ARGS__);        \
+            throw Fail{status};               \
+        }                                     \
+    } while (0)
+
+#define CK(ctx, call)                                                                              \
+    do {                                                                                           \
+        cudaError_t e_ = (call);                                                                   \
+        FAILIF(e_ != cudaSuccess, ctx, MURE_ERR_CUDA, "%s: %s", #call, cudaGetErrorString(e_));    \
+    } while (0)
+
+void *dalloc(mure_ctx *c, size_t bytes)
+{
+    if (bytes == 0) bytes = 16;
+    void *p = nullptr;
+    if (c->has_alloc) {
+        p = c->alloc.alloc(bytes, (void *)c->stream, c->alloc.user);
+    } else {
+        if (cudaMallocAsync(&p, bytes, c->stream) != cudaSuccess) {
+            cudaGetLastError();
+            p = nullptr;
+        }
+    }
+    FAILIF(!p, c, MURE_ERR_OOM, "device allocation of %zu bytes failed", bytes);
+    return p;
+}
+
+void dfree(mure_ctx *c, void *p)
+{
+    if (!p) return;
+    if (c->has_alloc) c->alloc.free(p, (void *)c->stream, c->alloc.user);
+    else cudaFreeAsync(p, c->stream);
+}
+
+// Device allocations owned by one call (freed on every exit path).
+struct Scratch {
+    mure_ctx *c;
+    std::vector<void *> ptrs;
+    explicit Scratch(mure_ctx *ctx) : c(ctx) {}
+    template <class T>
+    T *get(size_t n)
+    {
+        void *p = dalloc(c, n * sizeof(T));
+        ptrs.push_back(p);
+        return static_cast<T *>(p);
+    }
+    ~Scratch()
+    {
+        for (void *p : ptrs) dfree(c, p);
+    }
+};
+
+int64_t round_up(int64_t n, int64_t a) { return (n + a - 1) / a * a; }
+
+template <class F>
+mure_status run(mure_ctx *c, F &&fn)
+{
+    if (c) c->err.clear();
+    try {
+        fn();
+    } catch (const Fail &f) {
+        return f.st;
+    } catch (const std::bad_alloc &) {
+        set_err(c, "host allocation failed");
+        return MURE_ERR_OOM;
+    }
+    return MURE_OK;
+}
+
+void check_launch(mure_ctx *c)
+{
+    cudaError_t e = cudaGetLastError();
+    FAILIF(e != cudaSuccess, c, MURE_ERR_CUDA, "kernel launch: %s", cudaGetErrorString(e));
+}
+
+// ---------------------------------------------------------- model compilation --
+
+struct Shape {
+    int h, w, c;
+};
+
+bool weighted(int k) { return k == MURE_NODE_CONV2D || k == MURE_NODE_DENSE; }
+
+// Output shapes of all nodes (same rules as the network definition in the header).
+std::vector<Shape> node_shapes(mure_ctx *c, const mure_model_desc *d)
+{
+    std::vector<Shape> s(d->n_nodes);
+    const Shape in{d->in_h, d->in_w, d->in_c};
+    for (int v = 0; v < d->n_nodes; ++v) {
+        const mure_node &n = d->nodes[v];
+        FAILIF(n.in0 < -1 || n.in0 >= v, c, MURE_ERR_INVALID_ARG, "node %d: input %d is not an earlier node", v, n.in0);
+        const Shape a = n.in0 < 0 ? in : s[n.in0];
+        Shape o = a;
+        switch (n.kind) {
+        case MURE_NODE_CONV2D:
+            FAILIF(n.cin != a.c || n.stride < 1 || n.kh < 1 || n.kw < 1 || n.pad < 0 || n.cout < 1, c,
+                   MURE_ERR_INVALID_ARG, "node %d: bad conv geometry", v);
+            o = {(a.h + 2 * n.pad - n.kh) / n.stride + 1, (a.w + 2 * n.pad - n.kw) / n.stride + 1, n.cout};
+            FAILIF(o.h < 1 || o.w < 1, c, MURE_ERR_INVALID_ARG, "node %d: empty conv output", v);
+            FAILIF(!n.W || !n.b, c, MURE_ERR_INVALID_ARG, "node %d: NULL weights", v);
+            break;
+        case MURE_NODE_DENSE:
+            FAILIF(n.cin != a.h * a.w * a.c || n.cout < 1, c, MURE_ERR_INVALID_ARG, "node %d: dense fan-in mismatch", v);
+            FAILIF(!n.W || !n.b, c, MURE_ERR_INVALID_ARG, "node %d: NULL weights", v);
+            o = {1, 1, n.cout};
+            break;
+        case MURE_NODE_MAXPOOL2D:
+            FAILIF(n.kh < 1 || n.kw < 1 || n.stride < 1, c, MURE_ERR_INVALID_ARG, "node %d: bad pool", v);
+            o = {(a.h - n.kh) / n.stride + 1, (a.w - n.kw) / n.stride + 1, a.c};
+            FAILIF(o.h < 1 || o.w < 1, c, MURE_ERR_INVALID_ARG, "node %d: empty pool output", v);
+            break;
+        case MURE_NODE_FLATTEN:
+            o = {1, 1, a.h * a.w * a.c};
+            break;
+        case MURE_NODE_ADD: {
+            FAILIF(n.in1 < -1 || n.in1 >= v, c, MURE_ERR_INVALID_ARG, "node %d: bad second input", v);
+            const Shape b = n.in1 < 0 ? in : s[n.in1];
+            FAILIF(a.h != b.h || a.w != b.w || a.c != b.c, c, MURE_ERR_INVALID_ARG, "node %d: add shape mismatch", v);
+            break;
+        }
+        case MURE_NODE_GAP:
+            o = {1, 1, a.c};
+            break;
+        case MURE_NODE_SHORTCUT:
+            FAILIF(n.stride < 1 || n.cout < a.c, c, MURE_ERR_INVALID_ARG, "node %d: bad shortcut", v);
+            o = {(a.h - 1) / n.stride + 1, (a.w - 1) / n.stride + 1, n.cout};
+            break;
+        default:
+            FAILIF(true, c, MURE_ERR_INVALID_ARG, "node %d: unknown kind %d", v, n.kind);
+        }
+        FAILIF(n.act != MURE_ACT_NONE && n.act != MURE_ACT_RELU, c, MURE_ERR_INVALID_ARG, "node %d: bad activation", v);
+        s[v] = o;
+    }
+    return s;
+}
+
+TensorDim tdim(Shape s)
+{
+    TensorDim t{s.h, s.w, s.c, (int64_t)s.h * s.w * s.c, 0};
+    t.stride = round4(t.size);
+    return t;
+}
+
+// Group the graph into stages: weighted node + its tail of ADD / MAXPOOL / FLATTEN
+// / GAP up to the next weighted node (the dependence graph of Algorithm 2 read off
+// the nodes' inputs).
+void compile(mure_ctx *c, const mure_model_desc *d, mure_model *m)
+{
+    const std::vector<Shape> shp = node_shapes(c, d);
+    const Shape in{d->in_h, d->in_w, d->in_c};
+    auto shape_of = [&](int id) { return id < 0 ? in : shp[id]; };
+    std::vector<int> wn;
+    for (int v = 0; v < d->n_nodes; ++v)
+        if (weighted(d->nodes[v].kind)) wn.push_back(v);
+    FAILIF(wn.empty(), c, MURE_ERR_INVALID_ARG, "the network has no weighted node");
+    FAILIF(wn.back() != d->n_nodes - 1, c, MURE_ERR_UNSUPPORTED, "the output node must be the last weighted node");
+    const int L = (int)wn.size();
+    const Shape outs = shp[d->n_nodes - 1];
+    FAILIF(outs.h * outs.w * outs.c != d->n_classes, c, MURE_ERR_INVALID_ARG, "output size %d != n_classes %d",
+           outs.h * outs.w * outs.c, d->n_classes);
+    FAILIF(d->n_classes > kMaxClasses || d->n_classes < 1, c, MURE_ERR_UNSUPPORTED, "n_classes must be 1..%d",
+           kMaxClasses);
+    // stage_in[s] = node whose output is x_s (-1 = the network input)
+    std::vector<int> stage_in(L + 1, -2);
+    stage_in[0] = -1;
+    std::vector<char> used(d->n_nodes, 0);
+    m->st.resize(L);
+    m->xd.resize(L + 1);
+    m->zd.resize(L);
+    m->xd[0] = tdim(in);
+    for (int v = 0; v < L; ++v) {
+        const int nid = wn[v];
+        const mure_node &n = d->nodes[nid];
+        FAILIF(n.in0 != stage_in[v], c, MURE_ERR_UNSUPPORTED, "weighted node %d does not read the previous stage", nid);
+        used[nid] = 1;
+        Stage &S = m->st[v];
+        S = Stage{};
+        S.kind = n.kind;
+        const Shape a = shape_of(n.in0), z = shp[nid];
+        if (n.kind == MURE_NODE_CONV2D) {
+            S.ih = a.h; S.iw = a.w; S.ic = a.c; S.kh = n.kh; S.kw = n.kw; S.stride = n.stride; S.pad = n.pad;
+        } else {
+            S.ih = 1; S.iw = 1; S.ic = n.cin; S.kh = 1; S.kw = 1; S.stride = 1; S.pad = 0;
+        }
+        S.oh = z.h; S.ow = z.w; S.oc = z.c;
+        S.K = S.kh * S.kw * S.ic;
+        S.act1 = n.act;
+        S.skip_src = -1; S.sc_stride = 1; S.sc_c = 0; S.sk_w = 0;
+        S.macs = (int64_t)S.oh * S.ow * S.oc * S.K;
+        m->zd[v] = tdim(z);
+        int cur = nid;
+        const int end = v + 1 < L ? wn[v + 1] : d->n_nodes;
+        int phase = 0;  // 0: before ADD, 1: after ADD, 2: after pool, 3: after gap
+        for (int u = nid + 1; u < end; ++u) {
+            const mure_node &t = d->nodes[u];
+            if (t.kind == MURE_NODE_SHORTCUT) continue;  // a side branch, checked by its ADD
+            FAILIF(v + 1 == L, c, MURE_ERR_UNSUPPORTED, "nodes after the output layer");
+            used[u] = 1;
+            if (t.kind == MURE_NODE_ADD) {
+                FAILIF(phase != 0 || (t.in0 != cur && t.in1 != cur), c, MURE_ERR_UNSUPPORTED,
+                       "node %d: unsupported add placement", u);
+                int other = t.in0 == cur ? t.in1 : t.in0;
+                int sc_stride = 1;
+                if (other >= 0 && d->nodes[other].kind == MURE_NODE_SHORTCUT) {
+                    used[other] = 1;
+                    sc_stride = d->nodes[other].stride;
+                    other = d->nodes[other].in0;
+                }
+                int src = -1;
+                for (int s2 = 0; s2 <= v; ++s2)
+                    if (stage_in[s2] == other) src = s2;
+                FAILIF(src < 0, c, MURE_ERR_UNSUPPORTED, "node %d: skip input is not a stage input", u);
+                S.has_add = 1; S.skip_src = src; S.sc_stride = sc_stride;
+                S.sc_c = m->xd[src].c; S.sk_w = m->xd[src].w;
+                S.act2 = t.act;
+                phase = 1;
+            } else if (t.kind == MURE_NODE_MAXPOOL2D) {
+                FAILIF(t.in0 != cur || phase > 1 || t.kh != 2 || t.kw != 2 || t.stride != 2, c, MURE_ERR_UNSUPPORTED,
+                       "node %d: only one 2x2 stride-2 max pool per stage", u);
+                FAILIF(t.act != MURE_ACT_NONE, c, MURE_ERR_UNSUPPORTED, "node %d: activation on a pool", u);
+                S.pool = 1;
+                phase = 2;
+            } else if (t.kind == MURE_NODE_FLATTEN) {
+                FAILIF(t.in0 != cur, c, MURE_ERR_UNSUPPORTED, "node %d: flatten off the chain", u);
+            } else if (t.kind == MURE_NODE_GAP) {
+                FAILIF(t.in0 != cur || phase > 2, c, MURE_ERR_UNSUPPORTED, "node %d: unsupported gap", u);
+                FAILIF(t.act != MURE_ACT_NONE, c, MURE_ERR_UNSUPPORTED, "node %d: activation on a gap", u);
+                S.gap = 1;
+                phase = 3;
+            } else {
+                FAILIF(true, c, MURE_ERR_UNSUPPORTED, "node %d: unsupported node in a stage tail", u);
+            }
+            cur = u;
+        }
+        const Shape y = shp[cur];
+        S.yh = y.h; S.yw = y.w; S.yc = y.c;
+        stage_in[v + 1] = cur;
+        m->xd[v + 1] = tdim(y);
+        FAILIF(S.yc != S.oc && !S.gap && !(S.yh == 1 && S.yw == 1), c, MURE_ERR_UNSUPPORTED, "stage %d channels", v);
+    }
+    for (int u = 0; u < d->n_nodes; ++u)
+        FAILIF(!used[u], c, MURE_ERR_UNSUPPORTED, "node %d is not part of a supported stage", u);
+    m->L = L;
+    m->n_classes = d->n_classes;
+}
+
+// --------------------------------------------------------------- descriptors --
+
+struct Groups {
+    std::vector<int32_t> order;       // mutant ids grouped by layer (stable)
+    std::vector<int64_t> begin;       // [L+1] group boundaries in `order`
+};
+
+void check_table(mure_ctx *c, const mure_model *m, const mure_mutant *t, int64_t n, const int32_t *pool,
+                 int64_t pool_len)
+{
+    FAILIF(n < 0 || pool_len < 0, c, MURE_ERR_INVALID_ARG, "negative sizes");
+    FAILIF(n > 0 && !t, c, MURE_ERR_INVALID_ARG, "NULL mutant table");
+    FAILIF(pool_len > 0 && !pool, c, MURE_ERR_INVALID_ARG, "NULL neuron pool");
+    FAILIF(n > INT32_MAX, c, MURE_ERR_UNSUPPORTED, "more than 2^31 mutants");
+    std::vector<int64_t> seen;
+    for (int64_t i = 0; i < n; ++i) {
+        const mure_mutant &u = t[i];
+        FAILIF(u.layer < 0 || u.layer >= m->L, c, MURE_ERR_INVALID_ARG, "mutant %lld: layer %d out of range",
+               (long long)i, u.layer);
+        FAILIF(u.op < MURE_OP_GF || u.op > MURE_OP_IDENTITY, c, MURE_ERR_INVALID_ARG, "mutant %lld: bad op", (long long)i);
+        FAILIF(u.reserved != 0 || u.reserved2 != 0.f, c, MURE_ERR_INVALID_ARG, "mutant %lld: reserved fields", (long long)i);
+        FAILIF(u.n_neurons < 0 || u.neuron_off < 0 || u.neuron_off + u.n_neurons > pool_len, c, MURE_ERR_INVALID_ARG,
+               "mutant %lld: neuron range outside the pool", (long long)i);
+        FAILIF(u.op == MURE_OP_NS && (u.n_neurons & 1), c, MURE_ERR_INVALID_ARG, "mutant %lld: odd NS neuron count",
+               (long long)i);
+        const int oc = m->st[u.layer].oc;
+        seen.assign(pool + u.neuron_off, pool + u.neuron_off + u.n_neurons);
+        for (int64_t q = 0; q < u.n_neurons; ++q)
+            FAILIF(seen[q] < 0 || seen[q] >= oc, c, MURE_ERR_INVALID_ARG, "mutant %lld: neuron %lld out of range",
+                   (long long)i, (long long)seen[q]);
+        std::sort(seen.begin(), seen.end());
+        FAILIF(std::adjacent_find(seen.begin(), seen.end()) != seen.end(), c, MURE_ERR_INVALID_ARG,
+               "mutant %lld: repeated neuron", (long long)i);
+    }
+}
+
+Groups group_by_layer(const mure_model *m, const mure_mutant *t, int64_t n)
+{
+    Groups g;
+    g.begin.assign(m->L + 1, 0);
+    for (int64_t i = 0; i < n; ++i) g.begin[t[i].layer + 1]++;
+    for (int l = 0; l < m->L; ++l) g.begin[l + 1] += g.begin[l];
+    std::vector<int64_t> pos(g.begin.begin(), g.begin.end() - 1);
+    g.order.resize(n);
+    for (int64_t i = 0; i < n; ++i) g.order[pos[t[i].layer]++] = (int32_t)i;
+    return g;
+}
+
+// Descriptor arrays in group order, uploaded to the device in one copy.
+struct DevTable {
+    int32_t *op, *nn, *ids, *mid;
+    int64_t *noff, *poff;
+    float *patch;
+    int64_t n_jobs, patch_len;
+    std::vector<int> kmax_layer;
+};
+
+DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_mutant *t, int64_t n,
+                      const int32_t *pool, int64_t pool_len, const Groups &g, int ws_as_weights, float *patch_out,
+                      int64_t *ids_from_group)
+{
+    DevTable dt{};
+    std::vector<int32_t> op(n), nn(n), mid(n);
+    std::vector<int64_t> noff(n), poff(n, -1);
+    std::vector<SlotJob> jobs;
+    int64_t plen = 0, perm_len = 0;
+    for (int64_t k = 0; k < n; ++k) {
+        const int32_t i = g.order[k];
+        const mure_mutant &u = t[i];
+        op[k] = u.op;
+        nn[k] = u.op == MURE_OP_IDENTITY ? 0 : u.n_neurons;
+        noff[k] = u.neuron_off;
+        mid[k] = i;
+        if ((u.op == MURE_OP_GF || u.op == MURE_OP_WS) && u.n_neurons > 0) {
+            const int F = m->st[u.layer].K;
+            poff[k] = plen;
+            for (int q = 0; q < u.n_neurons; ++q) {
+                SlotJob jb{};
+                jb.layer = u.layer; jb.op = u.op; jb.F = F; jb.j = pool[u.neuron_off + q]; jb.q = q;
+                jb.param = u.param; jb.seed = u.seed;
+                jb.out_off = plen + (int64_t)q * F;
+                jb.perm_off = perm_len;
+                if (u.op == MURE_OP_WS) perm_len += F;
+                jobs.push_back(jb);
+            }
+            plen += (int64_t)u.n_neurons * F;
+        }
+        if (ids_from_group) ids_from_group[i] = poff[k];
+    }
+    dt.n_jobs = (int64_t)jobs.size();
+    dt.patch_len = plen;
+    // one staging buffer, one H2D copy
+    const size_t b_op = n * 4, b_nn = n * 4, b_mid = n * 4, b_noff = n * 8, b_poff = n * 8;
+    const size_t b_ids = (size_t)std::max<int64_t>(pool_len, 1) * 4, b_jobs = jobs.size() * sizeof(SlotJob);
+    size_t off = 0;
+    auto place = [&](size_t b) { size_t o = off; off = round_up(off + b, 256); return o; };
+    const size_t o_op = place(b_op), o_nn = place(b_nn), o_mid = place(b_mid), o_noff = place(b_noff),
+                 o_poff = place(b_poff), o_ids = place(b_ids), o_jobs = place(b_jobs);
+    std::vector<char> host(off);
+    memcpy(host.data() + o_op, op.data(), b_op);
+    memcpy(host.data() + o_nn, nn.data(), b_nn);
+    memcpy(host.data() + o_mid, mid.data(), b_mid);
+    memcpy(host.data() + o_noff, noff.data(), b_noff);
+    memcpy(host.data() + o_poff, poff.data(), b_poff);
+    if (pool_len > 0) memcpy(host.data() + o_ids, pool, pool_len * 4);
+    if (!jobs.empty()) memcpy(host.data() + o_jobs, jobs.data(), b_jobs);
+    char *dev = sc.get<char>(off);
+    CK(c, cudaMemcpyAsync(dev, host.data(), off, cudaMemcpyHostToDevice, c->stream));
+    dt.op = (int32_t *)(dev + o_op);
+    dt.nn = (int32_t *)(dev + o_nn);
+    dt.mid = (int32_t *)(dev + o_mid);
+    dt.noff = (int64_t *)(dev + o_noff);
+    dt.poff = (int64_t *)(dev + o_poff);
+    dt.ids = (int32_t *)(dev + o_ids);
+    dt.patch = plen ? sc.get<float>(plen) : nullptr;
+    if (!jobs.empty()) {
+        std::vector<const float *> Wp(m->L);
+        for (int l = 0; l < m->L; ++l) Wp[l] = m->st[l].W;
+        const float **Wd = sc.get<const float *>(m->L);
+        CK(c, cudaMemcpyAsync(Wd, Wp.data(), m->L * sizeof(float *), cudaMemcpyHostToDevice, c->stream));
+        ExpandArgs ea{};
+        ea.jobs = (const SlotJob *)(dev + o_jobs);
+        ea.n_jobs = dt.n_jobs;
+        ea.sigma = m->sigma_dev;
+        ea.W = Wd;
+        ea.patch = dt.patch;
+        ea.perm = perm_len ? sc.get<int32_t>(perm_len) : nullptr;
+        ea.ws_as_weights = ws_as_weights;
+        launch_expand(ea, c->stream);
+        check_launch(c);
+        if (patch_out) CK(c, cudaMemcpyAsync(patch_out, dt.patch, plen * 4, cudaMemcpyDeviceToHost, c->stream));
+    }
+    // the largest neuron count per layer bounds the delta kernel's warps per row
+    dt.kmax_layer.assign(m->L, 0);
+    for (int l = 0; l < m->L; ++l) {
+        int km = 0;
+        for (int64_t k = g.begin[l]; k < g.begin[l + 1]; ++k) km = std::max(km, nn[k]);
+        dt.kmax_layer[l] = km;
+    }
+    return dt;
+}
+
+// ---------------------------------------------------------------- evaluation --
+
+struct EvalCfg {
+    int64_t words32;
+    uint32_t *kill32;
+    unsigned long long *counters;   // [3]: killed, label-count sum, near ties
+    float *logits_out;              // device or null
+};
+
+// Per-row buffers of one batch: x_s for s in [s_lo, L], plus z (vanilla) and the
+// global-average-pooling map.
+struct Workspace {
+    std::vector<float *> xb;   // [L+1]
+    float *zb = nullptr;
+    int64_t z_stride = 0;
+    float *gap_tmp = nullptr;
+    int64_t rows = 0;
+};
+
+int64_t gap_map_stride(const Stage &S)
+{
+    const int mh = S.pool ? S.oh / 2 : S.oh, mw = S.pool ? S.ow / 2 : S.ow;
+    return round4((int64_t)mh * mw * S.oc);
+}
+
+// Bytes per batch row for a group at layer l (vanilla: every stage input from 1,
+// plus z_l).
+int64_t row_bytes(const mure_model *m, int l, bool vanilla)
+{
+    int64_t b = 0;
+    for (int s = vanilla ? 1 : l + 1; s <= m->L; ++s) b += m->xd[s].stride;
+    if (vanilla) b += m->zd[l].stride;
+    int64_t g = 0;
+    for (int v = vanilla ? 0 : l + 1; v < m->L; ++v)
+        if (m->st[v].gap) g = std::max(g, gap_map_stride(m->st[v]));
+    return (b + g) * 4;
+}
+
+void alloc_workspace(mure_ctx *c, Scratch &sc, const mure_model *m, int64_t rows, bool vanilla, int lmin,
+                     Workspace &ws)
+{
+    ws.rows = rows;
+    ws.xb.assign(m->L + 1, nullptr);
+    for (int s = vanilla ? 1 : lmin + 1; s <= m->L; ++s) ws.xb[s] = sc.get<float>(rows * m->xd[s].stride);
+    if (vanilla) {
+        int64_t zs = 0;
+        for (int l = 0; l < m->L; ++l) zs = std::max(zs, m->zd[l].stride);
+        ws.z_stride = zs;
+        ws.zb = sc.get<float>(rows * zs);
+    }
+    int64_t g = 0;
+    for (int v = 0; v < m->L; ++v)
+        if (m->st[v].gap) g = std::max(g, gap_map_stride(m->st[v]));
+    if (g) ws.gap_tmp = sc.get<float>(rows * g);
+}
+
+// One batch: G mutants of group l (starting at group position g0) x an input tile.
+int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevTable &dt, const EvalCfg &ec,
+              const Workspace &ws, int l, int64_t g0, RowMap rm, bool vanilla, int64_t &flops)
+{
+    cudaStream_t s = c->stream;
+    const int L = m->L;
+    int launches = 0;
+    PatchArgs pa{dt.op + g0, dt.nn + g0, dt.noff + g0, dt.ids, dt.poff + g0, dt.patch};
+    FinalArgs fa{};
+    fa.mutant_id = dt.mid + g0;
+    fa.label = ca->label;
+    fa.pred0 = ca->pred0;
+    fa.n_in = ca->n_in;
+    fa.kill32 = ec.kill32;
+    fa.words32 = ec.words32;
+    fa.logits_out = ec.logits_out;
+    fa.near_ties = ec.counters + 2;
+    fa.mode = 0;
+    const Src net_in{ca->x[0], m->xd[0].stride, 1};
+    // where row r finds stage input x_s: memo reads unmutated tensors (s <= l) from
+    // the cache; vanilla recomputes everything except the network input.
+    auto xsrc = [&](int s2) -> Src {
+        if (s2 == 0) return net_in;
+        if (!vanilla && s2 <= l) return Src{ca->x[s2], m->xd[s2].stride, 1};
+        return Src{ws.xb[s2], m->xd[s2].stride, 0};
+    };
+    auto skip_of = [&](const Stage &S) -> Src { return S.has_add ? xsrc(S.skip_src) : Src{nullptr, 0, 0}; };
+    const Stage &Sl = m->st[l];
+    if (vanilla) {
+        // the prefix, then layer l itself, from the inputs, row by row
+        for (int v = 0; v < l; ++v) {
+            launches += launch_stage_simt(m->st[v], xsrc(v), rm, nullptr, 0, skip_of(m->st[v]), ws.xb[v + 1],
+                                          m->xd[v + 1].stride, ws.gap_tmp, s);
+            flops += 2 * m->st[v].macs * rm.R;
+        }
+        if (l < L - 1) {
+            launches += launch_stage_simt(Sl, xsrc(l), rm, ws.zb, ws.z_stride, skip_of(Sl), ws.xb[l + 1],
+                                          m->xd[l + 1].stride, ws.gap_tmp, s);
+        } else {
+            FinalArgs f2 = fa;
+            f2.mode = 2;
+            f2.z_out = ws.zb;
+            f2.z_stride = ws.z_stride;
+            f2.logits_rows = ws.xb[L];
+            f2.x_stride = m->xd[L].stride;
+            launches += launch_final_dense(Sl, xsrc(l), rm, f2, s);
+        }
+        flops += 2 * Sl.macs * rm.R;
+        launches += launch_delta(Sl, Src{ws.zb, ws.z_stride, 0}, xsrc(l), skip_of(Sl), rm, pa, dt.kmax_layer[l],
+                                 ws.xb[l + 1], m->xd[l + 1].stride, s);
+    } else {
+        // memo rows start as the cached output of layer l, then the mutated channels
+        launches += launch_gather_rows(Src{ca->x[l + 1], m->xd[l + 1].stride, 1}, m->xd[l + 1].stride, rm,
+                                       ws.xb[l + 1], m->xd[l + 1].stride, s);
+        launches += launch_delta(Sl, Src{ca->z[l], m->zd[l].stride, 1}, xsrc(l), skip_of(Sl), rm, pa,
+                                 dt.kmax_layer[l], ws.xb[l + 1], m->xd[l + 1].stride, s);
+    }
+    // the suffix l+1 .. L-1 (Algorithm 4) and the fused kill epilogue
+    for (int v = l + 1; v < L - 1; ++v) {
+        launches += launch_stage_simt(m->st[v], xsrc(v), rm, nullptr, 0, skip_of(m->st[v]), ws.xb[v + 1],
+                                      m->xd[v + 1].stride, ws.gap_tmp, s);
+        flops += 2 * m->st[v].macs * rm.R;
+    }
+    if (l < L - 1) {
+        launches += launch_final_dense(m->st[L - 1], xsrc(L - 1), rm, fa, s);
+        flops += 2 * m->st[L - 1].macs * rm.R;
+    } else {
+        launches += launch_epilogue(Src{ws.xb[L], m->xd[L].stride, 0}, m->n_classes, rm, fa, s);
+    }
+    return launches;
+}
+
+struct Outputs {
+    uint64_t *kill_bits;
+    double *sA, *sB;
+    mure_eval_stats *stats;
+    const mure_eval_opts *opts;
+};
+
+void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure_mutant *t, int64_t n,
+              const int32_t *pool, int64_t pool_len, bool vanilla, const Outputs &out)
+{
+    const mure_eval_opts dflt{};
+    const mure_eval_opts *o = out.opts ? out.opts : &dflt;
+    FAILIF(n > 0 && ca->n_in > 0 && !out.kill_bits, c, MURE_ERR_INVALID_ARG, "NULL kill_bits");
+    cudaStream_t s = c->stream;
+    Scratch sc(c);
+    CK(c, cudaEventRecord(c->ev[0], s));
+    const Groups g = group_by_layer(m, t, n);
+    const int64_t words32 = ca->n_pad / 32;
+    mure_eval_stats st{};
+    st.n_rows = n * ca->n_in;
+    double sA = 0, sB = 0;
+    if (n > 0 && ca->n_in > 0) {
+        const DevTable dt = upload_table(c, sc, m, t, n, pool, pool_len, g, 0, nullptr, nullptr);
+        CK(c, cudaEventRecord(c->ev[1], s));
+        EvalCfg ec{};
+        ec.words32 = words32;
+        ec.kill32 = o->outputs_on_device ? reinterpret_cast<uint32_t *>(out.kill_bits)
+                                         : sc.get<uint32_t>((size_t)n * words32);
+        ec.counters = sc.get<unsigned long long>(4);
+        CK(c, cudaMemsetAsync(ec.counters, 0, 4 * sizeof(unsigned long long), s));
+        float *lg_dev = nullptr;
+        if (o->logits_out) {
+            lg_dev = o->outputs_on_device ? o->logits_out : sc.get<float>((size_t)n * ca->n_in * m->n_classes);
+        }
+        ec.logits_out = lg_dev;
+        // batch geometry: rows = mutants x input tile, bounded by the workspace cap
+        const int64_t cap = o->workspace_bytes > 0 ? o->workspace_bytes : (int64_t)8 << 30;
+        int lmin = m->L;
+        int64_t rb = 0;
+        for (int l = 0; l < m->L; ++l)
+            if (g.begin[l + 1] > g.begin[l]) { lmin = std::min(lmin, l); rb = std::max(rb, row_bytes(m, l, vanilla)); }
+        int64_t rows = std::max<int64_t>(cap / std::max<int64_t>(rb, 1), 64);
+        rows = std::min<int64_t>(rows, (int64_t)1 << 24);
+        int64_t T = std::min<int64_t>(ca->n_pad, rows / 64 * 64);
+        const int64_t Gmax = std::max<int64_t>(1, rows / T);
+        // never more rows than the largest group needs
+        int64_t gbig = 0;
+        for (int l = 0; l < m->L; ++l) gbig = std::max(gbig, g.begin[l + 1] - g.begin[l]);
+        rows = std::min(Gmax, gbig) * T;
+        Workspace ws;
+        alloc_workspace(c, sc, m, rows, vanilla, lmin, ws);
+        int64_t launches = 0, flops = 0;
+        for (int l = 0; l < m->L; ++l) {
+            const int64_t gs = g.begin[l], ge = g.begin[l + 1];
+            if (ge == gs) continue;
+            ++st.n_groups;
+            for (int64_t t0 = 0; t0 < ca->n_pad; t0 += T) {
+                const int Tt = (int)std::min<int64_t>(T, ca->n_pad - t0);
+                for (int64_t g0 = gs; g0 < ge; g0 += Gmax) {
+                    const int64_t G = std::min<int64_t>(Gmax, ge - g0);
+                    RowMap rm{t0, Tt, (int)(G * Tt)};
+                    launches += run_batch(c, m, ca, dt, ec, ws, l, g0, rm, vanilla, flops);
+                    check_launch(c);
+                    ++st.n_batches;
+                }
+            }
+        }
+        CK(c, cudaEventRecord(c->ev[2], s));
+        launches += launch_scores(ec.kill32, n, words32, ca->label, m->n_classes, ec.counters, s);
+        check_launch(c);
+        CK(c, cudaEventRecord(c->ev[3], s));
+        unsigned long long host_cnt[4];
+        CK(c, cudaMemcpyAsync(host_cnt, ec.counters, sizeof host_cnt, cudaMemcpyDeviceToHost, s));
+        if (!o->outputs_on_device) {
+            CK(c, cudaMemcpyAsync(out.kill_bits, ec.kill32, (size_t)n * words32 * 4, cudaMemcpyDeviceToHost, s));
+            if (o->logits_out)
+                CK(c, cudaMemcpyAsync(o->logits_out, lg_dev, (size_t)n * ca->n_in * m->n_classes * 4,
+                                      cudaMemcpyDeviceToHost, s));
+        }
+        CK(c, cudaEventRecord(c->ev[4], s));
+        CK(c, cudaStreamSynchronize(s));
+        CK(c, cudaGetLastError());
+        sA = (double)host_cnt[0] / (double)n;
+        sB = ca->n_label_values > 0 ? (double)host_cnt[1] / ((double)n * ca->n_label_values) : 0.0;
+        st.n_near_ties = (int64_t)host_cnt[2];
+        st.kernel_launches = launches + (dt.n_jobs ? 1 : 0);
+        st.flops = flops;
+        float ms = 0;
+        cudaEventElapsedTime(&ms, c->ev[0], c->ev[4]); st.ms_total = ms;
+        cudaEventElapsedTime(&ms, c->ev[0], c->ev[1]); st.ms_expand = ms;
+        cudaEventElapsedTime(&ms, c->ev[1], c->ev[2]); st.ms_suffix = ms;
+        cudaEventElapsedTime(&ms, c->ev[2], c->ev[3]); st.ms_score = ms;
+    } else if (n > 0 && out.kill_bits && o->outputs_on_device == 0) {
+        // no inputs: zero-width kill rows, nothing to write
+    }
+    if (out.sA) *out.sA = sA;
+    if (out.sB) *out.sB = sB;
+    if (out.stats) *out.stats = st;
+}
+
+// Original forward over X: the prefix cache (full) or, for vanilla, only the
+// network input, predictions and labels.
+mure_cache *build_cache(mure_model *m, const float *X, int64_t n_in, const int32_t *labels, int on_dev, bool full)
+{
+    mure_ctx *c = m->ctx;
+    FAILIF(n_in < 0, c, MURE_ERR_INVALID_ARG, "n_inputs < 0");
+    FAILIF(n_in > 0 && !X, c, MURE_ERR_INVALID_ARG, "NULL X");
+    FAILIF(n_in > ((int64_t)1 << 30), c, MURE_ERR_UNSUPPORTED, "more than 2^30 inputs");
+    std::vector<int32_t> lab_host;
+    if (labels && n_in > 0) {
+        lab_host.resize(n_in);
+        if (on_dev) CK(c, cudaMemcpy(lab_host.data(), labels, n_in * 4, cudaMemcpyDeviceToHost));
+        else memcpy(lab_host.data(), labels, n_in * 4);
+        for (int64_t t = 0; t < n_in; ++t)
+            FAILIF(lab_host[t] < 0 || lab_host[t] >= m->n_classes, c, MURE_ERR_INVALID_ARG, "label %d of input %lld",
+                   lab_host[t], (long long)t);
+    }
+    cudaStream_t s = c->stream;
+    auto *ca = new mure_cache();
+    ca->model = m;
+    ca->full = full;
+    ca->n_in = n_in;
+    ca->n_pad = round_up(n_in, kInputAlign);
+    const int L = m->L;
+    ca->x.assign(L + 1, nullptr);
+    ca->z.assign(L, nullptr);
+    struct Cleanup {
+        mure_cache *ca;
+        bool ok = false;
+        ~Cleanup()
+        {
+            if (!ok) mure_cache_free(ca);
+        }
+    } cl{ca};
+    const int64_t np = std::max<int64_t>(ca->n_pad, kInputAlign);
+    for (int s2 = 0; s2 <= L; ++s2) {
+        ca->x[s2] = (float *)dalloc(c, np * m->xd[s2].stride * 4);
+        CK(c, cudaMemsetAsync(ca->x[s2], 0, np * m->xd[s2].stride * 4, s));
+    }
+    for (int v = 0; v < L; ++v) {
+        ca->z[v] = (float *)dalloc(c, np * m->zd[v].stride * 4);
+        CK(c, cudaMemsetAsync(ca->z[v], 0, np * m->zd[v].stride * 4, s));
+    }
+    ca->pred0 = (int32_t *)dalloc(c, np * 4);
+    ca->label = (int32_t *)dalloc(c, np * 4);
+    CK(c, cudaMemsetAsync(ca->pred0, 0, np * 4, s));
+    CK(c, cudaMemsetAsync(ca->label, 0, np * 4, s));
+    if (n_in > 0) {
+        const int64_t sz = m->xd[0].size, str = m->xd[0].stride;
+        CK(c, cudaMemcpy2DAsync(ca->x[0], str * 4, X, sz * 4, sz * 4, n_in,
+                                on_dev ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, s));
+        Scratch sc(c);
+        int64_t g = 0;
+        for (int v = 0; v < L; ++v)
+            if (m->st[v].gap) g = std::max(g, gap_map_stride(m->st[v]));
+        float *gap_tmp = g ? sc.get<float>(ca->n_pad * g) : nullptr;
+        // intermediate activations: in the cache (full) or in scratch rows (vanilla
+        // only needs the predictions)
+        std::vector<float *> xs(L + 1), zs(L);
+        for (int s2 = 0; s2 <= L; ++s2) xs[s2] = ca->x[s2];
+        for (int v = 0; v < L; ++v) zs[v] = ca->z[v];
+        const RowMap rm{0, (int)ca->n_pad, (int)ca->n_pad};
+        for (int v = 0; v < L - 1; ++v) {
+            const Stage &S = m->st[v];
+            const Src skip = S.has_add ? Src{xs[S.skip_src], m->xd[S.skip_src].stride, 0} : Src{nullptr, 0, 0};
+            launch_stage_simt(S, Src{xs[v], m->xd[v].stride, 0}, rm, zs[v], m->zd[v].stride, skip, xs[v + 1],
+                              m->xd[v + 1].stride, gap_tmp, s);
+            check_launch(c);
+        }
+        FinalArgs fa{};
+        fa.mode = 1;
+        fa.z_out = zs[L - 1];
+        fa.z_stride = m->zd[L - 1].stride;
+        fa.x_out = xs[L];
+        fa.x_stride = m->xd[L].stride;
+        fa.pred_out = ca->pred0;
+        launch_final_dense(m->st[L - 1], Src{xs[L - 1], m->xd[L - 1].stride, 0}, rm, fa, s);
+        check_launch(c);
+        if (labels) CK(c, cudaMemcpyAsync(ca->label, lab_host.data(), n_in * 4, cudaMemcpyHostToDevice, s));
+        else CK(c, cudaMemcpyAsync(ca->label, ca->pred0, n_in * 4, cudaMemcpyDeviceToDevice, s));
+        uint32_t *mask = sc.get<uint32_t>(1);
+        CK(c, cudaMemsetAsync(mask, 0, 4, s));
+        launch_label_set(ca->label, n_in, mask, s);
+        check_launch(c);
+        uint32_t hm = 0;
+        CK(c, cudaMemcpyAsync(&hm, mask, 4, cudaMemcpyDeviceToHost, s));
+        CK(c, cudaStreamSynchronize(s));
+        ca->n_label_values = __builtin_popcount(hm);
+    }
+    CK(c, cudaStreamSynchronize(s));
+    cl.ok = true;
+    return ca;
+}
+
+}  // namespace
+
+// ====================================================================== ABI ==
+
+extern "C" {
+
+mure_status mure_create(int device, void *cuda_stream, const mure_allocator *alloc, mure_ctx **out)
+{
+    if (!out) return MURE_ERR_INVALID_ARG;
+    *out = nullptr;
+    int n = 0;
+    if (cudaGetDeviceCount(&n) != cudaSuccess) {
+        cudaGetLastError();
+        return MURE_ERR_CUDA;
+    }
+    if (device < 0 || device >= n) return MURE_ERR_INVALID_ARG;
+    if (alloc && (!alloc->alloc || !alloc->free)) return MURE_ERR_INVALID_ARG;
+    auto *c = new mure_ctx();
+    c->device = device;
+    c->stream = (cudaStream_t)cuda_stream;
+    if (alloc) { c->alloc = *alloc; c->has_alloc = true; }
+    mure_status st = run(c, [&] {
+        CK(c, cudaSetDevice(device));
+        CK(c, cudaDeviceGetAttribute(&c->n_sms, cudaDevAttrMultiProcessorCount, device));
+        for (auto &e : c->ev) CK(c, cudaEventCreate(&e));
+    });
+    if (st != MURE_OK) {
+        mure_destroy(c);
+        return st;
+    }
+    *out = c;
+    return MURE_OK;
+}
+
+void mure_destroy(mure_ctx *ctx)
+{
+    if (!ctx) return;
+    for (auto &e : ctx->ev)
+        if (e) cudaEventDestroy(e);
+    delete ctx;
+}
+
+const char *mure_last_error(const mure_ctx *ctx) { return ctx ? ctx->err.c_str() : "NULL context"; }
+
+mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **out)
+{
+    if (!c) return MURE_ERR_INVALID_ARG;
+    return run(c, [&] {
+        FAILIF(!d || !out || !d->nodes || d->n_nodes < 1, c, MURE_ERR_INVALID_ARG, "NULL model description");
+        *out = nullptr;
+        FAILIF(d->in_h < 1 || d->in_w < 1 || d->in_c < 1, c, MURE_ERR_INVALID_ARG, "bad input shape");
+        FAILIF(d->precision != MURE_PREC_FP32, c, MURE_ERR_UNSUPPORTED, "precision %d is not available",
+               d->precision);
+        CK(c, cudaSetDevice(c->device));
+        auto *m = new mure_model();
+        m->ctx = c;
+        m->precision = d->precision;
+        struct Cleanup {
+            mure_model *m;
+            bool ok = false;
+            ~Cleanup()
+            {
+                if (!ok) mure_model_free(m);
+            }
+        } cl{m};
+        compile(c, d, m);
+        std::vector<int> wn;
+        for (int v = 0; v < d->n_nodes; ++v)
+            if (weighted(d->nodes[v].kind)) wn.push_back(v);
+        std::vector<float> Wt;
+        for (int l = 0; l < m->L; ++l) {
+            Stage &S = m->st[l];
+            const mure_node &n = d->nodes[wn[l]];
+            const int64_t nw = (int64_t)S.oc * S.K;
+            S.W = (float *)dalloc(c, nw * 4);
+            S.Wt = (float *)dalloc(c, nw * 4);
+            S.b = (float *)dalloc(c, S.oc * 4);
+            Wt.resize(nw);
+            for (int o = 0; o < S.oc; ++o)
+                for (int k = 0; k < S.K; ++k) Wt[(int64_t)k * S.oc + o] = n.W[(int64_t)o * S.K + k];
+            CK(c, cudaMemcpyAsync(S.W, n.W, nw * 4, cudaMemcpyHostToDevice, c->stream));
+            CK(c, cudaMemcpyAsync(S.Wt, Wt.data(), nw * 4, cudaMemcpyHostToDevice, c->stream));
+            CK(c, cudaMemcpyAsync(S.b, n.b, S.oc * 4, cudaMemcpyHostToDevice, c->stream));
+            CK(c, cudaStreamSynchronize(c->stream));  // Wt is reused
+        }
+        // population std of every layer's weights (GF's sigma), fp64 on the device
+        {
+            Scratch sc(c);
+            std::vector<const float *> Wp(m->L);
+            std::vector<int64_t> cnt(m->L);
+            for (int l = 0; l < m->L; ++l) { Wp[l] = m->st[l].W; cnt[l] = (int64_t)m->st[l].oc * m->st[l].K; }
+            const float **Wd = sc.get<const float *>(m->L);
+            int64_t *nd = sc.get<int64_t>(m->L);
+            m->sigma_dev = (double *)dalloc(c, m->L * 8);
+            CK(c, cudaMemcpyAsync(Wd, Wp.data(), m->L * sizeof(float *), cudaMemcpyHostToDevice, c->stream));
+            CK(c, cudaMemcpyAsync(nd, cnt.data(), m->L * 8, cudaMemcpyHostToDevice, c->stream));
+            launch_layer_std(Wd, nd, m->L, m->sigma_dev, c->stream);
+            check_launch(c);
+            m->sigma_host.resize(m->L);
+            CK(c, cudaMemcpyAsync(m->sigma_host.data(), m->sigma_dev, m->L * 8, cudaMemcpyDeviceToHost, c->stream));
+            CK(c, cudaStreamSynchronize(c->stream));
+            for (int l = 0; l < m->L; ++l) m->st[l].sigma_std = (float)m->sigma_host[l];
+        }
+        cl.ok = true;
+        *out = m;
+    });
+}
+
+void mure_model_free(mure_model *m)
+{
+    if (!m) return;
+    for (auto &S : m->st) {
+        dfree(m->ctx, S.W);
+        dfree(m->ctx, S.Wt);
+        dfree(m->ctx, S.b);
+    }
+    dfree(m->ctx, m->sigma_dev);
+    cudaStreamSynchronize(m->ctx->stream);
+    delete m;
+}
+
+int32_t mure_model_n_layers(const mure_model *m) { return m ? m->L : -1; }
+
+mure_status mure_build_prefix_cache(mure_model *m, const float *X, int64_t n_inputs, const int32_t *labels,
+                                    int x_on_device, mure_cache **out)
+{
+    if (!m) return MURE_ERR_INVALID_ARG;
+    mure_ctx *c = m->ctx;
+    return run(c, [&] {
+        FAILIF(!out, c, MURE_ERR_INVALID_ARG, "NULL out");
+        *out = nullptr;
+        CK(c, cudaSetDevice(c->device));
+        *out = build_cache(m, X, n_inputs, labels, x_on_device, true);
+    });
+}
+
+void mure_cache_free(mure_cache *ca)
+{
+    if (!ca) return;
+    mure_ctx *c = ca->model->ctx;
+    for (float *p : ca->x) dfree(c, p);
+    for (float *p : ca->z) dfree(c, p);
+    dfree(c, ca->pred0);
+    dfree(c, ca->label);
+    cudaStreamSynchronize(c->stream);
+    delete ca;
+}
+
+mure_status mure_cache_outputs(mure_cache *ca, float *logits, int32_t *pred)
+{
+    if (!ca) return MURE_ERR_INVALID_ARG;
+    mure_ctx *c = ca->model->ctx;
+    return run(c, [&] {
+        const mure_model *m = ca->model;
+        if (ca->n_in == 0) return;
+        if (logits)
+            CK(c, cudaMemcpy2DAsync(logits, m->n_classes * 4, ca->x[m->L], m->xd[m->L].stride * 4, m->n_classes * 4,
+                                    ca->n_in, cudaMemcpyDeviceToHost, c->stream));
+        if (pred) CK(c, cudaMemcpyAsync(pred, ca->pred0, ca->n_in * 4, cudaMemcpyDeviceToHost, c->stream));
+        CK(c, cudaStreamSynchronize(c->stream));
+    });
+}
+
+mure_status mure_eval_mutants(mure_cache *ca, const mure_mutant *table, int64_t n_mutants, const int32_t *neuron_pool,
+                              int64_t pool_len, const mure_eval_opts *opts, uint64_t *kill_bits,
+                              double *score_killed_frac, double *score_deepmutation, mure_eval_stats *stats)
+{
+    if (!ca) return MURE_ERR_INVALID_ARG;
+    mure_ctx *c = ca->model->ctx;
+    return run(c, [&] {
+        CK(c, cudaSetDevice(c->device));
+        FAILIF(!ca->full, c, MURE_ERR_INVALID_ARG, "cache holds no activations");
+        check_table(c, ca->model, table, n_mutants, neuron_pool, pool_len);
+        evaluate(c, ca->model, ca, table, n_mutants, neuron_pool, pool_len, false,
+                 Outputs{kill_bits, score_killed_frac, score_deepmutation, stats, opts});
+    });
+}
+
+mure_status mure_eval_vanilla(mure_model *m, const float *X, int64_t n_inputs, const int32_t *labels, int x_on_device,
+                              const mure_mutant *table, int64_t n_mutants, const int32_t *neuron_pool,
+                              int64_t pool_len, const mure_eval_opts *opts, uint64_t *kill_bits,
+                              double *score_killed_frac, double *score_deepmutation, mure_eval_stats *stats)
+{
+    if (!m) return MURE_ERR_INVALID_ARG;
+    mure_ctx *c = m->ctx;
+    return run(c, [&] {
+        CK(c, cudaSetDevice(c->device));
+        check_table(c, m, table, n_mutants, neuron_pool, pool_len);
+        mure_cache *ca = build_cache(m, X, n_inputs, labels, x_on_device, false);
+        struct Free {
+            mure_cache *ca;
+            ~Free() { mure_cache_free(ca); }
+        } fr{ca};
+        evaluate(c, m, ca, table, n_mutants, neuron_pool, pool_len, true,
+                 Outputs{kill_bits, score_killed_frac, score_deepmutation, stats, opts});
+    });
+}
+
+mure_status mure_expand_patches(mure_model *m, const mure_mutant *table, int64_t n_mutants, const int32_t *neuron_pool,
+                                int64_t pool_len, float *out, int64_t out_len, int64_t *offsets)
+{
+    if (!m) return MURE_ERR_INVALID_ARG;
+    mure_ctx *c = m->ctx;
+    return run(c, [&] {
+        CK(c, cudaSetDevice(c->device));
+        check_table(c, m, table, n_mutants, neuron_pool, pool_len);
+        FAILIF(!offsets && n_mutants > 0, c, MURE_ERR_INVALID_ARG, "NULL offsets");
+        int64_t need = 0;
+        for (int64_t i = 0; i < n_mutants; ++i)
+            if (table[i].op == MURE_OP_GF || table[i].op == MURE_OP_WS)
+                need += (int64_t)table[i].n_neurons * m->st[table[i].layer].K;
+        FAILIF(need > out_len || (need > 0 && !out), c, MURE_ERR_INVALID_ARG, "out holds %lld values, %lld needed",
+               (long long)out_len, (long long)need);
+        // identity order so that offsets follow the table
+        Groups g;
+        g.order.resize(n_mutants);
+        std::iota(g.order.begin(), g.order.end(), 0);
+        g.begin.assign(m->L + 1, n_mutants);
+        g.begin[0] = 0;
+        Scratch sc(c);
+        upload_table(c, sc, m, table, n_mutants, neuron_pool, pool_len, g, 1, out, offsets);
+        CK(c, cudaStreamSynchronize(c->stream));
+    });
+}
+
+}  // extern "C"

@@ -1,0 +1,175 @@
+// Internal declarations of the GB300 mutation-testing library (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/mure.h"
+
+namespace mure {
+
+constexpr int kMaxClasses = 32;   // final-layer kernel keeps one accumulator per class
+constexpr int kInputAlign = 64;   // inputs are padded to a multiple of 64 (one kill word)
+
+// A weighted layer together with the unweighted nodes that turn its output into the
+// next weighted layer's input ("stage").  Post-ops in order: act1, + skip, act2,
+// 2x2/2 max pool, global average pool.
+struct Stage {
+    int kind;                 // MURE_NODE_CONV2D or MURE_NODE_DENSE
+    int ih, iw, ic;           // input x_v (dense: 1 x 1 x fan-in)
+    int kh, kw, stride, pad;
+    int oh, ow, oc;           // pre-activation z_v
+    int K;                    // fan-in kh*kw*ic
+    int act1;
+    int has_add, skip_src;    // skip tensor = x_{skip_src} (stage-input index)
+    int sc_stride, sc_c;      // shortcut subsampling stride and source channels
+    int sk_w;                 // width of the skip source tensor
+    int act2;
+    int pool, gap;
+    int yh, yw, yc;           // output x_{v+1}
+    int64_t macs;             // multiply-accumulates per row
+    float *W = nullptr;       // device [oc][K]
+    float *Wt = nullptr;      // device [K][oc] (the same weights, K-major rows)
+    float *b = nullptr;       // device [oc]
+    float sigma_std = 0.f;    // population std of W (host copy, fp32-rounded for info)
+};
+
+// Stage inputs x_s, s = 0..L (x_0 network input, x_L logits): shape and row stride.
+struct TensorDim {
+    int h, w, c;
+    int64_t size, stride;     // elements; stride = size rounded up to a multiple of 4
+};
+
+}  // namespace mure
+
+struct mure_ctx {
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    mure_allocator alloc{};
+    bool has_alloc = false;
+    std::string err;
+    cudaEvent_t ev[8]{};
+    int n_sms = 0;
+};
+
+struct mure_model {
+    mure_ctx *ctx = nullptr;
+    int precision = MURE_PREC_FP32;
+    int L = 0;
+    int n_classes = 0;
+    std::vector<mure::Stage> st;      // L stages
+    std::vector<mure::TensorDim> xd;  // L + 1 stage inputs
+    std::vector<mure::TensorDim> zd;  // L pre-activations
+    double *sigma_dev = nullptr;      // device [L] population std of each layer's W (fp64)
+    std::vector<double> sigma_host;
+};
+
+struct mure_cache {
+    mure_model *model = nullptr;
+    int64_t n_in = 0, n_pad = 0;
+    std::vector<float *> x;           // x[s], s = 0..L: [n_pad][xd[s].stride]
+    std::vector<float *> z;           // z[v], v = 0..L-1: [n_pad][zd[v].stride]
+    int32_t *pred0 = nullptr;         // [n_pad]
+    int32_t *label = nullptr;         // [n_pad]
+    int n_label_values = 0;           // |L|: distinct labels among the inputs
+    bool full = true;                 // false: only x[0] / pred0 / label (vanilla)
+};
+
+namespace mure {
+
+// ------------------------------------------------------------ kernel launchers --
+// All launchers queue on `s` and return the number of kernels launched.
+
+// Where a batch row reads a tensor: per row (row r at p + r*stride) or per input
+// (row r at p + (t0 + r % T)*stride, shared by the batch's mutants).
+struct Src {
+    const float *p;
+    int64_t stride;
+    int per_input;
+};
+
+struct RowMap {
+    int64_t t0;   // first input of the tile
+    int T;        // inputs per tile (multiple of 64)
+    int R;        // rows = mutants in the batch x T
+};
+
+// Stage v over R rows: z (optional) and y = post(act1(conv(x) + b)).
+int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip,
+                      float *y_out, int64_t y_stride, float *gap_tmp, cudaStream_t s);
+
+// Final dense layer (F -> C, C <= 32) over R rows, with the fused epilogue.
+struct FinalArgs {
+    const int32_t *mutant_id;   // [G] original mutant index of batch mutant g
+    const int32_t *label;       // [n_pad]
+    const int32_t *pred0;       // [n_pad]
+    int64_t n_in;
+    uint32_t *kill32;           // [n_mut][words32] (kill mode)
+    int64_t words32;
+    float *logits_rows;         // optional per-row logits [R][C] (pre-epilogue mode)
+    float *logits_out;          // optional [n_mut][n_in][C]
+    float *z_out;               // cache mode: z[L-1] rows; nullable
+    int64_t z_stride;
+    float *x_out;               // cache mode: logits rows x[L]; nullable
+    int64_t x_stride;
+    int32_t *pred_out;          // cache mode: pred0 [n_pad]
+    unsigned long long *near_ties;
+    int mode;                   // 0 = kill, 1 = cache build, 2 = write per-row logits only
+};
+int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s);
+
+// Kill epilogue on per-row logits (mutants of the output layer).
+int launch_epilogue(Src logits, int C, RowMap rm, const FinalArgs &fa, cudaStream_t s);
+
+// Copy per-input rows of a cached tensor into per-row batch rows.
+int launch_gather_rows(Src src, int64_t n_elems, RowMap rm, float *dst, int64_t dst_stride, cudaStream_t s);
+
+// Per-mutant patch data of a batch, in device memory.
+struct PatchArgs {
+    const int32_t *op;          // [G]
+    const int32_t *n_neurons;   // [G]
+    const int64_t *neuron_off;  // [G] into ids
+    const int32_t *ids;         // neuron pool
+    const int64_t *patch_off;   // [G] offset of slot 0 into patch (-1: none)
+    const float *patch;         // GF: sigma * n, WS: W[j][perm f] - W[j][f]; F per slot
+};
+
+// Rewrite the mutated neurons' channels of x_{l+1} rows (y) from z_l (and x_l for
+// GF/WS), the layer's post-ops and skip.
+int launch_delta(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *y,
+                 int64_t y_stride, cudaStream_t s);
+
+// Expand GF / WS descriptors into patches (see mure_expand_patches): one job per
+// (mutant, neuron slot).
+struct SlotJob {
+    int32_t layer, op, F, j, q, reserved;
+    float param, reserved2;
+    uint64_t seed;
+    int64_t out_off;   // F values at patch + out_off
+    int64_t perm_off;  // WS: F ints of permutation scratch
+};
+struct ExpandArgs {
+    const SlotJob *jobs;
+    int64_t n_jobs;
+    const double *sigma;        // [L] population std of each layer's weights
+    const float *const *W;      // [L] device weight pointers ([oc][K])
+    float *patch;
+    int32_t *perm;              // WS permutation scratch
+    int ws_as_weights;          // 1: WS patch holds the permuted weights (inspection)
+};
+int launch_expand(const ExpandArgs &ea, cudaStream_t s);
+
+// Population std of each layer's weights in fp64.
+int launch_layer_std(const float *const *W, const int64_t *n, int L, double *out, cudaStream_t s);
+
+// Score reduction: per mutant killed flag and |killingLabels|, summed.
+int launch_scores(const uint32_t *kill32, int64_t n_mut, int64_t words32, const int32_t *label, int n_classes,
+                  unsigned long long *totals /* [2]: killed, sum of label counts */, cudaStream_t s);
+
+// Distinct labels among n inputs (bitset of n_classes bits, <= 32 classes).
+int launch_label_set(const int32_t *label, int64_t n, uint32_t *mask, cudaStream_t s);
+
+}  // namespace mure

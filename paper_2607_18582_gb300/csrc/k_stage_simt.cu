@@ -1,0 +1,361 @@
+// Layer kernels of the FP32 arithmetic: implicit-GEMM convolution / dense on the
+// CUDA cores, the output layer with the fused argmax / compare / kill epilogue, and
+// small row-movement kernels.
+//
+// Determinism contract (what makes memoized == vanilla bit for bit): every output
+// element z[row][pos][n] is the fp32 FMA chain acc = fma(x_k, w_k, acc) over the
+// fan-in k = (ky, kx, ci) in ascending order starting from +0 (zero-padding taps
+// contribute x = 0), then z = acc + b[n].  Nothing depends on the batch size, the
+// tile a row lands in or the number of mutants, so one row gives the same bits in
+// the cache build, in a vanilla prefix and in a memoized suffix.
+#include "common.cuh"
+#include "device_util.cuh"
+
+namespace mure {
+
+struct StageParams {
+    const float *x; int64_t x_stride; int x_per_input;
+    int64_t t0; int T; int R;
+    int ih, iw, ic, kh, kw, stride, pad, oh, ow, oc, K;
+    const float *Wt;  // [K][oc]
+    const float *b;
+    int act1, has_add, act2, pool;
+    const float *skip; int64_t skip_stride; int skip_per_input; int sk_w, sk_c, sk_stride;
+    float *z; int64_t z_stride;
+    float *y; int64_t y_stride;
+    int P;   // GEMM rows per batch row: oh*ow, ordered (oy, ox), or with pooling
+             // 4 * (oh/2) * (ow/2) ordered (py, px, dy, dx)
+    int pw;  // pooled width
+};
+
+template <int BN>
+__global__ void __launch_bounds__(256) k_stage_simt(const StageParams p)
+{
+    constexpr int BM = 4096 / BN, BK = 16;
+    constexpr int A_SPLIT = 256 / BM, A_PER = BK / A_SPLIT;
+    constexpr int B_SPLIT = 256 / BN, B_PER = BK / B_SPLIT;
+    __shared__ __align__(16) float As[BK][BM];
+    __shared__ __align__(16) float Bs[BK][BN];
+
+    const int tid = threadIdx.x;
+    const int tn = tid % (BN / 4), tm = tid / (BN / 4);
+    const int64_t M = (int64_t)p.R * p.P;
+    const int64_t m0 = (int64_t)blockIdx.x * BM;
+    const int n0 = blockIdx.y * BN;
+
+    // this thread's A-load row
+    const int m_l = tid % BM, kl0 = (tid / BM) * A_PER;
+    const int64_t m = m0 + m_l;
+    const bool valid_m = m < M;
+    int iy0 = 0, ix0 = 0;
+    const float *xrow = p.x;
+    if (valid_m) {
+        const int64_t row = m / p.P;
+        const int q = (int)(m % p.P);
+        int oy, ox;
+        if (p.pool) {
+            const int w = q >> 2, sub = q & 3;
+            oy = 2 * (w / p.pw) + (sub >> 1);
+            ox = 2 * (w % p.pw) + (sub & 1);
+        } else {
+            oy = q / p.ow;
+            ox = q % p.ow;
+        }
+        iy0 = oy * p.stride - p.pad;
+        ix0 = ox * p.stride - p.pad;
+        xrow = p.x + (p.x_per_input ? (p.t0 + row % p.T) : row) * p.x_stride;
+    }
+    const int n_l = tid % BN, kb0 = (tid / BN) * B_PER;
+
+    float acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+
+    for (int k0 = 0; k0 < p.K; k0 += BK) {
+        {
+            int k = k0 + kl0;
+            int ci = k % p.ic, t = k / p.ic, kx = t % p.kw, ky = t / p.kw;
+#pragma unroll
+            for (int i = 0; i < A_PER; ++i) {
+                float v = 0.f;
+                if (valid_m && k + i < p.K) {
+                    const int iy = iy0 + ky, ix = ix0 + kx;
+                    if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw)
+                        v = __ldg(xrow + ((int64_t)iy * p.iw + ix) * p.ic + ci);
+                }
+                As[kl0 + i][m_l] = v;
+                if (++ci == p.ic) { ci = 0; if (++kx == p.kw) { kx = 0; ++ky; } }
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < B_PER; ++i) {
+            const int k = k0 + kb0 + i, n = n0 + n_l;
+            Bs[kb0 + i][n_l] = (k < p.K && n < p.oc) ? __ldg(p.Wt + (int64_t)k * p.oc + n) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int kk = 0; kk < BK; ++kk) {
+            const float4 a = *reinterpret_cast<const float4 *>(&As[kk][tm * 4]);
+            const float4 b = *reinterpret_cast<const float4 *>(&Bs[kk][tn * 4]);
+            const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+
+    // epilogue: bias, activation, skip, pooling
+    const int64_t mb = m0 + tm * 4;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const int n = n0 + tn * 4 + j;
+        if (n >= p.oc) continue;
+        const float bias = __ldg(p.b + n);
+        float win[4];
+        int64_t row = 0;
+        int py = 0, px = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int64_t mm = mb + i;
+            win[i] = 0.f;
+            if (mm >= M) continue;
+            row = mm / p.P;
+            const int q = (int)(mm % p.P);
+            int oy, ox;
+            if (p.pool) {
+                const int w = q >> 2, sub = q & 3;
+                py = w / p.pw; px = w % p.pw;
+                oy = 2 * py + (sub >> 1);
+                ox = 2 * px + (sub & 1);
+            } else {
+                oy = q / p.ow;
+                ox = q % p.ow;
+            }
+            const float z = acc[i][j] + bias;
+            if (p.z) p.z[row * p.z_stride + ((int64_t)oy * p.ow + ox) * p.oc + n] = z;
+            float v = act_apply(p.act1, z);
+            if (p.has_add) {
+                const float *sr = p.skip + (p.skip_per_input ? (p.t0 + row % p.T) : row) * p.skip_stride;
+                const float s = n < p.sk_c ? sr[((int64_t)oy * p.sk_stride * p.sk_w + ox * p.sk_stride) * p.sk_c + n] : 0.f;
+                v = act_apply(p.act2, v + s);
+            }
+            if (p.pool) win[i] = v;
+            else p.y[row * p.y_stride + ((int64_t)oy * p.ow + ox) * p.oc + n] = v;
+        }
+        if (p.pool && mb < M)
+            p.y[row * p.y_stride + ((int64_t)py * p.pw + px) * p.oc + n] = max4_first(win[0], win[1], win[2], win[3]);
+    }
+}
+
+// Global average pooling: y[r][c] = (sum over positions, ascending, in fp32) / P.
+__global__ void k_gap(const float *__restrict__ in, int64_t in_stride, int P, int C, int R, float *__restrict__ y,
+                      int64_t y_stride)
+{
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (int64_t)R * C) return;
+    const int64_t r = i / C;
+    const int c = (int)(i % C);
+    y[r * y_stride + c] = gap_sum(in + r * in_stride, P, C, c);
+}
+
+int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
+                      int64_t y_stride, float *gap_tmp, cudaStream_t s)
+{
+    if (rm.R <= 0) return 0;
+    StageParams p{};
+    p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
+    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
+    p.ih = S.ih; p.iw = S.iw; p.ic = S.ic; p.kh = S.kh; p.kw = S.kw; p.stride = S.stride; p.pad = S.pad;
+    p.oh = S.oh; p.ow = S.ow; p.oc = S.oc; p.K = S.K;
+    p.Wt = S.Wt; p.b = S.b;
+    p.act1 = S.act1; p.has_add = S.has_add; p.act2 = S.act2; p.pool = S.pool;
+    p.skip = skip.p; p.skip_stride = skip.stride; p.skip_per_input = skip.per_input;
+    p.sk_w = S.sk_w; p.sk_c = S.sc_c; p.sk_stride = S.sc_stride;
+    p.z = z_out; p.z_stride = z_stride;
+    // with global average pooling the post-op map goes to gap_tmp first
+    const int mh = S.pool ? S.oh / 2 : S.oh, mw = S.pool ? S.ow / 2 : S.ow;
+    const int64_t map_stride = round4((int64_t)mh * mw * S.oc);
+    p.y = S.gap ? gap_tmp : y_out;
+    p.y_stride = S.gap ? map_stride : y_stride;
+    p.pw = S.ow / 2;
+    p.P = S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
+    const int64_t M = (int64_t)rm.R * p.P;
+    int launches = 1;
+    if (S.oc <= 16) {
+        dim3 g((unsigned)((M + 255) / 256), (unsigned)((S.oc + 15) / 16));
+        k_stage_simt<16><<<g, 256, 0, s>>>(p);
+    } else if (S.oc <= 32) {
+        dim3 g((unsigned)((M + 127) / 128), (unsigned)((S.oc + 31) / 32));
+        k_stage_simt<32><<<g, 256, 0, s>>>(p);
+    } else {
+        dim3 g((unsigned)((M + 63) / 64), (unsigned)((S.oc + 63) / 64));
+        k_stage_simt<64><<<g, 256, 0, s>>>(p);
+    }
+    if (S.gap) {
+        const int64_t n = (int64_t)rm.R * S.oc;
+        k_gap<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(gap_tmp, map_stride, mh * mw, S.oc, rm.R, y_out, y_stride);
+        ++launches;
+    }
+    return launches;
+}
+
+// ------------------------------------------------------ output layer + epilogue --
+
+struct FinalParams {
+    const float *x; int64_t x_stride; int x_per_input;
+    int64_t t0; int T; int R;
+    int F, C, act;
+    const float *W;  // [C][F]
+    const float *b;
+    FinalArgs fa;
+};
+
+// Kill bits of one warp of rows (32 consecutive inputs of one mutant) and the
+// near-tie count.  v = the row's logits.
+__device__ __forceinline__ void epilogue_row(const FinalArgs &fa, int64_t t0, int T, int64_t row, bool in_range,
+                                             const float *v, int C)
+{
+    const int g = (int)(row / T);
+    const int64_t t = t0 + row % T;
+    const bool valid = in_range && t < fa.n_in;
+    int arg = 0;
+    bool near = false;
+    if (valid) {
+        arg = argmax_first(v, C);
+        near = near_tie(v, C, arg);
+    }
+    const bool kill = valid && fa.pred0[t] == fa.label[t] && arg != fa.label[t];
+    const unsigned kb = __ballot_sync(0xffffffffu, kill);
+    const unsigned nb = __ballot_sync(0xffffffffu, near);
+    const int lane = threadIdx.x & 31;
+    if (lane == 0 && in_range) {
+        const int mid = fa.mutant_id[g];
+        fa.kill32[(int64_t)mid * fa.words32 + (t >> 5)] = kb;
+        if (nb && fa.near_ties) atomicAdd(fa.near_ties, (unsigned long long)__popc(nb));
+    }
+    if (valid && fa.logits_out) {
+        float *o = fa.logits_out + ((int64_t)fa.mutant_id[g] * fa.n_in + t) * C;
+        for (int c = 0; c < C; ++c) o[c] = v[c];
+    }
+}
+
+__global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
+{
+    constexpr int RB = 128, FC = 32;
+    __shared__ float xs[RB][FC + 1];
+    __shared__ __align__(16) float ws[FC][kMaxClasses];
+    const int tid = threadIdx.x;
+    const int64_t row0 = (int64_t)blockIdx.x * RB;
+    const int64_t row = row0 + tid;
+    const bool in_range = row < p.R;
+    float acc[kMaxClasses];
+#pragma unroll
+    for (int c = 0; c < kMaxClasses; ++c) acc[c] = 0.f;
+    for (int f0 = 0; f0 < p.F; f0 += FC) {
+        for (int i = tid; i < RB * FC; i += RB) {
+            const int rl = i / FC, fl = i % FC;
+            const int64_t r = row0 + rl;
+            float v = 0.f;
+            if (r < p.R && f0 + fl < p.F)
+                v = __ldg(p.x + (p.x_per_input ? (p.t0 + r % p.T) : r) * p.x_stride + f0 + fl);
+            xs[rl][fl] = v;
+        }
+        for (int i = tid; i < FC * kMaxClasses; i += RB) {
+            const int fl = i / kMaxClasses, c = i % kMaxClasses;
+            ws[fl][c] = (c < p.C && f0 + fl < p.F) ? __ldg(p.W + (int64_t)c * p.F + f0 + fl) : 0.f;
+        }
+        __syncthreads();
+        const int fe = min(FC, p.F - f0);
+        for (int fl = 0; fl < fe; ++fl) {
+            const float xv = xs[tid][fl];
+#pragma unroll
+            for (int c = 0; c < kMaxClasses; ++c)
+                if (c < p.C) acc[c] = fmaf(xv, ws[fl][c], acc[c]);
+        }
+        __syncthreads();
+    }
+    float v[kMaxClasses];
+#pragma unroll
+    for (int c = 0; c < kMaxClasses; ++c) {
+        const float z = c < p.C ? acc[c] + __ldg(p.b + c) : 0.f;
+        if (in_range && c < p.C) {
+            if (p.fa.z_out) p.fa.z_out[row * p.fa.z_stride + c] = z;
+        }
+        acc[c] = z;
+        v[c] = act_apply(p.act, z);
+    }
+    if (p.fa.mode == 1) {  // cache build: logits rows and original predictions
+        if (in_range) {
+            for (int c = 0; c < p.C; ++c) p.fa.x_out[row * p.fa.x_stride + c] = v[c];
+            p.fa.pred_out[row] = argmax_first(v, p.C);
+        }
+        return;
+    }
+    if (p.fa.mode == 2) {  // per-row logits for a following delta + epilogue
+        if (in_range)
+            for (int c = 0; c < p.C; ++c) p.fa.logits_rows[row * p.fa.x_stride + c] = v[c];
+        return;
+    }
+    epilogue_row(p.fa, p.t0, p.T, row, in_range, v, p.C);
+}
+
+__global__ void __launch_bounds__(128) k_epilogue(const float *__restrict__ lg, int64_t stride, int C, int64_t t0, int T,
+                                                  int R, const FinalArgs fa)
+{
+    const int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const bool in_range = row < R;
+    float v[kMaxClasses];
+#pragma unroll
+    for (int c = 0; c < kMaxClasses; ++c) v[c] = (in_range && c < C) ? lg[row * stride + c] : 0.f;
+    epilogue_row(fa, t0, T, row, in_range, v, C);
+}
+
+int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s)
+{
+    if (rm.R <= 0) return 0;
+    FinalParams p{};
+    p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
+    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
+    p.F = S.K; p.C = S.oc; p.act = S.act1;
+    p.W = S.W; p.b = S.b;
+    p.fa = fa;
+    k_final_dense<<<(unsigned)((rm.R + 127) / 128), 128, 0, s>>>(p);
+    return 1;
+}
+
+int launch_epilogue(Src logits, int C, RowMap rm, const FinalArgs &fa, cudaStream_t s)
+{
+    if (rm.R <= 0) return 0;
+    k_epilogue<<<(unsigned)((rm.R + 127) / 128), 128, 0, s>>>(logits.p, logits.stride, C, rm.t0, rm.T, rm.R, fa);
+    return 1;
+}
+
+// ----------------------------------------------------------------- row copies --
+
+__global__ void k_gather_rows(const float4 *__restrict__ src, int64_t src_stride4, int64_t n4, int64_t t0, int T,
+                              int64_t R, float4 *__restrict__ dst, int64_t dst_stride4)
+{
+    const int64_t total = R * n4;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = i / n4, e = i % n4;
+        dst[r * dst_stride4 + e] = __ldg(src + (t0 + r % T) * src_stride4 + e);
+    }
+}
+
+int launch_gather_rows(Src src, int64_t n_elems, RowMap rm, float *dst, int64_t dst_stride, cudaStream_t s)
+{
+    if (rm.R <= 0) return 0;
+    const int64_t n4 = (n_elems + 3) / 4;
+    const int64_t total = (int64_t)rm.R * n4;
+    int64_t blocks = (total + 255) / 256;
+    if (blocks > 152 * 32) blocks = 152 * 32;
+    k_gather_rows<<<(unsigned)blocks, 256, 0, s>>>(reinterpret_cast<const float4 *>(src.p), src.stride / 4, n4, rm.t0,
+                                                   rm.T, rm.R, reinterpret_cast<float4 *>(dst), dst_stride / 4);
+    return 1;
+}
+
+}  // namespace mure
