@@ -1,0 +1,374 @@
+"""Benchmark of memoized DNN mutation testing on GB300.
+
+One step = the whole hot path over the workload: the prefix-activation cache of the
+inputs (Algorithm 1 lines 10-12), descriptor expansion and grouping, the delta and
+suffix kernels of every mutant group, the fused kill epilogue and the score
+reduction.  Default workload: LeNet-5 (28x28x1), 10,000 inputs, 2,000 mutants at a
+1% selection ratio (GF / NEB / NAI / NS), random He-normal weights.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+Prints one JSON line (rank 0).  N > 1 runs N independent replicas (one per GPU,
+launched by torchrun); the path has no cross-GPU exchange.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "mutant×input evals/sec at 1 GB300; suffix-GEMM tensor-pipe % of peak"
+UNIT = "evals/s"
+# CUDA-core fp32 peak of a GB300: 152 SMs x 128 FP32 lanes x 2 FLOP (FMA) x 2.07 GHz
+SIMT_FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
+L2_FLUSH_BYTES = 256 << 20
+
+WORKLOAD_TEXT = {
+    "lenet5": "LeNet-5 28x28x1 (conv5x5 6 pad2, pool, conv5x5 16, pool, FC 400-120-84-10), 10,000 inputs U[0,1], "
+              "2,000 single-layer mutants, 1% selection ratio, GF/NEB/NAI/NS, layer uniform over 5",
+    "mlp": "MLP 784-128-64-10, 1,000 inputs U[0,1], 200 mutants, 1% ratio",
+    "resnet20": "ResNet-20 32x32x3, 10,000 inputs N(0,1), 5,000 mutants, 1% ratio",
+    "vgg": "VGG-style 32x32x3 (8 weighted layers), 10,000 inputs N(0,1), 5,000 mutants, ratios 0.5/1/2/5%",
+}
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+# ------------------------------------------------------------------- clocks --
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device):
+        self.device = device
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "200", "-i", str(self.device)],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for l in getattr(self, "lines", []):
+            p = [x.strip() for x in l.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                mx.append(float(p[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, p[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------- ncu traffic file --
+
+def profiled_traffic(kernel_key, rows_per_launch):
+    """DRAM bytes per launch of the dominant kernel from its committed ncu summary,
+    scaled by rows; None when the summary is missing or the kernel source changed
+    since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", f"{kernel_key}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m_bytes = re.search(r"dram_bytes_per_row:\s*([0-9.eE+]+)", text)
+    m_sha = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
+    m_src = re.search(r"source_file:\s*(\S+)", text)
+    if not (m_bytes and m_sha and m_src):
+        return None
+    try:
+        cur = hashlib.sha256(open(os.path.join(ROOT, m_src.group(1)), "rb").read()).hexdigest()
+    except OSError:
+        return None
+    if cur != m_sha.group(1):
+        return None
+    return float(m_bytes.group(1)) * rows_per_launch
+
+
+# ------------------------------------------------------------- distributed --
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------- oracle leg --
+
+def oracle_sample(w, n_mut, n_in, seed=0):
+    from paper_2607_18582_gb300 import workloads as wl
+    idx = wl.stratified(w.table, w.model, max(1, n_mut // (w.model.n_layers() * 4)))
+    rng = np.random.default_rng(seed)
+    if len(idx) < n_mut:
+        rest = np.setdiff1d(np.arange(len(w.table)), idx)
+        idx = np.sort(np.concatenate([idx, rng.choice(rest, min(len(rest), n_mut - len(idx)), replace=False)]))
+    return w.table.subset(idx[:n_mut]), w.X[:n_in]
+
+
+def cpu_oracle_rate(w, n_mut, n_in, threads):
+    """Oracle (memoized, Algorithm 1 on the CPU) evals/s on a bounded sample."""
+    import oracle
+    table, X = oracle_sample(w, n_mut, n_in)
+    t = time.perf_counter()
+    oracle.memo(w.model, X, table, n_threads=threads, want_logits=False)
+    dt = time.perf_counter() - t
+    return len(table) * len(X) / dt, dt, f"{len(table)} stratified mutants x first {len(X)} inputs, oracle memoized mode"
+
+
+def run_reference(args, world, rank):
+    """The reference arm: the CPU oracle as it stands, on bounded samples."""
+    if rank != 0:
+        return 0
+    from paper_2607_18582_gb300 import workloads as wl
+    import oracle
+    oracle.build()
+    w = wl.workload(args.workload)
+    threads = os.cpu_count() or 1
+    n_mut, n_in = 40, 500
+    for _ in range(args.warmup):
+        cpu_oracle_rate(w, n_mut, n_in, threads)
+    t = time.perf_counter()
+    for _ in range(args.steps):
+        _, _, sample = cpu_oracle_rate(w, n_mut, n_in, threads)
+    dt = time.perf_counter() - t
+    value = args.steps * n_mut * n_in / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32 (fp64 accumulation)",
+            "data": "synthetic", "config": config_block(args, w),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_block(args, w):
+    small = any(getattr(args, k, None) is not None for k in ("n_inputs", "n_mutants", "only_layer"))
+    return {"workload": f"{args.workload}: {WORKLOAD_TEXT.get(args.workload, args.workload)}"
+                        + (" [reduced profiling case]" if small else ""),
+            "n_inputs": int(len(w.X)), "n_mutants": int(len(w.table)), "n_layers": w.model.n_layers(),
+            "seeds": {"model": 0, "inputs": 1, "mutants": 2},
+            "l2": "flushed between timed steps (256 MiB write, outside the step events)",
+            "parallelism": f"{args.gpus} independent replica(s), no cross-GPU exchange"}
+
+
+# ----------------------------------------------------------------- GPU leg --
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="lenet5")
+    ap.add_argument("--skip-cpu-baseline", action="store_true")
+    ap.add_argument("--skip-extras", action="store_true", help="no e2e / vanilla / clocks legs")
+    ap.add_argument("--n-inputs", type=int, default=None, help="smaller case (profiling): first n inputs")
+    ap.add_argument("--n-mutants", type=int, default=None, help="smaller case (profiling): first n mutants")
+    ap.add_argument("--only-layer", type=int, default=None, help="keep only the mutants of this layer")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        return run_reference(args, world, rank)
+
+    import torch
+    from paper_2607_18582_gb300 import mure, workloads as wl
+
+    dev = local
+    torch.cuda.set_device(dev)
+    w = wl.workload(args.workload, args.n_inputs, args.n_mutants)
+    if args.only_layer is not None:
+        w.table = w.table.subset(np.nonzero(w.table.layer == args.only_layer)[0])
+    n_evals = len(w.table) * len(w.X)
+    ctx = mure.mure_create(dev)
+    model = mure.mure_model_load(ctx, w.model)
+    X_dev = torch.from_numpy(w.X).to(f"cuda:{dev}")
+    arrays = mure.table_array(w.table)
+    W64 = (len(w.X) + 63) // 64
+    kill_dev = torch.empty((len(w.table), W64), dtype=torch.int64, device=f"cuda:{dev}")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=f"cuda:{dev}")
+    stream = torch.cuda.current_stream(dev)
+
+    def step(timing):
+        cache = mure.mure_build_prefix_cache(model, X_dev)
+        r = mure.mure_eval_mutants(cache, w.table, outputs_on_device=True, kill_out=kill_dev, kernel_timing=timing,
+                                   arrays=arrays)
+        del cache
+        return r
+
+    for _ in range(args.warmup):
+        step(True)
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    launches0 = mure.mure_kernel_launches(ctx)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    results = []
+    with ClockSampler(dev) as clk:
+        for i in range(args.steps):
+            flush.zero_()                       # evict L2 between steps (not timed)
+            evs[i][0].record(stream)
+            results.append(step(True))
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    launches = mure.mure_kernel_launches(ctx) - launches0
+    ms = [a.elapsed_time(b) for a, b in evs]
+    t_total = max_over_ranks(sum(ms) / 1e3, world)
+    value = world * args.steps * n_evals / t_total
+    last = results[-1]
+
+    # dominant kernel: the layer (or delta / gather) class with the largest device time
+    L = w.model.n_layers()
+    cls_ms = {f"layer{v}": sum(r["stats"]["ms_layer"][v] for r in results) for v in range(L)}
+    cls_ms["delta"] = sum(r["stats"]["ms_delta"] for r in results)
+    cls_ms["gather"] = sum(r["stats"]["ms_gather"] for r in results)
+    cls_ms["epilogue"] = sum(r["stats"]["ms_epilogue"] for r in results)
+    top = max(cls_ms, key=cls_ms.get)
+    roof = None
+    pk, pk_kind = peaks()
+    if top.startswith("layer"):
+        v = int(top[5:])
+        fl = sum(r["stats"]["flops_layer"][v] for r in results)
+        nl = sum(r["stats"]["launches_layer"][v] for r in results)
+        achieved = fl / (cls_ms[top] / 1e3) / 1e12
+        layer_node = w.model.nodes[w.model.layers()[v]]
+        rows = fl / 2 / w.model.layer_macs(v) / max(1, nl)   # rows per launch
+        roof = {"bound": "alu", "achieved": achieved, "peak": SIMT_FP32_PEAK_TFLOPS, "unit": "TFLOP/s",
+                "frac": achieved / SIMT_FP32_PEAK_TFLOPS,
+                "traffic": profiled_traffic(f"stage_simt_{args.workload}_layer{v}", rows),
+                "rows_per_launch": rows,
+                "kernel": f"k_stage_simt (layer {v}: {layer_node.kind} {layer_node.cin}->{layer_node.cout})",
+                "launches": nl, "ms_total": cls_ms[top],
+                "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz (no tensor cores on this path)",
+                "tensor_pipe_frac": 0.0}
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": 1e3 * t_total / args.steps, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+           "config": config_block(args, w), "roofline": roof, "gpu_launches": int(launches),
+           "kernel_ms_per_step": {k: v / args.steps for k, v in cls_ms.items()},
+           "scores": {"killed_frac": last["scoreA"], "deepmutation": last["scoreB"],
+                      "near_ties": last["stats"]["n_near_ties"]}}
+
+    if not args.skip_extras:
+        out["clocks"] = clk.summary()
+        # end to end through the C ABI with host buffers: pinned X in, kill bits out
+        X_pin = torch.from_numpy(w.X).pin_memory()
+        kill_host = np.zeros((len(w.table), W64), np.uint64)
+        k_e2e = max(3, min(args.steps, 5))
+
+        def step_e2e():
+            cache = mure.mure_build_prefix_cache(model, X_pin.numpy())
+            return mure.mure_eval_mutants(cache, w.table, kill_out=kill_host, arrays=arrays)
+
+        step_e2e()
+        times = []
+        for _ in range(k_e2e):
+            flush.zero_()
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            step_e2e()          # synchronous: returns with the kill bits in host memory
+            times.append(time.perf_counter() - t0)
+        e2e_t = max_over_ranks(sum(times) / k_e2e, world)
+        h2d = int(w.X.nbytes + arrays[0].nbytes + arrays[1].nbytes)
+        d2h = int(kill_host.nbytes + 32)
+        out["e2e"] = {"value": world * n_evals / e2e_t, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                      "d2h_bytes_per_step": d2h, "steps": k_e2e}
+        # the GPU vanilla mode (speed-up denominator), same kernels, no reuse
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        van = mure.mure_eval_vanilla(model, X_dev, w.table, outputs_on_device=True)
+        torch.cuda.synchronize()
+        tv = time.perf_counter() - t0
+        same = bool(torch.equal(van["kill_bits"], kill_dev))
+        t_m = t_total / args.steps
+        out["gpu_vanilla"] = {"value": n_evals / tv, "ms_per_step": 1e3 * tv, "speedup": tv / t_m,
+                              "gain": (tv - t_m) / tv, "kill_matrix_identical": same}
+    if rank == 0 and world == 1 and not args.skip_cpu_baseline:
+        import oracle
+        oracle.build()
+        threads = os.cpu_count() or 1
+        rate, dt, sample = cpu_oracle_rate(w, 400, 2000, threads)
+        out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
+                               "seconds": dt}
+    out["peaks"] = {"source": pk_kind, "hbm_gbs": pk.get("hbm_gbs"), "bf16_tflops": pk.get("bf16_tflops")}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

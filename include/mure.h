@@ -131,7 +131,8 @@ typedef struct {
 
 typedef struct {
     int32_t outputs_on_device; /* kill_bits / logits_out are device pointers */
-    int32_t reserved;
+    int32_t kernel_timing;     /* 1: time every kernel launch with CUDA events on the
+                                  context stream and report per-layer times in stats */
     int64_t workspace_bytes;   /* cap on per-batch scratch (0: 8 GiB) */
     float *logits_out;         /* nullable; [n_mutants][n_inputs][n_classes]: every
                                   mutant's logits (for parity checks; slows the run) */
@@ -148,7 +149,18 @@ typedef struct {
     int64_t n_batches;      /* (group, mutant chunk, input tile) batches */
     int64_t kernel_launches;/* library kernels launched by the call */
     int64_t flops;          /* analytic FLOPs of the layer kernels that ran */
+    /* with kernel_timing: device time and analytic FLOPs / bytes of the kernels of
+       each weighted layer (index = layer, up to MURE_MAX_TIMED_LAYERS), of the delta
+       kernel, of the row-gather copies and of the stand-alone kill epilogue */
+    double ms_layer[64];
+    int64_t flops_layer[64];
+    int64_t launches_layer[64];
+    double ms_delta, ms_gather, ms_epilogue;
+    int64_t bytes_gather;   /* bytes read + written by the row-gather copies */
+    int64_t launches_delta;
 } mure_eval_stats;
+
+#define MURE_MAX_TIMED_LAYERS 64
 
 typedef struct mure_ctx mure_ctx;
 typedef struct mure_model mure_model;
@@ -172,6 +184,9 @@ const char *mure_last_error(const mure_ctx *ctx);
  * supported shape, n_classes > 32, unknown precision), OOM, CUDA. */
 mure_status mure_model_load(mure_ctx *ctx, const mure_model_desc *desc, mure_model **out);
 void mure_model_free(mure_model *model);
+
+/* Kernels this context has launched since it was created (all calls). */
+int64_t mure_kernel_launches(const mure_ctx *ctx);
 
 /* Number of weighted layers L of a loaded model (or -1 for NULL). */
 int32_t mure_model_n_layers(const mure_model *model);

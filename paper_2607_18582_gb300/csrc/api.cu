@@ -108,6 +108,48 @@ void check_launch(mure_ctx *c)
     FAILIF(e != cudaSuccess, c, MURE_ERR_CUDA, "kernel launch: %s", cudaGetErrorString(e));
 }
 
+// Optional per-launch device timing: a pair of events around each launch, summed
+// per class (a layer's kernels, delta, gather, epilogue) once the stream is idle.
+struct KTimer {
+    mure_ctx *c;
+    bool on;
+    struct Rec {
+        int cls;
+        cudaEvent_t a, b;
+    };
+    std::vector<Rec> recs;
+    KTimer(mure_ctx *ctx, bool enabled) : c(ctx), on(enabled) {}
+    cudaEvent_t ev(size_t i)
+    {
+        while (c->evpool.size() <= i) {
+            cudaEvent_t e;
+            CK(c, cudaEventCreate(&e));
+            c->evpool.push_back(e);
+        }
+        return c->evpool[i];
+    }
+    void begin(int cls)
+    {
+        if (!on) return;
+        Rec r{cls, ev(2 * recs.size()), ev(2 * recs.size() + 1)};
+        CK(c, cudaEventRecord(r.a, c->stream));
+        recs.push_back(r);
+    }
+    void end()
+    {
+        if (on) CK(c, cudaEventRecord(recs.back().b, c->stream));
+    }
+    // after the stream is idle
+    void collect(std::vector<double> &ms)
+    {
+        for (const Rec &r : recs) {
+            float t = 0;
+            CK(c, cudaEventElapsedTime(&t, r.a, r.b));
+            if (r.cls >= 0 && r.cls < (int)ms.size()) ms[r.cls] += t;
+        }
+    }
+};
+
 // ---------------------------------------------------------- model compilation --
 
 struct Shape {
@@ -334,6 +376,8 @@ struct DevTable {
     float *patch;
     int64_t n_jobs, patch_len;
     std::vector<int> kmax_layer;
+    std::vector<int64_t> dot_prefix;   // [n+1] prefix sums of GF/WS neuron slots (group order)
+    int expand_launches = 0;
 };
 
 DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_mutant *t, int64_t n,
@@ -370,6 +414,9 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
     }
     dt.n_jobs = (int64_t)jobs.size();
     dt.patch_len = plen;
+    dt.dot_prefix.assign(n + 1, 0);
+    for (int64_t k = 0; k < n; ++k)
+        dt.dot_prefix[k + 1] = dt.dot_prefix[k] + ((op[k] == MURE_OP_GF || op[k] == MURE_OP_WS) ? nn[k] : 0);
     // one staging buffer, one H2D copy
     const size_t b_op = n * 4, b_nn = n * 4, b_mid = n * 4, b_noff = n * 8, b_poff = n * 8;
     const size_t b_ids = (size_t)std::max<int64_t>(pool_len, 1) * 4, b_jobs = jobs.size() * sizeof(SlotJob);
@@ -407,7 +454,7 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
         ea.patch = dt.patch;
         ea.perm = perm_len ? sc.get<int32_t>(perm_len) : nullptr;
         ea.ws_as_weights = ws_as_weights;
-        launch_expand(ea, c->stream);
+        dt.expand_launches = launch_expand(ea, c->stream);
         check_launch(c);
         if (patch_out) CK(c, cudaMemcpyAsync(patch_out, dt.patch, plen * 4, cudaMemcpyDeviceToHost, c->stream));
     }
@@ -478,12 +525,28 @@ void alloc_workspace(mure_ctx *c, Scratch &sc, const mure_model *m, int64_t rows
 }
 
 // One batch: G mutants of group l (starting at group position g0) x an input tile.
+struct Acct {
+    int64_t flops = 0;
+    std::vector<int64_t> flops_cls, launches_cls;   // [L + 3]
+    int64_t bytes_gather = 0;
+};
+
 int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevTable &dt, const EvalCfg &ec,
-              const Workspace &ws, int l, int64_t g0, RowMap rm, bool vanilla, int64_t &flops)
+              const Workspace &ws, int l, int64_t g0, RowMap rm, bool vanilla, Acct &acct, KTimer &tm)
 {
     cudaStream_t s = c->stream;
     const int L = m->L;
+    const int C_DELTA = L, C_GATHER = L + 1, C_EPI = L + 2;
     int launches = 0;
+    auto timed = [&](int cls, int64_t fl, auto &&launch) {
+        tm.begin(cls);
+        const int n = launch();
+        tm.end();
+        launches += n;
+        acct.launches_cls[cls] += n;
+        acct.flops_cls[cls] += fl;
+        acct.flops += fl;
+    };
     PatchArgs pa{dt.op + g0, dt.nn + g0, dt.noff + g0, dt.ids, dt.poff + g0, dt.patch};
     FinalArgs fa{};
     fa.mutant_id = dt.mid + g0;
@@ -504,17 +567,23 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         return Src{ws.xb[s2], m->xd[s2].stride, 0};
     };
     auto skip_of = [&](const Stage &S) -> Src { return S.has_add ? xsrc(S.skip_src) : Src{nullptr, 0, 0}; };
+    auto stage = [&](int v, float *z_out, int64_t z_stride) {
+        const Stage &S = m->st[v];
+        timed(v, 2 * S.macs * rm.R, [&] {
+            return launch_stage_simt(S, xsrc(v), rm, z_out, z_stride, skip_of(S), ws.xb[v + 1], m->xd[v + 1].stride,
+                                     ws.gap_tmp, s);
+        });
+    };
     const Stage &Sl = m->st[l];
+    // GF / WS recompute k channels' dot products; the other operators are copies
+    const int64_t G = rm.R / rm.T;
+    const int64_t delta_flops =
+        (dt.dot_prefix[g0 + G] - dt.dot_prefix[g0]) * rm.T * 2 * (int64_t)Sl.oh * Sl.ow * Sl.K;
     if (vanilla) {
         // the prefix, then layer l itself, from the inputs, row by row
-        for (int v = 0; v < l; ++v) {
-            launches += launch_stage_simt(m->st[v], xsrc(v), rm, nullptr, 0, skip_of(m->st[v]), ws.xb[v + 1],
-                                          m->xd[v + 1].stride, ws.gap_tmp, s);
-            flops += 2 * m->st[v].macs * rm.R;
-        }
+        for (int v = 0; v < l; ++v) stage(v, nullptr, 0);
         if (l < L - 1) {
-            launches += launch_stage_simt(Sl, xsrc(l), rm, ws.zb, ws.z_stride, skip_of(Sl), ws.xb[l + 1],
-                                          m->xd[l + 1].stride, ws.gap_tmp, s);
+            stage(l, ws.zb, ws.z_stride);
         } else {
             FinalArgs f2 = fa;
             f2.mode = 2;
@@ -522,29 +591,31 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
             f2.z_stride = ws.z_stride;
             f2.logits_rows = ws.xb[L];
             f2.x_stride = m->xd[L].stride;
-            launches += launch_final_dense(Sl, xsrc(l), rm, f2, s);
+            timed(l, 2 * Sl.macs * rm.R, [&] { return launch_final_dense(Sl, xsrc(l), rm, f2, s); });
         }
-        flops += 2 * Sl.macs * rm.R;
-        launches += launch_delta(Sl, Src{ws.zb, ws.z_stride, 0}, xsrc(l), skip_of(Sl), rm, pa, dt.kmax_layer[l],
-                                 ws.xb[l + 1], m->xd[l + 1].stride, s);
+        timed(C_DELTA, delta_flops, [&] {
+            return launch_delta(Sl, Src{ws.zb, ws.z_stride, 0}, xsrc(l), skip_of(Sl), rm, pa, dt.kmax_layer[l],
+                                ws.xb[l + 1], m->xd[l + 1].stride, s);
+        });
     } else {
         // memo rows start as the cached output of layer l, then the mutated channels
-        launches += launch_gather_rows(Src{ca->x[l + 1], m->xd[l + 1].stride, 1}, m->xd[l + 1].stride, rm,
-                                       ws.xb[l + 1], m->xd[l + 1].stride, s);
-        launches += launch_delta(Sl, Src{ca->z[l], m->zd[l].stride, 1}, xsrc(l), skip_of(Sl), rm, pa,
-                                 dt.kmax_layer[l], ws.xb[l + 1], m->xd[l + 1].stride, s);
+        acct.bytes_gather += 2 * (int64_t)rm.R * m->xd[l + 1].stride * 4;
+        timed(C_GATHER, 0, [&] {
+            return launch_gather_rows(Src{ca->x[l + 1], m->xd[l + 1].stride, 1}, m->xd[l + 1].stride, rm,
+                                      ws.xb[l + 1], m->xd[l + 1].stride, s);
+        });
+        timed(C_DELTA, delta_flops, [&] {
+            return launch_delta(Sl, Src{ca->z[l], m->zd[l].stride, 1}, xsrc(l), skip_of(Sl), rm, pa,
+                                dt.kmax_layer[l], ws.xb[l + 1], m->xd[l + 1].stride, s);
+        });
     }
     // the suffix l+1 .. L-1 (Algorithm 4) and the fused kill epilogue
-    for (int v = l + 1; v < L - 1; ++v) {
-        launches += launch_stage_simt(m->st[v], xsrc(v), rm, nullptr, 0, skip_of(m->st[v]), ws.xb[v + 1],
-                                      m->xd[v + 1].stride, ws.gap_tmp, s);
-        flops += 2 * m->st[v].macs * rm.R;
-    }
+    for (int v = l + 1; v < L - 1; ++v) stage(v, nullptr, 0);
     if (l < L - 1) {
-        launches += launch_final_dense(m->st[L - 1], xsrc(L - 1), rm, fa, s);
-        flops += 2 * m->st[L - 1].macs * rm.R;
+        const Stage &SL = m->st[L - 1];
+        timed(L - 1, 2 * SL.macs * rm.R, [&] { return launch_final_dense(SL, xsrc(L - 1), rm, fa, s); });
     } else {
-        launches += launch_epilogue(Src{ws.xb[L], m->xd[L].stride, 0}, m->n_classes, rm, fa, s);
+        timed(C_EPI, 0, [&] { return launch_epilogue(Src{ws.xb[L], m->xd[L].stride, 0}, m->n_classes, rm, fa, s); });
     }
     return launches;
 }
@@ -600,7 +671,11 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         rows = std::min(Gmax, gbig) * T;
         Workspace ws;
         alloc_workspace(c, sc, m, rows, vanilla, lmin, ws);
-        int64_t launches = 0, flops = 0;
+        int64_t launches = 0;
+        Acct acct;
+        acct.flops_cls.assign(m->L + 3, 0);
+        acct.launches_cls.assign(m->L + 3, 0);
+        KTimer tm(c, o->kernel_timing != 0);
         for (int l = 0; l < m->L; ++l) {
             const int64_t gs = g.begin[l], ge = g.begin[l + 1];
             if (ge == gs) continue;
@@ -610,7 +685,7 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
                 for (int64_t g0 = gs; g0 < ge; g0 += Gmax) {
                     const int64_t G = std::min<int64_t>(Gmax, ge - g0);
                     RowMap rm{t0, Tt, (int)(G * Tt)};
-                    launches += run_batch(c, m, ca, dt, ec, ws, l, g0, rm, vanilla, flops);
+                    launches += run_batch(c, m, ca, dt, ec, ws, l, g0, rm, vanilla, acct, tm);
                     check_launch(c);
                     ++st.n_batches;
                 }
@@ -634,8 +709,23 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         sA = (double)host_cnt[0] / (double)n;
         sB = ca->n_label_values > 0 ? (double)host_cnt[1] / ((double)n * ca->n_label_values) : 0.0;
         st.n_near_ties = (int64_t)host_cnt[2];
-        st.kernel_launches = launches + (dt.n_jobs ? 1 : 0);
-        st.flops = flops;
+        st.kernel_launches = launches + dt.expand_launches;
+        c->launches += st.kernel_launches;
+        st.flops = acct.flops;
+        if (tm.on) {
+            std::vector<double> ms(m->L + 3, 0.0);
+            tm.collect(ms);
+            for (int v = 0; v < m->L && v < MURE_MAX_TIMED_LAYERS; ++v) {
+                st.ms_layer[v] = ms[v];
+                st.flops_layer[v] = acct.flops_cls[v];
+                st.launches_layer[v] = acct.launches_cls[v];
+            }
+            st.ms_delta = ms[m->L];
+            st.ms_gather = ms[m->L + 1];
+            st.ms_epilogue = ms[m->L + 2];
+            st.launches_delta = acct.launches_cls[m->L];
+        }
+        st.bytes_gather = acct.bytes_gather;
         float ms = 0;
         cudaEventElapsedTime(&ms, c->ev[0], c->ev[4]); st.ms_total = ms;
         cudaEventElapsedTime(&ms, c->ev[0], c->ev[1]); st.ms_expand = ms;
@@ -714,8 +804,8 @@ mure_cache *build_cache(mure_model *m, const float *X, int64_t n_in, const int32
         for (int v = 0; v < L - 1; ++v) {
             const Stage &S = m->st[v];
             const Src skip = S.has_add ? Src{xs[S.skip_src], m->xd[S.skip_src].stride, 0} : Src{nullptr, 0, 0};
-            launch_stage_simt(S, Src{xs[v], m->xd[v].stride, 0}, rm, zs[v], m->zd[v].stride, skip, xs[v + 1],
-                              m->xd[v + 1].stride, gap_tmp, s);
+            c->launches += launch_stage_simt(S, Src{xs[v], m->xd[v].stride, 0}, rm, zs[v], m->zd[v].stride, skip,
+                                             xs[v + 1], m->xd[v + 1].stride, gap_tmp, s);
             check_launch(c);
         }
         FinalArgs fa{};
@@ -725,13 +815,13 @@ mure_cache *build_cache(mure_model *m, const float *X, int64_t n_in, const int32
         fa.x_out = xs[L];
         fa.x_stride = m->xd[L].stride;
         fa.pred_out = ca->pred0;
-        launch_final_dense(m->st[L - 1], Src{xs[L - 1], m->xd[L - 1].stride, 0}, rm, fa, s);
+        c->launches += launch_final_dense(m->st[L - 1], Src{xs[L - 1], m->xd[L - 1].stride, 0}, rm, fa, s);
         check_launch(c);
         if (labels) CK(c, cudaMemcpyAsync(ca->label, lab_host.data(), n_in * 4, cudaMemcpyHostToDevice, s));
         else CK(c, cudaMemcpyAsync(ca->label, ca->pred0, n_in * 4, cudaMemcpyDeviceToDevice, s));
         uint32_t *mask = sc.get<uint32_t>(1);
         CK(c, cudaMemsetAsync(mask, 0, 4, s));
-        launch_label_set(ca->label, n_in, mask, s);
+        c->launches += launch_label_set(ca->label, n_in, mask, s);
         check_launch(c);
         uint32_t hm = 0;
         CK(c, cudaMemcpyAsync(&hm, mask, 4, cudaMemcpyDeviceToHost, s));
@@ -782,6 +872,7 @@ void mure_destroy(mure_ctx *ctx)
     if (!ctx) return;
     for (auto &e : ctx->ev)
         if (e) cudaEventDestroy(e);
+    for (auto &e : ctx->evpool) cudaEventDestroy(e);
     delete ctx;
 }
 
@@ -839,7 +930,7 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             m->sigma_dev = (double *)dalloc(c, m->L * 8);
             CK(c, cudaMemcpyAsync(Wd, Wp.data(), m->L * sizeof(float *), cudaMemcpyHostToDevice, c->stream));
             CK(c, cudaMemcpyAsync(nd, cnt.data(), m->L * 8, cudaMemcpyHostToDevice, c->stream));
-            launch_layer_std(Wd, nd, m->L, m->sigma_dev, c->stream);
+            c->launches += launch_layer_std(Wd, nd, m->L, m->sigma_dev, c->stream);
             check_launch(c);
             m->sigma_host.resize(m->L);
             CK(c, cudaMemcpyAsync(m->sigma_host.data(), m->sigma_dev, m->L * 8, cudaMemcpyDeviceToHost, c->stream));
@@ -865,6 +956,8 @@ void mure_model_free(mure_model *m)
 }
 
 int32_t mure_model_n_layers(const mure_model *m) { return m ? m->L : -1; }
+
+int64_t mure_kernel_launches(const mure_ctx *ctx) { return ctx ? ctx->launches : -1; }
 
 mure_status mure_build_prefix_cache(mure_model *m, const float *X, int64_t n_inputs, const int32_t *labels,
                                     int x_on_device, mure_cache **out)
@@ -963,7 +1056,8 @@ mure_status mure_expand_patches(mure_model *m, const mure_mutant *table, int64_t
         g.begin.assign(m->L + 1, n_mutants);
         g.begin[0] = 0;
         Scratch sc(c);
-        upload_table(c, sc, m, table, n_mutants, neuron_pool, pool_len, g, 1, out, offsets);
+        const DevTable dt = upload_table(c, sc, m, table, n_mutants, neuron_pool, pool_len, g, 1, out, offsets);
+        c->launches += dt.expand_launches;
         CK(c, cudaStreamSynchronize(c->stream));
     });
 }

@@ -52,7 +52,9 @@ struct mure_ctx {
     bool has_alloc = false;
     std::string err;
     cudaEvent_t ev[8]{};
+    std::vector<cudaEvent_t> evpool;  // per-launch timing events, reused across calls
     int n_sms = 0;
+    int64_t launches = 0;             // kernels launched since creation
 };
 
 struct mure_model {

@@ -23,7 +23,7 @@ PRECISIONS = {"fp32": 0, "tf32x3": 1, "bf16": 2}
 
 # the exported entry points of include/mure.h
 EXPORTS = ("mure_create", "mure_destroy", "mure_last_error", "mure_model_load", "mure_model_free",
-           "mure_model_n_layers", "mure_build_prefix_cache", "mure_cache_free", "mure_cache_outputs",
+           "mure_model_n_layers", "mure_kernel_launches", "mure_build_prefix_cache", "mure_cache_free", "mure_cache_outputs",
            "mure_eval_mutants", "mure_eval_vanilla", "mure_expand_patches")
 
 
@@ -56,7 +56,7 @@ class _Allocator(C.Structure):
 
 
 class _Opts(C.Structure):
-    _fields_ = [("outputs_on_device", C.c_int32), ("reserved", C.c_int32), ("workspace_bytes", C.c_int64),
+    _fields_ = [("outputs_on_device", C.c_int32), ("kernel_timing", C.c_int32), ("workspace_bytes", C.c_int64),
                 ("logits_out", C.c_void_p)]
 
 
@@ -64,10 +64,16 @@ class _Stats(C.Structure):
     _fields_ = [("ms_total", C.c_double), ("ms_expand", C.c_double), ("ms_suffix", C.c_double),
                 ("ms_score", C.c_double), ("n_rows", C.c_int64), ("n_near_ties", C.c_int64),
                 ("n_groups", C.c_int64), ("n_batches", C.c_int64), ("kernel_launches", C.c_int64),
-                ("flops", C.c_int64)]
+                ("flops", C.c_int64), ("ms_layer", C.c_double * 64), ("flops_layer", C.c_int64 * 64),
+                ("launches_layer", C.c_int64 * 64), ("ms_delta", C.c_double), ("ms_gather", C.c_double),
+                ("ms_epilogue", C.c_double), ("bytes_gather", C.c_int64), ("launches_delta", C.c_int64)]
 
     def as_dict(self):
-        return {k: getattr(self, k) for k, _ in self._fields_}
+        out = {}
+        for k, _ in self._fields_:
+            v = getattr(self, k)
+            out[k] = list(v) if hasattr(v, "__len__") else v
+        return out
 
 
 _lib = None
@@ -92,6 +98,8 @@ def lib():
         L.mure_model_free.restype = None
         L.mure_model_n_layers.argtypes = [vp]
         L.mure_model_n_layers.restype = i32
+        L.mure_kernel_launches.argtypes = [vp]
+        L.mure_kernel_launches.restype = i64
         L.mure_build_prefix_cache.argtypes = [vp, vp, i64, vp, C.c_int, C.POINTER(vp)]
         L.mure_cache_free.argtypes = [vp]
         L.mure_cache_free.restype = None
@@ -103,7 +111,7 @@ def lib():
         L.mure_expand_patches.argtypes = [vp, vp, i64, vp, i64, vp, i64, vp]
         for name in EXPORTS:
             if name not in ("mure_destroy", "mure_model_free", "mure_cache_free", "mure_last_error",
-                            "mure_model_n_layers"):
+                            "mure_model_n_layers", "mure_kernel_launches"):
                 getattr(L, name).restype = C.c_int
         _lib = L
     return _lib
@@ -258,7 +266,7 @@ def table_array(table):
     return arr, pool, int(table.pool.size)
 
 
-def _eval_common(n_mut, n_in, n_classes, logits, outputs_on_device, workspace_bytes, kill_out):
+def _eval_common(n_mut, n_in, n_classes, logits, outputs_on_device, workspace_bytes, kill_out, kernel_timing=False):
     W64 = (n_in + 63) // 64
     if outputs_on_device:
         import torch
@@ -268,7 +276,7 @@ def _eval_common(n_mut, n_in, n_classes, logits, outputs_on_device, workspace_by
     else:
         kill = kill_out if kill_out is not None else np.zeros((max(n_mut, 1), max(W64, 1)), np.uint64)
         lg = np.zeros((n_mut, n_in, n_classes), np.float32) if logits else None
-    opts = _Opts(int(bool(outputs_on_device)), 0, int(workspace_bytes), _ptr(lg))
+    opts = _Opts(int(bool(outputs_on_device)), int(bool(kernel_timing)), int(workspace_bytes), _ptr(lg))
     return kill, lg, opts, W64
 
 
@@ -281,12 +289,12 @@ def _eval_result(kill, lg, sa, sb, st, n_mut, W64, outputs_on_device):
 
 
 def mure_eval_mutants(cache: Cache, table, logits: bool = False, outputs_on_device: bool = False,
-                      workspace_bytes: int = 0, kill_out=None):
+                      workspace_bytes: int = 0, kill_out=None, kernel_timing: bool = False, arrays=None):
     """Memoized mutation testing of `table` on the cached inputs."""
-    arr, pool, plen = table_array(table)
+    arr, pool, plen = arrays if arrays is not None else table_array(table)
     n = len(table)
     kill, lg, opts, W64 = _eval_common(n, cache.n_inputs, cache.model.src.n_classes, logits, outputs_on_device,
-                                       workspace_bytes, kill_out)
+                                       workspace_bytes, kill_out, kernel_timing)
     sa, sb, st = C.c_double(), C.c_double(), _Stats()
     cache.model.ctx.check(lib().mure_eval_mutants(cache.h, _ptr(arr), n, _ptr(pool), plen, C.byref(opts), _ptr(kill),
                                                   C.byref(sa), C.byref(sb), C.byref(st)))
@@ -294,19 +302,24 @@ def mure_eval_mutants(cache: Cache, table, logits: bool = False, outputs_on_devi
 
 
 def mure_eval_vanilla(model: Model, X, table, labels=None, logits: bool = False, outputs_on_device: bool = False,
-                      workspace_bytes: int = 0, kill_out=None):
+                      workspace_bytes: int = 0, kill_out=None, kernel_timing: bool = False):
     """Vanilla mutation testing: every mutant end to end from X."""
     X, labels, on_dev = _as_input(X, labels)
     arr, pool, plen = table_array(table)
     n = len(table)
     n_in = int(X.shape[0])
     kill, lg, opts, W64 = _eval_common(n, n_in, model.src.n_classes, logits, outputs_on_device, workspace_bytes,
-                                       kill_out)
+                                       kill_out, kernel_timing)
     sa, sb, st = C.c_double(), C.c_double(), _Stats()
     model.ctx.check(lib().mure_eval_vanilla(model.h, _ptr(X) if n_in else None, n_in, _ptr(labels), on_dev, _ptr(arr),
                                             n, _ptr(pool), plen, C.byref(opts), _ptr(kill), C.byref(sa), C.byref(sb),
                                             C.byref(st)))
     return _eval_result(kill, lg, sa, sb, st, n, W64, outputs_on_device)
+
+
+def mure_kernel_launches(ctx: Context) -> int:
+    """Kernels the context has launched since it was created."""
+    return int(lib().mure_kernel_launches(ctx.h))
 
 
 def mure_expand_patches(model: Model, table):

@@ -64,6 +64,34 @@ class Model:
     def layer_width(self, layer):
         return self.nodes[self.layers()[layer]].cout
 
+    def shapes(self):
+        """Output shape (H, W, C) of every node."""
+        out = []
+        for n in self.nodes:
+            h, w, c = self.in_shape if n.inputs[0] < 0 else out[n.inputs[0]]
+            if n.kind == "conv":
+                out.append(((h + 2 * n.pad - n.kh) // n.stride + 1, (w + 2 * n.pad - n.kw) // n.stride + 1, n.cout))
+            elif n.kind == "dense":
+                out.append((1, 1, n.cout))
+            elif n.kind == "maxpool":
+                out.append(((h - n.kh) // n.stride + 1, (w - n.kw) // n.stride + 1, c))
+            elif n.kind in ("flatten",):
+                out.append((1, 1, h * w * c))
+            elif n.kind == "gap":
+                out.append((1, 1, c))
+            elif n.kind == "shortcut":
+                out.append(((h - 1) // n.stride + 1, (w - 1) // n.stride + 1, n.cout))
+            else:
+                out.append((h, w, c))
+        return out
+
+    def layer_macs(self, layer):
+        """Multiply-accumulates of weighted layer `layer` on one input."""
+        v = self.layers()[layer]
+        n = self.nodes[v]
+        h, w, c = self.shapes()[v]
+        return h * w * c * (n.kh * n.kw * n.cin if n.kind == "conv" else n.cin)
+
 
 @dataclass
 class MutantTable:
