@@ -9,6 +9,7 @@ from __future__ import annotations
 
 import ctypes as C
 import os
+import sys
 
 import numpy as np
 
@@ -77,6 +78,13 @@ class _Stats(C.Structure):
 
 
 _lib = None
+# Allocator thunks stay alive for the life of the process: a context's C object may
+# still call them while Python tears objects down in arbitrary (cyclic-GC) order.
+_ALLOCATOR_KEEPALIVE = []
+
+
+def _finalizing():
+    return sys is None or sys.is_finalizing()
 
 
 def lib():
@@ -131,19 +139,35 @@ def _is_device(a):
 
 
 class Context:
+    """Owns a library context.  Models and caches made from it count as children; the
+    C context is destroyed only once none is alive (and never during interpreter
+    shutdown, when the process frees everything anyway)."""
+
     def __init__(self, handle, keep):
         self.h = handle
         self._keep = keep
+        self._children = 0
+        self._released = False
 
     def check(self, status):
         if status != 0:
             msg = lib().mure_last_error(self.h)
             raise MureError(status, msg.decode() if msg else "")
 
-    def __del__(self):
-        if getattr(self, "h", None):
+    def _child_gone(self):
+        self._children -= 1
+        if self._released and self._children == 0:
+            self._destroy()
+
+    def _destroy(self):
+        if self.h and not _finalizing():
             lib().mure_destroy(self.h)
-            self.h = None
+        self.h = None
+
+    def __del__(self):
+        self._released = True
+        if getattr(self, "h", None) and self._children == 0:
+            self._destroy()
 
 
 def mure_create(device: int = 0, stream=None, torch_allocator: bool = True) -> Context:
@@ -165,8 +189,13 @@ def mure_create(device: int = 0, stream=None, torch_allocator: bool = True) -> C
         def _free(ptr, strm, user):
             torch.cuda.caching_allocator_delete(ptr)
 
-        a = _Allocator(_ALLOC_FN(_alloc), _FREE_FN(_free), None)
+        def _free_guarded(ptr, strm, user):
+            if not _finalizing():
+                _free(ptr, strm, user)
+
+        a = _Allocator(_ALLOC_FN(_alloc), _FREE_FN(_free_guarded), None)
         keep += [a, a.alloc, a.free]
+        _ALLOCATOR_KEEPALIVE.append(keep)
         alloc_p = C.byref(a)
     out = C.c_void_p()
     st = lib().mure_create(device, handle_stream, alloc_p, C.byref(out))
@@ -178,15 +207,30 @@ def mure_create(device: int = 0, stream=None, torch_allocator: bool = True) -> C
 class Model:
     def __init__(self, ctx, handle, src):
         self.ctx, self.h, self.src = ctx, handle, src
+        ctx._children += 1
+        self._children = 0
+        self._released = False
 
     @property
     def n_layers(self):
         return lib().mure_model_n_layers(self.h)
 
-    def __del__(self):
-        if getattr(self, "h", None):
-            lib().mure_model_free(self.h)
+    def _child_gone(self):
+        self._children -= 1
+        if self._released and self._children == 0:
+            self._destroy()
+
+    def _destroy(self):
+        if self.h:
+            if not _finalizing():
+                lib().mure_model_free(self.h)
             self.h = None
+            self.ctx._child_gone()
+
+    def __del__(self):
+        self._released = True
+        if getattr(self, "h", None) and self._children == 0:
+            self._destroy()
 
 
 def mure_model_load(ctx: Context, model, precision: str = "fp32") -> Model:
@@ -210,11 +254,17 @@ def mure_model_load(ctx: Context, model, precision: str = "fp32") -> Model:
 class Cache:
     def __init__(self, model, handle, n_inputs):
         self.model, self.h, self.n_inputs = model, handle, n_inputs
+        model._children += 1
+
+    def free(self):
+        if getattr(self, "h", None):
+            if not _finalizing():
+                lib().mure_cache_free(self.h)
+            self.h = None
+            self.model._child_gone()
 
     def __del__(self):
-        if getattr(self, "h", None):
-            lib().mure_cache_free(self.h)
-            self.h = None
+        self.free()
 
 
 def _as_input(X, labels):
@@ -336,3 +386,4 @@ def mure_expand_patches(model: Model, table):
     offs = np.zeros(max(n, 1), np.int64)
     model.ctx.check(lib().mure_expand_patches(model.h, _ptr(arr), n, _ptr(pool), plen, _ptr(out), need, _ptr(offs)))
     return out[:need], offs[:n]
+
