@@ -243,6 +243,31 @@ mure_status mure_expand_patches(mure_model *model, const mure_mutant *table, int
                                 const int32_t *neuron_pool, int64_t pool_len, float *out, int64_t out_len,
                                 int64_t *offsets);
 
+/* mure_expand_patches without any device allocation.  The paper has no counterpart:
+ * this entry point exists for callers that cannot allocate device memory, such as an
+ * application whose own allocator has reserved the device's memory and cannot lend
+ * it, or a latency-critical loop that forbids allocator calls because cudaMalloc and
+ * cudaFree can synchronise the device.  It runs the same expansion kernel; the
+ * kernel's scratch (job table, per-layer weight pointers, WS permutation buffers)
+ * lives in one fixed device array of 8 MiB inside the library, which every GPU that
+ * loads the library holds until the process exits.  The call allocates no device
+ * memory.
+ *   out_dev   device buffer of out_len floats receiving the patches (same layout and
+ *             values as mure_expand_patches, i.e. GF noise and WS-permuted weights);
+ *   offsets   host [n_mutants]: offset of each mutant's first slot in out_dev, -1 for
+ *             operators without a patch.
+ * The first call on a device looks up the array's device address with that device
+ * current; make that first call before any stream capture on the device.  Every call
+ * shares the one array: calls whose device work overlaps (on different streams or
+ * host threads) race and must not be issued.  The kernel initialises every scratch
+ * entry it reads, so nothing carries over from an earlier call.  The call returns when
+ * the patches are in out_dev.  Errors: INVALID_ARG (descriptors as in
+ * mure_eval_mutants; out_len too small; descriptors needing more than the 8 MiB of
+ * scratch, with the needed size in mure_last_error), CUDA. */
+mure_status mure_expand_patches_noalloc(mure_model *model, const mure_mutant *table, int64_t n_mutants,
+                                        const int32_t *neuron_pool, int64_t pool_len, float *out_dev,
+                                        int64_t out_len, int64_t *offsets);
+
 #ifdef __cplusplus
 }
 #endif

@@ -25,7 +25,7 @@ PRECISIONS = {"fp32": 0, "tf32x3": 1, "bf16": 2}
 # the exported entry points of include/mure.h
 EXPORTS = ("mure_create", "mure_destroy", "mure_last_error", "mure_model_load", "mure_model_free",
            "mure_model_n_layers", "mure_kernel_launches", "mure_build_prefix_cache", "mure_cache_free", "mure_cache_outputs",
-           "mure_eval_mutants", "mure_eval_vanilla", "mure_expand_patches")
+           "mure_eval_mutants", "mure_eval_vanilla", "mure_expand_patches", "mure_expand_patches_noalloc")
 
 
 class MureError(RuntimeError):
@@ -117,6 +117,7 @@ def lib():
         L.mure_eval_vanilla.argtypes = [vp, vp, i64, vp, C.c_int, vp, i64, vp, i64, C.POINTER(_Opts), vp,
                                         C.POINTER(C.c_double), C.POINTER(C.c_double), C.POINTER(_Stats)]
         L.mure_expand_patches.argtypes = [vp, vp, i64, vp, i64, vp, i64, vp]
+        L.mure_expand_patches_noalloc.argtypes = [vp, vp, i64, vp, i64, vp, i64, vp]
         for name in EXPORTS:
             if name not in ("mure_destroy", "mure_model_free", "mure_cache_free", "mure_last_error",
                             "mure_model_n_layers", "mure_kernel_launches"):
@@ -387,3 +388,13 @@ def mure_expand_patches(model: Model, table):
     model.ctx.check(lib().mure_expand_patches(model.h, _ptr(arr), n, _ptr(pool), plen, _ptr(out), need, _ptr(offs)))
     return out[:need], offs[:n]
 
+
+def mure_expand_patches_noalloc(model: Model, table, out_dev):
+    """mure_expand_patches into a caller-provided CUDA float32 tensor, with no device
+    allocation by the library; returns the offsets (host)."""
+    arr, pool, plen = table_array(table)
+    n = len(table)
+    offs = np.zeros(max(n, 1), np.int64)
+    model.ctx.check(lib().mure_expand_patches_noalloc(model.h, _ptr(arr), n, _ptr(pool), plen, _ptr(out_dev),
+                                                      int(out_dev.numel()), _ptr(offs)))
+    return offs[:n]
