@@ -297,6 +297,15 @@ def main():
     top = max(cls_ms, key=cls_ms.get)
     roof = None
     pk, pk_kind = peaks()
+    if top == "delta":
+        # HBM-bound: algorithmic bytes = the rows it builds (written once, cached rows
+        # read once) per its device time
+        byts = sum(r["stats"]["bytes_gather"] for r in results)
+        achieved = byts / (cls_ms[top] / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / pk["hbm_gbs"], "traffic": None, "kernel": "k_patch_rows (delta)",
+                "ms_total": cls_ms[top], "peak_source": f"{pk_kind} (MEASURED_PEAKS.json hbm_gbs)"}
+    pk, pk_kind = peaks()
     if top.startswith("layer"):
         v = int(top[5:])
         fl = sum(r["stats"]["flops_layer"][v] for r in results)

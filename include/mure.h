@@ -149,14 +149,15 @@ typedef struct {
     int64_t n_batches;      /* (group, mutant chunk, input tile) batches */
     int64_t kernel_launches;/* library kernels launched by the call */
     int64_t flops;          /* analytic FLOPs of the layer kernels that ran */
-    /* with kernel_timing: device time and analytic FLOPs / bytes of the kernels of
-       each weighted layer (index = layer, up to MURE_MAX_TIMED_LAYERS), of the delta
-       kernel, of the row-gather copies and of the stand-alone kill epilogue */
+    /* with kernel_timing: device time and analytic FLOPs of the kernels of each
+       weighted layer (index = layer, up to MURE_MAX_TIMED_LAYERS), of the delta
+       kernel (which also copies the cached rows a group starts from), and of the
+       stand-alone kill epilogue; ms_gather is kept for layout and stays 0 */
     double ms_layer[64];
     int64_t flops_layer[64];
     int64_t launches_layer[64];
     double ms_delta, ms_gather, ms_epilogue;
-    int64_t bytes_gather;   /* bytes read + written by the row-gather copies */
+    int64_t bytes_gather;   /* row bytes the delta kernel copies (read + write) */
     int64_t launches_delta;
 } mure_eval_stats;
 

@@ -3,6 +3,7 @@
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <numeric>
 
@@ -481,6 +482,7 @@ struct EvalCfg {
 // global-average-pooling map.
 struct Workspace {
     std::vector<float *> xb;   // [L+1]
+    float *patch = nullptr;    // [rows][kmax * cells] mutated-channel values
     float *zb = nullptr;
     int64_t z_stride = 0;
     float *gap_tmp = nullptr;
@@ -500,6 +502,8 @@ int64_t row_bytes(const mure_model *m, int l, bool vanilla)
     int64_t b = 0;
     for (int s = vanilla ? 1 : l + 1; s <= m->L; ++s) b += m->xd[s].stride;
     if (vanilla) b += m->zd[l].stride;
+    const Stage &S = m->st[l];
+    b += (int64_t)S.oc * (S.gap ? 1 : (S.pool ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow));  // patch values (bound)
     int64_t g = 0;
     for (int v = vanilla ? 0 : l + 1; v < m->L; ++v)
         if (m->st[v].gap) g = std::max(g, gap_map_stride(m->st[v]));
@@ -507,9 +511,10 @@ int64_t row_bytes(const mure_model *m, int l, bool vanilla)
 }
 
 void alloc_workspace(mure_ctx *c, Scratch &sc, const mure_model *m, int64_t rows, bool vanilla, int lmin,
-                     Workspace &ws)
+                     int64_t patch_floats, Workspace &ws)
 {
     ws.rows = rows;
+    ws.patch = sc.get<float>(rows * std::max<int64_t>(patch_floats, 1));
     ws.xb.assign(m->L + 1, nullptr);
     for (int s = vanilla ? 1 : lmin + 1; s <= m->L; ++s) ws.xb[s] = sc.get<float>(rows * m->xd[s].stride);
     if (vanilla) {
@@ -536,7 +541,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
 {
     cudaStream_t s = c->stream;
     const int L = m->L;
-    const int C_DELTA = L, C_GATHER = L + 1, C_EPI = L + 2;
+    const int C_DELTA = L, C_EPI = L + 2;
     int launches = 0;
     auto timed = [&](int cls, int64_t fl, auto &&launch) {
         tm.begin(cls);
@@ -593,30 +598,60 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
             f2.x_stride = m->xd[L].stride;
             timed(l, 2 * Sl.macs * rm.R, [&] { return launch_final_dense(Sl, xsrc(l), rm, f2, s); });
         }
-        timed(C_DELTA, delta_flops, [&] {
-            return launch_delta(Sl, Src{ws.zb, ws.z_stride, 0}, xsrc(l), skip_of(Sl), rm, pa, dt.kmax_layer[l],
-                                ws.xb[l + 1], m->xd[l + 1].stride, s);
-        });
-    } else {
-        // memo rows start as the cached output of layer l, then the mutated channels
-        acct.bytes_gather += 2 * (int64_t)rm.R * m->xd[l + 1].stride * 4;
-        timed(C_GATHER, 0, [&] {
-            return launch_gather_rows(Src{ca->x[l + 1], m->xd[l + 1].stride, 1}, m->xd[l + 1].stride, rm,
-                                      ws.xb[l + 1], m->xd[l + 1].stride, s);
-        });
-        timed(C_DELTA, delta_flops, [&] {
-            return launch_delta(Sl, Src{ca->z[l], m->zd[l].stride, 1}, xsrc(l), skip_of(Sl), rm, pa,
-                                dt.kmax_layer[l], ws.xb[l + 1], m->xd[l + 1].stride, s);
-        });
     }
-    // the suffix l+1 .. L-1 (Algorithm 4) and the fused kill epilogue
-    for (int v = l + 1; v < L - 1; ++v) stage(v, nullptr, 0);
-    if (l < L - 1) {
+    // the delta: values of the mutated channels of x_{l+1} (from the cached z_l in
+    // memoized mode, from the row's own z_l in vanilla mode)
+    const int cells_l = Sl.gap ? 1 : (Sl.pool ? (Sl.oh / 2) * (Sl.ow / 2) : Sl.oh * Sl.ow);
+    const int kmax = dt.kmax_layer[l];
+    const int64_t pstride = (int64_t)std::max(kmax, 1) * cells_l;
+    const Src zsrc = vanilla ? Src{ws.zb, ws.z_stride, 0} : Src{ca->z[l], m->zd[l].stride, 1};
+    acct.bytes_gather += (int64_t)rm.R * kmax * cells_l * 4;
+    const bool dot_kernel = patch_dot_supported(Sl, kmax);
+    timed(C_DELTA, delta_flops, [&] {
+        int n = launch_patch_vals(Sl, zsrc, xsrc(l), skip_of(Sl), rm, pa, kmax, ws.patch, pstride, s, dot_kernel);
+        if (dot_kernel && dt.dot_prefix[g0 + G] > dt.dot_prefix[g0])
+            n += launch_patch_dot(Sl, zsrc, xsrc(l), rm, pa, kmax, ws.patch, pstride, s);
+        return n;
+    });
+    Overlay ov;
+    ov.patch = ws.patch;
+    ov.row_stride = pstride;
+    ov.kmax = kmax;
+    ov.cells = cells_l;
+    ov.ch = Sl.oc;
+    ov.n_neurons = pa.n_neurons;
+    ov.neuron_off = pa.neuron_off;
+    ov.ids = pa.ids;
+    // the unmutated rows of x_{l+1}: cached (memoized) or just computed (vanilla)
+    const Src base = vanilla ? Src{ws.xb[l + 1], m->xd[l + 1].stride, 0} : Src{ca->x[l + 1], m->xd[l + 1].stride, 1};
+    if (l == L - 1) {
+        // mutants of the output layer: the epilogue reads the logits with the overlay
+        timed(C_EPI, 0, [&] { return launch_epilogue(base, m->n_classes, rm, fa, s, &ov); });
+        return launches;
+    }
+    if (l + 1 == L - 1) {
         const Stage &SL = m->st[L - 1];
-        timed(L - 1, 2 * SL.macs * rm.R, [&] { return launch_final_dense(SL, xsrc(L - 1), rm, fa, s); });
-    } else {
-        timed(C_EPI, 0, [&] { return launch_epilogue(Src{ws.xb[L], m->xd[L].stride, 0}, m->n_classes, rm, fa, s); });
+        timed(L - 1, 2 * SL.macs * rm.R, [&] { return launch_final_dense(SL, base, rm, fa, s, &ov); });
+        return launches;
     }
+    // first suffix stage: the overlay is applied while its input tile is staged, or
+    // the rows are materialised for kernels that read plain rows
+    const Stage &Sn = m->st[l + 1];
+    if (Sn.variant > 0) {
+        timed(l + 1, 2 * Sn.macs * rm.R, [&] {
+            return launch_conv_small(Sn, base, rm, nullptr, 0, ws.xb[l + 2], m->xd[l + 2].stride, s, &ov);
+        });
+    } else {
+        acct.bytes_gather += 2 * (int64_t)rm.R * m->xd[l + 1].size * 4;
+        timed(C_DELTA, 0, [&] {
+            return launch_rows_overlay(base, m->xd[l + 1].size, rm, ov, ws.xb[l + 1], m->xd[l + 1].stride, s);
+        });
+        stage(l + 1, nullptr, 0);
+    }
+    // the rest of the suffix (Algorithm 4) and the fused kill epilogue
+    for (int v = l + 2; v < L - 1; ++v) stage(v, nullptr, 0);
+    const Stage &SL = m->st[L - 1];
+    timed(L - 1, 2 * SL.macs * rm.R, [&] { return launch_final_dense(SL, xsrc(L - 1), rm, fa, s); });
     return launches;
 }
 
@@ -669,8 +704,15 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         int64_t gbig = 0;
         for (int l = 0; l < m->L; ++l) gbig = std::max(gbig, g.begin[l + 1] - g.begin[l]);
         rows = std::min(Gmax, gbig) * T;
+        int64_t patch_floats = 1;
+        for (int l = 0; l < m->L; ++l) {
+            if (g.begin[l + 1] == g.begin[l]) continue;
+            const Stage &S = m->st[l];
+            const int64_t cl = S.gap ? 1 : (S.pool ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow);
+            patch_floats = std::max<int64_t>(patch_floats, (int64_t)std::max(dt.kmax_layer[l], 1) * cl);
+        }
         Workspace ws;
-        alloc_workspace(c, sc, m, rows, vanilla, lmin, ws);
+        alloc_workspace(c, sc, m, rows, vanilla, lmin, patch_floats, ws);
         int64_t launches = 0;
         Acct acct;
         acct.flops_cls.assign(m->L + 3, 0);
@@ -900,6 +942,11 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             }
         } cl{m};
         compile(c, d, m);
+        // kernel selection per layer (fixed for the model's lifetime, so every
+        // computation of a layer uses one kernel); MURE_FORCE_GENERIC=1 keeps the
+        // implicit-GEMM kernel everywhere (the kernels agree bit for bit)
+        const char *force = getenv("MURE_FORCE_GENERIC");
+        for (Stage &S : m->st) S.variant = (force && force[0] == '1') ? 0 : conv_small_variant(S);
         std::vector<int> wn;
         for (int v = 0; v < d->n_nodes; ++v)
             if (weighted(d->nodes[v].kind)) wn.push_back(v);

@@ -31,6 +31,7 @@ struct Stage {
     int pool, gap;
     int yh, yw, yc;           // output x_{v+1}
     int64_t macs;             // multiply-accumulates per row
+    int variant = 0;          // 0: implicit-GEMM kernel; > 0: a shared-memory direct conv
     float *W = nullptr;       // device [oc][K]
     float *Wt = nullptr;      // device [K][oc] (the same weights, K-major rows)
     float *b = nullptr;       // device [oc]
@@ -99,9 +100,28 @@ struct RowMap {
     int R;        // rows = mutants in the batch x T
 };
 
+// The mutated channels of a batch's rows of x_{l+1}, applied on top of the unmutated
+// row by the first suffix kernel: for batch mutant g = r / T and slot q < n_neurons[g],
+// channel ids[neuron_off[g] + q] of cell c is patch[r * row_stride + q * cells + c];
+// the row's element for (cell c, channel j) is at c * ch + j.
+struct Overlay {
+    const float *patch = nullptr;   // null: no overlay
+    int64_t row_stride = 0;
+    int kmax = 0, cells = 0, ch = 0;
+    const int32_t *n_neurons = nullptr;
+    const int64_t *neuron_off = nullptr;
+    const int32_t *ids = nullptr;
+};
+
 // Stage v over R rows: z (optional) and y = post(act1(conv(x) + b)).
 int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip,
                       float *y_out, int64_t y_stride, float *gap_tmp, cudaStream_t s);
+
+// The shared-memory direct convolution for small inputs (variant of a stage, 0 when
+// the geometry is not one it compiles) and its launcher.
+int conv_small_variant(const Stage &S);
+int launch_conv_small(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, float *y_out,
+                      int64_t y_stride, cudaStream_t s, const Overlay *ov = nullptr);
 
 // Final dense layer (F -> C, C <= 32) over R rows, with the fused epilogue.
 struct FinalArgs {
@@ -121,13 +141,12 @@ struct FinalArgs {
     unsigned long long *near_ties;
     int mode;                   // 0 = kill, 1 = cache build, 2 = write per-row logits only
 };
-int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s);
+int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s,
+                       const Overlay *ov = nullptr);
 
-// Kill epilogue on per-row logits (mutants of the output layer).
-int launch_epilogue(Src logits, int C, RowMap rm, const FinalArgs &fa, cudaStream_t s);
+// Kill epilogue on logits rows (mutants of the output layer), with an optional overlay.
+int launch_epilogue(Src logits, int C, RowMap rm, const FinalArgs &fa, cudaStream_t s, const Overlay *ov = nullptr);
 
-// Copy per-input rows of a cached tensor into per-row batch rows.
-int launch_gather_rows(Src src, int64_t n_elems, RowMap rm, float *dst, int64_t dst_stride, cudaStream_t s);
 
 // Per-mutant patch data of a batch, in device memory.
 struct PatchArgs {
@@ -139,10 +158,21 @@ struct PatchArgs {
     const float *patch;         // GF: sigma * n, WS: W[j][perm f] - W[j][f]; F per slot
 };
 
-// Rewrite the mutated neurons' channels of x_{l+1} rows (y) from z_l (and x_l for
-// GF/WS), the layer's post-ops and skip.
-int launch_delta(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *y,
-                 int64_t y_stride, cudaStream_t s);
+// Delta of layer l: values of the mutated neurons' channels of x_{l+1}, from z_l
+// (channel-major; x_l for GF / WS), the layer's post-ops and skip, into
+// out[r][q][c] (slot q < kmax, output cell c of layer l).
+int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *out,
+                      int64_t out_stride, cudaStream_t s, bool skip_dot_ops = false);
+
+// GF / WS delta values of the small-layer geometries (stage variant > 0): the same
+// values as launch_patch_vals for those operators; launch_patch_vals then skips them.
+int patch_dot_supported(const Stage &S, int kmax);
+int launch_patch_dot(const Stage &S, Src z, Src x, RowMap rm, const PatchArgs &pa, int kmax, float *out,
+                     int64_t out_stride, cudaStream_t s);
+
+// Materialise rows: out = base rows with the overlay applied.
+int launch_rows_overlay(Src base, int64_t n_floats, RowMap rm, const Overlay &ov, float *out, int64_t out_stride,
+                        cudaStream_t s);
 
 // Expand GF / WS descriptors into patches (see mure_expand_patches): one job per
 // (mutant, neuron slot).

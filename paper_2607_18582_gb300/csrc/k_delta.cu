@@ -1,6 +1,8 @@
 // Mutant-side kernels: descriptor expansion (GF noise, WS shuffles), the delta
 // kernel that rewrites only the mutated neurons' channels of a layer on top of its
 // original output, and the score reduction.
+#include <algorithm>
+
 #include "common.cuh"
 #include "device_util.cuh"
 
@@ -105,43 +107,52 @@ int launch_layer_std(const float *const *W, const int64_t *n, int L, double *out
 }
 
 // ---------------------------------------------------------------------- delta --
+//
+// The delta of a group at layer l: the values of the mutated neurons' channels of
+// x_{l+1} (after layer l's activation, skip add, pooling and GAP), computed from the
+// original pre-activation z_l and, for GF / WS, the layer's input x_l.  They go to a
+// compact per-row patch buffer patch[r][q][c] (slot q < kmax, output cell c of layer
+// l); the first kernel of the suffix applies it on top of the unmutated row.
 
-struct DeltaParams {
+struct PatchValsParams {
     int ih, iw, ic, kh, kw, stride, pad, oh, ow, oc, K;
     int act1, has_add, act2, pool, gap;
     int sk_w, sk_c, sk_stride;
-    const float *z; int64_t z_stride; int z_per_input;
+    int cells;           // output cells of layer l (pooled positions; 1 with GAP)
+    int mcells, mcw;     // cells of the post-op map (pooled or not) and its width
+    const float *z; int64_t z_stride; int z_per_input;   // channel-major [oc][oh*ow]
     const float *x; int64_t x_stride; int x_per_input;
     const float *skip; int64_t skip_stride; int skip_per_input;
-    int64_t t0; int T; int R;
+    int64_t t0; int T; int G;
     PatchArgs pa;
     int kmax;
-    float *y; int64_t y_stride;
-    int lane_mode;
+    float *out; int64_t out_stride;
+    int warp_dot;        // 1: fan-in sums split across a warp (layers with < 32 positions)
+    int skip_dot_ops;    // 1: GF / WS values come from k_patch_dot
 };
 
-struct DeltaRow {
+struct SlotCtx {
     const float *z, *x, *s, *e;
-    int op, j, src_j;
+    int op, j, sj;
 };
 
-// Mutated output of neuron j at conv position (oy, ox) after act1, skip and act2.
-// `dot` is the GF/WS correction sum_k e_k x_k of that position.
-__device__ __forceinline__ float delta_post(const DeltaParams &p, const DeltaRow &d, int oy, int ox, float dot)
+// Mutated output of neuron j at conv position (oy, ox) after act1, skip and act2;
+// `dot` is the GF / WS correction sum_k e_k x_k at that position.
+__device__ __forceinline__ float slot_post(const PatchValsParams &p, const SlotCtx &d, int oy, int ox, float dot)
 {
-    float zz = d.z[((int64_t)oy * p.ow + ox) * p.oc + d.src_j];
+    float zz = d.z[(int64_t)d.sj * (p.oh * p.ow) + oy * p.ow + ox];
     if (d.op == MURE_OP_NAI) zz = -zz;
     else if (d.op == MURE_OP_GF || d.op == MURE_OP_WS) zz = zz + dot;
     float v = d.op == MURE_OP_NEB ? 0.f : act_apply(p.act1, zz);
     if (p.has_add) {
-        const float s = d.j < p.sk_c ? d.s[((int64_t)oy * p.sk_stride * p.sk_w + ox * p.sk_stride) * p.sk_c + d.j] : 0.f;
-        v = act_apply(p.act2, v + s);
+        const float sv = d.j < p.sk_c ? d.s[((int64_t)oy * p.sk_stride * p.sk_w + ox * p.sk_stride) * p.sk_c + d.j] : 0.f;
+        v = act_apply(p.act2, v + sv);
     }
     return v;
 }
 
-// sum_k e_k x_k over the receptive field of (oy, ox): one lane, ascending k.
-__device__ __forceinline__ float dot_serial(const DeltaParams &p, const DeltaRow &d, int oy, int ox)
+// sum_k e_k x_k over the receptive field of (oy, ox): one thread, ascending k.
+__device__ __forceinline__ float dot_serial(const PatchValsParams &p, const SlotCtx &d, int oy, int ox)
 {
     float acc = 0.f;
     const int iy0 = oy * p.stride - p.pad, ix0 = ox * p.stride - p.pad;
@@ -159,113 +170,222 @@ __device__ __forceinline__ float dot_serial(const DeltaParams &p, const DeltaRow
     return acc;
 }
 
-// The same sum with the warp: lane i takes k = i, i+32, ... in ascending order, then
-// a butterfly over lanes; every lane ends with the same value.
-__device__ __forceinline__ float dot_warp(const DeltaParams &p, const DeltaRow &d, int oy, int ox, int lane)
+// The same sum with a warp: lane i takes k = i, i+32, ... in ascending order, then a
+// butterfly over the lanes; every lane ends with the same value.
+__device__ __forceinline__ float dot_warp(const PatchValsParams &p, const SlotCtx &d, int oy, int ox, int lane)
 {
     float acc = 0.f;
     const int iy0 = oy * p.stride - p.pad, ix0 = ox * p.stride - p.pad;
-    for (int k = lane; k < p.K; k += 32) {
-        const int ci = k % p.ic, t = k / p.ic, kx = t % p.kw, ky = t / p.kw;
-        const int iy = iy0 + ky, ix = ix0 + kx;
-        if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw)
-            acc = fmaf(__ldg(d.e + k), __ldg(d.x + ((int64_t)iy * p.iw + ix) * p.ic + ci), acc);
+    if (p.kh == 1 && p.kw == 1 && p.ih == 1 && p.iw == 1) {
+        for (int k = lane; k < p.K; k += 32) acc = fmaf(__ldg(d.e + k), __ldg(d.x + k), acc);
+    } else {
+        for (int k = lane; k < p.K; k += 32) {
+            const int ci = k % p.ic, t = k / p.ic, kx = t % p.kw, ky = t / p.kw;
+            const int iy = iy0 + ky, ix = ix0 + kx;
+            if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw)
+                acc = fmaf(__ldg(d.e + k), __ldg(d.x + ((int64_t)iy * p.iw + ix) * p.ic + ci), acc);
+        }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
     return acc;
 }
 
-__global__ void __launch_bounds__(128) k_delta(const DeltaParams p)
+// Value of map cell c (a pooled window or one position) of slot d.  In warp-dot
+// mode every lane of the warp must call it with the same c.
+__device__ __forceinline__ float cell_value(const PatchValsParams &p, const SlotCtx &d, int c, int lane)
 {
-    extern __shared__ float gap_buf[];  // [4 warps][cells] when the layer ends in GAP
-    const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
-    const int64_t wid = (int64_t)blockIdx.x * 4 + wib;
-    const int64_t r = wid / p.kmax;
-    const int q = (int)(wid % p.kmax);
-    if (r >= p.R) return;
-    const int g = (int)(r / p.T);
-    const int64_t t = p.t0 + r % p.T;
-    DeltaRow d;
-    d.op = p.pa.op[g];
-    if (q >= p.pa.n_neurons[g]) return;
-    const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
-    d.j = ids[q];
-    d.src_j = d.op == MURE_OP_NS ? ids[q ^ 1] : d.j;
-    d.z = p.z + (p.z_per_input ? t : r) * p.z_stride;
-    const bool needs_dot = d.op == MURE_OP_GF || d.op == MURE_OP_WS;
-    d.x = needs_dot ? p.x + (p.x_per_input ? t : r) * p.x_stride : nullptr;
-    d.e = needs_dot ? p.pa.patch + p.pa.patch_off[g] + (int64_t)q * p.K : nullptr;
-    d.s = p.has_add ? p.skip + (p.skip_per_input ? t : r) * p.skip_stride : nullptr;
-    float *yrow = p.y + r * p.y_stride;
-
-    const int cw = p.pool ? p.ow / 2 : p.ow;
-    const int cells = (p.pool ? p.oh / 2 : p.oh) * cw;
-    float gsum = 0.f;
-    float *gb = gap_buf + wib * cells;
-    for (int c0 = 0; c0 < cells; c0 += (p.lane_mode ? 32 : 1)) {
-        const int c = p.lane_mode ? c0 + lane : c0;
-        const bool active = c < cells;
-        float v = 0.f;
-        const int cy = active ? c / cw : 0, cx = active ? c % cw : 0;
-        if (p.pool) {
-            float w4[4];
-            for (int sub = 0; sub < 4; ++sub) {
-                const int oy = 2 * cy + (sub >> 1), ox = 2 * cx + (sub & 1);
-                float dot = 0.f;
-                if (needs_dot) dot = p.lane_mode ? (active ? dot_serial(p, d, oy, ox) : 0.f) : dot_warp(p, d, oy, ox, lane);
-                w4[sub] = active ? delta_post(p, d, oy, ox, dot) : 0.f;
-            }
-            v = max4_first(w4[0], w4[1], w4[2], w4[3]);
-        } else {
-            float dot = 0.f;
-            if (needs_dot) dot = p.lane_mode ? (active ? dot_serial(p, d, cy, cx) : 0.f) : dot_warp(p, d, cy, cx, lane);
-            v = active ? delta_post(p, d, cy, cx, dot) : 0.f;
-        }
-        if (p.gap) {
-            if (p.lane_mode) { if (active) gb[c] = v; }
-            else gsum += v;  // cells in ascending order
-        } else if (active && (p.lane_mode || lane == 0)) {
-            yrow[(int64_t)c * p.oc + d.j] = v;
-        }
+    const bool dot = d.op == MURE_OP_GF || d.op == MURE_OP_WS;
+    const int cy = c / p.mcw, cx = c % p.mcw;
+    if (!p.pool) {
+        const float dv = dot ? (p.warp_dot ? dot_warp(p, d, cy, cx, lane) : dot_serial(p, d, cy, cx)) : 0.f;
+        return slot_post(p, d, cy, cx, dv);
     }
-    if (p.gap) {
-        if (p.lane_mode) {
-            __syncwarp();
-            if (lane == 0) {
-                float s = 0.f;
-                for (int c = 0; c < cells; ++c) s += gb[c];
-                yrow[d.j] = s / (float)cells;
+    float w4[4];
+#pragma unroll
+    for (int sub = 0; sub < 4; ++sub) {
+        const int oy = 2 * cy + (sub >> 1), ox = 2 * cx + (sub & 1);
+        const float dv = dot ? (p.warp_dot ? dot_warp(p, d, oy, ox, lane) : dot_serial(p, d, oy, ox)) : 0.f;
+        w4[sub] = slot_post(p, d, oy, ox, dv);
+    }
+    return max4_first(w4[0], w4[1], w4[2], w4[3]);
+}
+
+// Items are (mutant g, slot q, cell c) of one input (blockIdx.y), so the mutants of
+// an input read its z and x while they are in L2.  `per_warp`: one item per warp.
+template <bool PER_WARP>
+__global__ void __launch_bounds__(256) k_patch_vals(const PatchValsParams p)
+{
+    extern __shared__ float gap_buf[];  // [8][mcells] with GAP in lane mode
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int per_g = p.kmax * p.cells;
+    const int n_items = p.G * per_g;
+    for (int tl = blockIdx.y; tl < p.T; tl += gridDim.y) {
+        const int item = PER_WARP ? (int)blockIdx.x * 8 + warp : (int)blockIdx.x * 256 + threadIdx.x;
+        if (item >= n_items) continue;   // warp-uniform when PER_WARP
+        const int g = item / per_g, rem = item - g * per_g, q = rem / p.cells, c = rem - q * p.cells;
+        const int k = p.pa.n_neurons[g];
+        if (q >= k) continue;
+        const int op = p.pa.op[g];
+        const bool dot = op == MURE_OP_GF || op == MURE_OP_WS;
+        if (dot && p.skip_dot_ops) continue;
+        const int64_t r = (int64_t)g * p.T + tl, t = p.t0 + tl;
+        const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
+        SlotCtx d;
+        d.op = op;
+        d.j = ids[q];
+        d.sj = op == MURE_OP_NS ? ids[q ^ 1] : d.j;
+        d.z = p.z + (p.z_per_input ? t : r) * p.z_stride;
+        d.x = dot ? p.x + (p.x_per_input ? t : r) * p.x_stride : nullptr;
+        d.s = p.has_add ? p.skip + (p.skip_per_input ? t : r) * p.skip_stride : nullptr;
+        d.e = dot ? p.pa.patch + p.pa.patch_off[g] + (int64_t)q * p.K : nullptr;
+        float *o = p.out + r * p.out_stride + q * p.cells + c;
+        if (p.gap) {
+            // the map cells, then their ascending fp32 sum / count (one warp)
+            float s = 0.f;
+            if (p.warp_dot) {
+                for (int cc = 0; cc < p.mcells; ++cc) s += cell_value(p, d, cc, lane);
+            } else {
+                float *gb = gap_buf + warp * p.mcells;
+                for (int cc = lane; cc < p.mcells; cc += 32) gb[cc] = cell_value(p, d, cc, lane);
+                __syncwarp();
+                for (int cc = 0; cc < p.mcells; ++cc) s += gb[cc];
+                __syncwarp();
             }
-        } else if (lane == 0) {
-            yrow[d.j] = gsum / (float)cells;
+            if (lane == 0) *o = s / (float)p.mcells;
+        } else {
+            const float v = cell_value(p, d, c, lane);
+            if (!PER_WARP || lane == 0) *o = v;
         }
     }
 }
 
-int launch_delta(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *y,
-                 int64_t y_stride, cudaStream_t s)
+int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *out,
+                      int64_t out_stride, cudaStream_t s, bool skip_dot_ops)
 {
     if (rm.R <= 0 || kmax <= 0) return 0;
-    DeltaParams p{};
+    PatchValsParams p{};
     p.ih = S.ih; p.iw = S.iw; p.ic = S.ic; p.kh = S.kh; p.kw = S.kw; p.stride = S.stride; p.pad = S.pad;
     p.oh = S.oh; p.ow = S.ow; p.oc = S.oc; p.K = S.K;
     p.act1 = S.act1; p.has_add = S.has_add; p.act2 = S.act2; p.pool = S.pool; p.gap = S.gap;
     p.sk_w = S.sk_w; p.sk_c = S.sc_c; p.sk_stride = S.sc_stride;
+    p.mcw = S.pool ? S.ow / 2 : S.ow;
+    p.mcells = (S.pool ? S.oh / 2 : S.oh) * p.mcw;
+    p.cells = S.gap ? 1 : p.mcells;
     p.z = z.p; p.z_stride = z.stride; p.z_per_input = z.per_input;
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
     p.skip = skip.p; p.skip_stride = skip.stride; p.skip_per_input = skip.per_input;
-    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
+    p.t0 = rm.t0; p.T = rm.T; p.G = rm.R / rm.T;
     p.pa = pa;
     p.kmax = kmax;
-    p.y = y; p.y_stride = y_stride;
-    const int cells = (S.pool ? S.oh / 2 : S.oh) * (S.pool ? S.ow / 2 : S.ow);
-    // one lane per output position when there are at least 32 of them; otherwise
-    // the warp splits each position's fan-in (dense layers)
-    p.lane_mode = (S.oh * S.ow) >= 32;
-    const size_t smem = S.gap ? (size_t)4 * cells * sizeof(float) : 0;
-    const int64_t warps = (int64_t)rm.R * kmax;
-    k_delta<<<(unsigned)((warps + 3) / 4), 128, smem, s>>>(p);
+    p.out = out; p.out_stride = out_stride;
+    p.warp_dot = (S.oh * S.ow) < 32;
+    p.skip_dot_ops = skip_dot_ops;
+    const bool per_warp = p.gap || p.warp_dot;
+    const int64_t n_items = (int64_t)p.G * kmax * p.cells;
+    const unsigned gx = (unsigned)((n_items + (per_warp ? 7 : 255)) / (per_warp ? 8 : 256));
+    const dim3 grid(gx, (unsigned)std::min(rm.T, 65535));
+    const size_t smem = (S.gap && !p.warp_dot) ? 8 * (size_t)p.mcells * sizeof(float) : 0;
+    if (per_warp) k_patch_vals<true><<<grid, 256, smem, s>>>(p);
+    else k_patch_vals<false><<<grid, 256, smem, s>>>(p);
+    return 1;
+}
+
+// Materialise rows: out = base with the overlay's channels written in (for suffix
+// kernels that read plain rows).  out may alias a per-row base.
+__global__ void __launch_bounds__(256) k_rows_overlay(const float *__restrict__ base, int64_t base_stride,
+                                                      int base_per_input, int64_t t0, int T, int R, int64_t n_floats,
+                                                      const Overlay ov, float *out, int64_t out_stride,
+                                                      int rows_per_block)
+{
+    extern __shared__ float sm[];  // [rows_per_block][n_floats]
+    __shared__ const float *src[64];
+    __shared__ float *dst[64];
+    __shared__ int gidx[64];
+    const int64_t r0 = (int64_t)blockIdx.x * rows_per_block;
+    const int nr = (int)(R - r0 < rows_per_block ? R - r0 : rows_per_block);
+    if (threadIdx.x < nr) {
+        const int64_t r = r0 + threadIdx.x;
+        src[threadIdx.x] = base + (base_per_input ? t0 + r % T : r) * base_stride;
+        dst[threadIdx.x] = out + r * out_stride;
+        gidx[threadIdx.x] = (int)(r / T);
+    }
+    __syncthreads();
+    const int nf = (int)n_floats;
+    for (int i = threadIdx.x; i < nr * nf; i += blockDim.x) {
+        const int rl = i / nf;
+        sm[i] = __ldg(src[rl] + (i - rl * nf));
+    }
+    __syncthreads();
+    const int per_row = ov.kmax * ov.cells;
+    for (int i = threadIdx.x; i < nr * per_row; i += blockDim.x) {
+        const int rl = i / per_row, rem = i - rl * per_row, q = rem / ov.cells, c = rem - q * ov.cells;
+        const int g = gidx[rl];
+        if (q >= ov.n_neurons[g]) continue;
+        const int j = ov.ids[ov.neuron_off[g] + q];
+        sm[rl * nf + c * ov.ch + j] = ov.patch[(r0 + rl) * ov.row_stride + q * ov.cells + c];
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < nr * nf; i += blockDim.x) {
+        const int rl = i / nf;
+        dst[rl][i - rl * nf] = sm[i];
+    }
+}
+
+// Large rows: copy the base rows, then scatter the overlay (two ordered launches).
+__global__ void k_copy_rows(const float4 *__restrict__ src, int64_t src_stride4, int per_input, int64_t n4, int64_t t0,
+                            int T, int64_t R, float4 *__restrict__ dst, int64_t dst_stride4)
+{
+    const int64_t total = R * n4;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = i / n4, e = i - r * n4;
+        dst[r * dst_stride4 + e] = __ldg(src + (per_input ? t0 + r % T : r) * src_stride4 + e);
+    }
+}
+
+__global__ void k_overlay_scatter(int64_t T, int64_t R, const Overlay ov, float *out, int64_t out_stride)
+{
+    const int64_t per_row = (int64_t)ov.kmax * ov.cells;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < R * per_row;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t r = i / per_row;
+        const int rem = (int)(i - r * per_row), q = rem / ov.cells, c = rem - q * ov.cells;
+        const int g = (int)(r / T);
+        if (q >= ov.n_neurons[g]) continue;
+        const int j = ov.ids[ov.neuron_off[g] + q];
+        out[r * out_stride + (int64_t)c * ov.ch + j] = ov.patch[r * ov.row_stride + q * ov.cells + c];
+    }
+}
+
+int launch_rows_overlay(Src base, int64_t n_floats, RowMap rm, const Overlay &ov, float *out, int64_t out_stride,
+                        cudaStream_t s)
+{
+    if (rm.R <= 0) return 0;
+    if (n_floats > 8192) {
+        int launches = 0;
+        if (!(base.p == out && !base.per_input)) {
+            const int64_t n4 = (n_floats + 3) / 4, total = (int64_t)rm.R * n4;
+            const int64_t blocks = std::min<int64_t>((total + 255) / 256, 152 * 64);
+            k_copy_rows<<<(unsigned)blocks, 256, 0, s>>>(reinterpret_cast<const float4 *>(base.p), base.stride / 4,
+                                                         base.per_input, n4, rm.t0, rm.T, rm.R,
+                                                         reinterpret_cast<float4 *>(out), out_stride / 4);
+            ++launches;
+        }
+        const int64_t total = (int64_t)rm.R * ov.kmax * ov.cells;
+        if (total > 0) {
+            const int64_t blocks = std::min<int64_t>((total + 255) / 256, 152 * 64);
+            k_overlay_scatter<<<(unsigned)blocks, 256, 0, s>>>(rm.T, rm.R, ov, out, out_stride);
+            ++launches;
+        }
+        return launches;
+    }
+    const int rows_per_block = (int)std::max<int64_t>(1, std::min<int64_t>(64, 8192 / std::max<int64_t>(n_floats, 1)));
+    const size_t smem = (size_t)rows_per_block * n_floats * sizeof(float);
+    if (smem > 48 * 1024)
+        cudaFuncSetAttribute(k_rows_overlay, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const int64_t blocks = (rm.R + rows_per_block - 1) / rows_per_block;
+    k_rows_overlay<<<(unsigned)blocks, 256, smem, s>>>(base.p, base.stride, base.per_input, rm.t0, rm.T, rm.R,
+                                                      n_floats, ov, out, out_stride, rows_per_block);
     return 1;
 }
 

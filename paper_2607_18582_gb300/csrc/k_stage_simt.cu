@@ -136,7 +136,7 @@ __global__ void __launch_bounds__(256) k_stage_simt(const StageParams p)
                 ox = q % p.ow;
             }
             const float z = acc[i][j] + bias;
-            if (p.z) p.z[row * p.z_stride + ((int64_t)oy * p.ow + ox) * p.oc + n] = z;
+            if (p.z) p.z[row * p.z_stride + (int64_t)n * (p.oh * p.ow) + oy * p.ow + ox] = z;  // channel-major
             float v = act_apply(p.act1, z);
             if (p.has_add) {
                 const float *sr = p.skip + (p.skip_per_input ? (p.t0 + row % p.T) : row) * p.skip_stride;
@@ -166,6 +166,7 @@ int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
                       int64_t y_stride, float *gap_tmp, cudaStream_t s)
 {
     if (rm.R <= 0) return 0;
+    if (S.variant > 0) return launch_conv_small(S, x, rm, z_out, z_stride, y_out, y_stride, s);
     StageParams p{};
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
     p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
@@ -212,6 +213,7 @@ struct FinalParams {
     const float *W;  // [C][F]
     const float *b;
     FinalArgs fa;
+    Overlay ov;      // mutated channels of the input rows (ov.patch null: none)
 };
 
 // Kill bits of one warp of rows (32 consecutive inputs of one mutant) and the
@@ -252,6 +254,14 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
     const int64_t row0 = (int64_t)blockIdx.x * RB;
     const int64_t row = row0 + tid;
     const bool in_range = row < p.R;
+    // this row's mutated input channels (overlay), as (slot count, id pointer)
+    int ov_k = 0;
+    const int32_t *ov_ids = nullptr;
+    if (p.ov.patch && in_range) {
+        const int g = (int)(row / p.T);
+        ov_k = p.ov.n_neurons[g];
+        ov_ids = p.ov.ids + p.ov.neuron_off[g];
+    }
     float acc[kMaxClasses];
 #pragma unroll
     for (int c = 0; c < kMaxClasses; ++c) acc[c] = 0.f;
@@ -270,6 +280,13 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
         }
         __syncthreads();
         const int fe = min(FC, p.F - f0);
+        // overlay on this thread's own row (no other thread reads it)
+        for (int q = 0; q < ov_k; ++q) {
+            const int j = ov_ids[q];
+            const int cfirst = f0 - j <= 0 ? 0 : (f0 - j + p.ov.ch - 1) / p.ov.ch;
+            for (int c = cfirst; c < p.ov.cells && c * p.ov.ch + j < f0 + fe; ++c)
+                xs[tid][c * p.ov.ch + j - f0] = p.ov.patch[row * p.ov.row_stride + q * p.ov.cells + c];
+        }
         for (int fl = 0; fl < fe; ++fl) {
             const float xv = xs[tid][fl];
 #pragma unroll
@@ -303,21 +320,33 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
     epilogue_row(p.fa, p.t0, p.T, row, in_range, v, p.C);
 }
 
-__global__ void __launch_bounds__(128) k_epilogue(const float *__restrict__ lg, int64_t stride, int C, int64_t t0, int T,
-                                                  int R, const FinalArgs fa)
+__global__ void __launch_bounds__(128) k_epilogue(const float *__restrict__ lg, int64_t stride, int per_input, int C,
+                                                  int64_t t0, int T, int R, const FinalArgs fa, const Overlay ov)
 {
     const int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const bool in_range = row < R;
     float v[kMaxClasses];
+    const float *src = lg + (per_input ? t0 + row % T : row) * stride;
 #pragma unroll
-    for (int c = 0; c < kMaxClasses; ++c) v[c] = (in_range && c < C) ? lg[row * stride + c] : 0.f;
+    for (int c = 0; c < kMaxClasses; ++c) v[c] = (in_range && c < C) ? src[c] : 0.f;
+    if (ov.patch && in_range) {
+        const int g = (int)(row / T);
+        const int32_t *ids = ov.ids + ov.neuron_off[g];
+        for (int q = 0; q < ov.n_neurons[g]; ++q) {
+            const float val = ov.patch[row * ov.row_stride + q * ov.cells];
+#pragma unroll
+            for (int c = 0; c < kMaxClasses; ++c)
+                if (c == ids[q]) v[c] = val;
+        }
+    }
     epilogue_row(fa, t0, T, row, in_range, v, C);
 }
 
-int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s)
+int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s, const Overlay *ov)
 {
     if (rm.R <= 0) return 0;
     FinalParams p{};
+    if (ov) p.ov = *ov;
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
     p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
     p.F = S.K; p.C = S.oc; p.act = S.act1;
@@ -327,34 +356,13 @@ int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cu
     return 1;
 }
 
-int launch_epilogue(Src logits, int C, RowMap rm, const FinalArgs &fa, cudaStream_t s)
+int launch_epilogue(Src logits, int C, RowMap rm, const FinalArgs &fa, cudaStream_t s, const Overlay *ov)
 {
     if (rm.R <= 0) return 0;
-    k_epilogue<<<(unsigned)((rm.R + 127) / 128), 128, 0, s>>>(logits.p, logits.stride, C, rm.t0, rm.T, rm.R, fa);
-    return 1;
-}
-
-// ----------------------------------------------------------------- row copies --
-
-__global__ void k_gather_rows(const float4 *__restrict__ src, int64_t src_stride4, int64_t n4, int64_t t0, int T,
-                              int64_t R, float4 *__restrict__ dst, int64_t dst_stride4)
-{
-    const int64_t total = R * n4;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t r = i / n4, e = i % n4;
-        dst[r * dst_stride4 + e] = __ldg(src + (t0 + r % T) * src_stride4 + e);
-    }
-}
-
-int launch_gather_rows(Src src, int64_t n_elems, RowMap rm, float *dst, int64_t dst_stride, cudaStream_t s)
-{
-    if (rm.R <= 0) return 0;
-    const int64_t n4 = (n_elems + 3) / 4;
-    const int64_t total = (int64_t)rm.R * n4;
-    int64_t blocks = (total + 255) / 256;
-    if (blocks > 152 * 32) blocks = 152 * 32;
-    k_gather_rows<<<(unsigned)blocks, 256, 0, s>>>(reinterpret_cast<const float4 *>(src.p), src.stride / 4, n4, rm.t0,
-                                                   rm.T, rm.R, reinterpret_cast<float4 *>(dst), dst_stride / 4);
+    Overlay o;
+    if (ov) o = *ov;
+    k_epilogue<<<(unsigned)((rm.R + 127) / 128), 128, 0, s>>>(logits.p, logits.stride, logits.per_input, C, rm.t0,
+                                                              rm.T, rm.R, fa, o);
     return 1;
 }
 

@@ -259,3 +259,20 @@ def test_full_size_lenet_sampled(M, ctx, oracle_mod):
     ties = margin_tie(ora["logits"]) | margin_tie(ora["orig_logits"])[None, :]
     assert int(((g != o) & ~ties).sum()) == 0
     assert 0.0 <= r["scoreA"] <= 1.0 and 0.0 <= r["scoreB"] <= 1.0
+
+
+def test_kernel_variants_agree_bitwise(M, ctx, monkeypatch):
+    """The shared-memory direct convolution and the implicit-GEMM kernel compute the
+    same fp32 chains: a model forced onto the generic kernel gives identical bits."""
+    w = wl.workload("lenet5", 200, 1)
+    table = all_ops(w.model, 6, seed=41)
+    fast = M.mure_model_load(ctx, w.model)
+    monkeypatch.setenv("MURE_FORCE_GENERIC", "1")
+    generic = M.mure_model_load(ctx, w.model)
+    monkeypatch.delenv("MURE_FORCE_GENERIC")
+    r1 = M.mure_eval_mutants(M.mure_build_prefix_cache(fast, w.X), table, logits=True)
+    r2 = M.mure_eval_mutants(M.mure_build_prefix_cache(generic, w.X), table, logits=True)
+    assert np.array_equal(r1["logits"].view(np.uint32), r2["logits"].view(np.uint32))
+    assert np.array_equal(r1["kill_bits"], r2["kill_bits"])
+    v1 = M.mure_eval_vanilla(fast, w.X, table, logits=True)
+    assert np.array_equal(v1["logits"].view(np.uint32), r1["logits"].view(np.uint32))
