@@ -234,6 +234,8 @@ def main():
     ap.add_argument("--n-inputs", type=int, default=None, help="smaller case (profiling): first n inputs")
     ap.add_argument("--n-mutants", type=int, default=None, help="smaller case (profiling): first n mutants")
     ap.add_argument("--only-layer", type=int, default=None, help="keep only the mutants of this layer")
+    ap.add_argument("--precision", default="tf32x3", choices=["fp32", "tf32x3"],
+                    help="layer arithmetic: fp32 CUDA-core chains, or tensor-core 3xTF32 for dense layers")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world, rank, local = dist_setup()
@@ -250,7 +252,7 @@ def main():
         w.table = w.table.subset(np.nonzero(w.table.layer == args.only_layer)[0])
     n_evals = len(w.table) * len(w.X)
     ctx = mure.mure_create(dev)
-    model = mure.mure_model_load(ctx, w.model)
+    model = mure.mure_model_load(ctx, w.model, precision=args.precision)
     X_dev = torch.from_numpy(w.X).to(f"cuda:{dev}")
     arrays = mure.table_array(w.table)
     W64 = (len(w.X) + 63) // 64

@@ -637,7 +637,11 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     // first suffix stage: the overlay is applied while its input tile is staged, or
     // the rows are materialised for kernels that read plain rows
     const Stage &Sn = m->st[l + 1];
-    if (Sn.variant > 0) {
+    if (Sn.tc) {
+        timed(l + 1, 2 * Sn.macs * rm.R, [&] {
+            return launch_tc_dense(Sn, base, rm, nullptr, 0, ws.xb[l + 2], m->xd[l + 2].stride, s, &ov);
+        });
+    } else if (Sn.variant > 0) {
         timed(l + 1, 2 * Sn.macs * rm.R, [&] {
             return launch_conv_small(Sn, base, rm, nullptr, 0, ws.xb[l + 2], m->xd[l + 2].stride, s, &ov);
         });
@@ -739,6 +743,8 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         CK(c, cudaEventRecord(c->ev[3], s));
         unsigned long long host_cnt[4];
         CK(c, cudaMemcpyAsync(host_cnt, ec.counters, sizeof host_cnt, cudaMemcpyDeviceToHost, s));
+        int dev_err = 0;
+        CK(c, cudaMemcpyAsync(&dev_err, c->err_dev, sizeof(int), cudaMemcpyDeviceToHost, s));
         if (!o->outputs_on_device) {
             CK(c, cudaMemcpyAsync(out.kill_bits, ec.kill32, (size_t)n * words32 * 4, cudaMemcpyDeviceToHost, s));
             if (o->logits_out)
@@ -748,6 +754,10 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         CK(c, cudaEventRecord(c->ev[4], s));
         CK(c, cudaStreamSynchronize(s));
         CK(c, cudaGetLastError());
+        if (dev_err) {
+            CK(c, cudaMemset(c->err_dev, 0, sizeof(int)));
+            FAILIF(true, c, MURE_ERR_TIMEOUT, "a device-side wait gave up (code %d)", dev_err);
+        }
         sA = (double)host_cnt[0] / (double)n;
         sB = ca->n_label_values > 0 ? (double)host_cnt[1] / ((double)n * ca->n_label_values) : 0.0;
         st.n_near_ties = (int64_t)host_cnt[2];
@@ -900,6 +910,8 @@ mure_status mure_create(int device, void *cuda_stream, const mure_allocator *all
         CK(c, cudaSetDevice(device));
         CK(c, cudaDeviceGetAttribute(&c->n_sms, cudaDevAttrMultiProcessorCount, device));
         for (auto &e : c->ev) CK(c, cudaEventCreate(&e));
+        CK(c, cudaMalloc(&c->err_dev, sizeof(int)));
+        CK(c, cudaMemset(c->err_dev, 0, sizeof(int)));
     });
     if (st != MURE_OK) {
         mure_destroy(c);
@@ -915,6 +927,7 @@ void mure_destroy(mure_ctx *ctx)
     for (auto &e : ctx->ev)
         if (e) cudaEventDestroy(e);
     for (auto &e : ctx->evpool) cudaEventDestroy(e);
+    if (ctx->err_dev) cudaFree(ctx->err_dev);
     delete ctx;
 }
 
@@ -927,8 +940,8 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
         FAILIF(!d || !out || !d->nodes || d->n_nodes < 1, c, MURE_ERR_INVALID_ARG, "NULL model description");
         *out = nullptr;
         FAILIF(d->in_h < 1 || d->in_w < 1 || d->in_c < 1, c, MURE_ERR_INVALID_ARG, "bad input shape");
-        FAILIF(d->precision != MURE_PREC_FP32, c, MURE_ERR_UNSUPPORTED, "precision %d is not available",
-               d->precision);
+        FAILIF(d->precision != MURE_PREC_FP32 && d->precision != MURE_PREC_TF32X3, c, MURE_ERR_UNSUPPORTED,
+               "precision %d is not available", d->precision);
         CK(c, cudaSetDevice(c->device));
         auto *m = new mure_model();
         m->ctx = c;
@@ -946,7 +959,13 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
         // computation of a layer uses one kernel); MURE_FORCE_GENERIC=1 keeps the
         // implicit-GEMM kernel everywhere (the kernels agree bit for bit)
         const char *force = getenv("MURE_FORCE_GENERIC");
-        for (Stage &S : m->st) S.variant = (force && force[0] == '1') ? 0 : conv_small_variant(S);
+        for (Stage &S : m->st) {
+            S.variant = (force && force[0] == '1') ? 0 : conv_small_variant(S);
+            S.err = c->err_dev;
+        }
+        // TF32X3: dense layers before the output layer run on the tensor cores
+        if (d->precision == MURE_PREC_TF32X3)
+            for (int l = 0; l + 1 < m->L; ++l) m->st[l].tc = tc_dense_supported(m->st[l]);
         std::vector<int> wn;
         for (int v = 0; v < d->n_nodes; ++v)
             if (weighted(d->nodes[v].kind)) wn.push_back(v);
@@ -965,6 +984,13 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             CK(c, cudaMemcpyAsync(S.Wt, Wt.data(), nw * 4, cudaMemcpyHostToDevice, c->stream));
             CK(c, cudaMemcpyAsync(S.b, n.b, S.oc * 4, cudaMemcpyHostToDevice, c->stream));
             CK(c, cudaStreamSynchronize(c->stream));  // Wt is reused
+            if (S.tc) {
+                const int64_t np = (int64_t)round_up16(S.oc) * round_up32(S.K);
+                S.Wtc_hi = (float *)dalloc(c, np * 4);
+                S.Wtc_lo = (float *)dalloc(c, np * 4);
+                c->launches += launch_split_weights(S, S.Wtc_hi, S.Wtc_lo, c->stream);
+                check_launch(c);
+            }
         }
         // population std of every layer's weights (GF's sigma), fp64 on the device
         {
@@ -996,6 +1022,8 @@ void mure_model_free(mure_model *m)
         dfree(m->ctx, S.W);
         dfree(m->ctx, S.Wt);
         dfree(m->ctx, S.b);
+        dfree(m->ctx, S.Wtc_hi);
+        dfree(m->ctx, S.Wtc_lo);
     }
     dfree(m->ctx, m->sigma_dev);
     cudaStreamSynchronize(m->ctx->stream);

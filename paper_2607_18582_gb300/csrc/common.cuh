@@ -32,6 +32,10 @@ struct Stage {
     int yh, yw, yc;           // output x_{v+1}
     int64_t macs;             // multiply-accumulates per row
     int variant = 0;          // 0: implicit-GEMM kernel; > 0: a shared-memory direct conv
+    int tc = 0;               // 1: tensor-core (tcgen05, 3xTF32) kernel
+    float *Wtc_hi = nullptr;  // tc: TF32 halves of W, zero-padded [round16(oc)][round32(K)]
+    float *Wtc_lo = nullptr;
+    int *err = nullptr;       // device error word of the context (bounded waits)
     float *W = nullptr;       // device [oc][K]
     float *Wt = nullptr;      // device [K][oc] (the same weights, K-major rows)
     float *b = nullptr;       // device [oc]
@@ -43,6 +47,9 @@ struct TensorDim {
     int h, w, c;
     int64_t size, stride;     // elements; stride = size rounded up to a multiple of 4
 };
+
+__host__ __device__ inline int round_up16(int n) { return (n + 15) & ~15; }
+__host__ __device__ inline int round_up32(int n) { return (n + 31) & ~31; }
 
 }  // namespace mure
 
@@ -56,6 +63,7 @@ struct mure_ctx {
     std::vector<cudaEvent_t> evpool;  // per-launch timing events, reused across calls
     int n_sms = 0;
     int64_t launches = 0;             // kernels launched since creation
+    int *err_dev = nullptr;           // device error word written by bounded waits
 };
 
 struct mure_model {
@@ -122,6 +130,13 @@ int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
 int conv_small_variant(const Stage &S);
 int launch_conv_small(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, float *y_out,
                       int64_t y_stride, cudaStream_t s, const Overlay *ov = nullptr);
+
+// Tensor-core dense layer (tcgen05, 3xTF32): which layers it takes, the weight split
+// done at model load, and the launcher (rows as for the stage kernel, plus overlay).
+int tc_dense_supported(const Stage &S);
+int launch_split_weights(const Stage &S, float *hi, float *lo, cudaStream_t s);
+int launch_tc_dense(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, float *y_out, int64_t y_stride,
+                    cudaStream_t s, const Overlay *ov = nullptr);
 
 // Final dense layer (F -> C, C <= 32) over R rows, with the fused epilogue.
 struct FinalArgs {

@@ -166,6 +166,7 @@ int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
                       int64_t y_stride, float *gap_tmp, cudaStream_t s)
 {
     if (rm.R <= 0) return 0;
+    if (S.tc) return launch_tc_dense(S, x, rm, z_out, z_stride, y_out, y_stride, s);
     if (S.variant > 0) return launch_conv_small(S, x, rm, z_out, z_stride, y_out, y_stride, s);
     StageParams p{};
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;

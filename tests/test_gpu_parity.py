@@ -57,10 +57,14 @@ def oracle_runs(oracle_mod):
     return get
 
 
+PRECISIONS = ["fp32", "tf32x3"]
+
+
+@pytest.mark.parametrize("prec", PRECISIONS)
 @pytest.mark.parametrize("name", list(CASES))
-def test_cache_build_matches_oracle(M, ctx, oracle_runs, name):
+def test_cache_build_matches_oracle(M, ctx, oracle_runs, name, prec):
     w, table, ora = oracle_runs(name)
-    model = M.mure_model_load(ctx, w.model)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
     cache = M.mure_build_prefix_cache(model, w.X)
     lg, pred = M.mure_cache_outputs(cache)
     ok, worst = logits_close(lg, ora["orig_logits"])
@@ -69,10 +73,11 @@ def test_cache_build_matches_oracle(M, ctx, oracle_runs, name):
     assert np.array_equal(pred[~ties], ora["orig_logits"].argmax(axis=1)[~ties])
 
 
+@pytest.mark.parametrize("prec", PRECISIONS)
 @pytest.mark.parametrize("name", list(CASES))
-def test_memoized_matches_oracle(M, ctx, oracle_runs, name):
+def test_memoized_matches_oracle(M, ctx, oracle_runs, name, prec):
     w, table, ora = oracle_runs(name)
-    model = M.mure_model_load(ctx, w.model)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
     cache = M.mure_build_prefix_cache(model, w.X)
     res = M.mure_eval_mutants(cache, table, logits=True)
     ok, worst = logits_close(res["logits"], ora["logits"])
@@ -84,10 +89,11 @@ def test_memoized_matches_oracle(M, ctx, oracle_runs, name):
     assert res["stats"]["n_rows"] == len(table) * len(w.X)
 
 
+@pytest.mark.parametrize("prec", PRECISIONS)
 @pytest.mark.parametrize("name", list(CASES))
-def test_memoized_equals_vanilla_bitwise(M, ctx, oracle_runs, name):
+def test_memoized_equals_vanilla_bitwise(M, ctx, oracle_runs, name, prec):
     w, table, _ = oracle_runs(name)
-    model = M.mure_model_load(ctx, w.model)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
     cache = M.mure_build_prefix_cache(model, w.X)
     memo = M.mure_eval_mutants(cache, table, logits=True)
     van = M.mure_eval_vanilla(model, w.X, table, logits=True)
@@ -158,12 +164,13 @@ def test_expanded_patches_bitexact(M, ctx, oracle_mod):
         assert mism <= max(1, total // 1_000_000), (mism, total)
 
 
-def test_batch_invariance(M, ctx):
+@pytest.mark.parametrize("prec", PRECISIONS)
+def test_batch_invariance(M, ctx, prec):
     """Tiny workspaces force many batches (input tiles, mutant chunks): results are
     bitwise identical to one large batch."""
     w = wl.workload("lenet5", 300, 1)
     table = all_ops(w.model, 6, seed=21)
-    model = M.mure_model_load(ctx, w.model)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
     cache = M.mure_build_prefix_cache(model, w.X)
     big = M.mure_eval_mutants(cache, table, logits=True)
     small = M.mure_eval_mutants(cache, table, logits=True, workspace_bytes=64 * 8 * 1024)
@@ -176,14 +183,15 @@ def test_batch_invariance(M, ctx):
     assert np.array_equal(sub["logits"].view(np.uint32), big["logits"][:, :70].view(np.uint32))
 
 
-def test_identity_mutants_never_killed(M, ctx):
-    w = wl.workload("resnet20", 96, 1)
+@pytest.mark.parametrize("name,prec", [("resnet20", "fp32"), ("mlp", "tf32x3"), ("lenet5", "tf32x3")])
+def test_identity_mutants_never_killed(M, ctx, name, prec):
+    w = wl.workload(name, 96, 1)
     rows = []
     for l in range(w.model.n_layers()):
         rows.append((l, "IDENTITY", [], 0.0, 0))
         rows.append((l, "GF", [0, 3], 0.0, 7))   # sigma multiplier 0
     table = wl.table_from_rows(rows)
-    model = M.mure_model_load(ctx, w.model)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
     cache = M.mure_build_prefix_cache(model, w.X)
     lg0, _ = M.mure_cache_outputs(cache)
     r = M.mure_eval_mutants(cache, table, logits=True)
