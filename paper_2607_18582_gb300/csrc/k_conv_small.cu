@@ -32,7 +32,7 @@ struct ConvSmallParams {
 // WP / HP padded input width / height, PAD zero padding, POOL: 2x2 max pool after
 // the activation.
 template <int KH, int KW, int IC, int OC, int OCT, int WP, int HP, int PAD, bool POOL>
-__global__ void __launch_bounds__(256, 2) k_conv_small(const ConvSmallParams p)
+__global__ void __launch_bounds__(256, 3) k_conv_small(const ConvSmallParams p)
 {
     constexpr int K = KH * KW * IC;
     constexpr int TILE = HP * WP * IC;
@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(256, 2) k_conv_small(const ConvSmallParams p)
     int base[4];
 #pragma unroll
     for (int s = 0; s < 4; ++s) base[s] = (oy[s] * WP + ox[s]) * IC;
-#pragma unroll
+#pragma unroll 1
     for (int ky = 0; ky < KH; ++ky)
 #pragma unroll
         for (int kx = 0; kx < KW; ++kx)
@@ -196,7 +196,7 @@ int launch_conv_small(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
 {
     if (rm.R <= 0) return 0;
     switch (S.variant) {
-    case 1: return launch_small<5, 5, 6, 16, 8, 14, 14, 0, true>(S, x, rm, z_out, z_stride, y_out, y_stride, s, ov);
+    case 1: return launch_small<5, 5, 6, 16, 4, 14, 14, 0, true>(S, x, rm, z_out, z_stride, y_out, y_stride, s, ov);
     case 2: return launch_small<5, 5, 1, 6, 6, 32, 32, 2, true>(S, x, rm, z_out, z_stride, y_out, y_stride, s, ov);
     }
     return 0;

@@ -211,37 +211,36 @@ __device__ __forceinline__ float cell_value(const PatchValsParams &p, const Slot
     return max4_first(w4[0], w4[1], w4[2], w4[3]);
 }
 
-// Items are (mutant g, slot q, cell c) of one input (blockIdx.y), so the mutants of
-// an input read its z and x while they are in L2.  `per_warp`: one item per warp.
-template <bool PER_WARP>
+// One warp per (mutant g, slot q) of one input (blockIdx.y), so the mutants of an
+// input read its z and x while they are in L2; the warp's lanes take the cells (one
+// lane per cell), or, for layers with fewer than 32 positions, share each cell's dot
+// product.
 __global__ void __launch_bounds__(256) k_patch_vals(const PatchValsParams p)
 {
     extern __shared__ float gap_buf[];  // [8][mcells] with GAP in lane mode
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int per_g = p.kmax * p.cells;
-    const int n_items = p.G * per_g;
+    const int item = (int)blockIdx.x * 8 + warp;     // warp-uniform
+    if (item >= p.G * p.kmax) return;
+    const int g = item / p.kmax, q = item - g * p.kmax;
+    if (q >= p.pa.n_neurons[g]) return;
+    const int op = p.pa.op[g];
+    const bool dot = op == MURE_OP_GF || op == MURE_OP_WS;
+    if (dot && p.skip_dot_ops) return;
+    const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
+    SlotCtx d;
+    d.op = op;
+    d.j = ids[q];
+    d.sj = op == MURE_OP_NS ? ids[q ^ 1] : d.j;
+    const float *e = dot ? p.pa.patch + p.pa.patch_off[g] + (int64_t)q * p.K : nullptr;
     for (int tl = blockIdx.y; tl < p.T; tl += gridDim.y) {
-        const int item = PER_WARP ? (int)blockIdx.x * 8 + warp : (int)blockIdx.x * 256 + threadIdx.x;
-        if (item >= n_items) continue;   // warp-uniform when PER_WARP
-        const int g = item / per_g, rem = item - g * per_g, q = rem / p.cells, c = rem - q * p.cells;
-        const int k = p.pa.n_neurons[g];
-        if (q >= k) continue;
-        const int op = p.pa.op[g];
-        const bool dot = op == MURE_OP_GF || op == MURE_OP_WS;
-        if (dot && p.skip_dot_ops) continue;
         const int64_t r = (int64_t)g * p.T + tl, t = p.t0 + tl;
-        const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
-        SlotCtx d;
-        d.op = op;
-        d.j = ids[q];
-        d.sj = op == MURE_OP_NS ? ids[q ^ 1] : d.j;
         d.z = p.z + (p.z_per_input ? t : r) * p.z_stride;
         d.x = dot ? p.x + (p.x_per_input ? t : r) * p.x_stride : nullptr;
         d.s = p.has_add ? p.skip + (p.skip_per_input ? t : r) * p.skip_stride : nullptr;
-        d.e = dot ? p.pa.patch + p.pa.patch_off[g] + (int64_t)q * p.K : nullptr;
-        float *o = p.out + r * p.out_stride + q * p.cells + c;
+        d.e = e;
+        float *o = p.out + r * p.out_stride + q * p.cells;
         if (p.gap) {
-            // the map cells, then their ascending fp32 sum / count (one warp)
+            // the map cells, then their ascending fp32 sum / count
             float s = 0.f;
             if (p.warp_dot) {
                 for (int cc = 0; cc < p.mcells; ++cc) s += cell_value(p, d, cc, lane);
@@ -252,10 +251,14 @@ __global__ void __launch_bounds__(256) k_patch_vals(const PatchValsParams p)
                 for (int cc = 0; cc < p.mcells; ++cc) s += gb[cc];
                 __syncwarp();
             }
-            if (lane == 0) *o = s / (float)p.mcells;
+            if (lane == 0) o[0] = s / (float)p.mcells;
+        } else if (p.warp_dot) {
+            for (int c = 0; c < p.cells; ++c) {
+                const float v = cell_value(p, d, c, lane);
+                if (lane == 0) o[c] = v;
+            }
         } else {
-            const float v = cell_value(p, d, c, lane);
-            if (!PER_WARP || lane == 0) *o = v;
+            for (int c = lane; c < p.cells; c += 32) o[c] = cell_value(p, d, c, lane);
         }
     }
 }
@@ -281,13 +284,10 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     p.out = out; p.out_stride = out_stride;
     p.warp_dot = (S.oh * S.ow) < 32;
     p.skip_dot_ops = skip_dot_ops;
-    const bool per_warp = p.gap || p.warp_dot;
-    const int64_t n_items = (int64_t)p.G * kmax * p.cells;
-    const unsigned gx = (unsigned)((n_items + (per_warp ? 7 : 255)) / (per_warp ? 8 : 256));
-    const dim3 grid(gx, (unsigned)std::min(rm.T, 65535));
+    const int64_t n_items = (int64_t)p.G * kmax;
+    const dim3 grid((unsigned)((n_items + 7) / 8), (unsigned)std::min(rm.T, 65535));
     const size_t smem = (S.gap && !p.warp_dot) ? 8 * (size_t)p.mcells * sizeof(float) : 0;
-    if (per_warp) k_patch_vals<true><<<grid, 256, smem, s>>>(p);
-    else k_patch_vals<false><<<grid, 256, smem, s>>>(p);
+    k_patch_vals<<<grid, 256, smem, s>>>(p);
     return 1;
 }
 

@@ -182,19 +182,11 @@ __global__ void __launch_bounds__(128, 1) k_tc_dense(const TcDenseParams p, int 
     const int nK = p.Kp / kTileK;
     uint32_t phase[kStages] = {0, 0};
     bool ok = true;
-    for (int kt = 0; kt < nK; ++kt) {
-        const int s = kt % kStages;
-        unsigned char *st = sm + s * stage_bytes;
-        if (kt >= kStages) {
-            // the MMAs that read this stage two tiles ago must be done
-            if (tid == 0) wait_ok = mbar_wait(smem_u32(&mbar[s]), phase[s]);
-            __syncthreads();
-            if (!wait_ok) { ok = false; break; }
-            phase[s] ^= 1;
-        }
-        const int k0 = kt * kTileK;
-        // A: one row per thread, 32 values, split into TF32 halves
-        float a[kTileK];
+    // registers of the next K-tile, loaded one tile ahead so that their latency
+    // overlaps the staging and MMAs of the current one
+    float a[kTileK];
+    float4 bh[kTileK / 4], bl[kTileK / 4];
+    auto load_tile = [&](int k0) {
 #pragma unroll
         for (int c = 0; c < kTileK / 4; ++c) {
             float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -210,6 +202,32 @@ __global__ void __launch_bounds__(128, 1) k_tc_dense(const TcDenseParams p, int 
             }
             a[4 * c] = v.x; a[4 * c + 1] = v.y; a[4 * c + 2] = v.z; a[4 * c + 3] = v.w;
         }
+        if (tid < Nt) {
+            const float4 *h = reinterpret_cast<const float4 *>(p.Whi + (int64_t)(n_base + tid) * p.Kp + k0);
+            const float4 *l = reinterpret_cast<const float4 *>(p.Wlo + (int64_t)(n_base + tid) * p.Kp + k0);
+#pragma unroll
+            for (int c = 0; c < kTileK / 4; ++c) { bh[c] = __ldg(h + c); bl[c] = __ldg(l + c); }
+        }
+    };
+    load_tile(0);
+    for (int kt = 0; kt < nK; ++kt) {
+        const int s = kt % kStages;
+        unsigned char *st = sm + s * stage_bytes;
+        const int k0 = kt * kTileK;
+        float ac[kTileK];
+        float4 bhc[kTileK / 4], blc[kTileK / 4];
+#pragma unroll
+        for (int i = 0; i < kTileK; ++i) ac[i] = a[i];
+#pragma unroll
+        for (int c = 0; c < kTileK / 4; ++c) { bhc[c] = bh[c]; blc[c] = bl[c]; }
+        if (kt + 1 < nK) load_tile(k0 + kTileK);
+        if (kt >= kStages) {
+            // the MMAs that read this stage two tiles ago must be done
+            if (tid == 0) wait_ok = mbar_wait(smem_u32(&mbar[s]), phase[s]);
+            __syncthreads();
+            if (!wait_ok) { ok = false; break; }
+            phase[s] ^= 1;
+        }
         for (int q = 0; q < ov_k; ++q) {
             // mutated channels: elements k = c * ch + j of this K-tile
             const int j = ov_ids[q];
@@ -218,29 +236,37 @@ __global__ void __launch_bounds__(128, 1) k_tc_dense(const TcDenseParams p, int 
                 const float pv = p.ov.patch[row * p.ov.row_stride + q * p.ov.cells + c];
 #pragma unroll
                 for (int i = 0; i < kTileK; ++i)
-                    if (k0 + i == c * p.ov.ch + j) a[i] = pv;
+                    if (k0 + i == c * p.ov.ch + j) ac[i] = pv;
             }
         }
 #pragma unroll
         for (int c = 0; c < kTileK / 4; ++c) {
             float4 hi, lo;
-            hi.x = tf32_rna(a[4 * c]);     lo.x = tf32_rna(a[4 * c] - hi.x);
-            hi.y = tf32_rna(a[4 * c + 1]); lo.y = tf32_rna(a[4 * c + 1] - hi.y);
-            hi.z = tf32_rna(a[4 * c + 2]); lo.z = tf32_rna(a[4 * c + 2] - hi.z);
-            hi.w = tf32_rna(a[4 * c + 3]); lo.w = tf32_rna(a[4 * c + 3] - hi.w);
+            hi.x = tf32_rna(ac[4 * c]);     lo.x = tf32_rna(ac[4 * c] - hi.x);
+            hi.y = tf32_rna(ac[4 * c + 1]); lo.y = tf32_rna(ac[4 * c + 1] - hi.y);
+            hi.z = tf32_rna(ac[4 * c + 2]); lo.z = tf32_rna(ac[4 * c + 2] - hi.z);
+            hi.w = tf32_rna(ac[4 * c + 3]); lo.w = tf32_rna(ac[4 * c + 3] - hi.w);
             const uint32_t off = sw128_off(tid, c);
             *reinterpret_cast<float4 *>(st + off) = hi;
             *reinterpret_cast<float4 *>(st + a_bytes + off) = lo;
         }
-        // B: rows of the pre-split weights
-        for (int n = tid; n < Nt; n += kTileM) {
-            const float4 *bh = reinterpret_cast<const float4 *>(p.Whi + (int64_t)(n_base + n) * p.Kp + k0);
-            const float4 *bl = reinterpret_cast<const float4 *>(p.Wlo + (int64_t)(n_base + n) * p.Kp + k0);
+        if (tid < Nt) {
+#pragma unroll
+            for (int c = 0; c < kTileK / 4; ++c) {
+                const uint32_t off = sw128_off(tid, c);
+                *reinterpret_cast<float4 *>(st + 2 * a_bytes + off) = bhc[c];
+                *reinterpret_cast<float4 *>(st + 2 * a_bytes + b_bytes + off) = blc[c];
+            }
+        }
+        // rows 128..255 of a 256-wide B tile
+        for (int n = tid + kTileM; n < Nt; n += kTileM) {
+            const float4 *h = reinterpret_cast<const float4 *>(p.Whi + (int64_t)(n_base + n) * p.Kp + k0);
+            const float4 *l = reinterpret_cast<const float4 *>(p.Wlo + (int64_t)(n_base + n) * p.Kp + k0);
 #pragma unroll
             for (int c = 0; c < kTileK / 4; ++c) {
                 const uint32_t off = sw128_off(n, c);
-                *reinterpret_cast<float4 *>(st + 2 * a_bytes + off) = __ldg(bh + c);
-                *reinterpret_cast<float4 *>(st + 2 * a_bytes + b_bytes + off) = __ldg(bl + c);
+                *reinterpret_cast<float4 *>(st + 2 * a_bytes + off) = __ldg(h + c);
+                *reinterpret_cast<float4 *>(st + 2 * a_bytes + b_bytes + off) = __ldg(l + c);
             }
         }
         // make the generic-proxy stores visible to the tensor core, then issue
