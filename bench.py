@@ -234,7 +234,7 @@ def main():
     ap.add_argument("--n-inputs", type=int, default=None, help="smaller case (profiling): first n inputs")
     ap.add_argument("--n-mutants", type=int, default=None, help="smaller case (profiling): first n mutants")
     ap.add_argument("--only-layer", type=int, default=None, help="keep only the mutants of this layer")
-    ap.add_argument("--precision", default="tf32x3", choices=["fp32", "tf32x3"],
+    ap.add_argument("--precision", default="tf32x3", choices=["fp32", "tf32x3", "tf32"],
                     help="layer arithmetic: fp32 CUDA-core chains, or tensor-core 3xTF32 for dense layers")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)

@@ -75,12 +75,15 @@ enum { MURE_ACT_NONE = 0, MURE_ACT_RELU = 1 };
 enum { MURE_OP_GF = 0, MURE_OP_NEB = 1, MURE_OP_NAI = 2, MURE_OP_NS = 3, MURE_OP_WS = 4, MURE_OP_IDENTITY = 5 };
 
 /* Arithmetic of the layer kernels.  FP32: fp32 FMA chains on the CUDA cores.
- * TF32X3: tensor cores (tcgen05), fp32 operands split into two TF32 halves, three
- * products per pair.  BF16: tensor cores, bf16 operands, fp32 accumulation (the
- * reduced-precision variant).  One model uses one arithmetic for every layer
- * computation (cache build, vanilla prefix and suffix), so memoized and vanilla
- * results stay bit-identical under every mode. */
-enum { MURE_PREC_FP32 = 0, MURE_PREC_TF32X3 = 1, MURE_PREC_BF16 = 2 };
+ * TF32X3: dense layers and convolutions of >= 16 outputs on the tensor cores
+ * (tcgen05), fp32 operands split into two TF32 halves, three products per pair
+ * (fp32-level accuracy); small LeNet-size convolutions stay on the CUDA cores.
+ * TF32: the same layer selection with one TF32 product (the reduced-precision
+ * variant; its kill verdicts are compared with the fp32 oracle's, not bit-matched).  BF16:
+ * reserved.  The output layer always uses the fp32 CUDA-core kernel.  One model uses
+ * one arithmetic for every layer computation (cache build, vanilla prefix and
+ * suffix), so memoized and vanilla results stay bit-identical under every mode. */
+enum { MURE_PREC_FP32 = 0, MURE_PREC_TF32X3 = 1, MURE_PREC_BF16 = 2, MURE_PREC_TF32 = 3 };
 
 /* One node.  in0/in1 are node ids (< this node's id) or -1 for the network input.
  * Weighted nodes (CONV2D, DENSE) are numbered 0..L-1 in node order: these numbers

@@ -14,6 +14,13 @@ using namespace mure;
 
 namespace {
 
+// MURE_TC_CONV=1 puts every convolution of a TF32X3 model on the tensor cores.
+bool tc_conv_forced()
+{
+    const char *e = getenv("MURE_TC_CONV");
+    return e && e[0] == '1';
+}
+
 // ------------------------------------------------------------------ plumbing --
 
 struct Fail {
@@ -635,13 +642,17 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         return launches;
     }
     // first suffix stage: the overlay is applied while its input tile is staged, or
-    // the rows are materialised for kernels that read plain rows
+    // the rows are materialised for kernels that read plain rows and whenever a later
+    // residual add reads x_{l+1} as its skip input
     const Stage &Sn = m->st[l + 1];
-    if (Sn.tc) {
+    bool skip_reader = false;
+    for (int v = l + 2; v < L; ++v) skip_reader |= m->st[v].has_add && m->st[v].skip_src == l + 1;
+    if (Sn.tc && !skip_reader) {
         timed(l + 1, 2 * Sn.macs * rm.R, [&] {
-            return launch_tc_dense(Sn, base, rm, nullptr, 0, ws.xb[l + 2], m->xd[l + 2].stride, s, &ov);
+            return launch_tc(Sn, base, rm, nullptr, 0, skip_of(Sn), ws.xb[l + 2], m->xd[l + 2].stride, ws.gap_tmp, s,
+                             &ov);
         });
-    } else if (Sn.variant > 0) {
+    } else if (Sn.variant > 0 && !skip_reader) {
         timed(l + 1, 2 * Sn.macs * rm.R, [&] {
             return launch_conv_small(Sn, base, rm, nullptr, 0, ws.xb[l + 2], m->xd[l + 2].stride, s, &ov);
         });
@@ -940,8 +951,8 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
         FAILIF(!d || !out || !d->nodes || d->n_nodes < 1, c, MURE_ERR_INVALID_ARG, "NULL model description");
         *out = nullptr;
         FAILIF(d->in_h < 1 || d->in_w < 1 || d->in_c < 1, c, MURE_ERR_INVALID_ARG, "bad input shape");
-        FAILIF(d->precision != MURE_PREC_FP32 && d->precision != MURE_PREC_TF32X3, c, MURE_ERR_UNSUPPORTED,
-               "precision %d is not available", d->precision);
+        FAILIF(d->precision != MURE_PREC_FP32 && d->precision != MURE_PREC_TF32X3 && d->precision != MURE_PREC_TF32,
+               c, MURE_ERR_UNSUPPORTED, "precision %d is not available", d->precision);
         CK(c, cudaSetDevice(c->device));
         auto *m = new mure_model();
         m->ctx = c;
@@ -963,9 +974,17 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             S.variant = (force && force[0] == '1') ? 0 : conv_small_variant(S);
             S.err = c->err_dev;
         }
-        // TF32X3: dense layers before the output layer run on the tensor cores
-        if (d->precision == MURE_PREC_TF32X3)
-            for (int l = 0; l + 1 < m->L; ++l) m->st[l].tc = tc_dense_supported(m->st[l]);
+        // tensor-core modes: layers before the output layer with >= 16 outputs run on
+        // the tensor cores (3xTF32, or one TF32 MMA in the reduced-precision variant);
+        // in TF32X3 the LeNet-size convolutions keep their CUDA-core kernel, which is
+        // faster there than the implicit GEMM
+        for (int l = 0; l + 1 < m->L; ++l) {
+            Stage &S = m->st[l];
+            const bool take = tc_supported(S) && (S.kind == MURE_NODE_DENSE || S.variant == 0 || tc_conv_forced());
+            if (take && d->precision == MURE_PREC_TF32X3) S.tc = 1;
+            else if (take && d->precision == MURE_PREC_TF32) S.tc = 2;
+            if (S.tc) S.variant = 0;
+        }
         std::vector<int> wn;
         for (int v = 0; v < d->n_nodes; ++v)
             if (weighted(d->nodes[v].kind)) wn.push_back(v);

@@ -32,7 +32,7 @@ struct Stage {
     int yh, yw, yc;           // output x_{v+1}
     int64_t macs;             // multiply-accumulates per row
     int variant = 0;          // 0: implicit-GEMM kernel; > 0: a shared-memory direct conv
-    int tc = 0;               // 1: tensor-core (tcgen05, 3xTF32) kernel
+    int tc = 0;               // tensor-core kernel: 1 = 3xTF32, 2 = one TF32 MMA (variant)
     float *Wtc_hi = nullptr;  // tc: TF32 halves of W, zero-padded [round16(oc)][round32(K)]
     float *Wtc_lo = nullptr;
     int *err = nullptr;       // device error word of the context (bounded waits)
@@ -131,12 +131,16 @@ int conv_small_variant(const Stage &S);
 int launch_conv_small(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, float *y_out,
                       int64_t y_stride, cudaStream_t s, const Overlay *ov = nullptr);
 
-// Tensor-core dense layer (tcgen05, 3xTF32): which layers it takes, the weight split
-// done at model load, and the launcher (rows as for the stage kernel, plus overlay).
-int tc_dense_supported(const Stage &S);
+// Tensor-core layers (tcgen05; 3xTF32, or one TF32 MMA in the reduced-precision
+// mode): which layers the kernel takes, the weight split done at model load, and the
+// launcher (arguments as for the stage kernel, plus the overlay).
+int tc_supported(const Stage &S);
 int launch_split_weights(const Stage &S, float *hi, float *lo, cudaStream_t s);
-int launch_tc_dense(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, float *y_out, int64_t y_stride,
-                    cudaStream_t s, const Overlay *ov = nullptr);
+int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
+              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov = nullptr);
+
+// Global average pooling of R rows of a [P][C] map.
+int launch_gap(const float *in, int64_t in_stride, int P, int C, int R, float *y, int64_t y_stride, cudaStream_t s);
 
 // Final dense layer (F -> C, C <= 32) over R rows, with the fused epilogue.
 struct FinalArgs {

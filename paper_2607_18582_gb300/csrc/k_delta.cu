@@ -232,6 +232,26 @@ __global__ void __launch_bounds__(256) k_patch_vals(const PatchValsParams p)
     d.j = ids[q];
     d.sj = op == MURE_OP_NS ? ids[q ^ 1] : d.j;
     const float *e = dot ? p.pa.patch + p.pa.patch_off[g] + (int64_t)q * p.K : nullptr;
+    if (!dot && (p.warp_dot || p.cells < 32)) {
+        // no fan-in sum and few cells: one input per lane, its cells in order (a GAP
+        // value is the same ascending sum over the map cells as below)
+        for (int tl = blockIdx.y * 32 + lane; tl < p.T; tl += gridDim.y * 32) {
+            const int64_t r = (int64_t)g * p.T + tl, t = p.t0 + tl;
+            d.z = p.z + (p.z_per_input ? t : r) * p.z_stride;
+            d.x = nullptr;
+            d.s = p.has_add ? p.skip + (p.skip_per_input ? t : r) * p.skip_stride : nullptr;
+            d.e = nullptr;
+            float *o = p.out + r * p.out_stride + q * p.cells;
+            if (p.gap) {
+                float s = 0.f;
+                for (int cc = 0; cc < p.mcells; ++cc) s += cell_value(p, d, cc, lane);
+                o[0] = s / (float)p.mcells;
+            } else {
+                for (int c = 0; c < p.cells; ++c) o[c] = cell_value(p, d, c, lane);
+            }
+        }
+        return;
+    }
     for (int tl = blockIdx.y; tl < p.T; tl += gridDim.y) {
         const int64_t r = (int64_t)g * p.T + tl, t = p.t0 + tl;
         d.z = p.z + (p.z_per_input ? t : r) * p.z_stride;
@@ -285,7 +305,11 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     p.warp_dot = (S.oh * S.ow) < 32;
     p.skip_dot_ops = skip_dot_ops;
     const int64_t n_items = (int64_t)p.G * kmax;
-    const dim3 grid((unsigned)((n_items + 7) / 8), (unsigned)std::min(rm.T, 65535));
+    // each warp walks several inputs (blockIdx.y, +gridDim.y, ...): enough blocks to
+    // fill the GPU, few enough that block scheduling stays negligible
+    const int64_t gx = (n_items + 7) / 8;
+    const int64_t gy = std::max<int64_t>(1, std::min<int64_t>(rm.T, (152 * 16 + gx - 1) / gx));
+    const dim3 grid((unsigned)gx, (unsigned)gy);
     const size_t smem = (S.gap && !p.warp_dot) ? 8 * (size_t)p.mcells * sizeof(float) : 0;
     k_patch_vals<<<grid, 256, smem, s>>>(p);
     return 1;

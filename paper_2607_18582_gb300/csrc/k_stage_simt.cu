@@ -166,7 +166,7 @@ int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
                       int64_t y_stride, float *gap_tmp, cudaStream_t s)
 {
     if (rm.R <= 0) return 0;
-    if (S.tc) return launch_tc_dense(S, x, rm, z_out, z_stride, y_out, y_stride, s);
+    if (S.tc) return launch_tc(S, x, rm, z_out, z_stride, skip, y_out, y_stride, gap_tmp, s);
     if (S.variant > 0) return launch_conv_small(S, x, rm, z_out, z_stride, y_out, y_stride, s);
     StageParams p{};
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
@@ -246,11 +246,63 @@ __device__ __forceinline__ void epilogue_row(const FinalArgs &fa, int64_t t0, in
     }
 }
 
+// argmax / near tie / kill of one row's logits held in registers (CP >= C, unrolled
+// and predicated): the same rules as argmax_first and near_tie.
+template <int CP>
+__device__ __forceinline__ int argmax_reg(const float (&v)[CP], int C)
+{
+    int best = 0;
+    float bv = v[0];
+    bool bnan = isnan(v[0]);
+#pragma unroll
+    for (int c = 1; c < CP; ++c)
+        if (c < C && !bnan && (isnan(v[c]) || v[c] > bv)) { best = c; bv = v[c]; bnan = isnan(v[c]); }
+    return best;
+}
+
+template <int CP>
+__device__ __forceinline__ void epilogue_reg(const FinalArgs &fa, int64_t t0, int T, int64_t row, bool in_range,
+                                             const float (&v)[CP], int C)
+{
+    const int g = (int)(row / T);
+    const int64_t t = t0 + row % T;
+    const bool valid = in_range && t < fa.n_in;
+    int arg = 0;
+    bool near = false;
+    if (valid) {
+        arg = argmax_reg<CP>(v, C);
+        float top = v[0], second = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < CP; ++c) if (c == arg) top = v[c];
+#pragma unroll
+        for (int c = 0; c < CP; ++c)
+            if (c < C && c != arg && v[c] > second) second = v[c];
+        near = C >= 2 && (top - second) < 1e-4f * fabsf(top);
+    }
+    const bool kill = valid && fa.pred0[t] == fa.label[t] && arg != fa.label[t];
+    const unsigned kb = __ballot_sync(0xffffffffu, kill);
+    const unsigned nb = __ballot_sync(0xffffffffu, near);
+    const int lane = threadIdx.x & 31;
+    if (lane == 0 && in_range) {
+        const int mid = fa.mutant_id[g];
+        fa.kill32[(int64_t)mid * fa.words32 + (t >> 5)] = kb;
+        if (nb && fa.near_ties) atomicAdd(fa.near_ties, (unsigned long long)__popc(nb));
+    }
+    if (valid && fa.logits_out) {
+        float *o = fa.logits_out + ((int64_t)fa.mutant_id[g] * fa.n_in + t) * C;
+#pragma unroll
+        for (int c = 0; c < CP; ++c)
+            if (c < C) o[c] = v[c];
+    }
+}
+
+// CP: the class count rounded up to a multiple of 4 (the accumulators kept per row).
+template <int CP>
 __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
 {
     constexpr int RB = 128, FC = 32;
     __shared__ float xs[RB][FC + 1];
-    __shared__ __align__(16) float ws[FC][kMaxClasses];
+    __shared__ __align__(16) float ws[FC][CP];
     const int tid = threadIdx.x;
     const int64_t row0 = (int64_t)blockIdx.x * RB;
     const int64_t row = row0 + tid;
@@ -263,20 +315,24 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
         ov_k = p.ov.n_neurons[g];
         ov_ids = p.ov.ids + p.ov.neuron_off[g];
     }
-    float acc[kMaxClasses];
+    __shared__ const float *xrow_of[RB];
+    float acc[CP];
 #pragma unroll
-    for (int c = 0; c < kMaxClasses; ++c) acc[c] = 0.f;
+    for (int c = 0; c < CP; ++c) acc[c] = 0.f;
+    {
+        const int64_t r = row0 + tid;
+        xrow_of[tid] = r < p.R ? p.x + (p.x_per_input ? (p.t0 + r % p.T) : r) * p.x_stride : nullptr;
+    }
+    __syncthreads();
     for (int f0 = 0; f0 < p.F; f0 += FC) {
+#pragma unroll 8
         for (int i = tid; i < RB * FC; i += RB) {
             const int rl = i / FC, fl = i % FC;
-            const int64_t r = row0 + rl;
-            float v = 0.f;
-            if (r < p.R && f0 + fl < p.F)
-                v = __ldg(p.x + (p.x_per_input ? (p.t0 + r % p.T) : r) * p.x_stride + f0 + fl);
-            xs[rl][fl] = v;
+            const float *xr = xrow_of[rl];
+            xs[rl][fl] = (xr && f0 + fl < p.F) ? __ldg(xr + f0 + fl) : 0.f;
         }
-        for (int i = tid; i < FC * kMaxClasses; i += RB) {
-            const int fl = i / kMaxClasses, c = i % kMaxClasses;
+        for (int i = tid; i < FC * CP; i += RB) {
+            const int fl = i / CP, c = i % CP;
             ws[fl][c] = (c < p.C && f0 + fl < p.F) ? __ldg(p.W + (int64_t)c * p.F + f0 + fl) : 0.f;
         }
         __syncthreads();
@@ -291,34 +347,41 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
         for (int fl = 0; fl < fe; ++fl) {
             const float xv = xs[tid][fl];
 #pragma unroll
-            for (int c = 0; c < kMaxClasses; ++c)
-                if (c < p.C) acc[c] = fmaf(xv, ws[fl][c], acc[c]);
+            for (int c4 = 0; c4 < CP; c4 += 4) {
+                const float4 w4 = *reinterpret_cast<const float4 *>(&ws[fl][c4]);
+                acc[c4] = fmaf(xv, w4.x, acc[c4]);
+                acc[c4 + 1] = fmaf(xv, w4.y, acc[c4 + 1]);
+                acc[c4 + 2] = fmaf(xv, w4.z, acc[c4 + 2]);
+                acc[c4 + 3] = fmaf(xv, w4.w, acc[c4 + 3]);
+            }
         }
         __syncthreads();
     }
-    float v[kMaxClasses];
+    float v[CP];
 #pragma unroll
-    for (int c = 0; c < kMaxClasses; ++c) {
+    for (int c = 0; c < CP; ++c) {
         const float z = c < p.C ? acc[c] + __ldg(p.b + c) : 0.f;
-        if (in_range && c < p.C) {
-            if (p.fa.z_out) p.fa.z_out[row * p.fa.z_stride + c] = z;
-        }
-        acc[c] = z;
+        if (in_range && c < p.C && p.fa.z_out) p.fa.z_out[row * p.fa.z_stride + c] = z;
         v[c] = act_apply(p.act, z);
     }
     if (p.fa.mode == 1) {  // cache build: logits rows and original predictions
         if (in_range) {
-            for (int c = 0; c < p.C; ++c) p.fa.x_out[row * p.fa.x_stride + c] = v[c];
-            p.fa.pred_out[row] = argmax_first(v, p.C);
+#pragma unroll
+            for (int c = 0; c < CP; ++c)
+                if (c < p.C) p.fa.x_out[row * p.fa.x_stride + c] = v[c];
+            p.fa.pred_out[row] = argmax_reg<CP>(v, p.C);
         }
         return;
     }
     if (p.fa.mode == 2) {  // per-row logits for a following delta + epilogue
-        if (in_range)
-            for (int c = 0; c < p.C; ++c) p.fa.logits_rows[row * p.fa.x_stride + c] = v[c];
+        if (in_range) {
+#pragma unroll
+            for (int c = 0; c < CP; ++c)
+                if (c < p.C) p.fa.logits_rows[row * p.fa.x_stride + c] = v[c];
+        }
         return;
     }
-    epilogue_row(p.fa, p.t0, p.T, row, in_range, v, p.C);
+    epilogue_reg<CP>(p.fa, p.t0, p.T, row, in_range, v, p.C);
 }
 
 __global__ void __launch_bounds__(128) k_epilogue(const float *__restrict__ lg, int64_t stride, int per_input, int C,
@@ -343,6 +406,14 @@ __global__ void __launch_bounds__(128) k_epilogue(const float *__restrict__ lg, 
     epilogue_row(fa, t0, T, row, in_range, v, C);
 }
 
+int launch_gap(const float *in, int64_t in_stride, int P, int C, int R, float *y, int64_t y_stride, cudaStream_t s)
+{
+    const int64_t n = (int64_t)R * C;
+    if (n <= 0) return 0;
+    k_gap<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(in, in_stride, P, C, R, y, y_stride);
+    return 1;
+}
+
 int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s, const Overlay *ov)
 {
     if (rm.R <= 0) return 0;
@@ -353,7 +424,13 @@ int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cu
     p.F = S.K; p.C = S.oc; p.act = S.act1;
     p.W = S.W; p.b = S.b;
     p.fa = fa;
-    k_final_dense<<<(unsigned)((rm.R + 127) / 128), 128, 0, s>>>(p);
+    const unsigned blocks = (unsigned)((rm.R + 127) / 128);
+    const int cp = (p.C + 3) & ~3;
+    if (cp <= 4) k_final_dense<4><<<blocks, 128, 0, s>>>(p);
+    else if (cp <= 8) k_final_dense<8><<<blocks, 128, 0, s>>>(p);
+    else if (cp <= 12) k_final_dense<12><<<blocks, 128, 0, s>>>(p);
+    else if (cp <= 16) k_final_dense<16><<<blocks, 128, 0, s>>>(p);
+    else k_final_dense<32><<<blocks, 128, 0, s>>>(p);
     return 1;
 }
 

@@ -1,18 +1,23 @@
-// Dense layers on the 5th-generation tensor cores (tcgen05) with fp32-level accuracy:
-// every fp32 operand a is split into two TF32 halves, a = a_hi + a_lo (a_hi = a
-// rounded to TF32, a_lo = the rounded remainder), and each product uses three MMAs,
-// a_hi*b_hi + a_hi*b_lo + a_lo*b_hi, accumulated in fp32 in tensor memory.
+// Dense and convolution layers on the 5th-generation tensor cores (tcgen05) with
+// fp32-level accuracy: every fp32 operand a is split into two TF32 halves, a = a_hi +
+// a_lo (a_hi = a rounded to TF32, a_lo = the rounded remainder), and each product
+// uses three MMAs, a_hi*b_hi + a_hi*b_lo + a_lo*b_hi, accumulated in fp32 in tensor
+// memory.  (The reduced-precision variant uses a_hi*b_hi alone.)
 //
-// One CTA of 4 warps computes a 128-row x N tile (N <= 256, a multiple of 16):
-//   - all 128 threads stage the K-tile (32 values per row) of A (batch rows, with the
-//     first suffix stage's mutated channels written over the cached rows) and of the
-//     pre-split weights, split A, and store both halves in the 128-byte-swizzled
+// The GEMM: M = (batch row, output position) pairs, K = the fan-in (ky, kx, ci), N =
+// output channels.  A convolution is an implicit GEMM: the producer threads gather
+// the im2col rows from the NHWC input.  One CTA of 4 warps computes a 128 x N tile
+// (N <= 256, a multiple of 16):
+//   - all 128 threads stage the K-tile (32 values per GEMM row) of A (batch rows, with
+//     the first suffix stage's mutated channels written over the cached rows) and of
+//     the pre-split weights, split A, and store the halves in the 128-byte-swizzled
 //     K-major layout the MMA reads;
 //   - thread 0 issues 4 K-steps x 3 MMAs (kind::tf32, M=128, K=8) per K-tile and
 //     commits them to the stage's mbarrier; two stages alternate, so staging tile
 //     k+1 overlaps the MMAs of tile k;
-//   - the epilogue reads the accumulator back with tcgen05.ld (thread = row = TMEM
-//     lane), adds the bias, applies the activation and writes z and y rows.
+//   - the epilogue reads the accumulator back with tcgen05.ld (thread = GEMM row =
+//     TMEM lane), adds the bias and applies activation, residual add and 2x2 max pool
+//     (the four positions of a window are four consecutive lanes).
 // The K order of the accumulation is fixed and independent of the row's position in
 // the tile, so a row gives the same bits in every batch (memoized == vanilla).
 // Every mbarrier wait is bounded; on expiry the kernel records an error code, waits
@@ -28,7 +33,6 @@ namespace {
 
 constexpr int kTileM = 128;
 constexpr int kTileK = 32;                  // fp32 / tf32 values per 128-byte row
-constexpr int kStages = 2;
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
 {
@@ -122,21 +126,73 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float *v)
 
 }  // namespace
 
-struct TcDenseParams {
+struct TcParams {
     const float *x; int64_t x_stride; int x_per_input;
     int64_t t0; int T; int R;
+    int dense;                   // 1: a dense layer (one GEMM row per batch row)
+    int ih, iw, ic, kh, kw, stride, pad, oh, ow;
+    int P, pool, pw;             // GEMM rows per batch row (ordered as k_stage_simt)
     int K, Kp, N, Np;            // fan-in (padded to 32), outputs (padded to 16)
     const float *Whi, *Wlo;      // [Np][Kp] TF32 halves of the weights
     const float *b;
-    int act;
+    int act1, has_add, act2;
+    const float *skip; int64_t skip_stride; int skip_per_input; int sk_w, sk_c, sk_stride;
     float *z; int64_t z_stride;
     float *y; int64_t y_stride;
+    int three;                   // 1: 3xTF32, 0: one TF32 MMA (reduced precision)
     Overlay ov;
     int *err;
 };
 
-// ncols: the power of two >= max(32, Np) tensor-memory columns this CTA allocates.
-__global__ void __launch_bounds__(128, 1) k_tc_dense(const TcDenseParams p, int ncols)
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, int src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// One thread's GEMM row of an M-tile: batch row, output position, input row, overlay.
+struct RowInfo {
+    int64_t row;
+    int oy, ox, py, px;
+    const float *xrow;
+    int ov_k;
+    const int32_t *ov_ids;
+    bool ok;
+};
+
+__device__ __forceinline__ RowInfo row_info(const TcParams &p, int64_t m)
+{
+    RowInfo ri{};
+    ri.ok = m < (int64_t)p.R * p.P;
+    if (!ri.ok) return ri;
+    ri.row = m / p.P;
+    const int q = (int)(m - ri.row * p.P);
+    if (p.pool) {
+        const int w = q >> 2, sub = q & 3;
+        ri.py = w / p.pw; ri.px = w % p.pw;
+        ri.oy = 2 * ri.py + (sub >> 1);
+        ri.ox = 2 * ri.px + (sub & 1);
+    } else {
+        ri.oy = q / p.ow;
+        ri.ox = q % p.ow;
+    }
+    ri.xrow = p.x + (p.x_per_input ? p.t0 + ri.row % p.T : ri.row) * p.x_stride;
+    if (p.ov.patch) {
+        const int g = (int)(ri.row / p.T);
+        ri.ov_k = p.ov.n_neurons[g];
+        ri.ov_ids = p.ov.ids + p.ov.neuron_off[g];
+    }
+    return ri;
+}
+
+// ncols: the power of two >= max(32, N tile) tensor-memory columns this CTA allocates.
+// DENSE: one GEMM row per batch row; THREE: 3xTF32 (else one TF32 product).
+// The CTA is persistent: it loops over M-tiles (blockIdx.x, += gridDim.x) with the
+// operand pipeline running D = S-1 K-steps ahead across tile boundaries.
+template <bool DENSE, bool THREE>
+__global__ void __launch_bounds__(128, 1) k_tc_gemm(const TcParams p, int ncols, int S)
 {
     extern __shared__ __align__(1024) unsigned char smraw[];
     // 1024-byte aligned operand stages: [stage][A_hi, A_lo, B_hi, B_lo]
@@ -144,12 +200,20 @@ __global__ void __launch_bounds__(128, 1) k_tc_dense(const TcDenseParams p, int 
     const int n_base = blockIdx.y * 256;            // this CTA's output columns
     const int Nt = min(256, p.Np - n_base);        // a multiple of 16
     const int a_bytes = kTileM * 128, b_bytes = Nt * 128;
-    const int stage_bytes = 2 * a_bytes + 2 * b_bytes;
-    __shared__ __align__(8) uint64_t mbar[kStages];
+    const int stage_bytes = THREE ? 2 * a_bytes + 2 * b_bytes : a_bytes + b_bytes;
+    const int b_off = THREE ? 2 * a_bytes : a_bytes;
+    constexpr int kMaxStages = 6;
+    __shared__ __align__(8) uint64_t mbar[kMaxStages];
     __shared__ uint32_t tmem_base_sh;
     __shared__ int wait_ok;   // thread 0's wait result, so every decision is CTA-uniform
     const int tid = threadIdx.x, warp = tid >> 5;
-    const int64_t m0 = (int64_t)blockIdx.x * kTileM;
+    const int D = S - 1;
+    const int64_t M = (int64_t)p.R * p.P;
+    const int64_t n_tiles = (M + kTileM - 1) / kTileM;
+    const int nK = p.Kp / kTileK;
+    // this CTA's tiles: blockIdx.x, blockIdx.x + gridDim.x, ...
+    const int64_t my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+    const int64_t total = my_tiles * nK;
 
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base_sh)),
@@ -157,116 +221,151 @@ __global__ void __launch_bounds__(128, 1) k_tc_dense(const TcDenseParams p, int 
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(smem_u32(&mbar[s]), 1);
+        for (int s = 0; s < S; ++s) mbar_init(smem_u32(&mbar[s]), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_base_sh;
+    // thread 0's bookkeeping of each stage's MMA commits (issued, waited for)
+    uint32_t issued[kMaxStages] = {0, 0, 0, 0, 0, 0}, waited[kMaxStages] = {0, 0, 0, 0, 0, 0};
+    auto wait_stage = [&](int s) -> bool {
+        while (waited[s] < issued[s]) {
+            if (!mbar_wait(smem_u32(&mbar[s]), waited[s] & 1)) return false;
+            ++waited[s];
+        }
+        return true;
+    };
 
-    // this thread's A row and its overlay
-    const int64_t row = m0 + tid;
-    const bool row_ok = row < p.R;
-    const float *arow = nullptr;
-    int ov_k = 0;
-    const int32_t *ov_ids = nullptr;
-    if (row_ok) {
-        arow = p.x + (p.x_per_input ? p.t0 + row % p.T : row) * p.x_stride;
-        if (p.ov.patch) {
-            const int g = (int)(row / p.T);
-            ov_k = p.ov.n_neurons[g];
-            ov_ids = p.ov.ids + p.ov.neuron_off[g];
-        }
-    }
-    const int nK = p.Kp / kTileK;
-    uint32_t phase[kStages] = {0, 0};
-    bool ok = true;
-    // registers of the next K-tile, loaded one tile ahead so that their latency
-    // overlaps the staging and MMAs of the current one
-    float a[kTileK];
-    float4 bh[kTileK / 4], bl[kTileK / 4];
-    auto load_tile = [&](int k0) {
+    // queue the copies of K-step j (tile j / nK, K-tile j % nK) into its stage
+    int64_t pf_tile = -1;
+    RowInfo pf{};
+    auto issue = [&](int64_t j) {
+        const int64_t tile = blockIdx.x + (j / nK) * gridDim.x;
+        const int kt = (int)(j % nK), s = (int)(j % S), k0 = kt * kTileK;
+        if (tile != pf_tile) { pf = row_info(p, tile * kTileM + tid); pf_tile = tile; }
+        const uint32_t st = smem_u32(sm + s * stage_bytes);
+        if (DENSE) {
 #pragma unroll
-        for (int c = 0; c < kTileK / 4; ++c) {
-            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (row_ok) {
+            for (int c = 0; c < kTileK / 4; ++c) {
                 const int kk = k0 + 4 * c;
-                if (kk + 3 < p.K) v = __ldg(reinterpret_cast<const float4 *>(arow + kk));
-                else {
-                    v.x = kk < p.K ? arow[kk] : 0.f;
-                    v.y = kk + 1 < p.K ? arow[kk + 1] : 0.f;
-                    v.z = kk + 2 < p.K ? arow[kk + 2] : 0.f;
-                    v.w = kk + 3 < p.K ? arow[kk + 3] : 0.f;
-                }
+                const int nb = pf.ok ? max(0, min(16, (p.K - kk) * 4)) : 0;
+                cp_async16(st + sw128_off(tid, c), nb ? (const void *)(pf.xrow + kk) : (const void *)p.b, nb);
             }
-            a[4 * c] = v.x; a[4 * c + 1] = v.y; a[4 * c + 2] = v.z; a[4 * c + 3] = v.w;
-        }
-        if (tid < Nt) {
-            const float4 *h = reinterpret_cast<const float4 *>(p.Whi + (int64_t)(n_base + tid) * p.Kp + k0);
-            const float4 *l = reinterpret_cast<const float4 *>(p.Wlo + (int64_t)(n_base + tid) * p.Kp + k0);
+        } else if ((p.ic & 3) == 0) {
 #pragma unroll
-            for (int c = 0; c < kTileK / 4; ++c) { bh[c] = __ldg(h + c); bl[c] = __ldg(l + c); }
+            for (int c = 0; c < kTileK / 4; ++c) {
+                const int kk = k0 + 4 * c;
+                const float *src = p.b;
+                int nb = 0;
+                if (pf.ok && kk < p.K) {
+                    const int ci = kk % p.ic, t = kk / p.ic, kx = t % p.kw, ky = t / p.kw;
+                    const int iy = pf.oy * p.stride - p.pad + ky, ix = pf.ox * p.stride - p.pad + kx;
+                    if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw) {
+                        src = pf.xrow + ((int64_t)iy * p.iw + ix) * p.ic + ci;
+                        nb = 16;
+                    }
+                }
+                cp_async16(st + sw128_off(tid, c), src, nb);
+            }
+        } else {
+            // channels not a multiple of 4: plain loads, fp32 stored in place
+            int ci = k0 % p.ic, t = k0 / p.ic, kx = t % p.kw, ky = t / p.kw;
+            float v[kTileK];
+#pragma unroll
+            for (int i = 0; i < kTileK; ++i) {
+                v[i] = 0.f;
+                if (pf.ok && k0 + i < p.K) {
+                    const int iy = pf.oy * p.stride - p.pad + ky, ix = pf.ox * p.stride - p.pad + kx;
+                    if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw)
+                        v[i] = __ldg(pf.xrow + ((int64_t)iy * p.iw + ix) * p.ic + ci);
+                }
+                if (++ci == p.ic) { ci = 0; if (++kx == p.kw) { kx = 0; ++ky; } }
+            }
+#pragma unroll
+            for (int c = 0; c < kTileK / 4; ++c)
+                *reinterpret_cast<float4 *>(sm + s * stage_bytes + sw128_off(tid, c)) =
+                    make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+        }
+        for (int n = tid; n < Nt; n += kTileM) {
+            const float *h = p.Whi + (int64_t)(n_base + n) * p.Kp + k0;
+            const float *l = p.Wlo + (int64_t)(n_base + n) * p.Kp + k0;
+#pragma unroll
+            for (int c = 0; c < kTileK / 4; ++c) {
+                cp_async16(st + b_off + sw128_off(n, c), h + 4 * c, 16);
+                if (THREE) cp_async16(st + b_off + b_bytes + sw128_off(n, c), l + 4 * c, 16);
+            }
         }
     };
-    load_tile(0);
-    for (int kt = 0; kt < nK; ++kt) {
-        const int s = kt % kStages;
+
+    bool ok = true;
+    for (int64_t j = 0; j < D; ++j) {
+        if (j < total) issue(j);
+        cp_async_commit();
+    }
+    int64_t cur_tile = -1;
+    RowInfo ri{};
+    for (int64_t it = 0; it < total; ++it) {
+        const int64_t tile = blockIdx.x + (it / nK) * gridDim.x;
+        const int kt = (int)(it % nK), s = (int)(it % S), k0 = kt * kTileK;
+        if (tile != cur_tile) { ri = row_info(p, tile * kTileM + tid); cur_tile = tile; }
         unsigned char *st = sm + s * stage_bytes;
-        const int k0 = kt * kTileK;
-        float ac[kTileK];
-        float4 bhc[kTileK / 4], blc[kTileK / 4];
-#pragma unroll
-        for (int i = 0; i < kTileK; ++i) ac[i] = a[i];
-#pragma unroll
-        for (int c = 0; c < kTileK / 4; ++c) { bhc[c] = bh[c]; blc[c] = bl[c]; }
-        if (kt + 1 < nK) load_tile(k0 + kTileK);
-        if (kt >= kStages) {
-            // the MMAs that read this stage two tiles ago must be done
-            if (tid == 0) wait_ok = mbar_wait(smem_u32(&mbar[s]), phase[s]);
-            __syncthreads();
-            if (!wait_ok) { ok = false; break; }
-            phase[s] ^= 1;
+        // copies of this K-step have landed (each thread waits for its own, the
+        // barrier makes everybody's visible)
+        switch (D) {   // all but the D-1 most recent groups complete
+        case 1: cp_async_wait<0>(); break;
+        case 2: cp_async_wait<1>(); break;
+        case 3: cp_async_wait<2>(); break;
+        case 4: cp_async_wait<3>(); break;
+        default: cp_async_wait<4>(); break;
         }
-        for (int q = 0; q < ov_k; ++q) {
-            // mutated channels: elements k = c * ch + j of this K-tile
-            const int j = ov_ids[q];
-            const int cfirst = k0 - j <= 0 ? 0 : (k0 - j + p.ov.ch - 1) / p.ov.ch;
-            for (int c = cfirst; c < p.ov.cells && c * p.ov.ch + j < k0 + kTileK; ++c) {
-                const float pv = p.ov.patch[row * p.ov.row_stride + q * p.ov.cells + c];
-#pragma unroll
-                for (int i = 0; i < kTileK; ++i)
-                    if (k0 + i == c * p.ov.ch + j) ac[i] = pv;
-            }
-        }
-#pragma unroll
-        for (int c = 0; c < kTileK / 4; ++c) {
-            float4 hi, lo;
-            hi.x = tf32_rna(ac[4 * c]);     lo.x = tf32_rna(ac[4 * c] - hi.x);
-            hi.y = tf32_rna(ac[4 * c + 1]); lo.y = tf32_rna(ac[4 * c + 1] - hi.y);
-            hi.z = tf32_rna(ac[4 * c + 2]); lo.z = tf32_rna(ac[4 * c + 2] - hi.z);
-            hi.w = tf32_rna(ac[4 * c + 3]); lo.w = tf32_rna(ac[4 * c + 3] - hi.w);
-            const uint32_t off = sw128_off(tid, c);
-            *reinterpret_cast<float4 *>(st + off) = hi;
-            *reinterpret_cast<float4 *>(st + a_bytes + off) = lo;
-        }
-        if (tid < Nt) {
+        __syncthreads();
+        // split this row's 32 values into TF32 halves (the mutated channels first)
+        {
+            float ac[kTileK];
 #pragma unroll
             for (int c = 0; c < kTileK / 4; ++c) {
+                const float4 v = *reinterpret_cast<const float4 *>(st + sw128_off(tid, c));
+                ac[4 * c] = v.x; ac[4 * c + 1] = v.y; ac[4 * c + 2] = v.z; ac[4 * c + 3] = v.w;
+            }
+            for (int q = 0; q < ri.ov_k; ++q) {
+                const int jn = ri.ov_ids[q];
+                if (DENSE) {
+                    const int cfirst = k0 - jn <= 0 ? 0 : (k0 - jn + p.ov.ch - 1) / p.ov.ch;
+                    for (int c = cfirst; c < p.ov.cells && c * p.ov.ch + jn < k0 + kTileK; ++c) {
+                        const float pv = p.ov.patch[ri.row * p.ov.row_stride + q * p.ov.cells + c];
+#pragma unroll
+                        for (int i = 0; i < kTileK; ++i)
+                            if (k0 + i == c * p.ov.ch + jn) ac[i] = pv;
+                    }
+                } else {
+                    int ci = k0 % p.ic, t = k0 / p.ic, kx = t % p.kw, ky = t / p.kw;
+#pragma unroll
+                    for (int i = 0; i < kTileK; ++i) {
+                        if (ci == jn && k0 + i < p.K) {
+                            const int iy = ri.oy * p.stride - p.pad + ky, ix = ri.ox * p.stride - p.pad + kx;
+                            if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw)
+                                ac[i] = p.ov.patch[ri.row * p.ov.row_stride + q * p.ov.cells + iy * p.iw + ix];
+                        }
+                        if (++ci == p.ic) { ci = 0; if (++kx == p.kw) { kx = 0; ++ky; } }
+                    }
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < kTileK / 4; ++c) {
+                float4 hi;
+                hi.x = tf32_rna(ac[4 * c]);
+                hi.y = tf32_rna(ac[4 * c + 1]);
+                hi.z = tf32_rna(ac[4 * c + 2]);
+                hi.w = tf32_rna(ac[4 * c + 3]);
                 const uint32_t off = sw128_off(tid, c);
-                *reinterpret_cast<float4 *>(st + 2 * a_bytes + off) = bhc[c];
-                *reinterpret_cast<float4 *>(st + 2 * a_bytes + b_bytes + off) = blc[c];
-            }
-        }
-        // rows 128..255 of a 256-wide B tile
-        for (int n = tid + kTileM; n < Nt; n += kTileM) {
-            const float4 *h = reinterpret_cast<const float4 *>(p.Whi + (int64_t)(n_base + n) * p.Kp + k0);
-            const float4 *l = reinterpret_cast<const float4 *>(p.Wlo + (int64_t)(n_base + n) * p.Kp + k0);
-#pragma unroll
-            for (int c = 0; c < kTileK / 4; ++c) {
-                const uint32_t off = sw128_off(n, c);
-                *reinterpret_cast<float4 *>(st + 2 * a_bytes + off) = __ldg(h + c);
-                *reinterpret_cast<float4 *>(st + 2 * a_bytes + b_bytes + off) = __ldg(l + c);
+                *reinterpret_cast<float4 *>(st + off) = hi;
+                if (THREE) {
+                    const float4 lo = make_float4(tf32_rna(ac[4 * c] - hi.x), tf32_rna(ac[4 * c + 1] - hi.y),
+                                                  tf32_rna(ac[4 * c + 2] - hi.z), tf32_rna(ac[4 * c + 3] - hi.w));
+                    *reinterpret_cast<float4 *>(st + a_bytes + off) = lo;
+                }
             }
         }
         // make the generic-proxy stores visible to the tensor core, then issue
@@ -274,67 +373,104 @@ __global__ void __launch_bounds__(128, 1) k_tc_dense(const TcDenseParams p, int 
         __syncthreads();
         if (tid == 0) {
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t sa = smem_u32(st), sal = sa + a_bytes, sb = sa + 2 * a_bytes, sbl = sb + b_bytes;
+            const uint32_t sa = smem_u32(st), sal = sa + a_bytes, sb = sa + b_off, sbl = sb + b_bytes;
             const uint32_t id = idesc_tf32(kTileM, Nt);
 #pragma unroll
             for (int ks = 0; ks < kTileK / 8; ++ks) {
                 const uint32_t adv = ks * 32;   // 8 TF32 values = 32 bytes along K
-                const uint32_t acc0 = (kt > 0 || ks > 0) ? 1u : 0u;
-                mma_tf32(tmem, sw128_desc(sal + adv), sw128_desc(sb + adv), id, acc0);   // a_lo * b_hi
-                mma_tf32(tmem, sw128_desc(sa + adv), sw128_desc(sbl + adv), id, 1u);     // a_hi * b_lo
-                mma_tf32(tmem, sw128_desc(sa + adv), sw128_desc(sb + adv), id, 1u);      // a_hi * b_hi
+                const uint32_t first = (kt > 0 || ks > 0) ? 1u : 0u;
+                if (THREE) {
+                    mma_tf32(tmem, sw128_desc(sal + adv), sw128_desc(sb + adv), id, first);   // a_lo * b_hi
+                    mma_tf32(tmem, sw128_desc(sa + adv), sw128_desc(sbl + adv), id, 1u);      // a_hi * b_lo
+                    mma_tf32(tmem, sw128_desc(sa + adv), sw128_desc(sb + adv), id, 1u);       // a_hi * b_hi
+                } else {
+                    mma_tf32(tmem, sw128_desc(sa + adv), sw128_desc(sb + adv), id, first);    // a_hi * b_hi
+                }
             }
             mma_commit(smem_u32(&mbar[s]));
+            ++issued[s];
         }
-    }
-    // wait for the outstanding commits (the last one covers every MMA issued)
-    if (ok) {
-        if (tid == 0) {
-            int good = 1;
-            for (int kt = max(0, nK - kStages); kt < nK && good; ++kt) {
-                const int s = kt % kStages;
-                good = mbar_wait(smem_u32(&mbar[s]), phase[s]);
+        // refill the stage the previous K-step's MMAs read, D steps ahead
+        if (it + D < total) {
+            if (tid == 0) wait_ok = wait_stage((int)((it + D) % S));
+            __syncthreads();
+            if (!wait_ok) { ok = false; break; }
+            issue(it + D);
+        }
+        cp_async_commit();
+        if (kt == nK - 1) {
+            // the tile's accumulator is complete once its last commit has arrived
+            if (tid == 0) wait_ok = wait_stage(s);
+            __syncthreads();
+            if (!wait_ok) { ok = false; break; }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            // epilogue: thread = GEMM row = TMEM lane (warp w holds lanes 32w .. 32w+31)
+            const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+            const float *srow = nullptr;
+            if (p.has_add && ri.ok) srow = p.skip + (p.skip_per_input ? p.t0 + ri.row % p.T : ri.row) * p.skip_stride;
+            float *yrow = ri.ok ? p.y + ri.row * p.y_stride : nullptr;
+            for (int n0 = 0; n0 < Nt; n0 += 16) {
+                float v[16];
+                tmem_ld16(lane_base + n0, v);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int n = n_base + n0 + i;
+                    const float zz = (ri.ok && n < p.N) ? v[i] + __ldg(p.b + n) : 0.f;
+                    if (p.z && ri.ok && n < p.N) {
+                        if (DENSE) p.z[ri.row * p.z_stride + n] = zz;
+                        else p.z[ri.row * p.z_stride + (int64_t)n * (p.oh * p.ow) + ri.oy * p.ow + ri.ox] = zz;
+                    }
+                    float val = act_apply(p.act1, zz);
+                    if (!DENSE && p.has_add && ri.ok && n < p.N) {
+                        const float sv = n < p.sk_c
+                            ? srow[((int64_t)ri.oy * p.sk_stride * p.sk_w + ri.ox * p.sk_stride) * p.sk_c + n]
+                            : 0.f;
+                        val = act_apply(p.act2, val + sv);
+                    }
+                    v[i] = val;
+                }
+                if (!DENSE && p.pool) {
+                    // lanes 4w .. 4w+3 hold the four positions of one pooling window
+                    const int lane = tid & 31;
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const float w1 = __shfl_down_sync(0xffffffffu, v[i], 1);
+                        const float w2 = __shfl_down_sync(0xffffffffu, v[i], 2);
+                        const float w3 = __shfl_down_sync(0xffffffffu, v[i], 3);
+                        if ((lane & 3) == 0) v[i] = max4_first(v[i], w1, w2, w3);
+                    }
+                    if (ri.ok && (lane & 3) == 0) {
+                        float *yo = yrow + ((int64_t)ri.py * p.pw + ri.px) * p.N;
+#pragma unroll
+                        for (int i = 0; i < 16; ++i)
+                            if (n_base + n0 + i < p.N) yo[n_base + n0 + i] = v[i];
+                    }
+                } else if (ri.ok) {
+                    float *yo = yrow + (DENSE ? 0 : ((int64_t)ri.oy * p.ow + ri.ox) * p.N);
+                    const int nb = n_base + n0;
+                    if (nb + 15 < p.N && ((p.N & 3) == 0)) {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c)
+                            *reinterpret_cast<float4 *>(yo + nb + 4 * c) =
+                                make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i)
+                            if (nb + i < p.N) yo[nb + i] = v[i];
+                    }
+                }
             }
-            wait_ok = good;
+            // the next tile's first MMA overwrites the accumulator only after every
+            // thread's reads (the barrier at the top of the next K-step)
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         }
-        __syncthreads();
-        ok = wait_ok != 0;
     }
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    cp_async_wait<0>();
     if (!ok) {
         if (tid == 0) {
             atomicExch(p.err, MURE_ERR_TIMEOUT);
             // a bounded chance for the tensor core to finish before the memory goes
-            const int last = nK - 1;
-            if (last >= 0) mbar_wait(smem_u32(&mbar[last % kStages]), phase[last % kStages]);
-        }
-    } else {
-        // epilogue: thread = row = TMEM lane (warp w holds lanes 32w .. 32w+31)
-        const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-        for (int n0 = 0; n0 < Nt; n0 += 16) {
-            float v[16];
-            tmem_ld16(lane_base + n0, v);
-            if (row_ok) {
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    const int n = n_base + n0 + 4 * c;
-                    float zz[4], yy[4];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        zz[i] = n + i < p.N ? v[4 * c + i] + __ldg(p.b + n + i) : 0.f;
-                        yy[i] = act_apply(p.act, zz[i]);
-                    }
-                    if (n + 3 < p.N) {
-                        if (p.z) *reinterpret_cast<float4 *>(p.z + row * p.z_stride + n) = make_float4(zz[0], zz[1], zz[2], zz[3]);
-                        *reinterpret_cast<float4 *>(p.y + row * p.y_stride + n) = make_float4(yy[0], yy[1], yy[2], yy[3]);
-                    } else {
-                        for (int i = 0; i < 4 && n + i < p.N; ++i) {
-                            if (p.z) p.z[row * p.z_stride + n + i] = zz[i];
-                            p.y[row * p.y_stride + n + i] = yy[i];
-                        }
-                    }
-                }
-            }
+            for (int s = 0; s < S; ++s) wait_stage(s);
         }
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -354,9 +490,13 @@ __global__ void k_split_weights(const float *__restrict__ W, int N, int K, int N
     lo[i] = tf32_rna(w - h);
 }
 
-int tc_dense_supported(const Stage &S)
+int tc_supported(const Stage &S)
 {
-    return S.kind == MURE_NODE_DENSE && S.oc >= 16 && !S.has_add && !S.pool && !S.gap;
+    if (S.oc < 16) return 0;
+    if (S.kind == MURE_NODE_DENSE) return !S.has_add && !S.pool && !S.gap;
+    // implicit-GEMM convolution: pooled maps need whole windows per warp (always true:
+    // a window is 4 consecutive GEMM rows and tiles start at multiples of 128)
+    return S.kind == MURE_NODE_CONV2D;
 }
 
 int launch_split_weights(const Stage &S, float *hi, float *lo, cudaStream_t s)
@@ -367,27 +507,53 @@ int launch_split_weights(const Stage &S, float *hi, float *lo, cudaStream_t s)
     return 1;
 }
 
-int launch_tc_dense(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, float *y_out, int64_t y_stride,
-                    cudaStream_t s, const Overlay *ov)
+int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
+              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov)
 {
     if (rm.R <= 0) return 0;
-    TcDenseParams p{};
+    TcParams p{};
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
     p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
+    p.dense = S.kind == MURE_NODE_DENSE;
+    p.ih = S.ih; p.iw = S.iw; p.ic = S.ic; p.kh = S.kh; p.kw = S.kw; p.stride = S.stride; p.pad = S.pad;
+    p.oh = S.oh; p.ow = S.ow;
+    p.pool = S.pool; p.pw = S.ow / 2;
+    p.P = p.dense ? 1 : (S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : S.oh * S.ow);
     p.K = S.K; p.Kp = round_up32(S.K); p.N = S.oc; p.Np = round_up16(S.oc);
-    p.Whi = S.Wtc_hi; p.Wlo = S.Wtc_lo; p.b = S.b; p.act = S.act1;
+    p.Whi = S.Wtc_hi; p.Wlo = S.Wtc_lo; p.b = S.b;
+    p.act1 = S.act1; p.has_add = S.has_add; p.act2 = S.act2;
+    p.skip = skip.p; p.skip_stride = skip.stride; p.skip_per_input = skip.per_input;
+    p.sk_w = S.sk_w; p.sk_c = S.sc_c; p.sk_stride = S.sc_stride;
     p.z = z_out; p.z_stride = z_stride;
-    p.y = y_out; p.y_stride = y_stride;
+    // with global average pooling the post-op map goes to gap_tmp first
+    const int mh = S.pool ? S.oh / 2 : S.oh, mw = S.pool ? S.ow / 2 : S.ow;
+    const int64_t map_stride = round4((int64_t)mh * mw * S.oc);
+    p.y = S.gap ? gap_tmp : y_out;
+    p.y_stride = S.gap ? map_stride : y_stride;
+    p.three = S.tc == 1;
     if (ov) p.ov = *ov;
     p.err = S.err;
     const int nt = std::min(256, p.Np);
     int ncols = 32;
     while (ncols < nt) ncols <<= 1;
-    const size_t smem = 1024 + (size_t)kStages * (2 * kTileM * 128 + 2 * nt * 128);
-    cudaFuncSetAttribute(k_tc_dense, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    const dim3 grid((unsigned)((rm.R + kTileM - 1) / kTileM), (unsigned)((p.Np + 255) / 256));
-    k_tc_dense<<<grid, kTileM, smem, s>>>(p, ncols);
-    return 1;
+    const size_t stage = p.three ? (2 * kTileM * 128 + 2 * nt * 128) : (kTileM * 128 + nt * 128);
+    const int n_stages = (int)std::min<size_t>(6, (220 * 1024 - 1024) / stage);   // 2 .. 6 stages
+    const size_t smem = 1024 + (size_t)n_stages * stage;
+    const int64_t M = (int64_t)rm.R * p.P;
+    const int64_t tiles = (M + kTileM - 1) / kTileM;
+    // persistent CTAs: one per SM (per N slice), each looping over M-tiles
+    const int n_sm = 152;
+    const int ny = (p.Np + 255) / 256;
+    const dim3 grid((unsigned)std::max<int64_t>(1, std::min<int64_t>(tiles, std::max(1, n_sm / ny))), (unsigned)ny);
+    auto go = [&](auto kern) {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        kern<<<grid, kTileM, smem, s>>>(p, ncols, n_stages);
+    };
+    if (p.dense) { if (p.three) go(k_tc_gemm<true, true>); else go(k_tc_gemm<true, false>); }
+    else { if (p.three) go(k_tc_gemm<false, true>); else go(k_tc_gemm<false, false>); }
+    int launches = 1;
+    if (S.gap) launches += launch_gap(gap_tmp, map_stride, mh * mw, S.oc, rm.R, y_out, y_stride, s);
+    return launches;
 }
 
 }  // namespace mure

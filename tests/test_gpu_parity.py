@@ -284,3 +284,37 @@ def test_kernel_variants_agree_bitwise(M, ctx, monkeypatch):
     assert np.array_equal(r1["kill_bits"], r2["kill_bits"])
     v1 = M.mure_eval_vanilla(fast, w.X, table, logits=True)
     assert np.array_equal(v1["logits"].view(np.uint32), r1["logits"].view(np.uint32))
+
+
+@pytest.mark.parametrize("name", list(CASES))
+def test_tf32_variant_verdicts(M, ctx, oracle_runs, name):
+    """The reduced-precision variant (one TF32 product per MAC on the tensor cores):
+    memoized == vanilla bit for bit, and its kill verdicts agree with the fp32 oracle
+    on nearly every (mutant, input) pair; the agreement rate is what is reported."""
+    w, table, ora = oracle_runs(name)
+    model = M.mure_model_load(ctx, w.model, precision="tf32")
+    cache = M.mure_build_prefix_cache(model, w.X)
+    memo = M.mure_eval_mutants(cache, table, logits=True)
+    van = M.mure_eval_vanilla(model, w.X, table, logits=True)
+    assert np.array_equal(memo["kill_bits"], van["kill_bits"])
+    assert np.array_equal(memo["logits"].view(np.uint32), van["logits"].view(np.uint32))
+    agree = (bits(memo["kill_bits"], len(w.X)) == bits(ora["kill_bits"], len(w.X))).mean()
+    assert agree >= 0.98, agree
+
+
+def test_tensor_core_conv_on_small_layers(M, ctx, oracle_mod, monkeypatch):
+    """The implicit-GEMM tensor-core convolution also runs LeNet's conv 6->16 (when
+    forced) within the fp32 tolerance of the oracle."""
+    w = wl.workload("lenet5", 130, 1)
+    table = all_ops(w.model, 6, seed=51)
+    ora = oracle_mod.vanilla(w.model, w.X, table)
+    monkeypatch.setenv("MURE_TC_CONV", "1")
+    model = M.mure_model_load(ctx, w.model, precision="tf32x3")
+    monkeypatch.delenv("MURE_TC_CONV")
+    r = M.mure_eval_mutants(M.mure_build_prefix_cache(model, w.X), table, logits=True)
+    ok, worst = logits_close(r["logits"], ora["logits"])
+    assert ok, worst
+    bad, _ = compare_kills(r["kill_bits"], ora["kill_bits"], ora["orig_logits"], ora["logits"], len(w.X))
+    assert bad == 0
+    v = M.mure_eval_vanilla(model, w.X, table, logits=True)
+    assert np.array_equal(v["logits"].view(np.uint32), r["logits"].view(np.uint32))
