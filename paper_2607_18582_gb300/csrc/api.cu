@@ -647,7 +647,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     const Stage &Sn = m->st[l + 1];
     bool skip_reader = false;
     for (int v = l + 2; v < L; ++v) skip_reader |= m->st[v].has_add && m->st[v].skip_src == l + 1;
-    if (Sn.tc && !skip_reader) {
+    if (Sn.tc && !skip_reader && tc_overlay_inline(Sn, ov)) {
         timed(l + 1, 2 * Sn.macs * rm.R, [&] {
             return launch_tc(Sn, base, rm, nullptr, 0, skip_of(Sn), ws.xb[l + 2], m->xd[l + 2].stride, ws.gap_tmp, s,
                              &ov);
@@ -767,7 +767,8 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         CK(c, cudaGetLastError());
         if (dev_err) {
             CK(c, cudaMemset(c->err_dev, 0, sizeof(int)));
-            FAILIF(true, c, MURE_ERR_TIMEOUT, "a device-side wait gave up (code %d)", dev_err);
+            FAILIF(true, c, dev_err == MURE_ERR_TIMEOUT ? MURE_ERR_TIMEOUT : MURE_ERR_UNSUPPORTED,
+                   "a device-side check failed (code %d)", dev_err);
         }
         sA = (double)host_cnt[0] / (double)n;
         sB = ca->n_label_values > 0 ? (double)host_cnt[1] / ((double)n * ca->n_label_values) : 0.0;
@@ -1004,10 +1005,8 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             CK(c, cudaMemcpyAsync(S.b, n.b, S.oc * 4, cudaMemcpyHostToDevice, c->stream));
             CK(c, cudaStreamSynchronize(c->stream));  // Wt is reused
             if (S.tc) {
-                const int64_t np = (int64_t)round_up16(S.oc) * round_up32(S.K);
-                S.Wtc_hi = (float *)dalloc(c, np * 4);
-                S.Wtc_lo = (float *)dalloc(c, np * 4);
-                c->launches += launch_split_weights(S, S.Wtc_hi, S.Wtc_lo, c->stream);
+                S.Wtc = (float *)dalloc(c, tc_weight_floats(S) * 4);
+                c->launches += launch_swizzle_weights(S, S.Wtc, c->stream);
                 check_launch(c);
             }
         }
@@ -1041,8 +1040,7 @@ void mure_model_free(mure_model *m)
         dfree(m->ctx, S.W);
         dfree(m->ctx, S.Wt);
         dfree(m->ctx, S.b);
-        dfree(m->ctx, S.Wtc_hi);
-        dfree(m->ctx, S.Wtc_lo);
+        dfree(m->ctx, S.Wtc);
     }
     dfree(m->ctx, m->sigma_dev);
     cudaStreamSynchronize(m->ctx->stream);

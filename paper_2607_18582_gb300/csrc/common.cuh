@@ -33,8 +33,7 @@ struct Stage {
     int64_t macs;             // multiply-accumulates per row
     int variant = 0;          // 0: implicit-GEMM kernel; > 0: a shared-memory direct conv
     int tc = 0;               // tensor-core kernel: 1 = 3xTF32, 2 = one TF32 MMA (variant)
-    float *Wtc_hi = nullptr;  // tc: TF32 halves of W, zero-padded [round16(oc)][round32(K)]
-    float *Wtc_lo = nullptr;
+    float *Wtc = nullptr;     // tc: TF32 halves of W in the tensor-core operand layout
     int *err = nullptr;       // device error word of the context (bounded waits)
     float *W = nullptr;       // device [oc][K]
     float *Wt = nullptr;      // device [K][oc] (the same weights, K-major rows)
@@ -135,7 +134,9 @@ int launch_conv_small(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
 // mode): which layers the kernel takes, the weight split done at model load, and the
 // launcher (arguments as for the stage kernel, plus the overlay).
 int tc_supported(const Stage &S);
-int launch_split_weights(const Stage &S, float *hi, float *lo, cudaStream_t s);
+int64_t tc_weight_floats(const Stage &S);
+int tc_overlay_inline(const Stage &S, const Overlay &ov);
+int launch_swizzle_weights(const Stage &S, float *out, cudaStream_t s);
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
               int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov = nullptr);
 

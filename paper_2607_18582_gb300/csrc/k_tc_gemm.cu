@@ -1,0 +1,767 @@
+// Dense and convolution layers on the 5th-generation tensor cores (tcgen05) with
+// fp32-level accuracy: every fp32 operand a is split into two TF32 halves, a = a_hi +
+// a_lo (a_hi = a rounded to TF32, a_lo = the rounded remainder), and each product
+// uses three MMAs, a_lo*b_hi + a_hi*b_lo + a_hi*b_hi, accumulated in fp32 in tensor
+// memory.  (The reduced-precision variant uses a_hi*b_hi alone.)
+//
+// The GEMM: M = (batch row, output position) pairs, K = the fan-in (ky, kx, ci), N =
+// output channels (a CTA takes a slice of <= 128).  A convolution is an implicit
+// GEMM: the producers gather the im2col rows from the NHWC input.  The CTA is
+// persistent (one per SM) and warp-specialised:
+//   warps 0-3  producers: thread = GEMM row = tensor-memory lane.  Each streams its
+//              row's 32-value K-steps into a private shared-memory ring with
+//              cp.async, several steps ahead (the first suffix stage's mutated
+//              channels are fetched from the patch buffer instead of the cached row),
+//              splits them into TF32 halves and stores the halves into a tensor-memory
+//              A stage (tcgen05.st); the MMA reads A from tensor memory, so the
+//              operand never goes through shared memory a second time;
+//   warp 8     one thread issues the MMAs (kind::tf32, M=128, K=8) and commits them
+//              to the stage barriers;
+//   warp 9     one thread moves the weights: pre-split, pre-swizzled K-step chunks
+//              (one bulk copy each), or the whole slice once when it fits;
+//   warps 4-7  epilogue: two accumulators alternate, so the bias / activation /
+//              residual / 2x2 pool / store of tile i overlaps the MMAs of tile i+1.
+// The K order of the accumulation is fixed and independent of the row's position in
+// the tile, so a row gives the same bits in every batch (memoized == vanilla).
+// Every wait is bounded; on expiry the kernel records an error code, stops every
+// role, lets its own copies and MMAs drain (bounded), frees its tensor memory and
+// returns.
+#include <algorithm>
+
+#include "common.cuh"
+#include "device_util.cuh"
+
+namespace mure {
+
+namespace {
+
+constexpr int kTileM = 128;
+constexpr int kTileK = 32;             // fp32 / tf32 values per 128-byte row
+constexpr int kNA = 4;                 // producer cp.async ring depth (K-steps)
+constexpr int kNB = 4;                 // streamed weight stages
+constexpr int kSlice = 128;            // output channels per CTA
+constexpr int kThreads = 320;          // 4 producer + 4 epilogue + MMA + weight warps
+constexpr int kAccCol = 0;             // two accumulators at columns 0 and 128
+constexpr int kACol = 256;             // A stages from column 256
+constexpr uint32_t kStageA = kTileM * 128;   // bytes of one producer ring slot
+constexpr long long kSpin = 2000000000LL;    // about a second at the SM clock
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ float tf32_rna(float x)
+{
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+    return __uint_as_float(r);
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row groups
+// 1024 bytes apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFF);          // start address
+    d |= (uint64_t)1 << 16;                          // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024 >> 4) << 32;                // stride byte offset: next 8-row group
+    d |= (uint64_t)1 << 46;                          // descriptor version
+    d |= (uint64_t)2 << 61;                          // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor, kind::tf32: D fp32, A and B tf32, both K-major, M x N.
+__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N)
+{
+    return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// Byte offset of 16-byte chunk `chunk` of row r in a 128-byte-swizzled K-major tile.
+__host__ __device__ __forceinline__ uint32_t sw128_off(int r, int chunk)
+{
+    return (uint32_t)(r * 128 + ((chunk ^ (r & 7)) << 4));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t a)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(a), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// The same with a suspend-time hint: a waiting thread sleeps until the phase
+// completes (or the hint expires) instead of taking issue slots from the producers.
+__device__ __forceinline__ bool mbar_try_sleep(uint32_t a, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(a), "r"(parity), "r"(20000u)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase of parity `parity`; false when another role has aborted or
+// about a second has passed (then this role aborts the CTA).
+template <bool SLEEP = false>
+__device__ __forceinline__ bool wait_phase(uint32_t a, uint32_t parity, volatile int *abort_flag)
+{
+    if (mbar_try(a, parity)) return true;
+    const long long t0 = clock64();
+    for (;;) {
+        if (SLEEP ? mbar_try_sleep(a, parity) : mbar_try(a, parity)) return true;
+        if (*abort_flag) return false;
+        if (clock64() - t0 > kSpin) { *abort_flag = 1; return false; }
+    }
+}
+
+// The same for a whole warp: every lane polls, the verdict is the warp's AND, so the
+// .sync.aligned tensor-memory instructions that follow see a converged warp.
+template <bool SLEEP = false>
+__device__ __forceinline__ bool warp_wait_phase(uint32_t a, uint32_t parity, volatile int *abort_flag)
+{
+    const bool ok = wait_phase<SLEEP>(a, parity, abort_flag);
+    return __all_sync(0xffffffffu, ok);
+}
+
+// Teardown wait: bounded, ignores the abort flag.
+__device__ __forceinline__ void wait_phase_drain(uint32_t a, uint32_t parity)
+{
+    const long long t0 = clock64();
+    while (!mbar_try(a, parity))
+        if (clock64() - t0 > kSpin) return;
+}
+
+// A from tensor memory, B from shared memory.
+__device__ __forceinline__ void mma_tf32_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc)
+{
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc));
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t mbar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t mbar)
+{
+    asm volatile("cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(mbar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float *v)
+{
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Thread t's 32 values go to lane (warp quadrant) t, columns taddr .. taddr+31.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float *v)
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+        "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+        "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+        "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+        "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+        "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+        "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+        "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+        "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+        "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+        "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+        : "memory");
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, int src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void *src, int src_bytes)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+}  // namespace
+
+struct TcParams {
+    const float *x; int64_t x_stride; int x_per_input;
+    int64_t t0; int T; int R;
+    int ih, iw, ic, kh, kw, stride, pad, oh, ow;
+    int P, pool, pw;             // GEMM rows per batch row (pooled maps: window-major)
+    int K, Kp, N, Np;            // fan-in (padded to 32), outputs (padded to 16)
+    const float *Wsw;            // pre-split, pre-swizzled weight chunks (see k_swizzle_weights)
+    int64_t w_slice_floats;      // distance between the N slices' chunk sequences
+    int b_resident;              // 1: the CTA's whole weight slice sits in shared memory
+    const float *b;
+    int act1, has_add, act2;
+    const float *skip; int64_t skip_stride; int skip_per_input; int sk_w, sk_c, sk_stride;
+    float *z; int64_t z_stride;
+    float *y; int64_t y_stride;
+    Overlay ov;                  // mutated channels of the input rows (ov.patch null: none)
+    int *err;
+};
+
+// Per producer ring slot, the overlay values of a row's K-step: up to kOvMax
+// (position, value) entries, the values fetched by cp.async into ov_val.
+constexpr int kOvMax = 8;
+constexpr uint32_t kOvSlotBytes = kTileM * (kOvMax * 4 + kOvMax + 4);   // values, positions, count
+
+// One GEMM row of an M-tile: batch row, output position, input row, overlay.
+struct RowInfo {
+    int64_t row;
+    int oy, ox, py, px;
+    const float *xrow;
+    int ov_k;
+    const int32_t *ov_ids;
+    const float *ov_patch;
+    int ov_pos[4], ov_c[4];   // dense overlay walk: next position j + c * ch of slots 0..3
+    bool ok;
+};
+
+template <bool DENSE, bool OVERLAY = true>
+__device__ __forceinline__ RowInfo row_info(const TcParams &p, int64_t m)
+{
+    RowInfo ri{};
+    ri.ok = m < (int64_t)p.R * p.P;
+    if (!ri.ok) return ri;
+    if (DENSE) {
+        ri.row = m;
+    } else {
+        ri.row = m / p.P;
+        const int q = (int)(m - ri.row * p.P);
+        if (p.pool) {
+            const int w = q >> 2, sub = q & 3;
+            ri.py = w / p.pw; ri.px = w % p.pw;
+            ri.oy = 2 * ri.py + (sub >> 1);
+            ri.ox = 2 * ri.px + (sub & 1);
+        } else {
+            ri.oy = q / p.ow;
+            ri.ox = q % p.ow;
+        }
+    }
+    ri.xrow = p.x + (p.x_per_input ? p.t0 + ri.row % p.T : ri.row) * p.x_stride;
+    if (OVERLAY && p.ov.patch) {
+        const int g = (int)(ri.row / p.T);
+        ri.ov_k = p.ov.n_neurons[g];
+        ri.ov_ids = p.ov.ids + p.ov.neuron_off[g];
+        ri.ov_patch = p.ov.patch + ri.row * p.ov.row_stride;
+        if (DENSE) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                ri.ov_c[q] = 0;
+                ri.ov_pos[q] = q < ri.ov_k ? ri.ov_ids[q] : 0;
+            }
+        }
+    }
+    return ri;
+}
+
+// Queue the cp.async copies of K-step k0 .. k0+31 of GEMM row `pf` into the 128-byte
+// row `slot` (swizzled like the MMA operand layout, so the read-back is free of bank
+// conflicts).  Values past the fan-in, outside the image (zero padding) or of rows
+// past the end are zero-filled.  The mutated channels of the first suffix stage:
+// their patch values are fetched into the slot's overlay entries (ov), written over
+// the staged row once it has landed.
+template <bool DENSE>
+__device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, int r, uint32_t slot, uint32_t ov,
+                                              int k0)
+{
+    const float *dummy = p.b;   // a valid address for zero-byte copies
+    int cnt = 0;
+    auto entry = [&](int pos, const float *src) {
+        if (cnt < kOvMax) {
+            cp_async4(ov + (uint32_t)(cnt * kTileM + r) * 4, src, 4);
+            asm volatile("st.shared.u8 [%0], %1;" ::"r"(ov + kTileM * kOvMax * 4 + cnt * kTileM + r), "r"(pos));
+        } else {
+            atomicExch(p.err, MURE_ERR_UNSUPPORTED);   // the host keeps the entry count in range
+        }
+        ++cnt;
+    };
+    if (DENSE) {
+        // overlay positions are c * ch + j (cell c of mutated channel j); the K-steps of a
+        // row come in ascending k, so each slot keeps a cursor
+        const int nq = min(pf.ov_k, 4);
+#pragma unroll
+        for (int c = 0; c < kTileK / 4; ++c) {
+            const int kk = k0 + 4 * c;
+            const int nb = pf.ok ? max(0, min(16, (p.K - kk) * 4)) : 0;
+            cp_async16(slot + sw128_off(r, c), nb ? (const void *)(pf.xrow + kk) : (const void *)dummy, nb);
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            if (q >= nq) break;
+            while (pf.ov_c[q] < p.ov.cells && pf.ov_pos[q] < k0 + kTileK) {
+                entry(pf.ov_pos[q] - k0, pf.ov_patch + q * p.ov.cells + pf.ov_c[q]);
+                pf.ov_pos[q] += p.ov.ch;
+                ++pf.ov_c[q];
+            }
+        }
+    } else if ((p.ic & 3) == 0) {
+        // 16-byte chunks: 4 channels of one input pixel
+        int ci = k0 % p.ic, t = k0 / p.ic, kx = t % p.kw, ky = t / p.kw;
+#pragma unroll
+        for (int c = 0; c < kTileK / 4; ++c) {
+            const int kk = k0 + 4 * c;
+            const int iy = pf.oy * p.stride - p.pad + ky, ix = pf.ox * p.stride - p.pad + kx;
+            const bool in = pf.ok && kk < p.K && (unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw;
+            cp_async16(slot + sw128_off(r, c), in ? pf.xrow + ((int64_t)iy * p.iw + ix) * p.ic + ci : dummy,
+                       in ? 16 : 0);
+            if (in)
+                for (int q = 0; q < pf.ov_k; ++q) {
+                    const int jn = pf.ov_ids[q];
+                    if (jn >= ci && jn < ci + 4) entry(4 * c + jn - ci, pf.ov_patch + q * p.ov.cells + iy * p.iw + ix);
+                }
+            ci += 4;
+            if (ci == p.ic) { ci = 0; if (++kx == p.kw) { kx = 0; ++ky; } }
+        }
+    } else {
+        // channel counts that are not a multiple of 4: 4-byte copies, the patch value
+        // taken directly for a mutated channel
+        int ci = k0 % p.ic, t = k0 / p.ic, kx = t % p.kw, ky = t / p.kw;
+        for (int i = 0; i < kTileK; ++i) {
+            const int k = k0 + i;
+            const int iy = pf.oy * p.stride - p.pad + ky, ix = pf.ox * p.stride - p.pad + kx;
+            const bool in = pf.ok && k < p.K && (unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw;
+            const float *src = in ? pf.xrow + ((int64_t)iy * p.iw + ix) * p.ic + ci : dummy;
+            if (in)
+                for (int q = 0; q < pf.ov_k; ++q)
+                    if (pf.ov_ids[q] == ci) src = pf.ov_patch + q * p.ov.cells + iy * p.iw + ix;
+            cp_async4(slot + sw128_off(r, i >> 2) + 4 * (i & 3), src, in ? 4 : 0);
+            if (++ci == p.ic) { ci = 0; if (++kx == p.kw) { kx = 0; ++ky; } }
+        }
+    }
+    if (p.ov.patch) asm volatile("st.shared.u8 [%0], %1;" ::"r"(ov + kTileM * kOvMax * 5 + r), "r"(min(cnt, kOvMax)));
+}
+
+// DENSE: one GEMM row per batch row; THREE: 3xTF32 (else one TF32 product).
+template <bool DENSE, bool THREE>
+__global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
+{
+    constexpr int kNT = THREE ? 4 : 8;             // tensor-memory A stages
+    constexpr int kAColsPerStage = THREE ? 64 : 32;
+    extern __shared__ __align__(1024) unsigned char smraw[];
+    __shared__ __align__(8) uint64_t bar_afull[kNT], bar_aempty[kNT], bar_bfull[kNB], bar_bempty[kNB];
+    __shared__ __align__(8) uint64_t bar_accfull[2], bar_accempty[2], bar_drain;
+    __shared__ uint32_t tmem_sh;
+    __shared__ int abort_sh;
+    __shared__ float bias_sh[kSlice];
+    volatile int *abort_flag = &abort_sh;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t sbase = (smem_u32(smraw) + 1023u) & ~1023u;
+    const int n_base = blockIdx.y * kSlice;
+    const int Nt = min(kSlice, p.Np - n_base);              // a multiple of 16
+    constexpr int planes = THREE ? 2 : 1;
+    const uint32_t b_step = (uint32_t)(planes * Nt * 128);  // one K-step of the weight slice
+    const int nK = p.Kp / kTileK;
+    const uint32_t b_region = sbase;
+    const uint32_t a_region = sbase + (p.b_resident ? (uint32_t)nK * b_step : (uint32_t)kNB * b_step);
+    const uint32_t ov_region = a_region + kNA * kStageA;    // kNA overlay slots (with an overlay)
+    const int64_t M = (int64_t)p.R * p.P;
+    const int64_t n_tiles = (M + kTileM - 1) / kTileM;
+    const int64_t my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+    const int64_t total = my_tiles * nK;
+    const float *wslice = p.Wsw + (int64_t)blockIdx.y * p.w_slice_floats;
+
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_sh)),
+                     "r"(512));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    for (int n = threadIdx.x; n < kSlice; n += kThreads) bias_sh[n] = n_base + n < p.N ? p.b[n_base + n] : 0.f;
+    if (threadIdx.x == 32) {
+        for (int s = 0; s < kNT; ++s) { mbar_init(smem_u32(&bar_afull[s]), 4); mbar_init(smem_u32(&bar_aempty[s]), 1); }
+        for (int s = 0; s < kNB; ++s) { mbar_init(smem_u32(&bar_bfull[s]), 1); mbar_init(smem_u32(&bar_bempty[s]), 1); }
+        for (int s = 0; s < 2; ++s) { mbar_init(smem_u32(&bar_accfull[s]), 1); mbar_init(smem_u32(&bar_accempty[s]), 4); }
+        mbar_init(smem_u32(&bar_drain), 1);
+        abort_sh = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tmem_sh;
+
+    if (warp < 4) {
+        // ------------------------------------------------------------ producers --
+        const int r = threadIdx.x;                        // GEMM row in the tile = TMEM lane
+        const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+        // issue cursor (tile i, K-tile kt, ring slot) runs kNA - 1 steps ahead
+        RowInfo pf{};
+        int64_t iss_i = 0, issued = 0;
+        int iss_kt = 0, iss_slot = 0;
+        auto issue_next = [&]() {
+            if (iss_kt == 0) pf = row_info<DENSE>(p, (blockIdx.x + iss_i * gridDim.x) * kTileM + r);
+            produce_issue<DENSE>(p, pf, r, a_region + (uint32_t)iss_slot * kStageA,
+                                 ov_region + (uint32_t)iss_slot * kOvSlotBytes, iss_kt * kTileK);
+            if (++iss_kt == nK) { iss_kt = 0; ++iss_i; }
+            if (++iss_slot == kNA) iss_slot = 0;
+            ++issued;
+        };
+        for (int s0 = 0; s0 < kNA - 1; ++s0) {
+            if (issued < total) issue_next();
+            cp_async_commit();
+        }
+        int slot_i = 0, t = 0;
+        uint32_t wraps = 0;                               // completed rounds of the A-stage ring
+        for (int64_t j = 0; j < total; ++j) {
+            if (issued < total) issue_next();
+            cp_async_commit();
+            cp_async_wait<kNA - 1>();                     // this thread's copies of step j
+            const uint32_t slot = a_region + (uint32_t)slot_i * kStageA;
+            if (p.ov.patch) {
+                // the row's overlay entries of this K-step, written over the landed copy
+                const uint32_t ov = ov_region + (uint32_t)slot_i * kOvSlotBytes;
+                uint32_t n;
+                asm volatile("ld.shared.u8 %0, [%1];" : "=r"(n) : "r"(ov + kTileM * kOvMax * 5 + r));
+                for (uint32_t e = 0; e < n; ++e) {
+                    uint32_t pos, val;
+                    asm volatile("ld.shared.u8 %0, [%1];" : "=r"(pos) : "r"(ov + kTileM * kOvMax * 4 + e * kTileM + r));
+                    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(val) : "r"(ov + (e * kTileM + r) * 4));
+                    asm volatile("st.shared.u32 [%0], %1;" ::"r"(slot + sw128_off(r, pos >> 2) + 4 * (pos & 3)), "r"(val)
+                                 : "memory");
+                }
+            }
+            if (++slot_i == kNA) slot_i = 0;
+            float hi[kTileK], lo[kTileK];
+#pragma unroll
+            for (int c = 0; c < kTileK / 4; ++c) {
+                float4 v;
+                asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                             : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                             : "r"(slot + sw128_off(r, c)));
+                hi[4 * c] = v.x; hi[4 * c + 1] = v.y; hi[4 * c + 2] = v.z; hi[4 * c + 3] = v.w;
+            }
+#pragma unroll
+            for (int i = 0; i < kTileK; ++i) {
+                const float h = tf32_rna(hi[i]);
+                if (THREE) lo[i] = tf32_rna(hi[i] - h);
+                hi[i] = h;
+            }
+            if (wraps >= 1 && !warp_wait_phase(smem_u32(&bar_aempty[t]), (wraps - 1) & 1, abort_flag)) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t ta = tmem + lane_off + kACol + t * kAColsPerStage;
+            tmem_st32(ta, hi);
+            if (THREE) tmem_st32(ta + 32, lo);
+            asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bar_afull[t]));
+            if (++t == kNT) { t = 0; ++wraps; }
+        }
+        cp_async_wait<0>();
+    } else if (warp < 8) {
+        // ------------------------------------------------------------- epilogue --
+        const int qd = warp & 3;
+        const uint32_t lane_off = (uint32_t)(qd * 32) << 16;
+        for (int64_t i = 0; i < my_tiles; ++i) {
+            const int a = (int)(i & 1);
+            if (!warp_wait_phase<true>(smem_u32(&bar_accfull[a]), (uint32_t)((i >> 1) & 1), abort_flag)) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const int64_t tile = blockIdx.x + i * gridDim.x;
+            const RowInfo ri = row_info<DENSE, false>(p, tile * kTileM + qd * 32 + lane);
+            const float *srow = nullptr;
+            if (p.has_add && ri.ok) srow = p.skip + (p.skip_per_input ? p.t0 + ri.row % p.T : ri.row) * p.skip_stride;
+            float *yrow = ri.ok ? p.y + ri.row * p.y_stride : nullptr;
+            for (int n0 = 0; n0 < Nt; n0 += 16) {
+                float v[16];
+                tmem_ld16(tmem + lane_off + kAccCol + a * 128 + n0, v);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int n = n_base + n0 + e;
+                    const float zz = (ri.ok && n < p.N) ? v[e] + bias_sh[n0 + e] : 0.f;
+                    if (p.z && ri.ok && n < p.N) {
+                        if (DENSE) p.z[ri.row * p.z_stride + n] = zz;
+                        else p.z[ri.row * p.z_stride + (int64_t)n * (p.oh * p.ow) + ri.oy * p.ow + ri.ox] = zz;
+                    }
+                    float val = act_apply(p.act1, zz);
+                    if (!DENSE && p.has_add && ri.ok && n < p.N) {
+                        const float sv = n < p.sk_c
+                            ? srow[((int64_t)ri.oy * p.sk_stride * p.sk_w + ri.ox * p.sk_stride) * p.sk_c + n]
+                            : 0.f;
+                        val = act_apply(p.act2, val + sv);
+                    }
+                    v[e] = val;
+                }
+                if (!DENSE && p.pool) {
+                    // lanes 4w .. 4w+3 hold the four positions of one pooling window
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const float w1 = __shfl_down_sync(0xffffffffu, v[e], 1);
+                        const float w2 = __shfl_down_sync(0xffffffffu, v[e], 2);
+                        const float w3 = __shfl_down_sync(0xffffffffu, v[e], 3);
+                        if ((lane & 3) == 0) v[e] = max4_first(v[e], w1, w2, w3);
+                    }
+                    if (ri.ok && (lane & 3) == 0) {
+                        float *yo = yrow + ((int64_t)ri.py * p.pw + ri.px) * p.N;
+#pragma unroll
+                        for (int e = 0; e < 16; ++e)
+                            if (n_base + n0 + e < p.N) yo[n_base + n0 + e] = v[e];
+                    }
+                } else if (ri.ok) {
+                    float *yo = yrow + (DENSE ? 0 : ((int64_t)ri.oy * p.ow + ri.ox) * p.N);
+                    const int nb = n_base + n0;
+                    if (nb + 15 < p.N && ((p.N & 3) == 0)) {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c)
+                            *reinterpret_cast<float4 *>(yo + nb + 4 * c) =
+                                make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e)
+                            if (nb + e < p.N) yo[nb + e] = v[e];
+                    }
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
+        }
+    } else if (warp == 8) {
+        // ------------------------------------------------------------------ MMA --
+        if (lane == 0) {
+            const uint32_t id = idesc_tf32(kTileM, Nt);
+            bool ok = true;
+            if (p.b_resident) ok = wait_phase(smem_u32(&bar_bfull[0]), 0, abort_flag);
+            int t = 0, sb = 0;
+            uint32_t t_wraps = 0, b_wraps = 0;
+            for (int64_t i = 0; ok && i < my_tiles; ++i) {
+                const int a = (int)(i & 1);
+                if (i >= 2 && !wait_phase(smem_u32(&bar_accempty[a]), (uint32_t)(((i >> 1) - 1) & 1), abort_flag)) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t d = tmem + kAccCol + a * 128;
+                for (int kt = 0; kt < nK; ++kt) {
+                    if (!wait_phase(smem_u32(&bar_afull[t]), t_wraps & 1, abort_flag)) { ok = false; break; }
+                    uint32_t bs;
+                    if (p.b_resident) {
+                        bs = b_region + (uint32_t)kt * b_step;
+                    } else {
+                        if (!wait_phase(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
+                        bs = b_region + (uint32_t)sb * b_step;
+                    }
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint32_t ta = tmem + kACol + t * kAColsPerStage;
+#pragma unroll
+                    for (int ks = 0; ks < kTileK / 8; ++ks) {
+                        const uint32_t first = (kt > 0 || ks > 0) ? 1u : 0u;
+                        const uint64_t bh = sw128_desc(bs + ks * 32);
+                        if (THREE) {
+                            const uint64_t bl = sw128_desc(bs + (uint32_t)Nt * 128 + ks * 32);
+                            mma_tf32_ts(d, ta + 32 + ks * 8, bh, id, first);   // a_lo * b_hi
+                            mma_tf32_ts(d, ta + ks * 8, bl, id, 1u);           // a_hi * b_lo
+                            mma_tf32_ts(d, ta + ks * 8, bh, id, 1u);           // a_hi * b_hi
+                        } else {
+                            mma_tf32_ts(d, ta + ks * 8, bh, id, first);        // a_hi * b_hi
+                        }
+                    }
+                    mma_commit(smem_u32(&bar_aempty[t]));
+                    if (++t == kNT) { t = 0; ++t_wraps; }
+                    if (!p.b_resident) {
+                        mma_commit(smem_u32(&bar_bempty[sb]));
+                        if (++sb == kNB) { sb = 0; ++b_wraps; }
+                    }
+                }
+                if (!ok) break;
+                mma_commit(smem_u32(&bar_accfull[a]));
+            }
+            // every MMA this thread issued has finished before the teardown
+            mma_commit(smem_u32(&bar_drain));
+            wait_phase_drain(smem_u32(&bar_drain), 0);
+        }
+    } else {
+        // -------------------------------------------------------------- weights --
+        if (lane == 0) {
+            if (p.b_resident) {
+                const uint32_t bytes = (uint32_t)nK * b_step;
+                mbar_expect_tx(smem_u32(&bar_bfull[0]), bytes);
+                for (uint32_t o = 0; o < bytes; o += 32768u)
+                    bulk_g2s(b_region + o, (const unsigned char *)wslice + o, min(32768u, bytes - o),
+                             smem_u32(&bar_bfull[0]));
+                wait_phase_drain(smem_u32(&bar_bfull[0]), 0);
+            } else {
+                int64_t j = 0;
+                int sb = 0, kt = 0;
+                uint32_t wraps = 0;
+                for (; j < total; ++j) {
+                    if (wraps >= 1 && !wait_phase(smem_u32(&bar_bempty[sb]), (wraps - 1) & 1, abort_flag)) break;
+                    mbar_expect_tx(smem_u32(&bar_bfull[sb]), b_step);
+                    bulk_g2s(b_region + (uint32_t)sb * b_step, (const unsigned char *)wslice + (size_t)kt * b_step,
+                             b_step, smem_u32(&bar_bfull[sb]));
+                    if (++kt == nK) kt = 0;
+                    if (++sb == kNB) { sb = 0; ++wraps; }
+                }
+                // the copies still in flight land before the shared memory is released
+                for (int64_t jj = std::max<int64_t>(0, j - kNB); jj < j; ++jj)
+                    wait_phase_drain(smem_u32(&bar_bfull[(int)(jj % kNB)]), (uint32_t)((jj / kNB) & 1));
+            }
+        }
+    }
+
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (threadIdx.x == 0 && abort_sh) atomicExch(p.err, MURE_ERR_TIMEOUT);
+    if (warp == 0) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512));
+    }
+}
+
+// Split fp32 weights [N][K] into TF32 halves laid out as the kernel's shared-memory
+// operand: for each 128-channel slice s and K-step kc, the hi plane then (3xTF32)
+// the lo plane, each Nt rows of 32 values in 128-byte-swizzled order.
+__global__ void k_swizzle_weights(const float *__restrict__ W, int N, int K, int Np, int Kp, int planes,
+                                  int64_t slice_floats, float *out)
+{
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (int64_t)Np * Kp) return;
+    const int n = (int)(i / Kp), k = (int)(i % Kp);
+    const float w = (n < N && k < K) ? W[(int64_t)n * K + k] : 0.f;
+    const float h = tf32_rna(w);
+    const int s = n / kSlice, nl = n % kSlice, Nt = min(kSlice, Np - s * kSlice);
+    const int kc = k / kTileK, kk = k % kTileK;
+    const int64_t chunk = (int64_t)s * slice_floats + (int64_t)kc * planes * Nt * kTileK;
+    const int64_t off = (sw128_off(nl, kk >> 2) >> 2) + (kk & 3);
+    out[chunk + off] = h;
+    if (planes == 2) out[chunk + (int64_t)Nt * kTileK + off] = tf32_rna(w - h);
+}
+
+int tc_supported(const Stage &S)
+{
+    if (S.oc < 16) return 0;
+    if (S.kind == MURE_NODE_DENSE) return !S.has_add && !S.pool && !S.gap;
+    // implicit-GEMM convolution: pooled maps need whole windows per warp (always true:
+    // a window is 4 consecutive GEMM rows and tiles start at multiples of 128)
+    return S.kind == MURE_NODE_CONV2D;
+}
+
+// Whether the tensor-core kernel can fetch a first-suffix overlay itself: at most
+// kOvMax patch values per row and K-step (dense: at most 4 mutated channels).
+int tc_overlay_inline(const Stage &S, const Overlay &ov)
+{
+    if (S.kind == MURE_NODE_DENSE) {
+        if (ov.kmax > 4) return 0;
+        const int per_slot = std::min(ov.cells, (kTileK + ov.ch - 1) / ov.ch + 1);
+        return ov.kmax * per_slot <= kOvMax;
+    }
+    if ((S.ic & 3) != 0) return 1;   // 4-byte copies take the patch value directly
+    const int pixels = (S.ic % kTileK == 0 || kTileK % S.ic == 0) ? std::max(1, kTileK / S.ic) : kTileK / S.ic + 2;
+    return ov.kmax * pixels <= kOvMax;
+}
+
+int64_t tc_weight_floats(const Stage &S)
+{
+    const int Np = round_up16(S.oc), Kp = round_up32(S.K), planes = S.tc == 1 ? 2 : 1;
+    const int64_t slice = (int64_t)planes * kSlice * Kp;
+    return slice * ((Np + kSlice - 1) / kSlice);
+}
+
+int launch_swizzle_weights(const Stage &S, float *out, cudaStream_t s)
+{
+    const int Np = round_up16(S.oc), Kp = round_up32(S.K), planes = S.tc == 1 ? 2 : 1;
+    const int64_t n = (int64_t)Np * Kp;
+    cudaMemsetAsync(out, 0, tc_weight_floats(S) * sizeof(float), s);
+    k_swizzle_weights<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(S.W, S.oc, S.K, Np, Kp, planes,
+                                                                   (int64_t)planes * kSlice * Kp, out);
+    return 1;
+}
+
+int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
+              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov)
+{
+    if (rm.R <= 0) return 0;
+    TcParams p{};
+    const bool dense = S.kind == MURE_NODE_DENSE;
+    p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
+    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
+    p.ih = S.ih; p.iw = S.iw; p.ic = S.ic; p.kh = S.kh; p.kw = S.kw; p.stride = S.stride; p.pad = S.pad;
+    p.oh = S.oh; p.ow = S.ow;
+    p.pool = S.pool; p.pw = S.ow / 2;
+    p.P = dense ? 1 : (S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : S.oh * S.ow);
+    p.K = S.K; p.Kp = round_up32(S.K); p.N = S.oc; p.Np = round_up16(S.oc);
+    const bool three = S.tc == 1;
+    const int planes = three ? 2 : 1;
+    p.Wsw = S.Wtc;
+    p.w_slice_floats = (int64_t)planes * kSlice * p.Kp;
+    p.b = S.b;
+    p.act1 = S.act1; p.has_add = S.has_add; p.act2 = S.act2;
+    p.skip = skip.p; p.skip_stride = skip.stride; p.skip_per_input = skip.per_input;
+    p.sk_w = S.sk_w; p.sk_c = S.sc_c; p.sk_stride = S.sc_stride;
+    p.z = z_out; p.z_stride = z_stride;
+    // with global average pooling the post-op map goes to gap_tmp first
+    const int mh = S.pool ? S.oh / 2 : S.oh, mw = S.pool ? S.ow / 2 : S.ow;
+    const int64_t map_stride = round4((int64_t)mh * mw * S.oc);
+    p.y = S.gap ? gap_tmp : y_out;
+    p.y_stride = S.gap ? map_stride : y_stride;
+    if (ov) p.ov = *ov;
+    p.err = S.err;
+    // shared memory: the weights (whole slice, or kNB K-steps), then the producer ring
+    const int nt_max = std::min(kSlice, p.Np);
+    const size_t b_step = (size_t)planes * nt_max * 128;
+    const size_t slice_bytes = b_step * (p.Kp / kTileK);
+    p.b_resident = slice_bytes <= 96 * 1024;
+    const size_t b_bytes = p.b_resident ? slice_bytes : kNB * b_step;
+    // at least 116 KiB so that one CTA (holding all 512 tensor-memory columns) runs per SM
+    const size_t ov_bytes = p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0;
+    const size_t smem = std::max<size_t>(1024 + b_bytes + (size_t)kNA * kStageA + ov_bytes, 116 * 1024);
+    const int64_t M = (int64_t)rm.R * p.P;
+    const int64_t tiles = (M + kTileM - 1) / kTileM;
+    static int n_sm = 0;
+    if (!n_sm) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+        if (n_sm <= 0) n_sm = 148;
+    }
+    const int ny = (p.Np + kSlice - 1) / kSlice;
+    const dim3 grid((unsigned)std::max<int64_t>(1, std::min<int64_t>(tiles, std::max(1, n_sm / ny))), (unsigned)ny);
+    auto go = [&](auto kern) {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        kern<<<grid, kThreads, smem, s>>>(p);
+    };
+    if (dense) { if (three) go(k_tc_gemm<true, true>); else go(k_tc_gemm<true, false>); }
+    else { if (three) go(k_tc_gemm<false, true>); else go(k_tc_gemm<false, false>); }
+    int launches = 1;
+    if (S.gap) launches += launch_gap(gap_tmp, map_stride, mh * mw, S.oc, rm.R, y_out, y_stride, s);
+    return launches;
+}
+
+}  // namespace mure
