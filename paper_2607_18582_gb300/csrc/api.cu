@@ -15,10 +15,14 @@ using namespace mure;
 namespace {
 
 // MURE_TC_CONV=1 puts every convolution of a TF32X3 model on the tensor cores.
-bool tc_conv_forced()
+// MURE_TC_CONV: in the tensor-core modes the LeNet-size convolution keeps its
+// CUDA-core kernel (faster there) unless this is "small" (the small-image mode) or
+// "generic" (the implicit-GEMM producers; the two tensor-core forms give identical
+// bits).
+std::string tc_conv_env()
 {
     const char *e = getenv("MURE_TC_CONV");
-    return e && e[0] == '1';
+    return e ? e : "";
 }
 
 // ------------------------------------------------------------------ plumbing --
@@ -647,7 +651,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     const Stage &Sn = m->st[l + 1];
     bool skip_reader = false;
     for (int v = l + 2; v < L; ++v) skip_reader |= m->st[v].has_add && m->st[v].skip_src == l + 1;
-    if (Sn.tc && !skip_reader && tc_overlay_inline(Sn, ov)) {
+    if (Sn.tc && !skip_reader && tc_overlay_inline(Sn, ov, rm.R / rm.T)) {
         timed(l + 1, 2 * Sn.macs * rm.R, [&] {
             return launch_tc(Sn, base, rm, nullptr, 0, skip_of(Sn), ws.xb[l + 2], m->xd[l + 2].stride, ws.gap_tmp, s,
                              &ov);
@@ -973,18 +977,23 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
         const char *force = getenv("MURE_FORCE_GENERIC");
         for (Stage &S : m->st) {
             S.variant = (force && force[0] == '1') ? 0 : conv_small_variant(S);
+            S.geo = S.variant;
             S.err = c->err_dev;
         }
         // tensor-core modes: layers before the output layer with >= 16 outputs run on
         // the tensor cores (3xTF32, or one TF32 MMA in the reduced-precision variant);
-        // in TF32X3 the LeNet-size convolutions keep their CUDA-core kernel, which is
-        // faster there than the implicit GEMM
+        // the LeNet-size convolution keeps its CUDA-core kernel unless MURE_TC_CONV asks
         for (int l = 0; l + 1 < m->L; ++l) {
             Stage &S = m->st[l];
-            const bool take = tc_supported(S) && (S.kind == MURE_NODE_DENSE || S.variant == 0 || tc_conv_forced());
+            const std::string env = tc_conv_env();
+            const bool small = tc_small_geometry(S) && (env == "small" || env == "generic");
+            const bool take = tc_supported(S) && (S.kind == MURE_NODE_DENSE || S.variant == 0 || small);
             if (take && d->precision == MURE_PREC_TF32X3) S.tc = 1;
             else if (take && d->precision == MURE_PREC_TF32) S.tc = 2;
-            if (S.tc) S.variant = 0;
+            if (S.tc) {
+                S.variant = 0;
+                S.tc_small = small && env != "generic";
+            }
         }
         std::vector<int> wn;
         for (int v = 0; v < d->n_nodes; ++v)

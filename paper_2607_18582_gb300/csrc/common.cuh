@@ -32,7 +32,9 @@ struct Stage {
     int yh, yw, yc;           // output x_{v+1}
     int64_t macs;             // multiply-accumulates per row
     int variant = 0;          // 0: implicit-GEMM kernel; > 0: a shared-memory direct conv
+    int geo = 0;              // > 0: a compiled small geometry (the delta's dot-product kernel)
     int tc = 0;               // tensor-core kernel: 1 = 3xTF32, 2 = one TF32 MMA (variant)
+    int tc_small = 0;         // tc: the small-image convolution mode
     float *Wtc = nullptr;     // tc: TF32 halves of W in the tensor-core operand layout
     int *err = nullptr;       // device error word of the context (bounded waits)
     float *W = nullptr;       // device [oc][K]
@@ -135,7 +137,8 @@ int launch_conv_small(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
 // launcher (arguments as for the stage kernel, plus the overlay).
 int tc_supported(const Stage &S);
 int64_t tc_weight_floats(const Stage &S);
-int tc_overlay_inline(const Stage &S, const Overlay &ov);
+int tc_overlay_inline(const Stage &S, const Overlay &ov, int64_t groups);
+int tc_small_geometry(const Stage &S);
 int launch_swizzle_weights(const Stage &S, float *out, cudaStream_t s);
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
               int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov = nullptr);

@@ -313,13 +313,13 @@ int launch_dot(const Stage &S, Src z, Src x, RowMap rm, const PatchArgs &pa, int
 
 // GF / WS delta values for the small-layer geometries (the neuron count per mutant
 // must be <= 8); 0 when the layer has no such kernel.
-int patch_dot_supported(const Stage &S, int kmax) { return S.variant > 0 && kmax <= 8 && !S.has_add && !S.gap; }
+int patch_dot_supported(const Stage &S, int kmax) { return S.geo > 0 && kmax <= 8 && !S.has_add && !S.gap; }
 
 int launch_patch_dot(const Stage &S, Src z, Src x, RowMap rm, const PatchArgs &pa, int kmax, float *out,
                      int64_t out_stride, cudaStream_t s)
 {
     if (rm.R <= 0) return 0;
-    switch (S.variant) {
+    switch (S.geo) {
     case 1: return launch_dot<5, 5, 6, 14, 14, 0, true>(S, z, x, rm, pa, kmax, out, out_stride, s);
     case 2: return launch_dot<5, 5, 1, 32, 32, 2, true>(S, z, x, rm, pa, kmax, out, out_stride, s);
     }

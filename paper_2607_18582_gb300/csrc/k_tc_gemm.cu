@@ -15,12 +15,15 @@
 //              splits them into TF32 halves and stores the halves into a tensor-memory
 //              A stage (tcgen05.st); the MMA reads A from tensor memory, so the
 //              operand never goes through shared memory a second time;
-//   warp 8     one thread issues the MMAs (kind::tf32, M=128, K=8) and commits them
-//              to the stage barriers;
-//   warp 9     one thread moves the weights: pre-split, pre-swizzled K-step chunks
+//   warps 8-10 MMA issue (kind::tf32, M=128, K=8): one thread issues an MMA only about
+//              every 120 cycles, whatever N is, so where tensor memory allows, a
+//              K-step's MMAs are dealt to up to three warps, each accumulating into its
+//              own partial accumulator; the epilogue adds the partials in a fixed order;
+//   warp 11    one thread moves the weights: pre-split, pre-swizzled K-step chunks
 //              (one bulk copy each), or the whole slice once when it fits;
-//   warps 4-7  epilogue: two accumulators alternate, so the bias / activation /
-//              residual / 2x2 pool / store of tile i overlaps the MMAs of tile i+1.
+//   warps 4-7  epilogue: two accumulator sets alternate, so the bias / activation /
+//              residual / 2x2 pool / store of tile i overlaps the MMAs of tile i+1;
+//              unpooled rows go out through shared memory in coalesced stores.
 // The K order of the accumulation is fixed and independent of the row's position in
 // the tile, so a row gives the same bits in every batch (memoized == vanilla).
 // Every wait is bounded; on expiry the kernel records an error code, stops every
@@ -38,17 +41,27 @@ namespace {
 constexpr int kTileM = 128;
 constexpr int kTileK = 32;             // fp32 / tf32 values per 128-byte row
 constexpr int kNA = 4;                 // producer cp.async ring depth (K-steps)
-constexpr int kNB = 4;                 // streamed weight stages
+constexpr int kNB = 3;                 // streamed weight stages
 constexpr int kSlice = 128;            // output channels per CTA
-constexpr int kThreads = 320;          // 4 producer + 4 epilogue + MMA + weight warps
-constexpr int kAccCol = 0;             // two accumulators at columns 0 and 128
-constexpr int kACol = 256;             // A stages from column 256
+constexpr int kThreads = 384;          // 4 producer + 4 epilogue + 3 MMA + weight warps
+constexpr int kEpiStride = 36;         // floats per row of an epilogue staging chunk (32 + pad)
+constexpr int kACol = 256;             // accumulators in columns 0..255, A stages from 256
 constexpr uint32_t kStageA = kTileM * 128;   // bytes of one producer ring slot
 constexpr long long kSpin = 2000000000LL;    // about a second at the SM clock
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
 {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// The high TF32 half of a finite fp32 value on the integer pipes: add half a unit in
+// the last TF32 place to the magnitude bits and clear the 13 low bits (round to
+// nearest, ties away from zero).  The remainder x - hi is exact in fp32; the MMA reads
+// only its top 19 bits.  (The conversion instruction runs on a slow pipe and was the
+// producers' bottleneck.)
+__device__ __forceinline__ float tf32_hi(float x)
+{
+    return __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
 }
 
 __device__ __forceinline__ float tf32_rna(float x)
@@ -109,28 +122,18 @@ __device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity)
     return ok != 0;
 }
 
-// The same with a suspend-time hint: a waiting thread sleeps until the phase
-// completes (or the hint expires) instead of taking issue slots from the producers.
-__device__ __forceinline__ bool mbar_try_sleep(uint32_t a, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}\n"
-        : "=r"(ok)
-        : "r"(a), "r"(parity), "r"(20000u)
-        : "memory");
-    return ok != 0;
-}
-
-// Wait for the phase of parity `parity`; false when another role has aborted or
-// about a second has passed (then this role aborts the CTA).
-template <bool SLEEP = false>
+// Wait for the phase of parity `parity`, polling every ~NS nanoseconds (a sleeping
+// warp leaves the issue slots of its SM sub-partition to the producers); false when
+// another role has aborted or about a second has passed (then this role aborts the
+// CTA).
+template <int NS = 0>
 __device__ __forceinline__ bool wait_phase(uint32_t a, uint32_t parity, volatile int *abort_flag)
 {
     if (mbar_try(a, parity)) return true;
     const long long t0 = clock64();
     for (;;) {
-        if (SLEEP ? mbar_try_sleep(a, parity) : mbar_try(a, parity)) return true;
+        if (NS > 0) __nanosleep(NS);
+        if (mbar_try(a, parity)) return true;
         if (*abort_flag) return false;
         if (clock64() - t0 > kSpin) { *abort_flag = 1; return false; }
     }
@@ -138,10 +141,10 @@ __device__ __forceinline__ bool wait_phase(uint32_t a, uint32_t parity, volatile
 
 // The same for a whole warp: every lane polls, the verdict is the warp's AND, so the
 // .sync.aligned tensor-memory instructions that follow see a converged warp.
-template <bool SLEEP = false>
+template <int NS = 0>
 __device__ __forceinline__ bool warp_wait_phase(uint32_t a, uint32_t parity, volatile int *abort_flag)
 {
-    const bool ok = wait_phase<SLEEP>(a, parity, abort_flag);
+    const bool ok = wait_phase<NS>(a, parity, abort_flag);
     return __all_sync(0xffffffffu, ok);
 }
 
@@ -160,6 +163,43 @@ __device__ __forceinline__ void mma_tf32_ts(uint32_t d_tmem, uint32_t a_tmem, ui
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
         " tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
         "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc));
+}
+
+// MMAs q = LO .. HI-1 of a K-step, q = ks * kTerms + term (3xTF32: a_lo*b_hi,
+// a_hi*b_lo, a_hi*b_hi for K8 step ks), into accumulator d; the first one overwrites
+// unless acc0.  Fully unrolled: the issuing thread has no other warps to hide the
+// latency of scalar work between MMAs, and an MMA predicated off still costs its issue
+// slot, so each issuing warp runs only its own block.
+template <bool THREE, int LO, int HI>
+__device__ __forceinline__ void mma_block(uint32_t d, uint32_t ta, uint64_t dh, uint64_t dl, uint32_t id, uint32_t acc0)
+{
+    constexpr int kTerms = THREE ? 3 : 1;
+#pragma unroll
+    for (int q = LO; q < HI; ++q) {
+        const int ks = q / kTerms, term = q % kTerms;
+        const uint32_t acc = q > LO ? 1u : acc0;
+        // K8 step ks starts 32 bytes further along the swizzled rows: +2 in the
+        // descriptor's 16-byte address field
+        if (!THREE || term == 2) mma_tf32_ts(d, ta + ks * 8, dh + 2 * ks, id, acc);    // a_hi * b_hi
+        else if (term == 0) mma_tf32_ts(d, ta + 32 + ks * 8, dh + 2 * ks, id, acc);   // a_lo * b_hi
+        else mma_tf32_ts(d, ta + ks * 8, dl + 2 * ks, id, acc);                       // a_hi * b_lo
+    }
+}
+
+// Warp w of n_mma issuing warps: the contiguous block w*kQ/n .. (w+1)*kQ/n of a K-step.
+template <bool THREE>
+__device__ __forceinline__ void mma_share(int nmma, int w, uint32_t d, uint32_t ta, uint64_t dh, uint64_t dl, uint32_t id,
+                                          uint32_t acc0)
+{
+    constexpr int Q = THREE ? 12 : 4;
+    switch (nmma * 4 + w) {
+    case 4: mma_block<THREE, 0, Q>(d, ta, dh, dl, id, acc0); break;
+    case 8: mma_block<THREE, 0, Q / 2>(d, ta, dh, dl, id, acc0); break;
+    case 9: mma_block<THREE, Q / 2, Q>(d, ta, dh, dl, id, acc0); break;
+    case 12: mma_block<THREE, 0, Q / 3>(d, ta, dh, dl, id, acc0); break;
+    case 13: mma_block<THREE, Q / 3, 2 * Q / 3>(d, ta, dh, dl, id, acc0); break;
+    default: mma_block<THREE, 2 * Q / 3, Q>(d, ta, dh, dl, id, acc0); break;
+    }
 }
 
 __device__ __forceinline__ void mma_commit(uint32_t mbar)
@@ -237,6 +277,8 @@ struct TcParams {
     float *z; int64_t z_stride;
     float *y; int64_t y_stride;
     Overlay ov;                  // mutated channels of the input rows (ov.patch null: none)
+    int n_mma;                   // MMA-issuing warps, each with its own partial accumulators
+    int acc_cols;                // tensor-memory columns of one partial accumulator
     int *err;
 };
 
@@ -295,17 +337,45 @@ __device__ __forceinline__ RowInfo row_info(const TcParams &p, int64_t m)
     return ri;
 }
 
-// Queue the cp.async copies of K-step k0 .. k0+31 of GEMM row `pf` into the 128-byte
-// row `slot` (swizzled like the MMA operand layout, so the read-back is free of bank
-// conflicts).  Values past the fan-in, outside the image (zero padding) or of rows
-// past the end are zero-filled.  The mutated channels of the first suffix stage:
-// their patch values are fetched into the slot's overlay entries (ov), written over
-// the staged row once it has landed.
+// The rows a producer lane copies for its warp: lane l copies 16-byte chunk l & 7 of
+// rows 4c + (l >> 3), c = 0..7, of the warp's 32 GEMM rows, so that one copy
+// instruction covers four whole 128-byte row segments (a thread copying its own row
+// would touch 32 rows per instruction and saturate the load/store unit).
+struct LoadRows {
+    const float *xrow[8];   // null: row past the end
+    int oy[8], ox[8];
+};
+
 template <bool DENSE>
-__device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, int r, uint32_t slot, uint32_t ov,
-                                              int k0)
+__device__ __forceinline__ void load_rows(const RowInfo &pf, LoadRows &lr)
+{
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+        const int src = 4 * c + (lane >> 3);
+        const unsigned long long xp =
+            __shfl_sync(0xffffffffu, (unsigned long long)(uintptr_t)(pf.ok ? pf.xrow : nullptr), src);
+        lr.xrow[c] = reinterpret_cast<const float *>((uintptr_t)xp);
+        if (!DENSE) {
+            lr.oy[c] = __shfl_sync(0xffffffffu, pf.oy, src);
+            lr.ox[c] = __shfl_sync(0xffffffffu, pf.ox, src);
+        }
+    }
+}
+
+// Queue the cp.async copies of K-step k0 .. k0+31 of the warp's 32 GEMM rows into
+// their 128-byte rows of `slot` (swizzled like the MMA operand layout, so that each
+// thread's read-back of its own row is free of bank conflicts).  Values past the
+// fan-in, outside the image (zero padding) or of rows past the end are zero-filled.
+// The mutated channels of the first suffix stage: the row owner (thread r) fetches
+// their patch values into the slot's overlay entries (ov), written over its row once
+// the copies have landed.
+template <bool DENSE>
+__device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, const LoadRows &lr, int r, uint32_t slot,
+                                              uint32_t ov, int k0)
 {
     const float *dummy = p.b;   // a valid address for zero-byte copies
+    const int lane = r & 31, wbase = r & ~31, ch = lane & 7;
     int cnt = 0;
     auto entry = [&](int pos, const float *src) {
         if (cnt < kOvMax) {
@@ -317,15 +387,17 @@ __device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, in
         ++cnt;
     };
     if (DENSE) {
+        const int kk = k0 + 4 * ch;
+        const int nbk = max(0, min(16, (p.K - kk) * 4));
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            const int row = wbase + 4 * c + (lane >> 3);
+            const int nb = lr.xrow[c] ? nbk : 0;
+            cp_async16(slot + sw128_off(row, ch), nb ? (const void *)(lr.xrow[c] + kk) : (const void *)dummy, nb);
+        }
         // overlay positions are c * ch + j (cell c of mutated channel j); the K-steps of a
         // row come in ascending k, so each slot keeps a cursor
         const int nq = min(pf.ov_k, 4);
-#pragma unroll
-        for (int c = 0; c < kTileK / 4; ++c) {
-            const int kk = k0 + 4 * c;
-            const int nb = pf.ok ? max(0, min(16, (p.K - kk) * 4)) : 0;
-            cp_async16(slot + sw128_off(r, c), nb ? (const void *)(pf.xrow + kk) : (const void *)dummy, nb);
-        }
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             if (q >= nq) break;
@@ -336,26 +408,37 @@ __device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, in
             }
         }
     } else if ((p.ic & 3) == 0) {
-        // 16-byte chunks: 4 channels of one input pixel
-        int ci = k0 % p.ic, t = k0 / p.ic, kx = t % p.kw, ky = t / p.kw;
+        // 16-byte chunks: 4 channels of one input pixel; this lane's chunk has the same
+        // (ky, kx, ci) in all its rows
+        const int kk = k0 + 4 * ch;
+        const int ci = kk % p.ic, t = kk / p.ic, kx = t % p.kw, ky = t / p.kw;
 #pragma unroll
-        for (int c = 0; c < kTileK / 4; ++c) {
-            const int kk = k0 + 4 * c;
-            const int iy = pf.oy * p.stride - p.pad + ky, ix = pf.ox * p.stride - p.pad + kx;
-            const bool in = pf.ok && kk < p.K && (unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw;
-            cp_async16(slot + sw128_off(r, c), in ? pf.xrow + ((int64_t)iy * p.iw + ix) * p.ic + ci : dummy,
+        for (int c = 0; c < 8; ++c) {
+            const int row = wbase + 4 * c + (lane >> 3);
+            const int iy = lr.oy[c] * p.stride - p.pad + ky, ix = lr.ox[c] * p.stride - p.pad + kx;
+            const bool in = lr.xrow[c] && kk < p.K && (unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw;
+            cp_async16(slot + sw128_off(row, ch), in ? lr.xrow[c] + ((int64_t)iy * p.iw + ix) * p.ic + ci : dummy,
                        in ? 16 : 0);
-            if (in)
-                for (int q = 0; q < pf.ov_k; ++q) {
-                    const int jn = pf.ov_ids[q];
-                    if (jn >= ci && jn < ci + 4) entry(4 * c + jn - ci, pf.ov_patch + q * p.ov.cells + iy * p.iw + ix);
-                }
-            ci += 4;
-            if (ci == p.ic) { ci = 0; if (++kx == p.kw) { kx = 0; ++ky; } }
+        }
+        if (pf.ov_k > 0) {
+            // the owner's mutated channels in its own row
+            int ci2 = k0 % p.ic, t2 = k0 / p.ic, kx2 = t2 % p.kw, ky2 = t2 / p.kw;
+            for (int c = 0; c < kTileK / 4; ++c) {
+                const int iy = pf.oy * p.stride - p.pad + ky2, ix = pf.ox * p.stride - p.pad + kx2;
+                const bool in = k0 + 4 * c < p.K && (unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw;
+                if (in)
+                    for (int q = 0; q < pf.ov_k; ++q) {
+                        const int jn = pf.ov_ids[q];
+                        if (jn >= ci2 && jn < ci2 + 4)
+                            entry(4 * c + jn - ci2, pf.ov_patch + q * p.ov.cells + iy * p.iw + ix);
+                    }
+                ci2 += 4;
+                if (ci2 == p.ic) { ci2 = 0; if (++kx2 == p.kw) { kx2 = 0; ++ky2; } }
+            }
         }
     } else {
-        // channel counts that are not a multiple of 4: 4-byte copies, the patch value
-        // taken directly for a mutated channel
+        // channel counts that are not a multiple of 4: 4-byte copies of the thread's own
+        // row, the patch value taken directly for a mutated channel
         int ci = k0 % p.ic, t = k0 / p.ic, kx = t % p.kw, ky = t / p.kw;
         for (int i = 0; i < kTileK; ++i) {
             const int k = k0 + i;
@@ -372,10 +455,73 @@ __device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, in
     if (p.ov.patch) asm volatile("st.shared.u8 [%0], %1;" ::"r"(ov + kTileM * kOvMax * 5 + r), "r"(min(cnt, kOvMax)));
 }
 
-// DENSE: one GEMM row per batch row; THREE: 3xTF32 (else one TF32 product).
-template <bool DENSE, bool THREE>
+// The small-image convolution mode: 5x5 filters over a 14 x 14 x 6 map, stride 1, no
+// padding, 2x2 max pool (LeNet-5's second convolution).  The producers stage whole
+// input maps in shared memory (copied with coalesced cp.async) and gather each GEMM
+// row's receptive field from there with compile-time offsets, two channels per load;
+// a 6-channel map is no fit for the 16-byte copies of the generic path.  A tile of
+// 128 GEMM rows spans at most NIMG maps.
+struct SmallConv {
+    static constexpr int IH = 14, IW = 14, IC = 6, KH = 5, KW = 5, OH = 10, OW = 10, PW = 5;
+    static constexpr int P = 4 * (OH / 2) * (OW / 2);        // GEMM rows per map (window-major)
+    static constexpr int K = KH * KW * IC, NKT = (K + kTileK - 1) / kTileK;
+    static constexpr int CELLS = IH * IW;                     // overlay cells of a mutated channel
+    static constexpr uint32_t IMG_B = IH * IW * IC * 4;       // bytes of one staged map
+    static constexpr int CH16 = IMG_B / 16;
+    static constexpr int MAXQ = 4;                            // mutated channels per row (overlay)
+    static constexpr int MAXG = 1024;                         // mutants per batch (overlay table)
+    static constexpr int NIMG = (kTileM - 1) / P + 2;         // maps per tile, at most
+    static constexpr uint32_t BUF_B = NIMG * IMG_B;           // one buffer of staged maps
+    static constexpr uint32_t OVST_B = NIMG * MAXQ * CELLS * 4;   // one buffer of staged patch values
+    static constexpr uint32_t TAB_B = MAXG * (1 + MAXQ) * 4;      // [g][count, channel ids]
+    static constexpr uint32_t BYTES = 2 * BUF_B + 2 * OVST_B + TAB_B;
+};
+static_assert(SmallConv::IMG_B % 16 == 0, "maps are copied in 16-byte chunks");
+static_assert((SmallConv::CELLS * 4) % 16 == 0, "patch values are copied in 16-byte chunks");
+
+__device__ __forceinline__ void named_bar_producers() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// K-step KT of a small-image GEMM row: 16 channel pairs at compile-time offsets from
+// the row's receptive-field origin `base` (k = (ky, kx, ci) with ci even, so every pair
+// is 8-byte aligned).
+template <int KT>
+__device__ __forceinline__ void small_gather(uint32_t base, float (&v)[kTileK])
+{
+    using G = SmallConv;
+#pragma unroll
+    for (int e = 0; e < kTileK / 2; ++e) {
+        const int k = KT * kTileK + 2 * e;
+        if (k < G::K) {
+            const uint32_t off = (uint32_t)(((k / (G::KW * G::IC)) * G::IW + (k / G::IC) % G::KW) * G::IC + k % G::IC) * 4;
+            asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v[2 * e]), "=f"(v[2 * e + 1]) : "r"(base + off));
+        } else {
+            v[2 * e] = 0.f;
+            v[2 * e + 1] = 0.f;
+        }
+    }
+}
+
+// The K-steps KT .. NKT-1 of a small-image row, each handed to `push`.
+template <int KT>
+struct SmallSteps {
+    template <class Push>
+    __device__ __forceinline__ static void run(uint32_t base, Push &push, bool &ok)
+    {
+        if constexpr (KT < SmallConv::NKT) {
+            float v[kTileK];
+            small_gather<KT>(base, v);
+            if (ok) ok = push(v);
+            SmallSteps<KT + 1>::run(base, push, ok);
+        }
+    }
+};
+
+// MODE 0: dense layer (one GEMM row per batch row); 1: implicit-GEMM convolution; 2:
+// the small-image convolution.  THREE: 3xTF32 (else one TF32 product).
+template <int MODE, bool THREE>
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
 {
+    constexpr bool DENSE = MODE == 0;
     constexpr int kNT = THREE ? 4 : 8;             // tensor-memory A stages
     constexpr int kAColsPerStage = THREE ? 64 : 32;
     extern __shared__ __align__(1024) unsigned char smraw[];
@@ -384,6 +530,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     __shared__ uint32_t tmem_sh;
     __shared__ int abort_sh;
     __shared__ float bias_sh[kSlice];
+    __shared__ __align__(16) float epi_stage[4][32 * kEpiStride];   // per epilogue warp: 32 rows x 32 values
+    __shared__ float *epi_ptr[4][32];                               // per epilogue warp: each row's output
     volatile int *abort_flag = &abort_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -408,11 +556,34 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     for (int n = threadIdx.x; n < kSlice; n += kThreads) bias_sh[n] = n_base + n < p.N ? p.b[n_base + n] : 0.f;
+    // small-image mode: staged maps, staged patch values, the batch's mutated-channel table
+    const uint32_t img_region = a_region;
+    const uint32_t ovst_region = img_region + 2 * SmallConv::BUF_B;
+    const uint32_t ovtab_region = ovst_region + 2 * SmallConv::OVST_B;
+    if (MODE == 2 && p.ov.patch) {
+        const int G = p.R / p.T;
+        for (int g = threadIdx.x; g < G; g += kThreads) {
+            const int n = p.ov.n_neurons[g];
+            const uint32_t tab = ovtab_region + (uint32_t)g * (1 + SmallConv::MAXQ) * 4;
+            asm volatile("st.shared.u32 [%0], %1;" ::"r"(tab), "r"(n));
+            for (int q = 0; q < SmallConv::MAXQ; ++q)
+                asm volatile("st.shared.u32 [%0], %1;" ::"r"(tab + 4 + 4 * q), "r"(q < n ? p.ov.ids[p.ov.neuron_off[g] + q] : 0));
+        }
+    }
     if (threadIdx.x == 32) {
-        for (int s = 0; s < kNT; ++s) { mbar_init(smem_u32(&bar_afull[s]), 4); mbar_init(smem_u32(&bar_aempty[s]), 1); }
-        for (int s = 0; s < kNB; ++s) { mbar_init(smem_u32(&bar_bfull[s]), 1); mbar_init(smem_u32(&bar_bempty[s]), 1); }
-        for (int s = 0; s < 2; ++s) { mbar_init(smem_u32(&bar_accfull[s]), 1); mbar_init(smem_u32(&bar_accempty[s]), 4); }
-        mbar_init(smem_u32(&bar_drain), 1);
+        for (int s = 0; s < kNT; ++s) {
+            mbar_init(smem_u32(&bar_afull[s]), 4);
+            mbar_init(smem_u32(&bar_aempty[s]), p.n_mma);
+        }
+        for (int s = 0; s < kNB; ++s) {
+            mbar_init(smem_u32(&bar_bfull[s]), 1);
+            mbar_init(smem_u32(&bar_bempty[s]), p.n_mma);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(smem_u32(&bar_accfull[s]), p.n_mma);
+            mbar_init(smem_u32(&bar_accempty[s]), 4);
+        }
+        mbar_init(smem_u32(&bar_drain), p.n_mma);
         abort_sh = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -425,59 +596,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
         // ------------------------------------------------------------ producers --
         const int r = threadIdx.x;                        // GEMM row in the tile = TMEM lane
         const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
-        // issue cursor (tile i, K-tile kt, ring slot) runs kNA - 1 steps ahead
-        RowInfo pf{};
-        int64_t iss_i = 0, issued = 0;
-        int iss_kt = 0, iss_slot = 0;
-        auto issue_next = [&]() {
-            if (iss_kt == 0) pf = row_info<DENSE>(p, (blockIdx.x + iss_i * gridDim.x) * kTileM + r);
-            produce_issue<DENSE>(p, pf, r, a_region + (uint32_t)iss_slot * kStageA,
-                                 ov_region + (uint32_t)iss_slot * kOvSlotBytes, iss_kt * kTileK);
-            if (++iss_kt == nK) { iss_kt = 0; ++iss_i; }
-            if (++iss_slot == kNA) iss_slot = 0;
-            ++issued;
-        };
-        for (int s0 = 0; s0 < kNA - 1; ++s0) {
-            if (issued < total) issue_next();
-            cp_async_commit();
-        }
-        int slot_i = 0, t = 0;
+        int t = 0;
         uint32_t wraps = 0;                               // completed rounds of the A-stage ring
-        for (int64_t j = 0; j < total; ++j) {
-            if (issued < total) issue_next();
-            cp_async_commit();
-            cp_async_wait<kNA - 1>();                     // this thread's copies of step j
-            const uint32_t slot = a_region + (uint32_t)slot_i * kStageA;
-            if (p.ov.patch) {
-                // the row's overlay entries of this K-step, written over the landed copy
-                const uint32_t ov = ov_region + (uint32_t)slot_i * kOvSlotBytes;
-                uint32_t n;
-                asm volatile("ld.shared.u8 %0, [%1];" : "=r"(n) : "r"(ov + kTileM * kOvMax * 5 + r));
-                for (uint32_t e = 0; e < n; ++e) {
-                    uint32_t pos, val;
-                    asm volatile("ld.shared.u8 %0, [%1];" : "=r"(pos) : "r"(ov + kTileM * kOvMax * 4 + e * kTileM + r));
-                    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(val) : "r"(ov + (e * kTileM + r) * 4));
-                    asm volatile("st.shared.u32 [%0], %1;" ::"r"(slot + sw128_off(r, pos >> 2) + 4 * (pos & 3)), "r"(val)
-                                 : "memory");
-                }
-            }
-            if (++slot_i == kNA) slot_i = 0;
-            float hi[kTileK], lo[kTileK];
-#pragma unroll
-            for (int c = 0; c < kTileK / 4; ++c) {
-                float4 v;
-                asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
-                             : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                             : "r"(slot + sw128_off(r, c)));
-                hi[4 * c] = v.x; hi[4 * c + 1] = v.y; hi[4 * c + 2] = v.z; hi[4 * c + 3] = v.w;
-            }
+        // split one K-step of this row into TF32 halves and hand it to the MMA warps
+        auto push = [&](float (&hi)[kTileK]) -> bool {
+            float lo[kTileK];
 #pragma unroll
             for (int i = 0; i < kTileK; ++i) {
-                const float h = tf32_rna(hi[i]);
-                if (THREE) lo[i] = tf32_rna(hi[i] - h);
+                const float h = tf32_hi(hi[i]);
+                if (THREE) lo[i] = hi[i] - h;
                 hi[i] = h;
             }
-            if (wraps >= 1 && !warp_wait_phase(smem_u32(&bar_aempty[t]), (wraps - 1) & 1, abort_flag)) break;
+            if (wraps >= 1 && !warp_wait_phase<32>(smem_u32(&bar_aempty[t]), (wraps - 1) & 1, abort_flag)) return false;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t ta = tmem + lane_off + kACol + t * kAColsPerStage;
             tmem_st32(ta, hi);
@@ -487,112 +617,265 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bar_afull[t]));
             if (++t == kNT) { t = 0; ++wraps; }
+            return true;
+        };
+        if constexpr (MODE == 2) {
+            using G = SmallConv;
+            // copies of tile i's maps (and patch values) into buffer i & 1
+            auto issue_tile = [&](int64_t i) {
+                const int64_t m0 = (blockIdx.x + i * gridDim.x) * kTileM;
+                const int64_t row0 = m0 / G::P;
+                const int nimg = (int)((min(m0 + kTileM, M) - 1) / G::P - row0) + 1;
+                const uint32_t buf = img_region + (uint32_t)(i & 1) * G::BUF_B;
+                for (int im = 0; im < nimg; ++im) {
+                    const int64_t row = row0 + im;
+                    const float *src = p.x + (p.x_per_input ? p.t0 + row % p.T : row) * p.x_stride;
+                    for (int c = r; c < G::CH16; c += kTileM) cp_async16(buf + im * G::IMG_B + c * 16, src + c * 4, 16);
+                }
+                if (p.ov.patch) {
+                    const uint32_t ovb = ovst_region + (uint32_t)(i & 1) * G::OVST_B;
+                    for (int im = 0; im < nimg; ++im) {
+                        const int64_t row = row0 + im;
+                        uint32_t k;
+                        asm volatile("ld.shared.u32 %0, [%1];" : "=r"(k) : "r"(ovtab_region + (uint32_t)(row / p.T) * (1 + G::MAXQ) * 4));
+                        const float *src = p.ov.patch + row * p.ov.row_stride;
+                        for (int c4 = r; c4 < (int)k * G::CELLS / 4; c4 += kTileM)
+                            cp_async16(ovb + (im * G::MAXQ * G::CELLS + c4 * 4) * 4, src + c4 * 4, 16);
+                    }
+                }
+            };
+            if (my_tiles > 0) issue_tile(0);
+            cp_async_commit();
+            bool ok = true;
+            for (int64_t i = 0; ok && i < my_tiles; ++i) {
+                cp_async_wait<0>();
+                named_bar_producers();                    // every copy of tile i has landed
+                if (i + 1 < my_tiles) issue_tile(i + 1);  // the other buffer: tile i-1 is done
+                cp_async_commit();
+                const int64_t m0 = (blockIdx.x + i * gridDim.x) * kTileM;
+                const int64_t row0 = m0 / G::P;
+                const uint32_t buf = img_region + (uint32_t)(i & 1) * G::BUF_B;
+                if (p.ov.patch) {
+                    // the mutants' channels written into the staged maps
+                    const int nimg = (int)((min(m0 + kTileM, M) - 1) / G::P - row0) + 1;
+                    const uint32_t ovb = ovst_region + (uint32_t)(i & 1) * G::OVST_B;
+                    for (int im = 0; im < nimg; ++im) {
+                        const uint32_t tab = ovtab_region + (uint32_t)((row0 + im) / p.T) * (1 + G::MAXQ) * 4;
+                        uint32_t k;
+                        asm volatile("ld.shared.u32 %0, [%1];" : "=r"(k) : "r"(tab));
+                        for (int idx = r; idx < (int)k * G::CELLS; idx += kTileM) {
+                            const int q = idx / G::CELLS, c = idx - q * G::CELLS;
+                            uint32_t jn, val;
+                            asm volatile("ld.shared.u32 %0, [%1];" : "=r"(jn) : "r"(tab + 4 + q * 4));
+                            asm volatile("ld.shared.u32 %0, [%1];" : "=r"(val) : "r"(ovb + (im * G::MAXQ * G::CELLS + idx) * 4));
+                            asm volatile("st.shared.u32 [%0], %1;" ::"r"(buf + im * G::IMG_B + (c * G::IC + jn) * 4), "r"(val)
+                                         : "memory");
+                        }
+                    }
+                    named_bar_producers();
+                }
+                // this thread's GEMM row: map, pooling window, position in the window
+                const int64_t m = m0 + r;
+                const bool in = m < M;
+                const int64_t row = in ? m / G::P : row0;
+                const int q = in ? (int)(m - row * G::P) : 0;
+                const int w = q >> 2, sub = q & 3;
+                const int oy = 2 * (w / G::PW) + (sub >> 1), ox = 2 * (w % G::PW) + (sub & 1);
+                const uint32_t base = buf + (uint32_t)(row - row0) * G::IMG_B + (uint32_t)((oy * G::IW + ox) * G::IC) * 4;
+                SmallSteps<0>::run(base, push, ok);
+            }
+            cp_async_wait<0>();
+        } else {
+            // issue cursor (tile i, K-tile kt, ring slot) runs kNA - 1 steps ahead
+            RowInfo pf{};
+            LoadRows lr{};
+            int64_t iss_i = 0, issued = 0;
+            int iss_kt = 0, iss_slot = 0;
+            auto issue_next = [&]() {
+                if (iss_kt == 0) {
+                    pf = row_info<DENSE>(p, (blockIdx.x + iss_i * gridDim.x) * kTileM + r);
+                    if (DENSE || (p.ic & 3) == 0) load_rows<DENSE>(pf, lr);
+                }
+                produce_issue<DENSE>(p, pf, lr, r, a_region + (uint32_t)iss_slot * kStageA,
+                                     ov_region + (uint32_t)iss_slot * kOvSlotBytes, iss_kt * kTileK);
+                if (++iss_kt == nK) { iss_kt = 0; ++iss_i; }
+                if (++iss_slot == kNA) iss_slot = 0;
+                ++issued;
+            };
+            for (int s0 = 0; s0 < kNA - 1; ++s0) {
+                if (issued < total) issue_next();
+                cp_async_commit();
+            }
+            int slot_i = 0;
+            for (int64_t j = 0; j < total; ++j) {
+                if (issued < total) issue_next();
+                cp_async_commit();
+                cp_async_wait<kNA - 1>();                 // this thread's copies of step j
+                __syncwarp();                             // ... and those of the warp's other lanes
+                const uint32_t slot = a_region + (uint32_t)slot_i * kStageA;
+                if (p.ov.patch) {
+                    // the row's overlay entries of this K-step, written over the landed copy
+                    const uint32_t ov = ov_region + (uint32_t)slot_i * kOvSlotBytes;
+                    uint32_t n;
+                    asm volatile("ld.shared.u8 %0, [%1];" : "=r"(n) : "r"(ov + kTileM * kOvMax * 5 + r));
+                    for (uint32_t e = 0; e < n; ++e) {
+                        uint32_t pos, val;
+                        asm volatile("ld.shared.u8 %0, [%1];" : "=r"(pos) : "r"(ov + kTileM * kOvMax * 4 + e * kTileM + r));
+                        asm volatile("ld.shared.u32 %0, [%1];" : "=r"(val) : "r"(ov + (e * kTileM + r) * 4));
+                        asm volatile("st.shared.u32 [%0], %1;" ::"r"(slot + sw128_off(r, pos >> 2) + 4 * (pos & 3)),
+                                     "r"(val)
+                                     : "memory");
+                    }
+                }
+                if (++slot_i == kNA) slot_i = 0;
+                float v[kTileK];
+#pragma unroll
+                for (int c = 0; c < kTileK / 4; ++c) {
+                    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                                 : "=f"(v[4 * c]), "=f"(v[4 * c + 1]), "=f"(v[4 * c + 2]), "=f"(v[4 * c + 3])
+                                 : "r"(slot + sw128_off(r, c)));
+                }
+                if (!push(v)) break;
+            }
+            cp_async_wait<0>();
         }
-        cp_async_wait<0>();
     } else if (warp < 8) {
         // ------------------------------------------------------------- epilogue --
         const int qd = warp & 3;
         const uint32_t lane_off = (uint32_t)(qd * 32) << 16;
         for (int64_t i = 0; i < my_tiles; ++i) {
             const int a = (int)(i & 1);
-            if (!warp_wait_phase<true>(smem_u32(&bar_accfull[a]), (uint32_t)((i >> 1) & 1), abort_flag)) break;
+            if (!warp_wait_phase<64>(smem_u32(&bar_accfull[a]), (uint32_t)((i >> 1) & 1), abort_flag)) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const int64_t tile = blockIdx.x + i * gridDim.x;
             const RowInfo ri = row_info<DENSE, false>(p, tile * kTileM + qd * 32 + lane);
             const float *srow = nullptr;
             if (p.has_add && ri.ok) srow = p.skip + (p.skip_per_input ? p.t0 + ri.row % p.T : ri.row) * p.skip_stride;
             float *yrow = ri.ok ? p.y + ri.row * p.y_stride : nullptr;
-            for (int n0 = 0; n0 < Nt; n0 += 16) {
-                float v[16];
-                tmem_ld16(tmem + lane_off + kAccCol + a * 128 + n0, v);
+            // unpooled outputs go through shared memory: one store instruction then
+            // covers 4 rows x 128 bytes instead of 32 rows x 16 bytes
+            float *stage = epi_stage[qd];
+            const bool vec = DENSE || (p.N & 3) == 0;
+            if (!(!DENSE && p.pool))
+                epi_ptr[qd][lane] = ri.ok ? yrow + (DENSE ? 0 : ((int64_t)ri.oy * p.ow + ri.ox) * p.N) : nullptr;
+            for (int n0 = 0; n0 < Nt; n0 += 32) {
+                const int nc = min(32, Nt - n0);
+                float v[32];
 #pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const int n = n_base + n0 + e;
-                    const float zz = (ri.ok && n < p.N) ? v[e] + bias_sh[n0 + e] : 0.f;
-                    if (p.z && ri.ok && n < p.N) {
-                        if (DENSE) p.z[ri.row * p.z_stride + n] = zz;
-                        else p.z[ri.row * p.z_stride + (int64_t)n * (p.oh * p.ow) + ri.oy * p.ow + ri.ox] = zz;
+                for (int h = 0; h < 32; h += 16) {
+                    if (h >= nc) break;
+                    float *vh = v + h;
+                    // the accumulator: the n_mma partials added in a fixed order
+                    const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_mma * p.acc_cols) + n0 + h;
+                    tmem_ld16(acc, vh);
+                    for (int w = 1; w < p.n_mma; ++w) {
+                        float u[16];
+                        tmem_ld16(acc + (uint32_t)(w * p.acc_cols), u);
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) vh[e] += u[e];
                     }
-                    float val = act_apply(p.act1, zz);
-                    if (!DENSE && p.has_add && ri.ok && n < p.N) {
-                        const float sv = n < p.sk_c
-                            ? srow[((int64_t)ri.oy * p.sk_stride * p.sk_w + ri.ox * p.sk_stride) * p.sk_c + n]
-                            : 0.f;
-                        val = act_apply(p.act2, val + sv);
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) vh[e] += bias_sh[n0 + h + e];   // padding channels hold 0
+                    if (p.z && ri.ok) {
+                        for (int e = 0; e < 16 && n_base + n0 + h + e < p.N; ++e) {
+                            const int n = n_base + n0 + h + e;
+                            if (DENSE) p.z[ri.row * p.z_stride + n] = vh[e];
+                            else p.z[ri.row * p.z_stride + (int64_t)n * (p.oh * p.ow) + ri.oy * p.ow + ri.ox] = vh[e];
+                        }
                     }
-                    v[e] = val;
+                    if (p.act1 == MURE_ACT_RELU) {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) vh[e] = act_apply(MURE_ACT_RELU, vh[e]);
+                    }
+                    if (!DENSE && p.has_add && ri.ok) {
+                        const float *sp = srow + ((int64_t)ri.oy * p.sk_stride * p.sk_w + ri.ox * p.sk_stride) * p.sk_c;
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const int n = n_base + n0 + h + e;
+                            const float sv = n < p.sk_c ? sp[n] : 0.f;
+                            vh[e] = act_apply(p.act2, vh[e] + sv);
+                        }
+                    }
+                    if (!DENSE && p.pool) {
+                        // lanes 4w .. 4w+3 hold the four positions of one pooling window
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const float w1 = __shfl_down_sync(0xffffffffu, vh[e], 1);
+                            const float w2 = __shfl_down_sync(0xffffffffu, vh[e], 2);
+                            const float w3 = __shfl_down_sync(0xffffffffu, vh[e], 3);
+                            if ((lane & 3) == 0) vh[e] = max4_first(vh[e], w1, w2, w3);
+                        }
+                        if (ri.ok && (lane & 3) == 0) {
+                            float *yo = yrow + ((int64_t)ri.py * p.pw + ri.px) * p.N + n_base + n0 + h;
+                            if (n_base + n0 + h + 15 < p.N && (p.N & 3) == 0) {
+#pragma unroll
+                                for (int c = 0; c < 4; ++c)
+                                    *reinterpret_cast<float4 *>(yo + 4 * c) =
+                                        make_float4(vh[4 * c], vh[4 * c + 1], vh[4 * c + 2], vh[4 * c + 3]);
+                            } else {
+#pragma unroll
+                                for (int e = 0; e < 16; ++e)
+                                    if (n_base + n0 + h + e < p.N) yo[e] = vh[e];
+                            }
+                        }
+                    }
                 }
-                if (!DENSE && p.pool) {
-                    // lanes 4w .. 4w+3 hold the four positions of one pooling window
+                if (!DENSE && p.pool) continue;
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        const float w1 = __shfl_down_sync(0xffffffffu, v[e], 1);
-                        const float w2 = __shfl_down_sync(0xffffffffu, v[e], 2);
-                        const float w3 = __shfl_down_sync(0xffffffffu, v[e], 3);
-                        if ((lane & 3) == 0) v[e] = max4_first(v[e], w1, w2, w3);
-                    }
-                    if (ri.ok && (lane & 3) == 0) {
-                        float *yo = yrow + ((int64_t)ri.py * p.pw + ri.px) * p.N;
+                for (int c = 0; c < 8; ++c)
+                    *reinterpret_cast<float4 *>(stage + lane * kEpiStride + 4 * c) =
+                        make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                __syncwarp();
 #pragma unroll
-                        for (int e = 0; e < 16; ++e)
-                            if (n_base + n0 + e < p.N) yo[n_base + n0 + e] = v[e];
-                    }
-                } else if (ri.ok) {
-                    float *yo = yrow + (DENSE ? 0 : ((int64_t)ri.oy * p.ow + ri.ox) * p.N);
-                    const int nb = n_base + n0;
-                    if (nb + 15 < p.N && ((p.N & 3) == 0)) {
-#pragma unroll
-                        for (int c = 0; c < 4; ++c)
-                            *reinterpret_cast<float4 *>(yo + nb + 4 * c) =
-                                make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < 16; ++e)
-                            if (nb + e < p.N) yo[nb + e] = v[e];
+                for (int k = 0; k < 8; ++k) {
+                    const int rr = 4 * k + (lane >> 3), c4 = lane & 7;
+                    float *dst = epi_ptr[qd][rr];
+                    const int n = n_base + n0 + 4 * c4;
+                    if (dst && 4 * c4 < nc && n < p.N) {
+                        const float4 val = *reinterpret_cast<const float4 *>(stage + rr * kEpiStride + 4 * c4);
+                        if (vec && n + 3 < p.N) {
+                            *reinterpret_cast<float4 *>(dst + n) = val;
+                        } else {
+                            dst[n] = val.x;
+                            if (n + 1 < p.N) dst[n + 1] = val.y;
+                            if (n + 2 < p.N) dst[n + 2] = val.z;
+                            if (n + 3 < p.N) dst[n + 3] = val.w;
+                        }
                     }
                 }
+                __syncwarp();
             }
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
         }
-    } else if (warp == 8) {
+    } else if (warp < 11) {
         // ------------------------------------------------------------------ MMA --
-        if (lane == 0) {
+        // a K-step's MMAs (K8 step ks, product term) are dealt round-robin to the n_mma
+        // issuing warps, each into its own partial accumulator: one thread issues an MMA
+        // only about every 120 cycles, whatever N is, so narrow layers need several
+        const int w = warp - 8;
+        if (lane == 0 && w < p.n_mma) {
+            const int nmma = p.n_mma;
             const uint32_t id = idesc_tf32(kTileM, Nt);
             bool ok = true;
-            if (p.b_resident) ok = wait_phase(smem_u32(&bar_bfull[0]), 0, abort_flag);
+            if (p.b_resident) ok = wait_phase<32>(smem_u32(&bar_bfull[0]), 0, abort_flag);
+            const uint64_t desc_b0 = sw128_desc(b_region);
+            const uint32_t b_step16 = b_step >> 4, lo16 = (uint32_t)Nt * 128 >> 4;
             int t = 0, sb = 0;
             uint32_t t_wraps = 0, b_wraps = 0;
             for (int64_t i = 0; ok && i < my_tiles; ++i) {
                 const int a = (int)(i & 1);
-                if (i >= 2 && !wait_phase(smem_u32(&bar_accempty[a]), (uint32_t)(((i >> 1) - 1) & 1), abort_flag)) break;
+                if (i >= 2 && !wait_phase<32>(smem_u32(&bar_accempty[a]), (uint32_t)(((i >> 1) - 1) & 1), abort_flag)) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                const uint32_t d = tmem + kAccCol + a * 128;
+                const uint32_t d = tmem + (uint32_t)((a * nmma + w) * p.acc_cols);
                 for (int kt = 0; kt < nK; ++kt) {
-                    if (!wait_phase(smem_u32(&bar_afull[t]), t_wraps & 1, abort_flag)) { ok = false; break; }
-                    uint32_t bs;
-                    if (p.b_resident) {
-                        bs = b_region + (uint32_t)kt * b_step;
-                    } else {
-                        if (!wait_phase(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
-                        bs = b_region + (uint32_t)sb * b_step;
-                    }
+                    if (!wait_phase<32>(smem_u32(&bar_afull[t]), t_wraps & 1, abort_flag)) { ok = false; break; }
+                    if (!p.b_resident &&
+                        !wait_phase<32>(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                    const uint32_t ta = tmem + kACol + t * kAColsPerStage;
-#pragma unroll
-                    for (int ks = 0; ks < kTileK / 8; ++ks) {
-                        const uint32_t first = (kt > 0 || ks > 0) ? 1u : 0u;
-                        const uint64_t bh = sw128_desc(bs + ks * 32);
-                        if (THREE) {
-                            const uint64_t bl = sw128_desc(bs + (uint32_t)Nt * 128 + ks * 32);
-                            mma_tf32_ts(d, ta + 32 + ks * 8, bh, id, first);   // a_lo * b_hi
-                            mma_tf32_ts(d, ta + ks * 8, bl, id, 1u);           // a_hi * b_lo
-                            mma_tf32_ts(d, ta + ks * 8, bh, id, 1u);           // a_hi * b_hi
-                        } else {
-                            mma_tf32_ts(d, ta + ks * 8, bh, id, first);        // a_hi * b_hi
-                        }
-                    }
+                    const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
+                    mma_share<THREE>(nmma, w, d, tmem + kACol + t * kAColsPerStage, dh, dl, id, kt > 0 ? 1u : 0u);
                     mma_commit(smem_u32(&bar_aempty[t]));
                     if (++t == kNT) { t = 0; ++t_wraps; }
                     if (!p.b_resident) {
@@ -603,7 +886,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                 if (!ok) break;
                 mma_commit(smem_u32(&bar_accfull[a]));
             }
-            // every MMA this thread issued has finished before the teardown
+            // every MMA of every issuing warp has finished before the teardown
             mma_commit(smem_u32(&bar_drain));
             wait_phase_drain(smem_u32(&bar_drain), 0);
         }
@@ -622,7 +905,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                 int sb = 0, kt = 0;
                 uint32_t wraps = 0;
                 for (; j < total; ++j) {
-                    if (wraps >= 1 && !wait_phase(smem_u32(&bar_bempty[sb]), (wraps - 1) & 1, abort_flag)) break;
+                    if (wraps >= 1 && !wait_phase<64>(smem_u32(&bar_bempty[sb]), (wraps - 1) & 1, abort_flag)) break;
                     mbar_expect_tx(smem_u32(&bar_bfull[sb]), b_step);
                     bulk_g2s(b_region + (uint32_t)sb * b_step, (const unsigned char *)wslice + (size_t)kt * b_step,
                              b_step, smem_u32(&bar_bfull[sb]));
@@ -673,10 +956,21 @@ int tc_supported(const Stage &S)
     return S.kind == MURE_NODE_CONV2D;
 }
 
+// Whether a convolution has the small-image mode's geometry.
+int tc_small_geometry(const Stage &S)
+{
+    using G = SmallConv;
+    return S.kind == MURE_NODE_CONV2D && S.ih == G::IH && S.iw == G::IW && S.ic == G::IC && S.kh == G::KH &&
+           S.kw == G::KW && S.stride == 1 && S.pad == 0 && S.pool && !S.has_add && !S.gap && S.oc >= 16 &&
+           S.oc <= kSlice;
+}
+
 // Whether the tensor-core kernel can fetch a first-suffix overlay itself: at most
 // kOvMax patch values per row and K-step (dense: at most 4 mutated channels).
-int tc_overlay_inline(const Stage &S, const Overlay &ov)
+int tc_overlay_inline(const Stage &S, const Overlay &ov, int64_t groups)
 {
+    if (S.tc_small)
+        return ov.kmax <= SmallConv::MAXQ && groups <= SmallConv::MAXG && ov.cells == SmallConv::CELLS;
     if (S.kind == MURE_NODE_DENSE) {
         if (ov.kmax > 4) return 0;
         const int per_slot = std::min(ov.cells, (kTileK + ov.ch - 1) / ov.ch + 1);
@@ -740,8 +1034,13 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     p.b_resident = slice_bytes <= 96 * 1024;
     const size_t b_bytes = p.b_resident ? slice_bytes : kNB * b_step;
     // at least 116 KiB so that one CTA (holding all 512 tensor-memory columns) runs per SM
-    const size_t ov_bytes = p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0;
-    const size_t smem = std::max<size_t>(1024 + b_bytes + (size_t)kNA * kStageA + ov_bytes, 116 * 1024);
+    const size_t a_bytes = S.tc_small ? (size_t)SmallConv::BYTES
+                                      : (size_t)kNA * kStageA + (p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0);
+    const size_t smem = std::max<size_t>(1024 + b_bytes + a_bytes, 116 * 1024);
+    // partial accumulators: two sets of n_mma in columns 0..255; a function of the layer
+    // alone, so a row's arithmetic never depends on the batch
+    p.acc_cols = round_up32(nt_max);
+    p.n_mma = std::max(1, std::min(3, kACol / (2 * p.acc_cols)));
     const int64_t M = (int64_t)rm.R * p.P;
     const int64_t tiles = (M + kTileM - 1) / kTileM;
     static int n_sm = 0;
@@ -757,8 +1056,9 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, kThreads, smem, s>>>(p);
     };
-    if (dense) { if (three) go(k_tc_gemm<true, true>); else go(k_tc_gemm<true, false>); }
-    else { if (three) go(k_tc_gemm<false, true>); else go(k_tc_gemm<false, false>); }
+    if (dense) { if (three) go(k_tc_gemm<0, true>); else go(k_tc_gemm<0, false>); }
+    else if (S.tc_small) { if (three) go(k_tc_gemm<2, true>); else go(k_tc_gemm<2, false>); }
+    else { if (three) go(k_tc_gemm<1, true>); else go(k_tc_gemm<1, false>); }
     int launches = 1;
     if (S.gap) launches += launch_gap(gap_tmp, map_stride, mh * mw, S.oc, rm.R, y_out, y_stride, s);
     return launches;
