@@ -129,6 +129,7 @@ struct PatchValsParams {
     float *out; int64_t out_stride;
     int warp_dot;        // 1: fan-in sums split across a warp (layers with < 32 positions)
     int skip_dot_ops;    // 1: GF / WS values come from k_patch_dot
+    int only_dot_ops;    // 1: the other operators come from k_patch_vals_staged
 };
 
 struct SlotCtx {
@@ -226,6 +227,7 @@ __global__ void __launch_bounds__(256) k_patch_vals(const PatchValsParams p)
     const int op = p.pa.op[g];
     const bool dot = op == MURE_OP_GF || op == MURE_OP_WS;
     if (dot && p.skip_dot_ops) return;
+    if (!dot && p.only_dot_ops) return;
     const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
     SlotCtx d;
     d.op = op;
@@ -283,6 +285,47 @@ __global__ void __launch_bounds__(256) k_patch_vals(const PatchValsParams p)
     }
 }
 
+// The operators without a fan-in sum (NAI, NEB, NS) of a convolution layer in
+// memoized mode, one input per block: the input's cached pre-activation maps are
+// staged in shared memory once and every mutant slot of the batch reads its channel
+// there (the mutants of a batch share the inputs).  The arithmetic is slot_post's,
+// so the values equal those of k_patch_vals bit for bit.
+__global__ void __launch_bounds__(256) k_patch_vals_staged(const PatchValsParams p)
+{
+    extern __shared__ float zs[];   // [oc][oh * ow] of the block's input, then the cell table
+    const int P = p.oh * p.ow, nz = p.oc * P;
+    int *coff = reinterpret_cast<int *>(zs + nz);   // cell -> top-left position of its window
+    const int tl = blockIdx.x;
+    const float *z = p.z + (p.t0 + tl) * p.z_stride;
+    for (int i = threadIdx.x; i < nz; i += blockDim.x) zs[i] = z[i];
+    for (int c = threadIdx.x; c < p.mcells; c += blockDim.x)
+        coff[c] = p.pool ? 2 * (c / p.mcw) * p.ow + 2 * (c % p.mcw) : c;
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int sl = warp; sl < p.G * p.kmax; sl += blockDim.x >> 5) {
+        const int g = sl / p.kmax, q = sl - g * p.kmax;
+        if (q >= p.pa.n_neurons[g]) continue;
+        const int op = p.pa.op[g];
+        if (op == MURE_OP_GF || op == MURE_OP_WS) continue;
+        const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
+        const int sj = op == MURE_OP_NS ? ids[q ^ 1] : ids[q];
+        const float *zc = zs + sj * P;
+        float *o = p.out + ((int64_t)g * p.T + tl) * p.out_stride + q * p.cells;
+        auto post = [&](float zz) {
+            if (op == MURE_OP_NAI) zz = -zz;
+            return op == MURE_OP_NEB ? 0.f : act_apply(p.act1, zz);
+        };
+        if (p.pool) {
+            for (int c = lane; c < p.cells; c += 32) {
+                const int b = coff[c];
+                o[c] = max4_first(post(zc[b]), post(zc[b + 1]), post(zc[b + p.ow]), post(zc[b + p.ow + 1]));
+            }
+        } else {
+            for (int c = lane; c < p.cells; c += 32) o[c] = post(zc[coff[c]]);
+        }
+    }
+}
+
 int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *out,
                       int64_t out_stride, cudaStream_t s, bool skip_dot_ops)
 {
@@ -311,8 +354,20 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     const int64_t gy = std::max<int64_t>(1, std::min<int64_t>(rm.T, (152 * 16 + gx - 1) / gx));
     const dim3 grid((unsigned)gx, (unsigned)gy);
     const size_t smem = (S.gap && !p.warp_dot) ? 8 * (size_t)p.mcells * sizeof(float) : 0;
+    // memoized convolution layers whose maps fit in shared memory: the non-dot
+    // operators per input, staged
+    const size_t staged_smem = ((size_t)S.oc * S.oh * S.ow + p.mcells) * 4;
+    const bool staged = z.per_input && S.kind == MURE_NODE_CONV2D && !S.has_add && !S.gap && p.mcells >= 32 &&
+                        staged_smem <= 48 * 1024;
+    int launches = 0;
+    if (staged) {
+        k_patch_vals_staged<<<(unsigned)rm.T, 256, staged_smem, s>>>(p);
+        ++launches;
+        if (skip_dot_ops) return launches;
+        p.only_dot_ops = 1;
+    }
     k_patch_vals<<<grid, 256, smem, s>>>(p);
-    return 1;
+    return launches + 1;
 }
 
 // Materialise rows: out = base with the overlay's channels written in (for suffix
