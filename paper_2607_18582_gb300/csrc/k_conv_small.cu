@@ -225,6 +225,7 @@ struct PatchDotParams {
     const float *e_all;
     float *out; int64_t out_stride;
     int cells, rows_per_block;
+    int oc;
 };
 
 template <int KH, int KW, int IC, int WP, int HP, int PAD, bool POOL, int KMAX>
@@ -286,6 +287,119 @@ __global__ void __launch_bounds__(256) k_patch_dot(const PatchDotParams p)
     }
 }
 
+// The same values in memoized mode, one input per block: the input's padded map and
+// its pre-activation maps are staged once, and every GF / WS slot of the batch (the
+// mutants share the inputs) is computed from there.  A thread takes one output cell
+// (a pooling window: four positions) for SG slots, so each filter tap costs 4 + SG
+// shared loads for 4 * SG FMAs.  Every sum is the same ascending fp32 chain as in
+// k_patch_dot, so the two kernels agree bit for bit.
+template <int KH, int KW, int IC, int WP, int HP, int PAD, bool POOL, int KMAX>
+__global__ void __launch_bounds__(256) k_patch_dot_in(const PatchDotParams p)
+{
+    constexpr int K = KH * KW * IC;
+    constexpr int TILE = HP * WP * IC;
+    constexpr int SG = 4;          // slots per thread
+    constexpr int SMAX = 32;       // slots whose filters are staged at a time
+    constexpr int NPOS = POOL ? 4 : 1;
+    extern __shared__ __align__(16) float sm[];
+    const int P = p.oh * p.ow;
+    float *xs = sm;                       // [TILE] zero-padded input map
+    float *es = xs + TILE;                // [SMAX][K] filter deltas
+    float *zsm = es + SMAX * K;           // [oc][P] pre-activation maps
+    __shared__ int sl_g[SMAX], sl_q[SMAX], sl_j[SMAX];
+    __shared__ int n_sl;
+    const int tl = blockIdx.x;
+    const int64_t t = p.t0 + tl;
+    const float *xin = p.x + t * p.x_stride;
+    for (int i = threadIdx.x; i < TILE; i += blockDim.x) {
+        const int ci = i % IC, pix = i / IC, px = pix % WP, py = pix / WP;
+        const int iy = py - PAD, ix = px - PAD;
+        xs[i] = ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw) ? __ldg(xin + (iy * p.iw + ix) * IC + ci)
+                                                                                  : 0.f;
+    }
+    const float *zin = p.z + t * p.z_stride;
+    for (int i = threadIdx.x; i < p.oc * P; i += blockDim.x) zsm[i] = __ldg(zin + i);
+    const int pw = POOL ? p.ow / 2 : p.ow;
+    // the batch's GF / WS slots, SMAX at a time (walking the groups in order)
+    int g_next = 0, q_next = 0;
+    for (;;) {
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int n = 0;
+            while (n < SMAX && g_next < p.G) {
+                const int op = p.op[g_next];
+                const int k = min(p.n_neurons[g_next], KMAX);
+                if ((op == MURE_OP_GF || op == MURE_OP_WS) && q_next < k) {
+                    sl_g[n] = g_next; sl_q[n] = q_next; sl_j[n] = p.ids[p.neuron_off[g_next] + q_next];
+                    ++n;
+                    ++q_next;
+                } else {
+                    ++g_next;
+                    q_next = 0;
+                }
+            }
+            n_sl = n;
+        }
+        __syncthreads();
+        const int ns = n_sl;
+        if (ns == 0) break;
+        for (int i = threadIdx.x; i < ns * K; i += blockDim.x) {
+            const int sl = i / K, kk = i - sl * K;
+            es[i] = __ldg(p.e_all + p.patch_off[sl_g[sl]] + (int64_t)sl_q[sl] * K + kk);
+        }
+        __syncthreads();
+        const int groups = (ns + SG - 1) / SG;
+        for (int it = threadIdx.x; it < groups * p.cells; it += blockDim.x) {
+            const int sg = it / p.cells, c = it - sg * p.cells;
+            const int cy = c / pw, cx = c - cy * pw;
+            int off[NPOS];
+#pragma unroll
+            for (int s2 = 0; s2 < NPOS; ++s2) {
+                const int oy = POOL ? 2 * cy + (s2 >> 1) : cy, ox = POOL ? 2 * cx + (s2 & 1) : cx;
+                off[s2] = (oy * WP + ox) * IC;
+            }
+            const int nsg = min(SG, ns - sg * SG);
+            const float *e0 = es + sg * SG * K;
+            float acc[SG][NPOS];
+#pragma unroll
+            for (int a = 0; a < SG; ++a)
+#pragma unroll
+                for (int s2 = 0; s2 < NPOS; ++s2) acc[a][s2] = 0.f;
+#pragma unroll 1
+            for (int ky = 0; ky < KH; ++ky)
+#pragma unroll
+                for (int kx = 0; kx < KW; ++kx)
+#pragma unroll
+                    for (int ci = 0; ci < IC; ++ci) {
+                        const int kk = (ky * KW + kx) * IC + ci, xo = (ky * WP + kx) * IC + ci;
+                        float xv[NPOS];
+#pragma unroll
+                        for (int s2 = 0; s2 < NPOS; ++s2) xv[s2] = xs[off[s2] + xo];
+#pragma unroll
+                        for (int a = 0; a < SG; ++a) {
+                            const float ev = e0[(a < nsg ? a : 0) * K + kk];
+#pragma unroll
+                            for (int s2 = 0; s2 < NPOS; ++s2) acc[a][s2] = fmaf(ev, xv[s2], acc[a][s2]);
+                        }
+                    }
+#pragma unroll
+            for (int a = 0; a < SG; ++a) {
+                if (a >= nsg) break;
+                const int sl = sg * SG + a;
+                const float *zr = zsm + sl_j[sl] * P;
+                float v4[NPOS];
+#pragma unroll
+                for (int s2 = 0; s2 < NPOS; ++s2) {
+                    const int oy = POOL ? 2 * cy + (s2 >> 1) : cy, ox = POOL ? 2 * cx + (s2 & 1) : cx;
+                    v4[s2] = act_apply(p.act1, zr[oy * p.ow + ox] + acc[a][s2]);
+                }
+                const int64_t r = (int64_t)sl_g[sl] * p.T + tl;
+                p.out[r * p.out_stride + sl_q[sl] * p.cells + c] = POOL ? max4_first(v4[0], v4[1], v4[2], v4[3]) : v4[0];
+            }
+        }
+    }
+}
+
 namespace {
 template <int KH, int KW, int IC, int WP, int HP, int PAD, bool POOL>
 int launch_dot(const Stage &S, Src z, Src x, RowMap rm, const PatchArgs &pa, int kmax, float *out, int64_t out_stride,
@@ -302,6 +416,17 @@ int launch_dot(const Stage &S, Src z, Src x, RowMap rm, const PatchArgs &pa, int
     p.out = out; p.out_stride = out_stride;
     p.cells = POOL ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
     p.rows_per_block = 8;
+    p.oc = S.oc;
+    if (z.per_input && x.per_input) {
+        // memoized: one block per input
+        const size_t smem2 = ((size_t)HP * WP * IC + 32 * (size_t)KH * KW * IC + (size_t)S.oc * S.oh * S.ow) * sizeof(float);
+        if (smem2 <= 96 * 1024) {
+            cudaFuncSetAttribute(k_patch_dot_in<KH, KW, IC, WP, HP, PAD, POOL, KMAX>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
+            k_patch_dot_in<KH, KW, IC, WP, HP, PAD, POOL, KMAX><<<(unsigned)rm.T, 256, smem2, s>>>(p);
+            return 1;
+        }
+    }
     const size_t smem = ((size_t)KMAX * KH * KW * IC + (size_t)p.rows_per_block * HP * WP * IC) * sizeof(float);
     cudaFuncSetAttribute(k_patch_dot<KH, KW, IC, WP, HP, PAD, POOL, KMAX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
