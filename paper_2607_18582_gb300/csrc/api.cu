@@ -15,10 +15,9 @@ using namespace mure;
 namespace {
 
 // MURE_TC_CONV=1 puts every convolution of a TF32X3 model on the tensor cores.
-// MURE_TC_CONV: in the tensor-core modes the LeNet-size convolution keeps its
-// CUDA-core kernel (faster there) unless this is "small" (the small-image mode) or
-// "generic" (the implicit-GEMM producers; the two tensor-core forms give identical
-// bits).
+// MURE_TC_CONV: in the tensor-core modes the LeNet-size convolution runs in the
+// small-image mode (a GEMM row per pooling window); "0" keeps its CUDA-core kernel,
+// "generic" runs it through the implicit-GEMM producers (one row per position).
 std::string tc_conv_env()
 {
     const char *e = getenv("MURE_TC_CONV");
@@ -982,11 +981,11 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
         }
         // tensor-core modes: layers before the output layer with >= 16 outputs run on
         // the tensor cores (3xTF32, or one TF32 MMA in the reduced-precision variant);
-        // the LeNet-size convolution keeps its CUDA-core kernel unless MURE_TC_CONV asks
+        // the LeNet-size convolution takes the small-image mode (MURE_TC_CONV above)
         for (int l = 0; l + 1 < m->L; ++l) {
             Stage &S = m->st[l];
             const std::string env = tc_conv_env();
-            const bool small = tc_small_geometry(S) && (env == "small" || env == "generic");
+            const bool small = tc_small_geometry(S) && env != "0";
             const bool take = tc_supported(S) && (S.kind == MURE_NODE_DENSE || S.variant == 0 || small);
             if (take && d->precision == MURE_PREC_TF32X3) S.tc = 1;
             else if (take && d->precision == MURE_PREC_TF32) S.tc = 2;
@@ -1015,7 +1014,13 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             CK(c, cudaStreamSynchronize(c->stream));  // Wt is reused
             if (S.tc) {
                 S.Wtc = (float *)dalloc(c, tc_weight_floats(S) * 4);
-                c->launches += launch_swizzle_weights(S, S.Wtc, c->stream);
+                const int64_t ntmp = tc_swizzle_tmp_floats(S);
+                float *tmp = ntmp ? (float *)dalloc(c, ntmp * 4) : nullptr;
+                c->launches += launch_swizzle_weights(S, S.Wtc, tmp, c->stream);
+                if (tmp) {
+                    CK(c, cudaStreamSynchronize(c->stream));
+                    dfree(c, tmp);
+                }
                 check_launch(c);
             }
         }

@@ -456,20 +456,28 @@ __device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, co
 }
 
 // The small-image convolution mode: 5x5 filters over a 14 x 14 x 6 map, stride 1, no
-// padding, 2x2 max pool (LeNet-5's second convolution).  The producers stage whole
-// input maps in shared memory (copied with coalesced cp.async) and gather each GEMM
-// row's receptive field from there with compile-time offsets, two channels per load;
-// a 6-channel map is no fit for the 16-byte copies of the generic path.  A tile of
-// 128 GEMM rows spans at most NIMG maps.
+// padding, 16 output channels, 2x2 max pool (LeNet-5's second convolution).  A GEMM
+// row is a pooling window rather than an output position: K is the window's 6 x 6 x 6
+// receptive field (216) and N = 4 positions x 16 channels = 64, with the weights
+// expanded once (zeros where a tap is outside a position's 5 x 5 filter).  With only
+// 16 output channels a per-position GEMM would have N = 16, where the MMA issue rate,
+// not the tensor core, is the limit; per window the layer takes a third of the MMA
+// instructions and of the gathers, and the epilogue pools inside each row.  The
+// producers stage whole input maps in shared memory (coalesced cp.async) and gather
+// each row's receptive field from there with compile-time offsets, 16 bytes per load
+// (a receptive-field row is 36 consecutive, 16-byte-aligned values).  A tile of 128
+// rows spans at most NIMG maps.
 struct SmallConv {
-    static constexpr int IH = 14, IW = 14, IC = 6, KH = 5, KW = 5, OH = 10, OW = 10, PW = 5;
-    static constexpr int P = 4 * (OH / 2) * (OW / 2);        // GEMM rows per map (window-major)
-    static constexpr int K = KH * KW * IC, NKT = (K + kTileK - 1) / kTileK;
+    static constexpr int IH = 14, IW = 14, IC = 6, KH = 5, KW = 5, OH = 10, OW = 10, PW = 5, OC = 16;
+    static constexpr int KU = KH + 1;                         // receptive field of a window: KU x KU
+    static constexpr int P = (OH / 2) * (OW / 2);             // GEMM rows (windows) per map
+    static constexpr int K = KU * KU * IC, NKT = (K + kTileK - 1) / kTileK;
+    static constexpr int N = 4 * OC;                          // GEMM columns: (window position, channel)
     static constexpr int CELLS = IH * IW;                     // overlay cells of a mutated channel
     static constexpr uint32_t IMG_B = IH * IW * IC * 4;       // bytes of one staged map
     static constexpr int CH16 = IMG_B / 16;
-    static constexpr int MAXQ = 4;                            // mutated channels per row (overlay)
-    static constexpr int MAXG = 1024;                         // mutants per batch (overlay table)
+    static constexpr int MAXQ = 2;                            // mutated channels per row (overlay)
+    static constexpr int MAXG = 256;                          // mutants per batch (overlay table)
     static constexpr int NIMG = (kTileM - 1) / P + 2;         // maps per tile, at most
     static constexpr uint32_t BUF_B = NIMG * IMG_B;           // one buffer of staged maps
     static constexpr uint32_t OVST_B = NIMG * MAXQ * CELLS * 4;   // one buffer of staged patch values
@@ -478,25 +486,28 @@ struct SmallConv {
 };
 static_assert(SmallConv::IMG_B % 16 == 0, "maps are copied in 16-byte chunks");
 static_assert((SmallConv::CELLS * 4) % 16 == 0, "patch values are copied in 16-byte chunks");
+static_assert((SmallConv::KU * SmallConv::IC) % 4 == 0 && (SmallConv::IW * SmallConv::IC * 4) % 16 == 0,
+              "receptive-field rows are 16-byte aligned runs of whole 4-value chunks");
 
 __device__ __forceinline__ void named_bar_producers() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-// K-step KT of a small-image GEMM row: 16 channel pairs at compile-time offsets from
-// the row's receptive-field origin `base` (k = (ky, kx, ci) with ci even, so every pair
-// is 8-byte aligned).
+// K-step KT of a window row: 8 chunks of 4 values at compile-time offsets from the
+// window's receptive-field origin `base`, k = (wy, wx, ci).
 template <int KT>
 __device__ __forceinline__ void small_gather(uint32_t base, float (&v)[kTileK])
 {
     using G = SmallConv;
+    constexpr int RUN = G::KU * G::IC;   // values per receptive-field row
 #pragma unroll
-    for (int e = 0; e < kTileK / 2; ++e) {
-        const int k = KT * kTileK + 2 * e;
+    for (int c = 0; c < kTileK / 4; ++c) {
+        const int k = KT * kTileK + 4 * c;
         if (k < G::K) {
-            const uint32_t off = (uint32_t)(((k / (G::KW * G::IC)) * G::IW + (k / G::IC) % G::KW) * G::IC + k % G::IC) * 4;
-            asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v[2 * e]), "=f"(v[2 * e + 1]) : "r"(base + off));
+            const uint32_t off = (uint32_t)((k / RUN) * G::IW * G::IC + k % RUN) * 4;
+            asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                         : "=f"(v[4 * c]), "=f"(v[4 * c + 1]), "=f"(v[4 * c + 2]), "=f"(v[4 * c + 3])
+                         : "r"(base + off));
         } else {
-            v[2 * e] = 0.f;
-            v[2 * e + 1] = 0.f;
+            v[4 * c] = v[4 * c + 1] = v[4 * c + 2] = v[4 * c + 3] = 0.f;
         }
     }
 }
@@ -555,7 +566,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                      "r"(512));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
-    for (int n = threadIdx.x; n < kSlice; n += kThreads) bias_sh[n] = n_base + n < p.N ? p.b[n_base + n] : 0.f;
+    for (int n = threadIdx.x; n < kSlice; n += kThreads) {
+        if (MODE == 2) bias_sh[n] = n < SmallConv::N ? p.b[n % SmallConv::OC] : 0.f;
+        else bias_sh[n] = n_base + n < p.N ? p.b[n_base + n] : 0.f;
+    }
     // small-image mode: staged maps, staged patch values, the batch's mutated-channel table
     const uint32_t img_region = a_region;
     const uint32_t ovst_region = img_region + 2 * SmallConv::BUF_B;
@@ -674,13 +688,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                     }
                     named_bar_producers();
                 }
-                // this thread's GEMM row: map, pooling window, position in the window
+                // this thread's GEMM row: map and pooling window
                 const int64_t m = m0 + r;
                 const bool in = m < M;
                 const int64_t row = in ? m / G::P : row0;
-                const int q = in ? (int)(m - row * G::P) : 0;
-                const int w = q >> 2, sub = q & 3;
-                const int oy = 2 * (w / G::PW) + (sub >> 1), ox = 2 * (w % G::PW) + (sub & 1);
+                const int w = in ? (int)(m - row * G::P) : 0;
+                const int oy = 2 * (w / G::PW), ox = 2 * (w % G::PW);
                 const uint32_t base = buf + (uint32_t)(row - row0) * G::IMG_B + (uint32_t)((oy * G::IW + ox) * G::IC) * 4;
                 SmallSteps<0>::run(base, push, ok);
             }
@@ -748,6 +761,50 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             if (!warp_wait_phase<64>(smem_u32(&bar_accfull[a]), (uint32_t)((i >> 1) & 1), abort_flag)) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const int64_t tile = blockIdx.x + i * gridDim.x;
+            if constexpr (MODE == 2) {
+                // a pooling window: columns n = s * OC + c for its position s = 2 dy + dx
+                using G = SmallConv;
+                const int64_t m = tile * kTileM + qd * 32 + lane;
+                const bool ok = m < M;
+                const int64_t row = ok ? m / G::P : 0;
+                const int w = ok ? (int)(m - row * G::P) : 0;
+                const int py = w / G::PW, px = w % G::PW;
+                const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_mma * p.acc_cols);
+                float v[G::N];
+#pragma unroll
+                for (int n0 = 0; n0 < G::N; n0 += 16) {
+                    tmem_ld16(acc + n0, v + n0);
+                    for (int w2 = 1; w2 < p.n_mma; ++w2) {
+                        float u[16];
+                        tmem_ld16(acc + (uint32_t)(w2 * p.acc_cols) + n0, u);
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) v[n0 + e] += u[e];
+                    }
+                }
+                float o[G::OC];
+#pragma unroll
+                for (int c = 0; c < G::OC; ++c) {
+                    float v4[4];
+#pragma unroll
+                    for (int s4 = 0; s4 < 4; ++s4) {
+                        const float zz = v[s4 * G::OC + c] + bias_sh[c];
+                        if (p.z && ok)
+                            p.z[row * p.z_stride + (int64_t)c * (G::OH * G::OW) + (2 * py + (s4 >> 1)) * G::OW + 2 * px + (s4 & 1)] = zz;
+                        v4[s4] = act_apply(p.act1, zz);
+                    }
+                    o[c] = max4_first(v4[0], v4[1], v4[2], v4[3]);
+                }
+                if (ok) {
+                    float *yo = p.y + row * p.y_stride + (int64_t)w * G::OC;
+#pragma unroll
+                    for (int c = 0; c < G::OC; c += 4)
+                        *reinterpret_cast<float4 *>(yo + c) = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+                }
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
+                continue;
+            }
             const RowInfo ri = row_info<DENSE, false>(p, tile * kTileM + qd * 32 + lane);
             const float *srow = nullptr;
             if (p.has_add && ri.ok) srow = p.skip + (p.skip_per_input ? p.t0 + ri.row % p.T : ri.row) * p.skip_stride;
@@ -961,8 +1018,7 @@ int tc_small_geometry(const Stage &S)
 {
     using G = SmallConv;
     return S.kind == MURE_NODE_CONV2D && S.ih == G::IH && S.iw == G::IW && S.ic == G::IC && S.kh == G::KH &&
-           S.kw == G::KW && S.stride == 1 && S.pad == 0 && S.pool && !S.has_add && !S.gap && S.oc >= 16 &&
-           S.oc <= kSlice;
+           S.kw == G::KW && S.stride == 1 && S.pad == 0 && S.pool && !S.has_add && !S.gap && S.oc == G::OC;
 }
 
 // Whether the tensor-core kernel can fetch a first-suffix overlay itself: at most
@@ -981,22 +1037,53 @@ int tc_overlay_inline(const Stage &S, const Overlay &ov, int64_t groups)
     return ov.kmax * pixels <= kOvMax;
 }
 
+// The GEMM's N and K: the small-image mode multiplies by the window-expanded weights.
+static int gemm_n(const Stage &S) { return S.tc_small ? SmallConv::N : S.oc; }
+static int gemm_k(const Stage &S) { return S.tc_small ? SmallConv::K : S.K; }
+
+// W [OC][(ky, kx, ci)] -> W' [(s, c)][(wy, wx, ci)]: the filter of window position
+// s = 2 dy + dx placed at offset (dy, dx) in the window's receptive field.
+__global__ void k_expand_window_weights(const float *__restrict__ W, float *out)
+{
+    using G = SmallConv;
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= G::N * G::K) return;
+    const int n = i / G::K, k = i % G::K;
+    const int sidx = n / G::OC, c = n % G::OC, dy = sidx >> 1, dx = sidx & 1;
+    const int wy = k / (G::KU * G::IC), wx = (k / G::IC) % G::KU, ci = k % G::IC;
+    const int ky = wy - dy, kx = wx - dx;
+    out[i] = ((unsigned)ky < (unsigned)G::KH && (unsigned)kx < (unsigned)G::KW)
+                 ? W[(int64_t)c * (G::KH * G::KW * G::IC) + (ky * G::KW + kx) * G::IC + ci]
+                 : 0.f;
+}
+
 int64_t tc_weight_floats(const Stage &S)
 {
-    const int Np = round_up16(S.oc), Kp = round_up32(S.K), planes = S.tc == 1 ? 2 : 1;
+    const int Np = round_up16(gemm_n(S)), Kp = round_up32(gemm_k(S)), planes = S.tc == 1 ? 2 : 1;
     const int64_t slice = (int64_t)planes * kSlice * Kp;
     return slice * ((Np + kSlice - 1) / kSlice);
 }
 
-int launch_swizzle_weights(const Stage &S, float *out, cudaStream_t s)
+// tmp: scratch of SmallConv::N * SmallConv::K floats for the small-image mode (else unused).
+int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t s)
 {
-    const int Np = round_up16(S.oc), Kp = round_up32(S.K), planes = S.tc == 1 ? 2 : 1;
+    const int N = gemm_n(S), K = gemm_k(S);
+    const int Np = round_up16(N), Kp = round_up32(K), planes = S.tc == 1 ? 2 : 1;
     const int64_t n = (int64_t)Np * Kp;
+    int launches = 1;
+    const float *W = S.W;
+    if (S.tc_small) {
+        k_expand_window_weights<<<(N * K + 255) / 256, 256, 0, s>>>(S.W, tmp);
+        W = tmp;
+        ++launches;
+    }
     cudaMemsetAsync(out, 0, tc_weight_floats(S) * sizeof(float), s);
-    k_swizzle_weights<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(S.W, S.oc, S.K, Np, Kp, planes,
+    k_swizzle_weights<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(W, N, K, Np, Kp, planes,
                                                                    (int64_t)planes * kSlice * Kp, out);
-    return 1;
+    return launches;
 }
+
+int64_t tc_swizzle_tmp_floats(const Stage &S) { return S.tc_small ? (int64_t)SmallConv::N * SmallConv::K : 0; }
 
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
               int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov)
@@ -1011,6 +1098,10 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     p.pool = S.pool; p.pw = S.ow / 2;
     p.P = dense ? 1 : (S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : S.oh * S.ow);
     p.K = S.K; p.Kp = round_up32(S.K); p.N = S.oc; p.Np = round_up16(S.oc);
+    if (S.tc_small) {
+        p.P = SmallConv::P;
+        p.K = SmallConv::K; p.Kp = round_up32(SmallConv::K); p.Np = SmallConv::N;
+    }
     const bool three = S.tc == 1;
     const int planes = three ? 2 : 1;
     p.Wsw = S.Wtc;
@@ -1031,7 +1122,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     const int nt_max = std::min(kSlice, p.Np);
     const size_t b_step = (size_t)planes * nt_max * 128;
     const size_t slice_bytes = b_step * (p.Kp / kTileK);
-    p.b_resident = slice_bytes <= 96 * 1024;
+    p.b_resident = slice_bytes <= (S.tc_small ? 112 : 96) * 1024;
     const size_t b_bytes = p.b_resident ? slice_bytes : kNB * b_step;
     // at least 116 KiB so that one CTA (holding all 512 tensor-memory columns) runs per SM
     const size_t a_bytes = S.tc_small ? (size_t)SmallConv::BYTES

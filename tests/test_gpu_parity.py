@@ -302,28 +302,29 @@ def test_tf32_variant_verdicts(M, ctx, oracle_runs, name):
     assert agree >= 0.98, agree
 
 
+@pytest.mark.parametrize("mode", ["small", "generic"])
 @pytest.mark.parametrize("prec", ["tf32x3", "tf32"])
-def test_tensor_core_conv_on_small_layers(M, ctx, oracle_mod, monkeypatch, prec):
-    """LeNet's conv 6->16 on the tensor cores: the small-image mode (maps staged in
-    shared memory) and the implicit-GEMM producers feed the same MMAs, so they give
-    identical bits; 3xTF32 stays within the fp32 tolerance of the oracle.  With 100
-    GEMM rows per map, 128-row tiles straddle up to three maps."""
+def test_tensor_core_conv_on_small_layers(M, ctx, oracle_mod, monkeypatch, prec, mode):
+    """LeNet's conv 6->16 on the tensor cores, in the small-image mode (a GEMM row per
+    pooling window, N = 4 positions x 16 channels, maps staged in shared memory) and
+    through the implicit-GEMM producers: memoized == vanilla bit for bit, 3xTF32 within
+    the fp32 tolerance of the oracle, the TF32 variant's verdicts nearly all agree.
+    With 25 windows per map, 128-row tiles straddle up to seven maps."""
     w = wl.workload("lenet5", 130, 1)
     table = all_ops(w.model, 6, seed=51)
     ora = oracle_mod.vanilla(w.model, w.X, table)
-    monkeypatch.setenv("MURE_TC_CONV", "small")
-    small = M.mure_model_load(ctx, w.model, precision=prec)
-    monkeypatch.setenv("MURE_TC_CONV", "generic")
-    generic = M.mure_model_load(ctx, w.model, precision=prec)
+    monkeypatch.setenv("MURE_TC_CONV", mode)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
     monkeypatch.delenv("MURE_TC_CONV")
-    r = M.mure_eval_mutants(M.mure_build_prefix_cache(small, w.X), table, logits=True)
-    r2 = M.mure_eval_mutants(M.mure_build_prefix_cache(generic, w.X), table, logits=True)
-    assert np.array_equal(r["logits"].view(np.uint32), r2["logits"].view(np.uint32))
-    assert np.array_equal(r["kill_bits"], r2["kill_bits"])
-    v = M.mure_eval_vanilla(small, w.X, table, logits=True)
+    r = M.mure_eval_mutants(M.mure_build_prefix_cache(model, w.X), table, logits=True)
+    v = M.mure_eval_vanilla(model, w.X, table, logits=True)
     assert np.array_equal(v["logits"].view(np.uint32), r["logits"].view(np.uint32))
+    assert np.array_equal(v["kill_bits"], r["kill_bits"])
     if prec == "tf32x3":
         ok, worst = logits_close(r["logits"], ora["logits"])
         assert ok, worst
         bad, _ = compare_kills(r["kill_bits"], ora["kill_bits"], ora["orig_logits"], ora["logits"], len(w.X))
         assert bad == 0
+    else:
+        agree = (bits(r["kill_bits"], len(w.X)) == bits(ora["kill_bits"], len(w.X))).mean()
+        assert agree >= 0.98, agree
