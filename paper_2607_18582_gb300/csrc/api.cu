@@ -388,6 +388,7 @@ struct DevTable {
     int64_t n_jobs, patch_len;
     std::vector<int> kmax_layer;
     std::vector<int64_t> dot_prefix;   // [n+1] prefix sums of GF/WS neuron slots (group order)
+    int32_t *dslot = nullptr;          // [dot_prefix[n]] GF/WS slots in group order: (group, slot q)
     int expand_launches = 0;
 };
 
@@ -428,13 +429,19 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
     dt.dot_prefix.assign(n + 1, 0);
     for (int64_t k = 0; k < n; ++k)
         dt.dot_prefix[k + 1] = dt.dot_prefix[k] + ((op[k] == MURE_OP_GF || op[k] == MURE_OP_WS) ? nn[k] : 0);
+    std::vector<int32_t> dslot;
+    dslot.reserve(2 * dt.dot_prefix[n]);
+    for (int64_t k = 0; k < n; ++k)
+        if (op[k] == MURE_OP_GF || op[k] == MURE_OP_WS)
+            for (int q = 0; q < nn[k]; ++q) { dslot.push_back((int32_t)k); dslot.push_back(q); }
     // one staging buffer, one H2D copy
     const size_t b_op = n * 4, b_nn = n * 4, b_mid = n * 4, b_noff = n * 8, b_poff = n * 8;
+    const size_t b_dslot = std::max<size_t>(dslot.size(), 1) * 4;
     const size_t b_ids = (size_t)std::max<int64_t>(pool_len, 1) * 4, b_jobs = jobs.size() * sizeof(SlotJob);
     size_t off = 0;
     auto place = [&](size_t b) { size_t o = off; off = round_up(off + b, 256); return o; };
     const size_t o_op = place(b_op), o_nn = place(b_nn), o_mid = place(b_mid), o_noff = place(b_noff),
-                 o_poff = place(b_poff), o_ids = place(b_ids), o_jobs = place(b_jobs);
+                 o_poff = place(b_poff), o_ids = place(b_ids), o_jobs = place(b_jobs), o_dslot = place(b_dslot);
     std::vector<char> host(off);
     memcpy(host.data() + o_op, op.data(), b_op);
     memcpy(host.data() + o_nn, nn.data(), b_nn);
@@ -443,6 +450,7 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
     memcpy(host.data() + o_poff, poff.data(), b_poff);
     if (pool_len > 0) memcpy(host.data() + o_ids, pool, pool_len * 4);
     if (!jobs.empty()) memcpy(host.data() + o_jobs, jobs.data(), b_jobs);
+    if (!dslot.empty()) memcpy(host.data() + o_dslot, dslot.data(), dslot.size() * 4);
     char *dev = sc.get<char>(off);
     CK(c, cudaMemcpyAsync(dev, host.data(), off, cudaMemcpyHostToDevice, c->stream));
     dt.op = (int32_t *)(dev + o_op);
@@ -451,6 +459,7 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
     dt.noff = (int64_t *)(dev + o_noff);
     dt.poff = (int64_t *)(dev + o_poff);
     dt.ids = (int32_t *)(dev + o_ids);
+    dt.dslot = (int32_t *)(dev + o_dslot);
     dt.patch = plen ? sc.get<float>(plen) : nullptr;
     if (!jobs.empty()) {
         std::vector<const float *> Wp(m->L);
@@ -563,6 +572,9 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         acct.flops += fl;
     };
     PatchArgs pa{dt.op + g0, dt.nn + g0, dt.noff + g0, dt.ids, dt.poff + g0, dt.patch};
+    pa.dslot = dt.dslot + 2 * dt.dot_prefix[g0];
+    pa.n_dslot = dt.dot_prefix[g0 + rm.R / rm.T] - dt.dot_prefix[g0];
+    pa.dslot_g0 = (int32_t)g0;
     FinalArgs fa{};
     fa.mutant_id = dt.mid + g0;
     fa.label = ca->label;

@@ -180,6 +180,9 @@ struct PatchArgs {
     const int32_t *ids;         // neuron pool
     const int64_t *patch_off;   // [G] offset of slot 0 into patch (-1: none)
     const float *patch;         // GF: sigma * n, WS: W[j][perm f] - W[j][f]; F per slot
+    const int32_t *dslot = nullptr;   // the batch's GF / WS slots: (global group, slot q) pairs
+    int64_t n_dslot = 0;
+    int32_t dslot_g0 = 0;             // global index of the batch's first group
 };
 
 // Delta of layer l: values of the mutated neurons' channels of x_{l+1}, from z_l

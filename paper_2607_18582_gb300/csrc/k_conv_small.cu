@@ -222,6 +222,7 @@ struct PatchDotParams {
     int ih, iw, oh, ow, act1;
     const int32_t *op, *n_neurons, *ids;
     const int64_t *neuron_off, *patch_off;
+    const int32_t *dslot; int64_t n_dslot; int32_t dslot_g0;   // the batch's GF / WS slots
     const float *e_all;
     float *out; int64_t out_stride;
     int cells, rows_per_block;
@@ -307,7 +308,6 @@ __global__ void __launch_bounds__(256) k_patch_dot_in(const PatchDotParams p)
     float *es = xs + TILE;                // [SMAX][K] filter deltas
     float *zsm = es + SMAX * K;           // [oc][P] pre-activation maps
     __shared__ int sl_g[SMAX], sl_q[SMAX], sl_j[SMAX];
-    __shared__ int n_sl;
     const int tl = blockIdx.x;
     const int64_t t = p.t0 + tl;
     const float *xin = p.x + t * p.x_stride;
@@ -320,29 +320,17 @@ __global__ void __launch_bounds__(256) k_patch_dot_in(const PatchDotParams p)
     const float *zin = p.z + t * p.z_stride;
     for (int i = threadIdx.x; i < p.oc * P; i += blockDim.x) zsm[i] = __ldg(zin + i);
     const int pw = POOL ? p.ow / 2 : p.ow;
-    // the batch's GF / WS slots, SMAX at a time (walking the groups in order)
-    int g_next = 0, q_next = 0;
-    for (;;) {
+    // the batch's GF / WS slots (listed by the host), SMAX at a time
+    for (int64_t s0 = 0; s0 < p.n_dslot; s0 += SMAX) {
+        const int ns = (int)(p.n_dslot - s0 < SMAX ? p.n_dslot - s0 : SMAX);
         __syncthreads();
-        if (threadIdx.x == 0) {
-            int n = 0;
-            while (n < SMAX && g_next < p.G) {
-                const int op = p.op[g_next];
-                const int k = min(p.n_neurons[g_next], KMAX);
-                if ((op == MURE_OP_GF || op == MURE_OP_WS) && q_next < k) {
-                    sl_g[n] = g_next; sl_q[n] = q_next; sl_j[n] = p.ids[p.neuron_off[g_next] + q_next];
-                    ++n;
-                    ++q_next;
-                } else {
-                    ++g_next;
-                    q_next = 0;
-                }
-            }
-            n_sl = n;
+        if (threadIdx.x < ns) {
+            const int g = p.dslot[2 * (s0 + threadIdx.x)] - p.dslot_g0, q = p.dslot[2 * (s0 + threadIdx.x) + 1];
+            sl_g[threadIdx.x] = g;
+            sl_q[threadIdx.x] = q;
+            sl_j[threadIdx.x] = p.ids[p.neuron_off[g] + q];
         }
         __syncthreads();
-        const int ns = n_sl;
-        if (ns == 0) break;
         for (int i = threadIdx.x; i < ns * K; i += blockDim.x) {
             const int sl = i / K, kk = i - sl * K;
             es[i] = __ldg(p.e_all + p.patch_off[sl_g[sl]] + (int64_t)sl_q[sl] * K + kk);
@@ -413,6 +401,7 @@ int launch_dot(const Stage &S, Src z, Src x, RowMap rm, const PatchArgs &pa, int
     p.ih = S.ih; p.iw = S.iw; p.oh = S.oh; p.ow = S.ow; p.act1 = S.act1;
     p.op = pa.op; p.n_neurons = pa.n_neurons; p.ids = pa.ids; p.neuron_off = pa.neuron_off;
     p.patch_off = pa.patch_off; p.e_all = pa.patch;
+    p.dslot = pa.dslot; p.n_dslot = pa.n_dslot; p.dslot_g0 = pa.dslot_g0;
     p.out = out; p.out_stride = out_stride;
     p.cells = POOL ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
     p.rows_per_block = 8;

@@ -326,6 +326,68 @@ __global__ void __launch_bounds__(256) k_patch_vals_staged(const PatchValsParams
     }
 }
 
+// Dense layers in memoized mode, kDenseIn inputs per block: the inputs' cached rows
+// x and pre-activations z are staged in shared memory; a thread per (slot, input)
+// copies the operators without a fan-in sum, a warp per GF / WS slot (the host's list)
+// keeps its delta row in registers and forms the dot products of the block's inputs
+// exactly as dot_warp does (lane i sums k = i, i+32, ... ascending, then a butterfly).
+constexpr int kDenseIn = 8;
+constexpr int kDenseKMax = 1024;
+
+__global__ void __launch_bounds__(256) k_patch_vals_dense_in(const PatchValsParams p)
+{
+    extern __shared__ float sm2[];
+    const int K = p.K, OC = p.oc;
+    float *xs = sm2;                     // [kDenseIn][K]
+    float *zs = xs + kDenseIn * K;       // [kDenseIn][OC]
+    const int tl0 = blockIdx.x * kDenseIn;
+    const int ni = min(kDenseIn, p.T - tl0);
+    for (int i = threadIdx.x; i < ni * K; i += blockDim.x) {
+        const int a = i / K, k = i - a * K;
+        xs[i] = __ldg(p.x + (p.t0 + tl0 + a) * p.x_stride + k);
+    }
+    for (int i = threadIdx.x; i < ni * OC; i += blockDim.x) {
+        const int a = i / OC, c = i - a * OC;
+        zs[i] = __ldg(p.z + (p.t0 + tl0 + a) * p.z_stride + c);
+    }
+    __syncthreads();
+    // operators without a fan-in sum
+    for (int it = threadIdx.x; it < p.G * p.kmax * kDenseIn; it += blockDim.x) {
+        const int sl = it / kDenseIn, a = it - sl * kDenseIn;
+        const int g = sl / p.kmax, q = sl - g * p.kmax;
+        if (a >= ni || q >= p.pa.n_neurons[g]) continue;
+        const int op = p.pa.op[g];
+        if (op == MURE_OP_GF || op == MURE_OP_WS) continue;
+        const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
+        const int sj = op == MURE_OP_NS ? ids[q ^ 1] : ids[q];
+        float zz = zs[a * OC + sj];
+        if (op == MURE_OP_NAI) zz = -zz;
+        p.out[((int64_t)g * p.T + tl0 + a) * p.out_stride + q] = op == MURE_OP_NEB ? 0.f : act_apply(p.act1, zz);
+    }
+    // GF / WS: a warp per slot
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kPer = kDenseKMax / 32;
+    for (int64_t s2 = warp; s2 < p.pa.n_dslot; s2 += blockDim.x >> 5) {
+        const int g = p.pa.dslot[2 * s2] - p.pa.dslot_g0, q = p.pa.dslot[2 * s2 + 1];
+        const int j = p.pa.ids[p.pa.neuron_off[g] + q];
+        const float *e = p.pa.patch + p.pa.patch_off[g] + (int64_t)q * K;
+        float ev[kPer];
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) ev[i] = lane + 32 * i < K ? __ldg(e + lane + 32 * i) : 0.f;
+        for (int a = 0; a < ni; ++a) {
+            const float *xa = xs + a * K;
+            float acc = 0.f;
+#pragma unroll
+            for (int i = 0; i < kPer; ++i)
+                if (lane + 32 * i < K) acc = fmaf(ev[i], xa[lane + 32 * i], acc);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+            if (lane == 0)
+                p.out[((int64_t)g * p.T + tl0 + a) * p.out_stride + q] = act_apply(p.act1, zs[a * OC + j] + acc);
+        }
+    }
+}
+
 int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *out,
                       int64_t out_stride, cudaStream_t s, bool skip_dot_ops)
 {
@@ -354,10 +416,19 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     const int64_t gy = std::max<int64_t>(1, std::min<int64_t>(rm.T, (152 * 16 + gx - 1) / gx));
     const dim3 grid((unsigned)gx, (unsigned)gy);
     const size_t smem = (S.gap && !p.warp_dot) ? 8 * (size_t)p.mcells * sizeof(float) : 0;
+    // memoized dense layers: all operators per block of inputs
+    if (z.per_input && x.per_input && S.kind == MURE_NODE_DENSE && !S.has_add && !S.gap && !S.pool &&
+        S.K <= kDenseKMax && S.oh * S.ow == 1) {
+        const size_t sm = (size_t)kDenseIn * (S.K + S.oc) * 4;
+        if (sm <= 48 * 1024) {
+            k_patch_vals_dense_in<<<(unsigned)((rm.T + kDenseIn - 1) / kDenseIn), 256, sm, s>>>(p);
+            return 1;
+        }
+    }
     // memoized convolution layers whose maps fit in shared memory: the non-dot
     // operators per input, staged
     const size_t staged_smem = ((size_t)S.oc * S.oh * S.ow + p.mcells) * 4;
-    const bool staged = z.per_input && S.kind == MURE_NODE_CONV2D && !S.has_add && !S.gap && p.mcells >= 32 &&
+    const bool staged = z.per_input && S.kind == MURE_NODE_CONV2D && !S.has_add && !S.gap &&
                         staged_smem <= 48 * 1024;
     int launches = 0;
     if (staged) {
