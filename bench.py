@@ -235,7 +235,8 @@ def main():
     ap.add_argument("--n-mutants", type=int, default=None, help="smaller case (profiling): first n mutants")
     ap.add_argument("--only-layer", type=int, default=None, help="keep only the mutants of this layer")
     ap.add_argument("--precision", default="tf32x3", choices=["fp32", "tf32x3", "tf32"],
-                    help="layer arithmetic: fp32 CUDA-core chains, or tensor-core 3xTF32 for dense layers")
+                    help="layer arithmetic: fp32 CUDA-core chains, tensor-core 3xTF32 (fp32-level), or one TF32 "
+                         "product per MAC (the reduced-precision variant)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world, rank, local = dist_setup()
@@ -305,27 +306,49 @@ def main():
         byts = sum(r["stats"]["bytes_gather"] for r in results)
         achieved = byts / (cls_ms[top] / 1e3) / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / pk["hbm_gbs"], "traffic": None, "kernel": "k_patch_rows (delta)",
+                "frac": achieved / pk["hbm_gbs"], "traffic": None, "kernel": "delta kernels (k_patch_*)",
                 "ms_total": cls_ms[top], "peak_source": f"{pk_kind} (MEASURED_PEAKS.json hbm_gbs)"}
     pk, pk_kind = peaks()
     if top.startswith("layer"):
         v = int(top[5:])
         fl = sum(r["stats"]["flops_layer"][v] for r in results)
         nl = sum(r["stats"]["launches_layer"][v] for r in results)
-        achieved = fl / (cls_ms[top] / 1e3) / 1e12
+        secs = cls_ms[top] / 1e3
+        achieved = fl / secs / 1e12
         layer_node = w.model.nodes[w.model.layers()[v]]
-        rows = fl / 2 / w.model.layer_macs(v) / max(1, nl)   # rows per launch
-        roof = {"bound": "alu", "achieved": achieved, "peak": SIMT_FP32_PEAK_TFLOPS, "unit": "TFLOP/s",
-                "frac": achieved / SIMT_FP32_PEAK_TFLOPS,
-                "traffic": profiled_traffic(f"stage_simt_{args.workload}_layer{v}", rows),
-                "rows_per_launch": rows,
-                "kernel": f"k_stage_simt (layer {v}: {layer_node.kind} {layer_node.cin}->{layer_node.cout})",
-                "launches": nl, "ms_total": cls_ms[top],
-                "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz (no tensor cores on this path)",
-                "tensor_pipe_frac": 0.0}
+        rows_total = fl / 2 / w.model.layer_macs(v)
+        rows = rows_total / max(1, nl)   # rows per launch
+        kname, macs_exec = model.layer_kernel(v)
+        desc = f"layer {v}: {layer_node.kind} {layer_node.cin}->{layer_node.cout}"
+        if kname in ("tc_gemm", "tc_window"):
+            # tensor cores: TF32 peak = measured bf16 x the nominal TF32 / bf16 ratio
+            # (1.1 / 2.25 PFLOP/s); 3xTF32 spends three TF32 products per fp32 MAC, so
+            # its fp32-equivalent peak is a third of that.  The step is long, so the
+            # sustained bf16 figure applies.
+            bf16 = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+            tf32_peak = bf16 * 1.1 / 2.25
+            terms = 3 if args.precision == "tf32x3" else 1
+            peak = tf32_peak / terms
+            key = "tc_window" if kname == "tc_window" else "tc_gemm"
+            roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                    "traffic": profiled_traffic(f"{key}_{args.workload}_layer{v}", rows), "rows_per_launch": rows,
+                    "kernel": f"k_tc_gemm ({'window GEMM' if kname == 'tc_window' else 'implicit GEMM'}, {desc})",
+                    "launches": nl, "ms_total": cls_ms[top],
+                    "peak_source": f"{pk_kind} bf16 sustained {bf16:.1f} TFLOP/s x 1.1/2.25 (TF32) / {terms} "
+                                   f"({args.precision}); achieved counts the layer's useful fp32 MACs x 2",
+                    "tensor_pipe_frac": terms * 2 * macs_exec * rows_total / secs / 1e12 / tf32_peak}
+        else:
+            key = "conv_small" if kname == "simt_small" else ("final_dense" if kname == "output" else "stage_simt")
+            roof = {"bound": "alu", "achieved": achieved, "peak": SIMT_FP32_PEAK_TFLOPS, "unit": "TFLOP/s",
+                    "frac": achieved / SIMT_FP32_PEAK_TFLOPS,
+                    "traffic": profiled_traffic(f"{key}_{args.workload}_layer{v}", rows), "rows_per_launch": rows,
+                    "kernel": f"k_{key} ({desc})", "launches": nl, "ms_total": cls_ms[top],
+                    "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz (CUDA cores)",
+                    "tensor_pipe_frac": 0.0}
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": 1e3 * t_total / args.steps, "higher_is_better": True,
-           "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+           "scaling": "weak", "vs_baseline": None, "dtype": {"fp32": "f32", "tf32x3": "tf32x3", "tf32": "tf32"}[args.precision],
+           "data": "synthetic",
            "config": config_block(args, w), "roofline": roof, "gpu_launches": int(launches),
            "kernel_ms_per_step": {k: v / args.steps for k, v in cls_ms.items()},
            "scores": {"killed_frac": last["scoreA"], "deepmutation": last["scoreB"],

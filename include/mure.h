@@ -195,6 +195,26 @@ int64_t mure_kernel_launches(const mure_ctx *ctx);
 /* Number of weighted layers L of a loaded model (or -1 for NULL). */
 int32_t mure_model_n_layers(const mure_model *model);
 
+/* Which kernel computes weighted layer `layer` of a loaded model (the choice is fixed
+ * when the model is loaded, so every computation of a layer uses one kernel), and the
+ * multiply-accumulates that kernel executes per batch row.  Kernel codes:
+ *   MURE_KERNEL_SIMT_GEMM    CUDA-core implicit GEMM (fp32 chains)
+ *   MURE_KERNEL_SIMT_SMALL   CUDA-core direct convolution for LeNet-size layers
+ *   MURE_KERNEL_TC_GEMM      tensor-core GEMM / implicit-GEMM convolution
+ *   MURE_KERNEL_TC_WINDOW    tensor-core GEMM over 2x2 pooling windows
+ *   MURE_KERNEL_OUTPUT       output layer with the fused argmax / kill epilogue
+ * macs_per_row counts the GEMM as executed (padding and, for the window form, the
+ * zero taps included; one product per MAC, whatever the precision mode).  Either
+ * output pointer may be NULL.  Errors: INVALID_ARG (NULL model, layer out of range). */
+typedef enum {
+    MURE_KERNEL_SIMT_GEMM = 0,
+    MURE_KERNEL_SIMT_SMALL = 1,
+    MURE_KERNEL_TC_GEMM = 2,
+    MURE_KERNEL_TC_WINDOW = 3,
+    MURE_KERNEL_OUTPUT = 4
+} mure_kernel;
+mure_status mure_model_layer_kernel(const mure_model *model, int32_t layer, int32_t *kernel, int64_t *macs_per_row);
+
 /* Build the prefix-activation cache (the memo table, Algorithm 3 and Algorithm 1
  * lines 11-12, kept for every layer so every cluster shares one table): one forward
  * pass of the original network over X [n_inputs][in_h][in_w][in_c] storing, per

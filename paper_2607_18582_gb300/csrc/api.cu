@@ -1075,6 +1075,25 @@ void mure_model_free(mure_model *m)
 
 int32_t mure_model_n_layers(const mure_model *m) { return m ? m->L : -1; }
 
+mure_status mure_model_layer_kernel(const mure_model *m, int32_t layer, int32_t *kernel, int64_t *macs_per_row)
+{
+    if (!m || layer < 0 || layer >= m->L) return MURE_ERR_INVALID_ARG;
+    const Stage &S = m->st[layer];
+    int32_t k = MURE_KERNEL_SIMT_GEMM;
+    int64_t macs = S.macs;
+    if (layer == m->L - 1) {
+        k = MURE_KERNEL_OUTPUT;
+    } else if (S.tc) {
+        k = S.tc_small ? MURE_KERNEL_TC_WINDOW : MURE_KERNEL_TC_GEMM;
+        macs = tc_macs_per_row(S);
+    } else if (S.variant > 0) {
+        k = MURE_KERNEL_SIMT_SMALL;
+    }
+    if (kernel) *kernel = k;
+    if (macs_per_row) *macs_per_row = macs;
+    return MURE_OK;
+}
+
 int64_t mure_kernel_launches(const mure_ctx *ctx) { return ctx ? ctx->launches : -1; }
 
 mure_status mure_build_prefix_cache(mure_model *m, const float *X, int64_t n_inputs, const int32_t *labels,

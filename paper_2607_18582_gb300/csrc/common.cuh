@@ -141,6 +141,7 @@ int tc_overlay_inline(const Stage &S, const Overlay &ov, int64_t groups);
 int tc_small_geometry(const Stage &S);
 int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t s);
 int64_t tc_swizzle_tmp_floats(const Stage &S);
+int64_t tc_macs_per_row(const Stage &S);
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
               int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov = nullptr);
 

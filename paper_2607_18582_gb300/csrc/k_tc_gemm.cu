@@ -45,7 +45,7 @@ constexpr int kNB = 3;                 // streamed weight stages
 constexpr int kSlice = 128;            // output channels per CTA
 constexpr int kThreads = 384;          // 4 producer + 4 epilogue + 3 MMA + weight warps
 constexpr int kEpiStride = 36;         // floats per row of an epilogue staging chunk (32 + pad)
-constexpr int kACol = 256;             // accumulators in columns 0..255, A stages from 256
+constexpr int kMaxNT = 8;              // tensor-memory A stages, at most
 constexpr uint32_t kStageA = kTileM * 128;   // bytes of one producer ring slot
 constexpr long long kSpin = 2000000000LL;    // about a second at the SM clock
 
@@ -279,6 +279,9 @@ struct TcParams {
     Overlay ov;                  // mutated channels of the input rows (ov.patch null: none)
     int n_mma;                   // MMA-issuing warps, each with its own partial accumulators
     int acc_cols;                // tensor-memory columns of one partial accumulator
+    int n_acc;                   // accumulator sets (tiles in flight): 1 or 2
+    int n_stages;                // tensor-memory A stages (<= kMaxNT), from column a_col
+    int a_col;
     int *err;
 };
 
@@ -533,7 +536,7 @@ template <int MODE, bool THREE>
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
 {
     constexpr bool DENSE = MODE == 0;
-    constexpr int kNT = THREE ? 4 : 8;             // tensor-memory A stages
+    constexpr int kNT = kMaxNT;                    // barrier slots; p.n_stages are used
     constexpr int kAColsPerStage = THREE ? 64 : 32;
     extern __shared__ __align__(1024) unsigned char smraw[];
     __shared__ __align__(8) uint64_t bar_afull[kNT], bar_aempty[kNT], bar_bfull[kNB], bar_bempty[kNB];
@@ -623,14 +626,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             }
             if (wraps >= 1 && !warp_wait_phase<32>(smem_u32(&bar_aempty[t]), (wraps - 1) & 1, abort_flag)) return false;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t ta = tmem + lane_off + kACol + t * kAColsPerStage;
+            const uint32_t ta = tmem + lane_off + p.a_col + t * kAColsPerStage;
             tmem_st32(ta, hi);
             if (THREE) tmem_st32(ta + 32, lo);
             asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bar_afull[t]));
-            if (++t == kNT) { t = 0; ++wraps; }
+            if (++t == p.n_stages) { t = 0; ++wraps; }
             return true;
         };
         if constexpr (MODE == 2) {
@@ -757,8 +760,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
         const int qd = warp & 3;
         const uint32_t lane_off = (uint32_t)(qd * 32) << 16;
         for (int64_t i = 0; i < my_tiles; ++i) {
-            const int a = (int)(i & 1);
-            if (!warp_wait_phase<64>(smem_u32(&bar_accfull[a]), (uint32_t)((i >> 1) & 1), abort_flag)) break;
+            const int a = p.n_acc == 2 ? (int)(i & 1) : 0;
+            const int64_t use = p.n_acc == 2 ? (i >> 1) : i;
+            if (!warp_wait_phase<64>(smem_u32(&bar_accfull[a]), (uint32_t)(use & 1), abort_flag)) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const int64_t tile = blockIdx.x + i * gridDim.x;
             if constexpr (MODE == 2) {
@@ -913,7 +917,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
         // only about every 120 cycles, whatever N is, so narrow layers need several
         const int w = warp - 8;
         if (lane == 0 && w < p.n_mma) {
-            const int nmma = p.n_mma;
+            const int nmma = p.n_mma, nacc = p.n_acc;
             const uint32_t id = idesc_tf32(kTileM, Nt);
             bool ok = true;
             if (p.b_resident) ok = wait_phase<32>(smem_u32(&bar_bfull[0]), 0, abort_flag);
@@ -922,8 +926,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             int t = 0, sb = 0;
             uint32_t t_wraps = 0, b_wraps = 0;
             for (int64_t i = 0; ok && i < my_tiles; ++i) {
-                const int a = (int)(i & 1);
-                if (i >= 2 && !wait_phase<32>(smem_u32(&bar_accempty[a]), (uint32_t)(((i >> 1) - 1) & 1), abort_flag)) break;
+                const int a = nacc == 2 ? (int)(i & 1) : 0;
+                const int64_t use = nacc == 2 ? (i >> 1) : i;
+                if (use >= 1 && !wait_phase<32>(smem_u32(&bar_accempty[a]), (uint32_t)((use - 1) & 1), abort_flag)) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t d = tmem + (uint32_t)((a * nmma + w) * p.acc_cols);
                 for (int kt = 0; kt < nK; ++kt) {
@@ -932,9 +937,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                         !wait_phase<32>(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                     const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
-                    mma_share<THREE>(nmma, w, d, tmem + kACol + t * kAColsPerStage, dh, dl, id, kt > 0 ? 1u : 0u);
+                    mma_share<THREE>(nmma, w, d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, kt > 0 ? 1u : 0u);
                     mma_commit(smem_u32(&bar_aempty[t]));
-                    if (++t == kNT) { t = 0; ++t_wraps; }
+                    if (++t == p.n_stages) { t = 0; ++t_wraps; }
                     if (!p.b_resident) {
                         mma_commit(smem_u32(&bar_bempty[sb]));
                         if (++sb == kNB) { sb = 0; ++b_wraps; }
@@ -1083,7 +1088,28 @@ int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t 
     return launches;
 }
 
+// Multiply-accumulates one batch row costs the tensor-core kernel, padding included.
+int64_t tc_macs_per_row(const Stage &S)
+{
+    const int64_t Np = round_up16(gemm_n(S)), Kp = round_up32(gemm_k(S));
+    if (S.kind == MURE_NODE_DENSE) return Np * Kp;
+    const int64_t P = S.tc_small ? SmallConv::P : (S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : (int64_t)S.oh * S.ow);
+    return P * Np * Kp;
+}
+
 int64_t tc_swizzle_tmp_floats(const Stage &S) { return S.tc_small ? (int64_t)SmallConv::N * SmallConv::K : 0; }
+
+// Tensor-memory layout (512 columns): n_acc sets of n_mma partial accumulators, then
+// n_stages A stages.  A function of the layer alone, so a row's arithmetic never
+// depends on the batch.
+static void tc_config(TcParams &p, int nt_max, bool three)
+{
+    p.acc_cols = round_up32(nt_max);
+    p.n_acc = 2;
+    p.n_mma = std::max(1, std::min(3, 256 / (2 * p.acc_cols)));
+    p.a_col = 256;
+    p.n_stages = three ? 4 : 8;
+}
 
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
               int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov)
@@ -1130,8 +1156,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     const size_t smem = std::max<size_t>(1024 + b_bytes + a_bytes, 116 * 1024);
     // partial accumulators: two sets of n_mma in columns 0..255; a function of the layer
     // alone, so a row's arithmetic never depends on the batch
-    p.acc_cols = round_up32(nt_max);
-    p.n_mma = std::max(1, std::min(3, kACol / (2 * p.acc_cols)));
+    tc_config(p, nt_max, three);
     const int64_t M = (int64_t)rm.R * p.P;
     const int64_t tiles = (M + kTileM - 1) / kTileM;
     static int n_sm = 0;

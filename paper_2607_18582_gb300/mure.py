@@ -24,7 +24,7 @@ PRECISIONS = {"fp32": 0, "tf32x3": 1, "bf16": 2, "tf32": 3}
 
 # the exported entry points of include/mure.h
 EXPORTS = ("mure_create", "mure_destroy", "mure_last_error", "mure_model_load", "mure_model_free",
-           "mure_model_n_layers", "mure_kernel_launches", "mure_build_prefix_cache", "mure_cache_free", "mure_cache_outputs",
+           "mure_model_n_layers", "mure_model_layer_kernel", "mure_kernel_launches", "mure_build_prefix_cache", "mure_cache_free", "mure_cache_outputs",
            "mure_eval_mutants", "mure_eval_vanilla", "mure_expand_patches", "mure_expand_patches_noalloc")
 
 
@@ -106,6 +106,7 @@ def lib():
         L.mure_model_free.restype = None
         L.mure_model_n_layers.argtypes = [vp]
         L.mure_model_n_layers.restype = i32
+        L.mure_model_layer_kernel.argtypes = [vp, i32, C.POINTER(i32), C.POINTER(i64)]
         L.mure_kernel_launches.argtypes = [vp]
         L.mure_kernel_launches.restype = i64
         L.mure_build_prefix_cache.argtypes = [vp, vp, i64, vp, C.c_int, C.POINTER(vp)]
@@ -215,6 +216,14 @@ class Model:
     @property
     def n_layers(self):
         return lib().mure_model_n_layers(self.h)
+
+    KERNELS = {0: "simt_gemm", 1: "simt_small", 2: "tc_gemm", 3: "tc_window", 4: "output"}
+
+    def layer_kernel(self, layer):
+        """(kernel name, executed multiply-accumulates per batch row) of a layer."""
+        k, macs = C.c_int32(), C.c_int64()
+        self.ctx.check(lib().mure_model_layer_kernel(self.h, int(layer), C.byref(k), C.byref(macs)))
+        return self.KERNELS.get(k.value, str(k.value)), macs.value
 
     def _child_gone(self):
         self._children -= 1
