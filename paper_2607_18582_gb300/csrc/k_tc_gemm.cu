@@ -167,9 +167,8 @@ __device__ __forceinline__ void mma_tf32_ts(uint32_t d_tmem, uint32_t a_tmem, ui
 
 // MMAs q = LO .. HI-1 of a K-step, q = ks * kTerms + term (3xTF32: a_lo*b_hi,
 // a_hi*b_lo, a_hi*b_hi for K8 step ks), into accumulator d; the first one overwrites
-// unless acc0.  Fully unrolled: the issuing thread has no other warps to hide the
-// latency of scalar work between MMAs, and an MMA predicated off still costs its issue
-// slot, so each issuing warp runs only its own block.
+// unless acc0.  Fully unrolled: scalar work between two MMAs adds its latency to the
+// issuing thread's MMA rate.
 template <bool THREE, int LO, int HI>
 __device__ __forceinline__ void mma_block(uint32_t d, uint32_t ta, uint64_t dh, uint64_t dl, uint32_t id, uint32_t acc0)
 {
@@ -183,22 +182,6 @@ __device__ __forceinline__ void mma_block(uint32_t d, uint32_t ta, uint64_t dh, 
         if (!THREE || term == 2) mma_tf32_ts(d, ta + ks * 8, dh + 2 * ks, id, acc);    // a_hi * b_hi
         else if (term == 0) mma_tf32_ts(d, ta + 32 + ks * 8, dh + 2 * ks, id, acc);   // a_lo * b_hi
         else mma_tf32_ts(d, ta + ks * 8, dl + 2 * ks, id, acc);                       // a_hi * b_lo
-    }
-}
-
-// Warp w of n_mma issuing warps: the contiguous block w*kQ/n .. (w+1)*kQ/n of a K-step.
-template <bool THREE>
-__device__ __forceinline__ void mma_share(int nmma, int w, uint32_t d, uint32_t ta, uint64_t dh, uint64_t dl, uint32_t id,
-                                          uint32_t acc0)
-{
-    constexpr int Q = THREE ? 12 : 4;
-    switch (nmma * 4 + w) {
-    case 4: mma_block<THREE, 0, Q>(d, ta, dh, dl, id, acc0); break;
-    case 8: mma_block<THREE, 0, Q / 2>(d, ta, dh, dl, id, acc0); break;
-    case 9: mma_block<THREE, Q / 2, Q>(d, ta, dh, dl, id, acc0); break;
-    case 12: mma_block<THREE, 0, Q / 3>(d, ta, dh, dl, id, acc0); break;
-    case 13: mma_block<THREE, Q / 3, 2 * Q / 3>(d, ta, dh, dl, id, acc0); break;
-    default: mma_block<THREE, 2 * Q / 3, Q>(d, ta, dh, dl, id, acc0); break;
     }
 }
 
@@ -466,10 +449,14 @@ __device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, co
 // 16 output channels a per-position GEMM would have N = 16, where the MMA issue rate,
 // not the tensor core, is the limit; per window the layer takes a third of the MMA
 // instructions and of the gathers, and the epilogue pools inside each row.  The
-// producers stage whole input maps in shared memory (coalesced cp.async) and gather
-// each row's receptive field from there with compile-time offsets, 16 bytes per load
-// (a receptive-field row is 36 consecutive, 16-byte-aligned values).  A tile of 128
-// rows spans at most NIMG maps.
+// loader warp stages a tile's whole input maps in shared memory (one bulk copy per
+// map) and the producers gather each row's receptive field from there with
+// compile-time offsets, 16 bytes per load (a receptive-field row is 36 consecutive,
+// 16-byte-aligned values).  A tile holds the windows of MAPS whole maps (125 of its
+// 128 rows; the other 3 are computed and dropped), so that three staging buffers fit
+// beside the resident weights and the loader runs two tiles ahead of the producers.
+// Each tile's maps are bulk copies (with per-input maps, from L2), and so are the
+// patch values of the tile's rows, which are consecutive in memory.
 struct SmallConv {
     static constexpr int IH = 14, IW = 14, IC = 6, KH = 5, KW = 5, OH = 10, OW = 10, PW = 5, OC = 16;
     static constexpr int KU = KH + 1;                         // receptive field of a window: KU x KU
@@ -478,21 +465,25 @@ struct SmallConv {
     static constexpr int N = 4 * OC;                          // GEMM columns: (window position, channel)
     static constexpr int CELLS = IH * IW;                     // overlay cells of a mutated channel
     static constexpr uint32_t IMG_B = IH * IW * IC * 4;       // bytes of one staged map
-    static constexpr int CH16 = IMG_B / 16;
     static constexpr int MAXQ = 2;                            // mutated channels per row (overlay)
     static constexpr int MAXG = 256;                          // mutants per batch (overlay table)
-    static constexpr int NIMG = (kTileM - 1) / P + 2;         // maps per tile, at most
-    static constexpr uint32_t BUF_B = NIMG * IMG_B;           // one buffer of staged maps
-    static constexpr uint32_t OVST_B = NIMG * MAXQ * CELLS * 4;   // one buffer of staged patch values
+    static constexpr int MAPS = kTileM / P;                   // maps per tile
+    static constexpr int ROWS = MAPS * P;                     // live rows of a tile
+    static constexpr int NBUF = 3;                            // staging buffers
+    static constexpr uint32_t BUF_B = MAPS * IMG_B;           // one buffer of staged maps
+    static constexpr uint32_t OVST_B = MAPS * MAXQ * CELLS * 4;   // one buffer of staged patch values
     static constexpr uint32_t TAB_B = MAXG * (1 + MAXQ) * 4;      // [g][count, channel ids]
-    static constexpr uint32_t BYTES = 2 * BUF_B + 2 * OVST_B + TAB_B;
+    static constexpr uint32_t BYTES = NBUF * (BUF_B + OVST_B) + TAB_B;
 };
-static_assert(SmallConv::IMG_B % 16 == 0, "maps are copied in 16-byte chunks");
-static_assert((SmallConv::CELLS * 4) % 16 == 0, "patch values are copied in 16-byte chunks");
+static_assert(SmallConv::IMG_B % 16 == 0, "maps are bulk copies of whole 16-byte chunks");
+
+// Tiles of the small-image mode over R rows: tile i holds rows MAPS*i .. MAPS*i+MAPS-1.
+__host__ __device__ __forceinline__ int64_t small_tiles(int64_t R) { return (R + SmallConv::MAPS - 1) / SmallConv::MAPS; }
+static_assert(2 * SmallConv::N * 128 * SmallConv::NKT <= 112 * 1024,
+              "the small-image mode keeps its weights resident (its loader warp stages the maps)");
+static_assert((SmallConv::CELLS * 4) % 16 == 0, "patch values are bulk copies of whole 16-byte chunks");
 static_assert((SmallConv::KU * SmallConv::IC) % 4 == 0 && (SmallConv::IW * SmallConv::IC * 4) % 16 == 0,
               "receptive-field rows are 16-byte aligned runs of whole 4-value chunks");
-
-__device__ __forceinline__ void named_bar_producers() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
 // K-step KT of a window row: 8 chunks of 4 values at compile-time offsets from the
 // window's receptive-field origin `base`, k = (wy, wx, ci).
@@ -541,6 +532,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     extern __shared__ __align__(1024) unsigned char smraw[];
     __shared__ __align__(8) uint64_t bar_afull[kNT], bar_aempty[kNT], bar_bfull[kNB], bar_bempty[kNB];
     __shared__ __align__(8) uint64_t bar_accfull[2], bar_accempty[2], bar_drain;
+    // small-image mode, per staging buffer: maps landed, overlay applied, producers done
+    __shared__ __align__(8) uint64_t bar_landed[SmallConv::NBUF], bar_ready[SmallConv::NBUF], bar_released[SmallConv::NBUF];
     __shared__ uint32_t tmem_sh;
     __shared__ int abort_sh;
     __shared__ float bias_sh[kSlice];
@@ -559,7 +552,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     const uint32_t a_region = sbase + (p.b_resident ? (uint32_t)nK * b_step : (uint32_t)kNB * b_step);
     const uint32_t ov_region = a_region + kNA * kStageA;    // kNA overlay slots (with an overlay)
     const int64_t M = (int64_t)p.R * p.P;
-    const int64_t n_tiles = (M + kTileM - 1) / kTileM;
+    const int64_t n_tiles = MODE == 2 ? small_tiles(p.R) : (M + kTileM - 1) / kTileM;
     const int64_t my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
     const int64_t total = my_tiles * nK;
     const float *wslice = p.Wsw + (int64_t)blockIdx.y * p.w_slice_floats;
@@ -575,8 +568,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     }
     // small-image mode: staged maps, staged patch values, the batch's mutated-channel table
     const uint32_t img_region = a_region;
-    const uint32_t ovst_region = img_region + 2 * SmallConv::BUF_B;
-    const uint32_t ovtab_region = ovst_region + 2 * SmallConv::OVST_B;
+    const uint32_t ovst_region = img_region + SmallConv::NBUF * SmallConv::BUF_B;
+    const uint32_t ovtab_region = ovst_region + SmallConv::NBUF * SmallConv::OVST_B;
     if (MODE == 2 && p.ov.patch) {
         const int G = p.R / p.T;
         for (int g = threadIdx.x; g < G; g += kThreads) {
@@ -590,17 +583,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     if (threadIdx.x == 32) {
         for (int s = 0; s < kNT; ++s) {
             mbar_init(smem_u32(&bar_afull[s]), 4);
-            mbar_init(smem_u32(&bar_aempty[s]), p.n_mma);
+            mbar_init(smem_u32(&bar_aempty[s]), 1);     // each K-step has one issuing warp
         }
         for (int s = 0; s < kNB; ++s) {
             mbar_init(smem_u32(&bar_bfull[s]), 1);
-            mbar_init(smem_u32(&bar_bempty[s]), p.n_mma);
+            mbar_init(smem_u32(&bar_bempty[s]), 1);
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(smem_u32(&bar_accfull[s]), p.n_mma);
             mbar_init(smem_u32(&bar_accempty[s]), 4);
         }
         mbar_init(smem_u32(&bar_drain), p.n_mma);
+        for (int s = 0; s < SmallConv::NBUF; ++s) {
+            mbar_init(smem_u32(&bar_landed[s]), 1);
+            mbar_init(smem_u32(&bar_ready[s]), 1);
+            mbar_init(smem_u32(&bar_released[s]), 4);
+        }
         abort_sh = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -608,6 +606,35 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_sh;
+
+    // small-image mode staging (warps 10 and 11).  A map's mutant g = row / T and input
+    // t0 + row % T (rows fit 32 bits).
+    using G2 = SmallConv;
+    auto tab_of = [&](uint32_t row) { return ovtab_region + (row / (uint32_t)p.T) * (1 + G2::MAXQ) * 4; };
+    // tile i's first row and its number of rows
+    auto tile_rows = [&](int64_t i, uint32_t &row0) {
+        row0 = (uint32_t)((blockIdx.x + i * gridDim.x) * G2::MAPS);
+        return (int)min((uint32_t)G2::MAPS, (uint32_t)p.R - row0);
+    };
+    // bulk copies of tile i into buffer b: a map per row and, in one piece, the rows'
+    // patch values (lane 0)
+    auto issue_tile = [&](int64_t i, int b) {
+        uint32_t row0;
+        const int nimg = tile_rows(i, row0);
+        const uint32_t buf = img_region + (uint32_t)b * G2::BUF_B;
+        const uint32_t bar = smem_u32(&bar_landed[b]);
+        const uint32_t pbytes = p.ov.patch ? (uint32_t)(nimg * p.ov.row_stride * 4) : 0u;
+        // the buffer was last read and written by generic loads and stores
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        mbar_expect_tx(bar, nimg * G2::IMG_B + pbytes);
+        for (int im = 0; im < nimg; ++im) {
+            const uint32_t row = row0 + im;
+            const int64_t xr = p.x_per_input ? p.t0 + row % (uint32_t)p.T : row;
+            bulk_g2s(buf + im * G2::IMG_B, p.x + xr * p.x_stride, G2::IMG_B, bar);
+        }
+        if (pbytes)
+            bulk_g2s(ovst_region + (uint32_t)b * G2::OVST_B, p.ov.patch + (int64_t)row0 * p.ov.row_stride, pbytes, bar);
+    };
 
     if (warp < 4) {
         // ------------------------------------------------------------ producers --
@@ -637,70 +664,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             return true;
         };
         if constexpr (MODE == 2) {
+            // warps 10 and 11 stage each tile's maps (mutated channels written in) in
+            // buffer i mod NBUF; the producers only gather from them
             using G = SmallConv;
-            // copies of tile i's maps (and patch values) into buffer i & 1
-            auto issue_tile = [&](int64_t i) {
-                const int64_t m0 = (blockIdx.x + i * gridDim.x) * kTileM;
-                const int64_t row0 = m0 / G::P;
-                const int nimg = (int)((min(m0 + kTileM, M) - 1) / G::P - row0) + 1;
-                const uint32_t buf = img_region + (uint32_t)(i & 1) * G::BUF_B;
-                for (int im = 0; im < nimg; ++im) {
-                    const int64_t row = row0 + im;
-                    const float *src = p.x + (p.x_per_input ? p.t0 + row % p.T : row) * p.x_stride;
-                    for (int c = r; c < G::CH16; c += kTileM) cp_async16(buf + im * G::IMG_B + c * 16, src + c * 4, 16);
-                }
-                if (p.ov.patch) {
-                    const uint32_t ovb = ovst_region + (uint32_t)(i & 1) * G::OVST_B;
-                    for (int im = 0; im < nimg; ++im) {
-                        const int64_t row = row0 + im;
-                        uint32_t k;
-                        asm volatile("ld.shared.u32 %0, [%1];" : "=r"(k) : "r"(ovtab_region + (uint32_t)(row / p.T) * (1 + G::MAXQ) * 4));
-                        const float *src = p.ov.patch + row * p.ov.row_stride;
-                        for (int c4 = r; c4 < (int)k * G::CELLS / 4; c4 += kTileM)
-                            cp_async16(ovb + (im * G::MAXQ * G::CELLS + c4 * 4) * 4, src + c4 * 4, 16);
-                    }
-                }
-            };
-            if (my_tiles > 0) issue_tile(0);
-            cp_async_commit();
+            // this thread's GEMM row: map r / P of the tile and its pooling window (the
+            // padding rows gather from map 0, which is always staged)
+            const int im = r < G::ROWS ? r / G::P : 0, w = r < G::ROWS ? r % G::P : 0;
+            const uint32_t off = (uint32_t)im * G::IMG_B + (uint32_t)((2 * (w / G::PW) * G::IW + 2 * (w % G::PW)) * G::IC) * 4;
             bool ok = true;
+            int b = 0;
+            uint32_t uses = 0;                            // completed rounds of the buffer ring
             for (int64_t i = 0; ok && i < my_tiles; ++i) {
-                cp_async_wait<0>();
-                named_bar_producers();                    // every copy of tile i has landed
-                if (i + 1 < my_tiles) issue_tile(i + 1);  // the other buffer: tile i-1 is done
-                cp_async_commit();
-                const int64_t m0 = (blockIdx.x + i * gridDim.x) * kTileM;
-                const int64_t row0 = m0 / G::P;
-                const uint32_t buf = img_region + (uint32_t)(i & 1) * G::BUF_B;
-                if (p.ov.patch) {
-                    // the mutants' channels written into the staged maps
-                    const int nimg = (int)((min(m0 + kTileM, M) - 1) / G::P - row0) + 1;
-                    const uint32_t ovb = ovst_region + (uint32_t)(i & 1) * G::OVST_B;
-                    for (int im = 0; im < nimg; ++im) {
-                        const uint32_t tab = ovtab_region + (uint32_t)((row0 + im) / p.T) * (1 + G::MAXQ) * 4;
-                        uint32_t k;
-                        asm volatile("ld.shared.u32 %0, [%1];" : "=r"(k) : "r"(tab));
-                        for (int idx = r; idx < (int)k * G::CELLS; idx += kTileM) {
-                            const int q = idx / G::CELLS, c = idx - q * G::CELLS;
-                            uint32_t jn, val;
-                            asm volatile("ld.shared.u32 %0, [%1];" : "=r"(jn) : "r"(tab + 4 + q * 4));
-                            asm volatile("ld.shared.u32 %0, [%1];" : "=r"(val) : "r"(ovb + (im * G::MAXQ * G::CELLS + idx) * 4));
-                            asm volatile("st.shared.u32 [%0], %1;" ::"r"(buf + im * G::IMG_B + (c * G::IC + jn) * 4), "r"(val)
-                                         : "memory");
-                        }
-                    }
-                    named_bar_producers();
-                }
-                // this thread's GEMM row: map and pooling window
-                const int64_t m = m0 + r;
-                const bool in = m < M;
-                const int64_t row = in ? m / G::P : row0;
-                const int w = in ? (int)(m - row * G::P) : 0;
-                const int oy = 2 * (w / G::PW), ox = 2 * (w % G::PW);
-                const uint32_t base = buf + (uint32_t)(row - row0) * G::IMG_B + (uint32_t)((oy * G::IW + ox) * G::IC) * 4;
-                SmallSteps<0>::run(base, push, ok);
+                if (!warp_wait_phase<32>(smem_u32(&bar_ready[b]), uses & 1, abort_flag)) break;
+                SmallSteps<0>::run(img_region + (uint32_t)b * G::BUF_B + off, push, ok);
+                // every gather of the tile has been consumed by push: the buffer is free
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bar_released[b]));
+                if (++b == G::NBUF) { b = 0; ++uses; }
             }
-            cp_async_wait<0>();
         } else {
             // issue cursor (tile i, K-tile kt, ring slot) runs kNA - 1 steps ahead
             RowInfo pf{};
@@ -768,10 +749,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             if constexpr (MODE == 2) {
                 // a pooling window: columns n = s * OC + c for its position s = 2 dy + dx
                 using G = SmallConv;
-                const int64_t m = tile * kTileM + qd * 32 + lane;
-                const bool ok = m < M;
-                const int64_t row = ok ? m / G::P : 0;
-                const int w = ok ? (int)(m - row * G::P) : 0;
+                const int rr = qd * 32 + lane;
+                const int64_t row = tile * G::MAPS + rr / G::P;
+                const bool ok = rr < G::ROWS && row < p.R;
+                const int w = rr % G::P;
                 const int py = w / G::PW, px = w % G::PW;
                 const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_mma * p.acc_cols);
                 float v[G::N];
@@ -910,20 +891,64 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
         }
+    } else if (MODE == 2 && warp == 10) {
+        // ------------------------------------------------ map staging: finish --
+        // Tile i once landed: each row's mutated channels are written over its map, and
+        // the buffer goes to the producers.
+        using G = SmallConv;
+        int b = 0;
+        uint32_t uses = 0;
+        for (int64_t i = 0; i < my_tiles; ++i) {
+            if (!warp_wait_phase<32>(smem_u32(&bar_landed[b]), uses & 1, abort_flag)) break;
+            if (p.ov.patch) {
+                uint32_t row0;
+                const int nimg = tile_rows(i, row0);
+                const uint32_t buf = img_region + (uint32_t)b * G::BUF_B;
+                const uint32_t ovb = ovst_region + (uint32_t)b * G::OVST_B;
+                constexpr int U = (G::CELLS + 31) / 32;
+                for (int im = 0; im < nimg; ++im) {
+                    const uint32_t tab = tab_of(row0 + im);
+                    uint32_t k;
+                    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(k) : "r"(tab));
+                    for (uint32_t q = 0; q < k; ++q) {
+                        uint32_t jn, val[U];
+                        asm volatile("ld.shared.u32 %0, [%1];" : "=r"(jn) : "r"(tab + 4 + q * 4));
+                        const uint32_t src = ovb + (uint32_t)(im * p.ov.row_stride + q * G::CELLS) * 4;
+                        const uint32_t dst = buf + im * G::IMG_B + jn * 4;
+#pragma unroll
+                        for (int u = 0; u < U; ++u)
+                            if (lane + 32 * u < G::CELLS)
+                                asm volatile("ld.shared.u32 %0, [%1];" : "=r"(val[u]) : "r"(src + (lane + 32 * u) * 4));
+#pragma unroll
+                        for (int u = 0; u < U; ++u)
+                            if (lane + 32 * u < G::CELLS)
+                                asm volatile("st.shared.u32 [%0], %1;" ::"r"(dst + (lane + 32 * u) * (G::IC * 4)), "r"(val[u])
+                                             : "memory");
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bar_ready[b]));
+            if (++b == G::NBUF) { b = 0; ++uses; }
+        }
     } else if (warp < 11) {
         // ------------------------------------------------------------------ MMA --
-        // a K-step's MMAs (K8 step ks, product term) are dealt round-robin to the n_mma
-        // issuing warps, each into its own partial accumulator: one thread issues an MMA
-        // only about every 120 cycles, whatever N is, so narrow layers need several
+        // The K-steps of a tile are dealt to the n_mma issuing warps by their index
+        // (kt mod n_mma = w), each warp into its own partial accumulator.  One thread
+        // issues an MMA only about every 60 cycles and then waits for its next stage,
+        // so while one warp waits the others keep the tensor pipe busy.  The split
+        // depends on kt alone: a row's partial sums never depend on its place in the
+        // batch.
         const int w = warp - 8;
         if (lane == 0 && w < p.n_mma) {
             const int nmma = p.n_mma, nacc = p.n_acc;
+            constexpr int Q = THREE ? 12 : 4;
             const uint32_t id = idesc_tf32(kTileM, Nt);
             bool ok = true;
             if (p.b_resident) ok = wait_phase<32>(smem_u32(&bar_bfull[0]), 0, abort_flag);
             const uint64_t desc_b0 = sw128_desc(b_region);
             const uint32_t b_step16 = b_step >> 4, lo16 = (uint32_t)Nt * 128 >> 4;
-            int t = 0, sb = 0;
+            int t = 0, sb = 0;                  // ring slots of K-step kt (every warp tracks every step)
             uint32_t t_wraps = 0, b_wraps = 0;
             for (int64_t i = 0; ok && i < my_tiles; ++i) {
                 const int a = nacc == 2 ? (int)(i & 1) : 0;
@@ -931,19 +956,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                 if (use >= 1 && !wait_phase<32>(smem_u32(&bar_accempty[a]), (uint32_t)((use - 1) & 1), abort_flag)) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t d = tmem + (uint32_t)((a * nmma + w) * p.acc_cols);
+                int own = 0;                    // kt mod n_mma
                 for (int kt = 0; kt < nK; ++kt) {
-                    if (!wait_phase<32>(smem_u32(&bar_afull[t]), t_wraps & 1, abort_flag)) { ok = false; break; }
-                    if (!p.b_resident &&
-                        !wait_phase<32>(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
-                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                    const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
-                    mma_share<THREE>(nmma, w, d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, kt > 0 ? 1u : 0u);
-                    mma_commit(smem_u32(&bar_aempty[t]));
-                    if (++t == p.n_stages) { t = 0; ++t_wraps; }
-                    if (!p.b_resident) {
-                        mma_commit(smem_u32(&bar_bempty[sb]));
-                        if (++sb == kNB) { sb = 0; ++b_wraps; }
+                    if (own == w) {
+                        if (!wait_phase<32>(smem_u32(&bar_afull[t]), t_wraps & 1, abort_flag)) { ok = false; break; }
+                        if (!p.b_resident &&
+                            !wait_phase<32>(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
+                        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                        const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
+                        // the warp's first K-step of the tile (kt = w) overwrites its partial sum
+                        mma_block<THREE, 0, Q>(d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, kt >= nmma ? 1u : 0u);
+                        mma_commit(smem_u32(&bar_aempty[t]));
+                        if (!p.b_resident) mma_commit(smem_u32(&bar_bempty[sb]));
                     }
+                    if (++own == nmma) own = 0;
+                    if (++t == p.n_stages) { t = 0; ++t_wraps; }
+                    if (!p.b_resident && ++sb == kNB) { sb = 0; ++b_wraps; }
                 }
                 if (!ok) break;
                 mma_commit(smem_u32(&bar_accfull[a]));
@@ -961,7 +989,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                 for (uint32_t o = 0; o < bytes; o += 32768u)
                     bulk_g2s(b_region + o, (const unsigned char *)wslice + o, min(32768u, bytes - o),
                              smem_u32(&bar_bfull[0]));
-                wait_phase_drain(smem_u32(&bar_bfull[0]), 0);
             } else {
                 int64_t j = 0;
                 int sb = 0, kt = 0;
@@ -979,6 +1006,28 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                     wait_phase_drain(smem_u32(&bar_bfull[(int)(jj % kNB)]), (uint32_t)((jj / kNB) & 1));
             }
         }
+        if constexpr (MODE == 2) {
+            // ------------------------------------------------ map staging: copies --
+            // tile j goes to buffer j mod NBUF once the producers have released the
+            // tile that held it (a bulk copy issue can stall for hundreds of cycles, so
+            // this warp does nothing else)
+            using G = SmallConv;
+            int64_t issued = 0;
+            int b = 0;
+            uint32_t uses = 0;
+            for (; issued < my_tiles; ++issued) {
+                if (issued >= G::NBUF && !warp_wait_phase<32>(smem_u32(&bar_released[b]), (uses - 1) & 1, abort_flag)) break;
+                if (lane == 0) issue_tile(issued, b);
+                __syncwarp();
+                if (++b == G::NBUF) { b = 0; ++uses; }
+            }
+            // the copies of the last tiles (the only ones that can still be in flight)
+            // land before the shared memory is released
+            if (lane == 0)
+                for (int64_t j = issued > G::NBUF ? issued - G::NBUF : 0; j < issued; ++j)
+                    wait_phase_drain(smem_u32(&bar_landed[j % G::NBUF]), (uint32_t)((j / G::NBUF) & 1));
+        }
+        if (lane == 0 && p.b_resident) wait_phase_drain(smem_u32(&bar_bfull[0]), 0);
     }
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -1093,11 +1142,22 @@ int64_t tc_macs_per_row(const Stage &S)
 {
     const int64_t Np = round_up16(gemm_n(S)), Kp = round_up32(gemm_k(S));
     if (S.kind == MURE_NODE_DENSE) return Np * Kp;
-    const int64_t P = S.tc_small ? SmallConv::P : (S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : (int64_t)S.oh * S.ow);
+    // the small-image mode runs a 128-row tile per SmallConv::MAPS maps
+    if (S.tc_small) return (kTileM * Np * Kp + SmallConv::MAPS / 2) / SmallConv::MAPS;
+    const int64_t P = S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : (int64_t)S.oh * S.ow;
     return P * Np * Kp;
 }
 
 int64_t tc_swizzle_tmp_floats(const Stage &S) { return S.tc_small ? (int64_t)SmallConv::N * SmallConv::K : 0; }
+
+// The longest run of the K-step sequence (tile after tile, nK steps each) between two
+// consecutive K-steps of one issuing warp, when K-step kt goes to warp kt mod m.
+static int mma_gap(int nK, int m)
+{
+    int g = nK > m ? m : 0;
+    for (int w = 0; w < m; ++w) g = std::max(g, nK - (w + m * ((nK - 1 - w) / m)) + w);
+    return g;
+}
 
 // Tensor-memory layout (512 columns): n_acc sets of n_mma partial accumulators, then
 // n_stages A stages.  A function of the layer alone, so a row's arithmetic never
@@ -1106,9 +1166,15 @@ static void tc_config(TcParams &p, int nt_max, bool three)
 {
     p.acc_cols = round_up32(nt_max);
     p.n_acc = 2;
-    p.n_mma = std::max(1, std::min(3, 256 / (2 * p.acc_cols)));
     p.a_col = 256;
     p.n_stages = three ? 4 : 8;
+    // An issuing warp waits on a ring slot's barrier by the parity of the slot's use
+    // count, which names the right phase only while the warp's consecutive K-steps are
+    // at most a ring's depth apart; every warp also has a K-step in every tile.
+    const int nK = p.Kp / kTileK, depth = p.b_resident ? p.n_stages : std::min(p.n_stages, kNB);
+    int m = std::max(1, std::min({3, 256 / (2 * p.acc_cols), nK}));
+    while (m > 1 && mma_gap(nK, m) > depth) --m;
+    p.n_mma = m;
 }
 
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
@@ -1157,8 +1223,9 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     // partial accumulators: two sets of n_mma in columns 0..255; a function of the layer
     // alone, so a row's arithmetic never depends on the batch
     tc_config(p, nt_max, three);
+    if (S.tc_small) p.n_mma = std::min(p.n_mma, 2);   // warp 10 stages maps in that mode
     const int64_t M = (int64_t)rm.R * p.P;
-    const int64_t tiles = (M + kTileM - 1) / kTileM;
+    const int64_t tiles = S.tc_small ? small_tiles(rm.R) : (M + kTileM - 1) / kTileM;
     static int n_sm = 0;
     if (!n_sm) {
         int dev = 0;
