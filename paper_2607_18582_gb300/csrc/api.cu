@@ -662,7 +662,22 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     const Stage &Sn = m->st[l + 1];
     bool skip_reader = false;
     for (int v = l + 2; v < L; ++v) skip_reader |= m->st[v].has_add && m->st[v].skip_src == l + 1;
+    // a tensor-core dense stage L-2 takes the output layer and the kill epilogue into
+    // its own epilogue (the rows of x_{L-1} are then never stored)
+    const Stage &SLast = m->st[L - 1];
+    const FinalFuse ff{SLast.W, SLast.b, SLast.oc, SLast.K, SLast.act1, fa};
+    auto fused_last = [&](Src x, const Overlay *ovp) {
+        const Stage &S = m->st[L - 2];
+        timed(L - 2, 2 * (S.macs + SLast.macs) * rm.R, [&] {
+            return launch_tc(S, x, rm, nullptr, 0, skip_of(S), ws.xb[L - 1], m->xd[L - 1].stride, ws.gap_tmp, s, ovp, &ff);
+        });
+    };
+    const bool fuse = L >= 2 && tc_final_fusable(m->st[L - 2], SLast);
     if (Sn.tc && !skip_reader && tc_overlay_inline(Sn, ov, rm.R / rm.T)) {
+        if (fuse && l + 1 == L - 2) {
+            fused_last(base, &ov);
+            return launches;
+        }
         timed(l + 1, 2 * Sn.macs * rm.R, [&] {
             return launch_tc(Sn, base, rm, nullptr, 0, skip_of(Sn), ws.xb[l + 2], m->xd[l + 2].stride, ws.gap_tmp, s,
                              &ov);
@@ -679,6 +694,11 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         stage(l + 1, nullptr, 0);
     }
     // the rest of the suffix (Algorithm 4) and the fused kill epilogue
+    if (fuse && l + 2 <= L - 2) {
+        for (int v = l + 2; v < L - 2; ++v) stage(v, nullptr, 0);
+        fused_last(xsrc(L - 2), nullptr);
+        return launches;
+    }
     for (int v = l + 2; v < L - 1; ++v) stage(v, nullptr, 0);
     const Stage &SL = m->st[L - 1];
     timed(L - 1, 2 * SL.macs * rm.R, [&] { return launch_final_dense(SL, xsrc(L - 1), rm, fa, s); });

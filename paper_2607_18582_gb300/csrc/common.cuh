@@ -142,8 +142,15 @@ int tc_small_geometry(const Stage &S);
 int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t s);
 int64_t tc_swizzle_tmp_floats(const Stage &S);
 int64_t tc_macs_per_row(const Stage &S);
+// The output layer (dense, C <= 12 classes) computed in the epilogue of the
+// tensor-core dense layer that feeds it, with the kill epilogue: W [C][F], bias b,
+// activation act.  The rows of the layer in between are then never stored.
+struct FinalFuse;
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
-              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov = nullptr);
+              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov = nullptr,
+              const FinalFuse *ff = nullptr);
+// Whether stage S (feeding the output layer SL) can take SL into its epilogue.
+int tc_final_fusable(const Stage &S, const Stage &SL);
 
 // Global average pooling of R rows of a [P][C] map.
 int launch_gap(const float *in, int64_t in_stride, int P, int C, int R, float *y, int64_t y_stride, cudaStream_t s);
@@ -168,6 +175,12 @@ struct FinalArgs {
 };
 int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s,
                        const Overlay *ov = nullptr);
+struct FinalFuse {
+    const float *W;   // [C][F]
+    const float *b;   // [C]
+    int C, F, act;
+    FinalArgs fa;     // kill mode
+};
 
 // Kill epilogue on logits rows (mutants of the output layer), with an optional overlay.
 int launch_epilogue(Src logits, int C, RowMap rm, const FinalArgs &fa, cudaStream_t s, const Overlay *ov = nullptr);

@@ -33,6 +33,7 @@
 
 #include "common.cuh"
 #include "device_util.cuh"
+#include "epilogue.cuh"
 
 namespace mure {
 
@@ -43,6 +44,7 @@ constexpr int kTileK = 32;             // fp32 / tf32 values per 128-byte row
 constexpr int kNA = 4;                 // producer cp.async ring depth (K-steps)
 constexpr int kNB = 3;                 // streamed weight stages
 constexpr int kSlice = 128;            // output channels per CTA
+constexpr int kFuseClasses = 12;       // classes of an output layer fused into a dense epilogue
 constexpr int kThreads = 384;          // 4 producer + 4 epilogue + 3 MMA + weight warps
 constexpr int kEpiStride = 36;         // floats per row of an epilogue staging chunk (32 + pad)
 constexpr int kMaxNT = 8;              // tensor-memory A stages, at most
@@ -266,6 +268,7 @@ struct TcParams {
     int n_stages;                // tensor-memory A stages (<= kMaxNT), from column a_col
     int a_col;
     int *err;
+    FinalFuse ff;                // the output layer computed in the epilogue (FCP > 0)
 };
 
 // Per producer ring slot, the overlay values of a row's K-step: up to kOvMax
@@ -522,10 +525,14 @@ struct SmallSteps {
 };
 
 // MODE 0: dense layer (one GEMM row per batch row); 1: implicit-GEMM convolution; 2:
-// the small-image convolution.  THREE: 3xTF32 (else one TF32 product).
-template <int MODE, bool THREE>
+// the small-image convolution.  THREE: 3xTF32 (else one TF32 product).  FCP > 0
+// (dense, one N slice): the output layer, with up to FCP classes, is computed from
+// each row's outputs in the epilogue, followed by the kill epilogue, and the rows
+// themselves are not stored.
+template <int MODE, bool THREE, int FCP = 0>
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
 {
+    static_assert(FCP == 0 || (MODE == 0 && FCP % 4 == 0), "the output layer is fused into dense layers only");
     constexpr bool DENSE = MODE == 0;
     constexpr int kNT = kMaxNT;                    // barrier slots; p.n_stages are used
     constexpr int kAColsPerStage = THREE ? 64 : 32;
@@ -551,6 +558,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     const uint32_t b_region = sbase;
     const uint32_t a_region = sbase + (p.b_resident ? (uint32_t)nK * b_step : (uint32_t)kNB * b_step);
     const uint32_t ov_region = a_region + kNA * kStageA;    // kNA overlay slots (with an overlay)
+    // FCP > 0: the output layer's weights as [F][FCP] (zeros beyond its C classes)
+    const uint32_t fw_region = (ov_region + (p.ov.patch ? kNA * kOvSlotBytes : 0) + 15u) & ~15u;
     const int64_t M = (int64_t)p.R * p.P;
     const int64_t n_tiles = MODE == 2 ? small_tiles(p.R) : (M + kTileM - 1) / kTileM;
     const int64_t my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
@@ -561,6 +570,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_sh)),
                      "r"(512));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    if constexpr (FCP > 0) {
+        for (int i = threadIdx.x; i < p.ff.F * FCP; i += kThreads) {
+            const int f = i / FCP, c = i % FCP;
+            const float wv = c < p.ff.C ? p.ff.W[(int64_t)c * p.ff.F + f] : 0.f;
+            asm volatile("st.shared.f32 [%0], %1;" ::"r"(fw_region + 4 * i), "f"(wv) : "memory");
+        }
     }
     for (int n = threadIdx.x; n < kSlice; n += kThreads) {
         if (MODE == 2) bias_sh[n] = n < SmallConv::N ? p.b[n % SmallConv::OC] : 0.f;
@@ -800,6 +816,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             const bool vec = DENSE || (p.N & 3) == 0;
             if (!(!DENSE && p.pool))
                 epi_ptr[qd][lane] = ri.ok ? yrow + (DENSE ? 0 : ((int64_t)ri.oy * p.ow + ri.ox) * p.N) : nullptr;
+            float facc[FCP > 0 ? FCP : 1];
+#pragma unroll
+            for (int c = 0; c < (FCP > 0 ? FCP : 1); ++c) facc[c] = 0.f;
             for (int n0 = 0; n0 < Nt; n0 += 32) {
                 const int nc = min(32, Nt - n0);
                 float v[32];
@@ -828,6 +847,27 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                     if (p.act1 == MURE_ACT_RELU) {
 #pragma unroll
                         for (int e = 0; e < 16; ++e) vh[e] = act_apply(MURE_ACT_RELU, vh[e]);
+                    }
+                    if constexpr (FCP > 0) {
+                        // the output layer: fp32 FMAs over the inputs f in ascending
+                        // order, as the output-layer kernel does
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const int f = n0 + h + e;
+                            if (f < p.N) {
+#pragma unroll
+                                for (int c4 = 0; c4 < FCP; c4 += 4) {
+                                    float4 w4;
+                                    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                                                 : "=f"(w4.x), "=f"(w4.y), "=f"(w4.z), "=f"(w4.w)
+                                                 : "r"(fw_region + (uint32_t)(f * FCP + c4) * 4));
+                                    facc[c4] = fmaf(vh[e], w4.x, facc[c4]);
+                                    facc[c4 + 1] = fmaf(vh[e], w4.y, facc[c4 + 1]);
+                                    facc[c4 + 2] = fmaf(vh[e], w4.z, facc[c4 + 2]);
+                                    facc[c4 + 3] = fmaf(vh[e], w4.w, facc[c4 + 3]);
+                                }
+                            }
+                        }
                     }
                     if (!DENSE && p.has_add && ri.ok) {
                         const float *sp = srow + ((int64_t)ri.oy * p.sk_stride * p.sk_w + ri.ox * p.sk_stride) * p.sk_c;
@@ -862,7 +902,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                         }
                     }
                 }
-                if (!DENSE && p.pool) continue;
+                if ((!DENSE && p.pool) || FCP > 0) continue;
 #pragma unroll
                 for (int c = 0; c < 8; ++c)
                     *reinterpret_cast<float4 *>(stage + lane * kEpiStride + 4 * c) =
@@ -890,6 +930,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
+            if constexpr (FCP > 0) {
+                // logits = act(acc + b), then argmax / kill as the output-layer kernel
+                float lv[FCP];
+#pragma unroll
+                for (int c = 0; c < FCP; ++c) lv[c] = c < p.ff.C ? act_apply(p.ff.act, facc[c] + __ldg(p.ff.b + c)) : 0.f;
+                epilogue_reg<FCP>(p.ff.fa, p.t0, p.T, ri.row, ri.ok, lv, p.ff.C);
+            }
         }
     } else if (MODE == 2 && warp == 10) {
         // ------------------------------------------------ map staging: finish --
@@ -1177,8 +1224,15 @@ static void tc_config(TcParams &p, int nt_max, bool three)
     p.n_mma = m;
 }
 
+int tc_final_fusable(const Stage &S, const Stage &SL)
+{
+    return S.tc && S.kind == MURE_NODE_DENSE && tc_supported(S) && round_up16(S.oc) <= kSlice &&
+           SL.kind == MURE_NODE_DENSE && SL.K == S.oc && SL.oc >= 1 && SL.oc <= kFuseClasses && !SL.has_add &&
+           !SL.gap && !SL.pool;
+}
+
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
-              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov)
+              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov, const FinalFuse *ff)
 {
     if (rm.R <= 0) return 0;
     TcParams p{};
@@ -1219,7 +1273,9 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     // at least 116 KiB so that one CTA (holding all 512 tensor-memory columns) runs per SM
     const size_t a_bytes = S.tc_small ? (size_t)SmallConv::BYTES
                                       : (size_t)kNA * kStageA + (p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0);
-    const size_t smem = std::max<size_t>(1024 + b_bytes + a_bytes, 116 * 1024);
+    if (ff) p.ff = *ff;
+    const size_t f_bytes = ff ? 16 + (size_t)ff->F * kFuseClasses * 4 : 0;
+    const size_t smem = std::max<size_t>(1024 + b_bytes + a_bytes + f_bytes, 116 * 1024);
     // partial accumulators: two sets of n_mma in columns 0..255; a function of the layer
     // alone, so a row's arithmetic never depends on the batch
     tc_config(p, nt_max, three);
@@ -1239,7 +1295,8 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, kThreads, smem, s>>>(p);
     };
-    if (dense) { if (three) go(k_tc_gemm<0, true>); else go(k_tc_gemm<0, false>); }
+    if (dense && ff) { if (three) go(k_tc_gemm<0, true, kFuseClasses>); else go(k_tc_gemm<0, false, kFuseClasses>); }
+    else if (dense) { if (three) go(k_tc_gemm<0, true>); else go(k_tc_gemm<0, false>); }
     else if (S.tc_small) { if (three) go(k_tc_gemm<2, true>); else go(k_tc_gemm<2, false>); }
     else { if (three) go(k_tc_gemm<1, true>); else go(k_tc_gemm<1, false>); }
     int launches = 1;
