@@ -506,6 +506,7 @@ struct Workspace {
     int64_t z_stride = 0;
     float *gap_tmp = nullptr;
     int64_t rows = 0;
+    TcDeltaWs dw;              // tensor-core delta scratch (GF / WS slots of a batch)
 };
 
 int64_t gap_map_stride(const Stage &S)
@@ -530,9 +531,24 @@ int64_t row_bytes(const mure_model *m, int l, bool vanilla)
 }
 
 void alloc_workspace(mure_ctx *c, Scratch &sc, const mure_model *m, int64_t rows, bool vanilla, int lmin,
-                     int64_t patch_floats, Workspace &ws)
+                     int64_t patch_floats, int delta_slots, int delta_k, Workspace &ws)
 {
     ws.rows = rows;
+    if (delta_slots > 0) {
+        int64_t nf = 0, ni = 0;
+        tc_delta_ws_size(delta_slots, delta_k, nf, ni);
+        const int64_t Np = (delta_slots + 127) / 128 * 128;
+        float *f = sc.get<float>(nf);
+        ws.dw.filt = f;
+        ws.dw.swz = f + Np * delta_k;
+        ws.dw.colb = ws.dw.swz + 2 * Np * round_up32(delta_k);
+        int32_t *ip = sc.get<int32_t>(ni);
+        ws.dw.colg = ip;
+        ws.dw.colq = ip + Np;
+        ws.dw.colj = ip + 2 * Np;
+        ws.dw.n_max = delta_slots;
+        ws.dw.k_max = delta_k;
+    }
     ws.patch = sc.get<float>(rows * std::max<int64_t>(patch_floats, 1));
     ws.xb.assign(m->L + 1, nullptr);
     for (int s = vanilla ? 1 : lmin + 1; s <= m->L; ++s) ws.xb[s] = sc.get<float>(rows * m->xd[s].stride);
@@ -628,13 +644,26 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     const int64_t pstride = (int64_t)std::max(kmax, 1) * cells_l;
     const Src zsrc = vanilla ? Src{ws.zb, ws.z_stride, 0} : Src{ca->z[l], m->zd[l].stride, 1};
     acct.bytes_gather += (int64_t)rm.R * kmax * cells_l * 4;
-    const bool dot_kernel = patch_dot_supported(Sl, kmax);
+    // GF / WS: on the tensor cores (one GEMM over the batch's inputs with every slot's
+    // mutated filter as an output channel), else the CUDA-core dot-product kernels
+    const bool tc_delta = tc_delta_supported(Sl, m->precision) && ws.dw.n_max > 0;
+    const bool dot_kernel = !tc_delta && patch_dot_supported(Sl, kmax);
+    const bool has_dot = dt.dot_prefix[g0 + G] > dt.dot_prefix[g0];
+    int delta_err = 0;
     timed(C_DELTA, delta_flops, [&] {
-        int n = launch_patch_vals(Sl, zsrc, xsrc(l), skip_of(Sl), rm, pa, kmax, ws.patch, pstride, s, dot_kernel);
-        if (dot_kernel && dt.dot_prefix[g0 + G] > dt.dot_prefix[g0])
+        int n = launch_patch_vals(Sl, zsrc, xsrc(l), skip_of(Sl), rm, pa, kmax, ws.patch, pstride, s,
+                                  dot_kernel || tc_delta);
+        if (tc_delta && has_dot) {
+            // the inputs' x_l and z_l: cached rows (memoized) or the batch's first
+            // mutant's recomputed rows (vanilla; the prefix up to layer l is unmutated)
+            const int d = launch_tc_delta(Sl, m->precision, zsrc, xsrc(l), rm, pa, ws.patch, pstride, ws.dw, s);
+            if (d < 0) delta_err = 1; else n += d;
+        } else if (dot_kernel && has_dot) {
             n += launch_patch_dot(Sl, zsrc, xsrc(l), rm, pa, kmax, ws.patch, pstride, s);
+        }
         return n;
     });
+    if (delta_err) return -1;
     Overlay ov;
     ov.patch = ws.patch;
     ov.row_stride = pstride;
@@ -761,8 +790,16 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
             const int64_t cl = S.gap ? 1 : (S.pool ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow);
             patch_floats = std::max<int64_t>(patch_floats, (int64_t)std::max(dt.kmax_layer[l], 1) * cl);
         }
+        // the tensor-core delta: slots of a batch at most G x kmax of its layer
+        int delta_slots = 0, delta_k = 0;
+        for (int l = 0; l < m->L; ++l) {
+            if (g.begin[l + 1] == g.begin[l] || !tc_delta_supported(m->st[l], m->precision)) continue;
+            const int64_t gb = std::min<int64_t>(Gmax, g.begin[l + 1] - g.begin[l]);
+            delta_slots = (int)std::max<int64_t>(delta_slots, gb * std::max(dt.kmax_layer[l], 1));
+            delta_k = std::max(delta_k, m->st[l].K);
+        }
         Workspace ws;
-        alloc_workspace(c, sc, m, rows, vanilla, lmin, patch_floats, ws);
+        alloc_workspace(c, sc, m, rows, vanilla, lmin, patch_floats, delta_slots, delta_k, ws);
         int64_t launches = 0;
         Acct acct;
         acct.flops_cls.assign(m->L + 3, 0);
@@ -777,7 +814,9 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
                 for (int64_t g0 = gs; g0 < ge; g0 += Gmax) {
                     const int64_t G = std::min<int64_t>(Gmax, ge - g0);
                     RowMap rm{t0, Tt, (int)(G * Tt)};
-                    launches += run_batch(c, m, ca, dt, ec, ws, l, g0, rm, vanilla, acct, tm);
+                    const int nb = run_batch(c, m, ca, dt, ec, ws, l, g0, rm, vanilla, acct, tm);
+                    FAILIF(nb < 0, c, MURE_ERR_UNSUPPORTED, "delta scratch too small for layer %d", l);
+                    launches += nb;
                     check_launch(c);
                     ++st.n_batches;
                 }

@@ -146,9 +146,22 @@ int64_t tc_macs_per_row(const Stage &S);
 // tensor-core dense layer that feeds it, with the kill epilogue: W [C][F], bias b,
 // activation act.  The rows of the layer in between are then never stored.
 struct FinalFuse;
+// Output of the tensor-core delta: column n < n of the GEMM is slot (g[n], q[n]) of the
+// batch, channel j[n] of the layer; the GEMM's sum is added to the pre-activation
+// z[row][j][position] before the post-ops, and the value for output cell c of input
+// row r goes to out[(g * T + r) * stride + q * cells + c].
+struct SlotStore {
+    float *out = nullptr;
+    int64_t stride = 0;
+    const int32_t *g = nullptr, *q = nullptr, *j = nullptr;
+    int n = 0, cells = 0, T = 0;
+    const float *z = nullptr;
+    int64_t z_stride = 0;
+    int z_per_input = 0;
+};
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
               int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov = nullptr,
-              const FinalFuse *ff = nullptr);
+              const FinalFuse *ff = nullptr, const SlotStore *ss = nullptr);
 // Whether stage S (feeding the output layer SL) can take SL into its epilogue.
 int tc_final_fusable(const Stage &S, const Stage &SL);
 
@@ -204,6 +217,23 @@ struct PatchArgs {
 // out[r][q][c] (slot q < kmax, output cell c of layer l).
 int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *out,
                       int64_t out_stride, cudaStream_t s, bool skip_dot_ops = false);
+
+// GF / WS delta values on the tensor cores (convolution layers, tensor-core precision
+// modes): one implicit GEMM over the batch's inputs whose output channels are the
+// weight deltas e of every GF / WS slot of the batch (128 per N slice, so a slot's
+// arithmetic never depends on the batch); the epilogue adds the cached pre-activation
+// z of the slot's channel (e = 0 gives z exactly), applies the layer's post-ops and
+// stores into the patch rows.  Scratch: filters, their swizzled halves and per-column tables
+// for up to n_max slots of fan-in up to k_max.
+struct TcDeltaWs {
+    float *filt = nullptr, *swz = nullptr, *colb = nullptr;
+    int32_t *colg = nullptr, *colq = nullptr, *colj = nullptr;
+    int n_max = 0, k_max = 0;
+};
+int tc_delta_supported(const Stage &S, int precision);
+void tc_delta_ws_size(int n_slots, int k_max, int64_t &floats, int64_t &ints);
+int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_inputs, const PatchArgs &pa, float *out,
+                    int64_t out_stride, const TcDeltaWs &dw, cudaStream_t s);
 
 // GF / WS delta values of the small-layer geometries (stage variant > 0): the same
 // values as launch_patch_vals for those operators; launch_patch_vals then skips them.

@@ -269,6 +269,7 @@ struct TcParams {
     int a_col;
     int *err;
     FinalFuse ff;                // the output layer computed in the epilogue (FCP > 0)
+    SlotStore slot;              // slot.out: the tensor-core delta's scattered store
 };
 
 // Per producer ring slot, the overlay values of a row's K-step: up to kOvMax
@@ -844,6 +845,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                             else p.z[ri.row * p.z_stride + (int64_t)n * (p.oh * p.ow) + ri.oy * p.ow + ri.ox] = vh[e];
                         }
                     }
+                    if (!DENSE && p.slot.out && ri.ok) {
+                        // the delta GEMM's sum on top of the slot channel's pre-activation
+                        const float *zr = p.slot.z + (p.slot.z_per_input ? p.t0 + ri.row : ri.row) * p.slot.z_stride +
+                                          ri.oy * p.ow + ri.ox;
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const int n = n_base + n0 + h + e;
+                            if (n < p.slot.n) vh[e] = __ldg(zr + (int64_t)__ldg(p.slot.j + n) * (p.oh * p.ow)) + vh[e];
+                        }
+                    }
                     if (p.act1 == MURE_ACT_RELU) {
 #pragma unroll
                         for (int e = 0; e < 16; ++e) vh[e] = act_apply(MURE_ACT_RELU, vh[e]);
@@ -878,6 +889,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                             vh[e] = act_apply(p.act2, vh[e] + sv);
                         }
                     }
+                    if (!DENSE && !p.pool && p.slot.out && ri.ok) {
+                        const int cell = ri.oy * p.ow + ri.ox;
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const int n = n_base + n0 + h + e;
+                            if (n < p.slot.n)
+                                p.slot.out[((int64_t)__ldg(p.slot.g + n) * p.slot.T + ri.row) * p.slot.stride +
+                                           (int64_t)__ldg(p.slot.q + n) * p.slot.cells + cell] = vh[e];
+                        }
+                    }
                     if (!DENSE && p.pool) {
                         // lanes 4w .. 4w+3 hold the four positions of one pooling window
 #pragma unroll
@@ -887,7 +908,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                             const float w3 = __shfl_down_sync(0xffffffffu, vh[e], 3);
                             if ((lane & 3) == 0) vh[e] = max4_first(vh[e], w1, w2, w3);
                         }
-                        if (ri.ok && (lane & 3) == 0) {
+                        if (p.slot.out) {
+                            if (ri.ok && (lane & 3) == 0) {
+                                const int cell = ri.py * p.pw + ri.px;
+#pragma unroll
+                                for (int e = 0; e < 16; ++e) {
+                                    const int n = n_base + n0 + h + e;
+                                    if (n < p.slot.n)
+                                        p.slot.out[((int64_t)__ldg(p.slot.g + n) * p.slot.T + ri.row) * p.slot.stride +
+                                                   (int64_t)__ldg(p.slot.q + n) * p.slot.cells + cell] = vh[e];
+                                }
+                            }
+                        } else if (ri.ok && (lane & 3) == 0) {
                             float *yo = yrow + ((int64_t)ri.py * p.pw + ri.px) * p.N + n_base + n0 + h;
                             if (n_base + n0 + h + 15 < p.N && (p.N & 3) == 0) {
 #pragma unroll
@@ -902,7 +934,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                         }
                     }
                 }
-                if ((!DENSE && p.pool) || FCP > 0) continue;
+                if ((!DENSE && p.pool) || FCP > 0 || p.slot.out) continue;
 #pragma unroll
                 for (int c = 0; c < 8; ++c)
                     *reinterpret_cast<float4 *>(stage + lane * kEpiStride + 4 * c) =
@@ -1232,7 +1264,8 @@ int tc_final_fusable(const Stage &S, const Stage &SL)
 }
 
 int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
-              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov, const FinalFuse *ff)
+              int64_t y_stride, float *gap_tmp, cudaStream_t s, const Overlay *ov, const FinalFuse *ff,
+              const SlotStore *ss)
 {
     if (rm.R <= 0) return 0;
     TcParams p{};
@@ -1274,11 +1307,15 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     const size_t a_bytes = S.tc_small ? (size_t)SmallConv::BYTES
                                       : (size_t)kNA * kStageA + (p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0);
     if (ff) p.ff = *ff;
+    if (ss) p.slot = *ss;
     const size_t f_bytes = ff ? 16 + (size_t)ff->F * kFuseClasses * 4 : 0;
     const size_t smem = std::max<size_t>(1024 + b_bytes + a_bytes + f_bytes, 116 * 1024);
     // partial accumulators: two sets of n_mma in columns 0..255; a function of the layer
     // alone, so a row's arithmetic never depends on the batch
     tc_config(p, nt_max, three);
+    // the delta GEMM: one issuing warp, so that a column's sum never depends on how many
+    // slots share its batch
+    if (ss) p.n_mma = 1;
     if (S.tc_small) p.n_mma = std::min(p.n_mma, 2);   // warp 10 stages maps in that mode
     const int64_t M = (int64_t)rm.R * p.P;
     const int64_t tiles = S.tc_small ? small_tiles(rm.R) : (M + kTileM - 1) / kTileM;
@@ -1302,6 +1339,78 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     int launches = 1;
     if (S.gap) launches += launch_gap(gap_tmp, map_stride, mh * mw, S.oc, rm.R, y_out, y_stride, s);
     return launches;
+}
+
+// ------------------------------------------------ tensor-core delta (GF / WS) --
+
+// Column n of the batch's delta GEMM: slot n (its pair (group, q) listed by the host)
+// takes the weight delta e of its neuron j (GF: the noise; WS: W[j][perm f] - W[j][f]);
+// columns past the slots are zero.  The column bias is 0: the epilogue adds the cached
+// pre-activation of channel j instead.  One thread per (column, k).
+__global__ void k_slot_filters(int K, const PatchArgs pa, int n_slot, int Np, float *filt, float *colb, int32_t *colg,
+                               int32_t *colq, int32_t *colj)
+{
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (int64_t)Np * K) return;
+    const int n = (int)(i / K), k = (int)(i - (int64_t)n * K);
+    if (n >= n_slot) {
+        filt[i] = 0.f;
+        if (k == 0) { colb[n] = 0.f; colg[n] = 0; colq[n] = 0; colj[n] = 0; }
+        return;
+    }
+    const int g = pa.dslot[2 * n] - pa.dslot_g0, q = pa.dslot[2 * n + 1];
+    filt[i] = pa.patch[pa.patch_off[g] + (int64_t)q * K + k];
+    if (k == 0) { colb[n] = 0.f; colg[n] = g; colq[n] = q; colj[n] = pa.ids[pa.neuron_off[g] + q]; }
+}
+
+// Layers with a compiled small geometry keep the CUDA-core dot-product kernel, which
+// stages each input once for all slots; the GEMM's gathers want channel counts that
+// are multiples of 4 (16-byte copies).
+int tc_delta_supported(const Stage &S, int precision)
+{
+    return precision != MURE_PREC_FP32 && S.kind == MURE_NODE_CONV2D && !S.has_add && !S.gap && S.geo == 0 &&
+           S.ic % 4 == 0;
+}
+
+void tc_delta_ws_size(int n_slots, int k_max, int64_t &floats, int64_t &ints)
+{
+    const int64_t Np = (int64_t)(n_slots + kSlice - 1) / kSlice * kSlice, Kp = round_up32(k_max);
+    floats = Np * k_max + 2 * Np * Kp + Np;   // filters, swizzled halves, biases
+    ints = 3 * Np;
+}
+
+int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_inputs, const PatchArgs &pa, float *out,
+                    int64_t out_stride, const TcDeltaWs &dw, cudaStream_t s)
+{
+    const int n = (int)pa.n_dslot;
+    if (n <= 0 || rm_inputs.R <= 0) return 0;
+    const int Np = round_up16(n), K = S.K, Kp = round_up32(K);
+    if (n > dw.n_max || K > dw.k_max) return -1;
+    const int planes = precision == MURE_PREC_TF32X3 ? 2 : 1;
+    k_slot_filters<<<(unsigned)(((int64_t)Np * K + 255) / 256), 256, 0, s>>>(K, pa, n, Np, dw.filt, dw.colb, dw.colg,
+                                                                         dw.colq, dw.colj);
+    k_swizzle_weights<<<(unsigned)(((int64_t)Np * Kp + 255) / 256), 256, 0, s>>>(dw.filt, Np, K, Np, Kp, planes,
+                                                                               (int64_t)planes * kSlice * Kp, dw.swz);
+    Stage D = S;
+    D.oc = Np;
+    D.tc = precision == MURE_PREC_TF32X3 ? 1 : 2;
+    D.tc_small = 0;
+    D.Wtc = dw.swz;
+    D.b = dw.colb;
+    SlotStore ss;
+    ss.out = out;
+    ss.stride = out_stride;
+    ss.g = dw.colg;
+    ss.q = dw.colq;
+    ss.j = dw.colj;
+    ss.z = z.p;
+    ss.z_stride = z.stride;
+    ss.z_per_input = z.per_input;
+    ss.n = n;
+    ss.cells = S.pool ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
+    ss.T = rm_inputs.T;
+    const RowMap rmT{rm_inputs.t0, rm_inputs.T, rm_inputs.T};
+    return 2 + launch_tc(D, x, rmT, nullptr, 0, Src{nullptr, 0, 0}, nullptr, 0, nullptr, s, nullptr, nullptr, &ss);
 }
 
 }  // namespace mure
