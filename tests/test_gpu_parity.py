@@ -183,6 +183,27 @@ def test_batch_invariance(M, ctx, prec):
     assert np.array_equal(sub["logits"].view(np.uint32), big["logits"][:, :70].view(np.uint32))
 
 
+@pytest.mark.parametrize("prec", ["tf32x3", "tf32"])
+def test_batch_invariance_tensor_core_delta(M, ctx, prec):
+    """GF / WS deltas of the generic convolutions run as one tensor-core GEMM per batch
+    whose output channels are the batch's slots: a slot's values must not depend on
+    how many other slots share its batch (many small batches vs one)."""
+    w = wl.workload("vgg", 64, 1)
+    rows = []
+    for l in range(1, w.model.n_layers() - 2):
+        for i in range(6):
+            rows.append((l, "GF" if i % 2 == 0 else "WS", [i, i + 7], 1.0 if i % 2 == 0 else 0.0, 100 + 7 * l + i))
+    table = wl.table_from_rows(rows)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
+    cache = M.mure_build_prefix_cache(model, w.X)
+    big = M.mure_eval_mutants(cache, table, logits=True)
+    small = M.mure_eval_mutants(cache, table, logits=True, workspace_bytes=32 << 20)
+    assert small["stats"]["n_batches"] > big["stats"]["n_batches"]
+    assert np.array_equal(big["logits"].view(np.uint32), small["logits"].view(np.uint32))
+    van = M.mure_eval_vanilla(model, w.X, table, logits=True)
+    assert np.array_equal(big["logits"].view(np.uint32), van["logits"].view(np.uint32))
+
+
 @pytest.mark.parametrize("name,prec", [("resnet20", "fp32"), ("mlp", "tf32x3"), ("lenet5", "tf32x3")])
 def test_identity_mutants_never_killed(M, ctx, name, prec):
     w = wl.workload(name, 96, 1)
