@@ -130,6 +130,38 @@ def profiled_traffic(kernel_key, rows_per_launch):
     return float(m_bytes.group(1)) * rows_per_launch
 
 
+def hbm_rates(w, results, cls_ms, pk, pk_kind):
+    """Achieved HBM bandwidth of the memory-bound kernel classes against the measured
+    copy bandwidth: the delta kernels (algorithmic bytes = the patch values they write;
+    the cached z / x rows that each input stages once for all mutants are not counted)
+    and the stand-alone output-layer kernel (its input rows read once, 1 bit written
+    per row).  CUDA-event times of the timed steps."""
+    out = {}
+    peak = pk["hbm_gbs"]
+    ms = cls_ms.get("delta", 0.0)
+    byts = sum(r["stats"]["bytes_gather"] for r in results)
+    if ms > 0 and byts > 0:
+        gbs = byts / (ms / 1e3) / 1e9
+        out["delta"] = {"kernels": "k_patch_* (delta)", "bytes": byts, "ms": ms, "achieved": gbs, "unit": "GB/s",
+                        "frac": gbs / peak, "bytes_counted": "patch values written"}
+    L = w.model.n_layers()
+    last = f"layer{L - 1}"
+    ms = cls_ms.get(last, 0.0)
+    fl = sum(r["stats"]["flops_layer"][L - 1] for r in results)
+    macs = w.model.layer_macs(L - 1)
+    if ms > 0 and fl > 0:
+        rows = fl / 2 / macs
+        node = w.model.nodes[w.model.layers()[L - 1]]
+        byts = rows * (node.cin * 4 + 1 / 8)
+        gbs = byts / (ms / 1e3) / 1e9
+        out["output_layer"] = {"kernels": "k_final_dense (output layer + kill, rows not fused into a dense epilogue)",
+                               "bytes": byts, "ms": ms, "achieved": gbs, "unit": "GB/s", "frac": gbs / peak,
+                               "bytes_counted": "input rows read once, kill bits written"}
+    out["peak"] = peak
+    out["peak_source"] = f"{pk_kind} (MEASURED_PEAKS.json hbm_gbs)"
+    return out
+
+
 # ------------------------------------------------------------- distributed --
 
 def dist_setup():
@@ -396,6 +428,7 @@ def main():
         rate, dt, sample = cpu_oracle_rate(w, 400, 2000, threads)
         out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
                                "seconds": dt}
+    out["hbm"] = hbm_rates(w, results, cls_ms, pk, pk_kind)
     out["peaks"] = {"source": pk_kind, "hbm_gbs": pk.get("hbm_gbs"), "bf16_tflops": pk.get("bf16_tflops")}
     if rank == 0:
         print(json.dumps(out), flush=True)

@@ -389,6 +389,8 @@ struct DevTable {
     std::vector<int> kmax_layer;
     std::vector<int64_t> dot_prefix;   // [n+1] prefix sums of GF/WS neuron slots (group order)
     int32_t *dslot = nullptr;          // [dot_prefix[n]] GF/WS slots in group order: (group, slot q)
+    std::vector<int64_t> val_prefix;   // [n+1] prefix sums of NEB/NAI/NS neuron slots (group order)
+    int4 *vslot = nullptr;             // [val_prefix[n]] those slots: (group, q, source channel, op)
     int expand_launches = 0;
 };
 
@@ -434,14 +436,25 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
     for (int64_t k = 0; k < n; ++k)
         if (op[k] == MURE_OP_GF || op[k] == MURE_OP_WS)
             for (int q = 0; q < nn[k]; ++q) { dslot.push_back((int32_t)k); dslot.push_back(q); }
+    // the operators without a fan-in sum: NS reads its partner neuron's channel
+    dt.val_prefix.assign(n + 1, 0);
+    std::vector<int4> vslot;
+    for (int64_t k = 0; k < n; ++k) {
+        const bool val = op[k] == MURE_OP_NEB || op[k] == MURE_OP_NAI || op[k] == MURE_OP_NS;
+        dt.val_prefix[k + 1] = dt.val_prefix[k] + (val ? nn[k] : 0);
+        if (val)
+            for (int q = 0; q < nn[k]; ++q)
+                vslot.push_back(make_int4((int)k, q, pool[noff[k] + (op[k] == MURE_OP_NS ? (q ^ 1) : q)], op[k]));
+    }
     // one staging buffer, one H2D copy
     const size_t b_op = n * 4, b_nn = n * 4, b_mid = n * 4, b_noff = n * 8, b_poff = n * 8;
-    const size_t b_dslot = std::max<size_t>(dslot.size(), 1) * 4;
+    const size_t b_dslot = std::max<size_t>(dslot.size(), 1) * 4, b_vslot = std::max<size_t>(vslot.size(), 1) * 16;
     const size_t b_ids = (size_t)std::max<int64_t>(pool_len, 1) * 4, b_jobs = jobs.size() * sizeof(SlotJob);
     size_t off = 0;
     auto place = [&](size_t b) { size_t o = off; off = round_up(off + b, 256); return o; };
     const size_t o_op = place(b_op), o_nn = place(b_nn), o_mid = place(b_mid), o_noff = place(b_noff),
-                 o_poff = place(b_poff), o_ids = place(b_ids), o_jobs = place(b_jobs), o_dslot = place(b_dslot);
+                 o_poff = place(b_poff), o_ids = place(b_ids), o_jobs = place(b_jobs), o_dslot = place(b_dslot),
+                 o_vslot = place(b_vslot);
     std::vector<char> host(off);
     memcpy(host.data() + o_op, op.data(), b_op);
     memcpy(host.data() + o_nn, nn.data(), b_nn);
@@ -451,6 +464,7 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
     if (pool_len > 0) memcpy(host.data() + o_ids, pool, pool_len * 4);
     if (!jobs.empty()) memcpy(host.data() + o_jobs, jobs.data(), b_jobs);
     if (!dslot.empty()) memcpy(host.data() + o_dslot, dslot.data(), dslot.size() * 4);
+    if (!vslot.empty()) memcpy(host.data() + o_vslot, vslot.data(), vslot.size() * 16);
     char *dev = sc.get<char>(off);
     CK(c, cudaMemcpyAsync(dev, host.data(), off, cudaMemcpyHostToDevice, c->stream));
     dt.op = (int32_t *)(dev + o_op);
@@ -460,6 +474,7 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
     dt.poff = (int64_t *)(dev + o_poff);
     dt.ids = (int32_t *)(dev + o_ids);
     dt.dslot = (int32_t *)(dev + o_dslot);
+    dt.vslot = (int4 *)(dev + o_vslot);
     dt.patch = plen ? sc.get<float>(plen) : nullptr;
     if (!jobs.empty()) {
         std::vector<const float *> Wp(m->L);
@@ -591,6 +606,8 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     pa.dslot = dt.dslot + 2 * dt.dot_prefix[g0];
     pa.n_dslot = dt.dot_prefix[g0 + rm.R / rm.T] - dt.dot_prefix[g0];
     pa.dslot_g0 = (int32_t)g0;
+    pa.vslot = dt.vslot + dt.val_prefix[g0];
+    pa.n_vslot = dt.val_prefix[g0 + rm.R / rm.T] - dt.val_prefix[g0];
     FinalArgs fa{};
     fa.mutant_id = dt.mid + g0;
     fa.label = ca->label;

@@ -210,6 +210,8 @@ struct PatchArgs {
     const int32_t *dslot = nullptr;   // the batch's GF / WS slots: (global group, slot q) pairs
     int64_t n_dslot = 0;
     int32_t dslot_g0 = 0;             // global index of the batch's first group
+    const int4 *vslot = nullptr;      // the batch's other slots: (global group, q, source channel, op)
+    int64_t n_vslot = 0;
 };
 
 // Delta of layer l: values of the mutated neurons' channels of x_{l+1}, from z_l

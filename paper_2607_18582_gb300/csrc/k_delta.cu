@@ -302,27 +302,22 @@ __global__ void __launch_bounds__(256) k_patch_vals_staged(const PatchValsParams
         coff[c] = p.pool ? 2 * (c / p.mcw) * p.ow + 2 * (c % p.mcw) : c;
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int sl = warp; sl < p.G * p.kmax; sl += blockDim.x >> 5) {
-        const int g = sl / p.kmax, q = sl - g * p.kmax;
-        if (q >= p.pa.n_neurons[g]) continue;
-        const int op = p.pa.op[g];
-        if (op == MURE_OP_GF || op == MURE_OP_WS) continue;
-        const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
-        const int sj = op == MURE_OP_NS ? ids[q ^ 1] : ids[q];
+    // the batch's NEB / NAI / NS slots (listed by the host), one warp per slot
+    for (int64_t sl = warp; sl < p.pa.n_vslot; sl += blockDim.x >> 5) {
+        const int4 e = p.pa.vslot[sl];
+        const int g = e.x - p.pa.dslot_g0, q = e.y, sj = e.z, op = e.w;
         const float *zc = zs + sj * P;
         float *o = p.out + ((int64_t)g * p.T + tl) * p.out_stride + q * p.cells;
         auto post = [&](float zz) {
             if (op == MURE_OP_NAI) zz = -zz;
             return op == MURE_OP_NEB ? 0.f : act_apply(p.act1, zz);
         };
-        if (p.pool) {
-            for (int c = lane; c < p.cells; c += 32) {
-                const int b = coff[c];
-                o[c] = max4_first(post(zc[b]), post(zc[b + 1]), post(zc[b + p.ow]), post(zc[b + p.ow + 1]));
-            }
-        } else {
-            for (int c = lane; c < p.cells; c += 32) o[c] = post(zc[coff[c]]);
-        }
+        auto cell = [&](int c) {
+            const int b = coff[c];
+            return p.pool ? max4_first(post(zc[b]), post(zc[b + 1]), post(zc[b + p.ow]), post(zc[b + p.ow + 1]))
+                          : post(zc[b]);
+        };
+        for (int c = lane; c < p.cells; c += 32) o[c] = cell(c);
     }
 }
 
@@ -432,8 +427,10 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
                         staged_smem <= 48 * 1024;
     int launches = 0;
     if (staged) {
-        k_patch_vals_staged<<<(unsigned)rm.T, 256, staged_smem, s>>>(p);
-        ++launches;
+        if (pa.n_vslot > 0) {
+            k_patch_vals_staged<<<(unsigned)rm.T, 256, staged_smem, s>>>(p);
+            ++launches;
+        }
         if (skip_dot_ops) return launches;
         p.only_dot_ops = 1;
     }
