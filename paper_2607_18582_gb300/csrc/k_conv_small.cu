@@ -290,18 +290,18 @@ __global__ void __launch_bounds__(256) k_patch_dot(const PatchDotParams p)
 
 // The same values in memoized mode, one input per block: the input's padded map and
 // its pre-activation maps are staged once, and every GF / WS slot of the batch (the
-// mutants share the inputs) is computed from there.  A thread takes one output cell
-// (a pooling window: four positions) for SG slots, so each filter tap costs 4 + SG
-// shared loads for 4 * SG FMAs.  Every sum is the same ascending fp32 chain as in
-// k_patch_dot, so the two kernels agree bit for bit.
-template <int KH, int KW, int IC, int WP, int HP, int PAD, bool POOL, int KMAX>
-__global__ void __launch_bounds__(256) k_patch_dot_in(const PatchDotParams p)
+// mutants share the inputs) is computed from there, SMAX slots' filters at a time.  A
+// thread takes CW output cells (pooling windows: 4 CW positions) for SG slots: each
+// filter tap costs 4 CW + SG shared loads (the slot loads are warp broadcasts) for
+// 4 CW SG FMAs.  Every sum is the same ascending fp32 chain as in k_patch_dot, so the
+// two kernels agree bit for bit.
+template <int KH, int KW, int IC, int WP, int HP, int PAD, bool POOL, int CW, int SG, int SMAX, int NT>
+__global__ void __launch_bounds__(NT) k_patch_dot_in(const PatchDotParams p)
 {
     constexpr int K = KH * KW * IC;
     constexpr int TILE = HP * WP * IC;
-    constexpr int SG = 4;          // slots per thread
-    constexpr int SMAX = 32;       // slots whose filters are staged at a time
     constexpr int NPOS = POOL ? 4 : 1;
+    constexpr int NP = CW * NPOS;          // positions per thread
     extern __shared__ __align__(16) float sm[];
     const int P = p.oh * p.ow;
     float *xs = sm;                       // [TILE] zero-padded input map
@@ -311,48 +311,53 @@ __global__ void __launch_bounds__(256) k_patch_dot_in(const PatchDotParams p)
     const int tl = blockIdx.x;
     const int64_t t = p.t0 + tl;
     const float *xin = p.x + t * p.x_stride;
-    for (int i = threadIdx.x; i < TILE; i += blockDim.x) {
+    for (int i = threadIdx.x; i < TILE; i += NT) {
         const int ci = i % IC, pix = i / IC, px = pix % WP, py = pix / WP;
         const int iy = py - PAD, ix = px - PAD;
         xs[i] = ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw) ? __ldg(xin + (iy * p.iw + ix) * IC + ci)
                                                                                   : 0.f;
     }
     const float *zin = p.z + t * p.z_stride;
-    for (int i = threadIdx.x; i < p.oc * P; i += blockDim.x) zsm[i] = __ldg(zin + i);
+    for (int i = threadIdx.x; i < p.oc * P; i += NT) zsm[i] = __ldg(zin + i);
     const int pw = POOL ? p.ow / 2 : p.ow;
+    const int chunks = (p.cells + CW - 1) / CW;
     // the batch's GF / WS slots (listed by the host), SMAX at a time
     for (int64_t s0 = 0; s0 < p.n_dslot; s0 += SMAX) {
         const int ns = (int)(p.n_dslot - s0 < SMAX ? p.n_dslot - s0 : SMAX);
         __syncthreads();
-        if (threadIdx.x < ns) {
-            const int g = p.dslot[2 * (s0 + threadIdx.x)] - p.dslot_g0, q = p.dslot[2 * (s0 + threadIdx.x) + 1];
-            sl_g[threadIdx.x] = g;
-            sl_q[threadIdx.x] = q;
-            sl_j[threadIdx.x] = p.ids[p.neuron_off[g] + q];
+        for (int i = threadIdx.x; i < ns; i += NT) {
+            const int g = p.dslot[2 * (s0 + i)] - p.dslot_g0, q = p.dslot[2 * (s0 + i) + 1];
+            sl_g[i] = g;
+            sl_q[i] = q;
+            sl_j[i] = p.ids[p.neuron_off[g] + q];
         }
         __syncthreads();
-        for (int i = threadIdx.x; i < ns * K; i += blockDim.x) {
+        for (int i = threadIdx.x; i < ns * K; i += NT) {
             const int sl = i / K, kk = i - sl * K;
             es[i] = __ldg(p.e_all + p.patch_off[sl_g[sl]] + (int64_t)sl_q[sl] * K + kk);
         }
         __syncthreads();
         const int groups = (ns + SG - 1) / SG;
-        for (int it = threadIdx.x; it < groups * p.cells; it += blockDim.x) {
-            const int sg = it / p.cells, c = it - sg * p.cells;
-            const int cy = c / pw, cx = c - cy * pw;
-            int off[NPOS];
-#pragma unroll
-            for (int s2 = 0; s2 < NPOS; ++s2) {
-                const int oy = POOL ? 2 * cy + (s2 >> 1) : cy, ox = POOL ? 2 * cx + (s2 & 1) : cx;
-                off[s2] = (oy * WP + ox) * IC;
-            }
+        for (int it = threadIdx.x; it < groups * chunks; it += NT) {
+            const int sg = it / chunks, ch = it - sg * chunks;
             const int nsg = min(SG, ns - sg * SG);
+            int off[NP];
+#pragma unroll
+            for (int w = 0; w < CW; ++w) {
+                const int c = min(ch * CW + w, p.cells - 1);   // a chunk past the last cell repeats it
+                const int cy = c / pw, cx = c - cy * pw;
+#pragma unroll
+                for (int s2 = 0; s2 < NPOS; ++s2) {
+                    const int oy = POOL ? 2 * cy + (s2 >> 1) : cy, ox = POOL ? 2 * cx + (s2 & 1) : cx;
+                    off[w * NPOS + s2] = (oy * WP + ox) * IC;
+                }
+            }
             const float *e0 = es + sg * SG * K;
-            float acc[SG][NPOS];
+            float acc[SG][NP];
 #pragma unroll
             for (int a = 0; a < SG; ++a)
 #pragma unroll
-                for (int s2 = 0; s2 < NPOS; ++s2) acc[a][s2] = 0.f;
+                for (int q2 = 0; q2 < NP; ++q2) acc[a][q2] = 0.f;
 #pragma unroll 1
             for (int ky = 0; ky < KH; ++ky)
 #pragma unroll
@@ -360,14 +365,14 @@ __global__ void __launch_bounds__(256) k_patch_dot_in(const PatchDotParams p)
 #pragma unroll
                     for (int ci = 0; ci < IC; ++ci) {
                         const int kk = (ky * KW + kx) * IC + ci, xo = (ky * WP + kx) * IC + ci;
-                        float xv[NPOS];
+                        float xv[NP];
 #pragma unroll
-                        for (int s2 = 0; s2 < NPOS; ++s2) xv[s2] = xs[off[s2] + xo];
+                        for (int q2 = 0; q2 < NP; ++q2) xv[q2] = xs[off[q2] + xo];
 #pragma unroll
                         for (int a = 0; a < SG; ++a) {
                             const float ev = e0[(a < nsg ? a : 0) * K + kk];
 #pragma unroll
-                            for (int s2 = 0; s2 < NPOS; ++s2) acc[a][s2] = fmaf(ev, xv[s2], acc[a][s2]);
+                            for (int q2 = 0; q2 < NP; ++q2) acc[a][q2] = fmaf(ev, xv[q2], acc[a][q2]);
                         }
                     }
 #pragma unroll
@@ -375,14 +380,20 @@ __global__ void __launch_bounds__(256) k_patch_dot_in(const PatchDotParams p)
                 if (a >= nsg) break;
                 const int sl = sg * SG + a;
                 const float *zr = zsm + sl_j[sl] * P;
-                float v4[NPOS];
+                float *orow = p.out + ((int64_t)sl_g[sl] * p.T + tl) * p.out_stride + sl_q[sl] * p.cells;
 #pragma unroll
-                for (int s2 = 0; s2 < NPOS; ++s2) {
-                    const int oy = POOL ? 2 * cy + (s2 >> 1) : cy, ox = POOL ? 2 * cx + (s2 & 1) : cx;
-                    v4[s2] = act_apply(p.act1, zr[oy * p.ow + ox] + acc[a][s2]);
+                for (int w = 0; w < CW; ++w) {
+                    const int c = ch * CW + w;
+                    if (c >= p.cells) break;
+                    const int cy = c / pw, cx = c - cy * pw;
+                    float v4[NPOS];
+#pragma unroll
+                    for (int s2 = 0; s2 < NPOS; ++s2) {
+                        const int oy = POOL ? 2 * cy + (s2 >> 1) : cy, ox = POOL ? 2 * cx + (s2 & 1) : cx;
+                        v4[s2] = act_apply(p.act1, zr[oy * p.ow + ox] + acc[a][w * NPOS + s2]);
+                    }
+                    orow[c] = POOL ? max4_first(v4[0], v4[1], v4[2], v4[3]) : v4[0];
                 }
-                const int64_t r = (int64_t)sl_g[sl] * p.T + tl;
-                p.out[r * p.out_stride + sl_q[sl] * p.cells + c] = POOL ? max4_first(v4[0], v4[1], v4[2], v4[3]) : v4[0];
             }
         }
     }
@@ -407,12 +418,15 @@ int launch_dot(const Stage &S, Src z, Src x, RowMap rm, const PatchArgs &pa, int
     p.rows_per_block = 8;
     p.oc = S.oc;
     if (z.per_input && x.per_input) {
-        // memoized: one block per input
-        const size_t smem2 = ((size_t)HP * WP * IC + 32 * (size_t)KH * KW * IC + (size_t)S.oc * S.oh * S.ow) * sizeof(float);
-        if (smem2 <= 96 * 1024) {
-            cudaFuncSetAttribute(k_patch_dot_in<KH, KW, IC, WP, HP, PAD, POOL, KMAX>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
-            k_patch_dot_in<KH, KW, IC, WP, HP, PAD, POOL, KMAX><<<(unsigned)rm.T, 256, smem2, s>>>(p);
+        // memoized: one block per input, a cell and four slots per thread (measured
+        // against two cells and / or eight slots per thread: more registers per thread
+        // cost more in occupancy than the fewer shared loads save)
+        constexpr int CW = 1, SG = 4, SMAX = 32, NT = 256;
+        const size_t smem2 = ((size_t)HP * WP * IC + (size_t)SMAX * KH * KW * IC + (size_t)S.oc * S.oh * S.ow) * sizeof(float);
+        if (smem2 <= 200 * 1024) {
+            auto kern = k_patch_dot_in<KH, KW, IC, WP, HP, PAD, POOL, CW, SG, SMAX, NT>;
+            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
+            kern<<<(unsigned)rm.T, NT, smem2, s>>>(p);
             return 1;
         }
     }
