@@ -561,6 +561,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     const uint32_t ov_region = a_region + kNA * kStageA;    // kNA overlay slots (with an overlay)
     // FCP > 0: the output layer's weights as [F][FCP] (zeros beyond its C classes)
     const uint32_t fw_region = (ov_region + (p.ov.patch ? kNA * kOvSlotBytes : 0) + 15u) & ~15u;
+    const float4 *fw4 = reinterpret_cast<const float4 *>(smraw + (fw_region - smem_u32(smraw)));
     const int64_t M = (int64_t)p.R * p.P;
     const int64_t n_tiles = MODE == 2 ? small_tiles(p.R) : (M + kTileM - 1) / kTileM;
     const int64_t my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
@@ -868,10 +869,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                             if (f < p.N) {
 #pragma unroll
                                 for (int c4 = 0; c4 < FCP; c4 += 4) {
-                                    float4 w4;
-                                    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
-                                                 : "=f"(w4.x), "=f"(w4.y), "=f"(w4.z), "=f"(w4.w)
-                                                 : "r"(fw_region + (uint32_t)(f * FCP + c4) * 4));
+                                    const float4 w4 = fw4[(f * FCP + c4) >> 2];
                                     facc[c4] = fmaf(vh[e], w4.x, facc[c4]);
                                     facc[c4 + 1] = fmaf(vh[e], w4.y, facc[c4 + 1]);
                                     facc[c4 + 2] = fmaf(vh[e], w4.z, facc[c4 + 2]);
