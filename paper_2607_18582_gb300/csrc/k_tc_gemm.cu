@@ -30,6 +30,8 @@
 // role, lets its own copies and MMAs drain (bounded), frees its tensor memory and
 // returns.
 #include <algorithm>
+#include <cuda.h>
+#include <cudaTypedefs.h>
 
 #include "common.cuh"
 #include "device_util.cuh"
@@ -270,6 +272,11 @@ struct TcParams {
     int *err;
     FinalFuse ff;                // the output layer computed in the epilogue (FCP > 0)
     SlotStore slot;              // slot.out: the tensor-core delta's scattered store
+    // dense layers: A tiles (128 rows x one K-step) by tensor-map copies from warp 10
+    // instead of the producers' 16-byte copies; the row coordinate of tile m0 is m0
+    // (rows) or m0 mod T (rows of T inputs, T a multiple of 128)
+    int a_tma;
+    CUtensorMap tmap_a;
 };
 
 // Per producer ring slot, the overlay values of a row's K-step: up to kOvMax
@@ -531,7 +538,7 @@ struct SmallSteps {
 // each row's outputs in the epilogue, followed by the kill epilogue, and the rows
 // themselves are not stored.
 template <int MODE, bool THREE, int FCP = 0>
-__global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
+__global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__ TcParams p)
 {
     static_assert(FCP == 0 || (MODE == 0 && FCP % 4 == 0), "the output layer is fused into dense layers only");
     constexpr bool DENSE = MODE == 0;
@@ -542,6 +549,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
     __shared__ __align__(8) uint64_t bar_accfull[2], bar_accempty[2], bar_drain;
     // small-image mode, per staging buffer: maps landed, overlay applied, producers done
     __shared__ __align__(8) uint64_t bar_landed[SmallConv::NBUF], bar_ready[SmallConv::NBUF], bar_released[SmallConv::NBUF];
+    // dense A tiles by tensor-map copies: slot landed, slot read by the producers
+    __shared__ __align__(8) uint64_t bar_alanded[kNA], bar_afree[kNA];
     __shared__ uint32_t tmem_sh;
     __shared__ int abort_sh;
     __shared__ float bias_sh[kSlice];
@@ -612,6 +621,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
             mbar_init(smem_u32(&bar_accempty[s]), 4);
         }
         mbar_init(smem_u32(&bar_drain), p.n_mma);
+        for (int s = 0; s < kNA; ++s) {
+            mbar_init(smem_u32(&bar_alanded[s]), 1);
+            mbar_init(smem_u32(&bar_afree[s]), 4);
+        }
         for (int s = 0; s < SmallConv::NBUF; ++s) {
             mbar_init(smem_u32(&bar_landed[s]), 1);
             mbar_init(smem_u32(&bar_ready[s]), 1);
@@ -699,6 +712,26 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&bar_released[b]));
                 if (++b == G::NBUF) { b = 0; ++uses; }
+            }
+        } else if (DENSE && p.a_tma) {
+            // A tiles land by tensor-map copies (warp 10); each thread reads its row
+            bool ok = true;
+            int slot_i = 0;
+            uint32_t slot_wraps = 0;
+            for (int64_t j = 0; ok && j < total; ++j) {
+                if (!warp_wait_phase<32>(smem_u32(&bar_alanded[slot_i]), slot_wraps & 1, abort_flag)) break;
+                const uint32_t slot = a_region + (uint32_t)slot_i * kStageA;
+                float v[kTileK];
+#pragma unroll
+                for (int c = 0; c < kTileK / 4; ++c) {
+                    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                                 : "=f"(v[4 * c]), "=f"(v[4 * c + 1]), "=f"(v[4 * c + 2]), "=f"(v[4 * c + 3])
+                                 : "r"(slot + sw128_off(r, c)));
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bar_afree[slot_i]));
+                if (++slot_i == kNA) { slot_i = 0; ++slot_wraps; }
+                ok = push(v);
             }
         } else {
             // issue cursor (tile i, K-tile kt, ring slot) runs kNA - 1 steps ahead
@@ -967,6 +1000,34 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcParams p)
                 for (int c = 0; c < FCP; ++c) lv[c] = c < p.ff.C ? act_apply(p.ff.act, facc[c] + __ldg(p.ff.b + c)) : 0.f;
                 epilogue_reg<FCP>(p.ff.fa, p.t0, p.T, ri.row, ri.ok, lv, p.ff.C);
             }
+        }
+    } else if (DENSE && warp == 10 && p.a_tma) {
+        // ------------------------------------------------------ A tiles by TMA --
+        if (lane == 0) {
+            const uint64_t tmap = reinterpret_cast<uint64_t>(&p.tmap_a);
+            int slot_i = 0, kt = 0;
+            uint32_t slot_wraps = 0;
+            int64_t i = 0, j = 0;
+            for (; j < total; ++j) {
+                if (slot_wraps >= 1 &&
+                    !wait_phase<32>(smem_u32(&bar_afree[slot_i]), (slot_wraps - 1) & 1, abort_flag))
+                    break;
+                // the producers' reads of the slot (generic proxy) before this copy's writes
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                const int64_t m0 = (blockIdx.x + i * gridDim.x) * kTileM;
+                const int row = (int)(p.x_per_input ? m0 % p.T : m0);
+                const uint32_t bar = smem_u32(&bar_alanded[slot_i]);
+                mbar_expect_tx(bar, (uint32_t)kStageA);
+                asm volatile(
+                    "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+                    ::"r"(a_region + (uint32_t)slot_i * kStageA), "l"(tmap), "r"(kt * kTileK), "r"(row), "r"(bar)
+                    : "memory");
+                if (++slot_i == kNA) { slot_i = 0; ++slot_wraps; }
+                if (++kt == nK) { kt = 0; ++i; }
+            }
+            // copies still in flight land before the shared memory is released
+            for (int64_t jj = j > kNA ? j - kNA : 0; jj < j; ++jj)
+                wait_phase_drain(smem_u32(&bar_alanded[jj % kNA]), (uint32_t)((jj / kNA) & 1));
         }
     } else if (MODE == 2 && warp == 10) {
         // ------------------------------------------------ map staging: finish --
@@ -1254,6 +1315,41 @@ static void tc_config(TcParams &p, int nt_max, bool three)
     p.n_mma = m;
 }
 
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no link to libcuda).
+static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    }
+    return fn;
+}
+
+// The A operand of a dense layer as a 2-D tensor [rows][K] with 128-byte swizzled
+// boxes of 128 rows x 32 values (the producers' shared-memory layout): false when
+// the rows of a tile are not consecutive in memory or the encoder is unavailable.
+static bool dense_a_tensor_map(const Stage &S, Src x, RowMap rm, CUtensorMap &map)
+{
+    if (x.per_input && rm.T % kTileM != 0) return false;
+    if ((x.stride * 4) % 16 != 0 || (reinterpret_cast<uintptr_t>(x.p) & 15) != 0) return false;
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+    if (!enc) return false;
+    const float *base = x.p + (x.per_input ? rm.t0 * x.stride : 0);
+    const cuuint64_t dims[2] = {(cuuint64_t)S.K, (cuuint64_t)(x.per_input ? rm.T : rm.R)};
+    const cuuint64_t strides[1] = {(cuuint64_t)x.stride * 4};
+    const cuuint32_t box[2] = {(cuuint32_t)kTileK, (cuuint32_t)kTileM};
+    const cuuint32_t estr[2] = {1, 1};
+    return enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int tc_final_fusable(const Stage &S, const Stage &SL)
 {
     return S.tc && S.kind == MURE_NODE_DENSE && tc_supported(S) && round_up16(S.oc) <= kSlice &&
@@ -1314,6 +1410,8 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     // the delta GEMM: one issuing warp, so that a column's sum never depends on how many
     // slots share its batch
     if (ss) p.n_mma = 1;
+    // dense rows without an overlay: A tiles by tensor-map copies from warp 10
+    p.a_tma = dense && !p.ov.patch && p.n_mma <= 2 && dense_a_tensor_map(S, x, rm, p.tmap_a) ? 1 : 0;
     if (S.tc_small) p.n_mma = std::min(p.n_mma, 2);   // warp 10 stages maps in that mode
     const int64_t M = (int64_t)rm.R * p.P;
     const int64_t tiles = S.tc_small ? small_tiles(rm.R) : (M + kTileM - 1) / kTileM;

@@ -183,6 +183,20 @@ def test_batch_invariance(M, ctx, prec):
     assert np.array_equal(sub["logits"].view(np.uint32), big["logits"][:, :70].view(np.uint32))
 
 
+def test_repeat_and_vanilla_bitwise_at_scale(M, ctx):
+    """A larger LeNet-5 run (many tiles per CTA, every copy ring wrapping many times):
+    two memoized evaluations and the vanilla one give the same bits.  Catches races
+    between the copy engines and the threads that read their buffers."""
+    w = wl.workload("lenet5", 4096, 400)
+    model = M.mure_model_load(ctx, w.model, precision="tf32x3")
+    cache = M.mure_build_prefix_cache(model, w.X)
+    a = M.mure_eval_mutants(cache, w.table)
+    b = M.mure_eval_mutants(cache, w.table)
+    assert np.array_equal(a["kill_bits"], b["kill_bits"])
+    van = M.mure_eval_vanilla(model, w.X, w.table)
+    assert np.array_equal(a["kill_bits"], van["kill_bits"])
+
+
 @pytest.mark.parametrize("prec", ["tf32x3", "tf32"])
 def test_batch_invariance_tensor_core_delta(M, ctx, prec):
     """GF / WS deltas of the generic convolutions run as one tensor-core GEMM per batch
