@@ -273,8 +273,7 @@ struct TcParams {
     FinalFuse ff;                // the output layer computed in the epilogue (FCP > 0)
     SlotStore slot;              // slot.out: the tensor-core delta's scattered store
     // dense layers: A tiles (128 rows x one K-step) by tensor-map copies from warp 10
-    // instead of the producers' 16-byte copies; the row coordinate of tile m0 is m0
-    // (rows) or m0 mod T (rows of T inputs, T a multiple of 128)
+    // instead of the producers' 16-byte copies; tile m0 starts at row coordinate m0
     int a_tma;
     CUtensorMap tmap_a;
 };
@@ -341,6 +340,7 @@ __device__ __forceinline__ RowInfo row_info(const TcParams &p, int64_t m)
 struct LoadRows {
     const float *xrow[8];   // null: row past the end
     int oy[8], ox[8];
+    int ci, kx, ky;         // convolution: (ky, kx, ci) of this lane's 4-value chunk at the next K-step
 };
 
 template <bool DENSE>
@@ -360,6 +360,16 @@ __device__ __forceinline__ void load_rows(const RowInfo &pf, LoadRows &lr)
     }
 }
 
+// The chunk cursor of a convolution's first K-step: k = 4 * (lane mod 8).
+__device__ __forceinline__ void chunk_cursor(const TcParams &p, LoadRows &lr)
+{
+    const int kk = 4 * ((threadIdx.x & 31) & 7);
+    const int t = kk / p.ic;
+    lr.ci = kk - t * p.ic;
+    lr.kx = t % p.kw;
+    lr.ky = t / p.kw;
+}
+
 // Queue the cp.async copies of K-step k0 .. k0+31 of the warp's 32 GEMM rows into
 // their 128-byte rows of `slot` (swizzled like the MMA operand layout, so that each
 // thread's read-back of its own row is free of bank conflicts).  Values past the
@@ -368,7 +378,7 @@ __device__ __forceinline__ void load_rows(const RowInfo &pf, LoadRows &lr)
 // their patch values into the slot's overlay entries (ov), written over its row once
 // the copies have landed.
 template <bool DENSE>
-__device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, const LoadRows &lr, int r, uint32_t slot,
+__device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, LoadRows &lr, int r, uint32_t slot,
                                               uint32_t ov, int k0)
 {
     const float *dummy = p.b;   // a valid address for zero-byte copies
@@ -408,7 +418,13 @@ __device__ __forceinline__ void produce_issue(const TcParams &p, RowInfo &pf, co
         // 16-byte chunks: 4 channels of one input pixel; this lane's chunk has the same
         // (ky, kx, ci) in all its rows
         const int kk = k0 + 4 * ch;
-        const int ci = kk % p.ic, t = kk / p.ic, kx = t % p.kw, ky = t / p.kw;
+        const int ci = lr.ci, kx = lr.kx, ky = lr.ky;
+        // the cursor of the next K-step, 32 values on (no divisions per K-step)
+        lr.ci += kTileK;
+        while (lr.ci >= p.ic) {
+            lr.ci -= p.ic;
+            if (++lr.kx == p.kw) { lr.kx = 0; ++lr.ky; }
+        }
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
             const int row = wbase + 4 * c + (lane >> 3);
@@ -743,6 +759,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 if (iss_kt == 0) {
                     pf = row_info<DENSE>(p, (blockIdx.x + iss_i * gridDim.x) * kTileM + r);
                     if (DENSE || (p.ic & 3) == 0) load_rows<DENSE>(pf, lr);
+                    if (!DENSE && (p.ic & 3) == 0) chunk_cursor(p, lr);
                 }
                 produce_issue<DENSE>(p, pf, lr, r, a_region + (uint32_t)iss_slot * kStageA,
                                      ov_region + (uint32_t)iss_slot * kOvSlotBytes, iss_kt * kTileK);
@@ -1015,7 +1032,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 // the producers' reads of the slot (generic proxy) before this copy's writes
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 const int64_t m0 = (blockIdx.x + i * gridDim.x) * kTileM;
-                const int row = (int)(p.x_per_input ? m0 % p.T : m0);
+                const int row = (int)m0;
                 const uint32_t bar = smem_u32(&bar_alanded[slot_i]);
                 mbar_expect_tx(bar, (uint32_t)kStageA);
                 asm volatile(
@@ -1332,16 +1349,18 @@ static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
 }
 
 // The A operand of a dense layer as a 2-D tensor [rows][K] with 128-byte swizzled
-// boxes of 128 rows x 32 values (the producers' shared-memory layout): false when
-// the rows of a tile are not consecutive in memory or the encoder is unavailable.
+// boxes of 128 rows x 32 values (the producers' shared-memory layout): false for
+// per-input rows, unaligned rows or without the encoder.
 static bool dense_a_tensor_map(const Stage &S, Src x, RowMap rm, CUtensorMap &map)
 {
-    if (x.per_input && rm.T % kTileM != 0) return false;
+    // rows of per-input tensors always carry a patch (the first suffix stage), so only
+    // row-per-row tensors take this path
+    if (x.per_input) return false;
     if ((x.stride * 4) % 16 != 0 || (reinterpret_cast<uintptr_t>(x.p) & 15) != 0) return false;
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (!enc) return false;
-    const float *base = x.p + (x.per_input ? rm.t0 * x.stride : 0);
-    const cuuint64_t dims[2] = {(cuuint64_t)S.K, (cuuint64_t)(x.per_input ? rm.T : rm.R)};
+    const float *base = x.p;
+    const cuuint64_t dims[2] = {(cuuint64_t)S.K, (cuuint64_t)rm.R};
     const cuuint64_t strides[1] = {(cuuint64_t)x.stride * 4};
     const cuuint32_t box[2] = {(cuuint32_t)kTileK, (cuuint32_t)kTileM};
     const cuuint32_t estr[2] = {1, 1};
