@@ -196,24 +196,39 @@ def max_over_ranks(x, world):
 
 # ---------------------------------------------------------------- oracle leg --
 
-def oracle_sample(w, n_mut, n_in, seed=0):
+def oracle_sample(w, n_mut, n_in, seed=0, with_index=False):
     from paper_2607_18582_gb300 import workloads as wl
     idx = wl.stratified(w.table, w.model, max(1, n_mut // (w.model.n_layers() * 4)))
     rng = np.random.default_rng(seed)
     if len(idx) < n_mut:
         rest = np.setdiff1d(np.arange(len(w.table)), idx)
         idx = np.sort(np.concatenate([idx, rng.choice(rest, min(len(rest), n_mut - len(idx)), replace=False)]))
-    return w.table.subset(idx[:n_mut]), w.X[:n_in]
+    idx = idx[:n_mut]
+    if with_index:
+        return w.table.subset(idx), w.X[:n_in], idx
+    return w.table.subset(idx), w.X[:n_in]
 
 
-def cpu_oracle_rate(w, n_mut, n_in, threads):
-    """Oracle (memoized, Algorithm 1 on the CPU) evals/s on a bounded sample."""
+def cpu_oracle_rate(w, n_mut, n_in, threads, gpu_kill=None):
+    """Oracle (memoized, Algorithm 1 on the CPU) evals/s on a bounded sample; with the
+    GPU's kill matrix of the whole workload, also the agreement of the GPU's kill
+    verdicts with the oracle's on that sample."""
     import oracle
-    table, X = oracle_sample(w, n_mut, n_in)
+    table, X, idx = oracle_sample(w, n_mut, n_in, with_index=True)
     t = time.perf_counter()
-    oracle.memo(w.model, X, table, n_threads=threads, want_logits=False)
+    res = oracle.memo(w.model, X, table, n_threads=threads, want_logits=False)
     dt = time.perf_counter() - t
-    return len(table) * len(X) / dt, dt, f"{len(table)} stratified mutants x first {len(X)} inputs, oracle memoized mode"
+    agree = None
+    if gpu_kill is not None:
+        n = len(X)
+        cols = np.arange(n)
+        ora = (np.asarray(res["kill_bits"], np.uint64)[:, cols // 64] >> (cols % 64).astype(np.uint64)) & np.uint64(1)
+        g = np.asarray(gpu_kill, np.uint64)[idx]
+        gpu = (g[:, cols // 64] >> (cols % 64).astype(np.uint64)) & np.uint64(1)
+        diff = int((ora != gpu).sum())
+        agree = {"verdicts": int(ora.size), "differ": diff, "agreement": 1.0 - diff / max(1, ora.size)}
+    return (len(table) * len(X) / dt, dt, f"{len(table)} stratified mutants x first {len(X)} inputs, oracle memoized mode",
+            agree)
 
 
 def run_reference(args, world, rank):
@@ -230,7 +245,7 @@ def run_reference(args, world, rank):
         cpu_oracle_rate(w, n_mut, n_in, threads)
     t = time.perf_counter()
     for _ in range(args.steps):
-        _, _, sample = cpu_oracle_rate(w, n_mut, n_in, threads)
+        _, _, sample, _ = cpu_oracle_rate(w, n_mut, n_in, threads)
     dt = time.perf_counter() - t
     value = args.steps * n_mut * n_in / dt
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
@@ -425,9 +440,12 @@ def main():
         import oracle
         oracle.build()
         threads = os.cpu_count() or 1
-        rate, dt, sample = cpu_oracle_rate(w, 400, 2000, threads)
+        rate, dt, sample, agree = cpu_oracle_rate(w, 400, 2000, threads, gpu_kill=kill_dev.cpu().numpy())
         out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
                                "seconds": dt}
+        # kill verdicts of the timed GPU run against the oracle's on the same sample
+        # (differences are expected only on near ties; the TF32 variant reports its rate)
+        out["oracle_agreement"] = agree
     out["hbm"] = hbm_rates(w, results, cls_ms, pk, pk_kind)
     out["peaks"] = {"source": pk_kind, "hbm_gbs": pk.get("hbm_gbs"), "bf16_tflops": pk.get("bf16_tflops")}
     if rank == 0:
