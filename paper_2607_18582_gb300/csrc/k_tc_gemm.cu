@@ -1111,7 +1111,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 if (use >= 1 && !wait_phase<32>(smem_u32(&bar_accempty[a]), (uint32_t)((use - 1) & 1), abort_flag)) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t d = tmem + (uint32_t)((a * nmma + w) * p.acc_cols);
-                int own = 0;                    // kt mod n_mma
+                // two warps keep dealing across tiles (an odd nK alternates which warp
+                // takes the extra K-step); the epilogue's p0 + p1 is commutative, so a
+                // row's sum does not depend on which partial holds which K-steps
+                int own = nmma == 2 ? (int)((i * nK) & 1) : 0;
+                bool first = true;              // the warp's first K-step of the tile overwrites
                 for (int kt = 0; kt < nK; ++kt) {
                     if (own == w) {
                         if (!wait_phase<32>(smem_u32(&bar_afull[t]), t_wraps & 1, abort_flag)) { ok = false; break; }
@@ -1119,8 +1123,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                             !wait_phase<32>(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
                         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                         const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
-                        // the warp's first K-step of the tile (kt = w) overwrites its partial sum
-                        mma_block<THREE, 0, Q>(d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, kt >= nmma ? 1u : 0u);
+                        mma_block<THREE, 0, Q>(d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, first ? 0u : 1u);
+                        first = false;
                         mma_commit(smem_u32(&bar_aempty[t]));
                         if (!p.b_resident) mma_commit(smem_u32(&bar_bempty[sb]));
                     }
