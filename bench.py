@@ -154,7 +154,7 @@ def hbm_rates(w, results, cls_ms, pk, pk_kind):
         node = w.model.nodes[w.model.layers()[L - 1]]
         byts = rows * (node.cin * 4 + 1 / 8)
         gbs = byts / (ms / 1e3) / 1e9
-        out["output_layer"] = {"kernels": "k_final_dense (output layer + kill, rows not fused into a dense epilogue)",
+        out["output_layer"] = {"kernels": "k_final_dense_rows / k_final_dense (output layer + kill, rows not fused into a dense epilogue)",
                                "bytes": byts, "ms": ms, "achieved": gbs, "unit": "GB/s", "frac": gbs / peak,
                                "bytes_counted": "input rows read once, kill bits written"}
     out["peak"] = peak
