@@ -132,8 +132,8 @@ def profiled_traffic(kernel_key, rows_per_launch):
 
 def hbm_rates(w, results, cls_ms, pk, pk_kind):
     """Achieved HBM bandwidth of the memory-bound kernel classes against the measured
-    copy bandwidth: the delta kernels (algorithmic bytes = the patch values they write;
-    the cached z / x rows that each input stages once for all mutants are not counted)
+    copy bandwidth: the delta kernels (algorithmic bytes = the patch values they write
+    and the cached z / x rows that each input of a batch stages once for all mutants)
     and the stand-alone output-layer kernel (its input rows read once, 1 bit written
     per row).  CUDA-event times of the timed steps."""
     out = {}
@@ -143,7 +143,7 @@ def hbm_rates(w, results, cls_ms, pk, pk_kind):
     if ms > 0 and byts > 0:
         gbs = byts / (ms / 1e3) / 1e9
         out["delta"] = {"kernels": "k_patch_* (delta)", "bytes": byts, "ms": ms, "achieved": gbs, "unit": "GB/s",
-                        "frac": gbs / peak, "bytes_counted": "patch values written"}
+                        "frac": gbs / peak, "bytes_counted": "patch values written + cached z / x rows read once per input and batch"}
     L = w.model.n_layers()
     last = f"layer{L - 1}"
     ms = cls_ms.get(last, 0.0)

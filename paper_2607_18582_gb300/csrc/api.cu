@@ -390,6 +390,7 @@ struct DevTable {
     std::vector<int64_t> dot_prefix;   // [n+1] prefix sums of GF/WS neuron slots (group order)
     int32_t *dslot = nullptr;          // [dot_prefix[n]] GF/WS slots in group order: (group, slot q)
     std::vector<int64_t> val_prefix;   // [n+1] prefix sums of NEB/NAI/NS neuron slots (group order)
+    std::vector<int64_t> copy_prefix;  // [n+1] the same for NEB/NS alone
     int4 *vslot = nullptr;             // [val_prefix[n]] those slots: (group, q, source channel, op)
     int expand_launches = 0;
 };
@@ -438,10 +439,12 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
             for (int q = 0; q < nn[k]; ++q) { dslot.push_back((int32_t)k); dslot.push_back(q); }
     // the operators without a fan-in sum: NS reads its partner neuron's channel
     dt.val_prefix.assign(n + 1, 0);
+    dt.copy_prefix.assign(n + 1, 0);
     std::vector<int4> vslot;
     for (int64_t k = 0; k < n; ++k) {
         const bool val = op[k] == MURE_OP_NEB || op[k] == MURE_OP_NAI || op[k] == MURE_OP_NS;
         dt.val_prefix[k + 1] = dt.val_prefix[k] + (val ? nn[k] : 0);
+        dt.copy_prefix[k + 1] = dt.copy_prefix[k] + ((op[k] == MURE_OP_NEB || op[k] == MURE_OP_NS) ? nn[k] : 0);
         if (val)
             for (int q = 0; q < nn[k]; ++q)
                 vslot.push_back(make_int4((int)k, q, pool[noff[k] + (op[k] == MURE_OP_NS ? (q ^ 1) : q)], op[k]));
@@ -660,16 +663,42 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     const int kmax = dt.kmax_layer[l];
     const int64_t pstride = (int64_t)std::max(kmax, 1) * cells_l;
     const Src zsrc = vanilla ? Src{ws.zb, ws.z_stride, 0} : Src{ca->z[l], m->zd[l].stride, 1};
-    acct.bytes_gather += (int64_t)rm.R * kmax * cells_l * 4;
     // GF / WS: on the tensor cores (one GEMM over the batch's inputs with every slot's
     // mutated filter as an output channel), else the CUDA-core dot-product kernels
     const bool tc_delta = tc_delta_supported(Sl, m->precision) && ws.dw.n_max > 0;
     const bool dot_kernel = !tc_delta && patch_dot_supported(Sl, kmax);
     const bool has_dot = dt.dot_prefix[g0 + G] > dt.dot_prefix[g0];
+    Overlay ov;
+    ov.patch = ws.patch;
+    ov.row_stride = pstride;
+    ov.kmax = kmax;
+    ov.cells = cells_l;
+    ov.ch = Sl.oc;
+    ov.n_neurons = pa.n_neurons;
+    ov.neuron_off = pa.neuron_off;
+    ov.ids = pa.ids;
+    bool skip_reader = false;
+    for (int v = l + 2; v < L; ++v) skip_reader |= m->st[v].has_add && m->st[v].skip_src == l + 1;
+    // the window GEMM as first suffix stage applies NEB (zeros) and NS (a swap of the
+    // two channels, which is the operator itself: the swapped neurons' channels are
+    // computed independently) on its staged maps, so the delta writes no values for
+    // them; x_{l+1} must come from the small-convolution kernel, whose pooled values
+    // the other operators' patches reproduce bit for bit
+    const bool win_ops = l + 2 < L && m->st[l + 1].tc && m->st[l + 1].tc_small && !skip_reader && !Sl.tc &&
+                         Sl.variant > 0 && tc_overlay_inline(m->st[l + 1], ov, G) &&
+                         !(l + 1 == L - 2 && tc_final_fusable(m->st[L - 2], m->st[L - 1]));
+    if (win_ops) ov.op = pa.op;
+    // the delta's algorithmic bytes: the patch values it writes (every mutated channel
+    // of every row, but those the window GEMM applies itself) and the rows it reads,
+    // z_l (and x_l for GF / WS) once per input of the batch (memoized) or per row
+    const int64_t slots = (dt.dot_prefix[g0 + G] - dt.dot_prefix[g0]) + (dt.val_prefix[g0 + G] - dt.val_prefix[g0]) -
+                          (win_ops ? dt.copy_prefix[g0 + G] - dt.copy_prefix[g0] : 0);
+    acct.bytes_gather += slots * rm.T * cells_l * 4;
+    acct.bytes_gather += (vanilla ? rm.R : (int64_t)rm.T) * (m->zd[l].size + (has_dot ? m->xd[l].size : 0)) * 4;
     int delta_err = 0;
     timed(C_DELTA, delta_flops, [&] {
         int n = launch_patch_vals(Sl, zsrc, xsrc(l), skip_of(Sl), rm, pa, kmax, ws.patch, pstride, s,
-                                  dot_kernel || tc_delta);
+                                  dot_kernel || tc_delta, win_ops);
         if (tc_delta && has_dot) {
             // the inputs' x_l and z_l: cached rows (memoized) or the batch's first
             // mutant's recomputed rows (vanilla; the prefix up to layer l is unmutated)
@@ -681,15 +710,6 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         return n;
     });
     if (delta_err) return -1;
-    Overlay ov;
-    ov.patch = ws.patch;
-    ov.row_stride = pstride;
-    ov.kmax = kmax;
-    ov.cells = cells_l;
-    ov.ch = Sl.oc;
-    ov.n_neurons = pa.n_neurons;
-    ov.neuron_off = pa.neuron_off;
-    ov.ids = pa.ids;
     // the unmutated rows of x_{l+1}: cached (memoized) or just computed (vanilla)
     const Src base = vanilla ? Src{ws.xb[l + 1], m->xd[l + 1].stride, 0} : Src{ca->x[l + 1], m->xd[l + 1].stride, 1};
     if (l == L - 1) {
@@ -706,8 +726,6 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     // the rows are materialised for kernels that read plain rows and whenever a later
     // residual add reads x_{l+1} as its skip input
     const Stage &Sn = m->st[l + 1];
-    bool skip_reader = false;
-    for (int v = l + 2; v < L; ++v) skip_reader |= m->st[v].has_add && m->st[v].skip_src == l + 1;
     // a tensor-core dense stage L-2 takes the output layer and the kill epilogue into
     // its own epilogue (the rows of x_{L-1} are then never stored)
     const Stage &SLast = m->st[L - 1];

@@ -120,6 +120,10 @@ struct Overlay {
     const int32_t *n_neurons = nullptr;
     const int64_t *neuron_off = nullptr;
     const int32_t *ids = nullptr;
+    // non-null (window GEMM only): per-group operator codes; NEB rows get their mutated
+    // channels zeroed and NS rows their channel pairs swapped in the staged maps, and
+    // the patch values of those rows are not read (the delta need not write them)
+    const int32_t *op = nullptr;
 };
 
 // Stage v over R rows: z (optional) and y = post(act1(conv(x) + b)).
@@ -218,7 +222,7 @@ struct PatchArgs {
 // (channel-major; x_l for GF / WS), the layer's post-ops and skip, into
 // out[r][q][c] (slot q < kmax, output cell c of layer l).
 int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *out,
-                      int64_t out_stride, cudaStream_t s, bool skip_dot_ops = false);
+                      int64_t out_stride, cudaStream_t s, bool skip_dot_ops = false, bool skip_copy_ops = false);
 
 // GF / WS delta values on the tensor cores (convolution layers, tensor-core precision
 // modes): one implicit GEMM over the batch's inputs whose output channels are the

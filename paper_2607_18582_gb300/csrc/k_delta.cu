@@ -130,6 +130,7 @@ struct PatchValsParams {
     int warp_dot;        // 1: fan-in sums split across a warp (layers with < 32 positions)
     int skip_dot_ops;    // 1: GF / WS values come from k_patch_dot
     int only_dot_ops;    // 1: the other operators come from k_patch_vals_staged
+    int skip_copy_ops;   // 1: NEB / NS slots are applied by the consumer (window GEMM)
 };
 
 struct SlotCtx {
@@ -307,6 +308,7 @@ __global__ void __launch_bounds__(256) k_patch_vals_staged(const PatchValsParams
     for (int64_t sl = warp; sl < p.pa.n_vslot; sl += blockDim.x >> 5) {
         const int4 e = p.pa.vslot[sl];
         const int g = e.x - p.pa.dslot_g0, q = e.y, sj = e.z, op = e.w;
+        if (p.skip_copy_ops && (op == MURE_OP_NEB || op == MURE_OP_NS)) continue;
         const float *zc = zs + sj * P;
         float *o = p.out + ((int64_t)g * p.T + tl) * p.out_stride + q * p.cells;
         auto post = [&](float zz) {
@@ -404,7 +406,7 @@ __global__ void __launch_bounds__(256) k_patch_vals_dense_in(const PatchValsPara
 }
 
 int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const PatchArgs &pa, int kmax, float *out,
-                      int64_t out_stride, cudaStream_t s, bool skip_dot_ops)
+                      int64_t out_stride, cudaStream_t s, bool skip_dot_ops, bool skip_copy_ops)
 {
     if (rm.R <= 0 || kmax <= 0) return 0;
     PatchValsParams p{};
@@ -424,6 +426,7 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     p.out = out; p.out_stride = out_stride;
     p.warp_dot = (S.oh * S.ow) < 32;
     p.skip_dot_ops = skip_dot_ops;
+    p.skip_copy_ops = skip_copy_ops;
     const int64_t n_items = (int64_t)p.G * kmax;
     // each warp walks several inputs (blockIdx.y, +gridDim.y, ...): enough blocks to
     // fill the GPU, few enough that block scheduling stays negligible

@@ -618,7 +618,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         for (int g = threadIdx.x; g < G; g += kThreads) {
             const int n = p.ov.n_neurons[g];
             const uint32_t tab = ovtab_region + (uint32_t)g * (1 + SmallConv::MAXQ) * 4;
-            asm volatile("st.shared.u32 [%0], %1;" ::"r"(tab), "r"(n));
+            // count, and in bits 16+ how the finisher writes the channels: 0 from the
+            // patch, 1 zeros (NEB), 2 swapped in pairs (NS)
+            const int op = p.ov.op ? p.ov.op[g] : -1;
+            const uint32_t how = op == MURE_OP_NEB ? 1u : op == MURE_OP_NS ? 2u : 0u;
+            asm volatile("st.shared.u32 [%0], %1;" ::"r"(tab), "r"((uint32_t)n | (how << 16)));
             for (int q = 0; q < SmallConv::MAXQ; ++q)
                 asm volatile("st.shared.u32 [%0], %1;" ::"r"(tab + 4 + 4 * q), "r"(q < n ? p.ov.ids[p.ov.neuron_off[g] + q] : 0));
         }
@@ -670,7 +674,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         const int nimg = tile_rows(i, row0);
         const uint32_t buf = img_region + (uint32_t)b * G2::BUF_B;
         const uint32_t bar = smem_u32(&bar_landed[b]);
-        const uint32_t pbytes = p.ov.patch ? (uint32_t)(nimg * p.ov.row_stride * 4) : 0u;
+        // the rows' patch values, unless every row of the tile is NEB / NS (or has no
+        // mutated channel): the finisher then reads none
+        bool need = false;
+        if (p.ov.patch)
+            for (int im = 0; im < nimg; ++im) {
+                uint32_t k;
+                asm volatile("ld.shared.u32 %0, [%1];" : "=r"(k) : "r"(tab_of(row0 + im)));
+                need |= (k >> 16) == 0 && (k & 0xffffu) != 0;
+            }
+        const uint32_t pbytes = need ? (uint32_t)(nimg * p.ov.row_stride * 4) : 0u;
         // the buffer was last read and written by generic loads and stores
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         mbar_expect_tx(bar, nimg * G2::IMG_B + pbytes);
@@ -1065,6 +1078,41 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     const uint32_t tab = tab_of(row0 + im);
                     uint32_t k;
                     asm volatile("ld.shared.u32 %0, [%1];" : "=r"(k) : "r"(tab));
+                    const uint32_t how = k >> 16;
+                    k &= 0xffffu;
+                    const uint32_t map = buf + im * G::IMG_B;
+                    if (how == 1) {
+                        // NEB: the channels' post-activation values are +0
+                        for (uint32_t q = 0; q < k; ++q) {
+                            uint32_t jn;
+                            asm volatile("ld.shared.u32 %0, [%1];" : "=r"(jn) : "r"(tab + 4 + q * 4));
+#pragma unroll
+                            for (int u = 0; u < U; ++u)
+                                if (lane + 32 * u < G::CELLS)
+                                    asm volatile("st.shared.u32 [%0], %1;" ::"r"(map + ((lane + 32 * u) * G::IC + jn) * 4), "r"(0u)
+                                                 : "memory");
+                        }
+                        continue;
+                    }
+                    if (how == 2) {
+                        // NS: channels q and q + 1 trade places (each lane its own cells)
+                        for (uint32_t q = 0; q + 1 < k; q += 2) {
+                            uint32_t ja, jb;
+                            asm volatile("ld.shared.u32 %0, [%1];" : "=r"(ja) : "r"(tab + 4 + q * 4));
+                            asm volatile("ld.shared.u32 %0, [%1];" : "=r"(jb) : "r"(tab + 8 + q * 4));
+#pragma unroll
+                            for (int u = 0; u < U; ++u)
+                                if (lane + 32 * u < G::CELLS) {
+                                    const uint32_t cell = map + (lane + 32 * u) * G::IC * 4;
+                                    uint32_t va, vb;
+                                    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(va) : "r"(cell + ja * 4));
+                                    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(vb) : "r"(cell + jb * 4));
+                                    asm volatile("st.shared.u32 [%0], %1;" ::"r"(cell + ja * 4), "r"(vb) : "memory");
+                                    asm volatile("st.shared.u32 [%0], %1;" ::"r"(cell + jb * 4), "r"(va) : "memory");
+                                }
+                        }
+                        continue;
+                    }
                     for (uint32_t q = 0; q < k; ++q) {
                         uint32_t jn, val[U];
                         asm volatile("ld.shared.u32 %0, [%1];" : "=r"(jn) : "r"(tab + 4 + q * 4));
