@@ -52,7 +52,7 @@ class _Model(C.Structure):
 
 
 class _Mutant(C.Structure):
-    _fields_ = [("layer", C.c_int32), ("op", C.c_int32), ("n_neurons", C.c_int32), ("reserved", C.c_int32),
+    _fields_ = [("layer", C.c_int32), ("op", C.c_int32), ("n_neurons", C.c_int32), ("tagged", C.c_int32),
                 ("neuron_off", C.c_int64), ("param", C.c_float), ("reserved2", C.c_float), ("seed", C.c_uint64)]
 
 
@@ -82,6 +82,8 @@ def lib():
             L.or_layer_std.restype = C.c_double
             L.or_layer_std.argtypes = [C.POINTER(_Model), C.c_int32]
             L.or_mutant_layer.argtypes = [C.POINTER(_Model), C.POINTER(_Mutant), _I32P, C.c_int64, _FP, _FP, _U8P]
+            L.or_mutant_layer_at.argtypes = [C.POINTER(_Model), C.POINTER(_Mutant), _I32P, C.c_int64, C.c_int32,
+                                             _FP, _FP, _U8P]
             L.or_forward.argtypes = [C.POINTER(_Model), _FP, C.c_int64, _FP, _I32P]
             L.or_forward_nodes.argtypes = [C.POINTER(_Model), _FP, _FP]
             L.or_scores.argtypes = [_U64P, C.c_int64, C.c_int64, _I32P, C.c_int32, _DP, _DP, C.POINTER(C.c_int64)]
@@ -133,8 +135,10 @@ def _check(rc):
 def _mutants(table):
     n = len(table)
     arr = (_Mutant * max(n, 1))()
+    tagged = getattr(table, "tagged", None)
     for i in range(n):
-        arr[i] = _Mutant(int(table.layer[i]), int(table.op[i]), int(table.n_neurons[i]), 0,
+        arr[i] = _Mutant(int(table.layer[i]), int(table.op[i]), int(table.n_neurons[i]),
+                         int(tagged[i]) if tagged is not None else 0,
                          int(table.neuron_off[i]), float(table.param[i]), 0.0, int(table.seed[i]))
     pool = np.ascontiguousarray(table.pool, np.int32)
     if pool.size == 0:
@@ -197,17 +201,19 @@ def layer_std(model, layer):
     return float(lib().or_layer_std(C.byref(OModel(model).c), layer))
 
 
-def mutant_layer(model, table, i):
-    """Materialised parameters of mutant i's mutated layer: (W', b', blocked)."""
+def mutant_layer(model, table, i, layer=None):
+    """Materialised parameters of weighted layer `layer` of mutant i (default: its
+    first mutated layer): (W', b', blocked)."""
     om = OModel(model)
-    v = model.layers()[int(table.layer[i])]
+    layer = int(table.layer[i]) if layer is None else int(layer)
+    v = model.layers()[layer]
     nd = model.nodes[v]
     W = np.zeros_like(nd.W)
     b = np.zeros_like(nd.b)
     blk = np.zeros(nd.cout, np.uint8)
     arr, pool, plen = _mutants(table)
-    _check(lib().or_mutant_layer(C.byref(om.c), C.byref(arr[i]), _ptr(pool, _I32P), plen,
-                                 _ptr(W, _FP), _ptr(b, _FP), _ptr(blk, _U8P)))
+    _check(lib().or_mutant_layer_at(C.byref(om.c), C.byref(arr[i]), _ptr(pool, _I32P), plen, layer,
+                                    _ptr(W, _FP), _ptr(b, _FP), _ptr(blk, _U8P)))
     return W, b, blk.astype(bool)
 
 

@@ -32,6 +32,12 @@
  *       NS  : swap (w[j0], b[j0]) with (w[j1], b[j1]) for each listed pair
  *       NEB : the output of neuron j is forced to 0 (after the layer's activation)
  *       IDENTITY : no change
+ *   - mutants over several layers (the paper's set mu(M') of mutated layers, Sec. 3.2;
+ *     DeepMutation's model-wide selection): a "tagged" descriptor lists
+ *     (layer << 20 | neuron) entries; the operator is applied to each listed neuron in
+ *     its own layer (GF's sigma from that layer's weights, slot q of the list keeping
+ *     its random stream), NS pairs lie in one layer, and the descriptor's layer is the
+ *     smallest listed one (mmi).
  *   - random numbers: SplitMix64 (Steele, Lea, Flood, OOPSLA 2014) used as a
  *     counter-based generator; Gaussians by the Box-Muller transform in fp64.
  *   - argmax: lowest index wins ties; a NaN counts as the maximum.
@@ -71,7 +77,7 @@ typedef struct {
 
 /* One mutant: first (and only) mutated weighted layer, operator, neuron ids. */
 typedef struct {
-    int32_t layer, op, n_neurons, reserved;
+    int32_t layer, op, n_neurons, tagged;   /* tagged: pool entries are (layer << 20 | neuron) */
     int64_t neuron_off; /* index into the neuron pool */
     float param;        /* GF: sigma multiplier */
     float reserved2;
@@ -336,43 +342,70 @@ double or_layer_std(const or_model *m, int32_t layer)
     return sqrt(ss / (double)n);
 }
 
+/* Layer and neuron of pool entry e of a mutant. */
+static int32_t entry_layer(const or_mutant *mu, int32_t e) { return mu->tagged ? (e >> 20) : mu->layer; }
+static int32_t entry_neuron(const or_mutant *mu, int32_t e) { return mu->tagged ? (e & 0xFFFFF) : e; }
+
 static int check_mutant(const or_model *m, const or_mutant *mu, const int32_t *pool, int64_t pool_len)
 {
     int L = or_n_layers(m);
     if (mu->layer < 0 || mu->layer >= L) return OR_EINVAL;
     if (mu->op < OR_OP_GF || mu->op > OR_OP_IDENTITY) return OR_EINVAL;
+    if (mu->tagged != 0 && mu->tagged != 1) return OR_EINVAL;
     if (mu->n_neurons < 0 || mu->neuron_off < 0 || mu->neuron_off + mu->n_neurons > pool_len) return OR_EINVAL;
     if (mu->op == OR_OP_NS && (mu->n_neurons & 1)) return OR_EINVAL;
-    const or_node *nd = &m->nodes[layer_node(m, mu->layer)];
+    int32_t lmin = L;
     for (int q = 0; q < mu->n_neurons; ++q) {
-        int32_t j = pool[mu->neuron_off + q];
-        if (j < 0 || j >= nd->cout) return OR_EINVAL;
+        int32_t e = pool[mu->neuron_off + q];
+        if (e < 0) return OR_EINVAL;
+        int32_t l = entry_layer(mu, e), j = entry_neuron(mu, e);
+        if (l < 0 || l >= L) return OR_EINVAL;
+        if (j >= m->nodes[layer_node(m, l)].cout) return OR_EINVAL;
+        if (l < lmin) lmin = l;
         for (int r = 0; r < q; ++r)
-            if (pool[mu->neuron_off + r] == j) return OR_EINVAL;
+            if (pool[mu->neuron_off + r] == e) return OR_EINVAL;
+        if (mu->op == OR_OP_NS && (q & 1) && entry_layer(mu, pool[mu->neuron_off + q - 1]) != l) return OR_EINVAL;
     }
+    if (mu->tagged && mu->n_neurons > 0 && lmin != mu->layer) return OR_EINVAL;
     return OR_OK;
 }
 
-/* Materialise the mutated layer of M': W_out/b_out receive a full copy of the
- * layer's parameters with the operator applied; blocked_out[c] = 1 for NEB neurons. */
-int or_mutant_layer(const or_model *m, const or_mutant *mu, const int32_t *pool, int64_t pool_len,
-                    float *W_out, float *b_out, uint8_t *blocked_out)
+/* Whether mutant mu changes weighted layer `layer`. */
+static int touches_layer(const or_mutant *mu, const int32_t *pool, int32_t layer)
+{
+    if (mu->op == OR_OP_IDENTITY) return 0;
+    if (!mu->tagged) return layer == mu->layer;
+    for (int q = 0; q < mu->n_neurons; ++q)
+        if (entry_layer(mu, pool[mu->neuron_off + q]) == layer) return 1;
+    return 0;
+}
+
+/* Materialise weighted layer `layer` of M': W_out/b_out receive a full copy of the
+ * layer's parameters with the operator applied to the mutant's neurons in that
+ * layer (slot q of the neuron list keeps random stream q); blocked_out[c] = 1 for
+ * NEB neurons. */
+int or_mutant_layer_at(const or_model *m, const or_mutant *mu, const int32_t *pool, int64_t pool_len,
+                       int32_t layer, float *W_out, float *b_out, uint8_t *blocked_out)
 {
     if (!m || !mu) return OR_EINVAL;
     int rc = check_mutant(m, mu, pool, pool_len);
     if (rc) return rc;
-    const or_node *nd = &m->nodes[layer_node(m, mu->layer)];
+    if (layer < 0 || layer >= or_n_layers(m)) return OR_EINVAL;
+    const or_node *nd = &m->nodes[layer_node(m, layer)];
     int64_t F = fan_in(nd);
     memcpy(W_out, nd->W, sizeof(float) * (size_t)(F * nd->cout));
     memcpy(b_out, nd->b, sizeof(float) * (size_t)nd->cout);
     memset(blocked_out, 0, (size_t)nd->cout);
-    const int32_t *ids = pool + mu->neuron_off;
+    const int32_t *ent = pool + mu->neuron_off;
+    /* slot q is in this layer: its neuron id, else -1 */
+#define SLOT_J(q) (entry_layer(mu, ent[q]) == layer ? entry_neuron(mu, ent[q]) : -1)
     switch (mu->op) {
     case OR_OP_GF: {
-        double sigma = (double)mu->param * or_layer_std(m, mu->layer);
+        double sigma = (double)mu->param * or_layer_std(m, layer);
         for (int q = 0; q < mu->n_neurons; ++q) {
+            if (SLOT_J(q) < 0) continue;
             uint64_t s = slot_seed(mu->seed, q);
-            float *w = W_out + (size_t)ids[q] * F;
+            float *w = W_out + (size_t)SLOT_J(q) * F;
             for (int64_t f = 0; f < F; ++f) {
                 float e = (float)(sigma * or_gauss(s, f));
                 w[f] = w[f] + e;
@@ -384,9 +417,10 @@ int or_mutant_layer(const or_model *m, const or_mutant *mu, const int32_t *pool,
         int32_t *perm = (int32_t *)malloc(sizeof(int32_t) * (size_t)F);
         if (!perm) return OR_ENOMEM;
         for (int q = 0; q < mu->n_neurons; ++q) {
+            if (SLOT_J(q) < 0) continue;
             or_fisher_yates(slot_seed(mu->seed, q), (int32_t)F, perm);
-            const float *src = nd->W + (size_t)ids[q] * F;
-            float *w = W_out + (size_t)ids[q] * F;
+            const float *src = nd->W + (size_t)SLOT_J(q) * F;
+            float *w = W_out + (size_t)SLOT_J(q) * F;
             for (int64_t f = 0; f < F; ++f) w[f] = src[perm[f]];
         }
         free(perm);
@@ -394,14 +428,16 @@ int or_mutant_layer(const or_model *m, const or_mutant *mu, const int32_t *pool,
     }
     case OR_OP_NAI:
         for (int q = 0; q < mu->n_neurons; ++q) {
-            float *w = W_out + (size_t)ids[q] * F;
+            if (SLOT_J(q) < 0) continue;
+            float *w = W_out + (size_t)SLOT_J(q) * F;
             for (int64_t f = 0; f < F; ++f) w[f] = -w[f];
-            b_out[ids[q]] = -b_out[ids[q]];
+            b_out[SLOT_J(q)] = -b_out[SLOT_J(q)];
         }
         break;
     case OR_OP_NS:
         for (int q = 0; q + 1 < mu->n_neurons; q += 2) {
-            int j0 = ids[q], j1 = ids[q + 1];
+            if (SLOT_J(q) < 0) continue;   /* a pair lies in one layer */
+            int j0 = SLOT_J(q), j1 = SLOT_J(q + 1);
             memcpy(W_out + (size_t)j0 * F, nd->W + (size_t)j1 * F, sizeof(float) * (size_t)F);
             memcpy(W_out + (size_t)j1 * F, nd->W + (size_t)j0 * F, sizeof(float) * (size_t)F);
             b_out[j0] = nd->b[j1];
@@ -409,12 +445,22 @@ int or_mutant_layer(const or_model *m, const or_mutant *mu, const int32_t *pool,
         }
         break;
     case OR_OP_NEB:
-        for (int q = 0; q < mu->n_neurons; ++q) blocked_out[ids[q]] = 1;
+        for (int q = 0; q < mu->n_neurons; ++q)
+            if (SLOT_J(q) >= 0) blocked_out[SLOT_J(q)] = 1;
         break;
     case OR_OP_IDENTITY:
         break;
     }
+#undef SLOT_J
     return OR_OK;
+}
+
+/* The mutant's first mutated layer (mmi), materialised. */
+int or_mutant_layer(const or_model *m, const or_mutant *mu, const int32_t *pool, int64_t pool_len,
+                    float *W_out, float *b_out, uint8_t *blocked_out)
+{
+    if (!mu) return OR_EINVAL;
+    return or_mutant_layer_at(m, mu, pool, pool_len, mu->layer, W_out, b_out, blocked_out);
 }
 
 /* ------------------------------------------------------------- forward -- */
@@ -469,6 +515,71 @@ static const float *forward_one(fwd_ws *w, const float *x, int mv, const float *
         const float *i0 = node_in(w, nd->in0, x);
         const float *i1 = nd->kind == OR_ADD ? node_in(w, nd->in1, x) : NULL;
         if (v == mv) node_fwd(m, w->shp, v, i0, i1, W, b, blocked, w->buf[v]);
+        else node_fwd(m, w->shp, v, i0, i1, nd->W, nd->b, NULL, w->buf[v]);
+    }
+    return w->buf[m->n_nodes - 1];
+}
+
+/* The layers one mutant changes, materialised (buffers per weighted node, allocated
+ * on first use and kept for the worker's later mutants). */
+typedef struct {
+    int V;
+    float **W, **b;
+    uint8_t **blk;
+    uint8_t *on;    /* [V]: node v runs with the mutated parameters */
+} mut_params;
+
+static void mp_free(mut_params *p)
+{
+    if (p->W) for (int v = 0; v < p->V; ++v) { free(p->W[v]); free(p->b[v]); free(p->blk[v]); }
+    free(p->W); free(p->b); free(p->blk); free(p->on);
+    memset(p, 0, sizeof(*p));
+}
+
+static int mp_init(mut_params *p, const or_model *m)
+{
+    memset(p, 0, sizeof(*p));
+    p->V = m->n_nodes;
+    p->W = (float **)calloc((size_t)p->V, sizeof(float *));
+    p->b = (float **)calloc((size_t)p->V, sizeof(float *));
+    p->blk = (uint8_t **)calloc((size_t)p->V, sizeof(uint8_t *));
+    p->on = (uint8_t *)calloc((size_t)p->V, 1);
+    if (!p->W || !p->b || !p->blk || !p->on) { mp_free(p); return OR_ENOMEM; }
+    return OR_OK;
+}
+
+static int mp_load(mut_params *p, const or_model *m, const or_mutant *mu, const int32_t *pool, int64_t pool_len)
+{
+    memset(p->on, 0, (size_t)p->V);
+    int L = or_n_layers(m);
+    for (int l = 0; l < L; ++l) {
+        /* the first mutated layer is always materialised (an identity copy where the
+         * operator changes nothing there) */
+        if (l != mu->layer && !touches_layer(mu, pool, l)) continue;
+        int v = layer_node(m, l);
+        const or_node *nd = &m->nodes[v];
+        if (!p->W[v]) {
+            p->W[v] = (float *)malloc(sizeof(float) * (size_t)(fan_in(nd) * nd->cout));
+            p->b[v] = (float *)malloc(sizeof(float) * (size_t)nd->cout);
+            p->blk[v] = (uint8_t *)malloc((size_t)nd->cout);
+            if (!p->W[v] || !p->b[v] || !p->blk[v]) return OR_ENOMEM;
+        }
+        int rc = or_mutant_layer_at(m, mu, pool, pool_len, l, p->W[v], p->b[v], p->blk[v]);
+        if (rc) return rc;
+        p->on[v] = 1;
+    }
+    return OR_OK;
+}
+
+/* Forward of the whole network on one input with the mutant's layers. */
+static const float *forward_mut(fwd_ws *w, const float *x, const mut_params *p)
+{
+    const or_model *m = w->m;
+    for (int v = 0; v < m->n_nodes; ++v) {
+        const or_node *nd = &m->nodes[v];
+        const float *i0 = node_in(w, nd->in0, x);
+        const float *i1 = nd->kind == OR_ADD ? node_in(w, nd->in1, x) : NULL;
+        if (p->on[v]) node_fwd(m, w->shp, v, i0, i1, p->W[v], p->b[v], p->blk[v], w->buf[v]);
         else node_fwd(m, w->shp, v, i0, i1, nd->W, nd->b, NULL, w->buf[v]);
     }
     return w->buf[m->n_nodes - 1];
@@ -594,35 +705,25 @@ static void *vanilla_worker(void *arg)
     van_job *j = (van_job *)arg;
     const or_model *m = j->m;
     fwd_ws w;
+    mut_params mp;
     if ((j->rc = ws_init(&w, m))) return NULL;
+    if ((j->rc = mp_init(&mp, m))) { ws_free(&w); return NULL; }
     size_t in_sz = (size_t)m->in_h * m->in_w * m->in_c;
     int64_t W64 = (j->kc.n_in + 63) / 64;
-    size_t maxp = 0, maxc = 0;
-    for (int v = 0; v < m->n_nodes; ++v)
-        if (is_weighted(m->nodes[v].kind)) {
-            size_t p = (size_t)fan_in(&m->nodes[v]) * m->nodes[v].cout;
-            if (p > maxp) maxp = p;
-            if ((size_t)m->nodes[v].cout > maxc) maxc = m->nodes[v].cout;
-        }
-    float *Wm = (float *)malloc(sizeof(float) * (maxp ? maxp : 1));
-    float *bm = (float *)malloc(sizeof(float) * (maxc ? maxc : 1));
-    uint8_t *blk = (uint8_t *)malloc(maxc ? maxc : 1);
-    if (!Wm || !bm || !blk) { j->rc = OR_ENOMEM; goto out; }
     for (int64_t i = j->i0; i < j->i1; ++i) {
         const or_mutant *mu = &j->mut[i];
-        /* Build M' from scratch: its mutated layer's parameters are materialised. */
-        if ((j->rc = or_mutant_layer(m, mu, j->pool, j->pool_len, Wm, bm, blk))) goto out;
-        int mv = layer_node(m, mu->layer);
+        /* Build M' from scratch: its mutated layers' parameters are materialised. */
+        if ((j->rc = mp_load(&mp, m, mu, j->pool, j->pool_len))) goto out;
         uint64_t *row = j->kill_bits + i * W64;
         memset(row, 0, sizeof(uint64_t) * (size_t)W64);
         for (int64_t t = 0; t < j->kc.n_in; ++t) {
-            const float *y = forward_one(&w, j->X + (size_t)t * in_sz, mv, Wm, bm, blk);
+            const float *y = forward_mut(&w, j->X + (size_t)t * in_sz, &mp);
             if (j->logits) memcpy(j->logits + ((size_t)i * j->kc.n_in + t) * m->n_classes, y, sizeof(float) * (size_t)m->n_classes);
             if (kill_pred(&j->kc, t, argmax_f(y, m->n_classes))) set_kill(row, t);
         }
     }
 out:
-    free(Wm); free(bm); free(blk);
+    mp_free(&mp);
     ws_free(&w);
     return NULL;
 }
@@ -739,30 +840,22 @@ static void *memo_worker(void *arg)
     memo_job *j = (memo_job *)arg;
     const or_model *m = j->m;
     fwd_ws w;
+    mut_params mp;
     if ((j->rc = ws_init(&w, m))) return NULL;
+    if ((j->rc = mp_init(&mp, m))) { ws_free(&w); return NULL; }
     int64_t W64 = (j->kc.n_in + 63) / 64;
     size_t in_sz = (size_t)m->in_h * m->in_w * m->in_c;
-    size_t maxp = 0, maxc = 0;
-    for (int v = 0; v < m->n_nodes; ++v)
-        if (is_weighted(m->nodes[v].kind)) {
-            size_t p = (size_t)fan_in(&m->nodes[v]) * m->nodes[v].cout;
-            if (p > maxp) maxp = p;
-            if ((size_t)m->nodes[v].cout > maxc) maxc = m->nodes[v].cout;
-        }
-    float *Wm = (float *)malloc(sizeof(float) * (maxp ? maxp : 1));
-    float *bm = (float *)malloc(sizeof(float) * (maxc ? maxc : 1));
-    uint8_t *blk = (uint8_t *)malloc(maxc ? maxc : 1);
-    if (!Wm || !bm || !blk) { j->rc = OR_ENOMEM; goto out; }
     for (int64_t k = j->k0; k < j->k1; ++k) {
         int64_t id = j->ids[k];
         const or_mutant *mu = &j->mut[id];
-        if ((j->rc = or_mutant_layer(m, mu, j->pool, j->pool_len, Wm, bm, blk))) goto out;
+        if ((j->rc = mp_load(&mp, m, mu, j->pool, j->pool_len))) goto out;
         int mmi = layer_node(m, mu->layer);
         uint64_t *row = j->kill_bits + id * W64;
         memset(row, 0, sizeof(uint64_t) * (size_t)W64);
         for (int64_t t = 0; t < j->kc.n_in; ++t) {
-            /* chopped mutant: nodes mmi..V-1, inputs p < mmi from the memo table
-             * (the fresh input layers u_k), p >= mmi from `past` (w.buf). */
+            /* chopped mutant: nodes mmi..V-1 (every mutated node is >= mmi), inputs
+             * p < mmi from the memo table (the fresh input layers u_k), p >= mmi from
+             * `past` (w.buf). */
             for (int v = mmi; v < m->n_nodes; ++v) {
                 const or_node *nd = &m->nodes[v];
                 const float *in[2] = {NULL, NULL};
@@ -776,7 +869,7 @@ static void *memo_worker(void *arg)
                         in[e] = w.buf[p];
                     }
                 }
-                if (v == mmi) node_fwd(m, w.shp, v, in[0], in[1], Wm, bm, blk, w.buf[v]);
+                if (mp.on[v]) node_fwd(m, w.shp, v, in[0], in[1], mp.W[v], mp.b[v], mp.blk[v], w.buf[v]);
                 else node_fwd(m, w.shp, v, in[0], in[1], nd->W, nd->b, NULL, w.buf[v]);
             }
             const float *y = w.buf[m->n_nodes - 1];
@@ -785,7 +878,7 @@ static void *memo_worker(void *arg)
         }
     }
 out:
-    free(Wm); free(bm); free(blk);
+    mp_free(&mp);
     ws_free(&w);
     return NULL;
 }

@@ -103,6 +103,9 @@ class MutantTable:
     seed: np.ndarray         # uint64 [n]
     pool: np.ndarray         # int32 [sum n_neurons]
     ratio: np.ndarray        # float64 [n] (bookkeeping only)
+    # int32 [n] or None (all 0): 1 = the pool entries are (layer << 20 | neuron), the
+    # mutant spans several layers and `layer` is the smallest of them
+    tagged: np.ndarray = None
 
     def __len__(self):
         return int(self.layer.shape[0])
@@ -119,7 +122,8 @@ class MutantTable:
         pool = np.concatenate(pools).astype(np.int32) if pools else np.zeros(0, np.int32)
         return MutantTable(self.layer[idx].copy(), self.op[idx].copy(), self.n_neurons[idx].copy(),
                            np.asarray(offs, np.int64), self.param[idx].copy(), self.seed[idx].copy(),
-                           pool, self.ratio[idx].copy())
+                           pool, self.ratio[idx].copy(),
+                           None if self.tagged is None else self.tagged[idx].copy())
 
 
 # ----------------------------------------------------------------- networks --
@@ -292,6 +296,61 @@ def mutants(model: Model, n: int, seed: int = 2, ratios=(0.01,), ops=CONFIG_OPS,
                        np.concatenate(pool).astype(np.int32) if pool else np.zeros(0, np.int32), rat)
 
 
+def modelwide_mutants(model: Model, n: int, seed: int = 2, ratio: float = 0.01, ops=CONFIG_OPS) -> MutantTable:
+    """Descriptor table of n mutants whose neurons are drawn over the whole model
+    (DeepMutation's model-wide selection ratio; the paper's set mu(M') of mutated
+    layers): k = max(1, round(ratio x all neurons)) distinct (layer, neuron) pairs,
+    uniform over the model's neurons; NS draws k / 2 pairs, each inside one layer
+    chosen with probability proportional to its width.  Entries are encoded
+    (layer << 20 | neuron) in layer order ("tagged"); `layer` is the smallest."""
+    rng = np.random.default_rng(seed)
+    L = model.n_layers()
+    widths = np.array([model.layer_width(l) for l in range(L)], np.int64)
+    total = int(widths.sum())
+    starts = np.concatenate([[0], np.cumsum(widths)])
+    lay = np.zeros(n, np.int32)
+    opv = np.zeros(n, np.int32)
+    nn = np.zeros(n, np.int32)
+    off = np.zeros(n, np.int64)
+    par = np.zeros(n, np.float32)
+    sd = np.zeros(n, np.uint64)
+    rat = np.full(n, ratio, np.float64)
+    pool = []
+    pos = 0
+    k = max(1, int(np.floor(ratio * total + 0.5)))
+    pair_w = np.where(widths >= 2, widths, 0).astype(np.float64)
+    for i in range(n):
+        op = ops[i % len(ops)]
+        if op == "NS":
+            chosen = set()
+            ent = []
+            for _ in range(max(1, k // 2)):
+                while True:
+                    l = int(rng.choice(L, p=pair_w / pair_w.sum()))
+                    a, b = (int(v) for v in rng.choice(int(widths[l]), size=2, replace=False))
+                    if (l, a) not in chosen and (l, b) not in chosen:
+                        break
+                chosen.update({(l, a), (l, b)})
+                ent.append((l, a, b))
+            ent.sort()
+            entries = [(l << 20) | j for l, a, b in ent for j in (a, b)]
+        else:
+            flat = np.sort(rng.choice(total, size=min(k, total), replace=False))
+            ls = np.searchsorted(starts, flat, side="right") - 1
+            entries = [(int(l) << 20) | int(f - starts[l]) for f, l in zip(flat, ls)]
+        lay[i] = min(e >> 20 for e in entries)
+        opv[i] = OP_INDEX[op]
+        nn[i] = len(entries)
+        off[i] = pos
+        par[i] = 0.1 if op == "GF" else 0.0
+        sd[i] = np.uint64(int(rng.integers(0, 2 ** 63 - 1)))
+        pool.append(np.array(entries, np.int32))
+        pos += len(entries)
+    return MutantTable(lay, opv, nn, off, par, sd,
+                       np.concatenate(pool).astype(np.int32) if pool else np.zeros(0, np.int32), rat,
+                       np.ones(n, np.int32))
+
+
 def concat(tables) -> MutantTable:
     """One table holding the rows of several, in order."""
     tables = list(tables)
@@ -300,10 +359,14 @@ def concat(tables) -> MutantTable:
         offs.append(t.neuron_off + pos)
         pos += t.pool.size
     cat = lambda f, dt: np.concatenate([getattr(t, f) for t in tables]).astype(dt) if tables else np.zeros(0, dt)
+    tagged = None
+    if any(t.tagged is not None for t in tables):
+        tagged = np.concatenate([t.tagged if t.tagged is not None else np.zeros(len(t), np.int32)
+                                 for t in tables]).astype(np.int32)
     return MutantTable(cat("layer", np.int32), cat("op", np.int32), cat("n_neurons", np.int32),
                        np.concatenate(offs).astype(np.int64) if tables else np.zeros(0, np.int64),
                        cat("param", np.float32), cat("seed", np.uint64), cat("pool", np.int32),
-                       cat("ratio", np.float64))
+                       cat("ratio", np.float64), tagged)
 
 
 def table_from_rows(rows) -> MutantTable:
@@ -351,6 +414,9 @@ CONFIGS = {
     "vgg": ("vgg", 10000, 5000, (0.005, 0.01, 0.02, 0.05), None),
     "resnet20": ("resnet20", 10000, 5000, (0.01,), None),
     "vgg_stress": ("vgg", 20000, 20000, (0.001, 0.01, 0.05, 0.10), 0.5),
+    # model-wide selection: each mutant's neurons drawn over all layers (1 % of them)
+    "lenet5_modelwide": ("lenet5", 10000, 2000, (0.01,), "model"),
+    "mlp_modelwide": ("mlp", 1000, 200, (0.01,), "model"),
 }
 
 
@@ -363,5 +429,8 @@ def workload(name: str, n_inputs: int | None = None, n_mutants: int | None = Non
     n_in = n_in if n_inputs is None else n_inputs
     n_mut = n_mut if n_mutants is None else n_mutants
     X = inputs(model, n_in, input_seed)
-    table = mutants(model, n_mut, mutant_seed, ratios=ratios, first_layer_share=skew)
+    if skew == "model":
+        table = modelwide_mutants(model, n_mut, mutant_seed, ratio=ratios[0])
+    else:
+        table = mutants(model, n_mut, mutant_seed, ratios=ratios, first_layer_share=skew)
     return Workload(name, model, X, table)
