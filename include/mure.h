@@ -110,12 +110,19 @@ typedef struct {
     const mure_node *nodes;
 } mure_model_desc;
 
-/* One mutant descriptor (the mutant map of Algorithm 1, with mu(M') = {layer}). */
+/* One mutant descriptor (the mutant map of Algorithm 1).  Untagged (tagged = 0):
+ * mu(M') = {layer}, the pool entries are neuron ids of that layer.  Tagged
+ * (tagged = 1): the mutant's set mu(M') may hold several layers (the paper's general
+ * case, Sec. 3.2; DeepMutation's model-wide selection ratio); each pool entry is
+ * (layer << 20) | neuron and `layer` must be the smallest listed layer (mmi).  The
+ * operator applies to every listed neuron in its own layer: GF's sigma comes from that
+ * layer's weights, pool slot q keeps random stream q whatever its layer, and NS pairs
+ * (consecutive entries) lie in one layer. */
 typedef struct {
-    int32_t layer;      /* first (and only) mutated weighted layer, 0..L-1 */
+    int32_t layer;      /* first mutated weighted layer (mmi), 0..L-1 */
     int32_t op;         /* MURE_OP_* */
-    int32_t n_neurons;  /* neuron ids at neuron_pool[neuron_off .. +n_neurons) */
-    int32_t reserved;   /* must be 0 */
+    int32_t n_neurons;  /* pool entries at neuron_pool[neuron_off .. +n_neurons) */
+    int32_t tagged;     /* 0: entries are neurons of `layer`; 1: (layer << 20) | neuron */
     int64_t neuron_off;
     float param;        /* GF: sigma multiplier (e.g. 0.1); ignored otherwise */
     float reserved2;    /* must be 0 */
@@ -262,7 +269,8 @@ mure_status mure_eval_vanilla(mure_model *model, const float *X, int64_t n_input
  * offset[i] + q * F_l, where offset is returned in offsets [n_mutants] (-1 for other
  * operators).  GF: the noise added to each fan-in weight, fl32(sigma * n_f).  WS:
  * the permuted weights W[j][perm[f]].  out_len is the capacity of out (host);
- * Errors: INVALID_ARG (descriptors, or out too small), OOM, CUDA. */
+ * Errors: INVALID_ARG (descriptors, or out too small), UNSUPPORTED (a tagged
+ * descriptor), OOM, CUDA. */
 mure_status mure_expand_patches(mure_model *model, const mure_mutant *table, int64_t n_mutants,
                                 const int32_t *neuron_pool, int64_t pool_len, float *out, int64_t out_len,
                                 int64_t *offsets);
@@ -286,7 +294,7 @@ mure_status mure_expand_patches(mure_model *model, const mure_mutant *table, int
  * host threads) race and must not be issued.  The kernel initialises every scratch
  * entry it reads, so nothing carries over from an earlier call.  The call returns when
  * the patches are in out_dev.  Errors: INVALID_ARG (descriptors as in
- * mure_eval_mutants; out_len too small; descriptors needing more than the 8 MiB of
+ * mure_eval_mutants, untagged only; out_len too small; descriptors needing more than the 8 MiB of
  * scratch, with the needed size in mure_last_error), CUDA. */
 mure_status mure_expand_patches_noalloc(mure_model *model, const mure_mutant *table, int64_t n_mutants,
                                         const int32_t *neuron_pool, int64_t pool_len, float *out_dev,

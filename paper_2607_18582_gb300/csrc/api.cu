@@ -352,16 +352,25 @@ void check_table(mure_ctx *c, const mure_model *m, const mure_mutant *t, int64_t
         FAILIF(u.layer < 0 || u.layer >= m->L, c, MURE_ERR_INVALID_ARG, "mutant %lld: layer %d out of range",
                (long long)i, u.layer);
         FAILIF(u.op < MURE_OP_GF || u.op > MURE_OP_IDENTITY, c, MURE_ERR_INVALID_ARG, "mutant %lld: bad op", (long long)i);
-        FAILIF(u.reserved != 0 || u.reserved2 != 0.f, c, MURE_ERR_INVALID_ARG, "mutant %lld: reserved fields", (long long)i);
+        FAILIF((u.tagged != 0 && u.tagged != 1) || u.reserved2 != 0.f, c, MURE_ERR_INVALID_ARG,
+               "mutant %lld: reserved fields", (long long)i);
         FAILIF(u.n_neurons < 0 || u.neuron_off < 0 || u.neuron_off + u.n_neurons > pool_len, c, MURE_ERR_INVALID_ARG,
                "mutant %lld: neuron range outside the pool", (long long)i);
         FAILIF(u.op == MURE_OP_NS && (u.n_neurons & 1), c, MURE_ERR_INVALID_ARG, "mutant %lld: odd NS neuron count",
                (long long)i);
-        const int oc = m->st[u.layer].oc;
         seen.assign(pool + u.neuron_off, pool + u.neuron_off + u.n_neurons);
-        for (int64_t q = 0; q < u.n_neurons; ++q)
-            FAILIF(seen[q] < 0 || seen[q] >= oc, c, MURE_ERR_INVALID_ARG, "mutant %lld: neuron %lld out of range",
-                   (long long)i, (long long)seen[q]);
+        int lmin = m->L;
+        for (int64_t q = 0; q < u.n_neurons; ++q) {
+            const int32_t e = seen[q];
+            const int l = u.tagged ? (e < 0 ? -1 : e >> 20) : u.layer, j = u.tagged ? (e & 0xFFFFF) : e;
+            FAILIF(e < 0 || l < 0 || l >= m->L || j >= m->st[l].oc, c, MURE_ERR_INVALID_ARG,
+                   "mutant %lld: neuron entry %lld out of range", (long long)i, (long long)e);
+            FAILIF(u.op == MURE_OP_NS && (q & 1) && (u.tagged ? seen[q - 1] >> 20 : u.layer) != l, c,
+                   MURE_ERR_INVALID_ARG, "mutant %lld: an NS pair across two layers", (long long)i);
+            lmin = std::min(lmin, l);
+        }
+        FAILIF(u.tagged && u.n_neurons > 0 && lmin != u.layer, c, MURE_ERR_INVALID_ARG,
+               "mutant %lld: layer %d is not its smallest listed layer %d", (long long)i, u.layer, lmin);
         std::sort(seen.begin(), seen.end());
         FAILIF(std::adjacent_find(seen.begin(), seen.end()) != seen.end(), c, MURE_ERR_INVALID_ARG,
                "mutant %lld: repeated neuron", (long long)i);
@@ -393,6 +402,14 @@ struct DevTable {
     std::vector<int64_t> copy_prefix;  // [n+1] the same for NEB/NS alone
     int4 *vslot = nullptr;             // [val_prefix[n]] those slots: (group, q, source channel, op)
     int expand_launches = 0;
+    // tagged mutants with neurons in layers after their first: per layer v, per
+    // mutant (group order) the count, the offset into ids and the GF / WS patch offset
+    // of its neurons in v (0 / -1 where it has none)
+    bool has_later = false;
+    int64_t n = 0;
+    std::vector<std::vector<int32_t>> nn_at_host;   // [L][n]
+    int32_t *nn_at = nullptr;                       // [L][n]
+    int64_t *noff_at = nullptr, *poff_at = nullptr; // [L][n]
 };
 
 DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_mutant *t, int64_t n,
@@ -400,30 +417,68 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
                       int64_t *ids_from_group)
 {
     DevTable dt{};
+    const int L = m->L;
+    dt.n = n;
     std::vector<int32_t> op(n), nn(n), mid(n);
     std::vector<int64_t> noff(n), poff(n, -1);
     std::vector<SlotJob> jobs;
+    // the neuron ids of each mutant, decoded and grouped by layer: its first layer's
+    // segment, then one segment per later layer (tagged descriptors), each in pool order
+    std::vector<int32_t> ids;
+    ids.reserve((size_t)pool_len);
+    std::vector<std::vector<int64_t>> noff_at, poff_at;
     int64_t plen = 0, perm_len = 0;
     for (int64_t k = 0; k < n; ++k) {
         const int32_t i = g.order[k];
         const mure_mutant &u = t[i];
         op[k] = u.op;
-        nn[k] = u.op == MURE_OP_IDENTITY ? 0 : u.n_neurons;
-        noff[k] = u.neuron_off;
         mid[k] = i;
-        if ((u.op == MURE_OP_GF || u.op == MURE_OP_WS) && u.n_neurons > 0) {
-            const int F = m->st[u.layer].K;
-            poff[k] = plen;
+        const bool patched = u.op == MURE_OP_GF || u.op == MURE_OP_WS;
+        auto layer_of = [&](int q) { return u.tagged ? pool[u.neuron_off + q] >> 20 : u.layer; };
+        auto neuron_of = [&](int q) { return u.tagged ? pool[u.neuron_off + q] & 0xFFFFF : pool[u.neuron_off + q]; };
+        // segment of layer v: ids, and the patches of GF / WS (slot q keeps stream q)
+        auto segment = [&](int v, int64_t &seg_off, int64_t &seg_poff) {
+            seg_off = (int64_t)ids.size();
+            const int F = m->st[v].K;
+            int cnt = 0;
             for (int q = 0; q < u.n_neurons; ++q) {
-                SlotJob jb{};
-                jb.layer = u.layer; jb.op = u.op; jb.F = F; jb.j = pool[u.neuron_off + q]; jb.q = q;
-                jb.param = u.param; jb.seed = u.seed;
-                jb.out_off = plen + (int64_t)q * F;
-                jb.perm_off = perm_len;
-                if (u.op == MURE_OP_WS) perm_len += F;
-                jobs.push_back(jb);
+                if (layer_of(q) != v) continue;
+                ids.push_back(neuron_of(q));
+                if (patched) {
+                    SlotJob jb{};
+                    jb.layer = v; jb.op = u.op; jb.F = F; jb.j = neuron_of(q); jb.q = q;
+                    jb.param = u.param; jb.seed = u.seed;
+                    jb.out_off = plen + (int64_t)cnt * F;
+                    jb.perm_off = perm_len;
+                    if (u.op == MURE_OP_WS) perm_len += F;
+                    jobs.push_back(jb);
+                }
+                ++cnt;
             }
-            plen += (int64_t)u.n_neurons * F;
+            seg_poff = patched && cnt > 0 ? plen : -1;
+            if (patched) plen += (int64_t)cnt * F;
+            return cnt;
+        };
+        int64_t so = 0, sp = -1;
+        const int c0 = segment(u.layer, so, sp);
+        nn[k] = u.op == MURE_OP_IDENTITY ? 0 : c0;
+        noff[k] = so;
+        poff[k] = sp;
+        if (u.tagged) {
+            for (int v = u.layer + 1; v < L; ++v) {
+                int64_t vo = 0, vp = -1;
+                const int cv = segment(v, vo, vp);
+                if (cv == 0 || u.op == MURE_OP_IDENTITY) continue;
+                if (!dt.has_later) {
+                    dt.has_later = true;
+                    dt.nn_at_host.assign(L, std::vector<int32_t>(n, 0));
+                    noff_at.assign(L, std::vector<int64_t>(n, 0));
+                    poff_at.assign(L, std::vector<int64_t>(n, -1));
+                }
+                dt.nn_at_host[v][k] = cv;
+                noff_at[v][k] = vo;
+                poff_at[v][k] = vp;
+            }
         }
         if (ids_from_group) ids_from_group[i] = poff[k];
     }
@@ -447,24 +502,32 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
         dt.copy_prefix[k + 1] = dt.copy_prefix[k] + ((op[k] == MURE_OP_NEB || op[k] == MURE_OP_NS) ? nn[k] : 0);
         if (val)
             for (int q = 0; q < nn[k]; ++q)
-                vslot.push_back(make_int4((int)k, q, pool[noff[k] + (op[k] == MURE_OP_NS ? (q ^ 1) : q)], op[k]));
+                vslot.push_back(make_int4((int)k, q, ids[noff[k] + (op[k] == MURE_OP_NS ? (q ^ 1) : q)], op[k]));
     }
     // one staging buffer, one H2D copy
     const size_t b_op = n * 4, b_nn = n * 4, b_mid = n * 4, b_noff = n * 8, b_poff = n * 8;
     const size_t b_dslot = std::max<size_t>(dslot.size(), 1) * 4, b_vslot = std::max<size_t>(vslot.size(), 1) * 16;
-    const size_t b_ids = (size_t)std::max<int64_t>(pool_len, 1) * 4, b_jobs = jobs.size() * sizeof(SlotJob);
+    const size_t b_ids = std::max<size_t>(ids.size(), 1) * 4, b_jobs = jobs.size() * sizeof(SlotJob);
+    const size_t b_later = dt.has_later ? (size_t)L * n : 0;
     size_t off = 0;
     auto place = [&](size_t b) { size_t o = off; off = round_up(off + b, 256); return o; };
     const size_t o_op = place(b_op), o_nn = place(b_nn), o_mid = place(b_mid), o_noff = place(b_noff),
                  o_poff = place(b_poff), o_ids = place(b_ids), o_jobs = place(b_jobs), o_dslot = place(b_dslot),
-                 o_vslot = place(b_vslot);
+                 o_vslot = place(b_vslot), o_nnat = place(b_later * 4), o_noffat = place(b_later * 8),
+                 o_poffat = place(b_later * 8);
     std::vector<char> host(off);
     memcpy(host.data() + o_op, op.data(), b_op);
     memcpy(host.data() + o_nn, nn.data(), b_nn);
     memcpy(host.data() + o_mid, mid.data(), b_mid);
     memcpy(host.data() + o_noff, noff.data(), b_noff);
     memcpy(host.data() + o_poff, poff.data(), b_poff);
-    if (pool_len > 0) memcpy(host.data() + o_ids, pool, pool_len * 4);
+    if (!ids.empty()) memcpy(host.data() + o_ids, ids.data(), ids.size() * 4);
+    if (dt.has_later)
+        for (int v = 0; v < L; ++v) {
+            memcpy(host.data() + o_nnat + (size_t)v * n * 4, dt.nn_at_host[v].data(), (size_t)n * 4);
+            memcpy(host.data() + o_noffat + (size_t)v * n * 8, noff_at[v].data(), (size_t)n * 8);
+            memcpy(host.data() + o_poffat + (size_t)v * n * 8, poff_at[v].data(), (size_t)n * 8);
+        }
     if (!jobs.empty()) memcpy(host.data() + o_jobs, jobs.data(), b_jobs);
     if (!dslot.empty()) memcpy(host.data() + o_dslot, dslot.data(), dslot.size() * 4);
     if (!vslot.empty()) memcpy(host.data() + o_vslot, vslot.data(), vslot.size() * 16);
@@ -478,6 +541,11 @@ DevTable upload_table(mure_ctx *c, Scratch &sc, const mure_model *m, const mure_
     dt.ids = (int32_t *)(dev + o_ids);
     dt.dslot = (int32_t *)(dev + o_dslot);
     dt.vslot = (int4 *)(dev + o_vslot);
+    if (dt.has_later) {
+        dt.nn_at = (int32_t *)(dev + o_nnat);
+        dt.noff_at = (int64_t *)(dev + o_noffat);
+        dt.poff_at = (int64_t *)(dev + o_poffat);
+    }
     dt.patch = plen ? sc.get<float>(plen) : nullptr;
     if (!jobs.empty()) {
         std::vector<const float *> Wp(m->L);
@@ -535,11 +603,17 @@ int64_t gap_map_stride(const Stage &S)
 
 // Bytes per batch row for a group at layer l (vanilla: every stage input from 1,
 // plus z_l).
-int64_t row_bytes(const mure_model *m, int l, bool vanilla)
+int64_t row_bytes(const mure_model *m, int l, bool vanilla, bool z_rows = false)
 {
     int64_t b = 0;
     for (int s = vanilla ? 1 : l + 1; s <= m->L; ++s) b += m->xd[s].stride;
-    if (vanilla) b += m->zd[l].stride;
+    if (z_rows) {
+        int64_t zs = 0;
+        for (int v = 0; v < m->L; ++v) zs = std::max(zs, m->zd[v].stride);
+        b += zs;
+    } else if (vanilla) {
+        b += m->zd[l].stride;
+    }
     const Stage &S = m->st[l];
     b += (int64_t)S.oc * (S.gap ? 1 : (S.pool ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow));  // patch values (bound)
     int64_t g = 0;
@@ -549,7 +623,7 @@ int64_t row_bytes(const mure_model *m, int l, bool vanilla)
 }
 
 void alloc_workspace(mure_ctx *c, Scratch &sc, const mure_model *m, int64_t rows, bool vanilla, int lmin,
-                     int64_t patch_floats, int delta_slots, int delta_k, Workspace &ws)
+                     int64_t patch_floats, int delta_slots, int delta_k, Workspace &ws, bool z_rows = false)
 {
     ws.rows = rows;
     if (delta_slots > 0) {
@@ -570,7 +644,7 @@ void alloc_workspace(mure_ctx *c, Scratch &sc, const mure_model *m, int64_t rows
     ws.patch = sc.get<float>(rows * std::max<int64_t>(patch_floats, 1));
     ws.xb.assign(m->L + 1, nullptr);
     for (int s = vanilla ? 1 : lmin + 1; s <= m->L; ++s) ws.xb[s] = sc.get<float>(rows * m->xd[s].stride);
-    if (vanilla) {
+    if (vanilla || z_rows) {
         int64_t zs = 0;
         for (int l = 0; l < m->L; ++l) zs = std::max(zs, m->zd[l].stride);
         ws.z_stride = zs;
@@ -684,7 +758,16 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     // computed independently) on its staged maps, so the delta writes no values for
     // them; x_{l+1} must come from the small-convolution kernel, whose pooled values
     // the other operators' patches reproduce bit for bit
-    const bool win_ops = l + 2 < L && m->st[l + 1].tc && m->st[l + 1].tc_small && !skip_reader && !Sl.tc &&
+    // tagged mutants of the batch with neurons in later layers: the largest count per
+    // later layer (their rows then take the materialised path below)
+    std::vector<int> kv(L, 0);
+    bool later = false;
+    if (dt.has_later)
+        for (int v = l + 1; v < L; ++v) {
+            for (int64_t k = g0; k < g0 + G; ++k) kv[v] = std::max(kv[v], dt.nn_at_host[v][k]);
+            later |= kv[v] > 0;
+        }
+    const bool win_ops = !later && l + 2 < L && m->st[l + 1].tc && m->st[l + 1].tc_small && !skip_reader && !Sl.tc &&
                          Sl.variant > 0 && tc_overlay_inline(m->st[l + 1], ov, G) &&
                          !(l + 1 == L - 2 && tc_final_fusable(m->st[L - 2], m->st[L - 1]));
     if (win_ops) ov.op = pa.op;
@@ -712,6 +795,67 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     if (delta_err) return -1;
     // the unmutated rows of x_{l+1}: cached (memoized) or just computed (vanilla)
     const Src base = vanilla ? Src{ws.xb[l + 1], m->xd[l + 1].stride, 0} : Src{ca->x[l + 1], m->xd[l + 1].stride, 1};
+    if (later) {
+        // mu(M') holds later layers too: the rows of x_{l+1} are materialised with layer
+        // l's patch, and after every later mutated layer v its own delta (computed from
+        // the rows' x_v and z_v) is written over the rows of x_{v+1}; the output layer's
+        // delta goes through the kill epilogue.  Memoized and vanilla rows take this
+        // same path, and its arithmetic equals the fused paths' (same kernels on the
+        // same values), so a mutant's bits do not depend on its batch.
+        timed(C_DELTA, 0, [&] {
+            return launch_rows_overlay(base, m->xd[l + 1].size, rm, ov, ws.xb[l + 1], m->xd[l + 1].stride, s);
+        });
+        const Src zrows{ws.zb, ws.z_stride, 0};
+        for (int v = l + 1; v < L; ++v) {
+            const Stage &Sv = m->st[v];
+            const bool mut = kv[v] > 0;
+            const int cells_v = Sv.gap ? 1 : (Sv.pool ? (Sv.oh / 2) * (Sv.ow / 2) : Sv.oh * Sv.ow);
+            const int64_t pstride_v = (int64_t)std::max(kv[v], 1) * cells_v;
+            PatchArgs pv{dt.op + g0, dt.nn_at ? dt.nn_at + (size_t)v * dt.n + g0 : nullptr,
+                         dt.noff_at ? dt.noff_at + (size_t)v * dt.n + g0 : nullptr, dt.ids,
+                         dt.poff_at ? dt.poff_at + (size_t)v * dt.n + g0 : nullptr, dt.patch};
+            Overlay ovv;
+            ovv.patch = ws.patch;
+            ovv.row_stride = pstride_v;
+            ovv.kmax = kv[v];
+            ovv.cells = cells_v;
+            ovv.ch = Sv.oc;
+            ovv.n_neurons = pv.n_neurons;
+            ovv.neuron_off = pv.neuron_off;
+            ovv.ids = pv.ids;
+            const int64_t dfl = mut ? 2 * (int64_t)kv[v] * rm.R * Sv.oh * Sv.ow * Sv.K : 0;
+            if (v < L - 1) {
+                stage(v, mut ? ws.zb : nullptr, ws.z_stride);
+                if (!mut) continue;
+                acct.bytes_gather += rm.R * ((int64_t)kv[v] * cells_v + m->zd[v].size + m->xd[v].size) * 4;
+                timed(C_DELTA, dfl, [&] {
+                    return launch_patch_vals(Sv, zrows, xsrc(v), skip_of(Sv), rm, pv, kv[v], ws.patch, pstride_v, s);
+                });
+                const Src xr{ws.xb[v + 1], m->xd[v + 1].stride, 0};
+                timed(C_DELTA, 0, [&] {
+                    return launch_rows_overlay(xr, m->xd[v + 1].size, rm, ovv, ws.xb[v + 1], m->xd[v + 1].stride, s);
+                });
+            } else if (mut) {
+                FinalArgs f2 = fa;
+                f2.mode = 2;
+                f2.z_out = ws.zb;
+                f2.z_stride = ws.z_stride;
+                f2.logits_rows = ws.xb[L];
+                f2.x_stride = m->xd[L].stride;
+                timed(v, 2 * Sv.macs * rm.R, [&] { return launch_final_dense(Sv, xsrc(v), rm, f2, s); });
+                acct.bytes_gather += rm.R * ((int64_t)kv[v] + m->zd[v].size + m->xd[v].size) * 4;
+                timed(C_DELTA, dfl, [&] {
+                    return launch_patch_vals(Sv, zrows, xsrc(v), skip_of(Sv), rm, pv, kv[v], ws.patch, pstride_v, s);
+                });
+                timed(C_EPI, 0, [&] {
+                    return launch_epilogue(Src{ws.xb[L], m->xd[L].stride, 0}, m->n_classes, rm, fa, s, &ovv);
+                });
+            } else {
+                timed(v, 2 * Sv.macs * rm.R, [&] { return launch_final_dense(Sv, xsrc(v), rm, fa, s); });
+            }
+        }
+        return launches;
+    }
     if (l == L - 1) {
         // mutants of the output layer: the epilogue reads the logits with the overlay
         timed(C_EPI, 0, [&] { return launch_epilogue(base, m->n_classes, rm, fa, s, &ov); });
@@ -809,7 +953,10 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         int lmin = m->L;
         int64_t rb = 0;
         for (int l = 0; l < m->L; ++l)
-            if (g.begin[l + 1] > g.begin[l]) { lmin = std::min(lmin, l); rb = std::max(rb, row_bytes(m, l, vanilla)); }
+            if (g.begin[l + 1] > g.begin[l]) {
+                lmin = std::min(lmin, l);
+                rb = std::max(rb, row_bytes(m, l, vanilla, dt.has_later));
+            }
         int64_t rows = std::max<int64_t>(cap / std::max<int64_t>(rb, 1), 64);
         rows = std::min<int64_t>(rows, (int64_t)1 << 24);
         int64_t T = std::min<int64_t>(ca->n_pad, rows / 64 * 64);
@@ -825,6 +972,14 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
             const int64_t cl = S.gap ? 1 : (S.pool ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow);
             patch_floats = std::max<int64_t>(patch_floats, (int64_t)std::max(dt.kmax_layer[l], 1) * cl);
         }
+        if (dt.has_later)   // later mutated layers of tagged mutants: their patches too
+            for (int v = 0; v < m->L; ++v) {
+                const Stage &S = m->st[v];
+                const int64_t cl = S.gap ? 1 : (S.pool ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow);
+                int km = 0;
+                for (int64_t k = 0; k < n; ++k) km = std::max(km, dt.nn_at_host[v][k]);
+                patch_floats = std::max<int64_t>(patch_floats, (int64_t)km * cl);
+            }
         // the tensor-core delta: slots of a batch at most G x kmax of its layer
         int delta_slots = 0, delta_k = 0;
         for (int l = 0; l < m->L; ++l) {
@@ -834,7 +989,7 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
             delta_k = std::max(delta_k, m->st[l].K);
         }
         Workspace ws;
-        alloc_workspace(c, sc, m, rows, vanilla, lmin, patch_floats, delta_slots, delta_k, ws);
+        alloc_workspace(c, sc, m, rows, vanilla, lmin, patch_floats, delta_slots, delta_k, ws, dt.has_later);
         int64_t launches = 0;
         Acct acct;
         acct.flops_cls.assign(m->L + 3, 0);
@@ -1273,6 +1428,9 @@ mure_status mure_expand_patches(mure_model *m, const mure_mutant *table, int64_t
     return run(c, [&] {
         CK(c, cudaSetDevice(c->device));
         check_table(c, m, table, n_mutants, neuron_pool, pool_len);
+        for (int64_t i = 0; i < n_mutants; ++i)
+            FAILIF(table[i].tagged, c, MURE_ERR_UNSUPPORTED, "mutant %lld: tagged descriptors have no flat patch layout",
+                   (long long)i);
         FAILIF(!offsets && n_mutants > 0, c, MURE_ERR_INVALID_ARG, "NULL offsets");
         int64_t need = 0;
         for (int64_t i = 0; i < n_mutants; ++i)

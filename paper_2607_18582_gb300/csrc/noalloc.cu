@@ -56,7 +56,7 @@ extern "C" mure_status mure_expand_patches_noalloc(mure_model *m, const mure_mut
     int64_t patch_len = 0, perm_len = 0;
     for (int64_t i = 0; i < n_mutants; ++i) {
         const mure_mutant &u = table[i];
-        if (u.layer < 0 || u.layer >= m->L || u.op < MURE_OP_GF || u.op > MURE_OP_IDENTITY || u.reserved != 0 ||
+        if (u.layer < 0 || u.layer >= m->L || u.op < MURE_OP_GF || u.op > MURE_OP_IDENTITY || u.tagged != 0 ||
             u.reserved2 != 0.f || u.n_neurons < 0 || u.neuron_off < 0 || u.neuron_off + u.n_neurons > pool_len ||
             (u.op == MURE_OP_NS && (u.n_neurons & 1)))
             return fail(c, MURE_ERR_INVALID_ARG, "invalid mutant descriptor " + std::to_string(i));

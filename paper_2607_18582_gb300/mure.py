@@ -45,7 +45,7 @@ class _ModelDesc(C.Structure):
                 ("n_nodes", C.c_int32), ("precision", C.c_int32), ("nodes", C.POINTER(_Node))]
 
 
-MUTANT_DTYPE = np.dtype([("layer", "<i4"), ("op", "<i4"), ("n_neurons", "<i4"), ("reserved", "<i4"),
+MUTANT_DTYPE = np.dtype([("layer", "<i4"), ("op", "<i4"), ("n_neurons", "<i4"), ("tagged", "<i4"),
                          ("neuron_off", "<i8"), ("param", "<f4"), ("reserved2", "<f4"), ("seed", "<u8")])
 
 _ALLOC_FN = C.CFUNCTYPE(C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p)
@@ -320,6 +320,8 @@ def table_array(table):
     arr["neuron_off"][:n] = table.neuron_off
     arr["param"][:n] = table.param
     arr["seed"][:n] = table.seed
+    if getattr(table, "tagged", None) is not None:
+        arr["tagged"][:n] = table.tagged
     pool = np.ascontiguousarray(table.pool, np.int32)
     if pool.size == 0:
         pool = np.zeros(1, np.int32)
