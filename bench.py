@@ -42,6 +42,9 @@ WORKLOAD_TEXT = {
     "resnet20": "ResNet-20 32x32x3, 10,000 inputs N(0,1), 5,000 mutants, 1% ratio",
     "vgg": "VGG-style 32x32x3 (8 weighted layers), 10,000 inputs N(0,1), 5,000 mutants, ratios 0.5/1/2/5%",
     "vgg_stress": "VGG-style 32x32x3, 20,000 inputs N(0,1), 20,000 mutants, ratios 0.1/1/5/10%, 50% on the first conv",
+    "lenet5_modelwide": "LeNet-5 28x28x1, 10,000 inputs U[0,1], 2,000 mutants over several layers: 1% of all 236 "
+                        "neurons drawn model-wide per mutant (tagged descriptors), GF/NEB/NAI/NS",
+    "mlp_modelwide": "MLP 784-128-64-10, 1,000 inputs U[0,1], 200 mutants, 1% of all neurons drawn model-wide",
 }
 
 
