@@ -377,7 +377,7 @@ void check_table(mure_ctx *c, const mure_model *m, const mure_mutant *t, int64_t
     }
 }
 
-Groups group_by_layer(const mure_model *m, const mure_mutant *t, int64_t n)
+Groups group_by_layer(const mure_model *m, const mure_mutant *t, int64_t n, const int32_t *pool)
 {
     Groups g;
     g.begin.assign(m->L + 1, 0);
@@ -386,6 +386,25 @@ Groups group_by_layer(const mure_model *m, const mure_mutant *t, int64_t n)
     std::vector<int64_t> pos(g.begin.begin(), g.begin.end() - 1);
     g.order.resize(n);
     for (int64_t i = 0; i < n; ++i) g.order[pos[t[i].layer]++] = (int32_t)i;
+    // inside a group, tagged mutants by the set of later layers they change (stable):
+    // batches then share their later mutated layers, single-layer mutants keep the
+    // fused paths, and a batch without mutated tail layers keeps the fused output layer
+    // (a mutant's bits never depend on its batch)
+    std::vector<uint64_t> key(n, 0);
+    bool any = false;
+    for (int64_t i = 0; i < n; ++i) {
+        const mure_mutant &u = t[i];
+        if (!u.tagged || u.op == MURE_OP_IDENTITY) continue;
+        for (int q = 0; q < u.n_neurons; ++q) {
+            const int v = pool[u.neuron_off + q] >> 20;
+            if (v > u.layer && v < 64) key[i] |= 1ull << v;
+        }
+        any |= key[i] != 0;
+    }
+    if (any)
+        for (int l = 0; l < m->L; ++l)
+            std::stable_sort(g.order.begin() + g.begin[l], g.order.begin() + g.begin[l + 1],
+                             [&](int32_t a, int32_t b) { return key[a] < key[b]; });
     return g;
 }
 
@@ -806,9 +825,22 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
             return launch_rows_overlay(base, m->xd[l + 1].size, rm, ov, ws.xb[l + 1], m->xd[l + 1].stride, s);
         });
         const Src zrows{ws.zb, ws.z_stride, 0};
+        const bool fuse_tail = L >= 2 && tc_final_fusable(m->st[L - 2], m->st[L - 1]) && kv[L - 2] == 0 &&
+                               kv[L - 1] == 0 && !m->st[L - 2].has_add;
         for (int v = l + 1; v < L; ++v) {
             const Stage &Sv = m->st[v];
             const bool mut = kv[v] > 0;
+            if (fuse_tail && v == L - 2) {
+                // no mutated neuron from here on: the output layer in the epilogue of the
+                // layer before it, as on the single-layer path
+                const Stage &SLast = m->st[L - 1];
+                const FinalFuse ff{SLast.W, SLast.b, SLast.oc, SLast.K, SLast.act1, fa};
+                timed(L - 2, 2 * (Sv.macs + SLast.macs) * rm.R, [&] {
+                    return launch_tc(Sv, xsrc(v), rm, nullptr, 0, skip_of(Sv), ws.xb[L - 1], m->xd[L - 1].stride,
+                                     ws.gap_tmp, s, nullptr, &ff);
+                });
+                break;
+            }
             const int cells_v = Sv.gap ? 1 : (Sv.pool ? (Sv.oh / 2) * (Sv.ow / 2) : Sv.oh * Sv.ow);
             const int64_t pstride_v = (int64_t)std::max(kv[v], 1) * cells_v;
             PatchArgs pv{dt.op + g0, dt.nn_at ? dt.nn_at + (size_t)v * dt.n + g0 : nullptr,
@@ -929,7 +961,7 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
     cudaStream_t s = c->stream;
     Scratch sc(c);
     CK(c, cudaEventRecord(c->ev[0], s));
-    const Groups g = group_by_layer(m, t, n);
+    const Groups g = group_by_layer(m, t, n, pool);
     const int64_t words32 = ca->n_pad / 32;
     mure_eval_stats st{};
     st.n_rows = n * ca->n_in;

@@ -543,7 +543,8 @@ int launch_rows_overlay(Src base, int64_t n_floats, RowMap rm, const Overlay &ov
                         cudaStream_t s)
 {
     if (rm.R <= 0) return 0;
-    if (n_floats > 8192) {
+    // large rows, or rows patched in place (only the mutated channels are written)
+    if (n_floats > 8192 || (base.p == out && !base.per_input)) {
         int launches = 0;
         if (!(base.p == out && !base.per_input)) {
             const int64_t n4 = (n_floats + 3) / 4, total = (int64_t)rm.R * n4;

@@ -357,7 +357,7 @@ __global__ void __launch_bounds__(128) k_epilogue(const float *__restrict__ lg, 
     epilogue_row(fa, t0, T, row, in_range, v, C);
 }
 
-// The output layer for per-input rows with a dense overlay of at most 4 channels: each
+// The output layer for rows (per input or per row) with a dense overlay: each
 // thread copies its own input row (16-byte loads, all in flight at once) into its own
 // shared-memory row, writes the mutated channels there and runs the same fp32 chain as
 // k_final_dense (f ascending, fmaf(x, w, acc)), so both kernels give the same bits.
@@ -378,7 +378,7 @@ __global__ void __launch_bounds__(128) k_final_dense_rows(const FinalParams p)
         ws[i] = c < p.C ? __ldg(p.W + (int64_t)c * p.F + fl) : 0.f;
     }
     if (in_range) {
-        const float4 *src = reinterpret_cast<const float4 *>(p.x + (p.t0 + row % p.T) * p.x_stride);
+        const float4 *src = reinterpret_cast<const float4 *>(p.x + (p.x_per_input ? p.t0 + row % p.T : row) * p.x_stride);
         float4 v[kRowsF / 4];
 #pragma unroll
         for (int i = 0; i < kRowsF / 4; ++i)
@@ -448,7 +448,7 @@ int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cu
     const int cp = (p.C + 3) & ~3;
     // per-input rows with a small dense overlay, mutants' kill epilogue only: each
     // thread stages its own row (measured on the LeNet-5 workload, FC 84-10 of the FC
-    // 120-84 mutants: 0.68 -> 0.56 ms per step)
+    // 120-84 mutants: 0.68 -> 0.56 ms per step; on row-per-row inputs it was slower)
     if (x.per_input && fa.mode == 0 && !fa.z_out && p.F <= kRowsF - 4 && p.F % 4 == 0 && cp == 12 &&
         (x.stride & 3) == 0 && (reinterpret_cast<uintptr_t>(x.p) & 15) == 0 && (!ov || (ov->cells == 1 && ov->kmax <= 4))) {
         const size_t smem = ((size_t)p.F * 12 + 128 * kRowsF) * sizeof(float);
