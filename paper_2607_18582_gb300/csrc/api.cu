@@ -821,15 +821,36 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         // delta goes through the kill epilogue.  Memoized and vanilla rows take this
         // same path, and its arithmetic equals the fused paths' (same kernels on the
         // same values), so a mutant's bits do not depend on its batch.
-        timed(C_DELTA, 0, [&] {
-            return launch_rows_overlay(base, m->xd[l + 1].size, rm, ov, ws.xb[l + 1], m->xd[l + 1].stride, s);
-        });
-        const Src zrows{ws.zb, ws.z_stride, 0};
+        // an unmutated first suffix stage reads the cached rows with the overlay, as on
+        // the single-layer path; otherwise the rows of x_{l+1} are materialised
+        int vstart = l + 1;
+        if (kv[l + 1] == 0 && l + 2 < L) {
+            const Stage &Sn = m->st[l + 1];
+            if (Sn.tc && !skip_reader && tc_overlay_inline(Sn, ov, G)) {
+                timed(l + 1, 2 * Sn.macs * rm.R, [&] {
+                    return launch_tc(Sn, base, rm, nullptr, 0, skip_of(Sn), ws.xb[l + 2], m->xd[l + 2].stride,
+                                     ws.gap_tmp, s, &ov);
+                });
+                vstart = l + 2;
+            } else if (Sn.variant > 0 && !skip_reader) {
+                timed(l + 1, 2 * Sn.macs * rm.R, [&] {
+                    return launch_conv_small(Sn, base, rm, nullptr, 0, ws.xb[l + 2], m->xd[l + 2].stride, s, &ov);
+                });
+                vstart = l + 2;
+            }
+        }
+        if (vstart == l + 1)
+            timed(C_DELTA, 0, [&] {
+                return launch_rows_overlay(base, m->xd[l + 1].size, rm, ov, ws.xb[l + 1], m->xd[l + 1].stride, s);
+            });
         const bool fuse_tail = L >= 2 && tc_final_fusable(m->st[L - 2], m->st[L - 1]) && kv[L - 2] == 0 &&
                                kv[L - 1] == 0 && !m->st[L - 2].has_add;
-        for (int v = l + 1; v < L; ++v) {
+        for (int v = vstart; v < L; ++v) {
             const Stage &Sv = m->st[v];
             const bool mut = kv[v] > 0;
+            // z_v rows at the layer's own stride (the buffer holds the largest)
+            const int64_t zst = m->zd[v].stride;
+            const Src zrows{ws.zb, zst, 0};
             if (fuse_tail && v == L - 2) {
                 // no mutated neuron from here on: the output layer in the epilogue of the
                 // layer before it, as on the single-layer path
@@ -857,7 +878,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
             ovv.ids = pv.ids;
             const int64_t dfl = mut ? 2 * (int64_t)kv[v] * rm.R * Sv.oh * Sv.ow * Sv.K : 0;
             if (v < L - 1) {
-                stage(v, mut ? ws.zb : nullptr, ws.z_stride);
+                stage(v, mut ? ws.zb : nullptr, zst);
                 if (!mut) continue;
                 acct.bytes_gather += rm.R * ((int64_t)kv[v] * cells_v + m->zd[v].size + m->xd[v].size) * 4;
                 timed(C_DELTA, dfl, [&] {
@@ -871,7 +892,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
                 FinalArgs f2 = fa;
                 f2.mode = 2;
                 f2.z_out = ws.zb;
-                f2.z_stride = ws.z_stride;
+                f2.z_stride = zst;
                 f2.logits_rows = ws.xb[L];
                 f2.x_stride = m->xd[L].stride;
                 timed(v, 2 * Sv.macs * rm.R, [&] { return launch_final_dense(Sv, xsrc(v), rm, f2, s); });
