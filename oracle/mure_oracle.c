@@ -21,7 +21,7 @@
  * stored in fp32; every dot product, sum and mean is accumulated in fp64 and rounded
  * to fp32 once.  Products of two fp32 values are exact in fp64.
  *
- * Readings of the paper used here (each is listed in the design doc):
+ * Readings of the paper used here:
  *   - neuron j of a weighted layer = output channel j (conv) / output unit j (dense)
  *     (Sec. 2.1: a conv filter's output channel is one neuron).
  *   - mutation operators (delegated by the paper to DeepMutation, Sec. 3.1):

@@ -154,3 +154,25 @@ def test_invalid_tagged_mutants_rejected(oracle_mod):
         t.layer[0] = layer
         with pytest.raises(oracle_mod.OracleError):
             oracle_mod.vanilla(w.model, w.X, t)
+
+
+@pytest.mark.parametrize("name", ["lenet5", "vgg", "resnet20", "mlp"])
+def test_modelwide_generator_structure(name):
+    """The model-wide tables are well formed: distinct (layer, neuron) entries in range,
+    `layer` the smallest listed one, NS pairs inside one layer, k from the ratio."""
+    w = wl.workload(name, 1, 1)
+    m = w.model
+    widths = [m.layer_width(l) for l in range(m.n_layers())]
+    t = wl.modelwide_mutants(m, 64, seed=13, ratio=0.01)
+    k = max(1, int(np.floor(0.01 * sum(widths) + 0.5)))
+    for i in range(len(t)):
+        a, n = int(t.neuron_off[i]), int(t.n_neurons[i])
+        ent = [(int(e) >> 20, int(e) & 0xFFFFF) for e in t.pool[a:a + n]]
+        assert len(set(ent)) == n
+        assert all(0 <= l < len(widths) and 0 <= j < widths[l] for l, j in ent)
+        assert int(t.layer[i]) == min(l for l, _ in ent)
+        if wl.OPS[int(t.op[i])] == "NS":
+            assert n == 2 * max(1, k // 2)
+            assert all(ent[q][0] == ent[q + 1][0] for q in range(0, n, 2))
+        else:
+            assert n == min(k, sum(widths))
