@@ -450,6 +450,13 @@ def main():
         # (differences are expected only on near ties; the TF32 variant reports its rate)
         out["oracle_agreement"] = agree
     out["hbm"] = hbm_rates(w, results, cls_ms, pk, pk_kind)
+    # the batched suffix's activation rows written and read back through device memory
+    # (not algorithmic bytes: ideally they would stay on chip)
+    rows_b = sum(r["stats"].get("bytes_rows", 0) for r in results)
+    evals = sum(r["stats"]["n_rows"] for r in results)
+    if evals > 0:
+        out["activation_rows"] = {"bytes_per_eval": rows_b / evals, "unit": "B",
+                                  "counted": "suffix stage output rows, written once and read once"}
     out["peaks"] = {"source": pk_kind, "hbm_gbs": pk.get("hbm_gbs"), "bf16_tflops": pk.get("bf16_tflops")}
     if rank == 0:
         print(json.dumps(out), flush=True)

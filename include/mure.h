@@ -169,6 +169,9 @@ typedef struct {
     double ms_delta, ms_gather, ms_epilogue;
     int64_t bytes_gather;   /* row bytes the delta kernel copies (read + write) */
     int64_t launches_delta;
+    int64_t bytes_rows;     /* activation rows the stage kernels write and the next stage
+                               reads back (2 x rows x row bytes): the device-memory traffic
+                               of the batched suffix beyond the algorithmic bytes */
 } mure_eval_stats;
 
 #define MURE_MAX_TIMED_LAYERS 64

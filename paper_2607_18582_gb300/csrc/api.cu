@@ -680,6 +680,7 @@ struct Acct {
     int64_t flops = 0;
     std::vector<int64_t> flops_cls, launches_cls;   // [L + 3]
     int64_t bytes_gather = 0;
+    int64_t bytes_rows = 0;
 };
 
 int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevTable &dt, const EvalCfg &ec,
@@ -725,6 +726,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     auto skip_of = [&](const Stage &S) -> Src { return S.has_add ? xsrc(S.skip_src) : Src{nullptr, 0, 0}; };
     auto stage = [&](int v, float *z_out, int64_t z_stride) {
         const Stage &S = m->st[v];
+        acct.bytes_rows += 2 * (int64_t)rm.R * m->xd[v + 1].size * 4;
         timed(v, 2 * S.macs * rm.R, [&] {
             return launch_stage_simt(S, xsrc(v), rm, z_out, z_stride, skip_of(S), ws.xb[v + 1], m->xd[v + 1].stride,
                                      ws.gap_tmp, s);
@@ -827,12 +829,14 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         if (kv[l + 1] == 0 && l + 2 < L) {
             const Stage &Sn = m->st[l + 1];
             if (Sn.tc && !skip_reader && tc_overlay_inline(Sn, ov, G)) {
+                acct.bytes_rows += 2 * (int64_t)rm.R * m->xd[l + 2].size * 4;
                 timed(l + 1, 2 * Sn.macs * rm.R, [&] {
                     return launch_tc(Sn, base, rm, nullptr, 0, skip_of(Sn), ws.xb[l + 2], m->xd[l + 2].stride,
                                      ws.gap_tmp, s, &ov);
                 });
                 vstart = l + 2;
             } else if (Sn.variant > 0 && !skip_reader) {
+                acct.bytes_rows += 2 * (int64_t)rm.R * m->xd[l + 2].size * 4;
                 timed(l + 1, 2 * Sn.macs * rm.R, [&] {
                     return launch_conv_small(Sn, base, rm, nullptr, 0, ws.xb[l + 2], m->xd[l + 2].stride, s, &ov);
                 });
@@ -939,11 +943,13 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
             fused_last(base, &ov);
             return launches;
         }
+        acct.bytes_rows += 2 * (int64_t)rm.R * m->xd[l + 2].size * 4;
         timed(l + 1, 2 * Sn.macs * rm.R, [&] {
             return launch_tc(Sn, base, rm, nullptr, 0, skip_of(Sn), ws.xb[l + 2], m->xd[l + 2].stride, ws.gap_tmp, s,
                              &ov);
         });
     } else if (Sn.variant > 0 && !skip_reader) {
+        acct.bytes_rows += 2 * (int64_t)rm.R * m->xd[l + 2].size * 4;
         timed(l + 1, 2 * Sn.macs * rm.R, [&] {
             return launch_conv_small(Sn, base, rm, nullptr, 0, ws.xb[l + 2], m->xd[l + 2].stride, s, &ov);
         });
@@ -1107,6 +1113,7 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
             st.launches_delta = acct.launches_cls[m->L];
         }
         st.bytes_gather = acct.bytes_gather;
+        st.bytes_rows = acct.bytes_rows;
         float ms = 0;
         cudaEventElapsedTime(&ms, c->ev[0], c->ev[4]); st.ms_total = ms;
         cudaEventElapsedTime(&ms, c->ev[0], c->ev[1]); st.ms_expand = ms;

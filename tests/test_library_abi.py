@@ -46,7 +46,7 @@ def test_struct_layouts_match_header():
     assert mure.MUTANT_DTYPE.fields["neuron_off"][1] == 16
     assert mure.MUTANT_DTYPE.fields["seed"][1] == 32
     assert ctypes.sizeof(mure._Opts) == 24
-    assert ctypes.sizeof(mure._Stats) == 4 * 8 + 6 * 8 + 64 * 8 * 3 + 3 * 8 + 2 * 8
+    assert ctypes.sizeof(mure._Stats) == 4 * 8 + 6 * 8 + 64 * 8 * 3 + 3 * 8 + 3 * 8
 
 
 def test_library_loads_and_fails_cleanly_without_gpu(libpath):
