@@ -1,0 +1,73 @@
+"""Host-side logic of bench.py on the CPU: the roofline traffic lookup (valid only while
+the kernel source is unchanged), the clock-record parsing, the HBM-rate arithmetic and
+the oracle sample."""
+import hashlib
+import os
+import sys
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+from paper_2607_18582_gb300 import workloads as wl  # noqa: E402
+
+
+def _profile(tmp_path, src_text, sha, per_row=2000.0):
+    (tmp_path / "profiles").mkdir(exist_ok=True)
+    (tmp_path / "src.cu").write_text(src_text)
+    (tmp_path / "profiles" / "k.md").write_text(
+        f"# summary\n\n    dram_bytes_per_row: {per_row}\n    source_file: src.cu\n    source_sha256: {sha}\n")
+
+
+def test_profiled_traffic_tracks_the_source(tmp_path, monkeypatch):
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    text = "kernel source\n"
+    _profile(tmp_path, text, hashlib.sha256(text.encode()).hexdigest(), 2000.0)
+    assert bench.profiled_traffic("k", 10.0) == 20000.0
+    (tmp_path / "src.cu").write_text(text + "// changed\n")
+    assert bench.profiled_traffic("k", 10.0) is None
+    assert bench.profiled_traffic("missing", 10.0) is None
+
+
+def test_clock_summary_parsing():
+    cs = bench.ClockSampler(0)
+    cs.lines = ["0, 2070, 2070, 900.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+                "0, 2040, 2070, 1390.0, 0x4, Not Active, Not Active, Not Active, Active",
+                "0, 2070, 2070, 950.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+                "garbage line"]
+    s = cs.summary()
+    assert s["sm_mhz"] == 2070.0 and s["sm_max_mhz"] == 2070.0 and s["samples"] == 3
+    assert s["reasons"] == ["sw_power_cap"]
+    empty = bench.ClockSampler(0)
+    empty.lines = []
+    assert empty.summary()["reasons"] == ["unsampled"]
+
+
+def test_hbm_rates_arithmetic():
+    w = wl.workload("lenet5", 4, 4)
+    L = w.model.n_layers()
+    rows = 1000
+    macs = w.model.layer_macs(L - 1)
+    results = [{"stats": {"bytes_gather": 6_799_300, "flops_layer": [0] * (L - 1) + [2 * macs * rows]}}]
+    out = bench.hbm_rates(w, results, {"delta": 1.0, f"layer{L - 1}": 2.0}, {"hbm_gbs": 6799.3}, "measured")
+    assert out["delta"]["achieved"] == pytest.approx(6.7993)            # 6.8 MB in 1 ms
+    assert out["delta"]["frac"] == pytest.approx(6.7993 / 6799.3)
+    node = w.model.nodes[w.model.layers()[L - 1]]
+    exp = rows * (node.cin * 4 + 1 / 8) / 2e-3 / 1e9
+    assert out["output_layer"]["achieved"] == pytest.approx(exp)
+
+
+@pytest.mark.parametrize("name", ["lenet5", "lenet5_modelwide"])
+def test_oracle_sample_is_stratified(name):
+    w = wl.workload(name, 50, 400)
+    sub, X, idx = bench.oracle_sample(w, 40, 20, with_index=True)
+    assert len(sub) == 40 and len(X) == 20 and len(np.unique(idx)) == 40
+    assert set(np.unique(sub.layer)) == set(np.unique(w.table.layer[:400]))
+    if w.table.tagged is not None:
+        assert np.array_equal(sub.tagged, w.table.tagged[idx])
+        for j, i in enumerate(idx):
+            a, n = int(w.table.neuron_off[i]), int(w.table.n_neurons[i])
+            b = int(sub.neuron_off[j])
+            assert np.array_equal(sub.pool[b:b + n], w.table.pool[a:a + n])
