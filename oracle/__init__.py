@@ -19,8 +19,8 @@ _SRC = os.path.join(_HERE, "mure_oracle.c")
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "libmure_oracle.so")
 
-KINDS = {"conv": 0, "dense": 1, "maxpool": 2, "flatten": 3, "add": 4, "gap": 5, "shortcut": 6}
-ACTS = {"none": 0, "relu": 1}
+KINDS = {"conv": 0, "dense": 1, "maxpool": 2, "flatten": 3, "add": 4, "gap": 5, "shortcut": 6, "dwconv": 7}
+ACTS = {"none": 0, "relu": 1, "relu6": 2}
 OPS = {"GF": 0, "NEB": 1, "NAI": 2, "NS": 3, "WS": 4, "IDENTITY": 5}
 
 

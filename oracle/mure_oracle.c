@@ -55,8 +55,8 @@
 /* ------------------------------------------------------------------ types -- */
 
 enum { OR_CONV = 0, OR_DENSE = 1, OR_MAXPOOL = 2, OR_FLATTEN = 3, OR_ADD = 4,
-       OR_GAP = 5, OR_SHORTCUT = 6 };
-enum { OR_ACT_NONE = 0, OR_ACT_RELU = 1 };
+       OR_GAP = 5, OR_SHORTCUT = 6, OR_DWCONV = 7 };
+enum { OR_ACT_NONE = 0, OR_ACT_RELU = 1, OR_ACT_RELU6 = 2 };
 enum { OR_OP_GF = 0, OR_OP_NEB = 1, OR_OP_NAI = 2, OR_OP_NS = 3, OR_OP_WS = 4,
        OR_OP_IDENTITY = 5 };
 enum { OR_OK = 0, OR_EINVAL = 1, OR_EUNSUP = 2, OR_ENOMEM = 3 };
@@ -66,7 +66,7 @@ typedef struct {
     int32_t kind, act, in0, in1;
     int32_t kh, kw, stride, pad; /* conv window / pool window / shortcut stride */
     int32_t cin, cout;           /* conv & dense fan-in channels / outputs; shortcut channels */
-    const float *W;              /* conv [cout][kh][kw][cin], dense [cout][cin] */
+    const float *W;              /* conv [cout][kh][kw][cin], dense [cout][cin], depthwise conv [c][kh][kw] */
     const float *b;              /* [cout] */
 } or_node;
 
@@ -137,7 +137,7 @@ void or_fisher_yates(uint64_t stream_seed, int32_t n, int32_t *perm)
 
 /* ------------------------------------------------------------- shapes -- */
 
-static int is_weighted(int kind) { return kind == OR_CONV || kind == OR_DENSE; }
+static int is_weighted(int kind) { return kind == OR_CONV || kind == OR_DENSE || kind == OR_DWCONV; }
 
 /* Output shape of every node; returns OR_EINVAL for an inconsistent graph. */
 int or_shapes(const or_model *m, int32_t *out_hwc /* [n_nodes][3] */)
@@ -156,6 +156,16 @@ int or_shapes(const or_model *m, int32_t *out_hwc /* [n_nodes][3] */)
             o.h = (a.h + 2 * nd->pad - nd->kh) / nd->stride + 1;
             o.w = (a.w + 2 * nd->pad - nd->kw) / nd->stride + 1;
             o.c = nd->cout;
+            if (o.h < 1 || o.w < 1) rc = OR_EINVAL;
+            break;
+        case OR_DWCONV:
+            /* depthwise: one kh x kw filter per channel (MobileNetV2, Table 1) */
+            if (nd->cin != a.c || nd->cout != a.c || nd->stride < 1 || nd->kh < 1 || nd->kw < 1 || nd->pad < 0) {
+                rc = OR_EINVAL;
+                break;
+            }
+            o.h = (a.h + 2 * nd->pad - nd->kh) / nd->stride + 1;
+            o.w = (a.w + 2 * nd->pad - nd->kw) / nd->stride + 1;
             if (o.h < 1 || o.w < 1) rc = OR_EINVAL;
             break;
         case OR_DENSE:
@@ -201,7 +211,12 @@ int or_shapes(const or_model *m, int32_t *out_hwc /* [n_nodes][3] */)
 
 /* --------------------------------------------------------- layer math -- */
 
-static float act_f(int act, float v) { return (act == OR_ACT_RELU) ? (v > 0.0f ? v : 0.0f) : v; }
+static float act_f(int act, float v)
+{
+    if (act == OR_ACT_RELU) return v > 0.0f ? v : 0.0f;
+    if (act == OR_ACT_RELU6) return v > 0.0f ? (v < 6.0f ? v : 6.0f) : 0.0f;
+    return v;
+}
 
 /* Conv2d, NHWC, zero padding, fp64 accumulation, then the activation. */
 static void conv_fwd(const or_node *nd, shape3 a, const float *x, shape3 o, const float *W,
@@ -223,6 +238,28 @@ static void conv_fwd(const or_node *nd, shape3 a, const float *x, shape3 o, cons
                     }
                 }
                 y[((size_t)oy * o.w + ox) * o.c + co] = act_f(nd->act, (float)acc);
+            }
+}
+
+/* Depthwise conv2d, NHWC: channel c is convolved with its own kh x kw filter. */
+static void dwconv_fwd(const or_node *nd, shape3 a, const float *x, shape3 o, const float *W,
+                       const float *b, float *y)
+{
+    for (int oy = 0; oy < o.h; ++oy)
+        for (int ox = 0; ox < o.w; ++ox)
+            for (int c = 0; c < o.c; ++c) {
+                double acc = (double)b[c];
+                for (int ky = 0; ky < nd->kh; ++ky) {
+                    int iy = oy * nd->stride - nd->pad + ky;
+                    if (iy < 0 || iy >= a.h) continue;
+                    for (int kx = 0; kx < nd->kw; ++kx) {
+                        int ix = ox * nd->stride - nd->pad + kx;
+                        if (ix < 0 || ix >= a.w) continue;
+                        acc += (double)W[((size_t)c * nd->kh + ky) * nd->kw + kx] *
+                               (double)x[((size_t)iy * a.w + ix) * a.c + c];
+                    }
+                }
+                y[((size_t)oy * o.w + ox) * o.c + c] = act_f(nd->act, (float)acc);
             }
 }
 
@@ -280,6 +317,7 @@ static void node_fwd(const or_model *m, const shape3 *shp, int v, const float *i
     size_t n = (size_t)o.h * o.w * o.c;
     switch (nd->kind) {
     case OR_CONV: conv_fwd(nd, a, in0, o, W, b, out); break;
+    case OR_DWCONV: dwconv_fwd(nd, a, in0, o, W, b, out); break;
     case OR_DENSE: dense_fwd(nd, in0, W, b, out); break;
     case OR_MAXPOOL: maxpool_fwd(nd, a, in0, o, out); break;
     case OR_FLATTEN: memcpy(out, in0, n * sizeof(float)); break;
@@ -325,7 +363,12 @@ int32_t or_n_layers(const or_model *m)
     return l;
 }
 
-static int64_t fan_in(const or_node *nd) { return nd->kind == OR_CONV ? (int64_t)nd->kh * nd->kw * nd->cin : nd->cin; }
+static int64_t fan_in(const or_node *nd)
+{
+    if (nd->kind == OR_CONV) return (int64_t)nd->kh * nd->kw * nd->cin;
+    if (nd->kind == OR_DWCONV) return (int64_t)nd->kh * nd->kw;   /* a channel sees its own input channel */
+    return nd->cin;
+}
 
 /* Population standard deviation (ddof 0) of a layer's weights, two passes in fp64. */
 double or_layer_std(const or_model *m, int32_t layer)
@@ -975,6 +1018,7 @@ int64_t or_node_macs(const or_model *m, int32_t v)
     const or_node *nd = &m->nodes[v];
     int64_t r = 0;
     if (nd->kind == OR_CONV) r = (int64_t)s[3 * v] * s[3 * v + 1] * nd->cout * nd->kh * nd->kw * nd->cin;
+    else if (nd->kind == OR_DWCONV) r = (int64_t)s[3 * v] * s[3 * v + 1] * nd->cout * nd->kh * nd->kw;
     else if (nd->kind == OR_DENSE) r = (int64_t)nd->cin * nd->cout;
     free(s);
     return r;

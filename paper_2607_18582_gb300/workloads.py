@@ -34,7 +34,7 @@ CONFIG_OPS = ("GF", "NEB", "NAI", "NS")
 
 @dataclass
 class Node:
-    kind: str                 # conv | dense | maxpool | flatten | add | gap | shortcut
+    kind: str                 # conv | dense | maxpool | flatten | add | gap | shortcut | dwconv
     inputs: tuple             # node ids; -1 = the model input
     act: str = "none"         # none | relu
     kh: int = 1
@@ -56,7 +56,7 @@ class Model:
 
     def layers(self):
         """Node ids of the weighted nodes (conv, dense) in node order."""
-        return [v for v, n in enumerate(self.nodes) if n.kind in ("conv", "dense")]
+        return [v for v, n in enumerate(self.nodes) if n.kind in ("conv", "dense", "dwconv")]
 
     def n_layers(self):
         return len(self.layers())
@@ -69,7 +69,7 @@ class Model:
         out = []
         for n in self.nodes:
             h, w, c = self.in_shape if n.inputs[0] < 0 else out[n.inputs[0]]
-            if n.kind == "conv":
+            if n.kind in ("conv", "dwconv"):
                 out.append(((h + 2 * n.pad - n.kh) // n.stride + 1, (w + 2 * n.pad - n.kw) // n.stride + 1, n.cout))
             elif n.kind == "dense":
                 out.append((1, 1, n.cout))
@@ -90,6 +90,8 @@ class Model:
         v = self.layers()[layer]
         n = self.nodes[v]
         h, w, c = self.shapes()[v]
+        if n.kind == "dwconv":
+            return h * w * c * n.kh * n.kw
         return h * w * c * (n.kh * n.kw * n.cin if n.kind == "conv" else n.cin)
 
 
@@ -151,6 +153,14 @@ class _Builder:
         oh = (h + 2 * pad - k) // stride + 1
         ow = (w + 2 * pad - k) // stride + 1
         return self._add(Node("conv", (x,), act, k, k, stride, pad, c, cout, W, b), (oh, ow, cout))
+
+    def dwconv(self, x, k, stride=1, pad=0, act="relu6"):
+        h, w, c = self.shape[x]
+        W = (self.rng.standard_normal((c, k, k)) * np.sqrt(2.0 / (k * k))).astype(np.float32)
+        b = self.rng.uniform(-0.05, 0.05, size=c).astype(np.float32)
+        oh = (h + 2 * pad - k) // stride + 1
+        ow = (w + 2 * pad - k) // stride + 1
+        return self._add(Node("dwconv", (x,), act, k, k, stride, pad, c, c, W, b), (oh, ow, c))
 
     def dense(self, x, cout, act="relu"):
         h, w, c = self.shape[x]
@@ -237,7 +247,27 @@ def resnet20(seed=0):
     return bld.m
 
 
-MODELS = {"mlp": mlp, "lenet5": lenet5, "vgg": vgg, "resnet20": resnet20}
+def mobilenetv2_tiny(seed=0):
+    """A small MobileNetV2-style network on 32x32x3 (the paper's MobileNetV2 family,
+    Table 1): conv3x3(16)+ReLU6, three inverted residual blocks (1x1 expansion x4 +
+    ReLU6, 3x3 depthwise + ReLU6, linear 1x1 projection; a residual add where the shape
+    is kept), conv1x1(64)+ReLU6, global average pooling, dense 10.  Oracle only: the
+    GPU library has no depthwise layer yet."""
+    bld = _Builder("mobilenetv2_tiny", (32, 32, 3), 10, seed)
+    x = bld.conv(-1, 16, 3, stride=1, pad=1, act="relu6")
+    for cout, stride in ((16, 1), (24, 2), (24, 1)):
+        cin = bld.shape[x][2]
+        h = bld.conv(x, 4 * cin, 1, act="relu6")
+        h = bld.dwconv(h, 3, stride=stride, pad=1, act="relu6")
+        h = bld.conv(h, cout, 1, act="none")
+        x = bld.add(h, x, act="none") if stride == 1 and cin == cout else h
+    x = bld.conv(x, 64, 1, act="relu6")
+    x = bld.gap(x)
+    bld.dense(x, 10, act="none")
+    return bld.m
+
+
+MODELS = {"mlp": mlp, "lenet5": lenet5, "vgg": vgg, "resnet20": resnet20, "mobilenetv2_tiny": mobilenetv2_tiny}
 
 
 # ------------------------------------------------------------------- inputs --
