@@ -84,6 +84,8 @@ def lib():
             L.or_mutant_layer.argtypes = [C.POINTER(_Model), C.POINTER(_Mutant), _I32P, C.c_int64, _FP, _FP, _U8P]
             L.or_mutant_layer_at.argtypes = [C.POINTER(_Model), C.POINTER(_Mutant), _I32P, C.c_int64, C.c_int32,
                                              _FP, _FP, _U8P]
+            L.or_unchanged_rows.argtypes = [C.POINTER(_Model), _FP, C.c_int64, C.POINTER(_Mutant), C.c_int64,
+                                            _I32P, C.c_int64, C.c_int32, _U64P]
             L.or_forward.argtypes = [C.POINTER(_Model), _FP, C.c_int64, _FP, _I32P]
             L.or_forward_nodes.argtypes = [C.POINTER(_Model), _FP, _FP]
             L.or_scores.argtypes = [_U64P, C.c_int64, C.c_int64, _I32P, C.c_int32, _DP, _DP, C.POINTER(C.c_int64)]
@@ -249,6 +251,20 @@ def _run(fn, model, X, table, labels, n_threads, want_logits, memo):
 def vanilla(model, X, table, labels=None, n_threads=None, want_logits=True):
     """Vanilla mutation testing (every mutant built and run end to end)."""
     return _run(lib().or_vanilla, model, X, table, labels, n_threads, want_logits, memo=False)
+
+
+def unchanged_rows(model, X, table, n_threads=None):
+    """Bits [n_mut][ceil(n_in/64)]: every layer the mutant changes gives, on that input,
+    the original output bit for bit (the row's suffix and prediction are the original's)."""
+    om = OModel(model)
+    X = np.ascontiguousarray(X, np.float32)
+    n_in, n_mut = X.shape[0], len(table)
+    arr, pool, plen = _mutants(table)
+    W64 = (n_in + 63) // 64
+    bits = np.zeros((max(n_mut, 1), max(W64, 1)), np.uint64)
+    _check(lib().or_unchanged_rows(C.byref(om.c), _ptr(X, _FP) if X.size else None, n_in, arr, n_mut,
+                                   _ptr(pool, _I32P), plen, n_threads or (os.cpu_count() or 1), _ptr(bits, _U64P)))
+    return bits[:n_mut, :W64]
 
 
 def memo(model, X, table, labels=None, n_threads=None, want_logits=True):

@@ -834,6 +834,79 @@ int or_vanilla(const or_model *m, const float *X, int64_t n_in, const int32_t *l
     return rc;
 }
 
+/* --------------------------------------------------- unchanged rows -- */
+
+/* Exact unchanged-row test (a reference for eliminating rows before their suffix): bit
+ * (i, t) is set when, on input t, the output of every node that mutant i changes equals
+ * the original network's output of that node bit for bit.  Then every later node, the
+ * logits and the prediction are the original's too, so kill(i, t) = 0 without running
+ * the suffix.  Bits as in the kill matrix: [n_mut][ceil(n_in/64)], LSB first. */
+typedef struct {
+    const or_model *m;
+    const float *X;
+    int64_t n_in;
+    const or_mutant *mut;
+    const int32_t *pool;
+    int64_t pool_len;
+    uint64_t *bits;
+    int64_t i0, i1;
+    int rc;
+} unch_job;
+
+static void *unchanged_worker(void *arg)
+{
+    unch_job *j = (unch_job *)arg;
+    const or_model *m = j->m;
+    fwd_ws w0, w1;
+    mut_params mp;
+    if ((j->rc = ws_init(&w0, m))) return NULL;
+    if ((j->rc = ws_init(&w1, m))) { ws_free(&w0); return NULL; }
+    if ((j->rc = mp_init(&mp, m))) { ws_free(&w0); ws_free(&w1); return NULL; }
+    size_t in_sz = (size_t)m->in_h * m->in_w * m->in_c;
+    int64_t W64 = (j->n_in + 63) / 64;
+    for (int64_t i = j->i0; i < j->i1; ++i) {
+        if ((j->rc = mp_load(&mp, m, &j->mut[i], j->pool, j->pool_len))) goto out;
+        uint64_t *row = j->bits + i * W64;
+        memset(row, 0, sizeof(uint64_t) * (size_t)W64);
+        for (int64_t t = 0; t < j->n_in; ++t) {
+            const float *x = j->X + (size_t)t * in_sz;
+            forward_one(&w0, x, -1, NULL, NULL, NULL);
+            forward_mut(&w1, x, &mp);
+            int same = 1;
+            for (int v = 0; v < m->n_nodes && same; ++v)
+                if (mp.on[v] && memcmp(w0.buf[v], w1.buf[v], sizeof(float) * w0.size[v]) != 0) same = 0;
+            if (same) set_kill(row, t);
+        }
+    }
+out:
+    mp_free(&mp);
+    ws_free(&w0);
+    ws_free(&w1);
+    return NULL;
+}
+
+int or_unchanged_rows(const or_model *m, const float *X, int64_t n_in, const or_mutant *mut, int64_t n_mut,
+                      const int32_t *pool, int64_t pool_len, int32_t n_threads, uint64_t *bits)
+{
+    int rc = check_model(m);
+    if (rc) return rc;
+    if (n_in < 0 || n_mut < 0 || (n_mut > 0 && !mut) || !bits) return OR_EINVAL;
+    for (int64_t i = 0; i < n_mut; ++i)
+        if ((rc = check_mutant(m, &mut[i], pool, pool_len))) return rc;
+    if (n_mut == 0) return OR_OK;
+    if (n_threads < 1) n_threads = 1;
+    if (n_threads > n_mut) n_threads = (int32_t)n_mut;
+    unch_job *jobs = (unch_job *)calloc((size_t)n_threads, sizeof(unch_job));
+    if (!jobs) return OR_ENOMEM;
+    for (int k = 0; k < n_threads; ++k)
+        jobs[k] = (unch_job){m, X, n_in, mut, pool, pool_len, bits, n_mut * k / n_threads,
+                             n_mut * (k + 1) / n_threads, OR_OK};
+    rc = run_workers(unchanged_worker, jobs, sizeof(unch_job), n_threads);
+    for (int k = 0; rc == OR_OK && k < n_threads; ++k) if (jobs[k].rc) rc = jobs[k].rc;
+    free(jobs);
+    return rc;
+}
+
 /* ------------------------------------------- memoized (Algorithms 1-4) -- */
 
 /* Algorithm 2: dg[v] = set of nodes v reads from (node ids; -1 = model input).
