@@ -247,6 +247,28 @@ def resnet20(seed=0):
     return bld.m
 
 
+def resnet10(seed=0):
+    """ResNet-10 on 32x32x3 (the paper's ResNet family, Table 1): stem conv, four
+    stages of one basic block each (16/32/64/128 channels), projection shortcuts (a
+    1x1 convolution of stride 2 in the skip branch where the shape changes), global
+    average pooling, FC 128-10.  The skip branch holds a weighted layer, so the
+    memoization boundary of a mutant depends on Algorithm 2's graph, not on a chain.
+    Oracle only: the GPU stage compiler takes option-A shortcuts."""
+    bld = _Builder("resnet10", (32, 32, 3), 10, seed)
+    x = bld.conv(-1, 16, 3, pad=1)
+    cin = 16
+    for s, c in enumerate((16, 32, 64, 128)):
+        stride = 1 if s == 0 else 2
+        a = bld.conv(x, c, 3, stride=stride, pad=1, act="relu")
+        bb = bld.conv(a, c, 3, stride=1, pad=1, act="none")
+        sc = x if (stride == 1 and cin == c) else bld.conv(x, c, 1, stride=stride, pad=0, act="none")
+        x = bld.add(bb, sc, act="relu")
+        cin = c
+    x = bld.gap(x)
+    bld.dense(x, 10, act="none")
+    return bld.m
+
+
 def mobilenetv2_tiny(seed=0):
     """A small MobileNetV2-style network on 32x32x3 (the paper's MobileNetV2 family,
     Table 1): conv3x3(16)+ReLU6, three inverted residual blocks (1x1 expansion x4 +
@@ -267,7 +289,8 @@ def mobilenetv2_tiny(seed=0):
     return bld.m
 
 
-MODELS = {"mlp": mlp, "lenet5": lenet5, "vgg": vgg, "resnet20": resnet20, "mobilenetv2_tiny": mobilenetv2_tiny}
+MODELS = {"mlp": mlp, "lenet5": lenet5, "vgg": vgg, "resnet20": resnet20, "resnet10": resnet10,
+          "mobilenetv2_tiny": mobilenetv2_tiny}
 
 
 # ------------------------------------------------------------------- inputs --
