@@ -19,7 +19,8 @@ _SRC = os.path.join(_HERE, "mure_oracle.c")
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "libmure_oracle.so")
 
-KINDS = {"conv": 0, "dense": 1, "maxpool": 2, "flatten": 3, "add": 4, "gap": 5, "shortcut": 6, "dwconv": 7}
+KINDS = {"conv": 0, "dense": 1, "maxpool": 2, "flatten": 3, "add": 4, "gap": 5, "shortcut": 6, "dwconv": 7, "embed": 8,
+         "lstm": 9}
 ACTS = {"none": 0, "relu": 1, "relu6": 2}
 OPS = {"GF": 0, "NEB": 1, "NAI": 2, "NS": 3, "WS": 4, "IDENTITY": 5}
 
@@ -211,12 +212,12 @@ def mutant_layer(model, table, i, layer=None):
     v = model.layers()[layer]
     nd = model.nodes[v]
     W = np.zeros_like(nd.W)
-    b = np.zeros_like(nd.b)
+    b = np.zeros_like(nd.b) if nd.b is not None else np.zeros(1, np.float32)   # an embedding has no bias
     blk = np.zeros(nd.cout, np.uint8)
     arr, pool, plen = _mutants(table)
     _check(lib().or_mutant_layer_at(C.byref(om.c), C.byref(arr[i]), _ptr(pool, _I32P), plen, layer,
                                     _ptr(W, _FP), _ptr(b, _FP), _ptr(blk, _U8P)))
-    return W, b, blk.astype(bool)
+    return W, (b if nd.b is not None else None), blk.astype(bool)
 
 
 def _run(fn, model, X, table, labels, n_threads, want_logits, memo):

@@ -32,6 +32,14 @@
  *       NS  : swap (w[j0], b[j0]) with (w[j1], b[j1]) for each listed pair
  *       NEB : the output of neuron j is forced to 0 (after the layer's activation)
  *       IDENTITY : no change
+ *   - recurrent models (Sec. 5.3: an embedding, two LSTM layers, a dense output): a
+ *     neuron of an embedding is one output channel (a column of the table, no bias);
+ *     a neuron of an LSTM layer is one unit, whose fan-in is the four gates' input and
+ *     recurrent weights (4 (cin + units) values) and whose biases are the four gate
+ *     biases.  The operators above act on these: NAI negates all of the unit's weights
+ *     and biases, NS swaps two units' weights and biases, WS shuffles the unit's whole
+ *     fan-in list, and NEB holds the unit's output h at 0 at every step (the
+ *     recurrence sees the 0 too).
  *   - mutants over several layers (the paper's set mu(M') of mutated layers, Sec. 3.2;
  *     DeepMutation's model-wide selection): a "tagged" descriptor lists
  *     (layer << 20 | neuron) entries; the operator is applied to each listed neuron in
@@ -55,7 +63,7 @@
 /* ------------------------------------------------------------------ types -- */
 
 enum { OR_CONV = 0, OR_DENSE = 1, OR_MAXPOOL = 2, OR_FLATTEN = 3, OR_ADD = 4,
-       OR_GAP = 5, OR_SHORTCUT = 6, OR_DWCONV = 7 };
+       OR_GAP = 5, OR_SHORTCUT = 6, OR_DWCONV = 7, OR_EMBED = 8, OR_LSTM = 9 };
 enum { OR_ACT_NONE = 0, OR_ACT_RELU = 1, OR_ACT_RELU6 = 2 };
 enum { OR_OP_GF = 0, OR_OP_NEB = 1, OR_OP_NAI = 2, OR_OP_NS = 3, OR_OP_WS = 4,
        OR_OP_IDENTITY = 5 };
@@ -64,10 +72,15 @@ enum { OR_OK = 0, OR_EINVAL = 1, OR_EUNSUP = 2, OR_ENOMEM = 3 };
 /* One node of the network DAG.  Inputs are node ids; -1 is the model input. */
 typedef struct {
     int32_t kind, act, in0, in1;
-    int32_t kh, kw, stride, pad; /* conv window / pool window / shortcut stride */
-    int32_t cin, cout;           /* conv & dense fan-in channels / outputs; shortcut channels */
-    const float *W;              /* conv [cout][kh][kw][cin], dense [cout][cin], depthwise conv [c][kh][kw] */
-    const float *b;              /* [cout] */
+    int32_t kh, kw, stride, pad; /* conv window / pool window / shortcut stride; LSTM: kh = 1 returns
+                                    every step's output, kh = 0 only the last one */
+    int32_t cin, cout;           /* conv & dense fan-in channels / outputs; shortcut channels;
+                                    embedding: vocabulary size / width; LSTM: input features / units */
+    const float *W;              /* conv [cout][kh][kw][cin], dense [cout][cin], depthwise conv [c][kh][kw],
+                                    embedding [cout][cin] (neuron j = column j of the table),
+                                    LSTM [cout][4][cin + cout] (unit j, gates i, f, g, o; input then
+                                    recurrent weights) */
+    const float *b;              /* [cout]; LSTM [cout][4]; embedding none */
 } or_node;
 
 typedef struct {
@@ -137,7 +150,13 @@ void or_fisher_yates(uint64_t stream_seed, int32_t n, int32_t *perm)
 
 /* ------------------------------------------------------------- shapes -- */
 
-static int is_weighted(int kind) { return kind == OR_CONV || kind == OR_DENSE || kind == OR_DWCONV; }
+static int is_weighted(int kind)
+{
+    return kind == OR_CONV || kind == OR_DENSE || kind == OR_DWCONV || kind == OR_EMBED || kind == OR_LSTM;
+}
+
+/* Biases a neuron owns: an LSTM unit one per gate, an embedding none. */
+static int n_bias(const or_node *nd) { return nd->kind == OR_LSTM ? 4 : nd->kind == OR_EMBED ? 0 : 1; }
 
 /* Output shape of every node; returns OR_EINVAL for an inconsistent graph. */
 int or_shapes(const or_model *m, int32_t *out_hwc /* [n_nodes][3] */)
@@ -194,6 +213,24 @@ int or_shapes(const or_model *m, int32_t *out_hwc /* [n_nodes][3] */)
             if (nd->stride < 1 || nd->cout < a.c) { rc = OR_EINVAL; break; }
             o.h = (a.h - 1) / nd->stride + 1;
             o.w = (a.w - 1) / nd->stride + 1;
+            o.c = nd->cout;
+            break;
+        case OR_EMBED:
+            /* token ids (one per position) from the model input to vectors of width cout */
+            if (nd->in0 != -1 || a.c != 1 || nd->cin < 1 || nd->cout < 1 || nd->act != OR_ACT_NONE) {
+                rc = OR_EINVAL;
+                break;
+            }
+            o.c = nd->cout;
+            break;
+        case OR_LSTM:
+            /* a sequence of a.w steps of a.c features */
+            if (a.h != 1 || nd->cin != a.c || nd->cout < 1 || nd->cout > 4096 || (nd->kh != 0 && nd->kh != 1) ||
+                nd->act != OR_ACT_NONE) {
+                rc = OR_EINVAL;
+                break;
+            }
+            o.w = nd->kh ? a.w : 1;
             o.c = nd->cout;
             break;
         default:
@@ -263,6 +300,53 @@ static void dwconv_fwd(const or_node *nd, shape3 a, const float *x, shape3 o, co
             }
 }
 
+/* Embedding lookup: position p holds token id x[p] (checked on entry), its output
+ * channel j is W[j][x[p]]. */
+static void embed_fwd(const or_node *nd, shape3 a, const float *x, const float *W, float *y)
+{
+    for (int p = 0; p < a.h * a.w; ++p) {
+        int32_t tok = (int32_t)x[p];
+        for (int j = 0; j < nd->cout; ++j) y[(size_t)p * nd->cout + j] = W[(size_t)j * nd->cin + tok];
+    }
+}
+
+static double sigmoid64(double v) { return 1.0 / (1.0 + exp(-v)); }
+
+/* LSTM with the Keras defaults (recurrent activation sigmoid, activation tanh), zero
+ * initial state.  Per step t and unit j, with u = [x_t, h_{t-1}]:
+ *   a_g = b[j][g] + sum_f W[j][g][f] u[f]   for the gates g = i, f, g, o
+ *   i = sigma(a_i), f = sigma(a_f), g = tanh(a_g), o = sigma(a_o)
+ *   c_t = f c_{t-1} + i g,   h_t = o tanh(c_t)
+ * Every stored value (a, the gates, c, h) is fp32; each sum and product is formed in
+ * fp64 and rounded once.  A blocked unit outputs h = 0 at every step, so the next
+ * step's gates see 0 too. */
+static void lstm_fwd(const or_node *nd, shape3 a, const float *x, const float *W, const float *b,
+                     const uint8_t *blocked, float *y)
+{
+    const int T = a.w, F = nd->cin, H = nd->cout, U = F + H;
+    float c[H], h[H], c2[H], h2[H];
+    for (int j = 0; j < H; ++j) { c[j] = 0.0f; h[j] = 0.0f; }
+    for (int t = 0; t < T; ++t) {
+        const float *xt = x + (size_t)t * F;
+        for (int j = 0; j < H; ++j) {
+            float gate[4];
+            for (int g = 0; g < 4; ++g) {
+                const float *wp = W + ((size_t)j * 4 + g) * U;
+                double acc = (double)b[4 * j + g];
+                for (int f = 0; f < F; ++f) acc += (double)wp[f] * (double)xt[f];
+                for (int k = 0; k < H; ++k) acc += (double)wp[F + k] * (double)h[k];
+                float pre = (float)acc;
+                gate[g] = g == 2 ? (float)tanh((double)pre) : (float)sigmoid64((double)pre);
+            }
+            c2[j] = (float)((double)gate[1] * (double)c[j] + (double)gate[0] * (double)gate[2]);
+            h2[j] = blocked && blocked[j] ? 0.0f : (float)((double)gate[3] * tanh((double)c2[j]));
+        }
+        for (int j = 0; j < H; ++j) { c[j] = c2[j]; h[j] = h2[j]; }
+        if (nd->kh) memcpy(y + (size_t)t * H, h, sizeof(float) * (size_t)H);
+    }
+    if (!nd->kh) memcpy(y, h, sizeof(float) * (size_t)H);
+}
+
 static void dense_fwd(const or_node *nd, const float *x, const float *W, const float *b, float *y)
 {
     for (int o = 0; o < nd->cout; ++o) {
@@ -326,11 +410,30 @@ static void node_fwd(const or_model *m, const shape3 *shp, int v, const float *i
         break;
     case OR_GAP: gap_fwd(a, in0, out); break;
     case OR_SHORTCUT: shortcut_fwd(nd, a, in0, o, out); break;
+    case OR_EMBED: embed_fwd(nd, a, in0, W, out); break;
+    case OR_LSTM: lstm_fwd(nd, a, in0, W, b, blocked, out); break;
     }
     if (blocked && is_weighted(nd->kind))
         for (size_t p = 0; p < (size_t)o.h * o.w; ++p)
             for (int c = 0; c < o.c; ++c)
                 if (blocked[c]) out[p * o.c + c] = 0.0f;
+}
+
+/* Token ids fed to embedding node v: every value an integer in [0, vocabulary). */
+static int check_tokens(const or_node *nd, const float *x, int64_t n)
+{
+    for (int64_t i = 0; i < n; ++i)
+        if (!(x[i] >= 0.0f && x[i] < (float)nd->cin && x[i] == floorf(x[i]))) return OR_EINVAL;
+    return OR_OK;
+}
+
+/* The model input checked against every embedding that reads it. */
+static int check_input(const or_model *m, const float *X, int64_t n)
+{
+    int64_t per = (int64_t)m->in_h * m->in_w * m->in_c;
+    for (int v = 0; v < m->n_nodes; ++v)
+        if (m->nodes[v].kind == OR_EMBED && n > 0 && check_tokens(&m->nodes[v], X, n * per)) return OR_EINVAL;
+    return OR_OK;
 }
 
 /* One node on one input, for pinning the layer functions against library routines. */
@@ -340,6 +443,8 @@ int or_node_forward(const or_model *m, int32_t v, const float *in0, const float 
     shape3 *shp = (shape3 *)malloc(sizeof(shape3) * (size_t)m->n_nodes);
     if (!shp) return OR_ENOMEM;
     int rc = or_shapes(m, (int32_t *)shp);
+    if (rc == OR_OK && m->nodes[v].kind == OR_EMBED)
+        rc = check_tokens(&m->nodes[v], in0, (int64_t)m->in_h * m->in_w * m->in_c);
     if (rc == OR_OK) node_fwd(m, shp, v, in0, in1, m->nodes[v].W, m->nodes[v].b, NULL, out);
     free(shp);
     return rc;
@@ -367,7 +472,8 @@ static int64_t fan_in(const or_node *nd)
 {
     if (nd->kind == OR_CONV) return (int64_t)nd->kh * nd->kw * nd->cin;
     if (nd->kind == OR_DWCONV) return (int64_t)nd->kh * nd->kw;   /* a channel sees its own input channel */
-    return nd->cin;
+    if (nd->kind == OR_LSTM) return 4 * ((int64_t)nd->cin + nd->cout);  /* four gates over [x_t, h_{t-1}] */
+    return nd->cin;   /* dense; embedding: the neuron's column of the table */
 }
 
 /* Population standard deviation (ddof 0) of a layer's weights, two passes in fp64. */
@@ -436,8 +542,9 @@ int or_mutant_layer_at(const or_model *m, const or_mutant *mu, const int32_t *po
     if (layer < 0 || layer >= or_n_layers(m)) return OR_EINVAL;
     const or_node *nd = &m->nodes[layer_node(m, layer)];
     int64_t F = fan_in(nd);
+    int nb = n_bias(nd);
     memcpy(W_out, nd->W, sizeof(float) * (size_t)(F * nd->cout));
-    memcpy(b_out, nd->b, sizeof(float) * (size_t)nd->cout);
+    if (nb) memcpy(b_out, nd->b, sizeof(float) * (size_t)nb * nd->cout);
     memset(blocked_out, 0, (size_t)nd->cout);
     const int32_t *ent = pool + mu->neuron_off;
     /* slot q is in this layer: its neuron id, else -1 */
@@ -474,7 +581,7 @@ int or_mutant_layer_at(const or_model *m, const or_mutant *mu, const int32_t *po
             if (SLOT_J(q) < 0) continue;
             float *w = W_out + (size_t)SLOT_J(q) * F;
             for (int64_t f = 0; f < F; ++f) w[f] = -w[f];
-            b_out[SLOT_J(q)] = -b_out[SLOT_J(q)];
+            for (int g = 0; g < nb; ++g) b_out[nb * SLOT_J(q) + g] = -b_out[nb * SLOT_J(q) + g];
         }
         break;
     case OR_OP_NS:
@@ -483,8 +590,10 @@ int or_mutant_layer_at(const or_model *m, const or_mutant *mu, const int32_t *po
             int j0 = SLOT_J(q), j1 = SLOT_J(q + 1);
             memcpy(W_out + (size_t)j0 * F, nd->W + (size_t)j1 * F, sizeof(float) * (size_t)F);
             memcpy(W_out + (size_t)j1 * F, nd->W + (size_t)j0 * F, sizeof(float) * (size_t)F);
-            b_out[j0] = nd->b[j1];
-            b_out[j1] = nd->b[j0];
+            for (int g = 0; g < nb; ++g) {
+                b_out[nb * j0 + g] = nd->b[nb * j1 + g];
+                b_out[nb * j1 + g] = nd->b[nb * j0 + g];
+            }
         }
         break;
     case OR_OP_NEB:
@@ -603,7 +712,7 @@ static int mp_load(mut_params *p, const or_model *m, const or_mutant *mu, const 
         const or_node *nd = &m->nodes[v];
         if (!p->W[v]) {
             p->W[v] = (float *)malloc(sizeof(float) * (size_t)(fan_in(nd) * nd->cout));
-            p->b[v] = (float *)malloc(sizeof(float) * (size_t)nd->cout);
+            p->b[v] = (float *)malloc(sizeof(float) * (size_t)(n_bias(nd) ? n_bias(nd) : 1) * nd->cout);
             p->blk[v] = (uint8_t *)malloc((size_t)nd->cout);
             if (!p->W[v] || !p->b[v] || !p->blk[v]) return OR_ENOMEM;
         }
@@ -655,6 +764,7 @@ int or_forward(const or_model *m, const float *X, int64_t n, float *logits, int3
 {
     int rc = check_model(m);
     if (rc) return rc;
+    if (n > 0 && (rc = check_input(m, X, n))) return rc;
     fwd_ws w;
     if ((rc = ws_init(&w, m))) return rc;
     size_t in_sz = (size_t)m->in_h * m->in_w * m->in_c;
@@ -672,6 +782,7 @@ int or_forward_nodes(const or_model *m, const float *x, float *all_out)
 {
     int rc = check_model(m);
     if (rc) return rc;
+    if ((rc = check_input(m, x, 1))) return rc;
     fwd_ws w;
     if ((rc = ws_init(&w, m))) return rc;
     forward_one(&w, x, -1, NULL, NULL, NULL);
@@ -891,6 +1002,7 @@ int or_unchanged_rows(const or_model *m, const float *X, int64_t n_in, const or_
     int rc = check_model(m);
     if (rc) return rc;
     if (n_in < 0 || n_mut < 0 || (n_mut > 0 && !mut) || !bits) return OR_EINVAL;
+    if (n_in > 0 && (rc = check_input(m, X, n_in))) return rc;
     for (int64_t i = 0; i < n_mut; ++i)
         if ((rc = check_mutant(m, &mut[i], pool, pool_len))) return rc;
     if (n_mut == 0) return OR_OK;
@@ -1093,6 +1205,8 @@ int64_t or_node_macs(const or_model *m, int32_t v)
     if (nd->kind == OR_CONV) r = (int64_t)s[3 * v] * s[3 * v + 1] * nd->cout * nd->kh * nd->kw * nd->cin;
     else if (nd->kind == OR_DWCONV) r = (int64_t)s[3 * v] * s[3 * v + 1] * nd->cout * nd->kh * nd->kw;
     else if (nd->kind == OR_DENSE) r = (int64_t)nd->cin * nd->cout;
+    else if (nd->kind == OR_LSTM)   /* steps x units x four gates x [x_t, h_{t-1}] */
+        r = (int64_t)(nd->in0 < 0 ? m->in_w : s[3 * nd->in0 + 1]) * nd->cout * 4 * (nd->cin + nd->cout);
     free(s);
     return r;
 }

@@ -28,23 +28,26 @@ from dataclasses import dataclass, field
 import numpy as np
 
 OPS = ("GF", "NEB", "NAI", "NS", "WS", "IDENTITY")
+WEIGHTED = ("conv", "dense", "dwconv", "embed", "lstm")
 OP_INDEX = {name: i for i, name in enumerate(OPS)}
 CONFIG_OPS = ("GF", "NEB", "NAI", "NS")
 
 
 @dataclass
 class Node:
-    kind: str                 # conv | dense | maxpool | flatten | add | gap | shortcut | dwconv
+    kind: str                 # conv | dense | maxpool | flatten | add | gap | shortcut | dwconv | embed | lstm
     inputs: tuple             # node ids; -1 = the model input
-    act: str = "none"         # none | relu
-    kh: int = 1
+    act: str = "none"         # none | relu | relu6
+    kh: int = 1               # lstm: 1 = every step's output, 0 = the last step's
     kw: int = 1
     stride: int = 1
     pad: int = 0
     cin: int = 0
     cout: int = 0
-    W: np.ndarray | None = None   # conv [cout][kh][kw][cin], dense [cout][cin], fp32
-    b: np.ndarray | None = None   # [cout], fp32
+    # conv [cout][kh][kw][cin], dense [cout][cin], dwconv [c][kh][kw], embed [cout][vocabulary]
+    # (channel-major), lstm [units][4][cin + units] (gates i, f, g, o; input then recurrent), fp32
+    W: np.ndarray | None = None
+    b: np.ndarray | None = None   # [cout]; lstm [units][4]; embed None
 
 
 @dataclass
@@ -55,8 +58,8 @@ class Model:
     nodes: list = field(default_factory=list)
 
     def layers(self):
-        """Node ids of the weighted nodes (conv, dense) in node order."""
-        return [v for v, n in enumerate(self.nodes) if n.kind in ("conv", "dense", "dwconv")]
+        """Node ids of the weighted nodes in node order."""
+        return [v for v, n in enumerate(self.nodes) if n.kind in WEIGHTED]
 
     def n_layers(self):
         return len(self.layers())
@@ -81,6 +84,10 @@ class Model:
                 out.append((1, 1, c))
             elif n.kind == "shortcut":
                 out.append(((h - 1) // n.stride + 1, (w - 1) // n.stride + 1, n.cout))
+            elif n.kind == "embed":
+                out.append((h, w, n.cout))
+            elif n.kind == "lstm":
+                out.append((1, w if n.kh else 1, n.cout))
             else:
                 out.append((h, w, c))
         return out
@@ -92,6 +99,11 @@ class Model:
         h, w, c = self.shapes()[v]
         if n.kind == "dwconv":
             return h * w * c * n.kh * n.kw
+        if n.kind == "embed":
+            return 0   # a table lookup
+        if n.kind == "lstm":
+            steps = (self.in_shape if n.inputs[0] < 0 else self.shapes()[n.inputs[0]])[1]
+            return steps * n.cout * 4 * (n.cin + n.cout)
         return h * w * c * (n.kh * n.kw * n.cin if n.kind == "conv" else n.cin)
 
 
@@ -170,6 +182,30 @@ class _Builder:
     def maxpool(self, x, k=2, stride=2):
         h, w, c = self.shape[x]
         return self._add(Node("maxpool", (x,), "none", k, k, stride), ((h - k) // stride + 1, (w - k) // stride + 1, c))
+
+    def embed(self, x, vocab, dim):
+        """Keras Embedding initialiser: U(-0.05, 0.05); stored channel-major."""
+        h, w, _ = self.shape[x]
+        W = self.rng.uniform(-0.05, 0.05, size=(dim, vocab)).astype(np.float32)
+        return self._add(Node("embed", (x,), "none", 1, 1, 1, 0, vocab, dim, W, None), (h, w, dim))
+
+    def lstm(self, x, units, sequences):
+        """Keras LSTM initialisers: Glorot-uniform input weights, orthogonal recurrent
+        weights, forget-gate bias 1; the other biases ~ U(-0.05, 0.05) so that every
+        bias path is exercised."""
+        _, T, c = self.shape[x]
+        lim = np.sqrt(6.0 / (c + 4 * units))
+        Wx = self.rng.uniform(-lim, lim, size=(c, 4 * units))
+        q, r = np.linalg.qr(self.rng.standard_normal((4 * units, units)))
+        Wh = (q * np.sign(np.diag(r))).T                        # [units][4 units], orthonormal rows
+        W = np.zeros((units, 4, c + units), np.float32)
+        for g in range(4):
+            W[:, g, :c] = Wx[:, g * units:(g + 1) * units].T
+            W[:, g, c:] = Wh[:, g * units:(g + 1) * units].T
+        b = self.rng.uniform(-0.05, 0.05, size=(units, 4)).astype(np.float32)
+        b[:, 1] = 1.0
+        return self._add(Node("lstm", (x,), "none", 1 if sequences else 0, 1, 1, 0, c, units, W, b),
+                         (1, T if sequences else 1, units))
 
     def flatten(self, x):
         h, w, c = self.shape[x]
@@ -289,14 +325,36 @@ def mobilenetv2_tiny(seed=0):
     return bld.m
 
 
+def rnn(seed=0, n_classes=2, vocab=20000, dim=128, units=(64, 64), steps=80, name="rnn_imdb"):
+    """The paper's RNN family (Sec. 5.3, Table 1): embedding, two LSTM layers (the
+    first returns every step), dense output.  Vocabulary 20,000, width 128 and 64
+    units per LSTM give exactly Table 1's sizes: 2,642,562 parameters with 2 classes
+    (IMDB) and 2,648,282 with 90 (Reuters).  Sequences of `steps` tokens.  Oracle
+    only: the GPU library has no recurrent layer yet."""
+    bld = _Builder(name, (1, steps, 1), n_classes, seed)
+    x = bld.embed(-1, vocab, dim)
+    x = bld.lstm(x, units[0], sequences=True)
+    for u in units[1:-1]:
+        x = bld.lstm(x, u, sequences=True)
+    x = bld.lstm(x, units[-1], sequences=False)
+    bld.dense(x, n_classes, act="none")
+    return bld.m
+
+
+def rnn_reuters(seed=0):
+    return rnn(seed, n_classes=90, name="rnn_reuters")
+
+
 MODELS = {"mlp": mlp, "lenet5": lenet5, "vgg": vgg, "resnet20": resnet20, "resnet10": resnet10,
-          "mobilenetv2_tiny": mobilenetv2_tiny}
+          "mobilenetv2_tiny": mobilenetv2_tiny, "rnn_imdb": rnn, "rnn_reuters": rnn_reuters}
 
 
 # ------------------------------------------------------------------- inputs --
 
 def inputs(model: Model, n: int, seed: int = 1, dist: str | None = None) -> np.ndarray:
     """n inputs of the model's shape, [n][H][W][C] float32."""
+    if model.nodes and model.nodes[0].kind == "embed":
+        return token_sequences(model, n, seed)
     if dist is None:
         dist = "uniform" if model.in_shape[2] == 1 else "normal"
     rng = np.random.default_rng(seed)
@@ -304,6 +362,22 @@ def inputs(model: Model, n: int, seed: int = 1, dist: str | None = None) -> np.n
     if dist == "uniform":
         return rng.random(shape, dtype=np.float32)
     return rng.standard_normal(shape, dtype=np.float32)
+
+
+def token_sequences(model: Model, n: int, seed: int = 1) -> np.ndarray:
+    """n token sequences for a model that starts with an embedding (IMDB / Reuters
+    stand-ins), [n][1][T][1] float32 holding integer ids: review lengths
+    ~ lognormal (median T / 2) clipped to [8, T], word ids 1 + Zipf(1.3) clipped to the
+    vocabulary (word frequencies in text are heavy-tailed), pre-padded with id 0 as
+    Keras' pad_sequences does."""
+    rng = np.random.default_rng(seed)
+    T, V = model.in_shape[1], model.nodes[0].cin
+    out = np.zeros((n, 1, T, 1), np.float32)
+    for t in range(n):
+        length = int(np.clip(np.round(np.exp(rng.normal(np.log(T / 2), 0.6))), min(8, T), T))
+        ids = np.minimum(rng.zipf(1.3, size=length), V - 1)
+        out[t, 0, T - length:, 0] = ids
+    return out
 
 
 # ------------------------------------------------------------------ mutants --
