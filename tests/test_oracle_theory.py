@@ -72,6 +72,31 @@ def test_cost_accounting_lemma4(oracle_mod):
     assert van - memo == saving >= 0
 
 
+def _lemma4_gain(oracle_mod, model, table):
+    """1 - memo / vanilla in MACs: memo computes each group's prefix once and every
+    mutant's suffix from its first mutated layer on; vanilla runs every mutant whole."""
+    macs = [oracle_mod.node_macs(model, v) for v in range(len(model.nodes))]
+    L = model.layers()
+    counts = np.bincount(table.layer, minlength=len(L))
+    memo = sum(sum(macs[:L[l]]) + c * sum(macs[L[l]:]) for l, c in enumerate(counts) if c)
+    return 1.0 - memo / (len(table) * sum(macs))
+
+
+@pytest.mark.parametrize("name", ["lenet5", "mlp"])
+def test_modelwide_ratio_trend(oracle_mod, name):
+    """RQ2 (Sec. 5.5): with neurons drawn over the whole model, a larger selection ratio
+    moves the first mutated layer earlier and shrinks the shared prefix, so the gain
+    falls as the ratio grows (1 %, 3 %, 5 %)."""
+    m = wl.MODELS[name](0)
+    tables = [wl.modelwide_mutants(m, 400, seed=2, ratio=r) for r in (0.01, 0.03, 0.05)]
+    first = [float(np.mean(t.layer)) for t in tables]
+    gains = [_lemma4_gain(oracle_mod, m, t) for t in tables]
+    assert first[0] > first[1] >= first[2]
+    assert gains[0] > gains[1] >= gains[2] >= 0.0
+    if name == "lenet5":
+        assert gains[0] > gains[1] > gains[2] > 0.3
+
+
 def test_identity_mutants_never_killed(oracle_mod):
     w = wl.workload("lenet5", 64, 1)
     m = w.model
