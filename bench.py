@@ -45,6 +45,10 @@ WORKLOAD_TEXT = {
     "lenet5_modelwide": "LeNet-5 28x28x1, 10,000 inputs U[0,1], 2,000 mutants over several layers: 1% of all 236 "
                         "neurons drawn model-wide per mutant (tagged descriptors), GF/NEB/NAI/NS",
     "mlp_modelwide": "MLP 784-128-64-10, 1,000 inputs U[0,1], 200 mutants, 1% of all neurons drawn model-wide",
+    "lenet5_modelwide_3": "LeNet-5 28x28x1, 10,000 inputs U[0,1], 2,000 mutants over several layers: 3% of all 236 "
+                          "neurons (7) drawn model-wide per mutant, GF/NEB/NAI/NS",
+    "lenet5_modelwide_5": "LeNet-5 28x28x1, 10,000 inputs U[0,1], 2,000 mutants over several layers: 5% of all 236 "
+                          "neurons (12) drawn model-wide per mutant, GF/NEB/NAI/NS",
 }
 
 

@@ -543,6 +543,9 @@ CONFIGS = {
     "vgg_stress": ("vgg", 20000, 20000, (0.001, 0.01, 0.05, 0.10), 0.5),
     # model-wide selection: each mutant's neurons drawn over all layers (1 % of them)
     "lenet5_modelwide": ("lenet5", 10000, 2000, (0.01,), "model"),
+    # the paper's RQ2 ratios (Sec. 5.5): 3 % and 5 % of all neurons per mutant
+    "lenet5_modelwide_3": ("lenet5", 10000, 2000, (0.03,), "model"),
+    "lenet5_modelwide_5": ("lenet5", 10000, 2000, (0.05,), "model"),
     "mlp_modelwide": ("mlp", 1000, 200, (0.01,), "model"),
 }
 

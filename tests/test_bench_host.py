@@ -59,7 +59,7 @@ def test_hbm_rates_arithmetic():
     assert out["output_layer"]["achieved"] == pytest.approx(exp)
 
 
-@pytest.mark.parametrize("name", ["lenet5", "lenet5_modelwide"])
+@pytest.mark.parametrize("name", ["lenet5", "lenet5_modelwide", "lenet5_modelwide_5"])
 def test_oracle_sample_is_stratified(name):
     w = wl.workload(name, 50, 400)
     sub, X, idx = bench.oracle_sample(w, 40, 20, with_index=True)

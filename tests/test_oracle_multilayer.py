@@ -118,7 +118,8 @@ def test_per_layer_materialisation(oracle_mod):
         assert not blk.any()
 
 
-@pytest.mark.parametrize("name,n_in,n_mut", [("lenet5_modelwide", 16, 40), ("mlp_modelwide", 24, 40)])
+@pytest.mark.parametrize("name,n_in,n_mut", [("lenet5_modelwide", 16, 40), ("mlp_modelwide", 24, 40),
+                                            ("lenet5_modelwide_5", 12, 40)])
 def test_theorem1_memo_equals_vanilla_modelwide(oracle_mod, name, n_in, n_mut):
     w = wl.workload(name, n_in, n_mut)
     assert (w.table.tagged == 1).all()
