@@ -199,6 +199,18 @@ const char *mure_last_error(const mure_ctx *ctx);
 mure_status mure_model_load(mure_ctx *ctx, const mure_model_desc *desc, mure_model **out);
 void mure_model_free(mure_model *model);
 
+/* Validate a network description and a mutant table on the host, without a context
+ * or a device: the checks mure_model_load runs on `desc` (its compilation into
+ * stages included) and those mure_eval_mutants / mure_eval_vanilla run on the table
+ * before any launch (Algorithm 1's inputs: every mutant's layer, operator, neuron
+ * range, NS pairing, repeated neurons, and for tagged descriptors each entry's
+ * layer and the smallest-layer rule).  n_mutants = 0 checks the description alone.
+ * Every pointer is the caller's and is only read.  Returns OK, INVALID_ARG or
+ * UNSUPPORTED; when msg != NULL the one-line reason ("" on success) is written there,
+ * NUL-terminated and cut to msg_len bytes. */
+mure_status mure_check_descriptors(const mure_model_desc *desc, const mure_mutant *table, int64_t n_mutants,
+                                   const int32_t *neuron_pool, int64_t pool_len, char *msg, size_t msg_len);
+
 /* Kernels this context has launched since it was created (all calls). */
 int64_t mure_kernel_launches(const mure_ctx *ctx);
 

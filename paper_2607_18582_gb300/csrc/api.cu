@@ -1269,15 +1269,26 @@ void mure_destroy(mure_ctx *ctx)
 
 const char *mure_last_error(const mure_ctx *ctx) { return ctx ? ctx->err.c_str() : "NULL context"; }
 
+namespace {
+
+// The checks of a network description's header (before its nodes are compiled).
+void check_desc(mure_ctx *c, const mure_model_desc *d)
+{
+    FAILIF(!d || !d->nodes || d->n_nodes < 1, c, MURE_ERR_INVALID_ARG, "NULL model description");
+    FAILIF(d->in_h < 1 || d->in_w < 1 || d->in_c < 1, c, MURE_ERR_INVALID_ARG, "bad input shape");
+    FAILIF(d->precision != MURE_PREC_FP32 && d->precision != MURE_PREC_TF32X3 && d->precision != MURE_PREC_TF32,
+           c, MURE_ERR_UNSUPPORTED, "precision %d is not available", d->precision);
+}
+
+}  // namespace
+
 mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **out)
 {
     if (!c) return MURE_ERR_INVALID_ARG;
     return run(c, [&] {
-        FAILIF(!d || !out || !d->nodes || d->n_nodes < 1, c, MURE_ERR_INVALID_ARG, "NULL model description");
+        FAILIF(!out, c, MURE_ERR_INVALID_ARG, "NULL output handle");
         *out = nullptr;
-        FAILIF(d->in_h < 1 || d->in_w < 1 || d->in_c < 1, c, MURE_ERR_INVALID_ARG, "bad input shape");
-        FAILIF(d->precision != MURE_PREC_FP32 && d->precision != MURE_PREC_TF32X3 && d->precision != MURE_PREC_TF32,
-               c, MURE_ERR_UNSUPPORTED, "precision %d is not available", d->precision);
+        check_desc(c, d);
         CK(c, cudaSetDevice(c->device));
         auto *m = new mure_model();
         m->ctx = c;
@@ -1478,6 +1489,21 @@ mure_status mure_eval_vanilla(mure_model *m, const float *X, int64_t n_inputs, c
         evaluate(c, m, ca, table, n_mutants, neuron_pool, pool_len, true,
                  Outputs{kill_bits, score_killed_frac, score_deepmutation, stats, opts});
     });
+}
+
+mure_status mure_check_descriptors(const mure_model_desc *d, const mure_mutant *table, int64_t n_mutants,
+                                   const int32_t *neuron_pool, int64_t pool_len, char *msg, size_t msg_len)
+{
+    // host state only: the error text and the compiled stages (no device is touched)
+    mure_ctx c;
+    mure_model m;
+    const mure_status st = run(&c, [&] {
+        check_desc(&c, d);
+        compile(&c, d, &m);
+        check_table(&c, &m, table, n_mutants, neuron_pool, pool_len);
+    });
+    if (msg && msg_len > 0) snprintf(msg, msg_len, "%s", c.err.c_str());
+    return st;
 }
 
 mure_status mure_expand_patches(mure_model *m, const mure_mutant *table, int64_t n_mutants, const int32_t *neuron_pool,

@@ -25,7 +25,8 @@ PRECISIONS = {"fp32": 0, "tf32x3": 1, "bf16": 2, "tf32": 3}
 # the exported entry points of include/mure.h
 EXPORTS = ("mure_create", "mure_destroy", "mure_last_error", "mure_model_load", "mure_model_free",
            "mure_model_n_layers", "mure_model_layer_kernel", "mure_kernel_launches", "mure_build_prefix_cache", "mure_cache_free", "mure_cache_outputs",
-           "mure_eval_mutants", "mure_eval_vanilla", "mure_expand_patches", "mure_expand_patches_noalloc")
+           "mure_eval_mutants", "mure_eval_vanilla", "mure_expand_patches", "mure_expand_patches_noalloc",
+           "mure_check_descriptors")
 
 
 class MureError(RuntimeError):
@@ -120,6 +121,7 @@ def lib():
                                         C.POINTER(C.c_double), C.POINTER(C.c_double), C.POINTER(_Stats)]
         L.mure_expand_patches.argtypes = [vp, vp, i64, vp, i64, vp, i64, vp]
         L.mure_expand_patches_noalloc.argtypes = [vp, vp, i64, vp, i64, vp, i64, vp]
+        L.mure_check_descriptors.argtypes = [C.POINTER(_ModelDesc), vp, i64, vp, i64, C.c_char_p, C.c_size_t]
         for name in EXPORTS:
             if name not in ("mure_destroy", "mure_model_free", "mure_cache_free", "mure_last_error",
                             "mure_model_n_layers", "mure_kernel_launches"):
@@ -244,8 +246,8 @@ class Model:
             self._destroy()
 
 
-def mure_model_load(ctx: Context, model, precision: str = "fp32") -> Model:
-    """Copy a network description (workloads.Model fields) to the device."""
+def _model_desc(model, precision):
+    """The C description of a network (workloads.Model fields) and the arrays it points to."""
     nodes = (_Node * len(model.nodes))()
     keep = []
     for v, n in enumerate(model.nodes):
@@ -257,6 +259,12 @@ def mure_model_load(ctx: Context, model, precision: str = "fp32") -> Model:
                          _ptr(W), _ptr(b))
     h, w, c = model.in_shape
     desc = _ModelDesc(h, w, c, model.n_classes, len(model.nodes), PRECISIONS[precision], nodes)
+    return desc, (keep, nodes)
+
+
+def mure_model_load(ctx: Context, model, precision: str = "fp32") -> Model:
+    """Copy a network description (workloads.Model fields) to the device."""
+    desc, keep = _model_desc(model, precision)
     out = C.c_void_p()
     ctx.check(lib().mure_model_load(ctx.h, C.byref(desc), C.byref(out)))
     return Model(ctx, out.value, model)
@@ -410,3 +418,15 @@ def mure_expand_patches_noalloc(model: Model, table, out_dev):
     model.ctx.check(lib().mure_expand_patches_noalloc(model.h, _ptr(arr), n, _ptr(pool), plen, _ptr(out_dev),
                                                       int(out_dev.numel()), _ptr(offs)))
     return offs[:n]
+
+
+def mure_check_descriptors(model, table=None, precision: str = "fp32"):
+    """Host-side validation of a network description and (optionally) a mutant table,
+    with no context and no device: (status, reason); status 0 = MURE_OK."""
+    desc, keep = _model_desc(model, precision)
+    arr, pool, plen = table_array(table) if table is not None else (None, None, 0)
+    n = len(table) if table is not None else 0
+    msg = C.create_string_buffer(512)
+    st = lib().mure_check_descriptors(C.byref(desc), _ptr(arr) if n else None, n,
+                                      _ptr(pool) if plen else None, plen, msg, 512)
+    return int(st), msg.value.decode()
