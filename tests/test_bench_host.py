@@ -71,3 +71,26 @@ def test_oracle_sample_is_stratified(name):
             a, n = int(w.table.neuron_off[i]), int(w.table.n_neurons[i])
             b = int(sub.neuron_off[j])
             assert np.array_equal(sub.pool[b:b + n], w.table.pool[a:a + n])
+
+
+@pytest.mark.timeout(600)
+def test_reference_arm_line_single_rank():
+    """`bench.py --impl reference` at N = 1: one JSON line with every key of the
+    contract; the oracle is timed on the host cores with no device copies."""
+    import json
+    import subprocess
+    p = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--steps", "1", "--warmup", "3",
+                        "--workload", "mlp"], cwd=ROOT, capture_output=True, text=True, timeout=580)
+    assert p.returncode == 0, p.stderr[-2000:]
+    lines = [l for l in p.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+              "vs_baseline", "dtype", "data", "config", "e2e", "cpu_baseline", "impl"):
+        assert k in d, k
+    assert d["impl"] == "reference" and d["n_gpus"] == 1 and d["steps"] == 1 and d["warmup"] == 3
+    assert d["value"] > 0 and d["higher_is_better"] is True and d["vs_baseline"] is None
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
+    assert d["config"]["workload"].startswith("mlp")
