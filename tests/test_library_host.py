@@ -134,3 +134,42 @@ def test_reason_fits_the_buffer():
     # a NULL buffer is allowed; a NULL description is an argument error
     assert mure.lib().mure_check_descriptors(ctypes.byref(desc), None, 0, None, 0, None, 0) == OK
     assert mure.lib().mure_check_descriptors(None, None, 0, None, 0, None, 0) == INVALID
+
+
+def _corrupt_model(model, rng):
+    """A copy of the network with one geometry field of one node changed."""
+    m = wl.Model(model.name, model.in_shape, model.n_classes,
+                 [wl.Node(n.kind, n.inputs, n.act, n.kh, n.kw, n.stride, n.pad, n.cin, n.cout, n.W, n.b)
+                  for n in model.nodes])
+    v = int(rng.integers(len(m.nodes)))
+    n = m.nodes[v]
+    field = str(rng.choice(["kh", "kw", "stride", "pad", "cin", "cout", "inputs", "n_classes"]))
+    if field == "inputs":
+        n.inputs = (int(rng.integers(-1, len(m.nodes))),) + tuple(n.inputs[1:])
+    elif field == "n_classes":
+        m.n_classes = int(rng.choice([model.n_classes - 1, model.n_classes + 1]))
+    else:
+        setattr(n, field, max(-1, getattr(n, field) + int(rng.choice([-2, -1, 1, 3]))))
+    return m
+
+
+@pytest.mark.parametrize("name", ["lenet5", "resnet20", "mlp"])
+def test_description_checks_cover_the_oracles(oracle_mod, name):
+    """A description the oracle's graph checks refuse is refused by the library too
+    (the library also refuses supported-shape violations the oracle can run)."""
+    base = wl.MODELS[name](0)
+    rng = np.random.default_rng(5)
+    refused_by_oracle = 0
+    for _ in range(80):
+        m = _corrupt_model(base, rng)
+        try:
+            sh = oracle_mod.OModel(m).shapes()
+            oracle_ok = int(np.prod(sh[-1])) == m.n_classes
+        except oracle_mod.OracleError:
+            oracle_ok = False
+        st, msg = mure.mure_check_descriptors(m)
+        if not oracle_ok:
+            refused_by_oracle += 1
+            assert st != OK, msg
+        assert (msg == "") == (st == OK)
+    assert refused_by_oracle >= 10
