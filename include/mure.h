@@ -214,6 +214,20 @@ mure_status mure_check_descriptors(const mure_model_desc *desc, const mure_mutan
 /* Kernels this context has launched since it was created (all calls). */
 int64_t mure_kernel_launches(const mure_ctx *ctx);
 
+/* Limit of the device-side waits of this context's tensor-core kernels, in SM clock
+ * cycles (0, the initial value, restores the default of 2e9 cycles, about a second at
+ * the SM clock).  The paper has no counterpart: this is failure detection.  Every
+ * wait of a role of those kernels (for operand copies, MMAs, tensor-memory stages or
+ * accumulators) gives up after the limit; the kernel then stops all its roles, lets
+ * its own copies and MMAs in flight land (those teardown waits keep the default limit
+ * whatever this setting), frees its tensor memory and returns, and the call that
+ * launched it returns TIMEOUT with the context still usable (that call's output
+ * buffers are then undefined).  A limit far below the
+ * kernels' normal waits makes calls fail on purpose (a test of that path).  Applies
+ * to launches queued after this call.  Errors: INVALID_ARG (NULL context, negative
+ * limit). */
+mure_status mure_set_wait_limit(mure_ctx *ctx, int64_t cycles);
+
 /* Number of weighted layers L of a loaded model (or -1 for NULL). */
 int32_t mure_model_n_layers(const mure_model *model);
 
@@ -303,14 +317,20 @@ mure_status mure_expand_patches(mure_model *model, const mure_mutant *table, int
  *             values as mure_expand_patches, i.e. GF noise and WS-permuted weights);
  *   offsets   host [n_mutants]: offset of each mutant's first slot in out_dev, -1 for
  *             operators without a patch.
- * The first call on a device looks up the array's device address with that device
- * current; make that first call before any stream capture on the device.  Every call
- * shares the one array: calls whose device work overlaps (on different streams or
- * host threads) race and must not be issued.  The kernel initialises every scratch
- * entry it reads, so nothing carries over from an earlier call.  The call returns when
- * the patches are in out_dev.  Errors: INVALID_ARG (descriptors as in
- * mure_eval_mutants, untagged only; out_len too small; descriptors needing more than the 8 MiB of
- * scratch, with the needed size in mure_last_error), CUDA. */
+ * The first call on a device that has work to do looks up the array's device address
+ * with that device current (a failed lookup is retried by the next call).  The call
+ * copies its job table from pageable host memory and waits for the context's stream,
+ * so it must never be issued while that stream, or any stream of the device, is being
+ * captured into a CUDA graph; it returns INVALID_ARG when it finds the context's stream
+ * capturing.  Every call shares the one array: calls whose device work overlaps (on
+ * different streams or host threads) race and must not be issued.  The kernel
+ * initialises every scratch entry it reads, so nothing carries over from an earlier
+ * call.  The call returns when the patches are in out_dev.  Errors: the descriptor
+ * checks of mure_eval_mutants with their status codes; UNSUPPORTED for tagged
+ * descriptors (as mure_expand_patches); INVALID_ARG for out_len too small (the needed
+ * count in mure_last_error), for descriptors needing more than the 8 MiB of scratch
+ * (the needed size in mure_last_error) and for a capturing stream; OOM when a host
+ * allocation fails; CUDA. */
 mure_status mure_expand_patches_noalloc(mure_model *model, const mure_mutant *table, int64_t n_mutants,
                                         const int32_t *neuron_pool, int64_t pool_len, float *out_dev,
                                         int64_t out_len, int64_t *offsets);

@@ -1225,6 +1225,16 @@ mure_cache *build_cache(mure_model *m, const float *X, int64_t n_in, const int32
 
 // ====================================================================== ABI ==
 
+namespace mure {
+
+mure_status check_table_status(mure_ctx *c, const mure_model *m, const mure_mutant *t, int64_t n, const int32_t *pool,
+                               int64_t pool_len)
+{
+    return run(c, [&] { check_table(c, m, t, n, pool, pool_len); });
+}
+
+}  // namespace mure
+
 extern "C" {
 
 mure_status mure_create(int device, void *cuda_stream, const mure_allocator *alloc, mure_ctx **out)
@@ -1310,6 +1320,7 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             S.variant = (force && force[0] == '1') ? 0 : conv_small_variant(S);
             S.geo = S.variant;
             S.err = c->err_dev;
+            S.wait_limit = &c->wait_limit;
         }
         // tensor-core modes: layers before the output layer with >= 16 outputs run on
         // the tensor cores (3xTF32, or one TF32 MMA in the reduced-precision variant);
@@ -1415,6 +1426,18 @@ mure_status mure_model_layer_kernel(const mure_model *m, int32_t layer, int32_t 
 }
 
 int64_t mure_kernel_launches(const mure_ctx *ctx) { return ctx ? ctx->launches : -1; }
+
+mure_status mure_set_wait_limit(mure_ctx *ctx, int64_t cycles)
+{
+    if (!ctx) return MURE_ERR_INVALID_ARG;
+    ctx->err.clear();
+    if (cycles < 0) {
+        ctx->err = "negative wait limit";
+        return MURE_ERR_INVALID_ARG;
+    }
+    ctx->wait_limit = cycles;
+    return MURE_OK;
+}
 
 mure_status mure_build_prefix_cache(mure_model *m, const float *X, int64_t n_inputs, const int32_t *labels,
                                     int x_on_device, mure_cache **out)

@@ -37,6 +37,7 @@ struct Stage {
     int tc_small = 0;         // tc: the small-image convolution mode
     float *Wtc = nullptr;     // tc: TF32 halves of W in the tensor-core operand layout
     int *err = nullptr;       // device error word of the context (bounded waits)
+    const int64_t *wait_limit = nullptr;   // host: the context's wait limit (0 = default)
     float *W = nullptr;       // device [oc][K]
     float *Wt = nullptr;      // device [K][oc] (the same weights, K-major rows)
     float *b = nullptr;       // device [oc]
@@ -65,6 +66,7 @@ struct mure_ctx {
     int n_sms = 0;
     int64_t launches = 0;             // kernels launched since creation
     int *err_dev = nullptr;           // device error word written by bounded waits
+    int64_t wait_limit = 0;           // limit of the device-side waits in SM cycles (0 = default)
 };
 
 struct mure_model {
@@ -250,6 +252,11 @@ int launch_patch_dot(const Stage &S, Src z, Src x, RowMap rm, const PatchArgs &p
 // Materialise rows: out = base rows with the overlay applied.
 int launch_rows_overlay(Src base, int64_t n_floats, RowMap rm, const Overlay &ov, float *out, int64_t out_stride,
                         cudaStream_t s);
+
+// The descriptor checks of mure_eval_mutants (status and last-error text), for entry
+// points outside the scheduler.
+mure_status check_table_status(mure_ctx *c, const mure_model *m, const mure_mutant *t, int64_t n, const int32_t *pool,
+                               int64_t pool_len);
 
 // Expand GF / WS descriptors into patches (see mure_expand_patches): one job per
 // (mutant, neuron slot).

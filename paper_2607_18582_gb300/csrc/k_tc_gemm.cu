@@ -51,7 +51,14 @@ constexpr int kThreads = 384;          // 4 producer + 4 epilogue + 3 MMA + weig
 constexpr int kEpiStride = 36;         // floats per row of an epilogue staging chunk (32 + pad)
 constexpr int kMaxNT = 8;              // tensor-memory A stages, at most
 constexpr uint32_t kStageA = kTileM * 128;   // bytes of one producer ring slot
-constexpr long long kSpin = 2000000000LL;    // about a second at the SM clock
+constexpr long long kSpin = 2000000000LL;    // default wait limit: about a second at the SM clock
+
+// The CTA's abort state: set by the role whose wait ran out (after `limit` cycles), seen
+// by every other role's waits.
+struct WaitCtl {
+    int abort;
+    long long limit;
+};
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
 {
@@ -128,31 +135,33 @@ __device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity)
 
 // Wait for the phase of parity `parity`, polling every ~NS nanoseconds (a sleeping
 // warp leaves the issue slots of its SM sub-partition to the producers); false when
-// another role has aborted or about a second has passed (then this role aborts the
+// another role has aborted or the wait limit has passed (then this role aborts the
 // CTA).
 template <int NS = 0>
-__device__ __forceinline__ bool wait_phase(uint32_t a, uint32_t parity, volatile int *abort_flag)
+__device__ __forceinline__ bool wait_phase(uint32_t a, uint32_t parity, volatile WaitCtl *abort_flag)
 {
     if (mbar_try(a, parity)) return true;
     const long long t0 = clock64();
     for (;;) {
         if (NS > 0) __nanosleep(NS);
         if (mbar_try(a, parity)) return true;
-        if (*abort_flag) return false;
-        if (clock64() - t0 > kSpin) { *abort_flag = 1; return false; }
+        if (abort_flag->abort) return false;
+        if (clock64() - t0 > abort_flag->limit) { abort_flag->abort = 1; return false; }
     }
 }
 
 // The same for a whole warp: every lane polls, the verdict is the warp's AND, so the
 // .sync.aligned tensor-memory instructions that follow see a converged warp.
 template <int NS = 0>
-__device__ __forceinline__ bool warp_wait_phase(uint32_t a, uint32_t parity, volatile int *abort_flag)
+__device__ __forceinline__ bool warp_wait_phase(uint32_t a, uint32_t parity, volatile WaitCtl *abort_flag)
 {
     const bool ok = wait_phase<NS>(a, parity, abort_flag);
     return __all_sync(0xffffffffu, ok);
 }
 
-// Teardown wait: bounded, ignores the abort flag.
+// Teardown wait: bounded by the default limit whatever the CTA's limit, ignores the
+// abort flag, so that copies and MMAs in flight land before shared and tensor memory
+// are released.
 __device__ __forceinline__ void wait_phase_drain(uint32_t a, uint32_t parity)
 {
     const long long t0 = clock64();
@@ -270,6 +279,7 @@ struct TcParams {
     int n_stages;                // tensor-memory A stages (<= kMaxNT), from column a_col
     int a_col;
     int *err;
+    long long spin;              // wait limit in SM cycles (0: the default, about a second)
     FinalFuse ff;                // the output layer computed in the epilogue (FCP > 0)
     SlotStore slot;              // slot.out: the tensor-core delta's scattered store
     // dense layers: A tiles (128 rows x one K-step) by tensor-map copies from warp 10
@@ -568,11 +578,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     // dense A tiles by tensor-map copies: slot landed, slot read by the producers
     __shared__ __align__(8) uint64_t bar_alanded[kNA], bar_afree[kNA];
     __shared__ uint32_t tmem_sh;
-    __shared__ int abort_sh;
+    __shared__ WaitCtl abort_sh;
     __shared__ float bias_sh[kSlice];
     __shared__ __align__(16) float epi_stage[4][32 * kEpiStride];   // per epilogue warp: 32 rows x 32 values
     __shared__ float *epi_ptr[4][32];                               // per epilogue warp: each row's output
-    volatile int *abort_flag = &abort_sh;
+    volatile WaitCtl *abort_flag = &abort_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t sbase = (smem_u32(smraw) + 1023u) & ~1023u;
@@ -650,7 +660,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             mbar_init(smem_u32(&bar_ready[s]), 1);
             mbar_init(smem_u32(&bar_released[s]), 4);
         }
-        abort_sh = 0;
+        abort_sh.abort = 0;
+        abort_sh.limit = p.spin > 0 ? p.spin : kSpin;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -1239,7 +1250,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
-    if (threadIdx.x == 0 && abort_sh) atomicExch(p.err, MURE_ERR_TIMEOUT);
+    if (threadIdx.x == 0 && abort_sh.abort) atomicExch(p.err, MURE_ERR_TIMEOUT);
     if (warp == 0) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512));
@@ -1462,6 +1473,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     p.y_stride = S.gap ? map_stride : y_stride;
     if (ov) p.ov = *ov;
     p.err = S.err;
+    p.spin = S.wait_limit ? *S.wait_limit : 0;
     // shared memory: the weights (whole slice, or kNB K-steps), then the producer ring
     const int nt_max = std::min(kSlice, p.Np);
     const size_t b_step = (size_t)planes * nt_max * 128;

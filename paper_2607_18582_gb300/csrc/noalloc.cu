@@ -10,6 +10,7 @@
 #include <algorithm>
 #include <cstring>
 #include <mutex>
+#include <new>
 #include <vector>
 
 #include "common.cuh"
@@ -21,14 +22,11 @@ constexpr size_t kNoallocScratchBytes = size_t(8) << 20;  // 8 MiB
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
 
 // Host code cannot use &g_noalloc_scratch as a device address (it names a host-side
-// stand-in), so each device's address is looked up once, with that device current.
+// stand-in), so each device's address is looked up with that device current and kept
+// once the lookup has succeeded; a failed lookup is retried by the next call.
 constexpr int kMaxDevices = 256;
-struct DeviceScratch {
-    std::once_flag once;
-    cudaError_t err = cudaSuccess;
-    unsigned char *ptr = nullptr;
-};
-DeviceScratch g_scratch[kMaxDevices];
+std::mutex g_scratch_mu;
+unsigned char *g_scratch_ptr[kMaxDevices] = {};
 
 size_t align256(size_t n) { return (n + 255) & ~size_t(255); }
 
@@ -38,37 +36,24 @@ mure_status fail(mure_ctx *c, mure_status st, const std::string &msg)
     return st;
 }
 
-}  // namespace
-
-extern "C" mure_status mure_expand_patches_noalloc(mure_model *m, const mure_mutant *table, int64_t n_mutants,
-                                                   const int32_t *neuron_pool, int64_t pool_len, float *out_dev,
-                                                   int64_t out_len, int64_t *offsets)
+mure_status expand_noalloc(mure_ctx *c, mure_model *m, const mure_mutant *table, int64_t n_mutants,
+                           const int32_t *neuron_pool, int64_t pool_len, float *out_dev, int64_t out_len,
+                           int64_t *offsets)
 {
-    if (!m) return MURE_ERR_INVALID_ARG;
-    mure_ctx *c = m->ctx;
-    c->err.clear();
-    if (n_mutants < 0 || pool_len < 0 || (n_mutants > 0 && (!table || !offsets)) || (pool_len > 0 && !neuron_pool))
-        return fail(c, MURE_ERR_INVALID_ARG, "NULL table, pool or offsets, or a negative size");
+    // the descriptor checks of mure_eval_mutants, then the flat-layout rule of
+    // mure_expand_patches: the same status codes as the allocating entry point
+    const mure_status st = mure::check_table_status(c, m, table, n_mutants, neuron_pool, pool_len);
+    if (st != MURE_OK) return st;
+    for (int64_t i = 0; i < n_mutants; ++i)
+        if (table[i].tagged)
+            return fail(c, MURE_ERR_UNSUPPORTED,
+                        "mutant " + std::to_string(i) + ": tagged descriptors have no flat patch layout");
+    if (n_mutants > 0 && !offsets) return fail(c, MURE_ERR_INVALID_ARG, "NULL offsets");
     if (c->device < 0 || c->device >= kMaxDevices) return fail(c, MURE_ERR_UNSUPPORTED, "device id out of range");
 
-    // validate the descriptors and lay out one expansion job per (mutant, neuron slot)
+    // one expansion job per (mutant, neuron slot) of the GF / WS descriptors
     std::vector<mure::SlotJob> jobs;
     int64_t patch_len = 0, perm_len = 0;
-    for (int64_t i = 0; i < n_mutants; ++i) {
-        const mure_mutant &u = table[i];
-        if (u.layer < 0 || u.layer >= m->L || u.op < MURE_OP_GF || u.op > MURE_OP_IDENTITY || u.tagged != 0 ||
-            u.reserved2 != 0.f || u.n_neurons < 0 || u.neuron_off < 0 || u.neuron_off + u.n_neurons > pool_len ||
-            (u.op == MURE_OP_NS && (u.n_neurons & 1)))
-            return fail(c, MURE_ERR_INVALID_ARG, "invalid mutant descriptor " + std::to_string(i));
-        const int oc = m->st[u.layer].oc;
-        for (int q = 0; q < u.n_neurons; ++q) {
-            const int32_t j = neuron_pool[u.neuron_off + q];
-            if (j < 0 || j >= oc) return fail(c, MURE_ERR_INVALID_ARG, "neuron id out of range in mutant " + std::to_string(i));
-            for (int r = 0; r < q; ++r)
-                if (neuron_pool[u.neuron_off + r] == j)
-                    return fail(c, MURE_ERR_INVALID_ARG, "repeated neuron in mutant " + std::to_string(i));
-        }
-    }
     std::vector<int64_t> offs(n_mutants, -1);
     for (int64_t i = 0; i < n_mutants; ++i) {
         const mure_mutant &u = table[i];
@@ -102,12 +87,29 @@ extern "C" mure_status mure_expand_patches_noalloc(mure_model *m, const mure_mut
         return MURE_OK;
     }
 
-    cudaError_t e = cudaSetDevice(c->device);
+    // the call copies from pageable host memory and waits for its stream: neither is
+    // allowed while the stream is being captured into a graph
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(c->stream, &cap);
+    if (e != cudaSuccess) return fail(c, MURE_ERR_CUDA, std::string("cudaStreamIsCapturing: ") + cudaGetErrorString(e));
+    if (cap != cudaStreamCaptureStatusNone)
+        return fail(c, MURE_ERR_INVALID_ARG, "the context's stream is being captured");
+    e = cudaSetDevice(c->device);
     if (e != cudaSuccess) return fail(c, MURE_ERR_CUDA, std::string("cudaSetDevice: ") + cudaGetErrorString(e));
-    DeviceScratch &ds = g_scratch[c->device];
-    std::call_once(ds.once, [&] { ds.err = cudaGetSymbolAddress((void **)&ds.ptr, g_noalloc_scratch); });
-    if (ds.err != cudaSuccess || !ds.ptr)
-        return fail(c, MURE_ERR_CUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(ds.err));
+    unsigned char *scratch = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_scratch_mu);
+        if (!g_scratch_ptr[c->device]) {
+            void *p = nullptr;
+            e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+            if (e != cudaSuccess || !p) {
+                cudaGetLastError();
+                return fail(c, MURE_ERR_CUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
+            }
+            g_scratch_ptr[c->device] = static_cast<unsigned char *>(p);
+        }
+        scratch = g_scratch_ptr[c->device];
+    }
 
     // one host staging copy of the job table and weight pointers into the scratch
     std::vector<unsigned char> host(o_perm);
@@ -115,17 +117,17 @@ extern "C" mure_status mure_expand_patches_noalloc(mure_model *m, const mure_mut
     for (int l = 0; l < m->L; ++l) Wp[l] = m->st[l].W;
     memcpy(host.data() + o_w, Wp.data(), m->L * sizeof(float *));
     memcpy(host.data() + o_jobs, jobs.data(), jobs.size() * sizeof(mure::SlotJob));
-    e = cudaMemcpyAsync(ds.ptr, host.data(), o_perm, cudaMemcpyHostToDevice, c->stream);
+    e = cudaMemcpyAsync(scratch, host.data(), o_perm, cudaMemcpyHostToDevice, c->stream);
     if (e != cudaSuccess) return fail(c, MURE_ERR_CUDA, std::string("cudaMemcpyAsync: ") + cudaGetErrorString(e));
     mure::ExpandArgs ea{};
-    ea.jobs = reinterpret_cast<const mure::SlotJob *>(ds.ptr + o_jobs);
+    ea.jobs = reinterpret_cast<const mure::SlotJob *>(scratch + o_jobs);
     ea.n_jobs = (int64_t)jobs.size();
     ea.sigma = m->sigma_dev;
-    ea.W = reinterpret_cast<const float *const *>(ds.ptr + o_w);
+    ea.W = reinterpret_cast<const float *const *>(scratch + o_w);
     ea.patch = out_dev;
     // the kernel initialises every permutation entry it reads, so nothing in the
     // scratch has to start at zero or survives from an earlier call
-    ea.perm = reinterpret_cast<int32_t *>(ds.ptr + o_perm);
+    ea.perm = reinterpret_cast<int32_t *>(scratch + o_perm);
     ea.ws_as_weights = 1;
     c->launches += mure::launch_expand(ea, c->stream);
     e = cudaGetLastError();
@@ -133,4 +135,23 @@ extern "C" mure_status mure_expand_patches_noalloc(mure_model *m, const mure_mut
     if (e != cudaSuccess) return fail(c, MURE_ERR_CUDA, std::string("expansion: ") + cudaGetErrorString(e));
     std::copy(offs.begin(), offs.end(), offsets);
     return MURE_OK;
+}
+
+}  // namespace
+
+extern "C" mure_status mure_expand_patches_noalloc(mure_model *m, const mure_mutant *table, int64_t n_mutants,
+                                                   const int32_t *neuron_pool, int64_t pool_len, float *out_dev,
+                                                   int64_t out_len, int64_t *offsets)
+{
+    if (!m) return MURE_ERR_INVALID_ARG;
+    mure_ctx *c = m->ctx;
+    c->err.clear();
+    // host containers sized by the caller's table: a failed host allocation is a
+    // status, never an exception across the C ABI
+    try {
+        return expand_noalloc(c, m, table, n_mutants, neuron_pool, pool_len, out_dev, out_len, offsets);
+    } catch (const std::bad_alloc &) {
+        c->err = "host allocation failed";
+        return MURE_ERR_OOM;
+    }
 }

@@ -26,7 +26,7 @@ PRECISIONS = {"fp32": 0, "tf32x3": 1, "bf16": 2, "tf32": 3}
 EXPORTS = ("mure_create", "mure_destroy", "mure_last_error", "mure_model_load", "mure_model_free",
            "mure_model_n_layers", "mure_model_layer_kernel", "mure_kernel_launches", "mure_build_prefix_cache", "mure_cache_free", "mure_cache_outputs",
            "mure_eval_mutants", "mure_eval_vanilla", "mure_expand_patches", "mure_expand_patches_noalloc",
-           "mure_check_descriptors")
+           "mure_check_descriptors", "mure_set_wait_limit")
 
 
 class MureError(RuntimeError):
@@ -122,6 +122,7 @@ def lib():
         L.mure_expand_patches.argtypes = [vp, vp, i64, vp, i64, vp, i64, vp]
         L.mure_expand_patches_noalloc.argtypes = [vp, vp, i64, vp, i64, vp, i64, vp]
         L.mure_check_descriptors.argtypes = [C.POINTER(_ModelDesc), vp, i64, vp, i64, C.c_char_p, C.c_size_t]
+        L.mure_set_wait_limit.argtypes = [vp, i64]
         for name in EXPORTS:
             if name not in ("mure_destroy", "mure_model_free", "mure_cache_free", "mure_last_error",
                             "mure_model_n_layers", "mure_kernel_launches"):
@@ -391,6 +392,11 @@ def mure_eval_vanilla(model: Model, X, table, labels=None, logits: bool = False,
 def mure_kernel_launches(ctx: Context) -> int:
     """Kernels the context has launched since it was created."""
     return int(lib().mure_kernel_launches(ctx.h))
+
+
+def mure_set_wait_limit(ctx: Context, cycles: int) -> None:
+    """Limit of the tensor-core kernels' device-side waits in SM cycles (0: default)."""
+    ctx.check(lib().mure_set_wait_limit(ctx.h, int(cycles)))
 
 
 def mure_expand_patches(model: Model, table):

@@ -284,12 +284,14 @@ def test_device_inputs_and_outputs(M, ctx):
 
 
 @pytest.mark.slow
-def test_full_size_lenet_sampled(M, ctx, oracle_mod):
-    """The benchmark's configuration (LeNet-5, 10,000 inputs, 2,000 mutants, one
-    batch geometry as the benchmark runs it), checked on a sample of mutants x
-    inputs that the oracle computes one by one."""
+@pytest.mark.parametrize("prec", PRECISIONS)
+def test_full_size_lenet_sampled(M, ctx, oracle_mod, prec):
+    """The LeNet-5 configuration at full size (10,000 inputs, 2,000 mutants, one
+    batch geometry as the benchmark runs it) in both fp32-level modes (CUDA-core fp32
+    chains and the benchmarked 3xTF32 tensor-core path), checked on a sample of
+    mutants x inputs that the oracle computes one by one."""
     w = wl.workload("lenet5")
-    model = M.mure_model_load(ctx, w.model)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
     cache = M.mure_build_prefix_cache(model, w.X)
     r = M.mure_eval_mutants(cache, w.table)
     rng = np.random.default_rng(0)

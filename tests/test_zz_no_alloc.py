@@ -59,3 +59,28 @@ def test_noalloc_rejects_tables_beyond_its_scratch(M):
     with pytest.raises(M.MureError) as ei:
         M.mure_expand_patches_noalloc(model, table, out)
     assert ei.value.status == 1 and "scratch" in str(ei.value)
+
+
+def test_noalloc_short_output_and_tables_without_patches(M):
+    """An output buffer one value short is refused with the needed count (nothing is
+    launched); a table whose operators have no patch (NEB, NS, NAI, IDENTITY) returns
+    offsets of -1 without touching the device; a tagged table is refused as the
+    allocating entry point refuses it."""
+    import torch
+    ctx = M.mure_create(0)
+    model = M.mure_model_load(ctx, wl.lenet5())
+    table = _table(model.src, 3)
+    ref_vals, _ = M.mure_expand_patches(model, table)
+    out = torch.zeros(ref_vals.size - 1, dtype=torch.float32, device="cuda")
+    with pytest.raises(M.MureError) as ei:
+        M.mure_expand_patches_noalloc(model, table, out)
+    assert ei.value.status == 1 and "needed" in str(ei.value)
+    rows = [(l, op, [0, 1] if op == "NS" else [0], 0.0, 0)
+            for l in range(model.src.n_layers()) for op in ("NEB", "NS", "NAI", "IDENTITY")]
+    rows = [(l, op, [] if op == "IDENTITY" else ids, p, s) for l, op, ids, p, s in rows]
+    offs = M.mure_expand_patches_noalloc(model, wl.table_from_rows(rows), out)
+    assert offs.tolist() == [-1] * len(rows)
+    tagged = wl.workload("lenet5_modelwide", 1, 4).table
+    with pytest.raises(M.MureError) as ei:
+        M.mure_expand_patches_noalloc(model, tagged, out)
+    assert ei.value.status == 2
