@@ -239,6 +239,8 @@ int32_t mure_model_n_layers(const mure_model *model);
  *   MURE_KERNEL_TC_GEMM      tensor-core GEMM / implicit-GEMM convolution
  *   MURE_KERNEL_TC_WINDOW    tensor-core GEMM over 2x2 pooling windows
  *   MURE_KERNEL_OUTPUT       output layer with the fused argmax / kill epilogue
+ *   MURE_KERNEL_TC_CONV      tensor-core convolution over input rows staged in shared
+ *                            memory (stride 1, input channels a multiple of 32)
  * macs_per_row counts the GEMM as executed (padding and, for the window form, the
  * zero taps included; one product per MAC, whatever the precision mode).  Either
  * output pointer may be NULL.  Errors: INVALID_ARG (NULL model, layer out of range). */
@@ -247,7 +249,8 @@ typedef enum {
     MURE_KERNEL_SIMT_SMALL = 1,
     MURE_KERNEL_TC_GEMM = 2,
     MURE_KERNEL_TC_WINDOW = 3,
-    MURE_KERNEL_OUTPUT = 4
+    MURE_KERNEL_OUTPUT = 4,
+    MURE_KERNEL_TC_CONV = 5
 } mure_kernel;
 mure_status mure_model_layer_kernel(const mure_model *model, int32_t layer, int32_t *kernel, int64_t *macs_per_row);
 

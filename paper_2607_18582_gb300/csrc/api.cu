@@ -14,10 +14,12 @@ using namespace mure;
 
 namespace {
 
-// MURE_TC_CONV=1 puts every convolution of a TF32X3 model on the tensor cores.
 // MURE_TC_CONV: in the tensor-core modes the LeNet-size convolution runs in the
 // small-image mode (a GEMM row per pooling window); "0" keeps its CUDA-core kernel,
 // "generic" runs it through the implicit-GEMM producers (one row per position).
+// Stride-1 convolutions with input channels a multiple of 32 take the staged mode
+// (each tile's input rows staged in shared memory by tensor-map copies); "gather"
+// keeps them on the producers' per-row gathers from device memory.
 std::string tc_conv_env()
 {
     const char *e = getenv("MURE_TC_CONV");
@@ -1335,6 +1337,7 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             if (S.tc) {
                 S.variant = 0;
                 S.tc_small = small && env != "generic";
+                S.tc_conv = !S.tc_small && env != "gather" && tc_conv_geometry(S);
             }
         }
         std::vector<int> wn;
@@ -1415,7 +1418,7 @@ mure_status mure_model_layer_kernel(const mure_model *m, int32_t layer, int32_t 
     if (layer == m->L - 1) {
         k = MURE_KERNEL_OUTPUT;
     } else if (S.tc) {
-        k = S.tc_small ? MURE_KERNEL_TC_WINDOW : MURE_KERNEL_TC_GEMM;
+        k = S.tc_small ? MURE_KERNEL_TC_WINDOW : S.tc_conv ? MURE_KERNEL_TC_CONV : MURE_KERNEL_TC_GEMM;
         macs = tc_macs_per_row(S);
     } else if (S.variant > 0) {
         k = MURE_KERNEL_SIMT_SMALL;

@@ -50,6 +50,7 @@ constexpr int kFuseClasses = 12;       // classes of an output layer fused into 
 constexpr int kThreads = 384;          // 4 producer + 4 epilogue + 3 MMA + weight warps
 constexpr int kEpiStride = 36;         // floats per row of an epilogue staging chunk (32 + pad)
 constexpr int kMaxNT = 8;              // tensor-memory A stages, at most
+constexpr int kNBufMax = 4;            // staging buffers (small-image and staged-convolution modes)
 constexpr uint32_t kStageA = kTileM * 128;   // bytes of one producer ring slot
 constexpr long long kSpin = 2000000000LL;    // default wait limit: about a second at the SM clock
 
@@ -286,6 +287,16 @@ struct TcParams {
     // instead of the producers' 16-byte copies; tile m0 starts at row coordinate m0
     int a_tma;
     CUtensorMap tmap_a;
+    // MODE 3 (staged convolution): each tile's input rows with their zero border, 32
+    // channels at a time, land by tensor-map copies in a ring of cv_nbuf buffers; the
+    // producers gather every tap's 32 values from there.  K order: (chunk, tap, channel)
+    int cv_taps;                 // K-steps per chunk (one filter tap each)
+    int cv_nchunk;               // chunks of 32 input channels
+    int cv_imgs, cv_rows;        // batch rows per tile; output rows per tile and batch row
+    int cv_hw, cv_hh;            // staged width and height (input pixels, border included)
+    uint32_t cv_img_bytes;       // one batch row's staged chunk in shared memory
+    int cv_nbuf;
+    CUtensorMap tmap_x;          // the input rows as [row][ih][iw][ic]: boxes {32, cv_hw, cv_hh, 1}
 };
 
 // Per producer ring slot, the overlay values of a row's K-step: up to kOvMax
@@ -513,6 +524,7 @@ struct SmallConv {
     static constexpr uint32_t BYTES = NBUF * (BUF_B + OVST_B) + TAB_B;
 };
 static_assert(SmallConv::IMG_B % 16 == 0, "maps are bulk copies of whole 16-byte chunks");
+static_assert(SmallConv::NBUF <= kNBufMax, "staging barriers");
 
 // Tiles of the small-image mode over R rows: tile i holds rows MAPS*i .. MAPS*i+MAPS-1.
 __host__ __device__ __forceinline__ int64_t small_tiles(int64_t R) { return (R + SmallConv::MAPS - 1) / SmallConv::MAPS; }
@@ -559,7 +571,7 @@ struct SmallSteps {
 };
 
 // MODE 0: dense layer (one GEMM row per batch row); 1: implicit-GEMM convolution; 2:
-// the small-image convolution.  THREE: 3xTF32 (else one TF32 product).  FCP > 0
+// the small-image convolution; 3: the staged convolution (see TcParams).  THREE: 3xTF32 (else one TF32 product).  FCP > 0
 // (dense, one N slice): the output layer, with up to FCP classes, is computed from
 // each row's outputs in the epilogue, followed by the kill epilogue, and the rows
 // themselves are not stored.
@@ -573,8 +585,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     extern __shared__ __align__(1024) unsigned char smraw[];
     __shared__ __align__(8) uint64_t bar_afull[kNT], bar_aempty[kNT], bar_bfull[kNB], bar_bempty[kNB];
     __shared__ __align__(8) uint64_t bar_accfull[2], bar_accempty[2], bar_drain;
-    // small-image mode, per staging buffer: maps landed, overlay applied, producers done
-    __shared__ __align__(8) uint64_t bar_landed[SmallConv::NBUF], bar_ready[SmallConv::NBUF], bar_released[SmallConv::NBUF];
+    // small-image and staged-convolution modes, per staging buffer: copies landed,
+    // overlay applied, producers done
+    __shared__ __align__(8) uint64_t bar_landed[kNBufMax], bar_ready[kNBufMax], bar_released[kNBufMax];
     // dense A tiles by tensor-map copies: slot landed, slot read by the producers
     __shared__ __align__(8) uint64_t bar_alanded[kNA], bar_afree[kNA];
     __shared__ uint32_t tmem_sh;
@@ -594,6 +607,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     const uint32_t b_region = sbase;
     const uint32_t a_region = sbase + (p.b_resident ? (uint32_t)nK * b_step : (uint32_t)kNB * b_step);
     const uint32_t ov_region = a_region + kNA * kStageA;    // kNA overlay slots (with an overlay)
+    const uint32_t cv_region = a_region;                    // MODE 3: the staging ring
+    const uint32_t cv_buf_bytes = MODE == 3 ? (uint32_t)p.cv_imgs * p.cv_img_bytes : 0u;
     // FCP > 0: the output layer's weights as [F][FCP] (zeros beyond its C classes)
     const uint32_t fw_region = (ov_region + (p.ov.patch ? kNA * kOvSlotBytes : 0) + 15u) & ~15u;
     const float4 *fw4 = reinterpret_cast<const float4 *>(smraw + (fw_region - smem_u32(smraw)));
@@ -655,7 +670,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             mbar_init(smem_u32(&bar_alanded[s]), 1);
             mbar_init(smem_u32(&bar_afree[s]), 4);
         }
-        for (int s = 0; s < SmallConv::NBUF; ++s) {
+        for (int s = 0; s < kNBufMax; ++s) {
             mbar_init(smem_u32(&bar_landed[s]), 1);
             mbar_init(smem_u32(&bar_ready[s]), 1);
             mbar_init(smem_u32(&bar_released[s]), 4);
@@ -752,6 +767,49 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&bar_released[b]));
                 if (++b == G::NBUF) { b = 0; ++uses; }
+            }
+        } else if constexpr (MODE == 3) {
+            // the tile's staged input rows, one 32-channel chunk at a time (zero border
+            // included, overlay written in by warp 10): this thread gathers its GEMM
+            // row's 32 values of each filter tap from the chunk, 16 bytes per load, in
+            // the 128-byte swizzle of the copies (line l holds chunk j at j ^ (l mod 8))
+            const bool fin = p.ov.patch != nullptr;
+            bool ok = true;
+            int64_t job = 0;
+            for (int64_t i = 0; ok && i < my_tiles; ++i) {
+                const int64_t m0 = (blockIdx.x + i * gridDim.x) * (int64_t)kTileM;
+                const RowInfo ri = row_info<false, false>(p, m0 + r);
+                const int64_t row0 = m0 / p.P;
+                const int oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / kTileM) * p.cv_rows;
+                // rows past the end gather from the tile's first staged row (dropped later)
+                const uint32_t im = ri.ok ? (uint32_t)(ri.row - row0) : 0u;
+                const int line0 = ri.ok ? (ri.oy - oy0) * p.cv_hw + ri.ox : 0;
+                for (int c = 0; c < p.cv_nchunk; ++c, ++job) {
+                    const int b = (int)(job % p.cv_nbuf);
+                    const uint32_t use = (uint32_t)(job / p.cv_nbuf);
+                    if (!warp_wait_phase<32>(smem_u32(fin ? &bar_ready[b] : &bar_landed[b]), use & 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + im * p.cv_img_bytes;
+                    int ky = 0, kx = 0;
+                    for (int tap = 0; tap < p.cv_taps; ++tap) {
+                        const uint32_t line = (uint32_t)(line0 + ky * p.cv_hw + kx);
+                        const uint32_t lb = base + line * 128u, sw = line & 7u;
+                        float v[kTileK];
+#pragma unroll
+                        for (int cc = 0; cc < kTileK / 4; ++cc)
+                            asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                                         : "=f"(v[4 * cc]), "=f"(v[4 * cc + 1]), "=f"(v[4 * cc + 2]), "=f"(v[4 * cc + 3])
+                                         : "r"(lb + ((((uint32_t)cc) ^ sw) << 4)));
+                        if (!push(v)) { ok = false; break; }
+                        if (++kx == p.kw) { kx = 0; ++ky; }
+                    }
+                    // every gather of the chunk has been consumed by push: the buffer is free
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&bar_released[b]));
+                    if (!ok) break;
+                }
             }
         } else if (DENSE && p.a_tma) {
             // A tiles land by tensor-map copies (warp 10); each thread reads its row
@@ -1145,6 +1203,52 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             if (lane == 0) mbar_arrive(smem_u32(&bar_ready[b]));
             if (++b == G::NBUF) { b = 0; ++uses; }
         }
+    } else if (MODE == 3 && warp == 10) {
+        // ------------------------------------------ staged convolution: overlay --
+        // With an overlay (the first suffix stage), each landed chunk gets the mutated
+        // channels of its batch rows written over the copied values, at every staged
+        // pixel inside the image, before the producers read it.
+        if (p.ov.patch) {
+            int64_t job = 0;
+            bool ok = true;
+            for (int64_t i = 0; ok && i < my_tiles; ++i) {
+                const int64_t m0 = (blockIdx.x + i * gridDim.x) * (int64_t)kTileM;
+                const int64_t row0 = m0 / p.P;
+                const int oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / kTileM) * p.cv_rows;
+                const int nimg = (int)min((int64_t)p.cv_imgs, (int64_t)p.R - row0);
+                const int ncell = p.cv_hw * p.cv_hh;
+                for (int c = 0; c < p.cv_nchunk; ++c, ++job) {
+                    const int b = (int)(job % p.cv_nbuf);
+                    if (!warp_wait_phase<32>(smem_u32(&bar_landed[b]), (uint32_t)(job / p.cv_nbuf) & 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    for (int im = 0; im < nimg; ++im) {
+                        const int64_t row = row0 + im;
+                        const int g = (int)(row / p.T);
+                        const int k = p.ov.n_neurons[g];
+                        const int32_t *ids = p.ov.ids + p.ov.neuron_off[g];
+                        const float *prow = p.ov.patch + row * p.ov.row_stride;
+                        const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + (uint32_t)im * p.cv_img_bytes;
+                        for (int q = 0; q < k; ++q) {
+                            const int jl = ids[q] - c * kTileK;
+                            if (jl < 0 || jl >= kTileK) continue;
+                            const float *pq = prow + (int64_t)q * p.ov.cells;
+                            for (int cell = lane; cell < ncell; cell += 32) {
+                                const int hy = cell / p.cv_hw, hx = cell - hy * p.cv_hw;
+                                const int iy = oy0 - p.pad + hy, ix = hx - p.pad;
+                                if ((unsigned)iy >= (unsigned)p.ih || (unsigned)ix >= (unsigned)p.iw) continue;
+                                const uint32_t a = base + (uint32_t)cell * 128u +
+                                                   ((((uint32_t)jl >> 2) ^ ((uint32_t)cell & 7u)) << 4) + ((uint32_t)jl & 3u) * 4u;
+                                asm volatile("st.shared.f32 [%0], %1;" ::"r"(a), "f"(__ldg(pq + iy * p.iw + ix)) : "memory");
+                            }
+                        }
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&bar_ready[b]));
+                }
+            }
+        }
     } else if (warp < 11) {
         // ------------------------------------------------------------------ MMA --
         // The K-steps of a tile are dealt to the n_mma issuing warps by their index
@@ -1200,7 +1304,81 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         }
     } else {
         // -------------------------------------------------------------- weights --
-        if (lane == 0) {
+        if (MODE == 3 && lane == 0) {
+            // one thread issues both rings in the order they are consumed, each copy as
+            // soon as its slot is free: the staged chunks (released by the producers)
+            // and the weight K-steps (released by the MMAs)
+            const int64_t n_jobs = my_tiles * p.cv_nchunk;
+            const int64_t n_b = p.b_resident ? 0 : total;
+            const uint32_t box_bytes = (uint32_t)p.cv_hw * p.cv_hh * 128u;
+            const uint64_t tmap = reinterpret_cast<uint64_t>(&p.tmap_x);
+            if (p.b_resident) {
+                const uint32_t bytes = (uint32_t)nK * b_step;
+                mbar_expect_tx(smem_u32(&bar_bfull[0]), bytes);
+                for (uint32_t o = 0; o < bytes; o += 32768u)
+                    bulk_g2s(b_region + o, (const unsigned char *)wslice + o, min(32768u, bytes - o),
+                             smem_u32(&bar_bfull[0]));
+            }
+            int64_t jc = 0, jb = 0;
+            long long t_idle = clock64();
+            while (jc < n_jobs || jb < n_b) {
+                bool moved = false;
+                if (jc < n_jobs) {
+                    const int b = (int)(jc % p.cv_nbuf);
+                    const int64_t use = jc / p.cv_nbuf;
+                    if (use == 0 || mbar_try(smem_u32(&bar_released[b]), (uint32_t)((use - 1) & 1))) {
+                        const int64_t i = jc / p.cv_nchunk;
+                        const int c = (int)(jc - i * p.cv_nchunk);
+                        const int64_t m0 = (blockIdx.x + i * gridDim.x) * (int64_t)kTileM;
+                        const int64_t row0 = m0 / p.P;
+                        const int oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / kTileM) * p.cv_rows;
+                        const int nimg = (int)min((int64_t)p.cv_imgs, (int64_t)p.R - row0);
+                        const uint32_t bar = smem_u32(&bar_landed[b]);
+                        // the buffer was last read (and written) through the generic proxy
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        mbar_expect_tx(bar, (uint32_t)nimg * box_bytes);
+                        for (int im = 0; im < nimg; ++im) {
+                            const int64_t row = row0 + im;
+                            const int src = (int)(p.x_per_input ? p.t0 + row % p.T : row);
+                            asm volatile(
+                                "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes "
+                                "[%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(cv_region + (uint32_t)b * cv_buf_bytes +
+                                                                              (uint32_t)im * p.cv_img_bytes),
+                                "l"(tmap), "r"(c * kTileK), "r"(-p.pad), "r"(oy0 - p.pad), "r"(src), "r"(bar)
+                                : "memory");
+                        }
+                        ++jc;
+                        moved = true;
+                    }
+                }
+                if (jb < n_b) {
+                    const int sb = (int)(jb % kNB);
+                    const int64_t use = jb / kNB;
+                    if (use == 0 || mbar_try(smem_u32(&bar_bempty[sb]), (uint32_t)((use - 1) & 1))) {
+                        mbar_expect_tx(smem_u32(&bar_bfull[sb]), b_step);
+                        bulk_g2s(b_region + (uint32_t)sb * b_step, (const unsigned char *)wslice + (size_t)(jb % nK) * b_step,
+                                 b_step, smem_u32(&bar_bfull[sb]));
+                        ++jb;
+                        moved = true;
+                    }
+                }
+                if (moved) {
+                    t_idle = clock64();
+                    continue;
+                }
+                if (abort_flag->abort) break;
+                if (clock64() - t_idle > abort_flag->limit) {
+                    abort_flag->abort = 1;
+                    break;
+                }
+                __nanosleep(32);
+            }
+            // the copies still in flight land before the shared memory is released
+            for (int64_t jj = jc > p.cv_nbuf ? jc - p.cv_nbuf : 0; jj < jc; ++jj)
+                wait_phase_drain(smem_u32(&bar_landed[jj % p.cv_nbuf]), (uint32_t)((jj / p.cv_nbuf) & 1));
+            for (int64_t jj = jb > kNB ? jb - kNB : 0; jj < jb; ++jj)
+                wait_phase_drain(smem_u32(&bar_bfull[(int)(jj % kNB)]), (uint32_t)((jj / kNB) & 1));
+        } else if (lane == 0) {
             if (p.b_resident) {
                 const uint32_t bytes = (uint32_t)nK * b_step;
                 mbar_expect_tx(smem_u32(&bar_bfull[0]), bytes);
@@ -1260,13 +1438,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
 // Split fp32 weights [N][K] into TF32 halves laid out as the kernel's shared-memory
 // operand: for each 128-channel slice s and K-step kc, the hi plane then (3xTF32)
 // the lo plane, each Nt rows of 32 values in 128-byte-swizzled order.
+// perm_ic > 0 (the staged convolution): K-step kc holds channels 32 (kc / taps) .. +31
+// of filter tap kc mod taps, i.e. the K order (chunk, tap, channel) of its producers.
 __global__ void k_swizzle_weights(const float *__restrict__ W, int N, int K, int Np, int Kp, int planes,
-                                  int64_t slice_floats, float *out)
+                                  int64_t slice_floats, float *out, int perm_ic, int taps)
 {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= (int64_t)Np * Kp) return;
     const int n = (int)(i / Kp), k = (int)(i % Kp);
-    const float w = (n < N && k < K) ? W[(int64_t)n * K + k] : 0.f;
+    int ks = k;
+    if (perm_ic > 0) {
+        const int kc = k / kTileK;
+        ks = (kc % taps) * perm_ic + (kc / taps) * kTileK + k % kTileK;
+    }
+    const float w = (n < N && k < K) ? W[(int64_t)n * K + ks] : 0.f;
     const float h = tf32_rna(w);
     const int s = n / kSlice, nl = n % kSlice, Nt = min(kSlice, Np - s * kSlice);
     const int kc = k / kTileK, kk = k % kTileK;
@@ -1293,10 +1478,49 @@ int tc_small_geometry(const Stage &S)
            S.kw == G::KW && S.stride == 1 && S.pad == 0 && S.pool && !S.has_add && !S.gap && S.oc == G::OC;
 }
 
+// The staged convolution's tile: 128 GEMM rows are whole output rows of one batch row
+// (maps of >= 128 positions) or whole maps of several batch rows; the staged input is
+// the rows they read, zero border included, one 32-channel chunk per buffer.
+struct ConvTile {
+    int imgs, rows, hw, hh;
+    uint32_t img_bytes;
+};
+
+static bool conv_tile(const Stage &S, ConvTile &t)
+{
+    if (S.kind != MURE_NODE_CONV2D || S.stride != 1 || S.ic % kTileK != 0) return false;
+    if (S.pool && ((S.oh & 1) || (S.ow & 1))) return false;
+    const int P = S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
+    if (P >= kTileM) {
+        // whole output rows per tile; pooled tiles hold whole rows of pooling windows
+        if (P % kTileM != 0 || kTileM % S.ow != 0) return false;
+        t.imgs = 1;
+        t.rows = kTileM / S.ow;
+        if (S.pool && (t.rows & 1)) return false;
+    } else {
+        if (kTileM % P != 0) return false;
+        t.imgs = kTileM / P;
+        t.rows = S.oh;
+    }
+    t.hw = S.ow + S.kw - 1;
+    t.hh = t.rows + S.kh - 1;
+    if (t.hw > 256 || t.hh > 256) return false;
+    t.img_bytes = (uint32_t)((t.hw * t.hh * 128 + 1023) & ~1023);
+    // at least two buffers beside the streamed weights (three K-steps of 128 channels)
+    return (size_t)t.imgs * t.img_bytes <= 48 * 1024;
+}
+
+int tc_conv_geometry(const Stage &S)
+{
+    ConvTile t;
+    return conv_tile(S, t) ? 1 : 0;
+}
+
 // Whether the tensor-core kernel can fetch a first-suffix overlay itself: at most
 // kOvMax patch values per row and K-step (dense: at most 4 mutated channels).
 int tc_overlay_inline(const Stage &S, const Overlay &ov, int64_t groups)
 {
+    if (S.tc_conv) return 1;   // warp 10 writes any number of mutated channels
     if (S.tc_small)
         return ov.kmax <= SmallConv::MAXQ && groups <= SmallConv::MAXG && ov.cells == SmallConv::CELLS;
     if (S.kind == MURE_NODE_DENSE) {
@@ -1351,7 +1575,8 @@ int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t 
     }
     cudaMemsetAsync(out, 0, tc_weight_floats(S) * sizeof(float), s);
     k_swizzle_weights<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(W, N, K, Np, Kp, planes,
-                                                                   (int64_t)planes * kSlice * Kp, out);
+                                                                   (int64_t)planes * kSlice * Kp, out,
+                                                                   S.tc_conv ? S.ic : 0, S.kh * S.kw);
     return launches;
 }
 
@@ -1432,6 +1657,40 @@ static bool dense_a_tensor_map(const Stage &S, Src x, RowMap rm, CUtensorMap &ma
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The input rows of a staged convolution as a 4-D tensor [row][ih][iw][ic] with boxes
+// {32 channels, hw, hh, 1 row}, 128-byte swizzled, zero-filled outside the image.
+static bool conv_x_tensor_map(const Stage &S, Src x, RowMap rm, const ConvTile &t, CUtensorMap &map)
+{
+    if ((x.stride * 4) % 16 != 0 || (reinterpret_cast<uintptr_t>(x.p) & 15) != 0) return false;
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+    if (!enc) return false;
+    const int64_t rows = x.per_input ? rm.t0 + rm.T : rm.R;
+    const cuuint64_t dims[4] = {(cuuint64_t)S.ic, (cuuint64_t)S.iw, (cuuint64_t)S.ih, (cuuint64_t)rows};
+    const cuuint64_t strides[3] = {(cuuint64_t)S.ic * 4, (cuuint64_t)S.iw * S.ic * 4, (cuuint64_t)x.stride * 4};
+    const cuuint32_t box[4] = {(cuuint32_t)kTileK, (cuuint32_t)t.hw, (cuuint32_t)t.hh, 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    return enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float *>(x.p), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Dynamic shared memory a k_tc_gemm instance may use: the device's opt-in maximum less
+// the kernel's static shared memory.
+template <class Kern>
+static size_t tc_dyn_smem_max(Kern kern)
+{
+    static size_t cached = 0;
+    if (!cached) {
+        int dev = 0, optin = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+        cudaFuncAttributes fa{};
+        cudaFuncGetAttributes(&fa, kern);
+        cached = optin > (int)fa.sharedSizeBytes ? (size_t)optin - fa.sharedSizeBytes : 0;
+    }
+    return cached;
+}
+
 int tc_final_fusable(const Stage &S, const Stage &SL)
 {
     return S.tc && S.kind == MURE_NODE_DENSE && tc_supported(S) && round_up16(S.oc) <= kSlice &&
@@ -1481,8 +1740,31 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     p.b_resident = slice_bytes <= (S.tc_small ? 112 : 96) * 1024;
     const size_t b_bytes = p.b_resident ? slice_bytes : kNB * b_step;
     // at least 116 KiB so that one CTA (holding all 512 tensor-memory columns) runs per SM
-    const size_t a_bytes = S.tc_small ? (size_t)SmallConv::BYTES
-                                      : (size_t)kNA * kStageA + (p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0);
+    size_t a_bytes = S.tc_small ? (size_t)SmallConv::BYTES
+                                : (size_t)kNA * kStageA + (p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0);
+    ConvTile ct{};
+    if (S.tc_conv) {
+        // the staged convolution: as many staging buffers (up to 4) as fit beside the
+        // weights; the weights' K order was fixed for it at model load
+        const bool ok = conv_tile(S, ct) && conv_x_tensor_map(S, x, rm, ct, p.tmap_x);
+        const size_t room = three ? tc_dyn_smem_max(k_tc_gemm<3, true>) : tc_dyn_smem_max(k_tc_gemm<3, false>);
+        const size_t buf = (size_t)ct.imgs * ct.img_bytes;
+        const int nbuf = ok && room > 1024 + b_bytes ? (int)std::min<size_t>(kNBufMax, (room - 1024 - b_bytes) / buf) : 0;
+        if (nbuf < 2) {
+            static const int unsupported = MURE_ERR_UNSUPPORTED;
+            cudaMemcpyAsync(S.err, &unsupported, sizeof(int), cudaMemcpyHostToDevice, s);
+            return 0;
+        }
+        p.cv_taps = S.kh * S.kw;
+        p.cv_nchunk = S.ic / kTileK;
+        p.cv_imgs = ct.imgs;
+        p.cv_rows = ct.rows;
+        p.cv_hw = ct.hw;
+        p.cv_hh = ct.hh;
+        p.cv_img_bytes = ct.img_bytes;
+        p.cv_nbuf = nbuf;
+        a_bytes = (size_t)nbuf * buf;
+    }
     if (ff) p.ff = *ff;
     if (ss) p.slot = *ss;
     const size_t f_bytes = ff ? 16 + (size_t)ff->F * kFuseClasses * 4 : 0;
@@ -1495,7 +1777,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     if (ss) p.n_mma = 1;
     // dense rows without an overlay: A tiles by tensor-map copies from warp 10
     p.a_tma = dense && !p.ov.patch && p.n_mma <= 2 && dense_a_tensor_map(S, x, rm, p.tmap_a) ? 1 : 0;
-    if (S.tc_small) p.n_mma = std::min(p.n_mma, 2);   // warp 10 stages maps in that mode
+    if (S.tc_small || S.tc_conv) p.n_mma = std::min(p.n_mma, 2);   // warp 10 stages maps in those modes
     const int64_t M = (int64_t)rm.R * p.P;
     const int64_t tiles = S.tc_small ? small_tiles(rm.R) : (M + kTileM - 1) / kTileM;
     static int n_sm = 0;
@@ -1514,6 +1796,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     if (dense && ff) { if (three) go(k_tc_gemm<0, true, kFuseClasses>); else go(k_tc_gemm<0, false, kFuseClasses>); }
     else if (dense) { if (three) go(k_tc_gemm<0, true>); else go(k_tc_gemm<0, false>); }
     else if (S.tc_small) { if (three) go(k_tc_gemm<2, true>); else go(k_tc_gemm<2, false>); }
+    else if (S.tc_conv) { if (three) go(k_tc_gemm<3, true>); else go(k_tc_gemm<3, false>); }
     else { if (three) go(k_tc_gemm<1, true>); else go(k_tc_gemm<1, false>); }
     int launches = 1;
     if (S.gap) launches += launch_gap(gap_tmp, map_stride, mh * mw, S.oc, rm.R, y_out, y_stride, s);
@@ -1569,7 +1852,8 @@ int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_input
     k_slot_filters<<<(unsigned)(((int64_t)Np * K + 255) / 256), 256, 0, s>>>(K, pa, n, Np, dw.filt, dw.colb, dw.colg,
                                                                          dw.colq, dw.colj);
     k_swizzle_weights<<<(unsigned)(((int64_t)Np * Kp + 255) / 256), 256, 0, s>>>(dw.filt, Np, K, Np, Kp, planes,
-                                                                               (int64_t)planes * kSlice * Kp, dw.swz);
+                                                                               (int64_t)planes * kSlice * Kp, dw.swz,
+                                                                               S.tc_conv ? S.ic : 0, S.kh * S.kw);
     Stage D = S;
     D.oc = Np;
     D.tc = precision == MURE_PREC_TF32X3 ? 1 : 2;

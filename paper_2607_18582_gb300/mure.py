@@ -221,7 +221,7 @@ class Model:
     def n_layers(self):
         return lib().mure_model_n_layers(self.h)
 
-    KERNELS = {0: "simt_gemm", 1: "simt_small", 2: "tc_gemm", 3: "tc_window", 4: "output"}
+    KERNELS = {0: "simt_gemm", 1: "simt_small", 2: "tc_gemm", 3: "tc_window", 4: "output", 5: "tc_conv"}
 
     def layer_kernel(self, layer):
         """(kernel name, executed multiply-accumulates per batch row) of a layer."""

@@ -365,3 +365,29 @@ def test_tensor_core_conv_on_small_layers(M, ctx, oracle_mod, monkeypatch, prec,
     else:
         agree = (bits(r["kill_bits"], len(w.X)) == bits(ora["kill_bits"], len(w.X))).mean()
         assert agree >= 0.98, agree
+
+
+@pytest.mark.parametrize("name", ["vgg", "resnet20"])
+def test_gather_mode_convolutions_match_oracle(M, ctx, oracle_runs, monkeypatch, name):
+    """Stride-1 convolutions with 32k input channels run by default on input rows
+    staged in shared memory (K order: 32-channel chunk, tap, channel); with
+    MURE_TC_CONV=gather they keep the per-row gathers from device memory (K order: tap,
+    channel).  Both orders are fixed per model, so each mode is memoized == vanilla bit
+    for bit and within the fp32 tolerance of the oracle; the model reports which kernel
+    each layer uses."""
+    w, table, ora = oracle_runs(name)
+    staged = M.mure_model_load(ctx, w.model, precision="tf32x3")
+    kinds = [staged.layer_kernel(l)[0] for l in range(w.model.n_layers())]
+    assert "tc_conv" in kinds, kinds
+    monkeypatch.setenv("MURE_TC_CONV", "gather")
+    gather = M.mure_model_load(ctx, w.model, precision="tf32x3")
+    monkeypatch.delenv("MURE_TC_CONV")
+    assert "tc_conv" not in [gather.layer_kernel(l)[0] for l in range(w.model.n_layers())]
+    for model in (staged, gather):
+        r = M.mure_eval_mutants(M.mure_build_prefix_cache(model, w.X), table, logits=True)
+        ok, worst = logits_close(r["logits"], ora["logits"])
+        assert ok, worst
+        bad, _ = compare_kills(r["kill_bits"], ora["kill_bits"], ora["orig_logits"], ora["logits"], len(w.X))
+        assert bad == 0
+        v = M.mure_eval_vanilla(model, w.X, table, logits=True)
+        assert np.array_equal(v["logits"].view(np.uint32), r["logits"].view(np.uint32))
