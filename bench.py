@@ -1,12 +1,16 @@
 """Benchmark of memoized DNN mutation testing on GB300.
 
-One step = the whole hot path over the workload: the prefix-activation cache of the
-inputs (Algorithm 1 lines 10-12), descriptor expansion and grouping, the delta and
-suffix kernels of every mutant group, the fused kill epilogue and the score
-reduction.  Default workload: LeNet-5 (28x28x1), 10,000 inputs, 2,000 mutants at a
-1% selection ratio (GF / NEB / NAI / NS), random He-normal weights.
+One step = the whole hot path over one batch of the workload: the prefix-activation
+cache of ALL the workload's inputs (Algorithm 1 lines 10-12), descriptor expansion and
+grouping, the delta and suffix kernels of every mutant group, the fused kill epilogue
+and the score reduction, for one slice of the mutant table.  The table is cut into S
+slices by a seeded random partition (each slice a uniform sample of the table's mix of
+layers, operators and ratios); S consecutive steps cover the whole table once, so the
+default 20 timed steps on the VGG workload (10,000 inputs x 5,000 mutants, S = 20) are
+exactly one full job, with the cache rebuilt every step.  Default workload: the
+VGG-style network, 10,000 inputs N(0,1), 5,000 mutants at 0.5 / 1 / 2 / 5 %.
 
-  python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference] [--workload NAME]
 
 Prints one JSON line (rank 0).  N > 1 runs N independent replicas (one per GPU,
 launched by torchrun); the path has no cross-GPU exchange.
@@ -34,6 +38,9 @@ UNIT = "evals/s"
 # CUDA-core fp32 peak of a GB300: 152 SMs x 128 FP32 lanes x 2 FLOP (FMA) x 2.07 GHz
 SIMT_FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
 L2_FLUSH_BYTES = 256 << 20
+
+# slices of the mutant table per full job (one slice per step)
+SLICES = {"vgg": 20, "vgg_stress": 20, "resnet20": 20}
 
 WORKLOAD_TEXT = {
     "lenet5": "LeNet-5 28x28x1 (conv5x5 6 pad2, pool, conv5x5 16, pool, FC 400-120-84-10), 10,000 inputs U[0,1], "
@@ -247,7 +254,8 @@ def run_reference(args, world, rank):
     oracle.build()
     w = wl.workload(args.workload)
     threads = os.cpu_count() or 1
-    n_mut, n_in = 40, 500
+    n_mut, n_base = cpu_sample_size(w)
+    n_in = max(1, n_base // 8)
     for _ in range(args.warmup):
         cpu_oracle_rate(w, n_mut, n_in, threads)
     t = time.perf_counter()
@@ -277,15 +285,88 @@ def config_block(args, w):
 
 # ----------------------------------------------------------------- GPU leg --
 
+def table_slices(n_mut, n_slices, seed=7):
+    """A seeded random partition of the table's row indices into n_slices slices
+    (sorted within each slice); slice k is step k's batch of mutants."""
+    n_slices = max(1, min(n_slices, n_mut)) if n_mut else 1
+    perm = np.random.default_rng(seed).permutation(n_mut)
+    return [np.sort(perm[k::n_slices]) for k in range(n_slices)]
+
+
+def analytic_flops(model, table):
+    """FLOPs the method must spend on a table (per input), memoized and vanilla: the
+    suffix layers after each mutant's first mutated layer l, the recomputed channels of
+    layer l for GF / WS (k neurons x the layer's MACs per neuron) and, in vanilla mode,
+    the prefix and the whole layer l (Lemma 4's cost model: vanilla - memo = the
+    prefix every mutant of a cluster shares)."""
+    L = model.n_layers()
+    macs = np.array([model.layer_macs(v) for v in range(L)], np.float64)
+    suffix = np.concatenate([np.cumsum(macs[::-1])[::-1][1:], [0.0]])   # sum over v > l
+    prefix = np.cumsum(macs)                                            # sum over v <= l
+    width = np.array([model.layer_width(v) for v in range(L)], np.float64)
+    l = table.layer.astype(np.int64)
+    dot = np.isin(table.op, [0, 4])          # GF, WS recompute their channels
+    delta = np.where(dot, table.n_neurons * macs[l] / width[l], 0.0)
+    memo = 2.0 * float((suffix[l] + delta).sum())
+    vanilla = 2.0 * float((prefix[l] + suffix[l] + delta).sum())
+    return memo, vanilla
+
+
+def measure_tensor_peaks(dev):
+    """Peaks of this GPU measured like the driver's bf16 figures: cuBLAS TF32 (fp32
+    operands, TF32 tensor cores) and fp32 CUDA-core GEMMs of 8192^3 (2 N^3 FLOP), best
+    of 10 back-to-back (burst), and TF32 back to back for about 2 s (sustained)."""
+    import torch
+    n = 8192
+    a = torch.randn(n, n, device=f"cuda:{dev}")
+    b = torch.randn(n, n, device=f"cuda:{dev}")
+    old = torch.backends.cuda.matmul.allow_tf32
+
+    def best(k):
+        ts = []
+        for _ in range(k):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            torch.matmul(a, b)
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1) / 1e3)
+        return 2.0 * n ** 3 / min(ts) / 1e12
+    try:
+        torch.backends.cuda.matmul.allow_tf32 = True
+        torch.matmul(a, b)
+        tf32 = best(10)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(1, int(2.0 * tf32 * 1e12 / (2.0 * n ** 3)))
+        e0.record()
+        for _ in range(reps):
+            torch.matmul(a, b)
+        e1.record()
+        torch.cuda.synchronize()
+        tf32_sus = reps * 2.0 * n ** 3 / (e0.elapsed_time(e1) / 1e3) / 1e12
+        torch.backends.cuda.matmul.allow_tf32 = False
+        torch.matmul(a, b)
+        fp32 = best(5)
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = old
+    del a, b
+    torch.cuda.empty_cache()
+    return {"tf32_tflops": tf32, "tf32_tflops_sustained": tf32_sus, "fp32_tflops": fp32,
+            "how": "torch.matmul fp32 8192^3 (2 N^3 FLOP): TF32 allowed best of 10 (burst) and back to back "
+                   f"~2 s ({reps} GEMMs, sustained); TF32 disallowed (CUDA cores) best of 5"}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="lenet5")
+    ap.add_argument("--workload", default="vgg")
+    ap.add_argument("--slices", type=int, default=None,
+                    help="slices of the mutant table (one per step); default per workload (VGG 20)")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
-    ap.add_argument("--skip-extras", action="store_true", help="no e2e / vanilla / clocks legs")
+    ap.add_argument("--skip-extras", action="store_true", help="no e2e / vanilla / stress / peaks legs")
     ap.add_argument("--n-inputs", type=int, default=None, help="smaller case (profiling): first n inputs")
     ap.add_argument("--n-mutants", type=int, default=None, help="smaller case (profiling): first n mutants")
     ap.add_argument("--only-layer", type=int, default=None, help="keep only the mutants of this layer")
@@ -306,25 +387,31 @@ def main():
     w = wl.workload(args.workload, args.n_inputs, args.n_mutants)
     if args.only_layer is not None:
         w.table = w.table.subset(np.nonzero(w.table.layer == args.only_layer)[0])
-    n_evals = len(w.table) * len(w.X)
+    n_slices = args.slices if args.slices is not None else SLICES.get(args.workload, 1)
+    slices = table_slices(len(w.table), n_slices)
+    tables = [w.table.subset(ix) for ix in slices]
+    arrays = [mure.table_array(t) for t in tables]
     ctx = mure.mure_create(dev)
     model = mure.mure_model_load(ctx, w.model, precision=args.precision)
     X_dev = torch.from_numpy(w.X).to(f"cuda:{dev}")
-    arrays = mure.table_array(w.table)
     W64 = (len(w.X) + 63) // 64
     kill_dev = torch.empty((len(w.table), W64), dtype=torch.int64, device=f"cuda:{dev}")
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=f"cuda:{dev}")
     stream = torch.cuda.current_stream(dev)
+    off = np.concatenate([[0], np.cumsum([len(t) for t in tables])])
+    # step k evaluates slice k mod S; its kill rows go to their table positions afterwards
+    kill_slices = [kill_dev[int(off[k]):int(off[k + 1])] for k in range(len(tables))]
 
-    def step(timing):
+    def step(k, timing=False):
+        j = k % len(tables)
         cache = mure.mure_build_prefix_cache(model, X_dev)
-        r = mure.mure_eval_mutants(cache, w.table, outputs_on_device=True, kill_out=kill_dev, kernel_timing=timing,
-                                   arrays=arrays)
+        r = mure.mure_eval_mutants(cache, tables[j], outputs_on_device=True, kill_out=kill_slices[j],
+                                   kernel_timing=timing, arrays=arrays[j])
         del cache
         return r
 
-    for _ in range(args.warmup):
-        step(True)
+    for i in range(args.warmup):
+        step(i)
     torch.cuda.synchronize()
     barrier(world)
     torch.cuda.synchronize()
@@ -335,7 +422,7 @@ def main():
         for i in range(args.steps):
             flush.zero_()                       # evict L2 between steps (not timed)
             evs[i][0].record(stream)
-            results.append(step(True))
+            results.append(step(i))
             evs[i][1].record(stream)
         torch.cuda.synchronize()
     barrier(world)
@@ -343,31 +430,52 @@ def main():
     launches = mure.mure_kernel_launches(ctx) - launches0
     ms = [a.elapsed_time(b) for a, b in evs]
     t_total = max_over_ranks(sum(ms) / 1e3, world)
-    value = world * args.steps * n_evals / t_total
+    step_evals = [len(tables[i % len(tables)]) * len(w.X) for i in range(args.steps)]
+    n_evals = sum(step_evals)
+    value = world * n_evals / t_total
     last = results[-1]
 
-    # dominant kernel: the layer (or delta / gather) class with the largest device time
+    # per-kernel device times from a separate pass with per-launch events (the timed
+    # steps above run without them): the first min(S, 3) slices, scaled per step
+    n_bd = min(len(tables), 3)
+    bd = []
+    cb_ms = []
+    for i in range(n_bd):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        cache = mure.mure_build_prefix_cache(model, X_dev)
+        e1.record(stream)
+        bd.append(mure.mure_eval_mutants(cache, tables[i], outputs_on_device=True, kill_out=kill_slices[i],
+                                         kernel_timing=True, arrays=arrays[i]))
+        torch.cuda.synchronize()
+        cb_ms.append(e0.elapsed_time(e1))
+        del cache
+    bd_evals = sum(len(tables[i]) * len(w.X) for i in range(n_bd))
+
     L = w.model.n_layers()
-    cls_ms = {f"layer{v}": sum(r["stats"]["ms_layer"][v] for r in results) for v in range(L)}
-    cls_ms["delta"] = sum(r["stats"]["ms_delta"] for r in results)
-    cls_ms["gather"] = sum(r["stats"]["ms_gather"] for r in results)
-    cls_ms["epilogue"] = sum(r["stats"]["ms_epilogue"] for r in results)
+    cls_ms = {f"layer{v}": sum(r["stats"]["ms_layer"][v] for r in bd) for v in range(L)}
+    cls_ms["delta"] = sum(r["stats"]["ms_delta"] for r in bd)
+    cls_ms["gather"] = sum(r["stats"]["ms_gather"] for r in bd)
+    cls_ms["epilogue"] = sum(r["stats"]["ms_epilogue"] for r in bd)
     top = max(cls_ms, key=cls_ms.get)
-    roof = None
     pk, pk_kind = peaks()
+    tp = None
+    if not args.skip_extras:
+        tp = measure_tensor_peaks(dev)
+    # the step is long: the sustained TF32 figure applies when a step runs >= 1 s
+    long_step = t_total / args.steps >= 1.0
+    roof = None
     if top == "delta":
-        # HBM-bound: algorithmic bytes = the rows it builds (written once, cached rows
-        # read once) per its device time
-        byts = sum(r["stats"]["bytes_gather"] for r in results)
+        byts = sum(r["stats"]["bytes_gather"] for r in bd)
         achieved = byts / (cls_ms[top] / 1e3) / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
                 "frac": achieved / pk["hbm_gbs"], "traffic": None, "kernel": "delta kernels (k_patch_*)",
                 "ms_total": cls_ms[top], "peak_source": f"{pk_kind} (MEASURED_PEAKS.json hbm_gbs)"}
-    pk, pk_kind = peaks()
     if top.startswith("layer"):
         v = int(top[5:])
-        fl = sum(r["stats"]["flops_layer"][v] for r in results)
-        nl = sum(r["stats"]["launches_layer"][v] for r in results)
+        fl = sum(r["stats"]["flops_layer"][v] for r in bd)
+        nl = sum(r["stats"]["launches_layer"][v] for r in bd)
         secs = cls_ms[top] / 1e3
         achieved = fl / secs / 1e12
         layer_node = w.model.nodes[w.model.layers()[v]]
@@ -375,99 +483,189 @@ def main():
         rows = rows_total / max(1, nl)   # rows per launch
         kname, macs_exec = model.layer_kernel(v)
         desc = f"layer {v}: {layer_node.kind} {layer_node.cin}->{layer_node.cout}"
-        if kname in ("tc_gemm", "tc_window"):
-            # tensor cores: TF32 peak = measured bf16 x the nominal TF32 / bf16 ratio
-            # (1.1 / 2.25 PFLOP/s); 3xTF32 spends three TF32 products per fp32 MAC, so
-            # its fp32-equivalent peak is a third of that.  The step is long, so the
-            # sustained bf16 figure applies.
-            bf16 = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
-            tf32_peak = bf16 * 1.1 / 2.25
+        if kname in ("tc_gemm", "tc_window", "tc_conv"):
+            # tensor cores: 3xTF32 spends three TF32 products per fp32 MAC, so its
+            # fp32-equivalent peak is a third of the measured TF32 peak
             terms = 3 if args.precision == "tf32x3" else 1
+            if tp:
+                tf32_peak = tp["tf32_tflops_sustained"] if long_step else tp["tf32_tflops"]
+                src = (f"measured here: cuBLAS TF32 {'sustained' if long_step else 'burst'} {tf32_peak:.1f} "
+                       f"TFLOP/s / {terms} ({args.precision})")
+            else:
+                bf16 = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+                tf32_peak = bf16 * 1.1 / 2.25
+                src = f"{pk_kind} bf16 sustained {bf16:.1f} TFLOP/s x 1.1/2.25 (TF32) / {terms} ({args.precision})"
             peak = tf32_peak / terms
-            key = "tc_window" if kname == "tc_window" else "tc_gemm"
+            label = {"tc_window": "window GEMM", "tc_conv": "staged convolution", "tc_gemm": "implicit GEMM"}[kname]
             roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                    "traffic": profiled_traffic(f"{key}_{args.workload}_layer{v}", rows), "rows_per_launch": rows,
-                    "kernel": f"k_tc_gemm ({'window GEMM' if kname == 'tc_window' else 'implicit GEMM'}, {desc})",
-                    "launches": nl, "ms_total": cls_ms[top],
-                    "peak_source": f"{pk_kind} bf16 sustained {bf16:.1f} TFLOP/s x 1.1/2.25 (TF32) / {terms} "
-                                   f"({args.precision}); achieved counts the layer's useful fp32 MACs x 2",
+                    "traffic": profiled_traffic(f"{kname}_{args.workload}_layer{v}", rows), "rows_per_launch": rows,
+                    "kernel": f"k_tc_gemm ({label}, {desc})", "launches": nl, "ms_total": cls_ms[top],
+                    "peak_source": src + "; achieved counts the layer's useful fp32 MACs x 2",
                     "tensor_pipe_frac": terms * 2 * macs_exec * rows_total / secs / 1e12 / tf32_peak}
         else:
             key = "conv_small" if kname == "simt_small" else ("final_dense" if kname == "output" else "stage_simt")
-            roof = {"bound": "alu", "achieved": achieved, "peak": SIMT_FP32_PEAK_TFLOPS, "unit": "TFLOP/s",
-                    "frac": achieved / SIMT_FP32_PEAK_TFLOPS,
+            fp32_peak = tp["fp32_tflops"] if tp else SIMT_FP32_PEAK_TFLOPS
+            roof = {"bound": "alu", "achieved": achieved, "peak": fp32_peak, "unit": "TFLOP/s",
+                    "frac": achieved / fp32_peak,
                     "traffic": profiled_traffic(f"{key}_{args.workload}_layer{v}", rows), "rows_per_launch": rows,
                     "kernel": f"k_{key} ({desc})", "launches": nl, "ms_total": cls_ms[top],
-                    "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz (CUDA cores)",
+                    "peak_source": ("measured here: cuBLAS fp32 (CUDA cores)" if tp else
+                                    "derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz (CUDA cores)"),
                     "tensor_pipe_frac": 0.0}
+    memo_fl, van_fl = analytic_flops(w.model, w.table)
+    cfg = config_block(args, w)
+    cfg["mutants_per_step"] = float(np.mean([len(tables[i % len(tables)]) for i in range(args.steps)]))
+    cfg["slices"] = len(tables)
+    cfg["step"] = (f"cache build over all {len(w.X):,} inputs + 1/{len(tables)} of the mutant table (a seeded random "
+                   f"partition; {len(tables)} steps = the whole table once)" if len(tables) > 1 else
+                   f"cache build over all {len(w.X):,} inputs + the whole mutant table")
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": 1e3 * t_total / args.steps, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": {"fp32": "f32", "tf32x3": "tf32x3", "tf32": "tf32"}[args.precision],
            "data": "synthetic",
-           "config": config_block(args, w), "roofline": roof, "gpu_launches": int(launches),
-           "kernel_ms_per_step": {k: v / args.steps for k, v in cls_ms.items()},
+           "config": cfg, "roofline": roof, "gpu_launches": int(launches),
+           "kernel_ms_per_step": {k: v / n_bd * (n_evals / args.steps) / (bd_evals / n_bd) for k, v in cls_ms.items()},
+           "kernel_breakdown": f"separate pass with per-launch events over slices 0..{n_bd - 1}, scaled to the mean "
+                               "step; the timed steps run without per-launch events",
            "scores": {"killed_frac": last["scoreA"], "deepmutation": last["scoreB"],
-                      "near_ties": last["stats"]["n_near_ties"]}}
+                      "near_ties": last["stats"]["n_near_ties"]},
+           "analytic_flops": {"memo_per_eval": memo_fl / len(w.table), "vanilla_per_eval": van_fl / len(w.table),
+                              "memo_over_vanilla": memo_fl / van_fl,
+                              "memo_tflops_achieved": memo_fl / len(w.table) * n_evals * world / t_total / 1e12}}
 
     if not args.skip_extras:
         out["clocks"] = clk.summary()
         # end to end through the C ABI with host buffers: pinned X in, kill bits out
         X_pin = torch.from_numpy(w.X).pin_memory()
-        kill_host = np.zeros((len(w.table), W64), np.uint64)
+        kill_host = [np.zeros((len(t), W64), np.uint64) for t in tables]
         k_e2e = max(3, min(args.steps, 5))
 
-        def step_e2e():
+        def step_e2e(k):
+            j = k % len(tables)
             cache = mure.mure_build_prefix_cache(model, X_pin.numpy())
-            return mure.mure_eval_mutants(cache, w.table, kill_out=kill_host, arrays=arrays)
+            return mure.mure_eval_mutants(cache, tables[j], kill_out=kill_host[j], arrays=arrays[j])
 
-        step_e2e()
-        times = []
-        for _ in range(k_e2e):
+        step_e2e(0)
+        times, ev_e2e = [], 0
+        for k in range(k_e2e):
             flush.zero_()
             torch.cuda.synchronize()
             t0 = time.perf_counter()
-            step_e2e()          # synchronous: returns with the kill bits in host memory
+            step_e2e(k)          # synchronous: returns with the kill bits in host memory
             times.append(time.perf_counter() - t0)
-        e2e_t = max_over_ranks(sum(times) / k_e2e, world)
-        h2d = int(w.X.nbytes + arrays[0].nbytes + arrays[1].nbytes)
-        d2h = int(kill_host.nbytes + 32)
-        out["e2e"] = {"value": world * n_evals / e2e_t, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            ev_e2e += len(tables[k % len(tables)]) * len(w.X)
+        e2e_t = max_over_ranks(sum(times), world)
+        h2d = int(w.X.nbytes + np.mean([a[0].nbytes + a[1].nbytes for a in arrays]))
+        d2h = int(np.mean([kh.nbytes for kh in kill_host]) + 32)
+        out["e2e"] = {"value": world * ev_e2e / e2e_t, "unit": UNIT, "h2d_bytes_per_step": h2d,
                       "d2h_bytes_per_step": d2h, "steps": k_e2e}
-        # the GPU vanilla mode (speed-up denominator), same kernels, no reuse
+        # the GPU vanilla mode (speed-up denominator), same kernels, no reuse: slice 0
         torch.cuda.synchronize()
         t0 = time.perf_counter()
-        van = mure.mure_eval_vanilla(model, X_dev, w.table, outputs_on_device=True)
+        van = mure.mure_eval_vanilla(model, X_dev, tables[0], outputs_on_device=True)
         torch.cuda.synchronize()
         tv = time.perf_counter() - t0
-        same = bool(torch.equal(van["kill_bits"], kill_dev))
-        t_m = t_total / args.steps
-        out["gpu_vanilla"] = {"value": n_evals / tv, "ms_per_step": 1e3 * tv, "speedup": tv / t_m,
-                              "gain": (tv - t_m) / tv, "kill_matrix_identical": same}
+        same = bool(torch.equal(van["kill_bits"], kill_slices[0]))
+        memo_s = float(np.mean([m / 1e3 for m in ms]))
+        m0, v0 = analytic_flops(w.model, tables[0])
+        van_rate = len(tables[0]) * len(w.X) / tv
+        memo_rate = n_evals / (t_total / world) / world if world else value
+        out["gpu_vanilla"] = {"value": van_rate, "ms_per_step": 1e3 * tv, "slice": 0,
+                              "speedup": memo_rate / van_rate, "gain": 1.0 - van_rate / memo_rate,
+                              "kill_matrix_identical": same,
+                              "achieved_tflops": v0 * len(w.X) / tv / 1e12,
+                              "analytic_flops_per_eval": v0 / len(tables[0])}
+        # the stress mix (half of the mutants on the first convolution, 0.1-10 %):
+        # one slice of its table over all its inputs, after a warm-up on a few mutants
+        if args.workload == "vgg" and args.n_inputs is None and args.n_mutants is None:
+            ws_ = wl.workload("vgg_stress")
+            st_sl = table_slices(len(ws_.table), SLICES["vgg_stress"])
+            tab = ws_.table.subset(st_sl[0])
+            Xs = torch.from_numpy(ws_.X).to(f"cuda:{dev}")
+            mure.mure_eval_mutants(mure.mure_build_prefix_cache(model, Xs), tab.subset(np.arange(24)))
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            cs = mure.mure_build_prefix_cache(model, Xs)
+            rs = mure.mure_eval_mutants(cs, tab, outputs_on_device=True)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            sm, sv = analytic_flops(ws_.model, tab)
+            t_s = e0.elapsed_time(e1) / 1e3
+            out["stress"] = {"workload": "vgg_stress: " + WORKLOAD_TEXT["vgg_stress"], "value": len(tab) * len(ws_.X) / t_s,
+                             "unit": UNIT, "ms_per_step": 1e3 * t_s,
+                             "step": f"cache build over all {len(ws_.X):,} inputs + 1/{SLICES['vgg_stress']} of the "
+                                     f"table ({len(tab)} mutants)",
+                             "memo_over_vanilla_flops": sm / sv, "killed_frac": rs["scoreA"]}
+            del cs, Xs
     if rank == 0 and world == 1 and not args.skip_cpu_baseline:
         import oracle
         oracle.build()
         threads = os.cpu_count() or 1
-        rate, dt, sample, agree = cpu_oracle_rate(w, 400, 2000, threads, gpu_kill=kill_dev.cpu().numpy())
+        n_mut, n_in = cpu_sample_size(w)
+        rate, dt, sample, agree = cpu_oracle_rate(w, n_mut, n_in, threads, gpu_kill=kill_dev.cpu().numpy())
         out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
                                "seconds": dt}
         # kill verdicts of the timed GPU run against the oracle's on the same sample
         # (differences are expected only on near ties; the TF32 variant reports its rate)
         out["oracle_agreement"] = agree
-    out["hbm"] = hbm_rates(w, results, cls_ms, pk, pk_kind)
+    out["hbm"] = hbm_rates(w, bd, cls_ms, pk, pk_kind)
+    # the cache build (a full forward over the inputs: tensor-bound), bytes for reference
+    cb_bytes = w.X.nbytes + cache_bytes(model, len(w.X))
+    cb_s = float(np.mean(cb_ms)) / 1e3
+    out["hbm"]["cache_build"] = {"kernels": "the layer kernels over all inputs (mure_build_prefix_cache)",
+                                 "bytes": cb_bytes, "ms": 1e3 * cb_s, "achieved": cb_bytes / cb_s / 1e9, "unit": "GB/s",
+                                 "frac": cb_bytes / cb_s / 1e9 / pk["hbm_gbs"],
+                                 "tflops": 2.0 * sum(w.model.layer_macs(v) for v in range(L)) * len(w.X) / cb_s / 1e12,
+                                 "bytes_counted": "inputs read + every cached x_v and z_v row written once",
+                                 "bound": "tensor (one forward pass over the inputs)"}
     # the batched suffix's activation rows written and read back through device memory
     # (not algorithmic bytes: ideally they would stay on chip)
-    rows_b = sum(r["stats"].get("bytes_rows", 0) for r in results)
-    evals = sum(r["stats"]["n_rows"] for r in results)
+    rows_b = sum(r["stats"].get("bytes_rows", 0) for r in bd)
+    evals = sum(r["stats"]["n_rows"] for r in bd)
     if evals > 0:
         out["activation_rows"] = {"bytes_per_eval": rows_b / evals, "unit": "B",
                                   "counted": "suffix stage output rows, written once and read once"}
     out["peaks"] = {"source": pk_kind, "hbm_gbs": pk.get("hbm_gbs"), "bf16_tflops": pk.get("bf16_tflops")}
+    if tp:
+        out["peaks"].update(tp)
     if rank == 0:
         print(json.dumps(out), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
     return 0
+
+
+def cache_bytes(model, n_inputs):
+    """Bytes of the prefix cache for n inputs: every weighted layer's input x_v and
+    pre-activation z_v and the logits (rows rounded up to 4 floats, inputs to a
+    multiple of 64), fp32."""
+    shapes = model.shapes()
+    n_pad = (n_inputs + 63) // 64 * 64
+    r4 = lambda n: (n + 3) // 4 * 4
+    per = r4(model.n_classes)
+    for v in model.layers():
+        nd = model.nodes[v]
+        src = nd.inputs[0]
+        ih, iw, ic = model.in_shape if src < 0 else shapes[src]
+        h, ww, c = shapes[v]
+        per += r4(ih * iw * ic) + r4(h * ww * c)
+    return n_pad * per * 4
+
+
+def cpu_sample_size(w):
+    """(stratified mutants, inputs) of the CPU-baseline sample; the reference arm times
+    the same mutants on fewer inputs per step (the oracle's rate is linear in the inputs
+    and depends on the mutants per cluster, so both arms see the same rate)."""
+    name = w.name
+    if name.startswith("vgg"):
+        return 128, 8
+    if name.startswith("resnet"):
+        return 160, 8
+    if name.startswith("mlp"):
+        return 200, 1000
+    return 400, 2000
 
 
 if __name__ == "__main__":
