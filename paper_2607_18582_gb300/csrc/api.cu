@@ -1338,6 +1338,7 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
                 S.variant = 0;
                 S.tc_small = small && env != "generic";
                 S.tc_conv = !S.tc_small && env != "gather" && tc_conv_geometry(S);
+                S.tc_wide = S.tc_conv && getenv("MURE_TC_NARROW") == nullptr && tc_wide_geometry(S);
             }
         }
         std::vector<int> wn;

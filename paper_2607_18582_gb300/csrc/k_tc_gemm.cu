@@ -45,7 +45,8 @@ constexpr int kTileM = 128;
 constexpr int kTileK = 32;             // fp32 / tf32 values per 128-byte row
 constexpr int kNA = 4;                 // producer cp.async ring depth (K-steps)
 constexpr int kNB = 3;                 // streamed weight stages
-constexpr int kSlice = 128;            // output channels per CTA
+constexpr int kSlice = 128;            // output channels per CTA (the default N slice)
+constexpr int kSliceMax = 256;         // wide slice: one N = 256 MMA per K8 step (staged convolutions)
 constexpr int kFuseClasses = 12;       // classes of an output layer fused into a dense epilogue
 constexpr int kThreads = 384;          // 4 producer + 4 epilogue + 3 MMA + weight warps
 constexpr int kEpiStride = 36;         // floats per row of an epilogue staging chunk (32 + pad)
@@ -278,6 +279,8 @@ struct TcParams {
     int acc_cols;                // tensor-memory columns of one partial accumulator
     int n_acc;                   // accumulator sets (tiles in flight): 1 or 2
     int n_stages;                // tensor-memory A stages (<= kMaxNT), from column a_col
+    int slice_w;                 // output channels per CTA: kSlice, or kSliceMax for a wide slice
+    int nb;                      // streamed weight stages (<= kNB)
     int a_col;
     int *err;
     long long spin;              // wait limit in SM cycles (0: the default, about a second)
@@ -592,20 +595,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     __shared__ __align__(8) uint64_t bar_alanded[kNA], bar_afree[kNA];
     __shared__ uint32_t tmem_sh;
     __shared__ WaitCtl abort_sh;
-    __shared__ float bias_sh[kSlice];
+    __shared__ float bias_sh[kSliceMax];
     __shared__ __align__(16) float epi_stage[4][32 * kEpiStride];   // per epilogue warp: 32 rows x 32 values
     __shared__ float *epi_ptr[4][32];                               // per epilogue warp: each row's output
     volatile WaitCtl *abort_flag = &abort_sh;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t sbase = (smem_u32(smraw) + 1023u) & ~1023u;
-    const int n_base = blockIdx.y * kSlice;
-    const int Nt = min(kSlice, p.Np - n_base);              // a multiple of 16
+    const int n_base = blockIdx.y * p.slice_w;
+    const int Nt = min(p.slice_w, p.Np - n_base);           // a multiple of 16
     constexpr int planes = THREE ? 2 : 1;
     const uint32_t b_step = (uint32_t)(planes * Nt * 128);  // one K-step of the weight slice
     const int nK = p.Kp / kTileK;
     const uint32_t b_region = sbase;
-    const uint32_t a_region = sbase + (p.b_resident ? (uint32_t)nK * b_step : (uint32_t)kNB * b_step);
+    const uint32_t a_region = sbase + (p.b_resident ? (uint32_t)nK * b_step : (uint32_t)p.nb * b_step);
     const uint32_t ov_region = a_region + kNA * kStageA;    // kNA overlay slots (with an overlay)
     const uint32_t cv_region = a_region;                    // MODE 3: the staging ring
     const uint32_t cv_buf_bytes = MODE == 3 ? (uint32_t)p.cv_imgs * p.cv_img_bytes : 0u;
@@ -630,7 +633,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             asm volatile("st.shared.f32 [%0], %1;" ::"r"(fw_region + 4 * i), "f"(wv) : "memory");
         }
     }
-    for (int n = threadIdx.x; n < kSlice; n += kThreads) {
+    for (int n = threadIdx.x; n < kSliceMax; n += kThreads) {
         if (MODE == 2) bias_sh[n] = n < SmallConv::N ? p.b[n % SmallConv::OC] : 0.f;
         else bias_sh[n] = n_base + n < p.N ? p.b[n_base + n] : 0.f;
     }
@@ -1293,7 +1296,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     }
                     if (++own == nmma) own = 0;
                     if (++t == p.n_stages) { t = 0; ++t_wraps; }
-                    if (!p.b_resident && ++sb == kNB) { sb = 0; ++b_wraps; }
+                    if (!p.b_resident && ++sb == p.nb) { sb = 0; ++b_wraps; }
                 }
                 if (!ok) break;
                 mma_commit(smem_u32(&bar_accfull[a]));
@@ -1352,8 +1355,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     }
                 }
                 if (jb < n_b) {
-                    const int sb = (int)(jb % kNB);
-                    const int64_t use = jb / kNB;
+                    const int sb = (int)(jb % p.nb);
+                    const int64_t use = jb / p.nb;
                     if (use == 0 || mbar_try(smem_u32(&bar_bempty[sb]), (uint32_t)((use - 1) & 1))) {
                         mbar_expect_tx(smem_u32(&bar_bfull[sb]), b_step);
                         bulk_g2s(b_region + (uint32_t)sb * b_step, (const unsigned char *)wslice + (size_t)(jb % nK) * b_step,
@@ -1376,8 +1379,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             // the copies still in flight land before the shared memory is released
             for (int64_t jj = jc > p.cv_nbuf ? jc - p.cv_nbuf : 0; jj < jc; ++jj)
                 wait_phase_drain(smem_u32(&bar_landed[jj % p.cv_nbuf]), (uint32_t)((jj / p.cv_nbuf) & 1));
-            for (int64_t jj = jb > kNB ? jb - kNB : 0; jj < jb; ++jj)
-                wait_phase_drain(smem_u32(&bar_bfull[(int)(jj % kNB)]), (uint32_t)((jj / kNB) & 1));
+            for (int64_t jj = jb > p.nb ? jb - p.nb : 0; jj < jb; ++jj)
+                wait_phase_drain(smem_u32(&bar_bfull[(int)(jj % p.nb)]), (uint32_t)((jj / p.nb) & 1));
         } else if (lane == 0) {
             if (p.b_resident) {
                 const uint32_t bytes = (uint32_t)nK * b_step;
@@ -1395,11 +1398,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     bulk_g2s(b_region + (uint32_t)sb * b_step, (const unsigned char *)wslice + (size_t)kt * b_step,
                              b_step, smem_u32(&bar_bfull[sb]));
                     if (++kt == nK) kt = 0;
-                    if (++sb == kNB) { sb = 0; ++wraps; }
+                    if (++sb == p.nb) { sb = 0; ++wraps; }
                 }
                 // the copies still in flight land before the shared memory is released
-                for (int64_t jj = std::max<int64_t>(0, j - kNB); jj < j; ++jj)
-                    wait_phase_drain(smem_u32(&bar_bfull[(int)(jj % kNB)]), (uint32_t)((jj / kNB) & 1));
+                for (int64_t jj = std::max<int64_t>(0, j - p.nb); jj < j; ++jj)
+                    wait_phase_drain(smem_u32(&bar_bfull[(int)(jj % p.nb)]), (uint32_t)((jj / p.nb) & 1));
             }
         }
         if constexpr (MODE == 2) {
@@ -1441,7 +1444,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
 // perm_ic > 0 (the staged convolution): K-step kc holds channels 32 (kc / taps) .. +31
 // of filter tap kc mod taps, i.e. the K order (chunk, tap, channel) of its producers.
 __global__ void k_swizzle_weights(const float *__restrict__ W, int N, int K, int Np, int Kp, int planes,
-                                  int64_t slice_floats, float *out, int perm_ic, int taps)
+                                  int64_t slice_floats, float *out, int perm_ic, int taps, int slice_w)
 {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= (int64_t)Np * Kp) return;
@@ -1453,7 +1456,7 @@ __global__ void k_swizzle_weights(const float *__restrict__ W, int N, int K, int
     }
     const float w = (n < N && k < K) ? W[(int64_t)n * K + ks] : 0.f;
     const float h = tf32_rna(w);
-    const int s = n / kSlice, nl = n % kSlice, Nt = min(kSlice, Np - s * kSlice);
+    const int s = n / slice_w, nl = n % slice_w, Nt = min(slice_w, Np - s * slice_w);
     const int kc = k / kTileK, kk = k % kTileK;
     const int64_t chunk = (int64_t)s * slice_floats + (int64_t)kc * planes * Nt * kTileK;
     const int64_t off = (sw128_off(nl, kk >> 2) >> 2) + (kk & 3);
@@ -1553,12 +1556,20 @@ __global__ void k_expand_window_weights(const float *__restrict__ W, float *out)
                  : 0.f;
 }
 
+// Output channels per CTA: one wide N = 256 slice for staged convolutions of exactly
+// 256 outputs (the MMA's tensor work per K-step then exceeds its issue cost), else
+// slices of 128.
+static int slice_width(const Stage &S) { return S.tc_wide ? kSliceMax : kSlice; }
+
 int64_t tc_weight_floats(const Stage &S)
 {
     const int Np = round_up16(gemm_n(S)), Kp = round_up32(gemm_k(S)), planes = S.tc == 1 ? 2 : 1;
-    const int64_t slice = (int64_t)planes * kSlice * Kp;
-    return slice * ((Np + kSlice - 1) / kSlice);
+    const int sw = slice_width(S);
+    const int64_t slice = (int64_t)planes * sw * Kp;
+    return slice * ((Np + sw - 1) / sw);
 }
+
+int tc_wide_geometry(const Stage &S) { return S.tc_conv && round_up16(S.oc) == kSliceMax; }
 
 // tmp: scratch of SmallConv::N * SmallConv::K floats for the small-image mode (else unused).
 int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t s)
@@ -1575,8 +1586,8 @@ int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t 
     }
     cudaMemsetAsync(out, 0, tc_weight_floats(S) * sizeof(float), s);
     k_swizzle_weights<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(W, N, K, Np, Kp, planes,
-                                                                   (int64_t)planes * kSlice * Kp, out,
-                                                                   S.tc_conv ? S.ic : 0, S.kh * S.kw);
+                                                                   (int64_t)planes * slice_width(S) * Kp, out,
+                                                                   S.tc_conv ? S.ic : 0, S.kh * S.kw, slice_width(S));
     return launches;
 }
 
@@ -1608,14 +1619,15 @@ static int mma_gap(int nK, int m)
 static void tc_config(TcParams &p, int nt_max, bool three)
 {
     p.acc_cols = round_up32(nt_max);
-    p.n_acc = 2;
+    // a wide slice's accumulator takes half of tensor memory: one set
+    p.n_acc = p.acc_cols > 128 ? 1 : 2;
     p.a_col = 256;
     p.n_stages = three ? 4 : 8;
     // An issuing warp waits on a ring slot's barrier by the parity of the slot's use
     // count, which names the right phase only while the warp's consecutive K-steps are
     // at most a ring's depth apart; every warp also has a K-step in every tile.
-    const int nK = p.Kp / kTileK, depth = p.b_resident ? p.n_stages : std::min(p.n_stages, kNB);
-    int m = std::max(1, std::min({3, 256 / (2 * p.acc_cols), nK}));
+    const int nK = p.Kp / kTileK, depth = p.b_resident ? p.n_stages : std::min(p.n_stages, p.nb);
+    int m = std::max(1, std::min({3, 256 / (p.n_acc * p.acc_cols), nK}));
     while (m > 1 && mma_gap(nK, m) > depth) --m;
     p.n_mma = m;
 }
@@ -1719,7 +1731,8 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     const bool three = S.tc == 1;
     const int planes = three ? 2 : 1;
     p.Wsw = S.Wtc;
-    p.w_slice_floats = (int64_t)planes * kSlice * p.Kp;
+    p.slice_w = slice_width(S);
+    p.w_slice_floats = (int64_t)planes * p.slice_w * p.Kp;
     p.b = S.b;
     p.act1 = S.act1; p.has_add = S.has_add; p.act2 = S.act2;
     p.skip = skip.p; p.skip_stride = skip.stride; p.skip_per_input = skip.per_input;
@@ -1734,11 +1747,13 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     p.err = S.err;
     p.spin = S.wait_limit ? *S.wait_limit : 0;
     // shared memory: the weights (whole slice, or kNB K-steps), then the producer ring
-    const int nt_max = std::min(kSlice, p.Np);
+    const int nt_max = std::min(p.slice_w, p.Np);
     const size_t b_step = (size_t)planes * nt_max * 128;
     const size_t slice_bytes = b_step * (p.Kp / kTileK);
     p.b_resident = slice_bytes <= (S.tc_small ? 112 : 96) * 1024;
-    const size_t b_bytes = p.b_resident ? slice_bytes : kNB * b_step;
+    // a wide slice streams 64 KiB per K-step: two stages in flight
+    p.nb = p.slice_w > kSlice ? 2 : kNB;
+    const size_t b_bytes = p.b_resident ? slice_bytes : p.nb * b_step;
     // at least 116 KiB so that one CTA (holding all 512 tensor-memory columns) runs per SM
     size_t a_bytes = S.tc_small ? (size_t)SmallConv::BYTES
                                 : (size_t)kNA * kStageA + (p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0);
@@ -1787,7 +1802,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
         cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
         if (n_sm <= 0) n_sm = 148;
     }
-    const int ny = (p.Np + kSlice - 1) / kSlice;
+    const int ny = (p.Np + p.slice_w - 1) / p.slice_w;
     const dim3 grid((unsigned)std::max<int64_t>(1, std::min<int64_t>(tiles, std::max(1, n_sm / ny))), (unsigned)ny);
     auto go = [&](auto kern) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -1853,9 +1868,10 @@ int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_input
                                                                          dw.colq, dw.colj);
     k_swizzle_weights<<<(unsigned)(((int64_t)Np * Kp + 255) / 256), 256, 0, s>>>(dw.filt, Np, K, Np, Kp, planes,
                                                                                (int64_t)planes * kSlice * Kp, dw.swz,
-                                                                               S.tc_conv ? S.ic : 0, S.kh * S.kw);
+                                                                               S.tc_conv ? S.ic : 0, S.kh * S.kw, kSlice);
     Stage D = S;
     D.oc = Np;
+    D.tc_wide = 0;   // the slot filters are laid out in slices of 128
     D.tc = precision == MURE_PREC_TF32X3 ? 1 : 2;
     D.tc_small = 0;
     D.Wtc = dw.swz;

@@ -94,3 +94,26 @@ def test_reference_arm_line_single_rank():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
     assert d["config"]["workload"].startswith("mlp")
+
+
+def test_slices_flops_and_cache_bytes():
+    """The step slices partition the table; the analytic FLOPs follow Lemma 4's cost
+    model (vanilla - memo = the prefixes); the cache size counts every cached row."""
+    w = wl.workload("vgg", 8, 400)
+    sl = bench.table_slices(len(w.table), 20)
+    assert sorted(np.concatenate(sl).tolist()) == list(range(400))
+    assert max(len(x) for x in sl) - min(len(x) for x in sl) <= 1
+    memo, van = bench.analytic_flops(w.model, w.table)
+    L = w.model.n_layers()
+    macs = [w.model.layer_macs(v) for v in range(L)]
+    prefix = sum(2 * sum(macs[:int(l) + 1]) for l in w.table.layer)
+    assert van - memo == pytest.approx(prefix)
+    assert 0 < memo < van
+    # a table of first-layer NEB mutants: the whole network but the first layer
+    t = wl.table_from_rows([(0, "NEB", [0], 0.0, 0)])
+    m1, v1 = bench.analytic_flops(w.model, t)
+    assert m1 == 2 * sum(macs[1:]) and v1 == 2 * sum(macs)
+    per = bench.cache_bytes(w.model, 64) / 64
+    # input 3072 + z 65536 per 32x32x64 map ... at least the inputs and outputs of every layer
+    assert per > 4 * sum(w.model.layer_width(v) for v in range(L))
+    assert bench.cache_bytes(w.model, 1) == bench.cache_bytes(w.model, 64)   # inputs padded to 64
