@@ -609,7 +609,12 @@ def main():
         oracle.build()
         threads = os.cpu_count() or 1
         n_mut, n_in = cpu_sample_size(w)
-        rate, dt, sample, agree = cpu_oracle_rate(w, n_mut, n_in, threads, gpu_kill=kill_dev.cpu().numpy())
+        # kill rows are stored slice after slice: put them back in table order
+        kd = kill_dev.cpu().numpy()
+        kill_table = np.empty_like(kd)
+        for j, ix in enumerate(slices):
+            kill_table[ix] = kd[int(off[j]):int(off[j + 1])]
+        rate, dt, sample, agree = cpu_oracle_rate(w, n_mut, n_in, threads, gpu_kill=kill_table)
         out["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
                                "seconds": dt}
         # kill verdicts of the timed GPU run against the oracle's on the same sample

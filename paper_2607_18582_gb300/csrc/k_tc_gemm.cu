@@ -293,13 +293,14 @@ struct TcParams {
     // MODE 3 (staged convolution): each tile's input rows with their zero border, 32
     // channels at a time, land by tensor-map copies in a ring of cv_nbuf buffers; the
     // producers gather every tap's 32 values from there.  K order: (chunk, tap, channel)
-    int cv_taps;                 // K-steps per chunk (one filter tap each)
-    int cv_nchunk;               // chunks of 32 input channels
+    int cv_cw;                   // channels per chunk: 32, or 16 (a K-step then holds two taps)
+    int cv_taps;                 // K-steps per chunk
+    int cv_nchunk;               // chunks of cv_cw input channels
     int cv_imgs, cv_rows;        // batch rows per tile; output rows per tile and batch row
     int cv_hw, cv_hh;            // staged width and height (input pixels, border included)
     uint32_t cv_img_bytes;       // one batch row's staged chunk in shared memory
     int cv_nbuf;
-    CUtensorMap tmap_x;          // the input rows as [row][ih][iw][ic]: boxes {32, cv_hw, cv_hh, 1}
+    CUtensorMap tmap_x;          // the input rows as [row][ih][iw][ic]: boxes {cv_cw, cv_hw, cv_hh, 1}
 };
 
 // Per producer ring slot, the overlay values of a row's K-step: up to kOvMax
@@ -772,10 +773,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 if (++b == G::NBUF) { b = 0; ++uses; }
             }
         } else if constexpr (MODE == 3) {
-            // the tile's staged input rows, one 32-channel chunk at a time (zero border
+            // the tile's staged input rows, one chunk of channels at a time (zero border
             // included, overlay written in by warp 10): this thread gathers its GEMM
-            // row's 32 values of each filter tap from the chunk, 16 bytes per load, in
-            // the 128-byte swizzle of the copies (line l holds chunk j at j ^ (l mod 8))
+            // row's values of each filter tap from the chunk, 16 bytes per load, in the
+            // 128-byte swizzle of the copies (byte b of the buffer sits at b ^ ((b >> 3)
+            // & 0x70)); a K-step is one tap of 32 channels or two taps of 16
             const bool fin = p.ov.patch != nullptr;
             bool ok = true;
             int64_t job = 0;
@@ -795,18 +797,31 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         break;
                     }
                     const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + im * p.cv_img_bytes;
-                    int ky = 0, kx = 0;
-                    for (int tap = 0; tap < p.cv_taps; ++tap) {
-                        const uint32_t line = (uint32_t)(line0 + ky * p.cv_hw + kx);
-                        const uint32_t lb = base + line * 128u, sw = line & 7u;
+                    const int ntap = p.kh * p.kw;
+                    const uint32_t lbytes = (uint32_t)p.cv_cw * 4u;
+                    int ky = 0, kx = 0, tap = 0;
+                    for (int ks = 0; ks < p.cv_taps; ++ks) {
                         float v[kTileK];
 #pragma unroll
-                        for (int cc = 0; cc < kTileK / 4; ++cc)
-                            asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
-                                         : "=f"(v[4 * cc]), "=f"(v[4 * cc + 1]), "=f"(v[4 * cc + 2]), "=f"(v[4 * cc + 3])
-                                         : "r"(lb + ((((uint32_t)cc) ^ sw) << 4)));
-                        if (!push(v)) { ok = false; break; }
+                        for (int cc = 0; cc < kTileK / 4; ++cc) {
+                            // 16-byte chunk cc: its tap (a new one every cv_cw / 4 chunks)
+                            if (cc > 0 && (cc * 4) % p.cv_cw == 0) {
+                                ++tap;
+                                if (++kx == p.kw) { kx = 0; ++ky; }
+                            }
+                            if (tap < ntap) {
+                                const uint32_t line = (uint32_t)(line0 + ky * p.cv_hw + kx);
+                                const uint32_t lin = line * lbytes + (uint32_t)((cc * 4) % p.cv_cw) * 4u;
+                                asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                                             : "=f"(v[4 * cc]), "=f"(v[4 * cc + 1]), "=f"(v[4 * cc + 2]), "=f"(v[4 * cc + 3])
+                                             : "r"(base + (lin ^ ((lin >> 3) & 0x70u))));
+                            } else {
+                                v[4 * cc] = v[4 * cc + 1] = v[4 * cc + 2] = v[4 * cc + 3] = 0.f;
+                            }
+                        }
+                        ++tap;
                         if (++kx == p.kw) { kx = 0; ++ky; }
+                        if (!push(v)) { ok = false; break; }
                     }
                     // every gather of the chunk has been consumed by push: the buffer is free
                     __syncwarp();
@@ -1234,16 +1249,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         const float *prow = p.ov.patch + row * p.ov.row_stride;
                         const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + (uint32_t)im * p.cv_img_bytes;
                         for (int q = 0; q < k; ++q) {
-                            const int jl = ids[q] - c * kTileK;
-                            if (jl < 0 || jl >= kTileK) continue;
+                            const int jl = ids[q] - c * p.cv_cw;
+                            if (jl < 0 || jl >= p.cv_cw) continue;
                             const float *pq = prow + (int64_t)q * p.ov.cells;
                             for (int cell = lane; cell < ncell; cell += 32) {
                                 const int hy = cell / p.cv_hw, hx = cell - hy * p.cv_hw;
                                 const int iy = oy0 - p.pad + hy, ix = hx - p.pad;
                                 if ((unsigned)iy >= (unsigned)p.ih || (unsigned)ix >= (unsigned)p.iw) continue;
-                                const uint32_t a = base + (uint32_t)cell * 128u +
-                                                   ((((uint32_t)jl >> 2) ^ ((uint32_t)cell & 7u)) << 4) + ((uint32_t)jl & 3u) * 4u;
-                                asm volatile("st.shared.f32 [%0], %1;" ::"r"(a), "f"(__ldg(pq + iy * p.iw + ix)) : "memory");
+                                const uint32_t lin = (uint32_t)cell * (uint32_t)p.cv_cw * 4u + (uint32_t)jl * 4u;
+                                asm volatile("st.shared.f32 [%0], %1;" ::"r"(base + (lin ^ ((lin >> 3) & 0x70u))),
+                                             "f"(__ldg(pq + iy * p.iw + ix))
+                                             : "memory");
                             }
                         }
                     }
@@ -1313,7 +1329,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             // and the weight K-steps (released by the MMAs)
             const int64_t n_jobs = my_tiles * p.cv_nchunk;
             const int64_t n_b = p.b_resident ? 0 : total;
-            const uint32_t box_bytes = (uint32_t)p.cv_hw * p.cv_hh * 128u;
+            const uint32_t box_bytes = (uint32_t)p.cv_hw * p.cv_hh * (uint32_t)p.cv_cw * 4u;
             const uint64_t tmap = reinterpret_cast<uint64_t>(&p.tmap_x);
             if (p.b_resident) {
                 const uint32_t bytes = (uint32_t)nK * b_step;
@@ -1347,7 +1363,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                                 "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes "
                                 "[%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(cv_region + (uint32_t)b * cv_buf_bytes +
                                                                               (uint32_t)im * p.cv_img_bytes),
-                                "l"(tmap), "r"(c * kTileK), "r"(-p.pad), "r"(oy0 - p.pad), "r"(src), "r"(bar)
+                                "l"(tmap), "r"(c * p.cv_cw), "r"(-p.pad), "r"(oy0 - p.pad), "r"(src), "r"(bar)
                                 : "memory");
                         }
                         ++jc;
@@ -1485,13 +1501,14 @@ int tc_small_geometry(const Stage &S)
 // (maps of >= 128 positions) or whole maps of several batch rows; the staged input is
 // the rows they read, zero border included, one 32-channel chunk per buffer.
 struct ConvTile {
-    int imgs, rows, hw, hh;
+    int imgs, rows, hw, hh, cw;
     uint32_t img_bytes;
 };
 
 static bool conv_tile(const Stage &S, ConvTile &t)
 {
-    if (S.kind != MURE_NODE_CONV2D || S.stride != 1 || S.ic % kTileK != 0) return false;
+    if (S.kind != MURE_NODE_CONV2D || S.stride != 1 || (S.ic % kTileK != 0 && S.ic != 16)) return false;
+    t.cw = S.ic == 16 ? 16 : kTileK;
     if (S.pool && ((S.oh & 1) || (S.ow & 1))) return false;
     const int P = S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
     if (P >= kTileM) {
@@ -1508,7 +1525,7 @@ static bool conv_tile(const Stage &S, ConvTile &t)
     t.hw = S.ow + S.kw - 1;
     t.hh = t.rows + S.kh - 1;
     if (t.hw > 256 || t.hh > 256) return false;
-    t.img_bytes = (uint32_t)((t.hw * t.hh * 128 + 1023) & ~1023);
+    t.img_bytes = (uint32_t)((t.hw * t.hh * t.cw * 4 + 1023) & ~1023);
     // at least two buffers beside the streamed weights (three K-steps of 128 channels)
     return (size_t)t.imgs * t.img_bytes <= 48 * 1024;
 }
@@ -1587,7 +1604,8 @@ int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t 
     cudaMemsetAsync(out, 0, tc_weight_floats(S) * sizeof(float), s);
     k_swizzle_weights<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(W, N, K, Np, Kp, planes,
                                                                    (int64_t)planes * slice_width(S) * Kp, out,
-                                                                   S.tc_conv ? S.ic : 0, S.kh * S.kw, slice_width(S));
+                                                                   S.tc_conv && S.ic > kTileK ? S.ic : 0, S.kh * S.kw,
+                                                                   slice_width(S));
     return launches;
 }
 
@@ -1679,7 +1697,7 @@ static bool conv_x_tensor_map(const Stage &S, Src x, RowMap rm, const ConvTile &
     const int64_t rows = x.per_input ? rm.t0 + rm.T : rm.R;
     const cuuint64_t dims[4] = {(cuuint64_t)S.ic, (cuuint64_t)S.iw, (cuuint64_t)S.ih, (cuuint64_t)rows};
     const cuuint64_t strides[3] = {(cuuint64_t)S.ic * 4, (cuuint64_t)S.iw * S.ic * 4, (cuuint64_t)x.stride * 4};
-    const cuuint32_t box[4] = {(cuuint32_t)kTileK, (cuuint32_t)t.hw, (cuuint32_t)t.hh, 1};
+    const cuuint32_t box[4] = {(cuuint32_t)t.cw, (cuuint32_t)t.hw, (cuuint32_t)t.hh, 1};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     return enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float *>(x.p), dims, strides, box, estr,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
@@ -1770,8 +1788,9 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
             cudaMemcpyAsync(S.err, &unsupported, sizeof(int), cudaMemcpyHostToDevice, s);
             return 0;
         }
-        p.cv_taps = S.kh * S.kw;
-        p.cv_nchunk = S.ic / kTileK;
+        p.cv_cw = ct.cw;
+        p.cv_taps = (S.kh * S.kw * ct.cw + kTileK - 1) / kTileK;
+        p.cv_nchunk = S.ic / ct.cw;
         p.cv_imgs = ct.imgs;
         p.cv_rows = ct.rows;
         p.cv_hw = ct.hw;
@@ -1868,7 +1887,8 @@ int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_input
                                                                          dw.colq, dw.colj);
     k_swizzle_weights<<<(unsigned)(((int64_t)Np * Kp + 255) / 256), 256, 0, s>>>(dw.filt, Np, K, Np, Kp, planes,
                                                                                (int64_t)planes * kSlice * Kp, dw.swz,
-                                                                               S.tc_conv ? S.ic : 0, S.kh * S.kw, kSlice);
+                                                                               S.tc_conv && S.ic > kTileK ? S.ic : 0,
+                                                                               S.kh * S.kw, kSlice);
     Stage D = S;
     D.oc = Np;
     D.tc_wide = 0;   // the slot filters are laid out in slices of 128
