@@ -293,14 +293,15 @@ struct TcParams {
     // MODE 3 (staged convolution): each tile's input rows with their zero border, 32
     // channels at a time, land by tensor-map copies in a ring of cv_nbuf buffers; the
     // producers gather every tap's 32 values from there.  K order: (chunk, tap, channel)
-    int cv_cw;                   // channels per chunk: 32, or 16 (a K-step then holds two taps)
+    int cv_cw;                   // channels per chunk: 32, or 16 (a K-step then holds two taps;
+                                 // the copies still stage 32-channel lines, the upper 16 zero-filled)
     int cv_taps;                 // K-steps per chunk
     int cv_nchunk;               // chunks of cv_cw input channels
     int cv_imgs, cv_rows;        // batch rows per tile; output rows per tile and batch row
     int cv_hw, cv_hh;            // staged width and height (input pixels, border included)
     uint32_t cv_img_bytes;       // one batch row's staged chunk in shared memory
     int cv_nbuf;
-    CUtensorMap tmap_x;          // the input rows as [row][ih][iw][ic]: boxes {cv_cw, cv_hw, cv_hh, 1}
+    CUtensorMap tmap_x;          // the input rows as [row][ih][iw][ic]: boxes {32, cv_hw, cv_hh, 1}
 };
 
 // Per producer ring slot, the overlay values of a row's K-step: up to kOvMax
@@ -774,10 +775,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             }
         } else if constexpr (MODE == 3) {
             // the tile's staged input rows, one chunk of channels at a time (zero border
-            // included, overlay written in by warp 10): this thread gathers its GEMM
-            // row's values of each filter tap from the chunk, 16 bytes per load, in the
-            // 128-byte swizzle of the copies (byte b of the buffer sits at b ^ ((b >> 3)
-            // & 0x70)); a K-step is one tap of 32 channels or two taps of 16
+            // included, overlay written in by warp 10), one 128-byte line per pixel:
+            // this thread gathers its GEMM row's values of each filter tap from the
+            // chunk, 16 bytes per load, in the 128-byte swizzle of the copies (byte b of
+            // the buffer sits at b ^ ((b >> 3) & 0x70)); a K-step is one tap of 32
+            // channels or two taps of 16
             const bool fin = p.ov.patch != nullptr;
             bool ok = true;
             int64_t job = 0;
@@ -798,7 +800,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     }
                     const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + im * p.cv_img_bytes;
                     const int ntap = p.kh * p.kw;
-                    const uint32_t lbytes = (uint32_t)p.cv_cw * 4u;
                     int ky = 0, kx = 0, tap = 0;
                     for (int ks = 0; ks < p.cv_taps; ++ks) {
                         float v[kTileK];
@@ -811,7 +812,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                             }
                             if (tap < ntap) {
                                 const uint32_t line = (uint32_t)(line0 + ky * p.cv_hw + kx);
-                                const uint32_t lin = line * lbytes + (uint32_t)((cc * 4) % p.cv_cw) * 4u;
+                                const uint32_t lin = line * 128u + (uint32_t)((cc * 4) % p.cv_cw) * 4u;
                                 asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
                                              : "=f"(v[4 * cc]), "=f"(v[4 * cc + 1]), "=f"(v[4 * cc + 2]), "=f"(v[4 * cc + 3])
                                              : "r"(base + (lin ^ ((lin >> 3) & 0x70u))));
@@ -1256,7 +1257,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                                 const int hy = cell / p.cv_hw, hx = cell - hy * p.cv_hw;
                                 const int iy = oy0 - p.pad + hy, ix = hx - p.pad;
                                 if ((unsigned)iy >= (unsigned)p.ih || (unsigned)ix >= (unsigned)p.iw) continue;
-                                const uint32_t lin = (uint32_t)cell * (uint32_t)p.cv_cw * 4u + (uint32_t)jl * 4u;
+                                const uint32_t lin = (uint32_t)cell * 128u + (uint32_t)jl * 4u;
                                 asm volatile("st.shared.f32 [%0], %1;" ::"r"(base + (lin ^ ((lin >> 3) & 0x70u))),
                                              "f"(__ldg(pq + iy * p.iw + ix))
                                              : "memory");
@@ -1329,7 +1330,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             // and the weight K-steps (released by the MMAs)
             const int64_t n_jobs = my_tiles * p.cv_nchunk;
             const int64_t n_b = p.b_resident ? 0 : total;
-            const uint32_t box_bytes = (uint32_t)p.cv_hw * p.cv_hh * (uint32_t)p.cv_cw * 4u;
+            const uint32_t box_bytes = (uint32_t)p.cv_hw * p.cv_hh * 128u;
             const uint64_t tmap = reinterpret_cast<uint64_t>(&p.tmap_x);
             if (p.b_resident) {
                 const uint32_t bytes = (uint32_t)nK * b_step;
@@ -1525,7 +1526,7 @@ static bool conv_tile(const Stage &S, ConvTile &t)
     t.hw = S.ow + S.kw - 1;
     t.hh = t.rows + S.kh - 1;
     if (t.hw > 256 || t.hh > 256) return false;
-    t.img_bytes = (uint32_t)((t.hw * t.hh * t.cw * 4 + 1023) & ~1023);
+    t.img_bytes = (uint32_t)((t.hw * t.hh * 128 + 1023) & ~1023);
     // at least two buffers beside the streamed weights (three K-steps of 128 channels)
     return (size_t)t.imgs * t.img_bytes <= 48 * 1024;
 }
@@ -1697,7 +1698,8 @@ static bool conv_x_tensor_map(const Stage &S, Src x, RowMap rm, const ConvTile &
     const int64_t rows = x.per_input ? rm.t0 + rm.T : rm.R;
     const cuuint64_t dims[4] = {(cuuint64_t)S.ic, (cuuint64_t)S.iw, (cuuint64_t)S.ih, (cuuint64_t)rows};
     const cuuint64_t strides[3] = {(cuuint64_t)S.ic * 4, (cuuint64_t)S.iw * S.ic * 4, (cuuint64_t)x.stride * 4};
-    const cuuint32_t box[4] = {(cuuint32_t)t.cw, (cuuint32_t)t.hw, (cuuint32_t)t.hh, 1};
+    // 32 channels per line whatever the chunk: a 16-channel tensor's lines get 16 zeros
+    const cuuint32_t box[4] = {(cuuint32_t)kTileK, (cuuint32_t)t.hw, (cuuint32_t)t.hh, 1};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     return enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float *>(x.p), dims, strides, box, estr,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
