@@ -1523,7 +1523,12 @@ static bool conv_tile(const Stage &S, ConvTile &t)
         t.imgs = kTileM / P;
         t.rows = S.oh;
     }
+    // staged width: the kw - 1 border columns, then padded (zero-filled columns past the
+    // image) to 4 mod 8 lines, so that the 8 lanes of a quarter warp reading a pooling
+    // window pair (lines b, b+1, b+hw, b+hw+1, b+2, ...) hit 8 different 16-byte bank
+    // groups of the 128-byte swizzle (line l's chunk c sits at c ^ (l mod 8))
     t.hw = S.ow + S.kw - 1;
+    t.hw += (4 - t.hw % 8 + 8) % 8;
     t.hh = t.rows + S.kh - 1;
     if (t.hw > 256 || t.hh > 256) return false;
     t.img_bytes = (uint32_t)((t.hw * t.hh * 128 + 1023) & ~1023);
