@@ -146,6 +146,16 @@ typedef struct {
     int64_t workspace_bytes;   /* cap on per-batch scratch (0: 8 GiB) */
     float *logits_out;         /* nullable; [n_mutants][n_inputs][n_classes]: every
                                   mutant's logits (for parity checks; slows the run) */
+    int32_t skip_unchanged;    /* mure_eval_mutants, 1: exact unchanged-row elimination.
+                                  A single-layer mutant's row whose input to the first
+                                  suffix layer (x_{l+1}: the mutated layer's output after
+                                  its activation, residual add and pooling) equals the
+                                  original bit for bit is not run: its suffix would repeat
+                                  the original forward pass, so its kill bit is 0 and its
+                                  logits are the original logits.  Results are identical
+                                  to 0 (the default); stats.n_rows_unchanged counts the
+                                  rows dropped.  Ignored by mure_eval_vanilla. */
+    int32_t reserved;          /* 0 */
 } mure_eval_opts;
 
 typedef struct {
@@ -172,6 +182,7 @@ typedef struct {
     int64_t bytes_rows;     /* activation rows the stage kernels write and the next stage
                                reads back (2 x rows x row bytes): the device-memory traffic
                                of the batched suffix beyond the algorithmic bytes */
+    int64_t n_rows_unchanged; /* rows not run by the unchanged-row elimination */
 } mure_eval_stats;
 
 #define MURE_MAX_TIMED_LAYERS 64

@@ -602,6 +602,7 @@ struct EvalCfg {
     uint32_t *kill32;
     unsigned long long *counters;   // [3]: killed, label-count sum, near ties
     float *logits_out;              // device or null
+    bool skip_unchanged = false;    // memoized: drop rows whose x_{l+1} equals the original
 };
 
 // Per-row buffers of one batch: x_s for s in [s_lo, L], plus z (vanilla) and the
@@ -614,6 +615,9 @@ struct Workspace {
     float *gap_tmp = nullptr;
     int64_t rows = 0;
     TcDeltaWs dw;              // tensor-core delta scratch (GF / WS slots of a batch)
+    // unchanged-row elimination: per-row flags, per-block counts, the compacted row
+    // list and its length
+    int32_t *uflags = nullptr, *ublk = nullptr, *lrow = nullptr, *ucount = nullptr;
 };
 
 int64_t gap_map_stride(const Stage &S)
@@ -683,6 +687,7 @@ struct Acct {
     std::vector<int64_t> flops_cls, launches_cls;   // [L + 3]
     int64_t bytes_gather = 0;
     int64_t bytes_rows = 0;
+    int64_t rows_unchanged = 0;
 };
 
 int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevTable &dt, const EvalCfg &ec,
@@ -915,6 +920,30 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         }
         return launches;
     }
+    // exact unchanged-row elimination (memoized mode): rows whose x_{l+1} equals the
+    // original bit for bit keep kill 0 and the original logits; the suffix runs on the
+    // others only, as a compacted batch (physical row r = logical row lrow[r]).  The
+    // first suffix stage must read its rows through the row map: not the window GEMM
+    // or the CUDA-core small convolution, which stage whole consecutive rows.
+    {
+        const Stage &S1 = m->st[std::min(l + 1, L - 1)];
+        const bool first_ok = l + 1 == L - 1 || !(S1.tc_small || (S1.variant > 0 && !S1.tc));
+        if (ec.skip_unchanged && l < L - 1 && first_ok) {
+            UnchangedArgs ua{ws.patch, pstride, cells_l, Sl.oc, pa.n_neurons, pa.neuron_off, pa.ids,
+                             ca->x[l + 1], m->xd[l + 1].stride, ca->x[L], m->xd[L].stride, m->n_classes, fa};
+            timed(C_DELTA, 0, [&] { return launch_unchanged(ua, rm, ws.uflags, ws.ublk, ws.lrow, ws.ucount, s); });
+            int32_t n_run = 0;
+            CK(c, cudaMemcpyAsync(&n_run, ws.ucount, sizeof n_run, cudaMemcpyDeviceToHost, s));
+            CK(c, cudaStreamSynchronize(s));
+            const int64_t valid = G * std::max<int64_t>(0, std::min<int64_t>(rm.T, ca->n_in - rm.t0));
+            acct.rows_unchanged += valid - n_run;
+            if (n_run == 0) return launches;
+            rm.R = n_run;
+            rm.lrow = ws.lrow;
+            fa.compact = 1;
+            fa.lrow = ws.lrow;
+        }
+    }
     if (l == L - 1) {
         // mutants of the output layer: the epilogue reads the logits with the overlay
         timed(C_EPI, 0, [&] { return launch_epilogue(base, m->n_classes, rm, fa, s, &ov); });
@@ -1051,6 +1080,16 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         }
         Workspace ws;
         alloc_workspace(c, sc, m, rows, vanilla, lmin, patch_floats, delta_slots, delta_k, ws, dt.has_later);
+        FAILIF(o->skip_unchanged != 0 && o->skip_unchanged != 1, c, MURE_ERR_INVALID_ARG, "skip_unchanged must be 0 or 1");
+        if (!vanilla && o->skip_unchanged) {
+            ec.skip_unchanged = true;
+            ws.uflags = sc.get<int32_t>(rows);
+            ws.ublk = sc.get<int32_t>(rows / 256 + 1);
+            ws.lrow = sc.get<int32_t>(rows);
+            ws.ucount = sc.get<int32_t>(1);
+            // compacted batches OR their kill bits in
+            CK(c, cudaMemsetAsync(ec.kill32, 0, (size_t)n * words32 * 4, s));
+        }
         int64_t launches = 0;
         Acct acct;
         acct.flops_cls.assign(m->L + 3, 0);
@@ -1116,6 +1155,7 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
         }
         st.bytes_gather = acct.bytes_gather;
         st.bytes_rows = acct.bytes_rows;
+        st.n_rows_unchanged = acct.rows_unchanged;
         float ms = 0;
         cudaEventElapsedTime(&ms, c->ev[0], c->ev[4]); st.ms_total = ms;
         cudaEventElapsedTime(&ms, c->ev[0], c->ev[1]); st.ms_expand = ms;

@@ -110,8 +110,23 @@ struct Src {
 struct RowMap {
     int64_t t0;   // first input of the tile
     int T;        // inputs per tile (multiple of 64)
-    int R;        // rows = mutants in the batch x T
+    int R;        // rows = mutants in the batch x T (or the rows left after compaction)
+    // compacted batch (unchanged rows removed): physical row r is logical row lrow[r]
+    // = g * T + input offset; null: physical = logical
+    const int32_t *lrow = nullptr;
 };
+
+// The logical row (mutant g = lr / T, input t0 + lr % T) of physical row r.  Per-input
+// sources (cached rows), the patch rows, the group tables and the kill bits are
+// indexed by it; the batch's own row buffers by r.
+__host__ __device__ __forceinline__ int64_t logical_row(const int32_t *lrow, int64_t r)
+{
+#ifdef __CUDA_ARCH__
+    return lrow ? (int64_t)__ldg(lrow + r) : r;
+#else
+    return lrow ? (int64_t)lrow[r] : r;
+#endif
+}
 
 // The mutated channels of a batch's rows of x_{l+1}, applied on top of the unmutated
 // row by the first suffix kernel: for batch mutant g = r / T and slot q < n_neurons[g],
@@ -195,6 +210,8 @@ struct FinalArgs {
     int32_t *pred_out;          // cache mode: pred0 [n_pad]
     unsigned long long *near_ties;
     int mode;                   // 0 = kill, 1 = cache build, 2 = write per-row logits only
+    int compact;                // kill mode on a compacted batch: kill bits OR-ed into a zeroed matrix
+    const int32_t *lrow;        // compacted batch: logical row of each physical row (else null)
 };
 int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cudaStream_t s,
                        const Overlay *ov = nullptr);
@@ -284,6 +301,30 @@ int launch_expand(const ExpandArgs &ea, cudaStream_t s);
 
 // Population std of each layer's weights in fp64.
 int launch_layer_std(const float *const *W, const int64_t *n, int L, double *out, cudaStream_t s);
+
+// Exact unchanged-row elimination (memoized mode).  Row r of a batch (mutant g =
+// r / T, input t0 + r % T) is unchanged when every mutated channel of its patch equals
+// the cached original x_{l+1} of its input bit for bit: its suffix then equals the
+// original forward pass, so its kill bit is 0 and its logits are the cached original
+// logits (written to logits_out when requested; its near tie is counted from them).
+// flags[r] = 1 for the rows still to run; lrow receives them in ascending order and
+// count their number.  Scratch: block_cnt of ceil(R / 256) ints.
+struct UnchangedArgs {
+    const float *patch;          // [R][kmax][cells] the delta's values
+    int64_t row_stride;
+    int cells, ch;               // cells of x_{l+1}; channels (layer l's outputs)
+    const int32_t *n_neurons;    // [G] of the batch
+    const int64_t *neuron_off;
+    const int32_t *ids;
+    const float *base;           // cached x_{l+1} rows (per input)
+    int64_t base_stride;
+    const float *logits;         // cached original logits rows (per input)
+    int64_t logits_stride;
+    int C;
+    FinalArgs fa;                // logits_out, near_ties, mutant ids, n_in
+};
+int launch_unchanged(const UnchangedArgs &ua, RowMap rm, int32_t *flags, int32_t *block_cnt, int32_t *lrow,
+                     int32_t *count, cudaStream_t s);
 
 // Score reduction: per mutant killed flag and |killingLabels|, summed.
 int launch_scores(const uint32_t *kill32, int64_t n_mut, int64_t words32, const int32_t *label, int n_classes,

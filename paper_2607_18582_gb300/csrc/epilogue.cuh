@@ -26,8 +26,9 @@ template <int CP>
 __device__ __forceinline__ void epilogue_reg(const FinalArgs &fa, int64_t t0, int T, int64_t row, bool in_range,
                                              const float (&v)[CP], int C)
 {
-    const int g = (int)(row / T);
-    const int64_t t = t0 + row % T;
+    const int64_t lr = in_range ? logical_row(fa.lrow, row) : row;
+    const int g = (int)(lr / T);
+    const int64_t t = t0 + lr % T;
     const bool valid = in_range && t < fa.n_in;
     int arg = 0;
     bool near = false;
@@ -45,7 +46,12 @@ __device__ __forceinline__ void epilogue_reg(const FinalArgs &fa, int64_t t0, in
     const unsigned kb = __ballot_sync(0xffffffffu, kill);
     const unsigned nb = __ballot_sync(0xffffffffu, near);
     const int lane = threadIdx.x & 31;
-    if (lane == 0 && in_range) {
+    if (fa.compact) {
+        // a compacted batch: the warp's rows are any (mutant, input) pairs; the matrix
+        // was zeroed, each killed row sets its own bit
+        if (kill) atomicOr(fa.kill32 + (int64_t)fa.mutant_id[g] * fa.words32 + (t >> 5), 1u << (t & 31));
+        if (lane == 0 && nb && fa.near_ties) atomicAdd(fa.near_ties, (unsigned long long)__popc(nb));
+    } else if (lane == 0 && in_range) {
         const int mid = fa.mutant_id[g];
         fa.kill32[(int64_t)mid * fa.words32 + (t >> 5)] = kb;
         if (nb && fa.near_ties) atomicAdd(fa.near_ties, (unsigned long long)__popc(nb));

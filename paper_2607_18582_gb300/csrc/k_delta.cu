@@ -478,19 +478,21 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
 __global__ void __launch_bounds__(256) k_rows_overlay(const float *__restrict__ base, int64_t base_stride,
                                                       int base_per_input, int64_t t0, int T, int R, int64_t n_floats,
                                                       const Overlay ov, float *out, int64_t out_stride,
-                                                      int rows_per_block)
+                                                      int rows_per_block, const int32_t *lrow)
 {
     extern __shared__ float sm[];  // [rows_per_block][n_floats]
     __shared__ const float *src[64];
     __shared__ float *dst[64];
     __shared__ int gidx[64];
+    __shared__ int64_t lidx[64];
     const int64_t r0 = (int64_t)blockIdx.x * rows_per_block;
     const int nr = (int)(R - r0 < rows_per_block ? R - r0 : rows_per_block);
     if (threadIdx.x < nr) {
-        const int64_t r = r0 + threadIdx.x;
-        src[threadIdx.x] = base + (base_per_input ? t0 + r % T : r) * base_stride;
+        const int64_t r = r0 + threadIdx.x, lr = logical_row(lrow, r);
+        src[threadIdx.x] = base + (base_per_input ? t0 + lr % T : r) * base_stride;
         dst[threadIdx.x] = out + r * out_stride;
-        gidx[threadIdx.x] = (int)(r / T);
+        gidx[threadIdx.x] = (int)(lr / T);
+        lidx[threadIdx.x] = lr;
     }
     __syncthreads();
     const int nf = (int)n_floats;
@@ -505,7 +507,7 @@ __global__ void __launch_bounds__(256) k_rows_overlay(const float *__restrict__ 
         const int g = gidx[rl];
         if (q >= ov.n_neurons[g]) continue;
         const int j = ov.ids[ov.neuron_off[g] + q];
-        sm[rl * nf + c * ov.ch + j] = ov.patch[(r0 + rl) * ov.row_stride + q * ov.cells + c];
+        sm[rl * nf + c * ov.ch + j] = ov.patch[lidx[rl] * ov.row_stride + q * ov.cells + c];
     }
     __syncthreads();
     for (int i = threadIdx.x; i < nr * nf; i += blockDim.x) {
@@ -516,26 +518,27 @@ __global__ void __launch_bounds__(256) k_rows_overlay(const float *__restrict__ 
 
 // Large rows: copy the base rows, then scatter the overlay (two ordered launches).
 __global__ void k_copy_rows(const float4 *__restrict__ src, int64_t src_stride4, int per_input, int64_t n4, int64_t t0,
-                            int T, int64_t R, float4 *__restrict__ dst, int64_t dst_stride4)
+                            int T, int64_t R, float4 *__restrict__ dst, int64_t dst_stride4, const int32_t *lrow)
 {
     const int64_t total = R * n4;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t r = i / n4, e = i - r * n4;
-        dst[r * dst_stride4 + e] = __ldg(src + (per_input ? t0 + r % T : r) * src_stride4 + e);
+        dst[r * dst_stride4 + e] = __ldg(src + (per_input ? t0 + logical_row(lrow, r) % T : r) * src_stride4 + e);
     }
 }
 
-__global__ void k_overlay_scatter(int64_t T, int64_t R, const Overlay ov, float *out, int64_t out_stride)
+__global__ void k_overlay_scatter(int64_t T, int64_t R, const Overlay ov, float *out, int64_t out_stride,
+                                  const int32_t *lrow)
 {
     const int64_t per_row = (int64_t)ov.kmax * ov.cells;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < R * per_row;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t r = i / per_row;
+        const int64_t r = i / per_row, lr = logical_row(lrow, r);
         const int rem = (int)(i - r * per_row), q = rem / ov.cells, c = rem - q * ov.cells;
-        const int g = (int)(r / T);
+        const int g = (int)(lr / T);
         if (q >= ov.n_neurons[g]) continue;
         const int j = ov.ids[ov.neuron_off[g] + q];
-        out[r * out_stride + (int64_t)c * ov.ch + j] = ov.patch[r * ov.row_stride + q * ov.cells + c];
+        out[r * out_stride + (int64_t)c * ov.ch + j] = ov.patch[lr * ov.row_stride + q * ov.cells + c];
     }
 }
 
@@ -551,13 +554,13 @@ int launch_rows_overlay(Src base, int64_t n_floats, RowMap rm, const Overlay &ov
             const int64_t blocks = std::min<int64_t>((total + 255) / 256, 152 * 64);
             k_copy_rows<<<(unsigned)blocks, 256, 0, s>>>(reinterpret_cast<const float4 *>(base.p), base.stride / 4,
                                                          base.per_input, n4, rm.t0, rm.T, rm.R,
-                                                         reinterpret_cast<float4 *>(out), out_stride / 4);
+                                                         reinterpret_cast<float4 *>(out), out_stride / 4, rm.lrow);
             ++launches;
         }
         const int64_t total = (int64_t)rm.R * ov.kmax * ov.cells;
         if (total > 0) {
             const int64_t blocks = std::min<int64_t>((total + 255) / 256, 152 * 64);
-            k_overlay_scatter<<<(unsigned)blocks, 256, 0, s>>>(rm.T, rm.R, ov, out, out_stride);
+            k_overlay_scatter<<<(unsigned)blocks, 256, 0, s>>>(rm.T, rm.R, ov, out, out_stride, rm.lrow);
             ++launches;
         }
         return launches;
@@ -568,7 +571,7 @@ int launch_rows_overlay(Src base, int64_t n_floats, RowMap rm, const Overlay &ov
         cudaFuncSetAttribute(k_rows_overlay, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     const int64_t blocks = (rm.R + rows_per_block - 1) / rows_per_block;
     k_rows_overlay<<<(unsigned)blocks, 256, smem, s>>>(base.p, base.stride, base.per_input, rm.t0, rm.T, rm.R,
-                                                      n_floats, ov, out, out_stride, rows_per_block);
+                                                      n_floats, ov, out, out_stride, rows_per_block, rm.lrow);
     return 1;
 }
 

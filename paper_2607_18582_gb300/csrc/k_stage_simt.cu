@@ -17,6 +17,7 @@ namespace mure {
 struct StageParams {
     const float *x; int64_t x_stride; int x_per_input;
     int64_t t0; int T; int R;
+    const int32_t *lrow;   // compacted batch: logical rows (per-input reads), else null
     int ih, iw, ic, kh, kw, stride, pad, oh, ow, oc, K;
     const float *Wt;  // [K][oc]
     const float *b;
@@ -64,7 +65,7 @@ __global__ void __launch_bounds__(256) k_stage_simt(const StageParams p)
         }
         iy0 = oy * p.stride - p.pad;
         ix0 = ox * p.stride - p.pad;
-        xrow = p.x + (p.x_per_input ? (p.t0 + row % p.T) : row) * p.x_stride;
+        xrow = p.x + (p.x_per_input ? (p.t0 + logical_row(p.lrow, row) % p.T) : row) * p.x_stride;
     }
     const int n_l = tid % BN, kb0 = (tid / BN) * B_PER;
 
@@ -140,7 +141,8 @@ __global__ void __launch_bounds__(256) k_stage_simt(const StageParams p)
             if (p.z) p.z[row * p.z_stride + (int64_t)n * (p.oh * p.ow) + oy * p.ow + ox] = z;  // channel-major
             float v = act_apply(p.act1, z);
             if (p.has_add) {
-                const float *sr = p.skip + (p.skip_per_input ? (p.t0 + row % p.T) : row) * p.skip_stride;
+                const float *sr =
+                    p.skip + (p.skip_per_input ? (p.t0 + logical_row(p.lrow, row) % p.T) : row) * p.skip_stride;
                 const float s = n < p.sk_c ? sr[((int64_t)oy * p.sk_stride * p.sk_w + ox * p.sk_stride) * p.sk_c + n] : 0.f;
                 v = act_apply(p.act2, v + s);
             }
@@ -171,7 +173,7 @@ int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
     if (S.variant > 0) return launch_conv_small(S, x, rm, z_out, z_stride, y_out, y_stride, s);
     StageParams p{};
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
-    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
+    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R; p.lrow = rm.lrow;
     p.ih = S.ih; p.iw = S.iw; p.ic = S.ic; p.kh = S.kh; p.kw = S.kw; p.stride = S.stride; p.pad = S.pad;
     p.oh = S.oh; p.ow = S.ow; p.oc = S.oc; p.K = S.K;
     p.Wt = S.Wt; p.b = S.b;
@@ -211,6 +213,7 @@ int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
 struct FinalParams {
     const float *x; int64_t x_stride; int x_per_input;
     int64_t t0; int T; int R;
+    const int32_t *lrow;   // compacted batch: logical rows (per-input reads, overlay), else null
     int F, C, act;
     const float *W;  // [C][F]
     const float *b;
@@ -223,8 +226,9 @@ struct FinalParams {
 __device__ __forceinline__ void epilogue_row(const FinalArgs &fa, int64_t t0, int T, int64_t row, bool in_range,
                                              const float *v, int C)
 {
-    const int g = (int)(row / T);
-    const int64_t t = t0 + row % T;
+    const int64_t lr = in_range ? logical_row(fa.lrow, row) : row;
+    const int g = (int)(lr / T);
+    const int64_t t = t0 + lr % T;
     const bool valid = in_range && t < fa.n_in;
     int arg = 0;
     bool near = false;
@@ -236,7 +240,12 @@ __device__ __forceinline__ void epilogue_row(const FinalArgs &fa, int64_t t0, in
     const unsigned kb = __ballot_sync(0xffffffffu, kill);
     const unsigned nb = __ballot_sync(0xffffffffu, near);
     const int lane = threadIdx.x & 31;
-    if (lane == 0 && in_range) {
+    if (fa.compact) {
+        // a compacted batch: the warp's rows are any (mutant, input) pairs; the matrix
+        // was zeroed, each killed row sets its own bit
+        if (kill) atomicOr(fa.kill32 + (int64_t)fa.mutant_id[g] * fa.words32 + (t >> 5), 1u << (t & 31));
+        if (lane == 0 && nb && fa.near_ties) atomicAdd(fa.near_ties, (unsigned long long)__popc(nb));
+    } else if (lane == 0 && in_range) {
         const int mid = fa.mutant_id[g];
         fa.kill32[(int64_t)mid * fa.words32 + (t >> 5)] = kb;
         if (nb && fa.near_ties) atomicAdd(fa.near_ties, (unsigned long long)__popc(nb));
@@ -261,8 +270,9 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
     // this row's mutated input channels (overlay), as (slot count, id pointer)
     int ov_k = 0;
     const int32_t *ov_ids = nullptr;
+    const int64_t lrow = in_range ? logical_row(p.lrow, row) : row;
     if (p.ov.patch && in_range) {
-        const int g = (int)(row / p.T);
+        const int g = (int)(lrow / p.T);
         ov_k = p.ov.n_neurons[g];
         ov_ids = p.ov.ids + p.ov.neuron_off[g];
     }
@@ -272,7 +282,8 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
     for (int c = 0; c < CP; ++c) acc[c] = 0.f;
     {
         const int64_t r = row0 + tid;
-        xrow_of[tid] = r < p.R ? p.x + (p.x_per_input ? (p.t0 + r % p.T) : r) * p.x_stride : nullptr;
+        xrow_of[tid] = r < p.R ? p.x + (p.x_per_input ? (p.t0 + logical_row(p.lrow, r) % p.T) : r) * p.x_stride
+                               : nullptr;
     }
     __syncthreads();
     for (int f0 = 0; f0 < p.F; f0 += FC) {
@@ -293,7 +304,7 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
             const int j = ov_ids[q];
             const int cfirst = f0 - j <= 0 ? 0 : (f0 - j + p.ov.ch - 1) / p.ov.ch;
             for (int c = cfirst; c < p.ov.cells && c * p.ov.ch + j < f0 + fe; ++c)
-                xs[tid][c * p.ov.ch + j - f0] = p.ov.patch[row * p.ov.row_stride + q * p.ov.cells + c];
+                xs[tid][c * p.ov.ch + j - f0] = p.ov.patch[lrow * p.ov.row_stride + q * p.ov.cells + c];
         }
         for (int fl = 0; fl < fe; ++fl) {
             const float xv = xs[tid][fl];
@@ -378,7 +389,8 @@ __global__ void __launch_bounds__(128) k_final_dense_rows(const FinalParams p)
         ws[i] = c < p.C ? __ldg(p.W + (int64_t)c * p.F + fl) : 0.f;
     }
     if (in_range) {
-        const float4 *src = reinterpret_cast<const float4 *>(p.x + (p.x_per_input ? p.t0 + row % p.T : row) * p.x_stride);
+        const int64_t lrow = logical_row(p.lrow, row);
+        const float4 *src = reinterpret_cast<const float4 *>(p.x + (p.x_per_input ? p.t0 + lrow % p.T : row) * p.x_stride);
         float4 v[kRowsF / 4];
 #pragma unroll
         for (int i = 0; i < kRowsF / 4; ++i)
@@ -387,10 +399,10 @@ __global__ void __launch_bounds__(128) k_final_dense_rows(const FinalParams p)
         for (int i = 0; i < kRowsF / 4; ++i)
             if (4 * i < p.F) *reinterpret_cast<float4 *>(xr + 4 * i) = v[i];
         if (p.ov.patch) {
-            const int g = (int)(row / p.T);
+            const int g = (int)(lrow / p.T);
             const int k = p.ov.n_neurons[g];
             const int32_t *ids = p.ov.ids + p.ov.neuron_off[g];
-            for (int q = 0; q < k; ++q) xr[ids[q]] = p.ov.patch[row * p.ov.row_stride + q];
+            for (int q = 0; q < k; ++q) xr[ids[q]] = p.ov.patch[lrow * p.ov.row_stride + q];
         }
     }
     __syncthreads();   // the weights
@@ -440,7 +452,7 @@ int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cu
     FinalParams p{};
     if (ov) p.ov = *ov;
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
-    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
+    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R; p.lrow = rm.lrow;
     p.F = S.K; p.C = S.oc; p.act = S.act1;
     p.W = S.W; p.b = S.b;
     p.fa = fa;

@@ -263,6 +263,7 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 struct TcParams {
     const float *x; int64_t x_stride; int x_per_input;
     int64_t t0; int T; int R;
+    const int32_t *lrow;         // compacted batch: logical row of each physical row, else null
     int ih, iw, ic, kh, kw, stride, pad, oh, ow;
     int P, pool, pw;             // GEMM rows per batch row (pooled maps: window-major)
     int K, Kp, N, Np;            // fan-in (padded to 32), outputs (padded to 16)
@@ -342,12 +343,15 @@ __device__ __forceinline__ RowInfo row_info(const TcParams &p, int64_t m)
             ri.ox = q % p.ow;
         }
     }
-    ri.xrow = p.x + (p.x_per_input ? p.t0 + ri.row % p.T : ri.row) * p.x_stride;
+    // per-input sources, the overlay and its group by the logical row; the batch's own
+    // row buffers by the physical row
+    const int64_t lr = logical_row(p.lrow, ri.row);
+    ri.xrow = p.x + (p.x_per_input ? p.t0 + lr % p.T : ri.row) * p.x_stride;
     if (OVERLAY && p.ov.patch) {
-        const int g = (int)(ri.row / p.T);
+        const int g = (int)(lr / p.T);
         ri.ov_k = p.ov.n_neurons[g];
         ri.ov_ids = p.ov.ids + p.ov.neuron_off[g];
-        ri.ov_patch = p.ov.patch + ri.row * p.ov.row_stride;
+        ri.ov_patch = p.ov.patch + lr * p.ov.row_stride;
         if (DENSE) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -961,7 +965,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             }
             const RowInfo ri = row_info<DENSE, false>(p, tile * kTileM + qd * 32 + lane);
             const float *srow = nullptr;
-            if (p.has_add && ri.ok) srow = p.skip + (p.skip_per_input ? p.t0 + ri.row % p.T : ri.row) * p.skip_stride;
+            if (p.has_add && ri.ok)
+                srow = p.skip + (p.skip_per_input ? p.t0 + logical_row(p.lrow, ri.row) % p.T : ri.row) * p.skip_stride;
             float *yrow = ri.ok ? p.y + ri.row * p.y_stride : nullptr;
             // unpooled outputs go through shared memory: one store instruction then
             // covers 4 rows x 128 bytes instead of 32 rows x 16 bytes
@@ -1243,7 +1248,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         break;
                     }
                     for (int im = 0; im < nimg; ++im) {
-                        const int64_t row = row0 + im;
+                        const int64_t row = logical_row(p.lrow, row0 + im);
                         const int g = (int)(row / p.T);
                         const int k = p.ov.n_neurons[g];
                         const int32_t *ids = p.ov.ids + p.ov.neuron_off[g];
@@ -1359,7 +1364,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         mbar_expect_tx(bar, (uint32_t)nimg * box_bytes);
                         for (int im = 0; im < nimg; ++im) {
                             const int64_t row = row0 + im;
-                            const int src = (int)(p.x_per_input ? p.t0 + row % p.T : row);
+                            const int src = (int)(p.x_per_input ? p.t0 + logical_row(p.lrow, row) % p.T : row);
                             asm volatile(
                                 "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes "
                                 "[%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(cv_region + (uint32_t)b * cv_buf_bytes +
@@ -1743,7 +1748,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     TcParams p{};
     const bool dense = S.kind == MURE_NODE_DENSE;
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
-    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R;
+    p.t0 = rm.t0; p.T = rm.T; p.R = rm.R; p.lrow = rm.lrow;
     p.ih = S.ih; p.iw = S.iw; p.ic = S.ic; p.kh = S.kh; p.kw = S.kw; p.stride = S.stride; p.pad = S.pad;
     p.oh = S.oh; p.ow = S.ow;
     p.pool = S.pool; p.pw = S.ow / 2;

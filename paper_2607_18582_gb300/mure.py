@@ -59,7 +59,7 @@ class _Allocator(C.Structure):
 
 class _Opts(C.Structure):
     _fields_ = [("outputs_on_device", C.c_int32), ("kernel_timing", C.c_int32), ("workspace_bytes", C.c_int64),
-                ("logits_out", C.c_void_p)]
+                ("logits_out", C.c_void_p), ("skip_unchanged", C.c_int32), ("reserved", C.c_int32)]
 
 
 class _Stats(C.Structure):
@@ -69,7 +69,7 @@ class _Stats(C.Structure):
                 ("flops", C.c_int64), ("ms_layer", C.c_double * 64), ("flops_layer", C.c_int64 * 64),
                 ("launches_layer", C.c_int64 * 64), ("ms_delta", C.c_double), ("ms_gather", C.c_double),
                 ("ms_epilogue", C.c_double), ("bytes_gather", C.c_int64), ("launches_delta", C.c_int64),
-                ("bytes_rows", C.c_int64)]
+                ("bytes_rows", C.c_int64), ("n_rows_unchanged", C.c_int64)]
 
     def as_dict(self):
         out = {}
@@ -338,7 +338,8 @@ def table_array(table):
     return arr, pool, int(table.pool.size)
 
 
-def _eval_common(n_mut, n_in, n_classes, logits, outputs_on_device, workspace_bytes, kill_out, kernel_timing=False):
+def _eval_common(n_mut, n_in, n_classes, logits, outputs_on_device, workspace_bytes, kill_out, kernel_timing=False,
+                 skip_unchanged=False):
     W64 = (n_in + 63) // 64
     if outputs_on_device:
         import torch
@@ -348,7 +349,8 @@ def _eval_common(n_mut, n_in, n_classes, logits, outputs_on_device, workspace_by
     else:
         kill = kill_out if kill_out is not None else np.zeros((max(n_mut, 1), max(W64, 1)), np.uint64)
         lg = np.zeros((n_mut, n_in, n_classes), np.float32) if logits else None
-    opts = _Opts(int(bool(outputs_on_device)), int(bool(kernel_timing)), int(workspace_bytes), _ptr(lg))
+    opts = _Opts(int(bool(outputs_on_device)), int(bool(kernel_timing)), int(workspace_bytes), _ptr(lg),
+                 int(bool(skip_unchanged)), 0)
     return kill, lg, opts, W64
 
 
@@ -361,12 +363,14 @@ def _eval_result(kill, lg, sa, sb, st, n_mut, W64, outputs_on_device):
 
 
 def mure_eval_mutants(cache: Cache, table, logits: bool = False, outputs_on_device: bool = False,
-                      workspace_bytes: int = 0, kill_out=None, kernel_timing: bool = False, arrays=None):
-    """Memoized mutation testing of `table` on the cached inputs."""
+                      workspace_bytes: int = 0, kill_out=None, kernel_timing: bool = False, arrays=None,
+                      skip_unchanged: bool = False):
+    """Memoized mutation testing of `table` on the cached inputs (skip_unchanged: the
+    exact unchanged-row elimination)."""
     arr, pool, plen = arrays if arrays is not None else table_array(table)
     n = len(table)
     kill, lg, opts, W64 = _eval_common(n, cache.n_inputs, cache.model.src.n_classes, logits, outputs_on_device,
-                                       workspace_bytes, kill_out, kernel_timing)
+                                       workspace_bytes, kill_out, kernel_timing, skip_unchanged)
     sa, sb, st = C.c_double(), C.c_double(), _Stats()
     cache.model.ctx.check(lib().mure_eval_mutants(cache.h, _ptr(arr), n, _ptr(pool), plen, C.byref(opts), _ptr(kill),
                                                   C.byref(sa), C.byref(sb), C.byref(st)))

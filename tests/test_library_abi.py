@@ -39,14 +39,31 @@ def test_library_exports_every_declared_symbol(libpath):
     assert set(mure.EXPORTS) == set(names)
 
 
-def test_struct_layouts_match_header():
+def _c_layout(tmp_path, struct, fields):
+    """sizeof and offsetof of a header struct, printed by a C program compiled against
+    include/mure.h with gcc."""
+    src = tmp_path / f"{struct}.c"
+    body = "".join(f'    printf("%zu\\n", offsetof({struct}, {f}));\n' for f in fields)
+    src.write_text(f'#include <stddef.h>\n#include <stdio.h>\n#include "mure.h"\nint main(void) {{\n'
+                   f'    printf("%zu\\n", sizeof({struct}));\n{body}    return 0;\n}}\n')
+    exe = tmp_path / f"{struct}.bin"
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.dirname(HEADER), str(src), "-o", str(exe)], check=True)
+    vals = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    return vals[0], vals[1:]
+
+
+def test_struct_layouts_match_header(tmp_path):
     from paper_2607_18582_gb300 import mure
-    assert ctypes.sizeof(mure._Node) == 10 * 4 + 2 * 8
-    assert mure.MUTANT_DTYPE.itemsize == 40
-    assert mure.MUTANT_DTYPE.fields["neuron_off"][1] == 16
-    assert mure.MUTANT_DTYPE.fields["seed"][1] == 32
-    assert ctypes.sizeof(mure._Opts) == 24
-    assert ctypes.sizeof(mure._Stats) == 4 * 8 + 6 * 8 + 64 * 8 * 3 + 3 * 8 + 3 * 8
+    for struct, cls in (("mure_node", mure._Node), ("mure_model_desc", mure._ModelDesc),
+                        ("mure_allocator", mure._Allocator), ("mure_eval_opts", mure._Opts),
+                        ("mure_eval_stats", mure._Stats)):
+        names = [f for f, _ in cls._fields_]
+        size, offs = _c_layout(tmp_path, struct, names)
+        assert ctypes.sizeof(cls) == size, struct
+        assert [getattr(cls, f).offset for f in names] == offs, struct
+    size, offs = _c_layout(tmp_path, "mure_mutant", list(mure.MUTANT_DTYPE.names))
+    assert mure.MUTANT_DTYPE.itemsize == size
+    assert [mure.MUTANT_DTYPE.fields[f][1] for f in mure.MUTANT_DTYPE.names] == offs
 
 
 def test_library_loads_and_fails_cleanly_without_gpu(libpath):
