@@ -574,6 +574,32 @@ def main():
                               "kill_matrix_identical": same,
                               "achieved_tflops": v0 * len(w.X) / tv / 1e12,
                               "analytic_flops_per_eval": v0 / len(tables[0])}
+        # exact unchanged-row elimination (rows whose first suffix input equals the
+        # original are not run): the same steps' throughput counting every row, and the
+        # share of rows dropped
+        k_u = min(len(tables), 3)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        dropped = rows_u = 0
+        t_u = 0.0
+        for k in range(k_u):
+            flush.zero_()
+            e0.record(stream)
+            cache = mure.mure_build_prefix_cache(model, X_dev)
+            ru = mure.mure_eval_mutants(cache, tables[k], outputs_on_device=True, kill_out=kill_slices[k],
+                                        arrays=arrays[k], skip_unchanged=True)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            del cache
+            t_u += e0.elapsed_time(e1) / 1e3
+            dropped += ru["stats"]["n_rows_unchanged"]
+            rows_u += ru["stats"]["n_rows"]
+        t_plain = sum(ms[i] for i in range(args.steps) if i % len(tables) < k_u) / 1e3
+        n_plain = sum(1 for i in range(args.steps) if i % len(tables) < k_u)
+        out["unchanged_rows"] = {"effective_value": rows_u / t_u, "unit": UNIT, "rows_dropped_frac": dropped / max(1, rows_u),
+                                 "steps": k_u, "plain_value_same_slices": (n_plain and
+                                     sum(len(tables[i % len(tables)]) * len(w.X) for i in range(args.steps)
+                                         if i % len(tables) < k_u) / t_plain) or None,
+                                 "counted": "every (mutant, input) row, dropped ones included, per second"}
         # the stress mix (half of the mutants on the first convolution, 0.1-10 %):
         # one slice of its table over all its inputs, after a warm-up on a few mutants
         if args.workload == "vgg" and args.n_inputs is None and args.n_mutants is None:

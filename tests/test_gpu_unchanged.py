@@ -51,8 +51,8 @@ def dead_heavy_table(model, seed):
     return wl.table_from_rows(rows)
 
 
-CASES = [("mlp", 160, "fp32"), ("lenet5", 140, "tf32x3"), ("vgg", 70, "tf32x3"), ("resnet20", 70, "tf32x3"),
-         ("resnet20", 70, "fp32")]
+CASES = [("mlp", 160, "fp32"), ("lenet5", 140, "tf32x3"), ("vgg", 48, "tf32x3"), ("resnet20", 48, "tf32x3"),
+         ("resnet20", 40, "fp32")]
 
 
 @pytest.mark.parametrize("name,n_in,prec", CASES)
