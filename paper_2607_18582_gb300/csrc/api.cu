@@ -261,11 +261,18 @@ void compile(mure_ctx *c, const mure_model_desc *d, mure_model *m)
     for (int v = 0; v < L; ++v) {
         const int nid = wn[v];
         const mure_node &n = d->nodes[nid];
-        FAILIF(n.in0 != stage_in[v], c, MURE_ERR_UNSUPPORTED, "weighted node %d does not read the previous stage", nid);
+        // a weighted node reads the previous stage's output x_v, or an earlier stage input
+        // x_s: a projection in a residual block's skip branch (Algorithm 2's graph is
+        // then not a chain), whose add must take x_v (checked below)
+        int in_src = -1;
+        for (int s2 = 0; s2 <= v; ++s2)
+            if (stage_in[s2] == n.in0) in_src = s2;
+        FAILIF(in_src < 0, c, MURE_ERR_UNSUPPORTED, "weighted node %d does not read a stage input", nid);
         used[nid] = 1;
         Stage &S = m->st[v];
         S = Stage{};
         S.kind = n.kind;
+        S.in_src = in_src;
         const Shape a = shape_of(n.in0), z = shp[nid];
         if (n.kind == MURE_NODE_CONV2D) {
             S.ih = a.h; S.iw = a.w; S.ic = a.c; S.kh = n.kh; S.kw = n.kw; S.stride = n.stride; S.pad = n.pad;
@@ -322,6 +329,8 @@ void compile(mure_ctx *c, const mure_model_desc *d, mure_model *m)
             }
             cur = u;
         }
+        FAILIF(S.in_src != v && !(S.has_add && S.skip_src == v && S.sc_stride == 1), c, MURE_ERR_UNSUPPORTED,
+               "weighted node %d reads an earlier stage input but its add does not take the previous stage", nid);
         const Shape y = shp[cur];
         S.yh = y.h; S.yw = y.w; S.yc = y.c;
         stage_in[v + 1] = cur;
@@ -735,7 +744,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         const Stage &S = m->st[v];
         acct.bytes_rows += 2 * (int64_t)rm.R * m->xd[v + 1].size * 4;
         timed(v, 2 * S.macs * rm.R, [&] {
-            return launch_stage_simt(S, xsrc(v), rm, z_out, z_stride, skip_of(S), ws.xb[v + 1], m->xd[v + 1].stride,
+            return launch_stage_simt(S, xsrc(S.in_src), rm, z_out, z_stride, skip_of(S), ws.xb[v + 1], m->xd[v + 1].stride,
                                      ws.gap_tmp, s);
         });
     };
@@ -756,7 +765,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
             f2.z_stride = ws.z_stride;
             f2.logits_rows = ws.xb[L];
             f2.x_stride = m->xd[L].stride;
-            timed(l, 2 * Sl.macs * rm.R, [&] { return launch_final_dense(Sl, xsrc(l), rm, f2, s); });
+            timed(l, 2 * Sl.macs * rm.R, [&] { return launch_final_dense(Sl, xsrc(Sl.in_src), rm, f2, s); });
         }
     }
     // the delta: values of the mutated channels of x_{l+1} (from the cached z_l in
@@ -779,7 +788,10 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     ov.n_neurons = pa.n_neurons;
     ov.neuron_off = pa.neuron_off;
     ov.ids = pa.ids;
-    bool skip_reader = false;
+    // x_{l+1} read other than as the first suffix stage's GEMM input (a later residual
+    // add, or the add of a projection in a skip branch that reads an earlier input):
+    // its rows are materialised with the patch
+    bool skip_reader = l + 1 < L && m->st[l + 1].in_src != l + 1;
     for (int v = l + 2; v < L; ++v) skip_reader |= m->st[v].has_add && m->st[v].skip_src == l + 1;
     // the window GEMM as first suffix stage applies NEB (zeros) and NS (a swap of the
     // two channels, which is the operator itself: the swapped neurons' channels are
@@ -805,18 +817,18 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     const int64_t slots = (dt.dot_prefix[g0 + G] - dt.dot_prefix[g0]) + (dt.val_prefix[g0 + G] - dt.val_prefix[g0]) -
                           (win_ops ? dt.copy_prefix[g0 + G] - dt.copy_prefix[g0] : 0);
     acct.bytes_gather += slots * rm.T * cells_l * 4;
-    acct.bytes_gather += (vanilla ? rm.R : (int64_t)rm.T) * (m->zd[l].size + (has_dot ? m->xd[l].size : 0)) * 4;
+    acct.bytes_gather += (vanilla ? rm.R : (int64_t)rm.T) * (m->zd[l].size + (has_dot ? m->xd[Sl.in_src].size : 0)) * 4;
     int delta_err = 0;
     timed(C_DELTA, delta_flops, [&] {
-        int n = launch_patch_vals(Sl, zsrc, xsrc(l), skip_of(Sl), rm, pa, kmax, ws.patch, pstride, s,
+        int n = launch_patch_vals(Sl, zsrc, xsrc(Sl.in_src), skip_of(Sl), rm, pa, kmax, ws.patch, pstride, s,
                                   dot_kernel || tc_delta, win_ops);
         if (tc_delta && has_dot) {
             // the inputs' x_l and z_l: cached rows (memoized) or the batch's first
             // mutant's recomputed rows (vanilla; the prefix up to layer l is unmutated)
-            const int d = launch_tc_delta(Sl, m->precision, zsrc, xsrc(l), rm, pa, ws.patch, pstride, ws.dw, s);
+            const int d = launch_tc_delta(Sl, m->precision, zsrc, xsrc(Sl.in_src), rm, pa, ws.patch, pstride, ws.dw, s);
             if (d < 0) delta_err = 1; else n += d;
         } else if (dot_kernel && has_dot) {
-            n += launch_patch_dot(Sl, zsrc, xsrc(l), rm, pa, kmax, ws.patch, pstride, s);
+            n += launch_patch_dot(Sl, zsrc, xsrc(Sl.in_src), rm, pa, kmax, ws.patch, pstride, s);
         }
         return n;
     });
@@ -868,7 +880,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
                 const Stage &SLast = m->st[L - 1];
                 const FinalFuse ff{SLast.W, SLast.b, SLast.oc, SLast.K, SLast.act1, fa};
                 timed(L - 2, 2 * (Sv.macs + SLast.macs) * rm.R, [&] {
-                    return launch_tc(Sv, xsrc(v), rm, nullptr, 0, skip_of(Sv), ws.xb[L - 1], m->xd[L - 1].stride,
+                    return launch_tc(Sv, xsrc(Sv.in_src), rm, nullptr, 0, skip_of(Sv), ws.xb[L - 1], m->xd[L - 1].stride,
                                      ws.gap_tmp, s, nullptr, &ff);
                 });
                 break;
@@ -893,7 +905,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
                 if (!mut) continue;
                 acct.bytes_gather += rm.R * ((int64_t)kv[v] * cells_v + m->zd[v].size + m->xd[v].size) * 4;
                 timed(C_DELTA, dfl, [&] {
-                    return launch_patch_vals(Sv, zrows, xsrc(v), skip_of(Sv), rm, pv, kv[v], ws.patch, pstride_v, s);
+                    return launch_patch_vals(Sv, zrows, xsrc(Sv.in_src), skip_of(Sv), rm, pv, kv[v], ws.patch, pstride_v, s);
                 });
                 const Src xr{ws.xb[v + 1], m->xd[v + 1].stride, 0};
                 timed(C_DELTA, 0, [&] {
@@ -906,16 +918,16 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
                 f2.z_stride = zst;
                 f2.logits_rows = ws.xb[L];
                 f2.x_stride = m->xd[L].stride;
-                timed(v, 2 * Sv.macs * rm.R, [&] { return launch_final_dense(Sv, xsrc(v), rm, f2, s); });
+                timed(v, 2 * Sv.macs * rm.R, [&] { return launch_final_dense(Sv, xsrc(Sv.in_src), rm, f2, s); });
                 acct.bytes_gather += rm.R * ((int64_t)kv[v] + m->zd[v].size + m->xd[v].size) * 4;
                 timed(C_DELTA, dfl, [&] {
-                    return launch_patch_vals(Sv, zrows, xsrc(v), skip_of(Sv), rm, pv, kv[v], ws.patch, pstride_v, s);
+                    return launch_patch_vals(Sv, zrows, xsrc(Sv.in_src), skip_of(Sv), rm, pv, kv[v], ws.patch, pstride_v, s);
                 });
                 timed(C_EPI, 0, [&] {
                     return launch_epilogue(Src{ws.xb[L], m->xd[L].stride, 0}, m->n_classes, rm, fa, s, &ovv);
                 });
             } else {
-                timed(v, 2 * Sv.macs * rm.R, [&] { return launch_final_dense(Sv, xsrc(v), rm, fa, s); });
+                timed(v, 2 * Sv.macs * rm.R, [&] { return launch_final_dense(Sv, xsrc(Sv.in_src), rm, fa, s); });
             }
         }
         return launches;
@@ -994,12 +1006,12 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     // the rest of the suffix (Algorithm 4) and the fused kill epilogue
     if (fuse && l + 2 <= L - 2) {
         for (int v = l + 2; v < L - 2; ++v) stage(v, nullptr, 0);
-        fused_last(xsrc(L - 2), nullptr);
+        fused_last(xsrc(m->st[L - 2].in_src), nullptr);
         return launches;
     }
     for (int v = l + 2; v < L - 1; ++v) stage(v, nullptr, 0);
     const Stage &SL = m->st[L - 1];
-    timed(L - 1, 2 * SL.macs * rm.R, [&] { return launch_final_dense(SL, xsrc(L - 1), rm, fa, s); });
+    timed(L - 1, 2 * SL.macs * rm.R, [&] { return launch_final_dense(SL, xsrc(SL.in_src), rm, fa, s); });
     return launches;
 }
 
@@ -1234,7 +1246,7 @@ mure_cache *build_cache(mure_model *m, const float *X, int64_t n_in, const int32
         for (int v = 0; v < L - 1; ++v) {
             const Stage &S = m->st[v];
             const Src skip = S.has_add ? Src{xs[S.skip_src], m->xd[S.skip_src].stride, 0} : Src{nullptr, 0, 0};
-            c->launches += launch_stage_simt(S, Src{xs[v], m->xd[v].stride, 0}, rm, zs[v], m->zd[v].stride, skip,
+            c->launches += launch_stage_simt(S, Src{xs[S.in_src], m->xd[S.in_src].stride, 0}, rm, zs[v], m->zd[v].stride, skip,
                                              xs[v + 1], m->xd[v + 1].stride, gap_tmp, s);
             check_launch(c);
         }

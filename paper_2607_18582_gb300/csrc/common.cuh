@@ -25,6 +25,8 @@ struct Stage {
     int K;                    // fan-in kh*kw*ic
     int act1;
     int has_add, skip_src;    // skip tensor = x_{skip_src} (stage-input index)
+    int in_src = -1;          // stage input the layer reads (x_v; an earlier x_s for a
+                              // projection in a skip branch, whose add then takes x_v)
     int sc_stride, sc_c;      // shortcut subsampling stride and source channels
     int sk_w;                 // width of the skip source tensor
     int act2;

@@ -88,9 +88,18 @@ def test_table_validation_agrees_with_oracle(oracle_mod, name):
 
 
 def test_unsupported_graphs_and_settings():
-    # a weighted layer in a skip branch (projection shortcut)
-    st, msg = mure.mure_check_descriptors(wl.resnet10())
-    assert st == UNSUPPORTED and "stage" in msg
+    # a weighted layer in a skip branch (ResNet-10's projection shortcuts) is a stage
+    # that reads an earlier stage input, its add taking the previous stage's output
+    for prec in ("fp32", "tf32x3", "tf32"):
+        assert mure.mure_check_descriptors(wl.resnet10(), precision=prec) == (OK, "")
+    # ... but not when that add skips the layer just before it (a dead branch)
+    m = wl.resnet10()
+    adds = [i for i, n in enumerate(m.nodes) if n.kind == "add"]
+    add = m.nodes[adds[1]]                      # the second block's add: (conv_b, projection)
+    conv_a = m.nodes[add.inputs[0]].inputs[0]
+    add.inputs = (conv_a, add.inputs[1])
+    st, msg = mure.mure_check_descriptors(m)
+    assert st == UNSUPPORTED and "earlier stage input" in msg
     # more classes than the output-layer kernel keeps accumulators for
     st, msg = mure.mure_check_descriptors(wl.mlp(widths=(784, 64, 40)))
     assert st == UNSUPPORTED and "n_classes" in msg
