@@ -51,10 +51,15 @@ enum {
     MURE_NODE_FLATTEN = 3,  /* reshape to a vector (no data movement in NHWC) */
     MURE_NODE_ADD = 4,      /* element-wise sum of in0 and in1 + activation */
     MURE_NODE_GAP = 5,      /* global average pooling over H and W */
-    MURE_NODE_SHORTCUT = 6  /* parameter-free residual shortcut: subsample by
+    MURE_NODE_SHORTCUT = 6, /* parameter-free residual shortcut: subsample by
                                `stride`, zero channels appended up to `cout` */
+    MURE_NODE_DWCONV = 7    /* depthwise 2-D convolution (MobileNetV2, Table 1): channel
+                               c of the output is a kh x kw filter over channel c of the
+                               input, + bias + activation; cin = cout = the input's
+                               channels, W [c][kh][kw]; neuron j = channel j, whose fan-in
+                               is its kh*kw filter */
 };
-enum { MURE_ACT_NONE = 0, MURE_ACT_RELU = 1 };
+enum { MURE_ACT_NONE = 0, MURE_ACT_RELU = 1, MURE_ACT_RELU6 = 2 /* min(max(v, 0), 6) */ };
 
 /* Mutation operators (Sec. 3.1; DeepMutation's weight-level mutators).  Neuron j of
  * a weighted layer is its output channel / output unit j (Sec. 2.1).

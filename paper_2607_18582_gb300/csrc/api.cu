@@ -169,7 +169,7 @@ struct Shape {
     int h, w, c;
 };
 
-bool weighted(int k) { return k == MURE_NODE_CONV2D || k == MURE_NODE_DENSE; }
+bool weighted(int k) { return k == MURE_NODE_CONV2D || k == MURE_NODE_DENSE || k == MURE_NODE_DWCONV; }
 
 // Output shapes of all nodes (same rules as the network definition in the header).
 std::vector<Shape> node_shapes(mure_ctx *c, const mure_model_desc *d)
@@ -187,6 +187,13 @@ std::vector<Shape> node_shapes(mure_ctx *c, const mure_model_desc *d)
                    MURE_ERR_INVALID_ARG, "node %d: bad conv geometry", v);
             o = {(a.h + 2 * n.pad - n.kh) / n.stride + 1, (a.w + 2 * n.pad - n.kw) / n.stride + 1, n.cout};
             FAILIF(o.h < 1 || o.w < 1, c, MURE_ERR_INVALID_ARG, "node %d: empty conv output", v);
+            FAILIF(!n.W || !n.b, c, MURE_ERR_INVALID_ARG, "node %d: NULL weights", v);
+            break;
+        case MURE_NODE_DWCONV:
+            FAILIF(n.cin != a.c || n.cout != a.c || n.stride < 1 || n.kh < 1 || n.kw < 1 || n.pad < 0, c,
+                   MURE_ERR_INVALID_ARG, "node %d: bad depthwise geometry", v);
+            o = {(a.h + 2 * n.pad - n.kh) / n.stride + 1, (a.w + 2 * n.pad - n.kw) / n.stride + 1, a.c};
+            FAILIF(o.h < 1 || o.w < 1, c, MURE_ERR_INVALID_ARG, "node %d: empty depthwise output", v);
             FAILIF(!n.W || !n.b, c, MURE_ERR_INVALID_ARG, "node %d: NULL weights", v);
             break;
         case MURE_NODE_DENSE:
@@ -218,7 +225,8 @@ std::vector<Shape> node_shapes(mure_ctx *c, const mure_model_desc *d)
         default:
             FAILIF(true, c, MURE_ERR_INVALID_ARG, "node %d: unknown kind %d", v, n.kind);
         }
-        FAILIF(n.act != MURE_ACT_NONE && n.act != MURE_ACT_RELU, c, MURE_ERR_INVALID_ARG, "node %d: bad activation", v);
+        FAILIF(n.act != MURE_ACT_NONE && n.act != MURE_ACT_RELU && n.act != MURE_ACT_RELU6, c, MURE_ERR_INVALID_ARG,
+               "node %d: bad activation", v);
         s[v] = o;
     }
     return s;
@@ -274,13 +282,14 @@ void compile(mure_ctx *c, const mure_model_desc *d, mure_model *m)
         S.kind = n.kind;
         S.in_src = in_src;
         const Shape a = shape_of(n.in0), z = shp[nid];
-        if (n.kind == MURE_NODE_CONV2D) {
+        if (n.kind == MURE_NODE_CONV2D || n.kind == MURE_NODE_DWCONV) {
             S.ih = a.h; S.iw = a.w; S.ic = a.c; S.kh = n.kh; S.kw = n.kw; S.stride = n.stride; S.pad = n.pad;
         } else {
             S.ih = 1; S.iw = 1; S.ic = n.cin; S.kh = 1; S.kw = 1; S.stride = 1; S.pad = 0;
         }
         S.oh = z.h; S.ow = z.w; S.oc = z.c;
-        S.K = S.kh * S.kw * S.ic;
+        // a depthwise neuron's fan-in is its own channel's filter
+        S.K = n.kind == MURE_NODE_DWCONV ? S.kh * S.kw : S.kh * S.kw * S.ic;
         S.act1 = n.act;
         S.skip_src = -1; S.sc_stride = 1; S.sc_c = 0; S.sk_w = 0;
         S.macs = (int64_t)S.oh * S.ow * S.oc * S.K;
@@ -329,6 +338,8 @@ void compile(mure_ctx *c, const mure_model_desc *d, mure_model *m)
             }
             cur = u;
         }
+        FAILIF(S.kind == MURE_NODE_DWCONV && (S.has_add || S.pool || S.gap), c, MURE_ERR_UNSUPPORTED,
+               "depthwise node %d: only an activation may follow it in its stage", nid);
         FAILIF(S.in_src != v && !(S.has_add && S.skip_src == v && S.sc_stride == 1), c, MURE_ERR_UNSUPPORTED,
                "weighted node %d reads an earlier stage input but its add does not take the previous stage", nid);
         const Shape y = shp[cur];

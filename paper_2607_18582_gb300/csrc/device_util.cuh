@@ -12,8 +12,13 @@ namespace mure {
 __host__ __device__ __forceinline__ int64_t round4(int64_t n) { return (n + 3) & ~int64_t(3); }
 
 // ReLU returns +0 for every non-positive input (and for NaN), so the sign of a zero
-// pre-activation never reaches later layers.
-__device__ __forceinline__ float act_apply(int act, float v) { return act == MURE_ACT_RELU ? (v > 0.f ? v : 0.f) : v; }
+// pre-activation never reaches later layers; ReLU6 also caps at 6.
+__device__ __forceinline__ float act_apply(int act, float v)
+{
+    if (act == MURE_ACT_RELU) return v > 0.f ? v : 0.f;
+    if (act == MURE_ACT_RELU6) return v > 0.f ? (v < 6.f ? v : 6.f) : 0.f;
+    return v;
+}
 
 // 2x2 max pool of one window, top-left first; a later element replaces the
 // running maximum only when strictly greater.

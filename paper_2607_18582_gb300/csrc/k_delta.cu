@@ -131,6 +131,7 @@ struct PatchValsParams {
     int skip_dot_ops;    // 1: GF / WS values come from k_patch_dot
     int only_dot_ops;    // 1: the other operators come from k_patch_vals_staged
     int skip_copy_ops;   // 1: NEB / NS slots are applied by the consumer (window GEMM)
+    int dw;              // depthwise layer: neuron j's fan-in is its kh x kw filter on input channel j
 };
 
 struct SlotCtx {
@@ -158,6 +159,18 @@ __device__ __forceinline__ float dot_serial(const PatchValsParams &p, const Slot
 {
     float acc = 0.f;
     const int iy0 = oy * p.stride - p.pad, ix0 = ox * p.stride - p.pad;
+    if (p.dw) {
+        // a depthwise neuron: its filter taps (ky, kx) on input channel j
+        for (int ky = 0; ky < p.kh; ++ky) {
+            const int iy = iy0 + ky;
+            for (int kx = 0; kx < p.kw; ++kx) {
+                const int ix = ix0 + kx;
+                if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw)
+                    acc = fmaf(__ldg(d.e + ky * p.kw + kx), __ldg(d.x + ((int64_t)iy * p.iw + ix) * p.ic + d.j), acc);
+            }
+        }
+        return acc;
+    }
     int k = 0;
     for (int ky = 0; ky < p.kh; ++ky) {
         const int iy = iy0 + ky;
@@ -178,7 +191,13 @@ __device__ __forceinline__ float dot_warp(const PatchValsParams &p, const SlotCt
 {
     float acc = 0.f;
     const int iy0 = oy * p.stride - p.pad, ix0 = ox * p.stride - p.pad;
-    if (p.kh == 1 && p.kw == 1 && p.ih == 1 && p.iw == 1) {
+    if (p.dw) {
+        for (int k = lane; k < p.K; k += 32) {
+            const int ky = k / p.kw, kx = k - ky * p.kw, iy = iy0 + ky, ix = ix0 + kx;
+            if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw)
+                acc = fmaf(__ldg(d.e + k), __ldg(d.x + ((int64_t)iy * p.iw + ix) * p.ic + d.j), acc);
+        }
+    } else if (p.kh == 1 && p.kw == 1 && p.ih == 1 && p.iw == 1) {
         for (int k = lane; k < p.K; k += 32) acc = fmaf(__ldg(d.e + k), __ldg(d.x + k), acc);
     } else {
         for (int k = lane; k < p.K; k += 32) {
@@ -427,6 +446,7 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     p.warp_dot = (S.oh * S.ow) < 32;
     p.skip_dot_ops = skip_dot_ops;
     p.skip_copy_ops = skip_copy_ops;
+    p.dw = S.kind == MURE_NODE_DWCONV;
     const int64_t n_items = (int64_t)p.G * kmax;
     // each warp walks several inputs (blockIdx.y, +gridDim.y, ...): enough blocks to
     // fill the GPU, few enough that block scheduling stays negligible
@@ -452,8 +472,8 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     // memoized convolution layers whose maps fit in shared memory: the non-dot
     // operators per input, staged
     const size_t staged_smem = ((size_t)S.oc * S.oh * S.ow + p.mcells) * 4;
-    const bool staged = z.per_input && S.kind == MURE_NODE_CONV2D && !S.has_add && !S.gap &&
-                        staged_smem <= 48 * 1024;
+    const bool staged = z.per_input && (S.kind == MURE_NODE_CONV2D || S.kind == MURE_NODE_DWCONV) && !S.has_add &&
+                        !S.gap && staged_smem <= 48 * 1024;
     int launches = 0;
     if (staged) {
         if (pa.n_vslot > 0) {

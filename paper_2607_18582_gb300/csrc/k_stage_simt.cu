@@ -165,11 +165,53 @@ __global__ void k_gap(const float *__restrict__ in, int64_t in_stride, int P, in
     y[r * y_stride + c] = gap_sum(in + r * in_stride, P, C, c);
 }
 
+// Depthwise convolution stage (MobileNetV2): output channel c at (oy, ox) is the fp32
+// FMA chain over its filter taps (ky, kx ascending, from +0) on input channel c, then
+// + b; the pre-activation goes to z (channel-major) when requested, act1 to y.  One
+// thread per (row, position, channel): consecutive threads read and write
+// consecutive channels, and the weights are read as Wt [tap][c].
+__global__ void __launch_bounds__(256) k_dwconv(const StageParams p)
+{
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t per_row = (int64_t)p.oh * p.ow * p.oc;
+    if (i >= (int64_t)p.R * per_row) return;
+    const int64_t row = i / per_row;
+    const int rem = (int)(i - row * per_row);
+    const int c = rem % p.oc, pos = rem / p.oc, oy = pos / p.ow, ox = pos - (pos / p.ow) * p.ow;
+    const float *xrow = p.x + (p.x_per_input ? p.t0 + logical_row(p.lrow, row) % p.T : row) * p.x_stride;
+    float acc = 0.f;
+    for (int ky = 0; ky < p.kh; ++ky) {
+        const int iy = oy * p.stride - p.pad + ky;
+        for (int kx = 0; kx < p.kw; ++kx) {
+            const int ix = ox * p.stride - p.pad + kx;
+            if ((unsigned)iy < (unsigned)p.ih && (unsigned)ix < (unsigned)p.iw)
+                acc = fmaf(__ldg(p.Wt + (int64_t)(ky * p.kw + kx) * p.oc + c),
+                           __ldg(xrow + ((int64_t)iy * p.iw + ix) * p.ic + c), acc);
+        }
+    }
+    const float z = acc + __ldg(p.b + c);
+    if (p.z) p.z[row * p.z_stride + (int64_t)c * (p.oh * p.ow) + pos] = z;
+    p.y[row * p.y_stride + (int64_t)pos * p.oc + c] = act_apply(p.act1, z);
+}
+
 int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, Src skip, float *y_out,
                       int64_t y_stride, float *gap_tmp, cudaStream_t s)
 {
     if (rm.R <= 0) return 0;
     if (S.tc) return launch_tc(S, x, rm, z_out, z_stride, skip, y_out, y_stride, gap_tmp, s);
+    if (S.kind == MURE_NODE_DWCONV) {
+        StageParams p{};
+        p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
+        p.t0 = rm.t0; p.T = rm.T; p.R = rm.R; p.lrow = rm.lrow;
+        p.ih = S.ih; p.iw = S.iw; p.ic = S.ic; p.kh = S.kh; p.kw = S.kw; p.stride = S.stride; p.pad = S.pad;
+        p.oh = S.oh; p.ow = S.ow; p.oc = S.oc; p.K = S.K;
+        p.Wt = S.Wt; p.b = S.b; p.act1 = S.act1;
+        p.z = z_out; p.z_stride = z_stride;
+        p.y = y_out; p.y_stride = y_stride;
+        const int64_t n = (int64_t)rm.R * S.oh * S.ow * S.oc;
+        k_dwconv<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(p);
+        return 1;
+    }
     if (S.variant > 0) return launch_conv_small(S, x, rm, z_out, z_stride, y_out, y_stride, s);
     StageParams p{};
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;

@@ -1012,9 +1012,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                             if (n < p.slot.n) vh[e] = __ldg(zr + (int64_t)__ldg(p.slot.j + n) * (p.oh * p.ow)) + vh[e];
                         }
                     }
-                    if (p.act1 == MURE_ACT_RELU) {
+                    if (p.act1 != MURE_ACT_NONE) {
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) vh[e] = act_apply(MURE_ACT_RELU, vh[e]);
+                        for (int e = 0; e < 16; ++e) vh[e] = act_apply(p.act1, vh[e]);
                     }
                     if constexpr (FCP > 0) {
                         // the output layer: fp32 FMAs over the inputs f in ascending

@@ -92,6 +92,9 @@ def test_unsupported_graphs_and_settings():
     # that reads an earlier stage input, its add taking the previous stage's output
     for prec in ("fp32", "tf32x3", "tf32"):
         assert mure.mure_check_descriptors(wl.resnet10(), precision=prec) == (OK, "")
+    # depthwise convolutions and ReLU6 (MobileNetV2)
+    for prec in ("fp32", "tf32x3"):
+        assert mure.mure_check_descriptors(wl.mobilenetv2_tiny(), precision=prec) == (OK, "")
     # ... but not when that add skips the layer just before it (a dead branch)
     m = wl.resnet10()
     adds = [i for i, n in enumerate(m.nodes) if n.kind == "add"]
