@@ -800,10 +800,11 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     ov.neuron_off = pa.neuron_off;
     ov.ids = pa.ids;
     // x_{l+1} read other than as the first suffix stage's GEMM input (a later residual
-    // add, or the add of a projection in a skip branch that reads an earlier input):
-    // its rows are materialised with the patch
+    // add, the add of a projection that reads an earlier input, or a later projection
+    // reading x_{l+1} itself): its rows are materialised with the patch
     bool skip_reader = l + 1 < L && m->st[l + 1].in_src != l + 1;
-    for (int v = l + 2; v < L; ++v) skip_reader |= m->st[v].has_add && m->st[v].skip_src == l + 1;
+    for (int v = l + 2; v < L; ++v)
+        skip_reader |= (m->st[v].has_add && m->st[v].skip_src == l + 1) || m->st[v].in_src == l + 1;
     // the window GEMM as first suffix stage applies NEB (zeros) and NS (a swap of the
     // two channels, which is the operator itself: the swapped neurons' channels are
     // computed independently) on its staged maps, so the delta writes no values for
