@@ -132,6 +132,7 @@ struct PatchValsParams {
     int only_dot_ops;    // 1: the other operators come from k_patch_vals_staged
     int skip_copy_ops;   // 1: NEB / NS slots are applied by the consumer (window GEMM)
     int dw;              // depthwise layer: neuron j's fan-in is its kh x kw filter on input channel j
+    const float *W, *b;  // the layer's weights [oc][K] and biases (depthwise NS)
 };
 
 struct SlotCtx {
@@ -139,12 +140,19 @@ struct SlotCtx {
     int op, j, sj;
 };
 
+// NS on a depthwise layer: the two neurons exchange filters and biases, but each filter
+// stays on its own output channel's input channel, so the mutated channel j is
+// recomputed, b[m] + sum_k W[m][k] x_j[k] (m its partner), not taken from channel m.
+__device__ __forceinline__ bool dw_switch(const PatchValsParams &p, int op) { return p.dw && op == MURE_OP_NS; }
+
 // Mutated output of neuron j at conv position (oy, ox) after act1, skip and act2;
-// `dot` is the GF / WS correction sum_k e_k x_k at that position.
+// `dot` is the GF / WS correction sum_k e_k x_k at that position (depthwise NS: the
+// partner's filter on channel j).
 __device__ __forceinline__ float slot_post(const PatchValsParams &p, const SlotCtx &d, int oy, int ox, float dot)
 {
     float zz = d.z[(int64_t)d.sj * (p.oh * p.ow) + oy * p.ow + ox];
-    if (d.op == MURE_OP_NAI) zz = -zz;
+    if (dw_switch(p, d.op)) zz = dot + __ldg(p.b + d.sj);   // the forward kernel's chain: taps from +0, then + b
+    else if (d.op == MURE_OP_NAI) zz = -zz;
     else if (d.op == MURE_OP_GF || d.op == MURE_OP_WS) zz = zz + dot;
     float v = d.op == MURE_OP_NEB ? 0.f : act_apply(p.act1, zz);
     if (p.has_add) {
@@ -216,7 +224,7 @@ __device__ __forceinline__ float dot_warp(const PatchValsParams &p, const SlotCt
 // mode every lane of the warp must call it with the same c.
 __device__ __forceinline__ float cell_value(const PatchValsParams &p, const SlotCtx &d, int c, int lane)
 {
-    const bool dot = d.op == MURE_OP_GF || d.op == MURE_OP_WS;
+    const bool dot = d.op == MURE_OP_GF || d.op == MURE_OP_WS || dw_switch(p, d.op);
     const int cy = c / p.mcw, cx = c % p.mcw;
     if (!p.pool) {
         const float dv = dot ? (p.warp_dot ? dot_warp(p, d, cy, cx, lane) : dot_serial(p, d, cy, cx)) : 0.f;
@@ -245,15 +253,18 @@ __global__ void __launch_bounds__(256) k_patch_vals(const PatchValsParams p)
     const int g = item / p.kmax, q = item - g * p.kmax;
     if (q >= p.pa.n_neurons[g]) return;
     const int op = p.pa.op[g];
-    const bool dot = op == MURE_OP_GF || op == MURE_OP_WS;
-    if (dot && p.skip_dot_ops) return;
+    const bool gfws = op == MURE_OP_GF || op == MURE_OP_WS;
+    const bool dot = gfws || dw_switch(p, op);
+    if (gfws && p.skip_dot_ops) return;
     if (!dot && p.only_dot_ops) return;
     const int32_t *ids = p.pa.ids + p.pa.neuron_off[g];
     SlotCtx d;
     d.op = op;
     d.j = ids[q];
     d.sj = op == MURE_OP_NS ? ids[q ^ 1] : d.j;
-    const float *e = dot ? p.pa.patch + p.pa.patch_off[g] + (int64_t)q * p.K : nullptr;
+    // the fan-in terms of the sum: GF / WS patch, or (depthwise NS) the partner's filter
+    const float *e = gfws ? p.pa.patch + p.pa.patch_off[g] + (int64_t)q * p.K
+                          : dot ? p.W + (int64_t)d.sj * p.K : nullptr;
     if (!dot && (p.warp_dot || p.cells < 32)) {
         // no fan-in sum and few cells: one input per lane, its cells in order (a GAP
         // value is the same ascending sum over the map cells as below)
@@ -447,6 +458,8 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     p.skip_dot_ops = skip_dot_ops;
     p.skip_copy_ops = skip_copy_ops;
     p.dw = S.kind == MURE_NODE_DWCONV;
+    p.W = S.W;
+    p.b = S.b;
     const int64_t n_items = (int64_t)p.G * kmax;
     // each warp walks several inputs (blockIdx.y, +gridDim.y, ...): enough blocks to
     // fill the GPU, few enough that block scheduling stays negligible
@@ -472,8 +485,8 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     // memoized convolution layers whose maps fit in shared memory: the non-dot
     // operators per input, staged
     const size_t staged_smem = ((size_t)S.oc * S.oh * S.ow + p.mcells) * 4;
-    const bool staged = z.per_input && (S.kind == MURE_NODE_CONV2D || S.kind == MURE_NODE_DWCONV) && !S.has_add &&
-                        !S.gap && staged_smem <= 48 * 1024;
+    const bool staged = z.per_input && S.kind == MURE_NODE_CONV2D && !S.has_add && !S.gap &&
+                        staged_smem <= 48 * 1024;
     int launches = 0;
     if (staged) {
         if (pa.n_vslot > 0) {
