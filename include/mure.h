@@ -53,11 +53,24 @@ enum {
     MURE_NODE_GAP = 5,      /* global average pooling over H and W */
     MURE_NODE_SHORTCUT = 6, /* parameter-free residual shortcut: subsample by
                                `stride`, zero channels appended up to `cout` */
-    MURE_NODE_DWCONV = 7    /* depthwise 2-D convolution (MobileNetV2, Table 1): channel
+    MURE_NODE_DWCONV = 7,   /* depthwise 2-D convolution (MobileNetV2, Table 1): channel
                                c of the output is a kh x kw filter over channel c of the
                                input, + bias + activation; cin = cout = the input's
                                channels, W [c][kh][kw]; neuron j = channel j, whose fan-in
                                is its kh*kw filter */
+    MURE_NODE_EMBED = 8,    /* embedding (the recurrent family of Table 1): the input is
+                               1 x T x 1 token ids held in floats (integers in [0, cin));
+                               output 1 x T x cout, position t channel j = W[j][id_t];
+                               W [cout][cin] (channel-major), b may be NULL (no bias);
+                               neuron j = channel j, whose fan-in is its cin table entries */
+    MURE_NODE_LSTM = 9      /* LSTM over the 1 x T x cin input sequence, cout units, zero
+                               initial state, gates i, f, g, o: pre = b + Wx x_t + Wh h,
+                               i, f, o = sigmoid, g = tanh, c = f c + i g, h = o tanh(c);
+                               W [cout][4][cin + cout] (a unit's gate rows: input weights,
+                               then recurrent weights), b [cout][4]; kh = 1: output every
+                               step (1 x T x cout), kh = 0: the last step (1 x 1 x cout);
+                               neuron j = unit j, whose fan-in is its 4 (cin + cout)
+                               weights (NEB holds h_j at 0 at every step) */
 };
 enum { MURE_ACT_NONE = 0, MURE_ACT_RELU = 1, MURE_ACT_RELU6 = 2 /* min(max(v, 0), 6) */ };
 

@@ -169,7 +169,11 @@ struct Shape {
     int h, w, c;
 };
 
-bool weighted(int k) { return k == MURE_NODE_CONV2D || k == MURE_NODE_DENSE || k == MURE_NODE_DWCONV; }
+bool weighted(int k)
+{
+    return k == MURE_NODE_CONV2D || k == MURE_NODE_DENSE || k == MURE_NODE_DWCONV || k == MURE_NODE_EMBED ||
+           k == MURE_NODE_LSTM;
+}
 
 // Output shapes of all nodes (same rules as the network definition in the header).
 std::vector<Shape> node_shapes(mure_ctx *c, const mure_model_desc *d)
@@ -195,6 +199,18 @@ std::vector<Shape> node_shapes(mure_ctx *c, const mure_model_desc *d)
             o = {(a.h + 2 * n.pad - n.kh) / n.stride + 1, (a.w + 2 * n.pad - n.kw) / n.stride + 1, a.c};
             FAILIF(o.h < 1 || o.w < 1, c, MURE_ERR_INVALID_ARG, "node %d: empty depthwise output", v);
             FAILIF(!n.W || !n.b, c, MURE_ERR_INVALID_ARG, "node %d: NULL weights", v);
+            break;
+        case MURE_NODE_EMBED:
+            FAILIF(a.h != 1 || a.c != 1 || n.cin < 1 || n.cout < 1, c, MURE_ERR_INVALID_ARG,
+                   "node %d: an embedding reads a 1 x T x 1 sequence of ids", v);
+            FAILIF(!n.W, c, MURE_ERR_INVALID_ARG, "node %d: NULL weights", v);
+            o = {1, a.w, n.cout};
+            break;
+        case MURE_NODE_LSTM:
+            FAILIF(a.h != 1 || n.cin != a.c || n.cout < 1 || (n.kh != 0 && n.kh != 1), c, MURE_ERR_INVALID_ARG,
+                   "node %d: bad LSTM geometry", v);
+            FAILIF(!n.W || !n.b, c, MURE_ERR_INVALID_ARG, "node %d: NULL weights", v);
+            o = {1, n.kh ? a.w : 1, n.cout};
             break;
         case MURE_NODE_DENSE:
             FAILIF(n.cin != a.h * a.w * a.c || n.cout < 1, c, MURE_ERR_INVALID_ARG, "node %d: dense fan-in mismatch", v);
@@ -284,15 +300,26 @@ void compile(mure_ctx *c, const mure_model_desc *d, mure_model *m)
         const Shape a = shape_of(n.in0), z = shp[nid];
         if (n.kind == MURE_NODE_CONV2D || n.kind == MURE_NODE_DWCONV) {
             S.ih = a.h; S.iw = a.w; S.ic = a.c; S.kh = n.kh; S.kw = n.kw; S.stride = n.stride; S.pad = n.pad;
+        } else if (n.kind == MURE_NODE_EMBED || n.kind == MURE_NODE_LSTM) {
+            // sequences: iw = T steps, ic = the input width (1 for the ids); kh = the
+            // LSTM's every-step flag
+            S.ih = 1; S.iw = a.w; S.ic = a.c; S.kh = n.kh; S.kw = 1; S.stride = 1; S.pad = 0;
         } else {
             S.ih = 1; S.iw = 1; S.ic = n.cin; S.kh = 1; S.kw = 1; S.stride = 1; S.pad = 0;
         }
         S.oh = z.h; S.ow = z.w; S.oc = z.c;
-        // a depthwise neuron's fan-in is its own channel's filter
-        S.K = n.kind == MURE_NODE_DWCONV ? S.kh * S.kw : S.kh * S.kw * S.ic;
+        // a depthwise neuron's fan-in is its own channel's filter; an embedding channel's
+        // its table entries; an LSTM unit's its four gates' input and recurrent weights
+        S.K = n.kind == MURE_NODE_DWCONV ? S.kh * S.kw
+              : n.kind == MURE_NODE_EMBED ? n.cin
+              : n.kind == MURE_NODE_LSTM  ? 4 * (S.ic + S.oc)
+                                          : S.kh * S.kw * S.ic;
+        S.vocab = n.kind == MURE_NODE_EMBED ? n.cin : 0;
         S.act1 = n.act;
         S.skip_src = -1; S.sc_stride = 1; S.sc_c = 0; S.sk_w = 0;
-        S.macs = (int64_t)S.oh * S.ow * S.oc * S.K;
+        S.macs = n.kind == MURE_NODE_EMBED ? 0
+                 : n.kind == MURE_NODE_LSTM  ? (int64_t)S.iw * S.oc * S.K
+                                             : (int64_t)S.oh * S.ow * S.oc * S.K;
         m->zd[v] = tdim(z);
         int cur = nid;
         const int end = v + 1 < L ? wn[v + 1] : d->n_nodes;
@@ -340,6 +367,12 @@ void compile(mure_ctx *c, const mure_model_desc *d, mure_model *m)
         }
         FAILIF(S.kind == MURE_NODE_DWCONV && (S.has_add || S.pool || S.gap), c, MURE_ERR_UNSUPPORTED,
                "depthwise node %d: only an activation may follow it in its stage", nid);
+        FAILIF((S.kind == MURE_NODE_EMBED || S.kind == MURE_NODE_LSTM) && (S.has_add || S.pool || S.gap || n.act), c,
+               MURE_ERR_UNSUPPORTED, "recurrent node %d: no activation, add or pooling in its stage", nid);
+        FAILIF(S.kind == MURE_NODE_EMBED && v != 0, c, MURE_ERR_UNSUPPORTED, "embedding node %d: only as the first layer",
+               nid);
+        FAILIF((S.kind == MURE_NODE_EMBED || S.kind == MURE_NODE_LSTM) && !recurrent_supported(S), c,
+               MURE_ERR_UNSUPPORTED, "LSTM node %d: at most 64 units and 128 inputs", nid);
         FAILIF(S.in_src != v && !(S.has_add && S.skip_src == v && S.sc_stride == 1), c, MURE_ERR_UNSUPPORTED,
                "weighted node %d reads an earlier stage input but its add does not take the previous stage", nid);
         const Shape y = shp[cur];
@@ -368,6 +401,8 @@ void check_table(mure_ctx *c, const mure_model *m, const mure_mutant *t, int64_t
     FAILIF(n > 0 && !t, c, MURE_ERR_INVALID_ARG, "NULL mutant table");
     FAILIF(pool_len > 0 && !pool, c, MURE_ERR_INVALID_ARG, "NULL neuron pool");
     FAILIF(n > INT32_MAX, c, MURE_ERR_UNSUPPORTED, "more than 2^31 mutants");
+    bool recurrent = false;
+    for (int v = 0; v < m->L; ++v) recurrent |= m->st[v].kind == MURE_NODE_EMBED || m->st[v].kind == MURE_NODE_LSTM;
     std::vector<int64_t> seen;
     for (int64_t i = 0; i < n; ++i) {
         const mure_mutant &u = t[i];
@@ -391,6 +426,8 @@ void check_table(mure_ctx *c, const mure_model *m, const mure_mutant *t, int64_t
                    MURE_ERR_INVALID_ARG, "mutant %lld: an NS pair across two layers", (long long)i);
             lmin = std::min(lmin, l);
         }
+        FAILIF(u.tagged && recurrent, c, MURE_ERR_UNSUPPORTED,
+               "mutant %lld: mutants over several layers of a recurrent network", (long long)i);
         FAILIF(u.tagged && u.n_neurons > 0 && lmin != u.layer, c, MURE_ERR_INVALID_ARG,
                "mutant %lld: layer %d is not its smallest listed layer %d", (long long)i, u.layer, lmin);
         std::sort(seen.begin(), seen.end());
@@ -764,6 +801,22 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
     const int64_t G = rm.R / rm.T;
     const int64_t delta_flops =
         (dt.dot_prefix[g0 + G] - dt.dot_prefix[g0]) * rm.T * 2 * (int64_t)Sl.oh * Sl.ow * Sl.K;
+    if (Sl.kind == MURE_NODE_LSTM) {
+        // a mutated LSTM layer: its recurrence spreads one unit's change to every unit
+        // from the first step on, so the layer itself is recomputed for every row from
+        // its input (cached in memoized mode, recomputed in vanilla mode) with the mutated
+        // units' rows rewritten, then the suffix runs from its output
+        if (vanilla)
+            for (int v = 0; v < l; ++v) stage(v, nullptr, 0);
+        acct.bytes_rows += 2 * (int64_t)rm.R * m->xd[l + 1].size * 4;
+        timed(l, 2 * Sl.macs * rm.R, [&] {
+            return launch_lstm(Sl, xsrc(Sl.in_src), rm, nullptr, 0, ws.xb[l + 1], m->xd[l + 1].stride, &pa, s);
+        });
+        for (int v = l + 1; v < L - 1; ++v) stage(v, nullptr, 0);
+        const Stage &SLr = m->st[L - 1];
+        timed(L - 1, 2 * SLr.macs * rm.R, [&] { return launch_final_dense(SLr, xsrc(SLr.in_src), rm, fa, s); });
+        return launches;
+    }
     if (vanilla) {
         // the prefix, then layer l itself, from the inputs, row by row
         for (int v = 0; v < l; ++v) stage(v, nullptr, 0);
@@ -1279,8 +1332,17 @@ mure_cache *build_cache(mure_model *m, const float *X, int64_t n_in, const int32
         check_launch(c);
         uint32_t hm = 0;
         CK(c, cudaMemcpyAsync(&hm, mask, 4, cudaMemcpyDeviceToHost, s));
+        int dev_err = 0;
+        CK(c, cudaMemcpyAsync(&dev_err, c->err_dev, sizeof(int), cudaMemcpyDeviceToHost, s));
         CK(c, cudaStreamSynchronize(s));
         ca->n_label_values = __builtin_popcount(hm);
+        if (dev_err) {
+            // a token id outside an embedding's table, or a bounded wait that gave up
+            CK(c, cudaMemset(c->err_dev, 0, sizeof(int)));
+            FAILIF(true, c, dev_err == MURE_ERR_TIMEOUT ? MURE_ERR_TIMEOUT : MURE_ERR_INVALID_ARG,
+                   "a device-side check failed while building the cache (code %d: %s)", dev_err,
+                   dev_err == MURE_ERR_INVALID_ARG ? "an input id outside the embedding's table" : "wait limit");
+        }
     }
     CK(c, cudaStreamSynchronize(s));
     cl.ok = true;
@@ -1415,13 +1477,16 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
             const int64_t nw = (int64_t)S.oc * S.K;
             S.W = (float *)dalloc(c, nw * 4);
             S.Wt = (float *)dalloc(c, nw * 4);
-            S.b = (float *)dalloc(c, S.oc * 4);
+            // an LSTM unit has four gate biases; an embedding has none (zeros)
+            const int64_t nb = S.kind == MURE_NODE_LSTM ? 4 * (int64_t)S.oc : S.oc;
+            S.b = (float *)dalloc(c, nb * 4);
             Wt.resize(nw);
             for (int o = 0; o < S.oc; ++o)
                 for (int k = 0; k < S.K; ++k) Wt[(int64_t)k * S.oc + o] = n.W[(int64_t)o * S.K + k];
             CK(c, cudaMemcpyAsync(S.W, n.W, nw * 4, cudaMemcpyHostToDevice, c->stream));
             CK(c, cudaMemcpyAsync(S.Wt, Wt.data(), nw * 4, cudaMemcpyHostToDevice, c->stream));
-            CK(c, cudaMemcpyAsync(S.b, n.b, S.oc * 4, cudaMemcpyHostToDevice, c->stream));
+            if (n.b) CK(c, cudaMemcpyAsync(S.b, n.b, nb * 4, cudaMemcpyHostToDevice, c->stream));
+            else CK(c, cudaMemsetAsync(S.b, 0, nb * 4, c->stream));
             CK(c, cudaStreamSynchronize(c->stream));  // Wt is reused
             if (S.tc) {
                 S.Wtc = (float *)dalloc(c, tc_weight_floats(S) * 4);

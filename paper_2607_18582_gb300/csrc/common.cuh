@@ -25,6 +25,7 @@ struct Stage {
     int K;                    // fan-in kh*kw*ic
     int act1;
     int has_add, skip_src;    // skip tensor = x_{skip_src} (stage-input index)
+    int vocab = 0;            // embedding: table entries (ids 0 .. vocab - 1)
     int in_src = -1;          // stage input the layer reads (x_v; an earlier x_s for a
                               // projection in a skip branch, whose add then takes x_v)
     int sc_stride, sc_c;      // shortcut subsampling stride and source channels
@@ -191,6 +192,17 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
               const FinalFuse *ff = nullptr, const SlotStore *ss = nullptr);
 // Whether stage S (feeding the output layer SL) can take SL into its epilogue.
 int tc_final_fusable(const Stage &S, const Stage &SL);
+
+// The recurrent family: embedding lookups and LSTM layers over R rows of sequences
+// (iw = steps).  launch_lstm with pa non-null recomputes a mutated LSTM layer: every row
+// of batch mutant g takes its mutated units' rewritten rows (GF / WS: W + e of the
+// patch, NAI: negated, NS: the partner's, NEB: h held at 0).
+int recurrent_supported(const Stage &S);
+int launch_embed(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, float *y_out, int64_t y_stride,
+                 cudaStream_t s);
+struct PatchArgs;
+int launch_lstm(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, float *y_out, int64_t y_stride,
+                const PatchArgs *pa, cudaStream_t s);
 
 // Global average pooling of R rows of a [P][C] map.
 int launch_gap(const float *in, int64_t in_stride, int P, int C, int R, float *y, int64_t y_stride, cudaStream_t s);

@@ -132,6 +132,8 @@ struct PatchValsParams {
     int only_dot_ops;    // 1: the other operators come from k_patch_vals_staged
     int skip_copy_ops;   // 1: NEB / NS slots are applied by the consumer (window GEMM)
     int dw;              // depthwise layer: neuron j's fan-in is its kh x kw filter on input channel j
+    int embed;           // embedding: channel j at step t is table entry W[j][id_t]; GF / WS add e[id_t]
+    int vocab;
     const float *W, *b;  // the layer's weights [oc][K] and biases (depthwise NS)
 };
 
@@ -166,6 +168,11 @@ __device__ __forceinline__ float slot_post(const PatchValsParams &p, const SlotC
 __device__ __forceinline__ float dot_serial(const PatchValsParams &p, const SlotCtx &d, int oy, int ox)
 {
     float acc = 0.f;
+    if (p.embed) {
+        // the one-hot input of an embedding: the term of the step's id
+        const int id = (int)__ldg(d.x + ox);
+        return (unsigned)id < (unsigned)p.vocab ? acc + __ldg(d.e + id) : acc;
+    }
     const int iy0 = oy * p.stride - p.pad, ix0 = ox * p.stride - p.pad;
     if (p.dw) {
         // a depthwise neuron: its filter taps (ky, kx) on input channel j
@@ -198,6 +205,11 @@ __device__ __forceinline__ float dot_serial(const PatchValsParams &p, const Slot
 __device__ __forceinline__ float dot_warp(const PatchValsParams &p, const SlotCtx &d, int oy, int ox, int lane)
 {
     float acc = 0.f;
+    if (p.embed) {
+        // one term: every lane returns it (no butterfly)
+        const int id = (int)__ldg(d.x + ox);
+        return (unsigned)id < (unsigned)p.vocab ? acc + __ldg(d.e + id) : acc;
+    }
     const int iy0 = oy * p.stride - p.pad, ix0 = ox * p.stride - p.pad;
     if (p.dw) {
         for (int k = lane; k < p.K; k += 32) {
@@ -458,6 +470,8 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     p.skip_dot_ops = skip_dot_ops;
     p.skip_copy_ops = skip_copy_ops;
     p.dw = S.kind == MURE_NODE_DWCONV;
+    p.embed = S.kind == MURE_NODE_EMBED;
+    p.vocab = S.vocab;
     p.W = S.W;
     p.b = S.b;
     const int64_t n_items = (int64_t)p.G * kmax;

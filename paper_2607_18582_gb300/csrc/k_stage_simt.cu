@@ -199,6 +199,8 @@ int launch_stage_simt(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_
 {
     if (rm.R <= 0) return 0;
     if (S.tc) return launch_tc(S, x, rm, z_out, z_stride, skip, y_out, y_stride, gap_tmp, s);
+    if (S.kind == MURE_NODE_EMBED) return launch_embed(S, x, rm, z_out, z_stride, y_out, y_stride, s);
+    if (S.kind == MURE_NODE_LSTM) return launch_lstm(S, x, rm, z_out, z_stride, y_out, y_stride, nullptr, s);
     if (S.kind == MURE_NODE_DWCONV) {
         StageParams p{};
         p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;

