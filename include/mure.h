@@ -224,7 +224,7 @@ const char *mure_last_error(const mure_ctx *ctx);
 /* Copy a network to the device and compile it into stages (Algorithm 2: the
  * dependence graph is read from the nodes' inputs).  Errors: INVALID_ARG
  * (inconsistent shapes, bad ids, NULL weights), UNSUPPORTED (graph outside the
- * supported shape, n_classes > 32, unknown precision), OOM, CUDA. */
+ * supported shape, n_classes > 96, unknown precision), OOM, CUDA. */
 mure_status mure_model_load(mure_ctx *ctx, const mure_model_desc *desc, mure_model **out);
 void mure_model_free(mure_model *model);
 

@@ -1326,16 +1326,17 @@ mure_cache *build_cache(mure_model *m, const float *X, int64_t n_in, const int32
         check_launch(c);
         if (labels) CK(c, cudaMemcpyAsync(ca->label, lab_host.data(), n_in * 4, cudaMemcpyHostToDevice, s));
         else CK(c, cudaMemcpyAsync(ca->label, ca->pred0, n_in * 4, cudaMemcpyDeviceToDevice, s));
-        uint32_t *mask = sc.get<uint32_t>(1);
-        CK(c, cudaMemsetAsync(mask, 0, 4, s));
+        uint32_t *mask = sc.get<uint32_t>(kLabelWords);
+        CK(c, cudaMemsetAsync(mask, 0, 4 * kLabelWords, s));
         c->launches += launch_label_set(ca->label, n_in, mask, s);
         check_launch(c);
-        uint32_t hm = 0;
-        CK(c, cudaMemcpyAsync(&hm, mask, 4, cudaMemcpyDeviceToHost, s));
+        uint32_t hm[kLabelWords] = {};
+        CK(c, cudaMemcpyAsync(hm, mask, 4 * kLabelWords, cudaMemcpyDeviceToHost, s));
         int dev_err = 0;
         CK(c, cudaMemcpyAsync(&dev_err, c->err_dev, sizeof(int), cudaMemcpyDeviceToHost, s));
         CK(c, cudaStreamSynchronize(s));
-        ca->n_label_values = __builtin_popcount(hm);
+        ca->n_label_values = 0;
+        for (int k = 0; k < kLabelWords; ++k) ca->n_label_values += __builtin_popcount(hm[k]);
         if (dev_err) {
             // a token id outside an embedding's table, or a bounded wait that gave up
             CK(c, cudaMemset(c->err_dev, 0, sizeof(int)));

@@ -11,7 +11,8 @@
 
 namespace mure {
 
-constexpr int kMaxClasses = 32;   // final-layer kernel keeps one accumulator per class
+constexpr int kMaxClasses = 96;   // final-layer kernel keeps one accumulator per class (Reuters: 90)
+constexpr int kLabelWords = kMaxClasses / 32;   // 32-bit words of a label set
 constexpr int kInputAlign = 64;   // inputs are padded to a multiple of 64 (one kill word)
 
 // A weighted layer together with the unweighted nodes that turn its output into the
@@ -344,7 +345,7 @@ int launch_unchanged(const UnchangedArgs &ua, RowMap rm, int32_t *flags, int32_t
 int launch_scores(const uint32_t *kill32, int64_t n_mut, int64_t words32, const int32_t *label, int n_classes,
                   unsigned long long *totals /* [2]: killed, sum of label counts */, cudaStream_t s);
 
-// Distinct labels among n inputs (bitset of n_classes bits, <= 32 classes).
+// Distinct labels among n inputs (bitset of kLabelWords words; mask zeroed by the caller).
 int launch_label_set(const int32_t *label, int64_t n, uint32_t *mask, cudaStream_t s);
 
 }  // namespace mure

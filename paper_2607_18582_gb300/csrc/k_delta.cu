@@ -630,24 +630,33 @@ __global__ void __launch_bounds__(128) k_scores(const uint32_t *__restrict__ kil
     const int lane = threadIdx.x & 31;
     const int64_t i = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
     if (i >= n_mut) return;
-    uint32_t any = 0, labels = 0;
+    // the set of killing labels as kLabelWords 32-bit words (up to kMaxClasses labels)
+    uint32_t any = 0, labels[kLabelWords] = {};
     for (int64_t w = lane; w < words32; w += 32) {
         uint32_t bits = kill32[i * words32 + w];
         any |= bits;
         while (bits) {
             const int b = __ffs(bits) - 1;
-            labels |= 1u << label[w * 32 + b];
+            const int lb = label[w * 32 + b];
+#pragma unroll
+            for (int k = 0; k < kLabelWords; ++k)
+                if ((lb >> 5) == k) labels[k] |= 1u << (lb & 31);
             bits &= bits - 1;
         }
     }
+    int count = 0;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        any |= __shfl_xor_sync(0xffffffffu, any, o);
-        labels |= __shfl_xor_sync(0xffffffffu, labels, o);
+    for (int o = 16; o > 0; o >>= 1) any |= __shfl_xor_sync(0xffffffffu, any, o);
+#pragma unroll
+    for (int k = 0; k < kLabelWords; ++k) {
+        uint32_t m = labels[k];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m |= __shfl_xor_sync(0xffffffffu, m, o);
+        count += __popc(m);
     }
     if (lane == 0) {
         if (any) atomicAdd(&totals[0], 1ull);
-        atomicAdd(&totals[1], (unsigned long long)__popc(labels));
+        atomicAdd(&totals[1], (unsigned long long)count);
     }
 }
 
@@ -662,12 +671,20 @@ int launch_scores(const uint32_t *kill32, int64_t n_mut, int64_t words32, const 
 
 __global__ void k_label_set(const int32_t *__restrict__ label, int64_t n, uint32_t *mask)
 {
-    uint32_t m = 0;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-        m |= 1u << label[i];
+    uint32_t m[kLabelWords] = {};
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const int lb = label[i];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) m |= __shfl_xor_sync(0xffffffffu, m, o);
-    if ((threadIdx.x & 31) == 0 && m) atomicOr(mask, m);
+        for (int k = 0; k < kLabelWords; ++k)
+            if ((lb >> 5) == k) m[k] |= 1u << (lb & 31);
+    }
+#pragma unroll
+    for (int k = 0; k < kLabelWords; ++k) {
+        uint32_t v = m[k];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v |= __shfl_xor_sync(0xffffffffu, v, o);
+        if ((threadIdx.x & 31) == 0 && v) atomicOr(mask + k, v);
+    }
 }
 
 int launch_label_set(const int32_t *label, int64_t n, uint32_t *mask, cudaStream_t s)

@@ -516,7 +516,8 @@ int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cu
     else if (cp <= 8) k_final_dense<8><<<blocks, 128, 0, s>>>(p);
     else if (cp <= 12) k_final_dense<12><<<blocks, 128, 0, s>>>(p);
     else if (cp <= 16) k_final_dense<16><<<blocks, 128, 0, s>>>(p);
-    else k_final_dense<32><<<blocks, 128, 0, s>>>(p);
+    else if (cp <= 32) k_final_dense<32><<<blocks, 128, 0, s>>>(p);
+    else k_final_dense<96><<<blocks, 128, 0, s>>>(p);
     return 1;
 }
 

@@ -42,12 +42,15 @@ def every_operator(model, per_layer, seed):
     return wl.concat(subs)
 
 
-@pytest.mark.parametrize("size", ["small", "imdb"])
+@pytest.mark.parametrize("size", ["small", "imdb", "reuters"])
 def test_recurrent_network_matches_oracle(M, ctx, oracle_mod, size):
     if size == "small":
         model, n_in, per_layer = small_rnn(), 160, 12
-    else:
+    elif size == "imdb":
         model, n_in, per_layer = wl.rnn(), 64, 6
+    else:
+        # 90 classes: the 96-accumulator output layer and 96-label score sets
+        model, n_in, per_layer = wl.rnn_reuters(), 64, 6
     X = wl.inputs(model, n_in, 1)
     table = every_operator(model, per_layer, 70)
     ora = oracle_mod.vanilla(model, X, table)

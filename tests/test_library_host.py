@@ -104,8 +104,11 @@ def test_unsupported_graphs_and_settings():
     st, msg = mure.mure_check_descriptors(m)
     assert st == UNSUPPORTED and "earlier stage input" in msg
     # more classes than the output-layer kernel keeps accumulators for
-    st, msg = mure.mure_check_descriptors(wl.mlp(widths=(784, 64, 40)))
+    st, msg = mure.mure_check_descriptors(wl.mlp(widths=(784, 64, 100)))
     assert st == UNSUPPORTED and "n_classes" in msg
+    # up to 96 classes: the Reuters-sized recurrent model (90)
+    assert mure.mure_check_descriptors(wl.mlp(widths=(784, 64, 40))) == (OK, "")
+    assert mure.mure_check_descriptors(wl.rnn_reuters()) == (OK, "")
     st, msg = mure.mure_check_descriptors(wl.lenet5(), precision="bf16")
     assert st == UNSUPPORTED and "precision" in msg
 
