@@ -171,6 +171,33 @@ __device__ __forceinline__ void wait_phase_drain(uint32_t a, uint32_t parity)
         if (clock64() - t0 > kSpin) return;
 }
 
+// The issuing warps' turn token: K-step g of the CTA's sequence may be issued once the
+// counter reads g (acquire), and its issuer then publishes g + 1 (release).  Bounded like
+// the barrier waits.
+__device__ __forceinline__ uint32_t turn_load(uint32_t a)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void turn_store(uint32_t a, uint32_t v)
+{
+    asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ bool wait_turn(uint32_t a, uint32_t g, volatile WaitCtl *abort_flag)
+{
+    if (turn_load(a) == g) return true;
+    const long long t0 = clock64();
+    for (;;) {
+        __nanosleep(20);   // leaves the issue slots to the epilogue warp of the sub-partition
+        if (turn_load(a) == g) return true;
+        if (abort_flag->abort) return false;
+        if (clock64() - t0 > abort_flag->limit) { abort_flag->abort = 1; return false; }
+    }
+}
+
 // A from tensor memory, B from shared memory.
 __device__ __forceinline__ void mma_tf32_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc)
 {
@@ -276,7 +303,11 @@ struct TcParams {
     float *z; int64_t z_stride;
     float *y; int64_t y_stride;
     Overlay ov;                  // mutated channels of the input rows (ov.patch null: none)
-    int n_mma;                   // MMA-issuing warps, each with its own partial accumulators
+    int n_mma;                   // MMA-issuing warps
+    int n_part;                  // partial accumulators per set: n_mma, or 1 when the warps
+                                 // take turns (mma_chain)
+    int mma_chain;               // 1: the issuing warps take the K-steps in turn, in K-step
+                                 // order, into one accumulator (a token passed in shared memory)
     int acc_cols;                // tensor-memory columns of one partial accumulator
     int n_acc;                   // accumulator sets (tiles in flight): 1 or 2
     int n_stages;                // tensor-memory A stages (<= kMaxNT), from column a_col
@@ -600,6 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     // dense A tiles by tensor-map copies: slot landed, slot read by the producers
     __shared__ __align__(8) uint64_t bar_alanded[kNA], bar_afree[kNA];
     __shared__ uint32_t tmem_sh;
+    __shared__ uint32_t mma_turn_sh;   // mma_chain: the next K-step to issue
     __shared__ WaitCtl abort_sh;
     __shared__ float bias_sh[kSliceMax];
     __shared__ __align__(16) float epi_stage[4][32 * kEpiStride];   // per epilogue warp: 32 rows x 32 values
@@ -685,6 +717,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             mbar_init(smem_u32(&bar_released[s]), 4);
         }
         abort_sh.abort = 0;
+        mma_turn_sh = 0;
         abort_sh.limit = p.spin > 0 ? p.spin : kSpin;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -804,28 +837,47 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     }
                     const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + im * p.cv_img_bytes;
                     const int ntap = p.kh * p.kw;
-                    int ky = 0, kx = 0, tap = 0;
+                    // the current tap and its line relative to line0 (ky * cv_hw + kx)
+                    int tap = 0, kx = 0, off = 0;
+                    auto next_tap = [&]() {
+                        ++tap;
+                        if (++kx == p.kw) {
+                            kx = 0;
+                            off += p.cv_hw - p.kw + 1;
+                        } else {
+                            ++off;
+                        }
+                    };
+                    // chunk cc of line l sits at l * 128 + (cc ^ (l mod 8)) * 16
+                    auto gather = [&](float *v, int nc) {
+                        const uint32_t l = (uint32_t)(line0 + off);
+                        const uint32_t a = base + l * 128u, sw = l & 7u;
+#pragma unroll
+                        for (int cc = 0; cc < 8; ++cc) {
+                            if (cc >= nc) break;
+                            asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                                         : "=f"(v[4 * cc]), "=f"(v[4 * cc + 1]), "=f"(v[4 * cc + 2]), "=f"(v[4 * cc + 3])
+                                         : "r"(a + (((uint32_t)cc ^ sw) << 4)));
+                        }
+                    };
                     for (int ks = 0; ks < p.cv_taps; ++ks) {
                         float v[kTileK];
-#pragma unroll
-                        for (int cc = 0; cc < kTileK / 4; ++cc) {
-                            // 16-byte chunk cc: its tap (a new one every cv_cw / 4 chunks)
-                            if (cc > 0 && (cc * 4) % p.cv_cw == 0) {
-                                ++tap;
-                                if (++kx == p.kw) { kx = 0; ++ky; }
-                            }
+                        if (p.cv_cw == kTileK) {
+                            gather(v, 8);
+                            next_tap();
+                        } else {
+                            // two taps of 16 channels (the first half of their lines); past
+                            // the last tap the K-step's second half is zero
+                            gather(v, 4);
+                            next_tap();
                             if (tap < ntap) {
-                                const uint32_t line = (uint32_t)(line0 + ky * p.cv_hw + kx);
-                                const uint32_t lin = line * 128u + (uint32_t)((cc * 4) % p.cv_cw) * 4u;
-                                asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
-                                             : "=f"(v[4 * cc]), "=f"(v[4 * cc + 1]), "=f"(v[4 * cc + 2]), "=f"(v[4 * cc + 3])
-                                             : "r"(base + (lin ^ ((lin >> 3) & 0x70u))));
+                                gather(v + 16, 4);
                             } else {
-                                v[4 * cc] = v[4 * cc + 1] = v[4 * cc + 2] = v[4 * cc + 3] = 0.f;
+#pragma unroll
+                                for (int e = 16; e < kTileK; ++e) v[e] = 0.f;
                             }
+                            next_tap();
                         }
-                        ++tap;
-                        if (++kx == p.kw) { kx = 0; ++ky; }
                         if (!push(v)) { ok = false; break; }
                     }
                     // every gather of the chunk has been consumed by push: the buffer is free
@@ -927,12 +979,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 const bool ok = rr < G::ROWS && row < p.R;
                 const int w = rr % G::P;
                 const int py = w / G::PW, px = w % G::PW;
-                const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_mma * p.acc_cols);
+                const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_part * p.acc_cols);
                 float v[G::N];
 #pragma unroll
                 for (int n0 = 0; n0 < G::N; n0 += 16) {
                     tmem_ld16(acc + n0, v + n0);
-                    for (int w2 = 1; w2 < p.n_mma; ++w2) {
+                    for (int w2 = 1; w2 < p.n_part; ++w2) {
                         float u[16];
                         tmem_ld16(acc + (uint32_t)(w2 * p.acc_cols) + n0, u);
 #pragma unroll
@@ -984,10 +1036,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 for (int h = 0; h < 32; h += 16) {
                     if (h >= nc) break;
                     float *vh = v + h;
-                    // the accumulator: the n_mma partials added in a fixed order
-                    const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_mma * p.acc_cols) + n0 + h;
+                    // the accumulator: the n_part partials added in a fixed order
+                    const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_part * p.acc_cols) + n0 + h;
                     tmem_ld16(acc, vh);
-                    for (int w = 1; w < p.n_mma; ++w) {
+                    for (int w = 1; w < p.n_part; ++w) {
                         float u[16];
                         tmem_ld16(acc + (uint32_t)(w * p.acc_cols), u);
 #pragma unroll
@@ -1053,7 +1105,34 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                                            (int64_t)__ldg(p.slot.q + n) * p.slot.cells + cell] = vh[e];
                         }
                     }
-                    if (!DENSE && p.pool) {
+                    if (MODE == 3 && p.pool && !p.slot.out && n_base + n0 + h + 15 < p.N && (p.N & 3) == 0) {
+                        // lanes 4w .. 4w+3 hold the four positions (a, b, c, d) of one
+                        // pooling window; two exchanges leave lane q with all four values
+                        // of channels (q & 1) * 8 + (q >> 1) * 4 + 0..3, pooled in the
+                        // order a, b, c, d, and stored as one 16-byte piece
+                        const int q = lane & 3;
+                        float P[8], Q[8];   // positions a / c (P) and b / d (Q) of 8 channels
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const float send = (q & 1) ? vh[i] : vh[8 + i];
+                            const float recv = __shfl_xor_sync(0xffffffffu, send, 1);
+                            const float own = (q & 1) ? vh[8 + i] : vh[i];
+                            P[i] = (q & 1) ? recv : own;
+                            Q[i] = (q & 1) ? own : recv;
+                        }
+                        float o4[4];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const float sp = (q & 2) ? P[i] : P[4 + i], sq = (q & 2) ? Q[i] : Q[4 + i];
+                            const float rp = __shfl_xor_sync(0xffffffffu, sp, 2), rq = __shfl_xor_sync(0xffffffffu, sq, 2);
+                            o4[i] = (q & 2) ? max4_first(rp, rq, P[4 + i], Q[4 + i]) : max4_first(P[i], Q[i], rp, rq);
+                        }
+                        if (ri.ok) {
+                            float *yo = yrow + ((int64_t)ri.py * p.pw + ri.px) * p.N + n_base + n0 + h + (q & 1) * 8 +
+                                        (q >> 1) * 4;
+                            *reinterpret_cast<float4 *>(yo) = make_float4(o4[0], o4[1], o4[2], o4[3]);
+                        }
+                    } else if (!DENSE && p.pool) {
                         // lanes 4w .. 4w+3 hold the four positions of one pooling window
 #pragma unroll
                         for (int e = 0; e < 16; ++e) {
@@ -1281,7 +1360,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         // issues an MMA only about every 60 cycles and then waits for its next stage,
         // so while one warp waits the others keep the tensor pipe busy.  The split
         // depends on kt alone: a row's partial sums never depend on its place in the
-        // batch.
+        // batch.  With mma_chain the warps share one accumulator and take the K-steps
+        // in turn: a warp issues K-step g only once the warp before it has issued g - 1
+        // (the token), so the MMAs reach the tensor pipe in K-step order, as from one
+        // warp, while each warp's barrier waits and commits overlap the other's issue.
         const int w = warp - 8;
         if (lane == 0 && w < p.n_mma) {
             const int nmma = p.n_mma, nacc = p.n_acc;
@@ -1298,7 +1380,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 const int64_t use = nacc == 2 ? (i >> 1) : i;
                 if (use >= 1 && !wait_phase<32>(smem_u32(&bar_accempty[a]), (uint32_t)((use - 1) & 1), abort_flag)) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                const uint32_t d = tmem + (uint32_t)((a * nmma + w) * p.acc_cols);
+                const bool chain = p.mma_chain != 0;
+                const uint32_t d = tmem + (uint32_t)((a * p.n_part + (chain ? 0 : w)) * p.acc_cols);
                 // two warps keep dealing across tiles (an odd nK alternates which warp
                 // takes the extra K-step); the epilogue's p0 + p1 is commutative, so a
                 // row's sum does not depend on which partial holds which K-steps
@@ -1309,10 +1392,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         if (!wait_phase<32>(smem_u32(&bar_afull[t]), t_wraps & 1, abort_flag)) { ok = false; break; }
                         if (!p.b_resident &&
                             !wait_phase<32>(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
+                        const uint32_t g = (uint32_t)(i * nK + kt);
+                        if (chain && !wait_turn(smem_u32(&mma_turn_sh), g, abort_flag)) { ok = false; break; }
                         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                         const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
-                        mma_block<THREE, 0, Q>(d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, first ? 0u : 1u);
+                        // shared accumulator: K-step 0 of the tile overwrites
+                        const uint32_t acc0 = chain ? (kt > 0 ? 1u : 0u) : (first ? 0u : 1u);
+                        mma_block<THREE, 0, Q>(d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, acc0);
                         first = false;
+                        if (chain) {
+                            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                            turn_store(smem_u32(&mma_turn_sh), g + 1);
+                        }
                         mma_commit(smem_u32(&bar_aempty[t]));
                         if (!p.b_resident) mma_commit(smem_u32(&bar_bempty[sb]));
                     }
@@ -1642,10 +1733,10 @@ static int mma_gap(int nK, int m)
     return g;
 }
 
-// Tensor-memory layout (512 columns): n_acc sets of n_mma partial accumulators, then
+// Tensor-memory layout (512 columns): n_acc sets of n_part partial accumulators, then
 // n_stages A stages.  A function of the layer alone, so a row's arithmetic never
 // depends on the batch.
-static void tc_config(TcParams &p, int nt_max, bool three)
+static void tc_config(TcParams &p, int nt_max, bool three, bool chain)
 {
     p.acc_cols = round_up32(nt_max);
     // a wide slice's accumulator takes half of tensor memory: one set
@@ -1659,6 +1750,15 @@ static void tc_config(TcParams &p, int nt_max, bool three)
     int m = std::max(1, std::min({3, 256 / (p.n_acc * p.acc_cols), nK}));
     while (m > 1 && mma_gap(nK, m) > depth) --m;
     p.n_mma = m;
+    p.n_part = m;
+    p.mma_chain = 0;
+    if (chain && nK >= 2 && mma_gap(nK, 2) <= depth) {
+        // two issuing warps in turn on one accumulator per set: two sets up to 128
+        // columns, one wide set
+        p.n_mma = 2;
+        p.n_part = 1;
+        p.mma_chain = 1;
+    }
 }
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point (no link to libcuda).
@@ -1815,15 +1915,19 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     if (ss) p.slot = *ss;
     const size_t f_bytes = ff ? 16 + (size_t)ff->F * kFuseClasses * 4 : 0;
     const size_t smem = std::max<size_t>(1024 + b_bytes + a_bytes + f_bytes, 116 * 1024);
-    // partial accumulators: two sets of n_mma in columns 0..255; a function of the layer
+    // partial accumulators: n_acc sets of n_part in columns 0..255; a function of the layer
     // alone, so a row's arithmetic never depends on the batch
-    tc_config(p, nt_max, three);
+    tc_config(p, nt_max, three, S.tc_conv != 0 && !ss);
     // the delta GEMM: one issuing warp, so that a column's sum never depends on how many
     // slots share its batch
-    if (ss) p.n_mma = 1;
+    if (ss) p.n_mma = p.n_part = 1;
     // dense rows without an overlay: A tiles by tensor-map copies from warp 10
     p.a_tma = dense && !p.ov.patch && p.n_mma <= 2 && dense_a_tensor_map(S, x, rm, p.tmap_a) ? 1 : 0;
-    if (S.tc_small || S.tc_conv) p.n_mma = std::min(p.n_mma, 2);   // warp 10 stages maps in those modes
+    if (S.tc_small || S.tc_conv) {
+        // warp 10 stages maps in those modes
+        p.n_mma = std::min(p.n_mma, 2);
+        if (!p.mma_chain) p.n_part = p.n_mma;
+    }
     const int64_t M = (int64_t)rm.R * p.P;
     const int64_t tiles = S.tc_small ? small_tiles(rm.R) : (M + kTileM - 1) / kTileM;
     static int n_sm = 0;
