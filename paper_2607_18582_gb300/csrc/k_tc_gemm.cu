@@ -227,6 +227,20 @@ __device__ __forceinline__ void mma_block(uint32_t d, uint32_t ta, uint64_t dh, 
     }
 }
 
+// The same three products per K8 step in two MMAs (merge_lo): a_hi * [b_hi | b_lo] with
+// instruction descriptor id2 (N = 2 Nt), then a_lo * b_hi with id1 (N = Nt).  A narrow MMA
+// occupies the tensor pipe about as long as one of twice its width, so two instructions
+// per K8 step instead of three.
+__device__ __forceinline__ void mma_block_merged(uint32_t d, uint32_t ta, uint64_t dh, uint32_t id2, uint32_t id1,
+                                                 uint32_t acc0)
+{
+#pragma unroll
+    for (int ks = 0; ks < 4; ++ks) {
+        mma_tf32_ts(d, ta + ks * 8, dh + 2 * ks, id2, ks > 0 ? 1u : acc0);   // a_hi * [b_hi | b_lo]
+        mma_tf32_ts(d, ta + 32 + ks * 8, dh + 2 * ks, id1, 1u);              // a_lo * b_hi
+    }
+}
+
 __device__ __forceinline__ void mma_commit(uint32_t mbar)
 {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar)
@@ -308,6 +322,10 @@ struct TcParams {
                                  // take turns (mma_chain)
     int mma_chain;               // 1: the issuing warps take the K-steps in turn, in K-step
                                  // order, into one accumulator (a token passed in shared memory)
+    int merge_lo;                // 3xTF32 with narrow slices (Nt <= 64): a_hi * [b_hi | b_lo] as
+                                 // one MMA of width 2 Nt (the lo weight panel follows the hi
+                                 // panel) plus a_lo * b_hi; the accumulator's columns Nt .. 2 Nt
+                                 // hold the a_hi * b_lo sums, added to columns 0 .. Nt last
     int acc_cols;                // tensor-memory columns of one partial accumulator
     int n_acc;                   // accumulator sets (tiles in flight): 1 or 2
     int n_stages;                // tensor-memory A stages (<= kMaxNT), from column a_col
@@ -736,7 +754,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         return (int)min((uint32_t)G2::MAPS, (uint32_t)p.R - row0);
     };
     // bulk copies of tile i into buffer b: a map per row and, in one piece, the rows'
-    // patch values (lane 0)
+    // patch values, each from its own lane of the calling warp (one thread's bulk copies
+    // complete one after another)
     auto issue_tile = [&](int64_t i, int b) {
         uint32_t row0;
         const int nimg = tile_rows(i, row0);
@@ -752,15 +771,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 need |= (k >> 16) == 0 && (k & 0xffffu) != 0;
             }
         const uint32_t pbytes = need ? (uint32_t)(nimg * p.ov.row_stride * 4) : 0u;
+        if (lane == 0) mbar_expect_tx(bar, nimg * G2::IMG_B + pbytes);
+        __syncwarp();
         // the buffer was last read and written by generic loads and stores
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        mbar_expect_tx(bar, nimg * G2::IMG_B + pbytes);
-        for (int im = 0; im < nimg; ++im) {
-            const uint32_t row = row0 + im;
+        if (lane < nimg) {
+            const uint32_t row = row0 + lane;
             const int64_t xr = p.x_per_input ? p.t0 + row % (uint32_t)p.T : row;
-            bulk_g2s(buf + im * G2::IMG_B, p.x + xr * p.x_stride, G2::IMG_B, bar);
+            bulk_g2s(buf + lane * G2::IMG_B, p.x + xr * p.x_stride, G2::IMG_B, bar);
         }
-        if (pbytes)
+        if (pbytes && lane == nimg)
             bulk_g2s(ovst_region + (uint32_t)b * G2::OVST_B, p.ov.patch + (int64_t)row0 * p.ov.row_stride, pbytes, bar);
     };
 
@@ -990,6 +1010,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
 #pragma unroll
                         for (int e = 0; e < 16; ++e) v[n0 + e] += u[e];
                     }
+                    if (p.merge_lo) {
+                        float u[16];
+                        tmem_ld16(acc + (uint32_t)G::N + n0, u);
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) v[n0 + e] += u[e];
+                    }
                 }
                 float o[G::OC];
 #pragma unroll
@@ -1042,6 +1068,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     for (int w = 1; w < p.n_part; ++w) {
                         float u[16];
                         tmem_ld16(acc + (uint32_t)(w * p.acc_cols), u);
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) vh[e] += u[e];
+                    }
+                    if (MODE == 3 && p.merge_lo) {
+                        float u[16];
+                        tmem_ld16(acc + (uint32_t)Nt, u);
 #pragma unroll
                         for (int e = 0; e < 16; ++e) vh[e] += u[e];
                     }
@@ -1307,52 +1339,113 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             if (++b == G::NBUF) { b = 0; ++uses; }
         }
     } else if (MODE == 3 && warp == 10) {
-        // ------------------------------------------ staged convolution: overlay --
-        // With an overlay (the first suffix stage), each landed chunk gets the mutated
-        // channels of its batch rows written over the copied values, at every staged
-        // pixel inside the image, before the producers read it.
-        if (p.ov.patch) {
-            int64_t job = 0;
-            bool ok = true;
-            for (int64_t i = 0; ok && i < my_tiles; ++i) {
-                const int64_t m0 = (blockIdx.x + i * gridDim.x) * (int64_t)kTileM;
-                const int64_t row0 = m0 / p.P;
-                const int oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / kTileM) * p.cv_rows;
-                const int nimg = (int)min((int64_t)p.cv_imgs, (int64_t)p.R - row0);
-                const int ncell = p.cv_hw * p.cv_hh;
-                for (int c = 0; c < p.cv_nchunk; ++c, ++job) {
-                    const int b = (int)(job % p.cv_nbuf);
-                    if (!warp_wait_phase<32>(smem_u32(&bar_landed[b]), (uint32_t)(job / p.cv_nbuf) & 1, abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    for (int im = 0; im < nimg; ++im) {
-                        const int64_t row = logical_row(p.lrow, row0 + im);
-                        const int g = (int)(row / p.T);
-                        const int k = p.ov.n_neurons[g];
-                        const int32_t *ids = p.ov.ids + p.ov.neuron_off[g];
-                        const float *prow = p.ov.patch + row * p.ov.row_stride;
-                        const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + (uint32_t)im * p.cv_img_bytes;
-                        for (int q = 0; q < k; ++q) {
-                            const int jl = ids[q] - c * p.cv_cw;
-                            if (jl < 0 || jl >= p.cv_cw) continue;
-                            const float *pq = prow + (int64_t)q * p.ov.cells;
-                            for (int cell = lane; cell < ncell; cell += 32) {
-                                const int hy = cell / p.cv_hw, hx = cell - hy * p.cv_hw;
-                                const int iy = oy0 - p.pad + hy, ix = hx - p.pad;
-                                if ((unsigned)iy >= (unsigned)p.ih || (unsigned)ix >= (unsigned)p.iw) continue;
-                                const uint32_t lin = (uint32_t)cell * 128u + (uint32_t)jl * 4u;
-                                asm volatile("st.shared.f32 [%0], %1;" ::"r"(base + (lin ^ ((lin >> 3) & 0x70u))),
-                                             "f"(__ldg(pq + iy * p.iw + ix))
-                                             : "memory");
-                            }
-                        }
-                    }
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(smem_u32(&bar_ready[b]));
+        // ------------------------------------- staged convolution: input staging --
+        // Lane 0 copies each job's input rows (tile i, chunk c: 32 channels of the rows
+        // with their zero border) into buffer job mod cv_nbuf as soon as the producers
+        // have released it.  With an overlay (the first suffix stage) the warp then
+        // writes the mutated channels of its batch rows over each landed chunk, at every
+        // staged pixel inside the image, before the producers read it.  (A thread's bulk
+        // copies complete one after another, so the weight ring has a thread of its own.)
+        const bool fin = p.ov.patch != nullptr;
+        const int64_t n_jobs = my_tiles * p.cv_nchunk;
+        const uint32_t box_bytes = (uint32_t)p.cv_hw * p.cv_hh * 128u;
+        const uint64_t tmap = reinterpret_cast<uint64_t>(&p.tmap_x);
+        // tile i's first batch row, its first staged output row and its rows
+        auto tile_geo = [&](int64_t i, int64_t &row0, int &oy0) {
+            const int64_t m0 = (blockIdx.x + i * gridDim.x) * (int64_t)kTileM;
+            row0 = m0 / p.P;
+            oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / kTileM) * p.cv_rows;
+            return (int)min((int64_t)p.cv_imgs, (int64_t)p.R - row0);
+        };
+        auto issue = [&](int64_t jc) {
+            const int b = (int)(jc % p.cv_nbuf);
+            const int64_t i = jc / p.cv_nchunk;
+            const int c = (int)(jc - i * p.cv_nchunk);
+            int64_t row0;
+            int oy0;
+            const int nimg = tile_geo(i, row0, oy0);
+            const uint32_t bar = smem_u32(&bar_landed[b]);
+            // the buffer was last read (and written) through the generic proxy
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_expect_tx(bar, (uint32_t)max(nimg, 0) * box_bytes);
+            for (int im = 0; im < nimg; ++im) {
+                const int64_t row = row0 + im;
+                const int src = (int)(p.x_per_input ? p.t0 + logical_row(p.lrow, row) % p.T : row);
+                asm volatile(
+                    "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes "
+                    "[%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(cv_region + (uint32_t)b * cv_buf_bytes +
+                                                                  (uint32_t)im * p.cv_img_bytes),
+                    "l"(tmap), "r"(c * p.cv_cw), "r"(-p.pad), "r"(oy0 - p.pad), "r"(src), "r"(bar)
+                    : "memory");
+            }
+        };
+        int64_t issued = 0;
+        bool ok = true;
+        // the job's buffer once the producers released its previous use (blocking or not)
+        auto try_issue = [&](bool block) -> bool {
+            const int b = (int)(issued % p.cv_nbuf);
+            const int64_t use = issued / p.cv_nbuf;
+            if (use >= 1) {
+                const uint32_t a = smem_u32(&bar_released[b]), par = (uint32_t)((use - 1) & 1);
+                if (block) {
+                    if (!warp_wait_phase<32>(a, par, abort_flag)) { ok = false; return false; }
+                } else if (!__all_sync(0xffffffffu, mbar_try(a, par))) {
+                    return false;
                 }
             }
+            if (lane == 0) issue(issued);
+            __syncwarp();
+            ++issued;
+            return true;
+        };
+        for (int64_t job = 0; ok && job < n_jobs; ++job) {
+            while (ok && issued <= job) try_issue(true);
+            if (!ok) break;
+            if (fin) {
+                const int b = (int)(job % p.cv_nbuf);
+                if (!warp_wait_phase<32>(smem_u32(&bar_landed[b]), (uint32_t)(job / p.cv_nbuf) & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                const int64_t i = job / p.cv_nchunk;
+                const int c = (int)(job - i * p.cv_nchunk);
+                int64_t row0;
+                int oy0;
+                const int nimg = tile_geo(i, row0, oy0);
+                const int ncell = p.cv_hw * p.cv_hh;
+                for (int im = 0; im < nimg; ++im) {
+                    const int64_t row = logical_row(p.lrow, row0 + im);
+                    const int g = (int)(row / p.T);
+                    const int k = p.ov.n_neurons[g];
+                    const int32_t *ids = p.ov.ids + p.ov.neuron_off[g];
+                    const float *prow = p.ov.patch + row * p.ov.row_stride;
+                    const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + (uint32_t)im * p.cv_img_bytes;
+                    for (int q = 0; q < k; ++q) {
+                        const int jl = ids[q] - c * p.cv_cw;
+                        if (jl < 0 || jl >= p.cv_cw) continue;
+                        const float *pq = prow + (int64_t)q * p.ov.cells;
+                        for (int cell = lane; cell < ncell; cell += 32) {
+                            const int hy = cell / p.cv_hw, hx = cell - hy * p.cv_hw;
+                            const int iy = oy0 - p.pad + hy, ix = hx - p.pad;
+                            if ((unsigned)iy >= (unsigned)p.ih || (unsigned)ix >= (unsigned)p.iw) continue;
+                            const uint32_t lin = (uint32_t)cell * 128u + (uint32_t)jl * 4u;
+                            asm volatile("st.shared.f32 [%0], %1;" ::"r"(base + (lin ^ ((lin >> 3) & 0x70u))),
+                                         "f"(__ldg(pq + iy * p.iw + ix))
+                                         : "memory");
+                        }
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bar_ready[b]));
+            }
+            // run ahead while buffers are free, without holding up the next job's overlay
+            while (ok && issued < n_jobs && issued < job + p.cv_nbuf && try_issue(!fin)) {
+            }
         }
+        // the copies still in flight land before the shared memory is released
+        if (lane == 0)
+            for (int64_t jj = issued > p.cv_nbuf ? issued - p.cv_nbuf : 0; jj < issued; ++jj)
+                wait_phase_drain(smem_u32(&bar_landed[jj % p.cv_nbuf]), (uint32_t)((jj / p.cv_nbuf) & 1));
     } else if (warp < 11) {
         // ------------------------------------------------------------------ MMA --
         // The K-steps of a tile are dealt to the n_mma issuing warps by their index
@@ -1368,7 +1461,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         if (lane == 0 && w < p.n_mma) {
             const int nmma = p.n_mma, nacc = p.n_acc;
             constexpr int Q = THREE ? 12 : 4;
-            const uint32_t id = idesc_tf32(kTileM, Nt);
+            const uint32_t id = idesc_tf32(kTileM, Nt), id2 = idesc_tf32(kTileM, 2 * Nt);
+            const bool merged = THREE && p.merge_lo;
             bool ok = true;
             if (p.b_resident) ok = wait_phase<32>(smem_u32(&bar_bfull[0]), 0, abort_flag);
             const uint64_t desc_b0 = sw128_desc(b_region);
@@ -1398,7 +1492,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
                         // shared accumulator: K-step 0 of the tile overwrites
                         const uint32_t acc0 = chain ? (kt > 0 ? 1u : 0u) : (first ? 0u : 1u);
-                        mma_block<THREE, 0, Q>(d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, acc0);
+                        if (merged) mma_block_merged(d, tmem + p.a_col + t * kAColsPerStage, dh, id2, id, acc0);
+                        else mma_block<THREE, 0, Q>(d, tmem + p.a_col + t * kAColsPerStage, dh, dl, id, acc0);
                         first = false;
                         if (chain) {
                             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -1421,13 +1516,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     } else {
         // -------------------------------------------------------------- weights --
         if (MODE == 3 && lane == 0) {
-            // one thread issues both rings in the order they are consumed, each copy as
-            // soon as its slot is free: the staged chunks (released by the producers)
-            // and the weight K-steps (released by the MMAs)
-            const int64_t n_jobs = my_tiles * p.cv_nchunk;
+            // the weight K-steps, each copy as soon as the MMAs have released its slot (the
+            // staged input rows come from warp 10)
             const int64_t n_b = p.b_resident ? 0 : total;
-            const uint32_t box_bytes = (uint32_t)p.cv_hw * p.cv_hh * 128u;
-            const uint64_t tmap = reinterpret_cast<uint64_t>(&p.tmap_x);
             if (p.b_resident) {
                 const uint32_t bytes = (uint32_t)nK * b_step;
                 mbar_expect_tx(smem_u32(&bar_bfull[0]), bytes);
@@ -1435,63 +1526,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     bulk_g2s(b_region + o, (const unsigned char *)wslice + o, min(32768u, bytes - o),
                              smem_u32(&bar_bfull[0]));
             }
-            int64_t jc = 0, jb = 0;
-            long long t_idle = clock64();
-            while (jc < n_jobs || jb < n_b) {
-                bool moved = false;
-                if (jc < n_jobs) {
-                    const int b = (int)(jc % p.cv_nbuf);
-                    const int64_t use = jc / p.cv_nbuf;
-                    if (use == 0 || mbar_try(smem_u32(&bar_released[b]), (uint32_t)((use - 1) & 1))) {
-                        const int64_t i = jc / p.cv_nchunk;
-                        const int c = (int)(jc - i * p.cv_nchunk);
-                        const int64_t m0 = (blockIdx.x + i * gridDim.x) * (int64_t)kTileM;
-                        const int64_t row0 = m0 / p.P;
-                        const int oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / kTileM) * p.cv_rows;
-                        const int nimg = (int)min((int64_t)p.cv_imgs, (int64_t)p.R - row0);
-                        const uint32_t bar = smem_u32(&bar_landed[b]);
-                        // the buffer was last read (and written) through the generic proxy
-                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                        mbar_expect_tx(bar, (uint32_t)nimg * box_bytes);
-                        for (int im = 0; im < nimg; ++im) {
-                            const int64_t row = row0 + im;
-                            const int src = (int)(p.x_per_input ? p.t0 + logical_row(p.lrow, row) % p.T : row);
-                            asm volatile(
-                                "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes "
-                                "[%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(cv_region + (uint32_t)b * cv_buf_bytes +
-                                                                              (uint32_t)im * p.cv_img_bytes),
-                                "l"(tmap), "r"(c * p.cv_cw), "r"(-p.pad), "r"(oy0 - p.pad), "r"(src), "r"(bar)
-                                : "memory");
-                        }
-                        ++jc;
-                        moved = true;
-                    }
-                }
-                if (jb < n_b) {
-                    const int sb = (int)(jb % p.nb);
-                    const int64_t use = jb / p.nb;
-                    if (use == 0 || mbar_try(smem_u32(&bar_bempty[sb]), (uint32_t)((use - 1) & 1))) {
-                        mbar_expect_tx(smem_u32(&bar_bfull[sb]), b_step);
-                        bulk_g2s(b_region + (uint32_t)sb * b_step, (const unsigned char *)wslice + (size_t)(jb % nK) * b_step,
-                                 b_step, smem_u32(&bar_bfull[sb]));
-                        ++jb;
-                        moved = true;
-                    }
-                }
-                if (moved) {
-                    t_idle = clock64();
-                    continue;
-                }
-                if (abort_flag->abort) break;
-                if (clock64() - t_idle > abort_flag->limit) {
-                    abort_flag->abort = 1;
-                    break;
-                }
-                __nanosleep(32);
+            int64_t jb = 0;
+            for (; jb < n_b; ++jb) {
+                const int sb = (int)(jb % p.nb);
+                const int64_t use = jb / p.nb;
+                if (use >= 1 && !wait_phase<32>(smem_u32(&bar_bempty[sb]), (uint32_t)((use - 1) & 1), abort_flag)) break;
+                mbar_expect_tx(smem_u32(&bar_bfull[sb]), b_step);
+                bulk_g2s(b_region + (uint32_t)sb * b_step, (const unsigned char *)wslice + (size_t)(jb % nK) * b_step,
+                         b_step, smem_u32(&bar_bfull[sb]));
             }
             // the copies still in flight land before the shared memory is released
-            for (int64_t jj = jc > p.cv_nbuf ? jc - p.cv_nbuf : 0; jj < jc; ++jj)
-                wait_phase_drain(smem_u32(&bar_landed[jj % p.cv_nbuf]), (uint32_t)((jj / p.cv_nbuf) & 1));
             for (int64_t jj = jb > p.nb ? jb - p.nb : 0; jj < jb; ++jj)
                 wait_phase_drain(smem_u32(&bar_bfull[(int)(jj % p.nb)]), (uint32_t)((jj / p.nb) & 1));
         } else if (lane == 0) {
@@ -1529,7 +1573,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             uint32_t uses = 0;
             for (; issued < my_tiles; ++issued) {
                 if (issued >= G::NBUF && !warp_wait_phase<32>(smem_u32(&bar_released[b]), (uses - 1) & 1, abort_flag)) break;
-                if (lane == 0) issue_tile(issued, b);
+                issue_tile(issued, b);
                 __syncwarp();
                 if (++b == G::NBUF) { b = 0; ++uses; }
             }
@@ -1738,7 +1782,7 @@ static int mma_gap(int nK, int m)
 // depends on the batch.
 static void tc_config(TcParams &p, int nt_max, bool three, bool chain)
 {
-    p.acc_cols = round_up32(nt_max);
+    p.acc_cols = round_up32(p.merge_lo ? 2 * nt_max : nt_max);
     // a wide slice's accumulator takes half of tensor memory: one set
     p.n_acc = p.acc_cols > 128 ? 1 : 2;
     p.a_col = 256;
@@ -1917,6 +1961,8 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     const size_t smem = std::max<size_t>(1024 + b_bytes + a_bytes + f_bytes, 116 * 1024);
     // partial accumulators: n_acc sets of n_part in columns 0..255; a function of the layer
     // alone, so a row's arithmetic never depends on the batch
+    // (the window GEMM keeps two partial accumulators: measured as fast, no merged MMAs)
+    p.merge_lo = S.tc_conv && three && !ss && nt_max <= 64 ? 1 : 0;
     tc_config(p, nt_max, three, S.tc_conv != 0 && !ss);
     // the delta GEMM: one issuing warp, so that a column's sum never depends on how many
     // slots share its batch
