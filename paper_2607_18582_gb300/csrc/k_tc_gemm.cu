@@ -171,33 +171,6 @@ __device__ __forceinline__ void wait_phase_drain(uint32_t a, uint32_t parity)
         if (clock64() - t0 > kSpin) return;
 }
 
-// The issuing warps' turn token: K-step g of the CTA's sequence may be issued once the
-// counter reads g (acquire), and its issuer then publishes g + 1 (release).  Bounded like
-// the barrier waits.
-__device__ __forceinline__ uint32_t turn_load(uint32_t a)
-{
-    uint32_t v;
-    asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
-    return v;
-}
-
-__device__ __forceinline__ void turn_store(uint32_t a, uint32_t v)
-{
-    asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
-}
-
-__device__ __forceinline__ bool wait_turn(uint32_t a, uint32_t g, volatile WaitCtl *abort_flag)
-{
-    if (turn_load(a) == g) return true;
-    const long long t0 = clock64();
-    for (;;) {
-        __nanosleep(20);   // leaves the issue slots to the epilogue warp of the sub-partition
-        if (turn_load(a) == g) return true;
-        if (abort_flag->abort) return false;
-        if (clock64() - t0 > abort_flag->limit) { abort_flag->abort = 1; return false; }
-    }
-}
-
 // A from tensor memory, B from shared memory.
 __device__ __forceinline__ void mma_tf32_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc)
 {
@@ -321,7 +294,7 @@ struct TcParams {
     int n_part;                  // partial accumulators per set: n_mma, or 1 when the warps
                                  // take turns (mma_chain)
     int mma_chain;               // 1: the issuing warps take the K-steps in turn, in K-step
-                                 // order, into one accumulator (a token passed in shared memory)
+                                 // order, into one accumulator (handed over by barrier arrivals)
     int merge_lo;                // 3xTF32 with narrow slices (Nt <= 64): a_hi * [b_hi | b_lo] as
                                  // one MMA of width 2 Nt (the lo weight panel follows the hi
                                  // panel) plus a_lo * b_hi; the accumulator's columns Nt .. 2 Nt
@@ -649,7 +622,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     // dense A tiles by tensor-map copies: slot landed, slot read by the producers
     __shared__ __align__(8) uint64_t bar_alanded[kNA], bar_afree[kNA];
     __shared__ uint32_t tmem_sh;
-    __shared__ uint32_t mma_turn_sh;   // mma_chain: the next K-step to issue
+    // mma_chain: warp w's turn comes with an arrival on bar_turn[w] from the other warp
+    __shared__ __align__(8) uint64_t bar_turn[2];
     __shared__ WaitCtl abort_sh;
     __shared__ float bias_sh[kSliceMax];
     __shared__ __align__(16) float epi_stage[4][32 * kEpiStride];   // per epilogue warp: 32 rows x 32 values
@@ -735,7 +709,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             mbar_init(smem_u32(&bar_released[s]), 4);
         }
         abort_sh.abort = 0;
-        mma_turn_sh = 0;
+        mbar_init(smem_u32(&bar_turn[0]), 1);
+        mbar_init(smem_u32(&bar_turn[1]), 1);
         abort_sh.limit = p.spin > 0 ? p.spin : kSpin;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -1455,14 +1430,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         // depends on kt alone: a row's partial sums never depend on its place in the
         // batch.  With mma_chain the warps share one accumulator and take the K-steps
         // in turn: a warp issues K-step g only once the warp before it has issued g - 1
-        // (the token), so the MMAs reach the tensor pipe in K-step order, as from one
-        // warp, while each warp's barrier waits and commits overlap the other's issue.
+        // (an arrival on the turn barrier), so the MMAs reach the tensor pipe in K-step
+        // order, as from one warp, while each warp's barrier waits and commits overlap
+        // the other's issue.  (A barrier is never two phases ahead of its waiter: the
+        // other warp's next turn waits for this warp's arrival.)
         const int w = warp - 8;
         if (lane == 0 && w < p.n_mma) {
             const int nmma = p.n_mma, nacc = p.n_acc;
             constexpr int Q = THREE ? 12 : 4;
             const uint32_t id = idesc_tf32(kTileM, Nt), id2 = idesc_tf32(kTileM, 2 * Nt);
-            const bool merged = THREE && p.merge_lo;
+            // (the window GEMM never takes these paths: compiled out of its latency-bound
+            // issuing loop)
+            const bool merged = MODE == 3 && THREE && p.merge_lo;
             bool ok = true;
             if (p.b_resident) ok = wait_phase<32>(smem_u32(&bar_bfull[0]), 0, abort_flag);
             const uint64_t desc_b0 = sw128_desc(b_region);
@@ -1474,7 +1453,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 const int64_t use = nacc == 2 ? (i >> 1) : i;
                 if (use >= 1 && !wait_phase<32>(smem_u32(&bar_accempty[a]), (uint32_t)((use - 1) & 1), abort_flag)) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                const bool chain = p.mma_chain != 0;
+                const bool chain = MODE != 2 && p.mma_chain != 0;
                 const uint32_t d = tmem + (uint32_t)((a * p.n_part + (chain ? 0 : w)) * p.acc_cols);
                 // two warps keep dealing across tiles (an odd nK alternates which warp
                 // takes the extra K-step); the epilogue's p0 + p1 is commutative, so a
@@ -1487,7 +1466,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         if (!p.b_resident &&
                             !wait_phase<32>(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
                         const uint32_t g = (uint32_t)(i * nK + kt);
-                        if (chain && !wait_turn(smem_u32(&mma_turn_sh), g, abort_flag)) { ok = false; break; }
+                        // K-step g goes to warp g mod 2; it waits for the other warp's
+                        // arrival after K-step g - 1, the ((g + w) / 2)-th on its barrier
+                        if (chain && g > 0 &&
+                            !wait_phase<0>(smem_u32(&bar_turn[w]), (((g + (uint32_t)w) >> 1) + 1) & 1, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
                         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                         const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
                         // shared accumulator: K-step 0 of the tile overwrites
@@ -1497,7 +1482,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         first = false;
                         if (chain) {
                             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-                            turn_store(smem_u32(&mma_turn_sh), g + 1);
+                            mbar_arrive(smem_u32(&bar_turn[1 - w]));
                         }
                         mma_commit(smem_u32(&bar_aempty[t]));
                         if (!p.b_resident) mma_commit(smem_u32(&bar_bempty[sb]));
@@ -1962,11 +1947,12 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     // partial accumulators: n_acc sets of n_part in columns 0..255; a function of the layer
     // alone, so a row's arithmetic never depends on the batch
     // (the window GEMM keeps two partial accumulators: measured as fast, no merged MMAs)
+    // (not in the delta GEMM, whose slice width depends on the slots of its batch)
     p.merge_lo = S.tc_conv && three && !ss && nt_max <= 64 ? 1 : 0;
-    tc_config(p, nt_max, three, S.tc_conv != 0 && !ss);
-    // the delta GEMM: one issuing warp, so that a column's sum never depends on how many
-    // slots share its batch
-    if (ss) p.n_mma = p.n_part = 1;
+    tc_config(p, nt_max, three, !S.tc_small);
+    // the delta GEMM: one issuing warp (or two in turn, which is the same sum), so that a
+    // column's sum never depends on how many slots share its batch
+    if (ss && !p.mma_chain) p.n_mma = p.n_part = 1;
     // dense rows without an overlay: A tiles by tensor-map copies from warp 10
     p.a_tma = dense && !p.ov.patch && p.n_mma <= 2 && dense_a_tensor_map(S, x, rm, p.tmap_a) ? 1 : 0;
     if (S.tc_small || S.tc_conv) {
