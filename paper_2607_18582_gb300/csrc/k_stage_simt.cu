@@ -390,6 +390,112 @@ __global__ void __launch_bounds__(128) k_final_dense(const FinalParams p)
     epilogue_reg<CP>(p.fa, p.t0, p.T, row, in_range, v, p.C);
 }
 
+// The same output layer with each warp on its own 32 rows (lane = row) and no block-wide
+// barrier after the weights are staged: the warp copies its rows' next 32 inputs (16-byte
+// loads, eight per lane) while it runs the FMAs of the current 32, through a per-warp
+// shared-memory tile.  Each row's sums are the same fp32 chain as k_final_dense's (f
+// ascending from +0, fmaf(x, w, acc), then + b), so both kernels give the same bits.
+// (One launch of k_final_dense on 6,144 rows of 512 inputs waited 256 us on its loads.)
+// Needs F a multiple of 4 and 16-byte aligned rows; the weights [F][CP] in dynamic shared
+// memory.
+template <int CP>
+__global__ void __launch_bounds__(128) k_final_dense_w(const FinalParams p)
+{
+    extern __shared__ __align__(16) float wsm[];   // [F][CP]
+    __shared__ float xs[4][32][33];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int i = threadIdx.x; i < p.F * CP; i += blockDim.x) {
+        const int f = i / CP, c = i - f * CP;
+        wsm[i] = c < p.C ? __ldg(p.W + (int64_t)c * p.F + f) : 0.f;
+    }
+    __syncthreads();
+    const int64_t row0 = (int64_t)blockIdx.x * 128 + warp * 32;
+    const int64_t row = row0 + lane;
+    const bool in_range = row < p.R;
+    int ov_k = 0;
+    const int32_t *ov_ids = nullptr;
+    const int64_t lrow = in_range ? logical_row(p.lrow, row) : row;
+    if (p.ov.patch && in_range) {
+        const int g = (int)(lrow / p.T);
+        ov_k = p.ov.n_neurons[g];
+        ov_ids = p.ov.ids + p.ov.neuron_off[g];
+    }
+    // this lane copies 16 bytes (inputs 4 (lane mod 8) .. +3) of rows 4i + lane / 8
+    const int fq = 4 * (lane & 7);
+    const float *src[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int64_t r = row0 + 4 * i + (lane >> 3);
+        src[i] = r < p.R ? p.x + (p.x_per_input ? (p.t0 + logical_row(p.lrow, r) % p.T) : r) * p.x_stride : nullptr;
+    }
+    auto load = [&](int f0, float4 (&v)[8]) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            v[i] = (src[i] && f0 + fq < p.F) ? __ldg(reinterpret_cast<const float4 *>(src[i] + f0 + fq))
+                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+    };
+    float acc[CP];
+#pragma unroll
+    for (int c = 0; c < CP; ++c) acc[c] = 0.f;
+    float4 cur[8];
+    load(0, cur);
+    for (int f0 = 0; f0 < p.F; f0 += 32) {
+        __syncwarp();
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            float *d = &xs[warp][4 * i + (lane >> 3)][fq];
+            d[0] = cur[i].x; d[1] = cur[i].y; d[2] = cur[i].z; d[3] = cur[i].w;
+        }
+        if (f0 + 32 < p.F) load(f0 + 32, cur);
+        __syncwarp();
+        const int fe = min(32, p.F - f0);
+        // overlay on this lane's own row (no other lane reads it)
+        for (int q = 0; q < ov_k; ++q) {
+            const int j = ov_ids[q];
+            const int cfirst = f0 - j <= 0 ? 0 : (f0 - j + p.ov.ch - 1) / p.ov.ch;
+            for (int c = cfirst; c < p.ov.cells && c * p.ov.ch + j < f0 + fe; ++c)
+                xs[warp][lane][c * p.ov.ch + j - f0] = p.ov.patch[lrow * p.ov.row_stride + q * p.ov.cells + c];
+        }
+        for (int fl = 0; fl < fe; ++fl) {
+            const float xv = xs[warp][lane][fl];
+            const float *wr = wsm + (f0 + fl) * CP;
+#pragma unroll
+            for (int c4 = 0; c4 < CP; c4 += 4) {
+                const float4 w4 = *reinterpret_cast<const float4 *>(wr + c4);
+                acc[c4] = fmaf(xv, w4.x, acc[c4]);
+                acc[c4 + 1] = fmaf(xv, w4.y, acc[c4 + 1]);
+                acc[c4 + 2] = fmaf(xv, w4.z, acc[c4 + 2]);
+                acc[c4 + 3] = fmaf(xv, w4.w, acc[c4 + 3]);
+            }
+        }
+    }
+    float v[CP];
+#pragma unroll
+    for (int c = 0; c < CP; ++c) {
+        const float z = c < p.C ? acc[c] + __ldg(p.b + c) : 0.f;
+        if (in_range && c < p.C && p.fa.z_out) p.fa.z_out[row * p.fa.z_stride + c] = z;
+        v[c] = act_apply(p.act, z);
+    }
+    if (p.fa.mode == 1) {  // cache build: logits rows and original predictions
+        if (in_range) {
+#pragma unroll
+            for (int c = 0; c < CP; ++c)
+                if (c < p.C) p.fa.x_out[row * p.fa.x_stride + c] = v[c];
+            p.fa.pred_out[row] = argmax_reg<CP>(v, p.C);
+        }
+        return;
+    }
+    if (p.fa.mode == 2) {  // per-row logits for a following delta + epilogue
+        if (in_range) {
+#pragma unroll
+            for (int c = 0; c < CP; ++c)
+                if (c < p.C) p.fa.logits_rows[row * p.fa.x_stride + c] = v[c];
+        }
+        return;
+    }
+    epilogue_reg<CP>(p.fa, p.t0, p.T, row, in_range, v, p.C);
+}
+
 __global__ void __launch_bounds__(128) k_epilogue(const float *__restrict__ lg, int64_t stride, int per_input, int C,
                                                   int64_t t0, int T, int R, const FinalArgs fa, const Overlay ov)
 {
@@ -510,6 +616,20 @@ int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cu
         const size_t smem = ((size_t)p.F * 12 + 128 * kRowsF) * sizeof(float);
         cudaFuncSetAttribute(k_final_dense_rows<12, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         k_final_dense_rows<12, 3><<<blocks, 128, smem, s>>>(p);
+        return 1;
+    }
+    // aligned rows of whole 16-byte pieces, weights that fit in shared memory: per-warp rows
+    // with the next inputs in flight
+    const size_t wbytes = (size_t)p.F * cp * sizeof(float);
+    if (p.F % 4 == 0 && (x.stride & 3) == 0 && (reinterpret_cast<uintptr_t>(x.p) & 15) == 0 && cp <= 12 &&
+        wbytes <= 96 * 1024) {
+        auto go = [&](auto kern) {
+            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)wbytes);
+            kern<<<blocks, 128, wbytes, s>>>(p);
+        };
+        if (cp <= 4) go(k_final_dense_w<4>);
+        else if (cp <= 8) go(k_final_dense_w<8>);
+        else go(k_final_dense_w<12>);
         return 1;
     }
     if (cp <= 4) k_final_dense<4><<<blocks, 128, 0, s>>>(p);
