@@ -14,6 +14,17 @@ using namespace mure;
 
 namespace {
 
+// Mutants per batch the input tile is sized for (MURE_BATCH_MUTANTS overrides; at least 1).
+int64_t batch_mutants()
+{
+    static int64_t v = 0;
+    if (!v) {
+        const char *e = getenv("MURE_BATCH_MUTANTS");
+        v = e && atoi(e) > 0 ? atoi(e) : 16;
+    }
+    return v;
+}
+
 // MURE_TC_CONV: in the tensor-core modes the LeNet-size convolution runs in the
 // small-image mode (a GEMM row per pooling window); "0" keeps its CUDA-core kernel,
 // "generic" runs it through the implicit-GEMM producers (one row per position).
@@ -1126,7 +1137,11 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
             }
         int64_t rows = std::max<int64_t>(cap / std::max<int64_t>(rb, 1), 64);
         rows = std::min<int64_t>(rows, (int64_t)1 << 24);
-        int64_t T = std::min<int64_t>(ca->n_pad, rows / 64 * 64);
+        // the input tile leaves room for batch_mutants() mutants per batch: the delta's
+        // tensor-core GEMM is as wide as a batch's mutated channels, and each cached input
+        // row staged by the delta kernels serves every mutant of the batch (rows per
+        // batch, and so the suffix's work per launch, stay the same)
+        int64_t T = std::min<int64_t>(ca->n_pad, std::max<int64_t>(64, rows / batch_mutants() / 64 * 64));
         const int64_t Gmax = std::max<int64_t>(1, rows / T);
         // never more rows than the largest group needs
         int64_t gbig = 0;
