@@ -295,6 +295,9 @@ struct TcParams {
                                  // take turns (mma_chain)
     int mma_chain;               // 1: the issuing warps take the K-steps in turn, in K-step
                                  // order, into one accumulator (handed over by barrier arrivals)
+    int cv_pair;                 // MODE 3: units of two 128-row tiles (rows r and 128 + r per
+                                 // producer thread; MMA warp w issues tile w; one weight stage
+                                 // serves both)
     int merge_lo;                // 3xTF32 with narrow slices (Nt <= 64): a_hi * [b_hi | b_lo] as
                                  // one MMA of width 2 Nt (the lo weight panel follows the hi
                                  // panel) plus a_lo * b_hi; the accumulator's columns Nt .. 2 Nt
@@ -646,7 +649,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     const uint32_t fw_region = (ov_region + (p.ov.patch ? kNA * kOvSlotBytes : 0) + 15u) & ~15u;
     const float4 *fw4 = reinterpret_cast<const float4 *>(smraw + (fw_region - smem_u32(smraw)));
     const int64_t M = (int64_t)p.R * p.P;
-    const int64_t n_tiles = MODE == 2 ? small_tiles(p.R) : (M + kTileM - 1) / kTileM;
+    // MODE 3 with cv_pair: a unit of two tiles (rows m0 .. m0 + 255) per iteration
+    const bool pair = MODE == 3 && p.cv_pair;
+    const int64_t TM = pair ? 2 * kTileM : kTileM;
+    const int64_t n_tiles = MODE == 2 ? small_tiles(p.R) : (M + TM - 1) / TM;
     const int64_t my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
     const int64_t total = my_tiles * nK;
     const float *wslice = p.Wsw + (int64_t)blockIdx.y * p.w_slice_floats;
@@ -688,11 +694,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
     if (threadIdx.x == 32) {
         for (int s = 0; s < kNT; ++s) {
             mbar_init(smem_u32(&bar_afull[s]), 4);
-            mbar_init(smem_u32(&bar_aempty[s]), 1);     // each K-step has one issuing warp
+            // each K-step has one issuing warp (two with tile pairs, one per tile)
+            mbar_init(smem_u32(&bar_aempty[s]), pair ? 2 : 1);
         }
         for (int s = 0; s < kNB; ++s) {
             mbar_init(smem_u32(&bar_bfull[s]), 1);
-            mbar_init(smem_u32(&bar_bempty[s]), 1);
+            mbar_init(smem_u32(&bar_bempty[s]), pair ? 2 : 1);
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(smem_u32(&bar_accfull[s]), p.n_mma);
@@ -786,6 +793,33 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             if (++t == p.n_stages) { t = 0; ++wraps; }
             return true;
         };
+        // tile pairs: the K-step of row r (part 0), then of row 128 + r (part 1), into one
+        // stage of 2 kAColsPerStage columns; the stage goes to the MMA warps after part 1
+        auto push_part = [&](float (&hi)[kTileK], int part) -> bool {
+            float lo[kTileK];
+#pragma unroll
+            for (int i = 0; i < kTileK; ++i) {
+                const float h = tf32_hi(hi[i]);
+                if (THREE) lo[i] = hi[i] - h;
+                hi[i] = h;
+            }
+            if (part == 0) {
+                if (wraps >= 1 && !warp_wait_phase<32>(smem_u32(&bar_aempty[t]), (wraps - 1) & 1, abort_flag))
+                    return false;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            }
+            const uint32_t ta = tmem + lane_off + p.a_col + (uint32_t)(t * 2 + part) * kAColsPerStage;
+            tmem_st32(ta, hi);
+            if (THREE) tmem_st32(ta + 32, lo);
+            asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");   // the registers are reused
+            if (part == 1) {
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bar_afull[t]));
+                if (++t == p.n_stages) { t = 0; ++wraps; }
+            }
+            return true;
+        };
         if constexpr (MODE == 2) {
             // warps 10 and 11 stage each tile's maps (mutated channels written in) in
             // buffer i mod NBUF; the producers only gather from them
@@ -816,13 +850,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
             bool ok = true;
             int64_t job = 0;
             for (int64_t i = 0; ok && i < my_tiles; ++i) {
-                const int64_t m0 = (blockIdx.x + i * gridDim.x) * (int64_t)kTileM;
-                const RowInfo ri = row_info<false, false>(p, m0 + r);
+                const int64_t m0 = (blockIdx.x + i * gridDim.x) * TM;
                 const int64_t row0 = m0 / p.P;
-                const int oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / kTileM) * p.cv_rows;
-                // rows past the end gather from the tile's first staged row (dropped later)
+                const int oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / TM) * p.cv_rows;
+                // rows past the end gather from the unit's first staged row (dropped later)
+                const RowInfo ri = row_info<false, false>(p, m0 + r);
                 const uint32_t im = ri.ok ? (uint32_t)(ri.row - row0) : 0u;
                 const int line0 = ri.ok ? (ri.oy - oy0) * p.cv_hw + ri.ox : 0;
+                // tile pairs: this thread's row of the second tile too
+                uint32_t im1 = 0;
+                int line1 = 0;
+                if (pair) {
+                    const RowInfo r1 = row_info<false, false>(p, m0 + kTileM + r);
+                    im1 = r1.ok ? (uint32_t)(r1.row - row0) : 0u;
+                    line1 = r1.ok ? (r1.oy - oy0) * p.cv_hw + r1.ox : 0;
+                }
                 for (int c = 0; c < p.cv_nchunk; ++c, ++job) {
                     const int b = (int)(job % p.cv_nbuf);
                     const uint32_t use = (uint32_t)(job / p.cv_nbuf);
@@ -830,9 +872,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         ok = false;
                         break;
                     }
-                    const uint32_t base = cv_region + (uint32_t)b * cv_buf_bytes + im * p.cv_img_bytes;
+                    const uint32_t buf = cv_region + (uint32_t)b * cv_buf_bytes;
+                    const uint32_t base = buf + im * p.cv_img_bytes, base1 = buf + im1 * p.cv_img_bytes;
                     const int ntap = p.kh * p.kw;
-                    // the current tap and its line relative to line0 (ky * cv_hw + kx)
+                    // the current tap and its line relative to a row's line0 (ky * cv_hw + kx)
                     int tap = 0, kx = 0, off = 0;
                     auto next_tap = [&]() {
                         ++tap;
@@ -844,9 +887,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         }
                     };
                     // chunk cc of line l sits at l * 128 + (cc ^ (l mod 8)) * 16
-                    auto gather = [&](float *v, int nc) {
-                        const uint32_t l = (uint32_t)(line0 + off);
-                        const uint32_t a = base + l * 128u, sw = l & 7u;
+                    auto gather = [&](float *v, int nc, uint32_t bse, int line) {
+                        const uint32_t l = (uint32_t)line;
+                        const uint32_t a = bse + l * 128u, sw = l & 7u;
 #pragma unroll
                         for (int cc = 0; cc < 8; ++cc) {
                             if (cc >= nc) break;
@@ -856,24 +899,38 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                         }
                     };
                     for (int ks = 0; ks < p.cv_taps; ++ks) {
-                        float v[kTileK];
-                        if (p.cv_cw == kTileK) {
-                            gather(v, 8);
-                            next_tap();
-                        } else {
-                            // two taps of 16 channels (the first half of their lines); past
-                            // the last tap the K-step's second half is zero
-                            gather(v, 4);
-                            next_tap();
-                            if (tap < ntap) {
-                                gather(v + 16, 4);
-                            } else {
-#pragma unroll
-                                for (int e = 16; e < kTileK; ++e) v[e] = 0.f;
-                            }
+                        // this K-step's taps: one of 32 channels, or two of 16 (the first
+                        // half of their lines; past the last tap the second half is zero)
+                        const int offa = off;
+                        next_tap();
+                        int offb = -1;
+                        if (p.cv_cw != kTileK) {
+                            if (tap < ntap) offb = off;
                             next_tap();
                         }
-                        if (!push(v)) { ok = false; break; }
+                        auto gather_k = [&](float (&v)[kTileK], uint32_t bse, int l0) {
+                            if (p.cv_cw == kTileK) {
+                                gather(v, 8, bse, l0 + offa);
+                            } else {
+                                gather(v, 4, bse, l0 + offa);
+                                if (offb >= 0) {
+                                    gather(v + 16, 4, bse, l0 + offb);
+                                } else {
+#pragma unroll
+                                    for (int e = 16; e < kTileK; ++e) v[e] = 0.f;
+                                }
+                            }
+                        };
+                        float v[kTileK];
+                        gather_k(v, base, line0);
+                        if (pair) {
+                            if (!push_part(v, 0)) { ok = false; break; }
+                            gather_k(v, base1, line1);
+                            if (!push_part(v, 1)) { ok = false; break; }
+                        } else if (!push(v)) {
+                            ok = false;
+                            break;
+                        }
                     }
                     // every gather of the chunk has been consumed by push: the buffer is free
                     __syncwarp();
@@ -1016,7 +1073,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
                 continue;
             }
-            const RowInfo ri = row_info<DENSE, false>(p, tile * kTileM + qd * 32 + lane);
+            // tile pairs: the unit's two tiles one after the other, each from its own
+            // accumulator; the accumulator set is released after the second
+            const int nsub = pair ? 2 : 1;
+            for (int sub = 0; sub < nsub; ++sub) {
+            const uint32_t abase = pair ? (uint32_t)((a * 2 + sub) * p.acc_cols) : (uint32_t)(a * p.n_part * p.acc_cols);
+            const RowInfo ri = row_info<DENSE, false>(p, (tile * nsub + sub) * kTileM + qd * 32 + lane);
             const float *srow = nullptr;
             if (p.has_add && ri.ok)
                 srow = p.skip + (p.skip_per_input ? p.t0 + logical_row(p.lrow, ri.row) % p.T : ri.row) * p.skip_stride;
@@ -1038,7 +1100,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     if (h >= nc) break;
                     float *vh = v + h;
                     // the accumulator: the n_part partials added in a fixed order
-                    const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_part * p.acc_cols) + n0 + h;
+                    const uint32_t acc = tmem + lane_off + abase + n0 + h;
                     tmem_ld16(acc, vh);
                     for (int w = 1; w < p.n_part; ++w) {
                         float u[16];
@@ -1199,15 +1261,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                 }
                 __syncwarp();
             }
-            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
+            if (sub == nsub - 1) {
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
+            }
             if constexpr (FCP > 0) {
                 // logits = act(acc + b), then argmax / kill as the output-layer kernel
                 float lv[FCP];
 #pragma unroll
                 for (int c = 0; c < FCP; ++c) lv[c] = c < p.ff.C ? act_apply(p.ff.act, facc[c] + __ldg(p.ff.b + c)) : 0.f;
                 epilogue_reg<FCP>(p.ff.fa, p.t0, p.T, ri.row, ri.ok, lv, p.ff.C);
+            }
             }
         }
     } else if (DENSE && warp == 10 && p.a_tma) {
@@ -1327,9 +1392,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         const uint64_t tmap = reinterpret_cast<uint64_t>(&p.tmap_x);
         // tile i's first batch row, its first staged output row and its rows
         auto tile_geo = [&](int64_t i, int64_t &row0, int &oy0) {
-            const int64_t m0 = (blockIdx.x + i * gridDim.x) * (int64_t)kTileM;
+            const int64_t m0 = (blockIdx.x + i * gridDim.x) * TM;
             row0 = m0 / p.P;
-            oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / kTileM) * p.cv_rows;
+            oy0 = p.cv_imgs > 1 ? 0 : (int)((m0 - row0 * p.P) / TM) * p.cv_rows;
             return (int)min((int64_t)p.cv_imgs, (int64_t)p.R - row0);
         };
         auto issue = [&](int64_t jc) {
@@ -1435,7 +1500,49 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
         // the other's issue.  (A barrier is never two phases ahead of its waiter: the
         // other warp's next turn waits for this warp's arrival.)
         const int w = warp - 8;
-        if (lane == 0 && w < p.n_mma) {
+        if (pair) {
+            // tile pairs: warp w issues tile w of each unit into its own accumulator, both
+            // warps side by side from the same A and weight stages (each stage is released
+            // by the commits of both)
+            if (lane == 0 && w < 2) {
+                constexpr int Q = THREE ? 12 : 4;
+                const uint32_t id = idesc_tf32(kTileM, Nt), id2 = idesc_tf32(kTileM, 2 * Nt);
+                const bool merged = THREE && p.merge_lo;
+                bool ok = true;
+                if (p.b_resident) ok = wait_phase<32>(smem_u32(&bar_bfull[0]), 0, abort_flag);
+                const uint64_t desc_b0 = sw128_desc(b_region);
+                const uint32_t b_step16 = b_step >> 4, lo16 = (uint32_t)Nt * 128 >> 4;
+                int t = 0, sb = 0;
+                uint32_t t_wraps = 0, b_wraps = 0;
+                for (int64_t i = 0; ok && i < my_tiles; ++i) {
+                    const int a = p.n_acc == 2 ? (int)(i & 1) : 0;
+                    const int64_t use = p.n_acc == 2 ? (i >> 1) : i;
+                    if (use >= 1 && !wait_phase<32>(smem_u32(&bar_accempty[a]), (uint32_t)((use - 1) & 1), abort_flag)) break;
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint32_t d = tmem + (uint32_t)((a * 2 + w) * p.acc_cols);
+                    for (int kt = 0; kt < nK; ++kt) {
+                        if (!wait_phase<32>(smem_u32(&bar_afull[t]), t_wraps & 1, abort_flag)) { ok = false; break; }
+                        if (!p.b_resident &&
+                            !wait_phase<32>(smem_u32(&bar_bfull[sb]), b_wraps & 1, abort_flag)) { ok = false; break; }
+                        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                        const uint64_t dh = desc_b0 + (uint64_t)((p.b_resident ? kt : sb) * b_step16), dl = dh + lo16;
+                        const uint32_t ta = tmem + p.a_col + (uint32_t)(t * 2 + w) * kAColsPerStage;
+                        const uint32_t acc0 = kt > 0 ? 1u : 0u;   // K-step 0 of the tile overwrites
+                        if (merged) mma_block_merged(d, ta, dh, id2, id, acc0);
+                        else mma_block<THREE, 0, Q>(d, ta, dh, dl, id, acc0);
+                        mma_commit(smem_u32(&bar_aempty[t]));
+                        if (!p.b_resident) mma_commit(smem_u32(&bar_bempty[sb]));
+                        if (++t == p.n_stages) { t = 0; ++t_wraps; }
+                        if (!p.b_resident && ++sb == p.nb) { sb = 0; ++b_wraps; }
+                    }
+                    if (!ok) break;
+                    mma_commit(smem_u32(&bar_accfull[a]));
+                }
+                // every MMA of both issuing warps has finished before the teardown
+                mma_commit(smem_u32(&bar_drain));
+                wait_phase_drain(smem_u32(&bar_drain), 0);
+            }
+        } else if (lane == 0 && w < p.n_mma) {
             const int nmma = p.n_mma, nacc = p.n_acc;
             constexpr int Q = THREE ? 12 : 4;
             const uint32_t id = idesc_tf32(kTileM, Nt), id2 = idesc_tf32(kTileM, 2 * Nt);
@@ -1631,21 +1738,23 @@ struct ConvTile {
     uint32_t img_bytes;
 };
 
-static bool conv_tile(const Stage &S, ConvTile &t)
+// The staged geometry of units of tm GEMM rows (one tile, or a pair of tiles), with at most
+// max_bytes of staged rows per buffer.
+static bool conv_tile(const Stage &S, ConvTile &t, int tm = kTileM, size_t max_bytes = 48 * 1024)
 {
     if (S.kind != MURE_NODE_CONV2D || S.stride != 1 || (S.ic % kTileK != 0 && S.ic != 16)) return false;
     t.cw = S.ic == 16 ? 16 : kTileK;
     if (S.pool && ((S.oh & 1) || (S.ow & 1))) return false;
     const int P = S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
-    if (P >= kTileM) {
+    if (P >= tm) {
         // whole output rows per tile; pooled tiles hold whole rows of pooling windows
-        if (P % kTileM != 0 || kTileM % S.ow != 0) return false;
+        if (P % tm != 0 || tm % S.ow != 0) return false;
         t.imgs = 1;
-        t.rows = kTileM / S.ow;
+        t.rows = tm / S.ow;
         if (S.pool && (t.rows & 1)) return false;
     } else {
-        if (kTileM % P != 0) return false;
-        t.imgs = kTileM / P;
+        if (tm % P != 0) return false;
+        t.imgs = tm / P;
         t.rows = S.oh;
     }
     // staged width: the kw - 1 border columns, then padded (zero-filled columns past the
@@ -1658,7 +1767,7 @@ static bool conv_tile(const Stage &S, ConvTile &t)
     if (t.hw > 256 || t.hh > 256) return false;
     t.img_bytes = (uint32_t)((t.hw * t.hh * 128 + 1023) & ~1023);
     // at least two buffers beside the streamed weights (three K-steps of 128 channels)
-    return (size_t)t.imgs * t.img_bytes <= 48 * 1024;
+    return (size_t)t.imgs * t.img_bytes <= max_bytes;
 }
 
 int tc_conv_geometry(const Stage &S)
@@ -1919,9 +2028,20 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     ConvTile ct{};
     if (S.tc_conv) {
         // the staged convolution: as many staging buffers (up to 4) as fit beside the
-        // weights; the weights' K order was fixed for it at model load
-        const bool ok = conv_tile(S, ct) && conv_x_tensor_map(S, x, rm, ct, p.tmap_x);
+        // weights; the weights' K order was fixed for it at model load.  Slices of up to
+        // 64 outputs (not the delta GEMM) take units of two tiles where two buffers of
+        // their staged rows fit (measured: conv 64->64 -14%, ResNet-20's 16- to 64-channel
+        // convolutions -9..-10%; at 128 outputs the pair's single accumulator set, which
+        // no longer overlaps the epilogue, made it 4-20% slower)
         const size_t room = three ? tc_dyn_smem_max(k_tc_gemm<3, true>) : tc_dyn_smem_max(k_tc_gemm<3, false>);
+        bool ok = false;
+        if (!ss && nt_max <= 64 && conv_tile(S, ct, 2 * kTileM, 64 * 1024) &&
+            room >= 1024 + b_bytes + 2 * (size_t)ct.imgs * ct.img_bytes)
+            ok = p.cv_pair = conv_x_tensor_map(S, x, rm, ct, p.tmap_x) ? 1 : 0;
+        if (!ok) {
+            p.cv_pair = 0;
+            ok = conv_tile(S, ct) && conv_x_tensor_map(S, x, rm, ct, p.tmap_x);
+        }
         const size_t buf = (size_t)ct.imgs * ct.img_bytes;
         const int nbuf = ok && room > 1024 + b_bytes ? (int)std::min<size_t>(kNBufMax, (room - 1024 - b_bytes) / buf) : 0;
         if (nbuf < 2) {
@@ -1948,7 +2068,9 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     // alone, so a row's arithmetic never depends on the batch
     // (the window GEMM keeps two partial accumulators: measured as fast, no merged MMAs)
     // (not in the delta GEMM, whose slice width depends on the slots of its batch)
-    p.merge_lo = S.tc_conv && three && !ss && nt_max <= 64 ? 1 : 0;
+    // (with tile pairs only up to 32 outputs, where two accumulator sets of the merged
+    // width still fit)
+    p.merge_lo = S.tc_conv && three && !ss && nt_max <= (p.cv_pair ? 32 : 64) ? 1 : 0;
     tc_config(p, nt_max, three, !S.tc_small);
     // the delta GEMM: one issuing warp (or two in turn, which is the same sum), so that a
     // column's sum never depends on how many slots share its batch
@@ -1960,8 +2082,18 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
         p.n_mma = std::min(p.n_mma, 2);
         if (!p.mma_chain) p.n_part = p.n_mma;
     }
+    if (p.cv_pair) {
+        // units of two tiles: MMA warp w issues tile w of a unit into its own accumulator,
+        // the two warps side by side; an A stage holds the K-step of both tiles
+        p.n_mma = 2;
+        p.n_part = 1;
+        p.mma_chain = 0;
+        p.n_acc = 4 * p.acc_cols <= 256 ? 2 : 1;
+        p.n_stages = three ? 2 : 4;
+    }
     const int64_t M = (int64_t)rm.R * p.P;
-    const int64_t tiles = S.tc_small ? small_tiles(rm.R) : (M + kTileM - 1) / kTileM;
+    const int64_t unit = p.cv_pair ? 2 * kTileM : kTileM;
+    const int64_t tiles = S.tc_small ? small_tiles(rm.R) : (M + unit - 1) / unit;
     static int n_sm = 0;
     if (!n_sm) {
         int dev = 0;
