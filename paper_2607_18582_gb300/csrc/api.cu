@@ -1353,11 +1353,15 @@ mure_cache *build_cache(mure_model *m, const float *X, int64_t n_in, const int32
         ca->n_label_values = 0;
         for (int k = 0; k < kLabelWords; ++k) ca->n_label_values += __builtin_popcount(hm[k]);
         if (dev_err) {
-            // a token id outside an embedding's table, or a bounded wait that gave up
+            // a token id outside an embedding's table, a bounded wait that gave up, or a
+            // layer geometry a launch refused
             CK(c, cudaMemset(c->err_dev, 0, sizeof(int)));
-            FAILIF(true, c, dev_err == MURE_ERR_TIMEOUT ? MURE_ERR_TIMEOUT : MURE_ERR_INVALID_ARG,
+            FAILIF(true, c,
+                   dev_err == MURE_ERR_TIMEOUT || dev_err == MURE_ERR_UNSUPPORTED ? (mure_status)dev_err : MURE_ERR_INVALID_ARG,
                    "a device-side check failed while building the cache (code %d: %s)", dev_err,
-                   dev_err == MURE_ERR_INVALID_ARG ? "an input id outside the embedding's table" : "wait limit");
+                   dev_err == MURE_ERR_INVALID_ARG   ? "an input id outside the embedding's table"
+                   : dev_err == MURE_ERR_UNSUPPORTED ? "a layer geometry the kernels refused"
+                                                     : "wait limit");
         }
     }
     CK(c, cudaStreamSynchronize(s));
@@ -1481,6 +1485,9 @@ mure_status mure_model_load(mure_ctx *c, const mure_model_desc *d, mure_model **
                 S.tc_small = small && env != "generic";
                 S.tc_conv = !S.tc_small && env != "gather" && tc_conv_geometry(S);
                 S.tc_wide = S.tc_conv && getenv("MURE_TC_NARROW") == nullptr && tc_wide_geometry(S);
+                // 16-channel 3x3 layers: a GEMM row per 2x2 output window (MURE_TC_NOWINDOW
+                // keeps a row per position)
+                S.tc_win = S.tc_conv && getenv("MURE_TC_NOWINDOW") == nullptr && tc_win_geometry(S);
             }
         }
         std::vector<int> wn;

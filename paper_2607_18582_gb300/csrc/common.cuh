@@ -41,6 +41,8 @@ struct Stage {
     int tc_small = 0;         // tc: the small-image convolution mode
     int tc_conv = 0;          // tc: the staged convolution mode (input rows staged per tile)
     int tc_wide = 0;          // tc_conv: all 256 outputs in one CTA (one N = 256 MMA per K8 step)
+    int tc_win = 0;           // tc_conv: a GEMM row per 2x2 output window (16-channel 3x3 layers:
+                              // N = 4 positions x 16 outputs over a 4x4 field of 16 channels)
     float *Wtc = nullptr;     // tc: TF32 halves of W in the tensor-core operand layout
     int *err = nullptr;       // device error word of the context (bounded waits)
     const int64_t *wait_limit = nullptr;   // host: the context's wait limit (0 = default)
@@ -168,6 +170,7 @@ int tc_overlay_inline(const Stage &S, const Overlay &ov, int64_t groups);
 int tc_small_geometry(const Stage &S);
 int tc_conv_geometry(const Stage &S);
 int tc_wide_geometry(const Stage &S);
+int tc_win_geometry(const Stage &S);
 int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t s);
 int64_t tc_swizzle_tmp_floats(const Stage &S);
 int64_t tc_macs_per_row(const Stage &S);

@@ -295,6 +295,10 @@ struct TcParams {
                                  // take turns (mma_chain)
     int mma_chain;               // 1: the issuing warps take the K-steps in turn, in K-step
                                  // order, into one accumulator (handed over by barrier arrivals)
+    int cv_win;                  // MODE 3: a GEMM row per 2x2 output window (rows: windows
+                                 // (py, px), origin (2 py, 2 px); N = 4 positions x N outputs;
+                                 // taps of a 4x4 field)
+    int cv_fw, cv_ntap;          // MODE 3: the taps' field width (kw, or 4) and count
     int cv_pair;                 // MODE 3: units of two 128-row tiles (rows r and 128 + r per
                                  // producer thread; MMA warp w issues tile w; one weight stage
                                  // serves both)
@@ -363,6 +367,11 @@ __device__ __forceinline__ RowInfo row_info(const TcParams &p, int64_t m)
             ri.py = w / p.pw; ri.px = w % p.pw;
             ri.oy = 2 * ri.py + (sub >> 1);
             ri.ox = 2 * ri.px + (sub & 1);
+        } else if (p.cv_win) {
+            // a 2x2 output window: its top-left position
+            ri.py = q / p.pw; ri.px = q % p.pw;
+            ri.oy = 2 * ri.py;
+            ri.ox = 2 * ri.px;
         } else {
             ri.oy = q / p.ow;
             ri.ox = q % p.ow;
@@ -874,14 +883,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
                     }
                     const uint32_t buf = cv_region + (uint32_t)b * cv_buf_bytes;
                     const uint32_t base = buf + im * p.cv_img_bytes, base1 = buf + im1 * p.cv_img_bytes;
-                    const int ntap = p.kh * p.kw;
-                    // the current tap and its line relative to a row's line0 (ky * cv_hw + kx)
+                    const int ntap = p.cv_ntap;
+                    // the current tap and its line relative to a row's line0 (ky * cv_hw + kx),
+                    // over the filter (or a window's 4x4 field)
                     int tap = 0, kx = 0, off = 0;
                     auto next_tap = [&]() {
                         ++tap;
-                        if (++kx == p.kw) {
+                        if (++kx == p.cv_fw) {
                             kx = 0;
-                            off += p.cv_hw - p.kw + 1;
+                            off += p.cv_hw - p.cv_fw + 1;
                         } else {
                             ++off;
                         }
@@ -1067,6 +1077,56 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
 #pragma unroll
                     for (int c = 0; c < G::OC; c += 4)
                         *reinterpret_cast<float4 *>(yo + c) = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
+                }
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bar_accempty[a]));
+                continue;
+            }
+            if (MODE == 3 && p.cv_win) {
+                // a 2x2 output window per row: columns s * N + c for position s = 2 dy + dx
+                const RowInfo ri = row_info<false, false>(p, tile * kTileM + qd * 32 + lane);
+                const uint32_t acc = tmem + lane_off + (uint32_t)(a * p.n_part * p.acc_cols);
+                const float *srow = nullptr;
+                if (p.has_add && ri.ok)
+                    srow = p.skip + (p.skip_per_input ? p.t0 + logical_row(p.lrow, ri.row) % p.T : ri.row) * p.skip_stride;
+#pragma unroll 1
+                for (int sp = 0; sp < 4; ++sp) {
+                    const int oy = ri.oy + (sp >> 1), ox = ri.ox + (sp & 1);
+                    float v[16];   // N == 16 outputs per position
+                    tmem_ld16(acc + (uint32_t)(sp * 16), v);
+                    for (int w2 = 1; w2 < p.n_part; ++w2) {
+                        float u[16];
+                        tmem_ld16(acc + (uint32_t)(w2 * p.acc_cols + sp * 16), u);
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) v[e] += u[e];
+                    }
+                    if (p.merge_lo) {
+                        float u[16];
+                        tmem_ld16(acc + (uint32_t)(Nt + sp * 16), u);
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) v[e] += u[e];
+                    }
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) v[e] += bias_sh[e];
+                    if (p.z && ri.ok)
+                        for (int e = 0; e < 16; ++e)
+                            p.z[ri.row * p.z_stride + (int64_t)e * (p.oh * p.ow) + oy * p.ow + ox] = v[e];
+                    if (p.act1 != MURE_ACT_NONE) {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) v[e] = act_apply(p.act1, v[e]);
+                    }
+                    if (p.has_add && ri.ok) {
+                        const float *skp = srow + ((int64_t)oy * p.sk_stride * p.sk_w + ox * p.sk_stride) * p.sk_c;
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) v[e] = act_apply(p.act2, v[e] + (e < p.sk_c ? skp[e] : 0.f));
+                    }
+                    if (ri.ok) {
+                        float *yo = p.y + ri.row * p.y_stride + ((int64_t)oy * p.ow + ox) * 16;
+#pragma unroll
+                        for (int c = 0; c < 4; ++c)
+                            *reinterpret_cast<float4 *>(yo + 4 * c) = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                    }
                 }
                 asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                 __syncwarp();
@@ -1740,13 +1800,19 @@ struct ConvTile {
 
 // The staged geometry of units of tm GEMM rows (one tile, or a pair of tiles), with at most
 // max_bytes of staged rows per buffer.
-static bool conv_tile(const Stage &S, ConvTile &t, int tm = kTileM, size_t max_bytes = 48 * 1024)
+static bool conv_tile(const Stage &S, ConvTile &t, int tm = kTileM, size_t max_bytes = 48 * 1024, bool win = false)
 {
     if (S.kind != MURE_NODE_CONV2D || S.stride != 1 || (S.ic % kTileK != 0 && S.ic != 16)) return false;
     t.cw = S.ic == 16 ? 16 : kTileK;
-    if (S.pool && ((S.oh & 1) || (S.ow & 1))) return false;
+    if ((S.pool || win) && ((S.oh & 1) || (S.ow & 1))) return false;
     const int P = S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
-    if (P >= tm) {
+    if (win) {
+        // whole rows of 2x2 windows: tm windows are 2 tm / (ow / 2) output rows
+        const int pw = S.ow / 2, Pw = (S.oh / 2) * pw;
+        if (S.pool || S.kh != 3 || S.kw != 3 || S.pad != 1 || Pw % tm != 0 || tm % pw != 0) return false;
+        t.imgs = 1;
+        t.rows = 2 * (tm / pw);
+    } else if (P >= tm) {
         // whole output rows per tile; pooled tiles hold whole rows of pooling windows
         if (P % tm != 0 || tm % S.ow != 0) return false;
         t.imgs = 1;
@@ -1768,6 +1834,14 @@ static bool conv_tile(const Stage &S, ConvTile &t, int tm = kTileM, size_t max_b
     t.img_bytes = (uint32_t)((t.hw * t.hh * 128 + 1023) & ~1023);
     // at least two buffers beside the streamed weights (three K-steps of 128 channels)
     return (size_t)t.imgs * t.img_bytes <= max_bytes;
+}
+
+// The window form of the staged mode: 16-channel 3x3 convolutions with 16 outputs,
+// stride 1, pad 1, no pooling, whose windows fill whole 128-row tiles.
+int tc_win_geometry(const Stage &S)
+{
+    ConvTile t;
+    return S.ic == 16 && S.oc == 16 && conv_tile(S, t, kTileM, 96 * 1024, true) ? 1 : 0;
 }
 
 int tc_conv_geometry(const Stage &S)
@@ -1794,8 +1868,8 @@ int tc_overlay_inline(const Stage &S, const Overlay &ov, int64_t groups)
 }
 
 // The GEMM's N and K: the small-image mode multiplies by the window-expanded weights.
-static int gemm_n(const Stage &S) { return S.tc_small ? SmallConv::N : S.oc; }
-static int gemm_k(const Stage &S) { return S.tc_small ? SmallConv::K : S.K; }
+static int gemm_n(const Stage &S) { return S.tc_small ? SmallConv::N : S.tc_win ? 4 * S.oc : S.oc; }
+static int gemm_k(const Stage &S) { return S.tc_small ? SmallConv::K : S.tc_win ? 16 * S.ic : S.K; }
 
 // W [OC][(ky, kx, ci)] -> W' [(s, c)][(wy, wx, ci)]: the filter of window position
 // s = 2 dy + dx placed at offset (dy, dx) in the window's receptive field.
@@ -1811,6 +1885,21 @@ __global__ void k_expand_window_weights(const float *__restrict__ W, float *out)
     out[i] = ((unsigned)ky < (unsigned)G::KH && (unsigned)kx < (unsigned)G::KW)
                  ? W[(int64_t)c * (G::KH * G::KW * G::IC) + (ky * G::KW + kx) * G::IC + ci]
                  : 0.f;
+}
+
+// The staged mode's windows: W [OC][(ky, kx, ci)] of a 3x3 filter -> W' [(s, c)][(wy, wx,
+// ci)] over the 4x4 field of a 2x2 output window, position s = 2 dy + dx's filter at
+// offset (dy, dx), zeros elsewhere.
+__global__ void k_expand_field_weights(const float *__restrict__ W, int oc, int ic, float *out)
+{
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int N = 4 * oc, K = 16 * ic;
+    if (i >= (int64_t)N * K) return;
+    const int n = (int)(i / K), k = (int)(i % K);
+    const int sidx = n / oc, c = n % oc, dy = sidx >> 1, dx = sidx & 1;
+    const int wy = k / (4 * ic), wx = (k / ic) % 4, ci = k % ic;
+    const int ky = wy - dy, kx = wx - dx;
+    out[i] = ((unsigned)ky < 3u && (unsigned)kx < 3u) ? W[(int64_t)c * (9 * ic) + (ky * 3 + kx) * ic + ci] : 0.f;
 }
 
 // Output channels per CTA: one wide N = 256 slice for staged convolutions of exactly
@@ -1840,6 +1929,10 @@ int launch_swizzle_weights(const Stage &S, float *out, float *tmp, cudaStream_t 
         k_expand_window_weights<<<(N * K + 255) / 256, 256, 0, s>>>(S.W, tmp);
         W = tmp;
         ++launches;
+    } else if (S.tc_win) {
+        k_expand_field_weights<<<(N * K + 255) / 256, 256, 0, s>>>(S.W, S.oc, S.ic, tmp);
+        W = tmp;
+        ++launches;
     }
     cudaMemsetAsync(out, 0, tc_weight_floats(S) * sizeof(float), s);
     k_swizzle_weights<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(W, N, K, Np, Kp, planes,
@@ -1856,11 +1949,15 @@ int64_t tc_macs_per_row(const Stage &S)
     if (S.kind == MURE_NODE_DENSE) return Np * Kp;
     // the small-image mode runs a 128-row tile per SmallConv::MAPS maps
     if (S.tc_small) return (kTileM * Np * Kp + SmallConv::MAPS / 2) / SmallConv::MAPS;
+    if (S.tc_win) return (int64_t)(S.oh / 2) * (S.ow / 2) * Np * Kp;
     const int64_t P = S.pool ? 4 * (S.oh / 2) * (S.ow / 2) : (int64_t)S.oh * S.ow;
     return P * Np * Kp;
 }
 
-int64_t tc_swizzle_tmp_floats(const Stage &S) { return S.tc_small ? (int64_t)SmallConv::N * SmallConv::K : 0; }
+int64_t tc_swizzle_tmp_floats(const Stage &S)
+{
+    return S.tc_small ? (int64_t)SmallConv::N * SmallConv::K : S.tc_win ? (int64_t)gemm_n(S) * gemm_k(S) : 0;
+}
 
 // The longest run of the K-step sequence (tile after tile, nK steps each) between two
 // consecutive K-steps of one issuing warp, when K-step kt goes to warp kt mod m.
@@ -1996,6 +2093,17 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
         p.P = SmallConv::P;
         p.K = SmallConv::K; p.Kp = round_up32(SmallConv::K); p.Np = SmallConv::N;
     }
+    p.cv_fw = S.kw;
+    p.cv_ntap = S.kh * S.kw;
+    if (S.tc_win) {
+        // GEMM rows = 2x2 windows, columns = (position, output), K = the 4x4 field
+        p.P = (S.oh / 2) * (S.ow / 2);
+        p.K = p.Kp = gemm_k(S);
+        p.Np = gemm_n(S);
+        p.cv_win = 1;
+        p.cv_fw = 4;
+        p.cv_ntap = 16;
+    }
     const bool three = S.tc == 1;
     const int planes = three ? 2 : 1;
     p.Wsw = S.Wtc;
@@ -2020,8 +2128,9 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     const size_t slice_bytes = b_step * (p.Kp / kTileK);
     p.b_resident = slice_bytes <= (S.tc_small ? 112 : 96) * 1024;
     // a wide slice streams 64 KiB per K-step: two stages in flight
-    p.nb = p.slice_w > kSlice ? 2 : kNB;
-    const size_t b_bytes = p.b_resident ? slice_bytes : p.nb * b_step;
+    // (the windows' staged rows leave room for two weight stages)
+    p.nb = p.slice_w > kSlice || S.tc_win ? 2 : kNB;
+    size_t b_bytes = p.b_resident ? slice_bytes : p.nb * b_step;
     // at least 116 KiB so that one CTA (holding all 512 tensor-memory columns) runs per SM
     size_t a_bytes = S.tc_small ? (size_t)SmallConv::BYTES
                                 : (size_t)kNA * kStageA + (p.ov.patch ? (size_t)kNA * kOvSlotBytes : 0);
@@ -2035,14 +2144,20 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
         // no longer overlaps the epilogue, made it 4-20% slower)
         const size_t room = three ? tc_dyn_smem_max(k_tc_gemm<3, true>) : tc_dyn_smem_max(k_tc_gemm<3, false>);
         bool ok = false;
-        if (!ss && nt_max <= 64 && conv_tile(S, ct, 2 * kTileM, 64 * 1024) &&
+        if (!ss && !S.tc_win && nt_max <= 64 && conv_tile(S, ct, 2 * kTileM, 64 * 1024) &&
             room >= 1024 + b_bytes + 2 * (size_t)ct.imgs * ct.img_bytes)
             ok = p.cv_pair = conv_x_tensor_map(S, x, rm, ct, p.tmap_x) ? 1 : 0;
         if (!ok) {
             p.cv_pair = 0;
-            ok = conv_tile(S, ct) && conv_x_tensor_map(S, x, rm, ct, p.tmap_x);
+            ok = conv_tile(S, ct, kTileM, S.tc_win ? 96 * 1024 : 48 * 1024, S.tc_win != 0) &&
+                 conv_x_tensor_map(S, x, rm, ct, p.tmap_x);
         }
         const size_t buf = (size_t)ct.imgs * ct.img_bytes;
+        if (p.b_resident && room < 1024 + b_bytes + 2 * buf) {
+            // resident weights would leave room for fewer than two staging buffers: stream them
+            p.b_resident = 0;
+            b_bytes = (size_t)p.nb * b_step;
+        }
         const int nbuf = ok && room > 1024 + b_bytes ? (int)std::min<size_t>(kNBufMax, (room - 1024 - b_bytes) / buf) : 0;
         if (nbuf < 2) {
             static const int unsupported = MURE_ERR_UNSUPPORTED;
@@ -2050,7 +2165,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
             return 0;
         }
         p.cv_cw = ct.cw;
-        p.cv_taps = (S.kh * S.kw * ct.cw + kTileK - 1) / kTileK;
+        p.cv_taps = (p.cv_ntap * ct.cw + kTileK - 1) / kTileK;
         p.cv_nchunk = S.ic / ct.cw;
         p.cv_imgs = ct.imgs;
         p.cv_rows = ct.rows;
@@ -2174,6 +2289,7 @@ int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_input
     D.tc_wide = 0;   // the slot filters are laid out in slices of 128
     D.tc = precision == MURE_PREC_TF32X3 ? 1 : 2;
     D.tc_small = 0;
+    D.tc_win = 0;   // the slot GEMM runs per output position
     D.Wtc = dw.swz;
     D.b = dw.colb;
     SlotStore ss;
