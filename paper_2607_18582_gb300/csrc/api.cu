@@ -901,7 +901,8 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
         if (tc_delta && has_dot) {
             // the inputs' x_l and z_l: cached rows (memoized) or the batch's first
             // mutant's recomputed rows (vanilla; the prefix up to layer l is unmutated)
-            const int d = launch_tc_delta(Sl, m->precision, zsrc, xsrc(Sl.in_src), rm, pa, ws.patch, pstride, ws.dw, s);
+            const int d = launch_tc_delta(Sl, m->precision, zsrc, xsrc(Sl.in_src), skip_of(Sl), rm, pa, ws.patch, pstride,
+                                          ws.dw, s);
             if (d < 0) delta_err = 1; else n += d;
         } else if (dot_kernel && has_dot) {
             n += launch_patch_dot(Sl, zsrc, xsrc(Sl.in_src), rm, pa, kmax, ws.patch, pstride, s);

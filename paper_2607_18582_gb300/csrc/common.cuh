@@ -279,7 +279,7 @@ struct TcDeltaWs {
 };
 int tc_delta_supported(const Stage &S, int precision);
 void tc_delta_ws_size(int n_slots, int k_max, int64_t &floats, int64_t &ints);
-int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_inputs, const PatchArgs &pa, float *out,
+int launch_tc_delta(const Stage &S, int precision, Src z, Src x, Src skip, RowMap rm_inputs, const PatchArgs &pa, float *out,
                     int64_t out_stride, const TcDeltaWs &dw, cudaStream_t s);
 
 // GF / WS delta values of the small-layer geometries (stage variant > 0): the same

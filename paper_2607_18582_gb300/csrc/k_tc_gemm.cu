@@ -621,7 +621,8 @@ struct SmallSteps {
 template <int MODE, bool THREE, int FCP = 0>
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__ TcParams p)
 {
-    static_assert(FCP == 0 || (MODE == 0 && FCP % 4 == 0), "the output layer is fused into dense layers only");
+    static_assert(FCP == 0 || (MODE == 0 && FCP % 4 == 0) || (MODE == 3 && FCP == -1),
+                  "the output layer is fused into dense layers only; -1: the staged mode's slot GEMM with a residual add");
     constexpr bool DENSE = MODE == 0;
     constexpr int kNT = kMaxNT;                    // barrier slots; p.n_stages are used
     constexpr int kAColsPerStage = THREE ? 64 : 32;
@@ -1220,7 +1221,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const __grid_constant__
 #pragma unroll
                         for (int e = 0; e < 16; ++e) {
                             const int n = n_base + n0 + h + e;
-                            const float sv = n < p.sk_c ? sp[n] : 0.f;
+                            // the delta GEMM of a residual-add layer (FCP < 0): column n is a
+                            // slot, its skip value that of the slot's channel
+                            const int ch = FCP < 0 ? (n < p.slot.n ? __ldg(p.slot.j + n) : p.sk_c) : n;
+                            const float sv = ch < p.sk_c ? sp[ch] : 0.f;
                             vh[e] = act_apply(p.act2, vh[e] + sv);
                         }
                     }
@@ -2225,6 +2229,7 @@ int launch_tc(const Stage &S, Src x, RowMap rm, float *z_out, int64_t z_stride, 
     if (dense && ff) { if (three) go(k_tc_gemm<0, true, kFuseClasses>); else go(k_tc_gemm<0, false, kFuseClasses>); }
     else if (dense) { if (three) go(k_tc_gemm<0, true>); else go(k_tc_gemm<0, false>); }
     else if (S.tc_small) { if (three) go(k_tc_gemm<2, true>); else go(k_tc_gemm<2, false>); }
+    else if (S.tc_conv && ss && S.has_add) { if (three) go(k_tc_gemm<3, true, -1>); else go(k_tc_gemm<3, false, -1>); }
     else if (S.tc_conv) { if (three) go(k_tc_gemm<3, true>); else go(k_tc_gemm<3, false>); }
     else { if (three) go(k_tc_gemm<1, true>); else go(k_tc_gemm<1, false>); }
     int launches = 1;
@@ -2259,8 +2264,9 @@ __global__ void k_slot_filters(int K, const PatchArgs pa, int n_slot, int Np, fl
 // are multiples of 4 (16-byte copies).
 int tc_delta_supported(const Stage &S, int precision)
 {
-    return precision != MURE_PREC_FP32 && S.kind == MURE_NODE_CONV2D && !S.has_add && !S.gap && S.geo == 0 &&
-           S.ic % 4 == 0;
+    // (a residual add: the staged mode's slot instantiation adds each slot's own skip channel)
+    return precision != MURE_PREC_FP32 && S.kind == MURE_NODE_CONV2D && !S.gap && S.geo == 0 && S.ic % 4 == 0 &&
+           (!S.has_add || S.tc_conv);
 }
 
 void tc_delta_ws_size(int n_slots, int k_max, int64_t &floats, int64_t &ints)
@@ -2270,7 +2276,7 @@ void tc_delta_ws_size(int n_slots, int k_max, int64_t &floats, int64_t &ints)
     ints = 3 * Np;
 }
 
-int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_inputs, const PatchArgs &pa, float *out,
+int launch_tc_delta(const Stage &S, int precision, Src z, Src x, Src skip, RowMap rm_inputs, const PatchArgs &pa, float *out,
                     int64_t out_stride, const TcDeltaWs &dw, cudaStream_t s)
 {
     const int n = (int)pa.n_dslot;
@@ -2305,7 +2311,9 @@ int launch_tc_delta(const Stage &S, int precision, Src z, Src x, RowMap rm_input
     ss.cells = S.pool ? (S.oh / 2) * (S.ow / 2) : S.oh * S.ow;
     ss.T = rm_inputs.T;
     const RowMap rmT{rm_inputs.t0, rm_inputs.T, rm_inputs.T};
-    return 2 + launch_tc(D, x, rmT, nullptr, 0, Src{nullptr, 0, 0}, nullptr, 0, nullptr, s, nullptr, nullptr, &ss);
+    // a residual add: the skip rows of the batch's inputs (per input, or the first
+    // mutant's rows), added to each slot's own channel
+    return 2 + launch_tc(D, x, rmT, nullptr, 0, skip, nullptr, 0, nullptr, s, nullptr, nullptr, &ss);
 }
 
 }  // namespace mure
