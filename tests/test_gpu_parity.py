@@ -218,6 +218,26 @@ def test_batch_invariance_tensor_core_delta(M, ctx, prec):
     assert np.array_equal(big["logits"].view(np.uint32), van["logits"].view(np.uint32))
 
 
+@pytest.mark.parametrize("prec", ["tf32x3", "tf32"])
+def test_batch_invariance_windows_pairs_residual_delta(M, ctx, prec):
+    """ResNet-20 on the tensor cores: its 16-channel convolutions run as 2x2 output
+    windows, its 16- to 64-channel ones in pairs of tiles, and the GF / WS deltas of the
+    convolutions with a residual add as the slot GEMM with each slot's skip channel:
+    every operator on every layer gives the same bits in many small batches as in a few
+    large ones, and memoized == vanilla bit for bit."""
+    w = wl.workload("resnet20", 128, 1)
+    table = all_ops(w.model, 6, seed=61)
+    model = M.mure_model_load(ctx, w.model, precision=prec)
+    cache = M.mure_build_prefix_cache(model, w.X)
+    big = M.mure_eval_mutants(cache, table, logits=True)
+    small = M.mure_eval_mutants(cache, table, logits=True, workspace_bytes=64 << 20)
+    assert small["stats"]["n_batches"] > big["stats"]["n_batches"]
+    assert np.array_equal(big["kill_bits"], small["kill_bits"])
+    assert np.array_equal(big["logits"].view(np.uint32), small["logits"].view(np.uint32))
+    van = M.mure_eval_vanilla(model, w.X, table, logits=True)
+    assert np.array_equal(big["logits"].view(np.uint32), van["logits"].view(np.uint32))
+
+
 @pytest.mark.parametrize("name,prec", [("resnet20", "fp32"), ("mlp", "tf32x3"), ("lenet5", "tf32x3")])
 def test_identity_mutants_never_killed(M, ctx, name, prec):
     w = wl.workload(name, 96, 1)
