@@ -189,18 +189,26 @@ typedef struct {
     int64_t flops;          /* analytic FLOPs of the layer kernels that ran */
     /* with kernel_timing: device time and analytic FLOPs of the kernels of each
        weighted layer (index = layer, up to MURE_MAX_TIMED_LAYERS), of the delta
-       kernel (which also copies the cached rows a group starts from), and of the
-       stand-alone kill epilogue; ms_gather is kept for layout and stays 0 */
+       kernels (which also copy the cached rows a group starts from), and of the
+       stand-alone kill epilogue.  Where the mutated layer's fan-in sums (GF / WS)
+       run in a kernel of their own, the delta's value kernels (NEB / NAI / NS: the
+       cached pre-activations read, the patch values written) are timed apart in
+       ms_delta_values; otherwise they are part of ms_delta */
     double ms_layer[64];
     int64_t flops_layer[64];
     int64_t launches_layer[64];
-    double ms_delta, ms_gather, ms_epilogue;
+    double ms_delta, ms_delta_values, ms_epilogue;
     int64_t bytes_gather;   /* row bytes the delta kernel copies (read + write) */
     int64_t launches_delta;
     int64_t bytes_rows;     /* activation rows the stage kernels write and the next stage
                                reads back (2 x rows x row bytes): the device-memory traffic
                                of the batched suffix beyond the algorithmic bytes */
     int64_t n_rows_unchanged; /* rows not run by the unchanged-row elimination */
+    int64_t launches_delta_values; /* with kernel_timing: launches timed in ms_delta_values */
+    int64_t bytes_delta_values;    /* algorithmic bytes of those value kernels: the patch
+                                      values they write and the cached pre-activation row
+                                      of each input of a batch, read once for all its
+                                      mutants (memoized), or each row's own (vanilla) */
 } mure_eval_stats;
 
 #define MURE_MAX_TIMED_LAYERS 64

@@ -755,6 +755,7 @@ struct Acct {
     std::vector<int64_t> flops_cls, launches_cls;   // [L + 3]
     int64_t bytes_gather = 0;
     int64_t bytes_rows = 0;
+    int64_t bytes_values = 0;
     int64_t rows_unchanged = 0;
 };
 
@@ -763,7 +764,7 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
 {
     cudaStream_t s = c->stream;
     const int L = m->L;
-    const int C_DELTA = L, C_EPI = L + 2;
+    const int C_DELTA = L, C_VALS = L + 1, C_EPI = L + 2;
     int launches = 0;
     auto timed = [&](int cls, int64_t fl, auto &&launch) {
         tm.begin(cls);
@@ -894,21 +895,34 @@ int run_batch(mure_ctx *c, const mure_model *m, const mure_cache *ca, const DevT
                           (win_ops ? dt.copy_prefix[g0 + G] - dt.copy_prefix[g0] : 0);
     acct.bytes_gather += slots * rm.T * cells_l * 4;
     acct.bytes_gather += (vanilla ? rm.R : (int64_t)rm.T) * (m->zd[l].size + (has_dot ? m->xd[Sl.in_src].size : 0)) * 4;
+    // where the fan-in sums (GF / WS) run in a kernel of their own, the value kernels
+    // (NEB / NAI / NS: the cached pre-activations read, the patch values written) are
+    // timed and counted apart: they are the memory-bound part of the delta
+    const bool values_only = dot_kernel || tc_delta;
+    if (values_only) {
+        const int64_t vslots = (dt.val_prefix[g0 + G] - dt.val_prefix[g0]) -
+                               (win_ops ? dt.copy_prefix[g0 + G] - dt.copy_prefix[g0] : 0);
+        if (vslots > 0)
+            acct.bytes_values += vslots * rm.T * cells_l * 4 + (vanilla ? rm.R : (int64_t)rm.T) * m->zd[l].size * 4;
+    }
+    timed(values_only ? C_VALS : C_DELTA, values_only ? 0 : delta_flops, [&] {
+        return launch_patch_vals(Sl, zsrc, xsrc(Sl.in_src), skip_of(Sl), rm, pa, kmax, ws.patch, pstride, s, values_only,
+                                 win_ops);
+    });
     int delta_err = 0;
-    timed(C_DELTA, delta_flops, [&] {
-        int n = launch_patch_vals(Sl, zsrc, xsrc(Sl.in_src), skip_of(Sl), rm, pa, kmax, ws.patch, pstride, s,
-                                  dot_kernel || tc_delta, win_ops);
-        if (tc_delta && has_dot) {
-            // the inputs' x_l and z_l: cached rows (memoized) or the batch's first
-            // mutant's recomputed rows (vanilla; the prefix up to layer l is unmutated)
+    if (tc_delta && has_dot) {
+        // the inputs' x_l and z_l: cached rows (memoized) or the batch's first
+        // mutant's recomputed rows (vanilla; the prefix up to layer l is unmutated)
+        timed(C_DELTA, delta_flops, [&] {
             const int d = launch_tc_delta(Sl, m->precision, zsrc, xsrc(Sl.in_src), skip_of(Sl), rm, pa, ws.patch, pstride,
                                           ws.dw, s);
-            if (d < 0) delta_err = 1; else n += d;
-        } else if (dot_kernel && has_dot) {
-            n += launch_patch_dot(Sl, zsrc, xsrc(Sl.in_src), rm, pa, kmax, ws.patch, pstride, s);
-        }
-        return n;
-    });
+            if (d < 0) delta_err = 1;
+            return std::max(d, 0);
+        });
+    } else if (dot_kernel && has_dot) {
+        timed(C_DELTA, delta_flops,
+              [&] { return launch_patch_dot(Sl, zsrc, xsrc(Sl.in_src), rm, pa, kmax, ws.patch, pstride, s); });
+    }
     if (delta_err) return -1;
     // the unmutated rows of x_{l+1}: cached (memoized) or just computed (vanilla)
     const Src base = vanilla ? Src{ws.xb[l + 1], m->xd[l + 1].stride, 0} : Src{ca->x[l + 1], m->xd[l + 1].stride, 1};
@@ -1242,12 +1256,14 @@ void evaluate(mure_ctx *c, const mure_model *m, const mure_cache *ca, const mure
                 st.launches_layer[v] = acct.launches_cls[v];
             }
             st.ms_delta = ms[m->L];
-            st.ms_gather = ms[m->L + 1];
+            st.ms_delta_values = ms[m->L + 1];
+            st.launches_delta_values = acct.launches_cls[m->L + 1];
             st.ms_epilogue = ms[m->L + 2];
             st.launches_delta = acct.launches_cls[m->L];
         }
         st.bytes_gather = acct.bytes_gather;
         st.bytes_rows = acct.bytes_rows;
+        st.bytes_delta_values = acct.bytes_values;
         st.n_rows_unchanged = acct.rows_unchanged;
         float ms = 0;
         cudaEventElapsedTime(&ms, c->ev[0], c->ev[4]); st.ms_total = ms;

@@ -68,9 +68,10 @@ class _Stats(C.Structure):
                 ("ms_score", C.c_double), ("n_rows", C.c_int64), ("n_near_ties", C.c_int64),
                 ("n_groups", C.c_int64), ("n_batches", C.c_int64), ("kernel_launches", C.c_int64),
                 ("flops", C.c_int64), ("ms_layer", C.c_double * 64), ("flops_layer", C.c_int64 * 64),
-                ("launches_layer", C.c_int64 * 64), ("ms_delta", C.c_double), ("ms_gather", C.c_double),
+                ("launches_layer", C.c_int64 * 64), ("ms_delta", C.c_double), ("ms_delta_values", C.c_double),
                 ("ms_epilogue", C.c_double), ("bytes_gather", C.c_int64), ("launches_delta", C.c_int64),
-                ("bytes_rows", C.c_int64), ("n_rows_unchanged", C.c_int64)]
+                ("bytes_rows", C.c_int64), ("n_rows_unchanged", C.c_int64), ("launches_delta_values", C.c_int64),
+                ("bytes_delta_values", C.c_int64)]
 
     def as_dict(self):
         out = {}

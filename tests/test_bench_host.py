@@ -50,10 +50,16 @@ def test_hbm_rates_arithmetic():
     L = w.model.n_layers()
     rows = 1000
     macs = w.model.layer_macs(L - 1)
-    results = [{"stats": {"bytes_gather": 6_799_300, "flops_layer": [0] * (L - 1) + [2 * macs * rows]}}]
-    out = bench.hbm_rates(w, results, {"delta": 1.0, f"layer{L - 1}": 2.0}, {"hbm_gbs": 6799.3}, "measured")
-    assert out["delta"]["achieved"] == pytest.approx(6.7993)            # 6.8 MB in 1 ms
+    results = [{"stats": {"bytes_gather": 6_799_300, "bytes_delta_values": 1_000_000,
+                          "flops_layer": [0] * (L - 1) + [2 * macs * rows]}}]
+    cls = {"delta": 0.75, "delta_values": 0.25, f"layer{L - 1}": 2.0}
+    out = bench.hbm_rates(w, results, cls, {"hbm_gbs": 6799.3}, "measured")
+    assert out["delta"]["achieved"] == pytest.approx(6.7993)            # 6.8 MB in 0.75 + 0.25 ms
     assert out["delta"]["frac"] == pytest.approx(6.7993 / 6799.3)
+    assert out["cache_read"]["achieved"] == pytest.approx(4.0)          # 1 MB in 0.25 ms
+    assert out["cache_read"]["frac"] == pytest.approx(4.0 / 6799.3)
+    # no value kernels timed apart: no cache-read entry
+    assert "cache_read" not in bench.hbm_rates(w, results, {"delta": 1.0}, {"hbm_gbs": 6799.3}, "measured")
     node = w.model.nodes[w.model.layers()[L - 1]]
     exp = rows * (node.cin * 4 + 1 / 8) / 2e-3 / 1e9
     assert out["output_layer"]["achieved"] == pytest.approx(exp)
