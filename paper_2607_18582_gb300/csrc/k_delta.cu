@@ -476,9 +476,14 @@ int launch_patch_vals(const Stage &S, Src z, Src x, Src skip, RowMap rm, const P
     p.b = S.b;
     const int64_t n_items = (int64_t)p.G * kmax;
     // each warp walks several inputs (blockIdx.y, +gridDim.y, ...): enough blocks to
-    // fill the GPU, few enough that block scheduling stays negligible
+    // fill the GPU, few enough that block scheduling stays negligible.  Without fan-in
+    // sums in the launch, a layer of fewer than 32 cells takes a lane per input (32 inputs
+    // per block row), so more than ceil(T / 32) block rows would only idle (ncu: 4 x 608
+    // blocks for 2,048 inputs of VGG's conv 256->256, most of them empty)
     const int64_t gx = (n_items + 7) / 8;
-    const int64_t gy = std::max<int64_t>(1, std::min<int64_t>(rm.T, (152 * 16 + gx - 1) / gx));
+    const bool lane_per_input = skip_dot_ops && S.kind != MURE_NODE_DWCONV && (p.warp_dot || p.cells < 32);
+    const int64_t gy = std::max<int64_t>(1, std::min<int64_t>(lane_per_input ? (rm.T + 31) / 32 : rm.T,
+                                                              (152 * 16 + gx - 1) / gx));
     const dim3 grid((unsigned)gx, (unsigned)gy);
     const size_t smem = (S.gap && !p.warp_dot) ? 8 * (size_t)p.mcells * sizeof(float) : 0;
     // memoized dense layers: all operators per block of inputs

@@ -260,6 +260,7 @@ struct FinalParams {
     const int32_t *lrow;   // compacted batch: logical rows (per-input reads, overlay), else null
     int F, C, act;
     const float *W;  // [C][F]
+    const float *Wt; // [F][C] (the same weights, input-major)
     const float *b;
     FinalArgs fa;
     Overlay ov;      // mutated channels of the input rows (ov.patch null: none)
@@ -496,6 +497,153 @@ __global__ void __launch_bounds__(128) k_final_dense_w(const FinalParams p)
     epilogue_reg<CP>(p.fa, p.t0, p.T, row, in_range, v, p.C);
 }
 
+// The output layer of 9 to 12 classes with a block's 32 rows shared by its four warps:
+// warp w keeps classes w, w+4 and w+8 of every row (lane = row), so a warp's serial
+// instruction stream is a quarter of k_final_dense_w's (which keeps all classes of its
+// rows in one warp: ncu showed each of its blocks issue-bound at one warp per scheduler,
+// about 32 us per block whatever the grid, a third of it spent on a strided weight
+// fill).  A class's sum is the same fp32 chain as k_final_dense's (f ascending from +0,
+// fmaf(x, w, acc), then + b), so the bits equal those of the other output-layer kernels.
+// The weights come from the input-major copy Wt [F][C] with 16-byte loads all in flight;
+// each warp copies the rows' next 32 inputs (16-byte loads) into its own tile of 36-float
+// lines (16-byte stores and loads without bank conflicts) while it runs the FMAs of the
+// current 32; the warps' sums meet in shared memory and warp 0 runs the epilogue.  Needs
+// F a multiple of 4 and 16-byte aligned rows; dynamic shared memory [F][4][4] (class c at
+// [f][c mod 4][c / 4]).
+constexpr int kSplitLine = 36;
+
+__global__ void __launch_bounds__(128) k_final_dense_split(const FinalParams p)
+{
+    extern __shared__ __align__(16) float wsm[];   // [F][4][4]
+    __shared__ __align__(16) float xs[4][32][kSplitLine];
+    __shared__ float sums[32][13];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int i = threadIdx.x; i < p.F * 16; i += 128) wsm[i] = 0.f;
+    const int64_t row0 = (int64_t)blockIdx.x * 32;
+    const int64_t row = row0 + lane;
+    const bool in_range = row < p.R;
+    int ov_k = 0;
+    const int32_t *ov_ids = nullptr;
+    const int64_t lrow = in_range ? logical_row(p.lrow, row) : row;
+    if (p.ov.patch && in_range) {
+        const int g = (int)(lrow / p.T);
+        ov_k = p.ov.n_neurons[g];
+        ov_ids = p.ov.ids + p.ov.neuron_off[g];
+    }
+    // this lane copies 16 bytes (inputs 4 (lane mod 8) .. +3) of rows 4i + lane / 8
+    const int fq = 4 * (lane & 7);
+    const float *src[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const int64_t r = row0 + 4 * i + (lane >> 3);
+        src[i] = r < p.R ? p.x + (p.x_per_input ? (p.t0 + logical_row(p.lrow, r) % p.T) : r) * p.x_stride : nullptr;
+    }
+    auto load = [&](int f0, float4 (&v)[8]) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            v[i] = (src[i] && f0 + fq < p.F) ? __ldg(reinterpret_cast<const float4 *>(src[i] + f0 + fq))
+                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+    };
+    float4 cur[8];
+    load(0, cur);
+    __syncthreads();   // padding zeroed before the weights are placed
+    {
+        const int n4 = p.F * p.C / 4;
+        const float4 *w4p = reinterpret_cast<const float4 *>(p.Wt);
+        for (int i0 = threadIdx.x; i0 < n4; i0 += 8 * 128) {
+            float4 v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int i = i0 + u * 128;
+                v[u] = i < n4 ? __ldg(w4p + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int i = i0 + u * 128;
+                if (i >= n4) continue;
+                int f = 4 * i / p.C, c = 4 * i - f * p.C;
+                const float e[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    wsm[f * 16 + (c & 3) * 4 + (c >> 2)] = e[k];
+                    if (++c == p.C) { c = 0; ++f; }
+                }
+            }
+        }
+    }
+    __syncthreads();   // the weights
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f;
+    const float *wq = wsm + 4 * warp;
+    const float *xr = &xs[warp][lane][0];
+    for (int f0 = 0; f0 < p.F; f0 += 32) {
+        __syncwarp();
+#pragma unroll
+        for (int i = 0; i < 8; ++i) *reinterpret_cast<float4 *>(&xs[warp][4 * i + (lane >> 3)][fq]) = cur[i];
+        if (f0 + 32 < p.F) load(f0 + 32, cur);
+        __syncwarp();
+        const int fe = min(32, p.F - f0);
+        // overlay on this lane's own row (no other lane reads it)
+        for (int q = 0; q < ov_k; ++q) {
+            const int j = ov_ids[q];
+            const int cfirst = f0 - j <= 0 ? 0 : (f0 - j + p.ov.ch - 1) / p.ov.ch;
+            for (int c = cfirst; c < p.ov.cells && c * p.ov.ch + j < f0 + fe; ++c)
+                xs[warp][lane][c * p.ov.ch + j - f0] = p.ov.patch[lrow * p.ov.row_stride + q * p.ov.cells + c];
+        }
+        if (fe == 32) {
+#pragma unroll
+            for (int f4 = 0; f4 < 32; f4 += 4) {
+                const float4 x4 = *reinterpret_cast<const float4 *>(xr + f4);
+                const float xq[4] = {x4.x, x4.y, x4.z, x4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float4 w4 = *reinterpret_cast<const float4 *>(wq + (f0 + f4 + e) * 16);
+                    a0 = fmaf(xq[e], w4.x, a0);
+                    a1 = fmaf(xq[e], w4.y, a1);
+                    a2 = fmaf(xq[e], w4.z, a2);
+                }
+            }
+        } else {
+            for (int fl = 0; fl < fe; ++fl) {
+                const float xv = xr[fl];
+                const float4 w4 = *reinterpret_cast<const float4 *>(wq + (f0 + fl) * 16);
+                a0 = fmaf(xv, w4.x, a0);
+                a1 = fmaf(xv, w4.y, a1);
+                a2 = fmaf(xv, w4.z, a2);
+            }
+        }
+    }
+    sums[lane][warp] = a0;
+    sums[lane][warp + 4] = a1;
+    sums[lane][warp + 8] = a2;
+    __syncthreads();
+    if (warp != 0) return;
+    float v[12];
+#pragma unroll
+    for (int c = 0; c < 12; ++c) {
+        const float z = c < p.C ? sums[lane][c] + __ldg(p.b + c) : 0.f;
+        if (in_range && c < p.C && p.fa.z_out) p.fa.z_out[row * p.fa.z_stride + c] = z;
+        v[c] = act_apply(p.act, z);
+    }
+    if (p.fa.mode == 1) {  // cache build: logits rows and original predictions
+        if (in_range) {
+#pragma unroll
+            for (int c = 0; c < 12; ++c)
+                if (c < p.C) p.fa.x_out[row * p.fa.x_stride + c] = v[c];
+            p.fa.pred_out[row] = argmax_reg<12>(v, p.C);
+        }
+        return;
+    }
+    if (p.fa.mode == 2) {  // per-row logits for a following delta + epilogue
+        if (in_range) {
+#pragma unroll
+            for (int c = 0; c < 12; ++c)
+                if (c < p.C) p.fa.logits_rows[row * p.fa.x_stride + c] = v[c];
+        }
+        return;
+    }
+    epilogue_reg<12>(p.fa, p.t0, p.T, row, in_range, v, p.C);
+}
+
 __global__ void __launch_bounds__(128) k_epilogue(const float *__restrict__ lg, int64_t stride, int per_input, int C,
                                                   int64_t t0, int T, int R, const FinalArgs fa, const Overlay ov)
 {
@@ -604,7 +752,7 @@ int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cu
     p.x = x.p; p.x_stride = x.stride; p.x_per_input = x.per_input;
     p.t0 = rm.t0; p.T = rm.T; p.R = rm.R; p.lrow = rm.lrow;
     p.F = S.K; p.C = S.oc; p.act = S.act1;
-    p.W = S.W; p.b = S.b;
+    p.W = S.W; p.Wt = S.Wt; p.b = S.b;
     p.fa = fa;
     const unsigned blocks = (unsigned)((rm.R + 127) / 128);
     const int cp = (p.C + 3) & ~3;
@@ -629,7 +777,12 @@ int launch_final_dense(const Stage &S, Src x, RowMap rm, const FinalArgs &fa, cu
         };
         if (cp <= 4) go(k_final_dense_w<4>);
         else if (cp <= 8) go(k_final_dense_w<8>);
-        else go(k_final_dense_w<12>);
+        else {
+            // 9 to 12 classes: a block's 32 rows shared by four warps
+            const size_t sbytes = (size_t)p.F * 16 * sizeof(float);
+            cudaFuncSetAttribute(k_final_dense_split, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sbytes);
+            k_final_dense_split<<<(unsigned)((rm.R + 31) / 32), 128, sbytes, s>>>(p);
+        }
         return 1;
     }
     if (cp <= 4) k_final_dense<4><<<blocks, 128, 0, s>>>(p);
